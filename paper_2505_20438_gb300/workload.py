@@ -1,0 +1,215 @@
+"""Seeded synthetic inputs for smashed-KV decode attention.
+
+This module only draws inputs: bf16 query/key/value bits, per-slot token
+counts, slot counts and page tables.  It holds none of the attention, RoPE or
+append arithmetic, so both the CUDA path and the CPU oracle can be fed from it
+without sharing any of the method's code.
+
+Workloads stand in for the paper's decode workloads (short-context GSM8K /
+HumanEval / MGSM and long-context MultiNews / LongBench decoding, Sec. 4.3 and
+Fig. 5); the datasets and trained weights are not used.  A slot is one
+"smashed" KV entry that stands for 1..4 tokens (Sec. 3.1 and Sec. 3.6, token
+fusion), with at most 4 tokens per macro-step (Sec. 4.1).
+
+Token counts per slot follow a geometric law with p = 0.5 whose tail is folded
+into 4: P(1)=1/2, P(2)=1/4, P(3)=1/8, P(4)=1/8 (mean 1.875).
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Optional, Sequence
+
+import numpy as np
+
+# Maximum micro-step size: a macro-step emits (so a slot fuses) at most 4 tokens (Sec. 4.1).
+MAX_TOKENS_PER_SLOT = 4
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    """Shape and value distribution of one decode-attention workload."""
+
+    name: str
+    batch: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    page_slots: int
+    layers: int
+    slots: int = 0                       # slots per sequence (uniform batches)
+    slot_range: Optional[tuple] = None   # inclusive (lo, hi) for ragged batches
+    value_scale: float = 1.0             # std of q, K, V
+    seed: int = 0
+    pool_factor: float = 1.25            # pool pages / pages needed
+    scatter_pages: bool = True           # random page table vs sequential
+    attend_then_append: bool = False     # step order stated by the workload
+
+    @property
+    def group(self) -> int:
+        return self.n_q_heads // self.n_kv_heads
+
+
+# Tiny CPU-checkable case: 1 sequence, 8/2 heads, d=64, 2 pages of 128 slots.  The cache
+# is built by 255 appends at slot positions 0..254; the decode step appends slot 255 (so
+# positions run 0..255 and the 256 slots fill both pages) and attends over all 256.
+C0_TINY = Workload("tiny_b1_h8x2_d64_s256_p128", batch=1, n_q_heads=8, n_kv_heads=2,
+                   head_dim=64, page_slots=128, layers=1, slots=255, value_scale=1.0,
+                   seed=0, pool_factor=1.0, scatter_pages=False)
+# Llama-3-8B-shaped layer: batch 8, 32/8 heads, d=128, 4096 slots, 16-slot scattered pages.
+C1_LLAMA8B = Workload("llama8b_layer_b8_s4096", batch=8, n_q_heads=32, n_kv_heads=8,
+                      head_dim=128, page_slots=16, layers=1, slots=4096,
+                      value_scale=1.0 / math.sqrt(128.0), seed=1)
+# Ragged serving batch: 64 sequences, slots uniform in [512, 8192], attend then append.
+C2_RAGGED = Workload("ragged_b64_s512to8192", batch=64, n_q_heads=32, n_kv_heads=8,
+                     head_dim=128, page_slots=16, layers=1, slot_range=(512, 8192),
+                     value_scale=1.0, seed=2, attend_then_append=True)
+# Long context: batch 4, 65536 slots (~123k tokens at 1.875 tokens per slot).
+C3_LONG = Workload("long_b4_s65536", batch=4, n_q_heads=32, n_kv_heads=8, head_dim=128,
+                   page_slots=16, layers=1, slots=65536, value_scale=1.0, seed=3)
+
+
+def c4_sweep(batch: int, slots: int = 2048, layers: int = 32) -> Workload:
+    """32-layer decode stack of the Llama-8B layer shape, starting from 2048 slots."""
+    return Workload(f"stack_l{layers}_b{batch}_s{slots}", batch=batch, n_q_heads=32,
+                    n_kv_heads=8, head_dim=128, page_slots=16, layers=layers, slots=slots,
+                    value_scale=1.0 / math.sqrt(128.0), seed=4)
+
+
+WORKLOADS = {w.name: w for w in (C0_TINY, C1_LLAMA8B, C2_RAGGED, C3_LONG)}
+
+
+def scaled(w: Workload, **changes) -> Workload:
+    """Same workload with some fields replaced (smaller parity cases)."""
+    return dataclasses.replace(w, **changes)
+
+
+# ----------------------------------------------------------------------------
+# draws
+# ----------------------------------------------------------------------------
+
+def rng_for(seed: int, stream: int = 0) -> np.random.Generator:
+    """Independent PCG64 stream per (seed, purpose)."""
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, stream])))
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to bf16 (nearest, ties to even) and return the raw uint16 bits.
+
+    Used only to turn drawn normals into bf16 inputs; finite inputs only.
+    """
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    rounded = u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))
+    return (rounded >> np.uint32(16)).astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def normal_bf16(rng: np.random.Generator, shape: Sequence[int], scale: float = 1.0,
+                block: int = 1 << 24) -> np.ndarray:
+    """bf16 bits of N(0, scale^2) draws, generated in blocks to bound host memory."""
+    n = int(np.prod(shape))
+    out = np.empty(n, dtype=np.uint16)
+    for s in range(0, n, block):
+        e = min(n, s + block)
+        x = rng.standard_normal(e - s, dtype=np.float32)
+        if scale != 1.0:
+            x *= np.float32(scale)
+        out[s:e] = f32_to_bf16_bits(x)
+    return out.reshape(shape)
+
+
+def ntok_capped_geometric(rng: np.random.Generator, shape, p: float = 0.5,
+                          cap: int = MAX_TOKENS_PER_SLOT) -> np.ndarray:
+    """Tokens fused into each slot: geometric(p) on {1, 2, ...}, tail folded into `cap`."""
+    return np.minimum(rng.geometric(p, size=shape), cap).astype(np.int32)
+
+
+def slot_counts(w: Workload, rng: np.random.Generator) -> np.ndarray:
+    if w.slot_range is not None:
+        lo, hi = w.slot_range
+        return rng.integers(lo, hi + 1, size=w.batch).astype(np.int32)
+    return np.full(w.batch, w.slots, dtype=np.int32)
+
+
+def pages_needed(max_slots: int, page_slots: int) -> int:
+    return -(-max_slots // page_slots)
+
+
+def page_table(rng: np.random.Generator, batch: int, max_pages: int, pool_pages: int,
+               scatter: bool = True) -> np.ndarray:
+    """[batch][max_pages] distinct page ids drawn from a pool of `pool_pages`."""
+    need = batch * max_pages
+    if need > pool_pages:
+        raise ValueError(f"pool of {pool_pages} pages cannot hold {need}")
+    ids = rng.permutation(pool_pages)[:need] if scatter else np.arange(need)
+    return ids.astype(np.int32).reshape(batch, max_pages)
+
+
+@dataclasses.dataclass
+class HostCase:
+    """A whole decode-attention case on the host (bf16 as uint16 bits)."""
+
+    w: Workload
+    num_slots: np.ndarray        # [B] int32: slots already in the cache
+    max_slots: int               # capacity per sequence (slots)
+    pool_pages: int
+    page_table: np.ndarray       # [B][max_pages] int32
+    k: np.ndarray                # [B][Lmax][Hkv][d] uint16 (already rotated keys)
+    v: np.ndarray                # [B][Lmax][Hkv][d] uint16
+    slot_ntok: np.ndarray        # [B][Lmax] int32
+    slot_pos: np.ndarray         # [B][Lmax] int32 (slot index)
+    q: np.ndarray                # [B][Hq][d] uint16 (already rotated query)
+    k_new: np.ndarray            # [B][Hkv][d] uint16 (unrotated key of the new slot)
+    v_new: np.ndarray            # [B][Hkv][d] uint16
+    ntok_new: np.ndarray         # [B] int32
+
+    @property
+    def lmax(self) -> int:
+        return self.k.shape[1]
+
+
+def make_case(w: Workload, extra_slots: int = 1, num_slots: Optional[np.ndarray] = None,
+              pool_pages: Optional[int] = None) -> HostCase:
+    """Draw every input of workload `w` on the host from its seed.
+
+    `extra_slots` is the headroom per sequence for appends after the cache is filled.
+    """
+    counts = slot_counts(w, rng_for(w.seed, 1)) if num_slots is None else \
+        np.asarray(num_slots, dtype=np.int32)
+    lmax = int(counts.max()) if counts.size else 0
+    max_slots = lmax + extra_slots
+    max_pages = pages_needed(max(max_slots, 1), w.page_slots)
+    if pool_pages is None:
+        pool_pages = int(math.ceil(w.batch * max_pages * w.pool_factor))
+    pt = page_table(rng_for(w.seed, 2), w.batch, max_pages, pool_pages, w.scatter_pages)
+    shape = (w.batch, lmax, w.n_kv_heads, w.head_dim)
+    k = normal_bf16(rng_for(w.seed, 3), shape, w.value_scale)
+    v = normal_bf16(rng_for(w.seed, 4), shape, w.value_scale)
+    ntok = ntok_capped_geometric(rng_for(w.seed, 5), (w.batch, lmax))
+    pos = np.broadcast_to(np.arange(lmax, dtype=np.int32), (w.batch, lmax)).copy()
+    for b in range(w.batch):           # slots past a sequence's length are unused
+        ntok[b, counts[b]:] = 0
+        pos[b, counts[b]:] = 0
+    q = normal_bf16(rng_for(w.seed, 6), (w.batch, w.n_q_heads, w.head_dim), w.value_scale)
+    k_new = normal_bf16(rng_for(w.seed, 7), (w.batch, w.n_kv_heads, w.head_dim), w.value_scale)
+    v_new = normal_bf16(rng_for(w.seed, 8), (w.batch, w.n_kv_heads, w.head_dim), w.value_scale)
+    ntok_new = ntok_capped_geometric(rng_for(w.seed, 9), (w.batch,))
+    return HostCase(w, counts, max_slots, pool_pages, pt, k, v, ntok, pos, q, k_new, v_new,
+                    ntok_new)
+
+
+def device_normal_bf16(shape, scale: float, seed: int, device="cuda"):
+    """bf16 N(0, scale^2) tensor drawn on the device from a seeded torch generator.
+
+    Used where host generation would dominate start-up time (full-size bench workloads).
+    """
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    x = torch.randn(*shape, generator=g, device=device, dtype=torch.float32)
+    if scale != 1.0:
+        x.mul_(scale)
+    return x.to(torch.bfloat16)
