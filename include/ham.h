@@ -1,0 +1,218 @@
+/*
+ * ham.h -- C ABI of the GB300 (sm_103a) smashed-KV decode-attention library, libham.so.
+ *
+ * Method: HAMburger (Liu & Zhang, arXiv 2505.20438).  A macro-step is one forward of the
+ * base model that stores ONE key/value set for the whole group of 1..4 tokens it fused
+ * (Sec. 3.1; Sec. 3.6 "Token Fusion"); the cache therefore holds one "slot" per macro-step,
+ * and each decode step attends over the slots and appends the slot just produced.  The
+ * merged embedding enters the base model at an offset position reflecting the fused token
+ * count (Sec. 3.2).  With one token per slot everything reduces to the base model's own
+ * decode (Sec. 3.4).  Decoding reads the whole cache every step and is bound by memory
+ * bandwidth (Sec. 2.3, KV-cache compression).
+ *
+ * Conventions
+ *  - Every call returns an int status (ham_status).  No exception or abort crosses the ABI.
+ *    On failure ham_last_error() gives a message (thread-local, valid until the next call
+ *    on the same thread).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Calls
+ *    taking a stream are asynchronous unless stated otherwise.
+ *  - bf16 tensors are raw 16-bit bfloat16 values, row-major, 16-byte aligned device memory
+ *    owned by the caller.  The library owns the KV pool, page tables, counters and its
+ *    scratch; ham_kv_free releases them.
+ *  - Kernels never trap.  A bad value that can only be seen on the device (a page id outside
+ *    the pool, a full sequence, a token count < 1, a bounded wait that ran out) is recorded
+ *    in a device error word and the offending write is skipped; ham_kv_status or
+ *    ham_slot_lengths report it as HAM_EDEVICE.
+ */
+#ifndef HAM_H
+#define HAM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define HAM_ABI_VERSION 1
+
+typedef enum ham_status {
+  HAM_OK = 0,
+  HAM_EINVAL = 1,       /* bad argument seen on the host; nothing was launched */
+  HAM_ENOMEM = 2,       /* device or pinned-host allocation failed */
+  HAM_ECAPACITY = 3,    /* configuration does not fit (pool smaller than the page tables) */
+  HAM_ECUDA = 4,        /* a CUDA runtime call failed (message has the CUDA error) */
+  HAM_EDEVICE = 5,      /* a kernel recorded an error in the device error word */
+  HAM_EUNSUPPORTED = 6  /* shape outside the compiled kernels (head_dim, group size) */
+} ham_status;
+
+/* Device error word values (ham_kv_status). The first error recorded wins. */
+enum {
+  HAM_DEVERR_NONE = 0,
+  HAM_DEVERR_CAPACITY = 1,  /* append into a sequence already holding max_slots_per_seq */
+  HAM_DEVERR_NTOK = 2,      /* token count < 1 for a new slot */
+  HAM_DEVERR_PAGE = 3,      /* page-table entry outside [0, pool_pages) */
+  HAM_DEVERR_SLOTS = 4,     /* slot counter outside [0, max_slots_per_seq] */
+  HAM_DEVERR_TIMEOUT = 5    /* a bounded wait inside a kernel ran out */
+};
+
+/* Position given to a new slot when ham_kv_append gets pos == NULL (Sec. 3.2). */
+enum {
+  HAM_POS_SLOT = 0,   /* the slot index, i.e. the macro-step number */
+  HAM_POS_TOKEN = 1   /* tokens already in the sequence: the position of the group's first token */
+};
+
+enum { HAM_DTYPE_BF16 = 0, HAM_DTYPE_F32 = 1 };
+
+typedef struct ham_kv ham_kv; /* opaque handle: one paged smashed-KV cache, all layers */
+
+typedef struct ham_config {
+  int32_t layers;            /* >= 1 */
+  int32_t batch;             /* sequences, 1..4096 */
+  int32_t n_q_heads;         /* query heads */
+  int32_t n_kv_heads;        /* KV heads; n_q_heads / n_kv_heads in {1, 2, 4, 8} */
+  int32_t head_dim;          /* 64 or 128 */
+  int32_t page_slots;        /* slots per page, a multiple of 16 */
+  int32_t max_slots_per_seq; /* capacity of one sequence, in slots */
+  int32_t pos_mode;          /* HAM_POS_SLOT or HAM_POS_TOKEN */
+  int64_t pool_pages;        /* pages in the pool; 0 = batch * ceil(max_slots_per_seq / page_slots) */
+  double rope_base;          /* RoPE base (10000 for Llama-style models) */
+  uint64_t page_seed;        /* 0: sequence b gets pages [b*P, (b+1)*P); else a seeded shuffle */
+} ham_config;
+
+typedef struct ham_kv_info {
+  ham_config cfg;            /* with pool_pages resolved */
+  int32_t max_pages_per_seq; /* page-table row length = ceil(max_slots_per_seq / page_slots) */
+  int32_t attn_ctas;         /* CTAs of one attention launch */
+  int32_t num_sms;           /* SMs of the device the handle lives on */
+  int32_t device;            /* CUDA device ordinal */
+  int64_t pool_bytes;        /* K+V bytes of ONE layer's pool */
+  int64_t scratch_bytes;     /* split-attention partials + tickets */
+} ham_kv_info;
+
+/* ------------------------------------------------------------------------------------
+ * The four calls of a macro-step
+ * ------------------------------------------------------------------------------------ */
+
+/* Allocate a paged smashed-KV cache on the current CUDA device (synchronous).
+ *
+ * Device layout (one allocation; every pointer below lives inside it):
+ *   K pool, V pool of layer l  [pool_pages][n_kv_heads][page_slots][head_dim] bf16
+ *   slot_pos, slot_ntok        [pool_pages][page_slots] int32   (shared by all layers)
+ *   page table                 [batch][max_pages_per_seq] int32
+ *   num_slots                  [layers][batch] int32,  num_tokens [layers][batch] int64
+ * Slot n of sequence b is row n % page_slots of page page_table[b][n / page_slots].
+ * Every sequence starts empty.  Pages are reserved at allocation (page_seed), so appends
+ * never need the host.  Errors: HAM_EINVAL (bad config), HAM_ECAPACITY (pool_pages <
+ * batch * max_pages_per_seq), HAM_EUNSUPPORTED, HAM_ENOMEM, HAM_ECUDA.  *out is NULL on
+ * failure. */
+int ham_kv_alloc(const ham_config *cfg, ham_kv **out);
+
+/* Free everything the handle owns (synchronizes the device first).  NULL is a no-op. */
+int ham_kv_free(ham_kv *kv);
+
+/* Append the slot of this macro-step to every sequence of one layer (Sec. 3.1: one KV set
+ * per macro-step; Sec. 3.2: its position).  One fused kernel: for each sequence b, with
+ * n = num_slots[layer][b] and position p = pos[b] (or, if pos == NULL, n for HAM_POS_SLOT
+ * and num_tokens[layer][b] for HAM_POS_TOKEN):
+ *   K row of slot n  <- RoPE(k_new[b], p)   (rotate-half, theta_i = p * base^(-2i/d),
+ *                                            computed in fp64, stored bf16 round-to-nearest-even)
+ *   V row of slot n  <- v_new[b]             (bit copy)
+ *   q_inout[b]       <- RoPE(q_inout[b], p)  (if q_inout != NULL, in place)
+ *   slot_pos = p, slot_ntok = ntok[b], num_slots += 1, num_tokens += ntok[b]
+ * q_inout  nullable, device bf16 [batch][n_q_heads][head_dim]
+ * k_new, v_new      device bf16 [batch][n_kv_heads][head_dim]
+ * pos      nullable, device int32 [batch];  ntok  device int32 [batch], each >= 1
+ * A full sequence or ntok < 1 skips that sequence and sets the device error word.
+ * Host errors: HAM_EINVAL (NULL / unaligned pointer, layer out of range), HAM_ECUDA. */
+int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
+                  const void *v_new, const int32_t *pos, const int32_t *ntok, void *stream);
+
+/* One decode step of one layer: every query head attends over all slots of its sequence
+ * (softmax(q K^T / sqrt(head_dim)) V over the slot list; no weighting by token count).
+ * Query head h reads KV head h / (n_q_heads / n_kv_heads).  Split-KV: the slots of all
+ * (sequence, KV head) pairs are cut into equal contiguous ranges, one per CTA, and the
+ * partial softmax states of a pair are merged by the last CTA that finishes it.  Sequences
+ * with no slots give 0.  Slot counts are read on the device (no host sync).
+ * q    device bf16 [batch][n_q_heads][head_dim], already rotated (e.g. by ham_kv_append)
+ * out  device bf16 [batch][n_q_heads][head_dim]
+ * Host errors: HAM_EINVAL, HAM_ECUDA.  Calls on one handle must not overlap in time (they
+ * share the handle's scratch); serialize them on one stream. */
+int ham_decode_attn(ham_kv *kv, int32_t layer, const void *q, void *out, void *stream);
+
+/* Slot and token counts of every sequence after the last layer's appends (synchronous:
+ * copies on `stream`, then waits for it).  num_slots_host [batch], num_tokens_host [batch]
+ * (either may be NULL).  Returns HAM_EDEVICE if the device error word is set. */
+int ham_slot_lengths(ham_kv *kv, int32_t *num_slots_host, int64_t *num_tokens_host,
+                     void *stream);
+
+/* ------------------------------------------------------------------------------------
+ * Helpers: inspection, test set-up, tuning
+ * ------------------------------------------------------------------------------------ */
+
+/* Message of the last failed call on this thread ("" if none). */
+const char *ham_last_error(void);
+
+/* Sizes and resolved settings of a handle. */
+int ham_kv_get_info(const ham_kv *kv, ham_kv_info *info);
+
+/* Same as ham_decode_attn with the output type chosen: HAM_DTYPE_BF16 or HAM_DTYPE_F32
+ * (fp32 output, for tight comparisons). */
+int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out,
+                       int32_t out_dtype, void *stream);
+
+/* Per-layer counters (synchronous, like ham_slot_lengths). */
+int ham_kv_layer_lengths(ham_kv *kv, int32_t layer, int32_t *num_slots_host,
+                         int64_t *num_tokens_host, void *stream);
+
+/* Read and clear the device error word (synchronizes `stream`).  *device_code (nullable)
+ * gets the HAM_DEVERR_* value.  Returns HAM_EDEVICE if it was set. */
+int ham_kv_status(ham_kv *kv, void *stream, int32_t *device_code);
+
+/* Replace the page table with host_pt [batch][max_pages_per_seq] (synchronous).  Entries
+ * must lie in [0, pool_pages) and no page may appear twice; else HAM_EINVAL and nothing
+ * changes.  Existing slot contents are NOT moved. */
+int ham_kv_set_page_table(ham_kv *kv, const int32_t *host_pt);
+
+/* Copy the page table to host_pt [batch][max_pages_per_seq] (synchronous). */
+int ham_kv_get_page_table(const ham_kv *kv, int32_t *host_pt);
+
+/* Load a logical cache into one layer: slot j < counts[b] of sequence b gets
+ * k_log/v_log[b][j] (bit copy, no RoPE: keys are taken as already rotated) and, if given,
+ * slot_pos = pos[b][j], slot_ntok = ntok[b][j] (defaults: j and 1).  Sets
+ * num_slots[layer][b] = counts[b] and num_tokens[layer][b] = sum of the ntok.
+ * k_log, v_log  device bf16 [batch][lmax][n_kv_heads][head_dim]
+ * pos, ntok     nullable device int32 [batch][lmax];  counts  device int32 [batch]
+ * A count outside [0, min(lmax, max_slots_per_seq)] sets the device error word. */
+int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
+                const int32_t *pos, const int32_t *ntok, const int32_t *counts, int32_t lmax,
+                void *stream);
+
+/* Copy one layer's raw pools and the slot metadata out (device or pinned host destinations,
+ * cudaMemcpyDefault).  k_dst, v_dst: pool_bytes / 2 bytes each; pos_dst, ntok_dst:
+ * pool_pages * page_slots int32 each.  Any destination may be NULL. */
+int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *pos_dst,
+                  int32_t *ntok_dst, void *stream);
+
+/* Set every sequence of every layer back to 0 slots / 0 tokens (pages stay reserved). */
+int ham_kv_reset(ham_kv *kv, void *stream);
+
+/* Number of CTAs one attention launch uses (0 = default: SMs x resident CTAs per SM).
+ * Range 1 .. 8 x SMs.  Any value gives the same result up to fp32 summation order. */
+int ham_kv_set_attn_ctas(ham_kv *kv, int32_t ctas);
+
+/* Host evaluation of the split plan the attention kernel uses (no GPU needed).  Chunks are
+ * 16 slots; the chunks of (sequence b, KV head g), b-major, are numbered contiguously (W in
+ * all).  The first min(ctas, W) CTAs get equal non-empty ranges, CTA c the chunks
+ * [cta_begin[c], cta_begin[c+1]); the others stay idle.  For each segment
+ * s = b*n_kv_heads+g, seg_first_cta[s] .. seg_last_cta[s] are exactly the CTAs that touch
+ * it (-1, -1 if empty).
+ * cta_begin [ctas+1] int64; seg_first_cta, seg_last_cta [batch*n_kv_heads] int32. */
+int ham_split_plan(int32_t batch, int32_t n_kv_heads, const int32_t *num_slots_host,
+                   int32_t ctas, int64_t *cta_begin, int32_t *seg_first_cta,
+                   int32_t *seg_last_cta);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* HAM_H */

@@ -1,0 +1,122 @@
+// Internal declarations of libham.so (not installed; the public ABI is include/ham.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ham.h"
+
+namespace ham {
+
+// A chunk is the unit of the split plan and of one TMA stage: 16 consecutive slots of one
+// (sequence, KV head) pair.  Pages hold a multiple of 16 slots, so a chunk never straddles
+// two pages and its K (or V) rows are one contiguous 16 * head_dim * 2-byte block.
+constexpr int kChunkSlots = 16;
+constexpr int kMaxBatch = 4096;
+
+// ---------------------------------------------------------------------------------------
+// Split plan.  The chunks of all (sequence b, KV head g) segments are numbered b-major,
+// then g, then chunk index; W is their total.  Of the launched CTAs, C = min(launched, W)
+// take part and CTA c < C takes chunks [floor(c W / C), floor((c+1) W / C)), never empty
+// because W >= C.  So the CTAs touching a segment are exactly owner(first chunk) ..
+// owner(last chunk).  A CTA writes one partial per segment it touches, at index c + s,
+// which is unique because (c, s) only ever grows along the chunk order.
+// ---------------------------------------------------------------------------------------
+__host__ __device__ inline int32_t plan_ctas(int64_t W, int32_t launched) {
+  return (int32_t)(W < (int64_t)launched ? W : (int64_t)launched);
+}
+__host__ __device__ inline int64_t plan_cta_begin(int64_t W, int32_t C, int64_t c) {
+  return (W * c) / C;
+}
+// CTA that owns chunk x (0 <= x < W): the largest c with floor(c W / C) <= x.
+__host__ __device__ inline int32_t plan_owner(int64_t W, int32_t C, int64_t x) {
+  return (int32_t)(((x + 1) * (int64_t)C - 1) / W);
+}
+__host__ __device__ inline int32_t chunks_of(int32_t slots) {
+  return (slots + kChunkSlots - 1) / kChunkSlots;
+}
+
+// Everything one attention launch needs; all pointers are device pointers.
+struct AttnView {
+  const uint16_t *k_pool;      // this layer: [pool_pages][n_kv_heads][page_slots][head_dim]
+  const uint16_t *v_pool;
+  const int32_t *page_table;   // [batch][max_pages]
+  const int32_t *num_slots;    // [batch] of this layer
+  const uint16_t *q;           // [batch][n_q_heads][head_dim]
+  void *out;                   // [batch][n_q_heads][head_dim], bf16 or f32
+  float *part_acc;             // scratch [(ctas + batch*n_kv_heads)][group][head_dim]
+  float2 *part_ml;             // scratch [(ctas + batch*n_kv_heads)][group]: (max, sum)
+  uint32_t *tickets;           // scratch [batch*n_kv_heads], zero between launches
+  int32_t *err;                // device error word
+  int64_t pool_pages;
+  int32_t batch, n_kv_heads, page_slots, max_pages, max_slots;
+  int32_t ctas;
+};
+
+struct AppendView {
+  uint16_t *k_pool, *v_pool;   // this layer
+  int32_t *slot_pos, *slot_ntok;
+  const int32_t *page_table;
+  int32_t *num_slots;          // [batch] of this layer
+  int64_t *num_tokens;         // [batch] of this layer
+  const double *inv_freq;      // [head_dim / 2]: base^(-2i/d)
+  uint16_t *q;                 // nullable
+  const uint16_t *k_new, *v_new;
+  const int32_t *pos;          // nullable
+  const int32_t *ntok;
+  int32_t *err;
+  int64_t pool_pages;
+  int32_t batch, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots, pos_mode;
+};
+
+struct FillView {
+  uint16_t *k_pool, *v_pool;
+  int32_t *slot_pos, *slot_ntok;
+  const int32_t *page_table;
+  int32_t *num_slots;
+  int64_t *num_tokens;
+  const uint16_t *k_log, *v_log;
+  const int32_t *pos, *ntok, *counts;
+  int32_t *err;
+  int64_t pool_pages;
+  int32_t batch, n_kv_heads, head_dim, page_slots, max_pages, max_slots, lmax;
+};
+
+// Launchers (return cudaError_t of the launch; argument checks are done by the callers).
+cudaError_t launch_attention(const AttnView &v, int head_dim, int group, int out_dtype,
+                             cudaStream_t stream);
+// CTAs of one SM for the attention kernel of this shape (0 if the shape is not compiled).
+int attention_ctas_per_sm(int head_dim, int group, int batch);
+bool attention_supported(int head_dim, int group);
+cudaError_t launch_append(const AppendView &v, cudaStream_t stream);
+cudaError_t launch_fill(const FillView &v, cudaStream_t stream);
+
+// Device error word: keep the first error.
+__device__ inline void record_error(int32_t *err, int32_t code) {
+  if (err) atomicCAS(err, 0, code);
+}
+
+}  // namespace ham
+
+// Library-internal handle (opaque to users).
+struct ham_kv {
+  ham_config cfg;
+  int device = 0;
+  int num_sms = 0;
+  int32_t max_pages = 0;
+  int32_t attn_ctas = 0;        // 0: default
+  int32_t max_ctas = 0;         // scratch is sized for this many CTAs
+  int64_t pool_elems = 0;       // bf16 elements of ONE pool (K or V) of one layer
+  uint16_t *pool = nullptr;     // [layers][2][pool_elems]
+  uint8_t *meta = nullptr;      // everything else, carved below
+  int32_t *slot_pos = nullptr, *slot_ntok = nullptr, *page_table = nullptr;
+  int32_t *num_slots = nullptr; // [layers][batch]
+  int64_t *num_tokens = nullptr;
+  double *inv_freq = nullptr;
+  int32_t *err = nullptr;
+  float *part_acc = nullptr;
+  float2 *part_ml = nullptr;
+  uint32_t *tickets = nullptr;
+  int64_t scratch_bytes = 0;
+  void *host_stage = nullptr;   // pinned: counters and error word read-back
+};

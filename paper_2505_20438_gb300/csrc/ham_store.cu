@@ -1,0 +1,567 @@
+// Paged smashed-KV store: allocation, page tables, counters, fill/export and the C ABI
+// entry points that are not kernels of the decode path.
+//
+// A macro-step of HAMburger stores one KV set for all tokens it fused (Sec. 3.1, Sec. 3.6
+// "Token Fusion"), so the store is a per-sequence list of slots, each with the position it
+// was rotated at (Sec. 3.2) and its token count.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <vector>
+
+#include "ham_internal.cuh"
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+int fail(int status, const char *fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+  va_end(ap);
+  return status;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+  return fail(HAM_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define HAM_CUDA(call)                                   \
+  do {                                                   \
+    cudaError_t e_ = (call);                             \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call);  \
+  } while (0)
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+uint64_t splitmix64(uint64_t &s) {
+  uint64_t z = (s += 0x9E3779B97F4A7C15ull);
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Page ids of every sequence: sequential for seed 0, else the first batch*max_pages ids of
+// a seeded Fisher-Yates shuffle of the pool.
+std::vector<int32_t> reserve_pages(int32_t batch, int32_t max_pages, int64_t pool_pages,
+                                   uint64_t seed) {
+  std::vector<int32_t> ids((size_t)pool_pages);
+  for (int64_t i = 0; i < pool_pages; ++i) ids[(size_t)i] = (int32_t)i;
+  if (seed != 0) {
+    uint64_t s = seed;
+    for (int64_t i = pool_pages - 1; i > 0; --i) {
+      int64_t j = (int64_t)(splitmix64(s) % (uint64_t)(i + 1));
+      std::swap(ids[(size_t)i], ids[(size_t)j]);
+    }
+  }
+  ids.resize((size_t)batch * (size_t)max_pages);
+  return ids;
+}
+
+int check_layer(const ham_kv *kv, int32_t layer) {
+  if (!kv) return fail(HAM_EINVAL, "null handle");
+  if (layer < 0 || layer >= kv->cfg.layers)
+    return fail(HAM_EINVAL, "layer %d outside [0, %d)", layer, kv->cfg.layers);
+  return HAM_OK;
+}
+
+// Run host code on the handle's device, restoring the caller's device afterwards.
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+    else prev = -1;
+  }
+  ~DeviceGuard() {
+    if (prev >= 0) cudaSetDevice(prev);
+  }
+};
+
+uint16_t *layer_pool(const ham_kv *kv, int32_t layer, int which) {
+  return kv->pool + ((size_t)layer * 2 + (size_t)which) * (size_t)kv->pool_elems;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------------------------
+// fill kernel (test and bench set-up: logical cache -> pages)
+// ------------------------------------------------------------------------------------
+namespace ham {
+
+__global__ void fill_rows_kernel(FillView v) {
+  const int32_t b = blockIdx.y;
+  const int32_t count = v.counts[b];
+  if (count < 0 || count > v.lmax || count > v.max_slots) return;  // reported by fill_meta
+  const int vec_per_row = v.head_dim / 8;  // 16-byte vectors per (slot, KV head) row
+  const int64_t vec_per_slot = (int64_t)v.n_kv_heads * vec_per_row;
+  const int64_t first = (int64_t)blockIdx.x * 16;  // 16 slots per block
+  for (int64_t idx = threadIdx.x; idx < 16 * vec_per_slot; idx += blockDim.x) {
+    const int64_t j = first + idx / vec_per_slot;
+    if (j >= count) continue;
+    const int32_t g = (int32_t)((idx % vec_per_slot) / vec_per_row);
+    const int32_t e = (int32_t)(idx % vec_per_row);
+    const int32_t page = v.page_table[(int64_t)b * v.max_pages + j / v.page_slots];
+    if (page < 0 || page >= v.pool_pages) {
+      record_error(v.err, HAM_DEVERR_PAGE);
+      continue;
+    }
+    const int64_t dst = (((int64_t)page * v.n_kv_heads + g) * v.page_slots + j % v.page_slots) *
+                        v.head_dim / 8 + e;
+    const int64_t src = (((int64_t)b * v.lmax + j) * v.n_kv_heads + g) * vec_per_row + e;
+    reinterpret_cast<uint4 *>(v.k_pool)[dst] = reinterpret_cast<const uint4 *>(v.k_log)[src];
+    reinterpret_cast<uint4 *>(v.v_pool)[dst] = reinterpret_cast<const uint4 *>(v.v_log)[src];
+  }
+}
+
+__global__ void fill_meta_kernel(FillView v) {
+  const int32_t b = blockIdx.x;
+  const int32_t count = v.counts[b];
+  __shared__ long long partial[32];
+  if (count < 0 || count > v.lmax || count > v.max_slots) {
+    if (threadIdx.x == 0) record_error(v.err, HAM_DEVERR_SLOTS);
+    return;
+  }
+  long long tokens = 0;
+  for (int32_t j = threadIdx.x; j < count; j += blockDim.x) {
+    const int32_t page = v.page_table[(int64_t)b * v.max_pages + j / v.page_slots];
+    const int32_t t = v.ntok ? v.ntok[(int64_t)b * v.lmax + j] : 1;
+    tokens += t;
+    if (page < 0 || page >= v.pool_pages) continue;  // reported by fill_rows
+    const int64_t m = (int64_t)page * v.page_slots + j % v.page_slots;
+    v.slot_pos[m] = v.pos ? v.pos[(int64_t)b * v.lmax + j] : j;
+    v.slot_ntok[m] = t;
+  }
+  for (int o = 16; o > 0; o >>= 1) tokens += __shfl_xor_sync(0xffffffffu, tokens, o);
+  if ((threadIdx.x & 31) == 0) partial[threadIdx.x / 32] = tokens;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long total = 0;
+    for (int w = 0; w < (int)(blockDim.x / 32); ++w) total += partial[w];
+    v.num_slots[b] = count;
+    v.num_tokens[b] = total;
+  }
+}
+
+cudaError_t launch_fill(const FillView &v, cudaStream_t stream) {
+  if (v.lmax > 0) {
+    dim3 grid((unsigned)((v.lmax + 15) / 16), (unsigned)v.batch);
+    fill_rows_kernel<<<grid, 256, 0, stream>>>(v);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  fill_meta_kernel<<<v.batch, 256, 0, stream>>>(v);
+  return cudaGetLastError();
+}
+
+}  // namespace ham
+
+// ------------------------------------------------------------------------------------
+// C ABI
+// ------------------------------------------------------------------------------------
+extern "C" {
+
+const char *ham_last_error(void) { return g_last_error; }
+
+int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
+  if (!out) return fail(HAM_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (!cfg_in) return fail(HAM_EINVAL, "config is NULL");
+  ham_config cfg = *cfg_in;
+  if (cfg.layers < 1 || cfg.batch < 1 || cfg.batch > ham::kMaxBatch || cfg.n_q_heads < 1 ||
+      cfg.n_kv_heads < 1 || cfg.n_q_heads % cfg.n_kv_heads != 0)
+    return fail(HAM_EINVAL, "bad shape: layers %d batch %d (max %d) heads %d/%d", cfg.layers,
+                cfg.batch, ham::kMaxBatch, cfg.n_q_heads, cfg.n_kv_heads);
+  if (cfg.page_slots < ham::kChunkSlots || cfg.page_slots % ham::kChunkSlots != 0)
+    return fail(HAM_EINVAL, "page_slots %d must be a positive multiple of %d", cfg.page_slots,
+                ham::kChunkSlots);
+  if (cfg.max_slots_per_seq < 1)
+    return fail(HAM_EINVAL, "max_slots_per_seq %d must be >= 1", cfg.max_slots_per_seq);
+  if (cfg.pos_mode != HAM_POS_SLOT && cfg.pos_mode != HAM_POS_TOKEN)
+    return fail(HAM_EINVAL, "pos_mode %d", cfg.pos_mode);
+  if (!(cfg.rope_base > 1.0) || !std::isfinite(cfg.rope_base))
+    return fail(HAM_EINVAL, "rope_base must be finite and > 1");
+  const int group = cfg.n_q_heads / cfg.n_kv_heads;
+  if (!ham::attention_supported(cfg.head_dim, group))
+    return fail(HAM_EUNSUPPORTED, "head_dim %d / group %d not compiled (head_dim 64 or 128, "
+                "group 1, 2, 4 or 8)", cfg.head_dim, group);
+  const int64_t max_pages =
+      ((int64_t)cfg.max_slots_per_seq + cfg.page_slots - 1) / cfg.page_slots;
+  const int64_t need_pages = (int64_t)cfg.batch * max_pages;
+  if (need_pages > INT32_MAX) return fail(HAM_EINVAL, "page table too large");
+  // The attention kernel counts 16-slot chunks of the whole batch in int32.
+  if ((int64_t)cfg.batch * ham::chunks_of(cfg.max_slots_per_seq) * cfg.n_kv_heads > INT32_MAX)
+    return fail(HAM_EINVAL, "batch * max_slots_per_seq too large");
+  if (cfg.pool_pages == 0) cfg.pool_pages = need_pages;
+  if (cfg.pool_pages < need_pages)
+    return fail(HAM_ECAPACITY, "pool of %lld pages < %lld pages reserved by the page tables",
+                (long long)cfg.pool_pages, (long long)need_pages);
+  if (cfg.pool_pages > INT32_MAX) return fail(HAM_EINVAL, "pool_pages above int32 range");
+
+  int dev = 0;
+  HAM_CUDA(cudaGetDevice(&dev));
+  int sms = 0;
+  HAM_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+
+  ham_kv *kv = new ham_kv();
+  kv->cfg = cfg;
+  kv->device = dev;
+  kv->num_sms = sms;
+  kv->max_pages = (int32_t)max_pages;
+  kv->max_ctas = 8 * sms;
+  kv->pool_elems = cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots * cfg.head_dim;
+
+  const size_t pool_bytes = (size_t)cfg.layers * 2 * (size_t)kv->pool_elems * sizeof(uint16_t);
+  const size_t slots_meta = (size_t)cfg.pool_pages * cfg.page_slots * sizeof(int32_t);
+  const size_t n_seg = (size_t)cfg.batch * cfg.n_kv_heads;
+  const size_t n_part = (size_t)kv->max_ctas + n_seg;
+  size_t off = 0;
+  auto carve = [&](size_t bytes) {
+    size_t at = off;
+    off = round_up(off + bytes, 256);
+    return at;
+  };
+  const size_t o_pos = carve(slots_meta), o_ntok = carve(slots_meta);
+  const size_t o_pt = carve((size_t)need_pages * sizeof(int32_t));
+  const size_t o_ns = carve((size_t)cfg.layers * cfg.batch * sizeof(int32_t));
+  const size_t o_nt = carve((size_t)cfg.layers * cfg.batch * sizeof(int64_t));
+  const size_t o_if = carve((size_t)(cfg.head_dim / 2) * sizeof(double));
+  const size_t o_err = carve(sizeof(int32_t));
+  const size_t o_acc = carve(n_part * group * cfg.head_dim * sizeof(float));
+  const size_t o_ml = carve(n_part * group * sizeof(float2));
+  const size_t o_tk = carve(n_seg * sizeof(uint32_t));
+  kv->scratch_bytes = (int64_t)(off - o_acc);
+
+  cudaError_t e = cudaMalloc(&kv->pool, pool_bytes);
+  if (e != cudaSuccess) {
+    delete kv;
+    cudaGetLastError();
+    return fail(HAM_ENOMEM, "cudaMalloc of %zu pool bytes: %s", pool_bytes, cudaGetErrorString(e));
+  }
+  e = cudaMalloc(&kv->meta, off);
+  if (e == cudaSuccess) e = cudaMallocHost(&kv->host_stage, 256 + (size_t)cfg.batch * 16);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    ham_kv_free(kv);
+    return fail(HAM_ENOMEM, "allocation of the cache metadata failed");
+  }
+  kv->slot_pos = reinterpret_cast<int32_t *>(kv->meta + o_pos);
+  kv->slot_ntok = reinterpret_cast<int32_t *>(kv->meta + o_ntok);
+  kv->page_table = reinterpret_cast<int32_t *>(kv->meta + o_pt);
+  kv->num_slots = reinterpret_cast<int32_t *>(kv->meta + o_ns);
+  kv->num_tokens = reinterpret_cast<int64_t *>(kv->meta + o_nt);
+  kv->inv_freq = reinterpret_cast<double *>(kv->meta + o_if);
+  kv->err = reinterpret_cast<int32_t *>(kv->meta + o_err);
+  kv->part_acc = reinterpret_cast<float *>(kv->meta + o_acc);
+  kv->part_ml = reinterpret_cast<float2 *>(kv->meta + o_ml);
+  kv->tickets = reinterpret_cast<uint32_t *>(kv->meta + o_tk);
+
+  // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits.
+  e = cudaMemset(kv->pool, 0, pool_bytes);
+  if (e == cudaSuccess) e = cudaMemset(kv->meta, 0, off);
+  std::vector<int32_t> pt = reserve_pages(cfg.batch, kv->max_pages, cfg.pool_pages, cfg.page_seed);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(kv->page_table, pt.data(), pt.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  // RoPE frequencies theta_i / pos = base^(-2i/d), fp64 (rotate-half pairs (i, i + d/2)).
+  std::vector<double> inv_freq((size_t)cfg.head_dim / 2);
+  for (int i = 0; i < cfg.head_dim / 2; ++i)
+    inv_freq[(size_t)i] = pow(cfg.rope_base, -(2.0 * (double)i) / (double)cfg.head_dim);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(kv->inv_freq, inv_freq.data(), inv_freq.size() * sizeof(double),
+                   cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    int rc = cuda_fail(e, "initialising the cache");
+    ham_kv_free(kv);
+    return rc;
+  }
+  *out = kv;
+  return HAM_OK;
+}
+
+int ham_kv_free(ham_kv *kv) {
+  if (!kv) return HAM_OK;
+  DeviceGuard guard(kv->device);
+  cudaDeviceSynchronize();
+  if (kv->pool) cudaFree(kv->pool);
+  if (kv->meta) cudaFree(kv->meta);
+  if (kv->host_stage) cudaFreeHost(kv->host_stage);
+  delete kv;
+  return HAM_OK;
+}
+
+int ham_kv_get_info(const ham_kv *kv, ham_kv_info *info) {
+  if (!kv || !info) return fail(HAM_EINVAL, "null argument");
+  memset(info, 0, sizeof *info);
+  info->cfg = kv->cfg;
+  info->max_pages_per_seq = kv->max_pages;
+  const int group = kv->cfg.n_q_heads / kv->cfg.n_kv_heads;
+  int per_sm = ham::attention_ctas_per_sm(kv->cfg.head_dim, group, kv->cfg.batch);
+  info->attn_ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->num_sms * (per_sm > 0 ? per_sm : 1);
+  info->num_sms = kv->num_sms;
+  info->device = kv->device;
+  info->pool_bytes = 2 * kv->pool_elems * (int64_t)sizeof(uint16_t);
+  info->scratch_bytes = kv->scratch_bytes;
+  return HAM_OK;
+}
+
+int ham_kv_set_attn_ctas(ham_kv *kv, int32_t ctas) {
+  if (!kv) return fail(HAM_EINVAL, "null handle");
+  if (ctas < 0 || ctas > kv->max_ctas)
+    return fail(HAM_EINVAL, "ctas %d outside [0, %d]", ctas, kv->max_ctas);
+  kv->attn_ctas = ctas;
+  return HAM_OK;
+}
+
+int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
+                  const void *v_new, const int32_t *pos, const int32_t *ntok, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!k_new || !v_new || !ntok) return fail(HAM_EINVAL, "k_new, v_new and ntok are required");
+  if (!aligned16(k_new) || !aligned16(v_new) || (q_inout && !aligned16(q_inout)))
+    return fail(HAM_EINVAL, "q/k/v must be 16-byte aligned");
+  if (((uintptr_t)ntok & 3u) || ((uintptr_t)pos & 3u))
+    return fail(HAM_EINVAL, "pos/ntok must be 4-byte aligned");
+  DeviceGuard guard(kv->device);
+  ham::AppendView v{};
+  v.k_pool = layer_pool(kv, layer, 0);
+  v.v_pool = layer_pool(kv, layer, 1);
+  v.slot_pos = kv->slot_pos;
+  v.slot_ntok = kv->slot_ntok;
+  v.page_table = kv->page_table;
+  v.num_slots = kv->num_slots + (size_t)layer * kv->cfg.batch;
+  v.num_tokens = kv->num_tokens + (size_t)layer * kv->cfg.batch;
+  v.inv_freq = kv->inv_freq;
+  v.q = static_cast<uint16_t *>(q_inout);
+  v.k_new = static_cast<const uint16_t *>(k_new);
+  v.v_new = static_cast<const uint16_t *>(v_new);
+  v.pos = pos;
+  v.ntok = ntok;
+  v.err = kv->err;
+  v.pool_pages = kv->cfg.pool_pages;
+  v.batch = kv->cfg.batch;
+  v.n_q_heads = kv->cfg.n_q_heads;
+  v.n_kv_heads = kv->cfg.n_kv_heads;
+  v.head_dim = kv->cfg.head_dim;
+  v.page_slots = kv->cfg.page_slots;
+  v.max_pages = kv->max_pages;
+  v.max_slots = kv->cfg.max_slots_per_seq;
+  v.pos_mode = kv->cfg.pos_mode;
+  cudaError_t e = ham::launch_append(v, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  return HAM_OK;
+}
+
+int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int32_t out_dtype,
+                       void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!q || !out) return fail(HAM_EINVAL, "q and out are required");
+  if (!aligned16(q) || !aligned16(out)) return fail(HAM_EINVAL, "q/out must be 16-byte aligned");
+  if (out_dtype != HAM_DTYPE_BF16 && out_dtype != HAM_DTYPE_F32)
+    return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
+  DeviceGuard guard(kv->device);
+  const int group = kv->cfg.n_q_heads / kv->cfg.n_kv_heads;
+  int ctas = kv->attn_ctas;
+  if (ctas <= 0) {
+    int per_sm = ham::attention_ctas_per_sm(kv->cfg.head_dim, group, kv->cfg.batch);
+    if (per_sm <= 0) return fail(HAM_ECUDA, "attention kernel cannot be resident on an SM");
+    ctas = kv->num_sms * per_sm;
+    if (ctas > kv->max_ctas) ctas = kv->max_ctas;
+  }
+  ham::AttnView v{};
+  v.k_pool = layer_pool(kv, layer, 0);
+  v.v_pool = layer_pool(kv, layer, 1);
+  v.page_table = kv->page_table;
+  v.num_slots = kv->num_slots + (size_t)layer * kv->cfg.batch;
+  v.q = static_cast<const uint16_t *>(q);
+  v.out = out;
+  v.part_acc = kv->part_acc;
+  v.part_ml = kv->part_ml;
+  v.tickets = kv->tickets;
+  v.err = kv->err;
+  v.pool_pages = kv->cfg.pool_pages;
+  v.batch = kv->cfg.batch;
+  v.n_kv_heads = kv->cfg.n_kv_heads;
+  v.page_slots = kv->cfg.page_slots;
+  v.max_pages = kv->max_pages;
+  v.max_slots = kv->cfg.max_slots_per_seq;
+  v.ctas = ctas;
+  cudaError_t e = ham::launch_attention(v, kv->cfg.head_dim, group, out_dtype,
+                                        static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+  return HAM_OK;
+}
+
+int ham_decode_attn(ham_kv *kv, int32_t layer, const void *q, void *out, void *stream) {
+  return ham_decode_attn_ex(kv, layer, q, out, HAM_DTYPE_BF16, stream);
+}
+
+int ham_kv_layer_lengths(ham_kv *kv, int32_t layer, int32_t *num_slots_host,
+                         int64_t *num_tokens_host, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  DeviceGuard guard(kv->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int B = kv->cfg.batch;
+  uint8_t *h = static_cast<uint8_t *>(kv->host_stage);
+  int32_t *h_err = reinterpret_cast<int32_t *>(h);
+  int64_t *h_tok = reinterpret_cast<int64_t *>(h + 64);
+  int32_t *h_slots = reinterpret_cast<int32_t *>(h + 64 + (size_t)B * 8);
+  HAM_CUDA(cudaMemcpyAsync(h_slots, kv->num_slots + (size_t)layer * B, B * sizeof(int32_t),
+                           cudaMemcpyDeviceToHost, s));
+  HAM_CUDA(cudaMemcpyAsync(h_tok, kv->num_tokens + (size_t)layer * B, B * sizeof(int64_t),
+                           cudaMemcpyDeviceToHost, s));
+  HAM_CUDA(cudaMemcpyAsync(h_err, kv->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+  HAM_CUDA(cudaStreamSynchronize(s));
+  if (num_slots_host) memcpy(num_slots_host, h_slots, B * sizeof(int32_t));
+  if (num_tokens_host) memcpy(num_tokens_host, h_tok, B * sizeof(int64_t));
+  if (*h_err != 0) return fail(HAM_EDEVICE, "device error word = %d", *h_err);
+  return HAM_OK;
+}
+
+int ham_slot_lengths(ham_kv *kv, int32_t *num_slots_host, int64_t *num_tokens_host,
+                     void *stream) {
+  if (!kv) return fail(HAM_EINVAL, "null handle");
+  return ham_kv_layer_lengths(kv, kv->cfg.layers - 1, num_slots_host, num_tokens_host, stream);
+}
+
+int ham_kv_status(ham_kv *kv, void *stream, int32_t *device_code) {
+  if (!kv) return fail(HAM_EINVAL, "null handle");
+  DeviceGuard guard(kv->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int32_t *h_err = static_cast<int32_t *>(kv->host_stage);
+  HAM_CUDA(cudaMemcpyAsync(h_err, kv->err, sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+  HAM_CUDA(cudaMemsetAsync(kv->err, 0, sizeof(int32_t), s));
+  HAM_CUDA(cudaStreamSynchronize(s));
+  if (device_code) *device_code = *h_err;
+  if (*h_err != 0) {
+    // A kernel that gave up mid-way may have left split tickets behind: clear them.
+    const size_t n_seg = (size_t)kv->cfg.batch * kv->cfg.n_kv_heads;
+    HAM_CUDA(cudaMemsetAsync(kv->tickets, 0, n_seg * sizeof(uint32_t), s));
+    HAM_CUDA(cudaStreamSynchronize(s));
+    return fail(HAM_EDEVICE, "device error word = %d", *h_err);
+  }
+  return HAM_OK;
+}
+
+int ham_kv_set_page_table(ham_kv *kv, const int32_t *host_pt) {
+  if (!kv || !host_pt) return fail(HAM_EINVAL, "null argument");
+  const size_t n = (size_t)kv->cfg.batch * kv->max_pages;
+  std::vector<uint8_t> used((size_t)kv->cfg.pool_pages, 0);
+  for (size_t i = 0; i < n; ++i) {
+    int32_t p = host_pt[i];
+    if (p < 0 || p >= kv->cfg.pool_pages)
+      return fail(HAM_EINVAL, "page table entry %zu = %d outside [0, %lld)", i, p,
+                  (long long)kv->cfg.pool_pages);
+    if (used[(size_t)p]++) return fail(HAM_EINVAL, "page %d appears twice", p);
+  }
+  DeviceGuard guard(kv->device);
+  HAM_CUDA(cudaDeviceSynchronize());
+  HAM_CUDA(cudaMemcpy(kv->page_table, host_pt, n * sizeof(int32_t), cudaMemcpyHostToDevice));
+  return HAM_OK;
+}
+
+int ham_kv_get_page_table(const ham_kv *kv, int32_t *host_pt) {
+  if (!kv || !host_pt) return fail(HAM_EINVAL, "null argument");
+  DeviceGuard guard(kv->device);
+  HAM_CUDA(cudaMemcpy(host_pt, kv->page_table,
+                      (size_t)kv->cfg.batch * kv->max_pages * sizeof(int32_t),
+                      cudaMemcpyDeviceToHost));
+  return HAM_OK;
+}
+
+int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
+                const int32_t *pos, const int32_t *ntok, const int32_t *counts, int32_t lmax,
+                void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!counts || lmax < 0 || (lmax > 0 && (!k_log || !v_log)))
+    return fail(HAM_EINVAL, "counts, lmax >= 0 and (for lmax > 0) k_log, v_log are required");
+  if ((k_log && !aligned16(k_log)) || (v_log && !aligned16(v_log)))
+    return fail(HAM_EINVAL, "k_log/v_log must be 16-byte aligned");
+  DeviceGuard guard(kv->device);
+  ham::FillView v{};
+  v.k_pool = layer_pool(kv, layer, 0);
+  v.v_pool = layer_pool(kv, layer, 1);
+  v.slot_pos = kv->slot_pos;
+  v.slot_ntok = kv->slot_ntok;
+  v.page_table = kv->page_table;
+  v.num_slots = kv->num_slots + (size_t)layer * kv->cfg.batch;
+  v.num_tokens = kv->num_tokens + (size_t)layer * kv->cfg.batch;
+  v.k_log = static_cast<const uint16_t *>(k_log);
+  v.v_log = static_cast<const uint16_t *>(v_log);
+  v.pos = pos;
+  v.ntok = ntok;
+  v.counts = counts;
+  v.err = kv->err;
+  v.pool_pages = kv->cfg.pool_pages;
+  v.batch = kv->cfg.batch;
+  v.n_kv_heads = kv->cfg.n_kv_heads;
+  v.head_dim = kv->cfg.head_dim;
+  v.page_slots = kv->cfg.page_slots;
+  v.max_pages = kv->max_pages;
+  v.max_slots = kv->cfg.max_slots_per_seq;
+  v.lmax = lmax;
+  cudaError_t e = ham::launch_fill(v, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "fill launch");
+  return HAM_OK;
+}
+
+int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *pos_dst,
+                  int32_t *ntok_dst, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  DeviceGuard guard(kv->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t pool_bytes = (size_t)kv->pool_elems * sizeof(uint16_t);
+  const size_t meta_bytes = (size_t)kv->cfg.pool_pages * kv->cfg.page_slots * sizeof(int32_t);
+  if (k_dst) HAM_CUDA(cudaMemcpyAsync(k_dst, layer_pool(kv, layer, 0), pool_bytes, cudaMemcpyDefault, s));
+  if (v_dst) HAM_CUDA(cudaMemcpyAsync(v_dst, layer_pool(kv, layer, 1), pool_bytes, cudaMemcpyDefault, s));
+  if (pos_dst) HAM_CUDA(cudaMemcpyAsync(pos_dst, kv->slot_pos, meta_bytes, cudaMemcpyDefault, s));
+  if (ntok_dst) HAM_CUDA(cudaMemcpyAsync(ntok_dst, kv->slot_ntok, meta_bytes, cudaMemcpyDefault, s));
+  return HAM_OK;
+}
+
+int ham_kv_reset(ham_kv *kv, void *stream) {
+  if (!kv) return fail(HAM_EINVAL, "null handle");
+  DeviceGuard guard(kv->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t n = (size_t)kv->cfg.layers * kv->cfg.batch;
+  HAM_CUDA(cudaMemsetAsync(kv->num_slots, 0, n * sizeof(int32_t), s));
+  HAM_CUDA(cudaMemsetAsync(kv->num_tokens, 0, n * sizeof(int64_t), s));
+  return HAM_OK;
+}
+
+int ham_split_plan(int32_t batch, int32_t n_kv_heads, const int32_t *num_slots_host,
+                   int32_t ctas, int64_t *cta_begin, int32_t *seg_first_cta,
+                   int32_t *seg_last_cta) {
+  if (batch < 1 || n_kv_heads < 1 || ctas < 1 || !num_slots_host)
+    return fail(HAM_EINVAL, "bad plan arguments");
+  std::vector<int64_t> cum((size_t)batch + 1, 0);
+  for (int32_t b = 0; b < batch; ++b) {
+    if (num_slots_host[b] < 0) return fail(HAM_EINVAL, "negative slot count");
+    cum[(size_t)b + 1] = cum[(size_t)b] + ham::chunks_of(num_slots_host[b]);
+  }
+  const int64_t W = (int64_t)n_kv_heads * cum[(size_t)batch];
+  const int32_t C = ham::plan_ctas(W, ctas);  // CTAs that get chunks; the rest stay idle
+  if (cta_begin)
+    for (int32_t c = 0; c <= ctas; ++c)
+      cta_begin[c] = C ? ham::plan_cta_begin(W, C, c < C ? c : C) : 0;
+  for (int32_t b = 0; b < batch; ++b) {
+    const int64_t nch = cum[(size_t)b + 1] - cum[(size_t)b];
+    for (int32_t g = 0; g < n_kv_heads; ++g) {
+      const int64_t s = (int64_t)b * n_kv_heads + g;
+      const int64_t x0 = (int64_t)n_kv_heads * cum[(size_t)b] + g * nch;
+      const int32_t first = nch ? ham::plan_owner(W, C, x0) : -1;
+      const int32_t last = nch ? ham::plan_owner(W, C, x0 + nch - 1) : -1;
+      if (seg_first_cta) seg_first_cta[s] = first;
+      if (seg_last_cta) seg_last_cta[s] = last;
+    }
+  }
+  return HAM_OK;
+}
+
+}  // extern "C"

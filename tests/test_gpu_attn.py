@@ -1,0 +1,149 @@
+"""GPU: split-KV decode attention matches the oracle (max-abs <= 2e-2, mean-abs <= 2e-3)."""
+import os
+import sys
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2505_20438_gb300 import ham
+from paper_2505_20438_gb300 import workload as wl
+
+from gpu_helpers import (MAX_ABS, MEAN_ABS, assert_parity, dev_bf16, dev_i32, gpu_cache,
+                         gpu_decode, small_case)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("hq,hkv,d,page,counts,scale", [
+    (8, 2, 64, 16, (37, 80), 1.0),                    # ragged tails inside a chunk
+    (8, 2, 64, 128, (256,), 1.0),                     # the tiny shape, 2 pages of 128
+    (32, 8, 128, 16, (1, 100, 1000), 1.0 / np.sqrt(128)),
+    (32, 8, 128, 16, (0, 17, 0, 4097), 1.0),          # empty sequences
+    (32, 8, 128, 32, (513, 2047), 1.0),
+    (8, 8, 128, 16, (300, 33), 1.0),                  # group 1
+    (16, 8, 128, 16, (300, 33), 1.0),                 # group 2
+    (64, 8, 128, 16, (300, 33), 1.0),                 # group 8
+    (8, 1, 64, 16, (300, 33), 1.0),                   # group 8, d 64
+    (2, 2, 64, 16, (70,), 1.0),                       # group 1, d 64
+])
+def test_decode_matches_oracle(hq, hkv, d, page, counts, scale):
+    case = small_case(batch=len(counts), hq=hq, hkv=hkv, d=d, page=page, counts=counts,
+                      scale=scale, seed=sum(counts) % 97)
+    ref = oracle.OracleCache.from_case(case).decode_attn(case.q)
+    kv = gpu_cache(case)
+    out32 = gpu_decode(kv, case.q, f32=True)
+    out16 = gpu_decode(kv, case.q, f32=False)
+    assert_parity(out16, ref, what="bf16 out")
+    assert_parity(out32, ref, max_abs=1e-4, mean_abs=1e-5, what="f32 out")
+    for b, n in enumerate(counts):                     # empty sequences give exactly 0
+        if n == 0:
+            assert np.all(out16[b] == 0) and np.all(out32[b] == 0)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+@pytest.mark.parametrize("ctas", [1, 2, 7, 152, 0, 1216])
+def test_split_count_invariance(ctas):
+    case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(2000, 35, 901), seed=11)
+    ref = oracle.OracleCache.from_case(case).decode_attn(case.q)
+    kv = gpu_cache(case)
+    ham.ham_kv_set_attn_ctas(kv, ctas)
+    out = gpu_decode(kv, case.q, f32=True)
+    assert_parity(out, ref, max_abs=1e-4, mean_abs=1e-5, what=f"ctas={ctas}")
+
+
+def test_repeated_launches_reuse_tickets():
+    """Split tickets are reset by the combining CTA: back-to-back launches agree exactly."""
+    case = small_case(batch=2, hq=32, hkv=8, d=128, page=16, counts=(3000, 1500), seed=12)
+    kv = gpu_cache(case)
+    outs = [gpu_decode(kv, case.q, f32=True) for _ in range(4)]
+    for o in outs[1:]:
+        assert np.array_equal(o, outs[0])
+
+
+def test_page_permutation_is_bitwise_invariant():
+    """The split plan depends on logical slot indices only: other pages, same bits."""
+    case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(700, 64, 1500), seed=13,
+                      pool_factor=2.0)
+    kv_a = gpu_cache(case)
+    perm = wl.rng_for(99).permutation(case.pool_pages)[: case.page_table.size]
+    kv_b = gpu_cache(case, page_table=perm.reshape(case.page_table.shape).astype(np.int32))
+    a = gpu_decode(kv_a, case.q, f32=True)
+    b = gpu_decode(kv_b, case.q, f32=True)
+    assert np.array_equal(a, b)
+
+
+def test_special_cases():
+    # one slot: the output is that slot's V
+    case = small_case(batch=2, hq=32, hkv=8, d=128, counts=(1, 1), seed=14)
+    out = gpu_decode(gpu_cache(case), case.q, f32=True)
+    v0 = wl.bf16_bits_to_f32(case.v[:, 0]).astype(np.float64)
+    for h in range(32):
+        assert np.allclose(out[:, h], v0[:, h // 4], atol=1e-6)
+    # a planted key far above the rest: online rescaling picks it wherever it sits
+    case = small_case(batch=1, hq=32, hkv=8, d=128, counts=(3000,), scale=0.05, seed=15)
+    q = wl.bf16_bits_to_f32(case.q[0, 0]).astype(np.float64)
+    for j, score in ((2999, 60.0), (5, 40.0), (1600, 50.0)):
+        case.k[0, j, 0] = wl.f32_to_bf16_bits((q * (score * np.sqrt(128) / (q @ q))).astype(np.float32))
+    ref = oracle.OracleCache.from_case(case).decode_attn(case.q)
+    out = gpu_decode(gpu_cache(case), case.q, f32=True)
+    assert_parity(out, ref, max_abs=1e-4, mean_abs=1e-5, what="planted")
+    v = wl.bf16_bits_to_f32(case.v[0, 2999, 0]).astype(np.float64)
+    assert np.allclose(out[0, 0], v, atol=1e-3)
+
+
+def test_tiny_workload_step_matches_fixture():
+    """The tiny workload end to end on the GPU (255 appends, then append + attend)."""
+    here = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+    sys.path.insert(0, here)
+    try:
+        import make_golden
+    finally:
+        sys.path.remove(here)
+    w = wl.C0_TINY
+    empty = wl.make_case(w, num_slots=np.zeros(1, np.int32), extra_slots=256)
+    prefill = wl.make_case(w)
+    kv = gpu_cache(empty, fill=False)
+    assert kv.max_pages == 2 and kv.pool_pages == 2
+    for n in range(w.slots):
+        ham.ham_kv_append(kv, 0, None, dev_bf16(prefill.k[:, n]), dev_bf16(prefill.v[:, n]),
+                          None, dev_i32(prefill.slot_ntok[:, n]))
+    q = dev_bf16(prefill.q)
+    ham.ham_kv_append(kv, 0, q, dev_bf16(prefill.k_new), dev_bf16(prefill.v_new), None,
+                      dev_i32(prefill.ntok_new))
+    import torch
+    out = torch.full(q.shape, float("nan"), dtype=torch.float32, device="cuda")
+    ham.ham_decode_attn_ex(kv, 0, q, out)
+    got = out.cpu().numpy().astype(np.float64)
+    lines = open(os.path.join(here, "tiny_step_oracle.txt")).read().splitlines()
+    ref = np.array([float(l) for l in lines if not l.startswith("#")]).reshape(got.shape)
+    assert_parity(got, ref, max_abs=1e-4, mean_abs=1e-5, what="tiny step")
+    slots, tokens = ham.ham_slot_lengths(kv)
+    ref_out, oc = make_golden.tiny_step()
+    assert list(slots) == [256] and list(tokens) == list(oc.num_tokens)
+
+
+# ---------------------------------------------------------------------------------------
+# full-size workloads, in the bench's launch configuration
+# ---------------------------------------------------------------------------------------
+
+def _full_size(w, sample_heads=None):
+    case = wl.make_case(w, extra_slots=4)
+    oc = oracle.OracleCache.from_case(case)
+    ref = oc.decode_attn(case.q)
+    kv = gpu_cache(case)
+    out = gpu_decode(kv, case.q, f32=False)
+    assert_parity(out, ref, what=w.name)
+    slots, _ = ham.ham_slot_lengths(kv)
+    assert np.array_equal(slots, case.num_slots)
+    return case, kv
+
+
+@pytest.mark.parametrize("w", [wl.C1_LLAMA8B, wl.C2_RAGGED, wl.C3_LONG], ids=lambda w: w.name)
+def test_full_size_workloads(w):
+    case, kv = _full_size(w)
+    # attend-then-append stays consistent: the appended slot is visible to the next step
+    ham.ham_kv_append(kv, 0, None, dev_bf16(case.k_new), dev_bf16(case.v_new), None,
+                      dev_i32(case.ntok_new))
+    slots, _ = ham.ham_slot_lengths(kv)
+    assert np.array_equal(slots, case.num_slots + 1)
