@@ -1,0 +1,540 @@
+#!/usr/bin/env python3
+"""Benchmark of smashed-KV decode attention (HAMburger macro-step hot path) on GB300.
+
+One step = one macro-step of one layer for the whole batch, through the C ABI:
+    ham_kv_append   (RoPE of q and k at the new slot's position, append of the slot)
+    ham_decode_attn (split-KV attention over all slots, combine)
+The default workload is the Llama-3-8B-shaped layer: batch 8, 32 query / 8 KV heads,
+head_dim 128, 4096 slots per sequence in 16-slot pages scattered over a shared pool.
+
+Timing: steps are captured in CUDA graphs (64 steps per graph) and replayed; the timed
+region is bracketed by a barrier and a device synchronize.  Four independent caches are
+rotated so each step reads a cache last touched three steps earlier (4 x 128 MiB of KV,
+far above the 129 MB L2).  After each graph the four caches are rolled back to 4096 slots
+(ham_kv_set_lengths), so the attended length stays 4097..4112.  The attention kernel's
+own duration comes from CUDA events recorded around each of its launches inside the graph.
+
+Prints ONE JSON line on rank 0.  `--impl reference` times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "macro-steps/s and achieved HBM GB/s (% of GB300 peak) for smashed-KV decode attn"
+UNIT = "macro-steps/s"
+GRAPH_STEPS = 64
+CACHES = 4
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=40960)
+    p.add_argument("--warmup", type=int, default=640)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="llama8b_layer_b8_s4096")
+    p.add_argument("--e2e-steps", type=int, default=2000)
+    p.add_argument("--cpu-seconds", type=float, default=12.0,
+                   help="CPU work budget of the oracle baseline sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+# ---------------------------------------------------------------------------------------
+# environment helpers
+# ---------------------------------------------------------------------------------------
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def measured_peak_hbm():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured (MEASURED_PEAKS.json hbm_gbs)"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for name in ("ham_attn.cu", "ham_internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2505_20438_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload_name):
+    """dram read+write bytes per attention launch from the committed ncu summary, if it was
+    taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", f"decode_attn_{workload_name}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    src = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", text)
+    tr = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
+    if not src or not tr or src.group(1) != kernel_source_hash():
+        return None
+    return int(tr.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 200 ms while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        except OSError:
+            pass
+        finally:
+            if self.path and os.path.exists(self.path):
+                os.remove(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        # samples "under load": the SM clock above half of its maximum
+        mx = num(rows[-1][2])
+        loaded = [x for x in sm if mx is None or x > 0.5 * mx] or sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None, "sm_max_mhz": mx,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max((num(r[3]) or 0.0) for r in rows)}
+
+
+# ---------------------------------------------------------------------------------------
+# workload
+# ---------------------------------------------------------------------------------------
+
+def workload(name):
+    from paper_2505_20438_gb300 import workload as wl
+    if name not in wl.WORKLOADS:
+        raise SystemExit(f"unknown workload {name}; choose from {sorted(wl.WORKLOADS)}")
+    w = wl.WORKLOADS[name]
+    if w.slot_range is not None or w.layers != 1:
+        raise SystemExit(f"bench times uniform single-layer workloads; {name} is a parity case")
+    return w
+
+
+def config_dict(w):
+    return {"workload": w.name, "batch": w.batch, "n_q_heads": w.n_q_heads,
+            "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim, "slots": w.slots,
+            "page_slots": w.page_slots, "pages": "scattered by a seeded shuffle of a shared pool",
+            "tokens_per_slot": "geometric p=0.5 capped at 4 (mean 1.875)",
+            "step": "ham_kv_append (RoPE q,k + append) then ham_decode_attn over all slots",
+            "l2": f"{CACHES} independent caches rotated ({CACHES} x "
+                  f"{w.batch * w.slots * w.n_kv_heads * w.head_dim * 4 / 2**20:.0f} MiB KV "
+                  "> 129 MB L2)",
+            "graph": f"{GRAPH_STEPS} steps per CUDA graph, rollback to {w.slots} slots per graph"}
+
+
+def attn_bytes(w, L):
+    """Algorithmic bytes of one attention launch with L slots per sequence: K and V of every
+    slot once, q in, out, and the page-table entries."""
+    kv = w.batch * L * w.n_kv_heads * w.head_dim * 2 * 2
+    qo = 2 * w.batch * w.n_q_heads * w.head_dim * 2
+    pt = w.batch * math.ceil(L / w.page_slots) * 4
+    return kv + qo + pt
+
+
+def append_bytes(w):
+    """Algorithmic bytes of one append: q read+write, k_new/v_new in, K/V rows out, metadata."""
+    return (2 * w.batch * w.n_q_heads * w.head_dim * 2 + 4 * w.batch * w.n_kv_heads * w.head_dim
+            + w.batch * 4 * 6)
+
+
+# ---------------------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------------------
+
+def build_caches(w, device_index, rank):
+    import numpy as np
+    import torch
+
+    from paper_2505_20438_gb300 import ham
+    from paper_2505_20438_gb300 import workload as wl
+
+    caches = []
+    max_slots = w.slots + GRAPH_STEPS // CACHES + 16
+    for r in range(CACHES):
+        seed = 1000 * w.seed + 10 * rank + r
+        kv = ham.ham_kv_alloc(1, w.batch, w.n_q_heads, w.n_kv_heads, w.head_dim, w.page_slots,
+                              max_slots, pool_pages=int(math.ceil(
+                                  w.batch * math.ceil(max_slots / w.page_slots) * w.pool_factor)),
+                              page_seed=seed + 1)
+        shape = (w.batch, w.slots, w.n_kv_heads, w.head_dim)
+        k = wl.device_normal_bf16(shape, w.value_scale, seed * 7 + 1)
+        v = wl.device_normal_bf16(shape, w.value_scale, seed * 7 + 2)
+        rng = wl.rng_for(seed, 5)
+        ntok = wl.ntok_capped_geometric(rng, (w.batch, w.slots))
+        counts = torch.full((w.batch,), w.slots, dtype=torch.int32, device="cuda")
+        ham.ham_kv_fill(kv, 0, k, v, counts, ntok=torch.from_numpy(ntok).cuda())
+        del k, v
+        tokens = torch.from_numpy(ntok.sum(axis=1).astype(np.int64)).cuda()
+        c = {
+            "kv": kv, "counts": counts, "tokens": tokens,
+            "q": wl.device_normal_bf16((w.batch, w.n_q_heads, w.head_dim), w.value_scale, seed * 7 + 3),
+            "k_new": wl.device_normal_bf16((w.batch, w.n_kv_heads, w.head_dim), w.value_scale, seed * 7 + 4),
+            "v_new": wl.device_normal_bf16((w.batch, w.n_kv_heads, w.head_dim), w.value_scale, seed * 7 + 5),
+            "ntok_new": torch.from_numpy(wl.ntok_capped_geometric(rng, (w.batch,))).cuda(),
+            "out": torch.empty((w.batch, w.n_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda"),
+            "mean_ntok": float(ntok.mean()),
+        }
+        caches.append(c)
+    torch.cuda.synchronize()
+    return caches
+
+
+def run_ours(args, w):
+    import torch
+
+    from paper_2505_20438_gb300 import build as build_mod
+    from paper_2505_20438_gb300 import ham
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    build_mod.build()
+    caches = build_caches(w, local_rank, rank)
+    stream = torch.cuda.Stream()
+    n_graph = max(1, math.ceil(args.steps / GRAPH_STEPS))
+    n_warm = max(1, math.ceil(max(args.warmup, 3) / GRAPH_STEPS))
+    steps = n_graph * GRAPH_STEPS
+
+    def one_step(c):
+        ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
+        ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+
+    def rollback():
+        for c in caches:
+            ham.ham_kv_set_lengths(c["kv"], 0, c["counts"], c["tokens"])
+
+    # eager warm-up (first launches configure the kernels outside of capture)
+    with torch.cuda.stream(stream):
+        for i in range(2 * CACHES):
+            one_step(caches[i % CACHES])
+        rollback()
+    stream.synchronize()
+
+    try:
+        ev = [(torch.cuda.Event(enable_timing=True, external=True),
+               torch.cuda.Event(enable_timing=True, external=True)) for _ in range(GRAPH_STEPS)]
+        per_launch_method = ("CUDA events around every ham_decode_attn (attention + combine "
+                             "kernels) of the last graph replay of the timed region")
+    except TypeError:
+        ev = None
+        per_launch_method = "attention-only graph, CUDA events around the replay"
+
+    def capture(with_events):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(GRAPH_STEPS):
+                c = caches[i % CACHES]
+                ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
+                if with_events:
+                    ev[i][0].record()
+                ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+                if with_events:
+                    ev[i][1].record()
+            rollback()
+        return g
+
+    # the timed loop replays an event-free graph (events would cut the programmatic
+    # dependent launch between kernels); the last replay is an identical graph with events
+    graph = capture(False)
+    probe = capture(True) if ev is not None else graph
+    launches_per_graph = 3 * GRAPH_STEPS + CACHES   # append, attention, combine; rollbacks
+
+    # attended lengths inside one graph: cache i % 4 sees w.slots + 1 + i // 4 slots
+    lengths = [w.slots + 1 + i // CACHES for i in range(GRAPH_STEPS)]
+    attn_bytes_graph = sum(attn_bytes(w, L) for L in lengths)
+    step_bytes_graph = attn_bytes_graph + GRAPH_STEPS * append_bytes(w)
+
+    with torch.cuda.stream(stream):          # replay() launches on the current stream
+        for _ in range(n_warm):
+            graph.replay()
+        probe.replay()
+    torch.cuda.synchronize()
+    for c in caches:
+        if ham.ham_kv_status(c["kv"]) != ham.HAM_DEVERR_NONE:
+            raise RuntimeError("device error during warm-up")
+
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks, torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(n_graph - 1):
+            graph.replay()
+        probe.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed_ms = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([elapsed_ms], device="cuda", dtype=torch.float64)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(tt.item())
+        torch.distributed.barrier()
+
+    # attention kernel duration (last replay of the timed region)
+    if ev is not None:
+        attn_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(GRAPH_STEPS)]
+    else:
+        g2 = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g2, stream=stream):
+            for i in range(GRAPH_STEPS):
+                c = caches[i % CACHES]
+                ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            a0.record(stream)
+            g2.replay()
+            a1.record(stream)
+        torch.cuda.synchronize()
+        attn_ms = [a0.elapsed_time(a1) / GRAPH_STEPS] * GRAPH_STEPS
+    for c in caches:
+        if ham.ham_kv_status(c["kv"]) != ham.HAM_DEVERR_NONE:
+            raise RuntimeError("device error during the timed region")
+
+    peak, peak_src = measured_peak_hbm()
+    attn_gbs = attn_bytes_graph / (sum(attn_ms) * 1e-3) / 1e9
+    ms_per_step = elapsed_ms / steps
+    value = world * steps / (elapsed_ms * 1e-3)
+    step_gbs = world * n_graph * step_bytes_graph / (elapsed_ms * 1e-3) / 1e9
+    mean_ntok = statistics.mean(c["mean_ntok"] for c in caches)
+
+    e2e = run_e2e(args, w, caches, stream, rollback, world)
+
+    traffic = profiled_traffic(w.name)
+    result = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+        "steps": steps, "warmup": n_warm * GRAPH_STEPS, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "accum_dtype": "f32", "data": "synthetic", "config": config_dict(w),
+        "kv_gbs": round(step_gbs, 1),
+        "kv_frac_of_measured_peak": round(step_gbs / world / peak, 4),
+        "kv_frac_of_8tbs_spec": round(step_gbs / world / 8000.0, 4),
+        "slots_per_s": round(value * w.batch, 1),
+        "tokens_per_s": round(value * w.batch * mean_ntok, 1),
+        "roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
+                     "unit": "GB/s", "frac": round(attn_gbs / peak, 4), "traffic": traffic,
+                     "kernel": "decode_attn_kernel<128,bf16> + combine_kernel<bf16>",
+                     "avg_launch_us": round(1e3 * statistics.mean(attn_ms), 3),
+                     "algorithmic_bytes_per_launch": int(attn_bytes_graph / GRAPH_STEPS),
+                     "peak_source": peak_src, "duration_method": per_launch_method},
+        "gpu_launches": n_graph * launches_per_graph * world,
+        "e2e": e2e,
+        "clocks": clocks.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def run_e2e(args, w, caches, stream, rollback, world):
+    """Same steps through the public API with pinned host inputs copied in and the output
+    copied back and read on the host every step."""
+    import torch
+
+    from paper_2505_20438_gb300 import ham
+
+    host = []
+    for c in caches:
+        host.append({k: c[k].cpu().pin_memory() for k in ("q", "k_new", "v_new", "ntok_new")})
+        host[-1]["out"] = torch.empty(c["out"].shape, dtype=c["out"].dtype).pin_memory()
+    h2d = sum(host[0][k].numel() * host[0][k].element_size() for k in ("q", "k_new", "v_new", "ntok_new"))
+    d2h = host[0]["out"].numel() * host[0]["out"].element_size()
+    n = max(GRAPH_STEPS, (args.e2e_steps // GRAPH_STEPS) * GRAPH_STEPS)
+    checksum = 0.0
+    with torch.cuda.stream(stream):
+        for i in range(2 * CACHES):        # warm the eager path
+            c, h = caches[i % CACHES], host[i % CACHES]
+            ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
+            ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+        rollback()
+        stream.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        t = time.perf_counter()
+        for i in range(n):
+            c, h = caches[i % CACHES], host[i % CACHES]
+            for k in ("q", "k_new", "v_new", "ntok_new"):
+                c[k].copy_(h[k], non_blocking=True)
+            ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
+            ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+            h["out"].copy_(c["out"], non_blocking=True)
+            stream.synchronize()
+            checksum += float(h["out"][0, 0, 0])      # the host reads the step's result
+            if (i + 1) % GRAPH_STEPS == 0:
+                rollback()
+        stream.synchronize()
+        dt = time.perf_counter() - t
+    if world > 1:
+        tt = torch.tensor([dt], device="cuda", dtype=torch.float64)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        dt = float(tt.item())
+    return {"value": round(world * n / dt, 2), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": n,
+            "path": "pinned host -> device copies, ham_kv_append, ham_decode_attn, "
+                    "device -> pinned host copy, host sync, every step (eager)",
+            "finite": math.isfinite(checksum)}
+
+
+# ---------------------------------------------------------------------------------------
+# CPU oracle: baseline leg and reference arm
+# ---------------------------------------------------------------------------------------
+
+def oracle_case(w):
+    import oracle
+    from paper_2505_20438_gb300 import workload as wl
+    oracle.build()
+    case = wl.make_case(w, extra_slots=4)
+    return oracle, case, oracle.OracleCache.from_case(case)
+
+
+def cpu_baseline(w, seconds):
+    """Full macro-steps (append + attention of every head) of the oracle for ~`seconds`."""
+    oracle, case, oc = oracle_case(w)
+    n, t0 = 0, time.perf_counter()
+    while True:
+        q = case.q.copy()
+        oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q)
+        oc.decode_attn(q)
+        oc.num_slots[:] = case.num_slots          # keep the workload at its slot count
+        n += 1
+        dt = time.perf_counter() - t0
+        if dt >= seconds or n >= 10000:
+            break
+    return {"value": round(n / dt, 4), "unit": UNIT, "cores": oracle.max_threads(),
+            "kind": "oracle",
+            "sample": f"{n} full macro-steps (append + attention of all {w.batch * w.n_q_heads} "
+                      f"query heads over {w.slots} slots) of {w.name}, fp64 C oracle, "
+                      f"OpenMP over (sequence, head)"}
+
+
+def run_reference(args, w):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    import dataclasses
+
+    import oracle
+    from paper_2505_20438_gb300 import workload as wl
+    oracle.build()
+    steps = max(1, args.steps)
+    warm = max(3, args.warmup)
+    # Each step runs the oracle as it stands (append + OpenMP attention of every head) on a
+    # sub-case of the workload: fewer sequences, or one sequence with fewer slots, sized so
+    # the whole run is about 40 full macro-steps of oracle work.  Attention work is linear
+    # in the slot count, so the value is scaled by the sampled fraction of slots.
+    frac = min(1.0, 40.0 / (steps + warm))
+    if frac * w.batch >= 1.0:
+        sub_b, sub_l = max(1, int(round(frac * w.batch))), w.slots
+    else:
+        sub_b, sub_l = 1, max(16, int(round(frac * w.batch * w.slots)))
+    sub = dataclasses.replace(w, batch=sub_b, slots=sub_l)
+    case = wl.make_case(sub, extra_slots=4)
+    oc = oracle.OracleCache.from_case(case)
+    def one():
+        q = case.q.copy()
+        oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q)
+        oc.decode_attn(q)
+        oc.num_slots[:] = case.num_slots
+    for _ in range(warm):
+        one()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+    dt = time.perf_counter() - t0
+    share = (sub_b * sub_l) / (w.batch * w.slots)
+    value = steps * share / dt
+    sample = (f"each step: append + attention of all heads for {sub_b} sequence(s) x {sub_l} "
+              f"slots = {share:.4f} of a {w.name} macro-step; {steps} steps timed")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+        "n_gpus": world, "steps": steps, "warmup": warm,
+        "ms_per_step": round(1e3 / value, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config_dict(w),
+        "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": oracle.max_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main():
+    args = parse_args()
+    w = workload(args.workload)
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

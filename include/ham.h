@@ -87,7 +87,7 @@ typedef struct ham_kv_info {
   int32_t num_sms;           /* SMs of the device the handle lives on */
   int32_t device;            /* CUDA device ordinal */
   int64_t pool_bytes;        /* K+V bytes of ONE layer's pool */
-  int64_t scratch_bytes;     /* split-attention partials + tickets */
+  int64_t scratch_bytes;     /* split-attention partials and per-segment CTA ranges */
 } ham_kv_info;
 
 /* ------------------------------------------------------------------------------------
@@ -131,9 +131,10 @@ int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
 /* One decode step of one layer: every query head attends over all slots of its sequence
  * (softmax(q K^T / sqrt(head_dim)) V over the slot list; no weighting by token count).
  * Query head h reads KV head h / (n_q_heads / n_kv_heads).  Split-KV: the slots of all
- * (sequence, KV head) pairs are cut into equal contiguous ranges, one per CTA, and the
- * partial softmax states of a pair are merged by the last CTA that finishes it.  Sequences
- * with no slots give 0.  Slot counts are read on the device (no host sync).
+ * (sequence, KV head) pairs are cut into equal contiguous ranges, one per CTA, and a second
+ * kernel merges the partial softmax states of pairs that span several CTAs (two launches on
+ * `stream`, the second with programmatic dependent launch).  Sequences with no slots give 0.
+ * Slot counts are read on the device (no host sync).
  * q    device bf16 [batch][n_q_heads][head_dim], already rotated (e.g. by ham_kv_append)
  * out  device bf16 [batch][n_q_heads][head_dim]
  * Host errors: HAM_EINVAL, HAM_ECUDA.  Calls on one handle must not overlap in time (they
@@ -193,6 +194,14 @@ int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
  * pool_pages * page_slots int32 each.  Any destination may be NULL. */
 int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *pos_dst,
                   int32_t *ntok_dst, void *stream);
+
+/* Set the slot and token counters of one layer from device arrays (e.g. to roll back the
+ * slots of a rejected macro-step): num_slots [batch] int32, num_tokens [batch] int64
+ * (nullable: tokens unchanged).  Slots at or past the new count are free and the next
+ * append overwrites them.  A count outside [0, max_slots_per_seq] sets the device error
+ * word and leaves that sequence unchanged.  One small kernel; can be captured in a graph. */
+int ham_kv_set_lengths(ham_kv *kv, int32_t layer, const int32_t *num_slots,
+                       const int64_t *num_tokens, void *stream);
 
 /* Set every sequence of every layer back to 0 slots / 0 tokens (pages stay reserved). */
 int ham_kv_reset(ham_kv *kv, void *stream);

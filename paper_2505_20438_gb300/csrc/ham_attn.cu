@@ -4,31 +4,33 @@
 // Sec. 3.6 "Token Fusion"), so a decode step is plain softmax attention of each query head
 // over the slot list of its sequence, scale 1/sqrt(d), query head h reading KV head h / G
 // (Llama-3.2 base model, Sec. 4.1).  Decoding re-reads the whole cache every step and is
-// bound by memory bandwidth (Sec. 2.3), so the kernel is built around moving every K/V
-// byte from HBM exactly once per (sequence, KV head):
+// bound by memory bandwidth (Sec. 2.3), so the kernel moves every K/V byte from HBM once
+// per (sequence, KV head) and keeps everything else off the critical path:
 //
 //  * Split plan: the 16-slot chunks of all (sequence, KV head) segments are numbered
-//    contiguously and cut into gridDim.x equal ranges, one per CTA (ham_internal.cuh).
-//    Ragged batches balance for free; the plan is computed on the device from the slot
-//    counters, so the launch never waits on the host.
-//  * Producer warp: one lane issues 1-D bulk copies (cp.async.bulk, the TMA engine) of a
-//    chunk's K rows and V rows (each one contiguous block inside a page) into a ring of
-//    shared-memory stages, completing on an mbarrier, with an L2 evict-first hint.  The
-//    query heads of a segment ride on the first stage of the segment.
-//  * Consumer warps: a chunk's 16 slots are split over the consumer warps; a slot's
-//    head_dim values are spread over kLanesPerSlot lanes (16-byte conflict-free shared
-//    loads).  q.k partials of the G heads use packed fp32 FMAs (__ffma2_rn), then a
-//    reduce-scatter over the slot's lanes leaves each lane one head's score, with no
-//    selects because every lane keeps its heads in the order (i XOR its own head).  The
-//    online softmax is fp32 in the exp2 domain with a lazy running max (rescale only when
-//    a score exceeds the running max by more than 2^8).
-//  * Combine: at the end of a segment the consumer warps merge their states in shared
-//    memory; a segment covered by one CTA is written directly, otherwise the CTA writes a
-//    partial (max, sum, acc) and the last CTA to finish the segment (atomic ticket) merges
-//    the partials in CTA order, so the result does not depend on timing or page ids.
+//    contiguously and cut into equal ranges, one per CTA (ham_internal.cuh).  Ragged
+//    batches balance for free; the plan is computed on the device from the slot counters,
+//    so the launch never waits on the host.
+//  * Producer warp: one lane issues TMA tensor copies (cp.async.bulk.tensor, 128-byte
+//    swizzle) of a chunk's K rows and V rows into a shared-memory ring, completing on
+//    mbarriers, with an L2 evict-first hint.  The swizzle keeps the ldmatrix reads below
+//    free of bank conflicts (head_dim 64) or 2-way (head_dim 128).  The query heads of a
+//    segment ride on the first stage of that segment (1-D bulk copy).
+//  * Consumer warp: the G query heads of the group are padded to 8 and a chunk is a
+//    16 x head_dim x 8 contraction on the tensor cores (mma.sync m16n8k16, bf16 in, fp32
+//    accumulate): S^T = K Q^T with slots as rows, then O^T += V^T P^T with P^T moved into
+//    the B-operand layout by movmatrix.  The online softmax is fp32 in the exp2 domain with
+//    a lazy running max (rescale only when a score exceeds it by more than 2^8).
+//  * Combine: a segment covered by one CTA is written directly; otherwise each CTA writes a
+//    partial (max, sum, acc) and a second, fully parallel kernel (one thread per output
+//    element, launched with programmatic dependent launch so its launch overlaps this
+//    kernel's tail) merges the partials in CTA order.  The result does not depend on
+//    timing or page ids.  (A fused last-CTA merge was measured first: one warp merging
+//    ~15 partials through L2 serialised 12-18 us at the end of every launch.)
 //
 // Every wait is bounded (about 2 s); a wait that runs out records HAM_DEVERR_TIMEOUT,
 // lets the CTA's copies land and returns.  No trap, no unbounded spin.
+#include <cuda.h>
 #include <cuda_bf16.h>
 
 #include <mutex>
@@ -43,6 +45,7 @@ constexpr uint32_t kFull = 0xffffffffu;
 constexpr float kRescaleSlack = 8.0f;              // log2 units
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // bounded waits: 2 s
 constexpr int kFirst = 1, kLast = 2, kPageOk = 4;  // stage flags
+constexpr int kMaxGroup = 8;                       // heads padded to the MMA's N = 8
 
 // ------------------------------------------------------------------------------------
 // PTX wrappers
@@ -61,6 +64,9 @@ __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
 }
 __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
@@ -85,15 +91,7 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
-// 1-D bulk copy global -> shared through the TMA engine; 16-byte aligned, size % 16 == 0.
-__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes,
-                                          uint64_t *bar, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
-      : "memory");
-}
+// 1-D bulk copy global -> shared (TMA engine); 16-byte aligned, size % 16 == 0.
 __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes,
                                           uint64_t *bar) {
   asm volatile(
@@ -102,17 +100,59 @@ __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t b
       "l"(src), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
 }
+// Rank-3 tiled TMA copy of the box at (x, y, z) of `map` into shared memory.
+__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int x, int y,
+                                            int z, uint64_t *bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)),
+      "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+// D += A * B for one 16x8x16 tile: A 16x16 bf16 (row), B 16x8 bf16 (col), D fp32.
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                          uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// Two fp32 -> packed bf16 (round to nearest even): lo in bits 0..15, hi in 16..31.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
-}
-// Two bf16 packed in a 32-bit word (element 2j low, 2j+1 high) -> exact fp32 pair.
-__device__ __forceinline__ float2 bf16x2_to_float2(uint32_t w) {
-  return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
-}
-__device__ __forceinline__ uint32_t word_of(const uint4 &v, int j) {
-  return j == 0 ? v.x : j == 1 ? v.y : j == 2 ? v.z : v.w;
 }
 
 // One thread waits on an mbarrier phase, bounded.  honor_abort: give up early once another
@@ -145,42 +185,6 @@ __device__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort_fl
   }
 }
 
-// ------------------------------------------------------------------------------------
-// Shape of one kernel instance
-// ------------------------------------------------------------------------------------
-constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
-
-template <int D, int G, int E>
-struct Shape {
-  static constexpr int kLanesPerSlot = D / E;                  // lanes sharing one slot row
-  static constexpr int kSlotsPerWarp = 32 / kLanesPerSlot;
-  static constexpr int kConsumerWarps = kChunkSlots / kSlotsPerWarp;
-  static constexpr int kPieces = E / 8;                        // 16-byte pieces per lane
-  static constexpr int kHeadLanes = kLanesPerSlot / G;         // lanes left holding one head
-  static constexpr int kChunkBytes = kChunkSlots * D * 2;      // K (or V) rows of a chunk
-  static constexpr int kStageBytes = 2 * kChunkBytes;
-  static constexpr int kStages = D == 128 ? 8 : 12;
-  static constexpr int kQBufs = kStages + 1;
-  static constexpr int kQBytes = G * D * 2;
-  static constexpr int kThreads = 32 * (kConsumerWarps + 1);
-  static constexpr int kConsumerThreads = 32 * kConsumerWarps;
-  // q and acc take 4*G*E/2 registers; two CTAs per SM while that leaves room (~200/thread)
-  static constexpr int kMinBlocks = kThreads * (2 * G * E + 48) <= 32768 ? 2 : 1;
-  // shared memory map
-  static constexpr int kOffQ = kStages * kStageBytes;
-  static constexpr int kOffBar = kOffQ + kQBufs * kQBytes;
-  static constexpr int kOffInfo = align_up(kOffBar + (2 * kStages + 1) * 8, 16);
-  static constexpr int kOffMergeAcc = kOffInfo + kStages * 16;
-  static constexpr int kOffMergeML = kOffMergeAcc + kConsumerWarps * G * D * 4;
-  static constexpr int kOffFlags = kOffMergeML + kConsumerWarps * G * 8;
-  static constexpr int kOffCum = kOffFlags + 16;
-  static size_t smem_bytes(int batch) { return (size_t)kOffCum + 4u * (2u * batch + 1u); }
-
-  static_assert(D % E == 0 && E % 8 == 0, "lane slice must be whole 16-byte pieces");
-  static_assert(32 % kLanesPerSlot == 0 && kChunkSlots % kSlotsPerWarp == 0, "lane layout");
-  static_assert(G >= 1 && G <= kLanesPerSlot && kLanesPerSlot % G == 0, "group vs lanes");
-};
-
 template <typename OutT>
 __device__ __forceinline__ void store_out(void *out, int64_t i, float x) {
   if constexpr (std::is_same<OutT, float>::value)
@@ -189,67 +193,83 @@ __device__ __forceinline__ void store_out(void *out, int64_t i, float x) {
     static_cast<__nv_bfloat16 *>(out)[i] = __float2bfloat16_rn(x);
 }
 
-// Reduce-scatter of the G partial scores over the kLanesPerSlot lanes of a slot.  v[i]
-// holds the lane's partial of head (i ^ hsel); afterwards the return value is the full
-// score of head hsel.  (Partner lane c ^ m has hsel ^ (G/2...) so its upper half holds the
-// heads of our lower half.)
-template <int G, int LPS>
-__device__ __forceinline__ float reduce_scores(float (&v)[G]) {
-#pragma unroll
-  for (int n = G, m = LPS / 2; n > 1; n >>= 1, m >>= 1) {
-#pragma unroll
-    for (int i = 0; i < n / 2; ++i) v[i] += __shfl_xor_sync(kFull, v[i + n / 2], m);
-  }
-  float s = v[0];
-#pragma unroll
-  for (int m = LPS / (2 * G); m >= 1; m >>= 1) s += __shfl_xor_sync(kFull, s, m);
-  return s;
-}
+// ------------------------------------------------------------------------------------
+// Shape of one kernel instance
+// ------------------------------------------------------------------------------------
+constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
-// Consumer-warp barrier on an mbarrier (bounded; returns false on timeout/abort).
-__device__ __forceinline__ bool consumer_sync(uint64_t *bar, uint32_t &phase,
-                                              volatile int *flags) {
-  __syncwarp();
-  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
-  const bool ok = warp_wait(bar, phase, flags);
-  phase ^= 1u;
-  return ok;
+template <int D>
+struct Shape {
+  static constexpr int kChunkBytes = kChunkSlots * D * 2;   // K (or V) rows of one chunk
+  static constexpr int kStageBytes = 2 * kChunkBytes;
+  static constexpr int kStages = 32768 / kStageBytes;       // 32 KiB ring
+  static constexpr int kQBufs = kStages + 1;
+  static constexpr int kQBytes = kMaxGroup * D * 2;
+  static constexpr int kThreads = 64;                       // consumer warp, producer warp
+  static constexpr int kSteps = D / 16;                     // k-steps of q.k, m-tiles of p.v
+  static constexpr int kLinesPerRow = D / 64;               // 128-byte swizzle lines per row
+  // shared memory map (offsets from a 1024-byte aligned base)
+  static constexpr int kOffQ = kStages * kStageBytes;
+  static constexpr int kOffBar = kOffQ + kQBufs * kQBytes;
+  static constexpr int kOffInfo = align_up(kOffBar + (2 * kStages) * 8, 16);
+  static constexpr int kOffFlags = kOffInfo + kStages * 16;
+  static constexpr int kOffCum = kOffFlags + 16;
+  static size_t smem_bytes(int batch) {
+    return 1024 + (size_t)kOffCum + 4u * (2u * batch + 1u);
+  }
+  static_assert(D == 64 || D == 128, "head_dim 64 or 128");
+  static_assert(kStages >= 2, "ring depth");
+};
+
+// Byte offset of the 16-byte piece `c` (elements c*8 .. c*8+7) of slot row `slot` inside a
+// chunk tile written by the swizzled TMA copy: rows are split into 128-byte lines
+// (line = slot * D/64 + c / 8) and the piece index inside a line is XORed with line % 8.
+template <int D>
+__device__ __forceinline__ uint32_t tile_offset(int slot, int c) {
+  const int line = slot * Shape<D>::kLinesPerRow + (c >> 3);
+  return (uint32_t)(line * 128 + (((c & 7) ^ (line & 7)) << 4));
 }
 
 // ------------------------------------------------------------------------------------
 // The kernel
 // ------------------------------------------------------------------------------------
-template <int D, int G, int E, typename OutT>
-__global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMinBlocks)
-    decode_attn_kernel(const AttnView v) {
-  using S = Shape<D, G, E>;
-  constexpr int LPS = S::kLanesPerSlot;
-  extern __shared__ __align__(128) uint8_t smem[];
+template <int D, typename OutT>
+__global__ void __launch_bounds__(Shape<D>::kThreads)
+    decode_attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                       const __grid_constant__ CUtensorMap tmap_v, const AttnView v) {
+  using S = Shape<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t *stages = smem;
   uint8_t *qbufs = smem + S::kOffQ;
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + S::kOffBar);
   uint64_t *empty = full + S::kStages;
-  uint64_t *sync_bar = empty + S::kStages;
   int4 *info = reinterpret_cast<int4 *>(smem + S::kOffInfo);
-  float *merge_acc = reinterpret_cast<float *>(smem + S::kOffMergeAcc);
-  float2 *merge_ml = reinterpret_cast<float2 *>(smem + S::kOffMergeML);
-  volatile int *flags = reinterpret_cast<volatile int *>(smem + S::kOffFlags);  // abort, last
+  volatile int *flags = reinterpret_cast<volatile int *>(smem + S::kOffFlags);  // abort
   int32_t *cum = reinterpret_cast<int32_t *>(smem + S::kOffCum);  // [B+1] chunk prefix
   int32_t *lens = cum + v.batch + 1;                               // [B] slots
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int B = v.batch, Hkv = v.n_kv_heads;
+  const int B = v.batch, Hkv = v.n_kv_heads, G = v.group;
 
   if (tid == 0) {
     for (int s = 0; s < S::kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], S::kConsumerWarps);
+      mbar_init(&empty[s], 1);
     }
-    mbar_init(sync_bar, S::kConsumerWarps);
     flags[0] = 0;
-    flags[1] = 0;
     fence_mbar_init();
   }
+  if (tid == 32) {
+    prefetch_tensormap(&tmap_k);
+    prefetch_tensormap(&tmap_v);
+  }
+  // Programmatic dependent launch: everything above overlaps the previous kernel's tail;
+  // slot counters, q and the pools are read only after it has completed.  The combine
+  // kernel that follows may be scheduled now (it waits for this grid to finish).
+  grid_dependency_wait();
+  grid_launch_dependents();
   if (warp == 0) {  // chunks per sequence and their prefix sums
     int run = 0;
     for (int b0 = 0; b0 < B; b0 += 32) {
@@ -285,6 +305,7 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
     if (cum[b + 1] != cum[b]) continue;
     for (int idx = tid; idx < G * D; idx += blockDim.x)
       store_out<OutT>(v.out, (int64_t)s * G * D + idx, 0.f);
+    if (tid == 0) v.seg_range[s] = make_int2(-1, -1);
   }
   // Only min(gridDim.x, W) CTAs take part, so that every range holds at least one chunk:
   // the CTAs touching a segment are then exactly first..last (no idle CTA in between).
@@ -295,13 +316,13 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
   const int nchunks = (int)(x1 - x0);
 
   // ---------------------------------------------------------------- producer warp
-  if (warp == S::kConsumerWarps) {
+  if (warp == 1) {
     const uint64_t pol = policy_evict_first();
+    const uint32_t qbytes = (uint32_t)(G * D * 2);
     int it = 0, nseg = 0;
     for (int base = 0; base < nchunks; base += 32) {
       const int nb = min(32, nchunks - base);
-      int seg = 0, valid = 0, fl = 0;
-      long long off = 0;
+      int seg = 0, valid = 0, fl = 0, row0 = 0;
       if (lane < nb) {  // decode chunk x0 + base + lane
         const int64_t x = x0 + base + lane;
         int lo = 0, hi = B - 1;
@@ -318,8 +339,7 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
         const int slot0 = c * kChunkSlots;
         const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
         const bool page_ok = page >= 0 && page < v.pool_pages;
-        off = (((long long)(page_ok ? page : 0) * Hkv + g) * v.page_slots +
-               slot0 % v.page_slots) * D;
+        row0 = ((page_ok ? page : 0) * Hkv + g) * v.page_slots + slot0 % v.page_slots;
         fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
              ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
       }
@@ -328,7 +348,7 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
         const int s_seg = __shfl_sync(kFull, seg, j);
         const int s_valid = __shfl_sync(kFull, valid, j);
         const int s_fl = __shfl_sync(kFull, fl, j);
-        const long long s_off = __shfl_sync(kFull, off, j);
+        const int s_row = __shfl_sync(kFull, row0, j);
         int failed = 0;
         if (lane == 0) {
           const int stage = it % S::kStages;
@@ -342,18 +362,18 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
             if (s_fl & kFirst) qb = nseg++ % S::kQBufs;
             info[stage] = make_int4(s_seg, s_valid, s_fl, qb);
             uint32_t bytes = (s_fl & kPageOk) ? (uint32_t)S::kStageBytes : 0u;
-            if (qb >= 0) bytes += S::kQBytes;
+            if (qb >= 0) bytes += qbytes;
             if (bytes) mbar_arrive_tx(&full[stage], bytes);
             else mbar_arrive(&full[stage]);
             uint8_t *dst = stages + stage * S::kStageBytes;
             if (s_fl & kPageOk) {
-              bulk_load(dst, v.k_pool + s_off, S::kChunkBytes, &full[stage], pol);
-              bulk_load(dst + S::kChunkBytes, v.v_pool + s_off, S::kChunkBytes, &full[stage], pol);
+              tma_load_3d(dst, &tmap_k, 0, 0, s_row, &full[stage], pol);
+              tma_load_3d(dst + S::kChunkBytes, &tmap_v, 0, 0, s_row, &full[stage], pol);
             } else {
               record_error(v.err, HAM_DEVERR_PAGE);
             }
             if (qb >= 0)
-              bulk_load(qbufs + qb * S::kQBytes, v.q + (int64_t)s_seg * G * D, S::kQBytes,
+              bulk_load(qbufs + qb * S::kQBytes, v.q + (int64_t)s_seg * G * D, qbytes,
                         &full[stage]);
           }
         }
@@ -373,24 +393,26 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
     return;
   }
 
-  // ---------------------------------------------------------------- consumer warps
-  const int sg = lane / LPS, c = lane % LPS;
-  const int hsel = c / S::kHeadLanes;           // the head this lane's score ends up in
-  const int slot = warp * S::kSlotsPerWarp + sg;  // slot within the chunk
-  const int ctid = warp * 32 + lane;
+  // ---------------------------------------------------------------- consumer warp
+  // Fragment coordinates (mma.sync m16n8k16): row r0 / r0 + 8, column pair 2 * cq.
+  const int r0 = lane >> 2, cq = lane & 3;
+  const int h0 = 2 * cq, h1 = 2 * cq + 1;  // the two heads of this lane's S / O columns
+  const bool hv0 = h0 < G, hv1 = h1 < G;
   const float qscale = rsqrtf((float)D) * 1.4426950408889634f;  // 1/sqrt(d) * log2(e)
+  // ldmatrix row addresses (per lane) inside a chunk tile
+  const int a_slot = 8 * ((lane >> 3) & 1) + (lane & 7);  // K as A: rows 0-15, k-halves
+  const int a_half = lane >> 4;
+  const int v_slot = 8 * (lane >> 4) + (lane & 7);        // V^T as A (transposed load)
+  const int v_half = (lane >> 3) & 1;
 
-  float2 q2[G][E / 2];   // [i]: head (i ^ hsel), this lane's elements, pre-scaled
-  float2 acc[G][E / 2];  // same head order
-  float m[G];            // running max per head (same order), uniform over the warp
-  float l_own = 0.f;     // running sum of this lane's head over its slots
+  uint32_t qb[S::kSteps][2];  // B fragments of Q^T for the current segment
+  float o[S::kSteps][4];      // O^T fragments: rows = head_dim, columns = heads
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
 #pragma unroll
-  for (int i = 0; i < G; ++i) {
-    m[i] = -INFINITY;
-#pragma unroll
-    for (int e = 0; e < E / 2; ++e) acc[i][e] = make_float2(0.f, 0.f);
+  for (int t = 0; t < S::kSteps; ++t) {
+    o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
+    qb[t][0] = qb[t][1] = 0u;
   }
-  uint32_t sync_phase = 0;
 
   for (int it = 0; it < nchunks; ++it) {
     const int stage = it % S::kStages;
@@ -402,86 +424,85 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
       return;
     }
     const int4 inf = info[stage];
-    if (inf.z & kFirst) {  // query heads of a new segment
-      const uint8_t *qb = qbufs + inf.w * S::kQBytes;
+    if (inf.z & kFirst) {  // Q^T fragments of a new segment (heads >= G are zero)
+      const uint16_t *q = reinterpret_cast<const uint16_t *>(qbufs + inf.w * S::kQBytes);
 #pragma unroll
-      for (int i = 0; i < G; ++i) {
-        const uint8_t *qh = qb + (i ^ hsel) * D * 2;
-#pragma unroll
-        for (int t = 0; t < S::kPieces; ++t) {
-          const uint4 w = *reinterpret_cast<const uint4 *>(qh + (t * LPS + c) * 16);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const float2 f = bf16x2_to_float2(word_of(w, j));
-            q2[i][t * 4 + j] = make_float2(f.x * qscale, f.y * qscale);
-          }
+      for (int t = 0; t < S::kSteps; ++t) {
+        if (r0 < G) {
+          qb[t][0] = *reinterpret_cast<const uint32_t *>(q + r0 * D + 16 * t + 2 * cq);
+          qb[t][1] = *reinterpret_cast<const uint32_t *>(q + r0 * D + 16 * t + 8 + 2 * cq);
+        } else {
+          qb[t][0] = qb[t][1] = 0u;
         }
       }
     }
     if (inf.z & kPageOk) {
-      const uint8_t *kb = stages + stage * S::kStageBytes + slot * (D * 2);
-      const uint8_t *vb = kb + S::kChunkBytes;
-      const bool valid = slot < inf.y;
-      uint4 kr[S::kPieces], vr[S::kPieces];
-#pragma unroll
-      for (int t = 0; t < S::kPieces; ++t)
-        kr[t] = *reinterpret_cast<const uint4 *>(kb + (t * LPS + c) * 16);
-#pragma unroll
-      for (int t = 0; t < S::kPieces; ++t)
-        vr[t] = *reinterpret_cast<const uint4 *>(vb + (t * LPS + c) * 16);
-      // q.k partials, two elements per packed FMA
-      float2 part[G];
-#pragma unroll
-      for (int i = 0; i < G; ++i) part[i] = make_float2(0.f, 0.f);
-#pragma unroll
-      for (int t = 0; t < S::kPieces; ++t) {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const float2 kf = bf16x2_to_float2(word_of(kr[t], j));
-#pragma unroll
-          for (int i = 0; i < G; ++i) part[i] = __ffma2_rn(q2[i][t * 4 + j], kf, part[i]);
+      uint8_t *kt = stages + stage * S::kStageBytes;
+      uint8_t *vt = kt + S::kChunkBytes;
+      const int nvalid = inf.y;
+      if (nvalid < kChunkSlots) {  // rows past the sequence end never reach the MMA
+        for (int i = lane; i < (kChunkSlots - nvalid) * (D / 8); i += 32) {
+          const int slot = nvalid + i / (D / 8), c = i % (D / 8);
+          *reinterpret_cast<uint4 *>(vt + tile_offset<D>(slot, c)) = make_uint4(0, 0, 0, 0);
         }
+        __syncwarp();
       }
-      float sc[G];
+      const uint32_t kbase = smem_u32(kt), vbase = smem_u32(vt);
+      // S^T (16 slots x 8 heads) = K (16 x D) . Q^T (D x 8), two accumulators for ILP
+      float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int i = 0; i < G; ++i) sc[i] = part[i].x + part[i].y;
-      float s = reduce_scores<G, LPS>(sc);
-      s = valid ? s : -INFINITY;
-      float tmax = s;
+      for (int t = 0; t < S::kSteps; ++t) {
+        uint32_t a[4];
+        ldmatrix_x4(a, kbase + tile_offset<D>(a_slot, 2 * t + a_half));
+        if (t & 1) mma_16816(sb, a, qb[t][0], qb[t][1]);
+        else mma_16816(sa, a, qb[t][0], qb[t][1]);
+      }
+      const bool v0 = r0 < nvalid, v1 = r0 + 8 < nvalid;
+      const float x0 = (v0 && hv0) ? (sa[0] + sb[0]) * qscale : -INFINITY;
+      const float x1 = (v0 && hv1) ? (sa[1] + sb[1]) * qscale : -INFINITY;
+      const float x2 = (v1 && hv0) ? (sa[2] + sb[2]) * qscale : -INFINITY;
+      const float x3 = (v1 && hv1) ? (sa[3] + sb[3]) * qscale : -INFINITY;
+      float t0 = fmaxf(x0, x2), t1 = fmaxf(x1, x3);
 #pragma unroll
-      for (int o = LPS; o < 32; o <<= 1) tmax = fmaxf(tmax, __shfl_xor_sync(kFull, tmax, o));
-      if (__any_sync(kFull, tmax > m[0] + kRescaleSlack)) {
+      for (int off = 4; off < 32; off <<= 1) {
+        t0 = fmaxf(t0, __shfl_xor_sync(kFull, t0, off));
+        t1 = fmaxf(t1, __shfl_xor_sync(kFull, t1, off));
+      }
+      if (__any_sync(kFull, t0 > m0 + kRescaleSlack || t1 > m1 + kRescaleSlack)) {
+        const float n0 = fmaxf(m0, t0), n1 = fmaxf(m1, t1);
+        const float a0 = (n0 == -INFINITY) ? 1.f : ex2(m0 - n0);
+        const float a1 = (n1 == -INFINITY) ? 1.f : ex2(m1 - n1);
 #pragma unroll
-        for (int i = 0; i < G; ++i) {
-          const float tm = __shfl_sync(kFull, tmax, (i ^ hsel) * S::kHeadLanes);
-          const float mn = fmaxf(m[i], tm);
-          const float alpha = (mn == -INFINITY) ? 1.f : ex2(m[i] - mn);
-#pragma unroll
-          for (int e = 0; e < E / 2; ++e) acc[i][e] = __fmul2_rn(acc[i][e], make_float2(alpha, alpha));
-          if (i == 0) l_own *= alpha;
-          m[i] = mn;
+        for (int t = 0; t < S::kSteps; ++t) {
+          o[t][0] *= a0;
+          o[t][2] *= a0;
+          o[t][1] *= a1;
+          o[t][3] *= a1;
         }
+        l0 *= a0;
+        l1 *= a1;
+        m0 = n0;
+        m1 = n1;
       }
-      const float p = valid ? ex2(s - m[0]) : 0.f;
-      l_own += p;
-      float ph[G];
+      const float p0 = (x0 == -INFINITY) ? 0.f : ex2(x0 - m0);
+      const float p1 = (x1 == -INFINITY) ? 0.f : ex2(x1 - m1);
+      const float p2 = (x2 == -INFINITY) ? 0.f : ex2(x2 - m0);
+      const float p3 = (x3 == -INFINITY) ? 0.f : ex2(x3 - m1);
+      const uint32_t pk0 = pack_bf16x2(p0, p1);  // slot r0:     heads h0, h1
+      const uint32_t pk1 = pack_bf16x2(p2, p3);  // slot r0 + 8: heads h0, h1
+      // the softmax sum uses the same rounded weights the MMA sees
+      l0 += __uint_as_float(pk0 << 16) + __uint_as_float(pk1 << 16);
+      l1 += __uint_as_float(pk0 & 0xFFFF0000u) + __uint_as_float(pk1 & 0xFFFF0000u);
+      const uint32_t bp0 = movmatrix_trans(pk0);  // P^T B fragment, slots 0-7
+      const uint32_t bp1 = movmatrix_trans(pk1);  // slots 8-15
+      // O^T (D x 8 heads) += V^T (D x 16 slots) . P^T (16 slots x 8 heads)
 #pragma unroll
-      for (int i = 0; i < G; ++i)
-        ph[i] = __shfl_sync(kFull, p, sg * LPS + (i ^ hsel) * S::kHeadLanes);
-      if (!valid) {
-#pragma unroll
-        for (int t = 0; t < S::kPieces; ++t) vr[t] = make_uint4(0u, 0u, 0u, 0u);
+      for (int t = 0; t < S::kSteps; ++t) {
+        uint32_t a[4];
+        ldmatrix_x4_trans(a, vbase + tile_offset<D>(v_slot, 2 * t + v_half));
+        mma_16816(o[t], a, bp0, bp1);
       }
-#pragma unroll
-      for (int t = 0; t < S::kPieces; ++t) {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const float2 vf = bf16x2_to_float2(word_of(vr[t], j));
-#pragma unroll
-          for (int i = 0; i < G; ++i)
-            acc[i][t * 4 + j] = __ffma2_rn(make_float2(ph[i], ph[i]), vf, acc[i][t * 4 + j]);
-        }
-      }
+      if (nvalid < kChunkSlots) fence_proxy_async_smem();  // zeroed rows vs the next TMA
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[stage]);
@@ -491,115 +512,126 @@ __global__ void __launch_bounds__(Shape<D, G, E>::kThreads, Shape<D, G, E>::kMin
     // ------------------------------------------------------------ end of a segment
     const int seg = inf.x;
 #pragma unroll
-    for (int o = LPS; o < 32; o <<= 1) {  // sum the warp's slot groups
-#pragma unroll
-      for (int i = 0; i < G; ++i) {
-#pragma unroll
-        for (int e = 0; e < E / 2; ++e) {
-          acc[i][e].x += __shfl_xor_sync(kFull, acc[i][e].x, o);
-          acc[i][e].y += __shfl_xor_sync(kFull, acc[i][e].y, o);
-        }
-      }
-      l_own += __shfl_xor_sync(kFull, l_own, o);
+    for (int off = 4; off < 32; off <<= 1) {
+      l0 += __shfl_xor_sync(kFull, l0, off);
+      l1 += __shfl_xor_sync(kFull, l1, off);
     }
-    if (sg == 0) {
-#pragma unroll
-      for (int i = 0; i < G; ++i) {
-        float *dst = merge_acc + (warp * G + (i ^ hsel)) * D;
-#pragma unroll
-        for (int t = 0; t < S::kPieces; ++t) {
-          float4 *d4 = reinterpret_cast<float4 *>(dst + (t * LPS + c) * 8);
-          d4[0] = make_float4(acc[i][t * 4 + 0].x, acc[i][t * 4 + 0].y, acc[i][t * 4 + 1].x,
-                              acc[i][t * 4 + 1].y);
-          d4[1] = make_float4(acc[i][t * 4 + 2].x, acc[i][t * 4 + 2].y, acc[i][t * 4 + 3].x,
-                              acc[i][t * 4 + 3].y);
-        }
-      }
-      if (c % S::kHeadLanes == 0) merge_ml[warp * G + hsel] = make_float2(m[0], l_own);
-    }
-    bool ok = consumer_sync(sync_bar, sync_phase, flags);
-
     const int b = seg / Hkv, g = seg - b * Hkv;
     const int nch = cum[b + 1] - cum[b];
     const int64_t X0 = (int64_t)Hkv * cum[b] + (int64_t)g * nch;
     const int first = plan_owner(W, C, X0), last = plan_owner(W, C, X0 + nch - 1);
-    const bool multi = first != last;
-    const int64_t pidx = (int64_t)blockIdx.x + seg;
-    if (ok) {
-      for (int idx = ctid; idx < G * D; idx += S::kConsumerThreads) {
-        const int h = idx / D, d = idx - h * D;
-        float M = -INFINITY;
+    const int64_t obase = (int64_t)seg * G * D;
+    if (first == last) {  // the whole segment is ours: normalise and store
+      const float i0 = 1.f / l0, i1 = 1.f / l1;
 #pragma unroll
-        for (int w = 0; w < S::kConsumerWarps; ++w) M = fmaxf(M, merge_ml[w * G + h].x);
-        float num = 0.f, den = 0.f;
-#pragma unroll
-        for (int w = 0; w < S::kConsumerWarps; ++w) {
-          const float2 ml = merge_ml[w * G + h];
-          const float f = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
-          num += f * merge_acc[(w * G + h) * D + d];
-          den += f * ml.y;
+      for (int t = 0; t < S::kSteps; ++t) {
+        const int d0 = 16 * t + r0;
+        if (hv0) {
+          store_out<OutT>(v.out, obase + (int64_t)h0 * D + d0, o[t][0] * i0);
+          store_out<OutT>(v.out, obase + (int64_t)h0 * D + d0 + 8, o[t][2] * i0);
         }
-        if (!multi) {
-          store_out<OutT>(v.out, ((int64_t)seg * G + h) * D + d, num / den);
-        } else {
-          v.part_acc[(pidx * G + h) * D + d] = num;
-          if (d == 0) v.part_ml[pidx * G + h] = make_float2(M, den);
+        if (hv1) {
+          store_out<OutT>(v.out, obase + (int64_t)h1 * D + d0, o[t][1] * i1);
+          store_out<OutT>(v.out, obase + (int64_t)h1 * D + d0 + 8, o[t][3] * i1);
         }
       }
-    }
-    if (ok && multi) {
-      __threadfence();
-      ok = consumer_sync(sync_bar, sync_phase, flags);
-      if (ok && ctid == 0) {
-        const uint32_t ticket = atomicAdd(&v.tickets[seg], 1u);
-        flags[1] = (ticket == (uint32_t)(last - first)) ? 1 : 0;
-      }
-      if (ok) ok = consumer_sync(sync_bar, sync_phase, flags);
-      if (ok && flags[1]) {  // last CTA of the segment: merge the partials in CTA order
-        __threadfence();
-        for (int idx = ctid; idx < G * D; idx += S::kConsumerThreads) {
-          const int h = idx / D, d = idx - h * D;
-          float M = -INFINITY;
-          for (int k = first; k <= last; ++k)
-            M = fmaxf(M, __ldcg(&v.part_ml[((int64_t)k + seg) * G + h]).x);
-          float num = 0.f, den = 0.f;
-          for (int k = first; k <= last; ++k) {
-            const int64_t pk = (int64_t)k + seg;
-            const float2 ml = __ldcg(&v.part_ml[pk * G + h]);
-            const float f = ex2(ml.x - M);
-            num += f * __ldcg(&v.part_acc[(pk * G + h) * D + d]);
-            den += f * ml.y;
-          }
-          store_out<OutT>(v.out, ((int64_t)seg * G + h) * D + d, num / den);
+    } else {  // partial state of this CTA; the combine kernel merges first..last
+      const int64_t pidx = (int64_t)blockIdx.x + seg;
+      float *pacc = v.part_acc + pidx * G * D;
+#pragma unroll
+      for (int t = 0; t < S::kSteps; ++t) {
+        const int d0 = 16 * t + r0;
+        if (hv0) {
+          pacc[h0 * D + d0] = o[t][0];
+          pacc[h0 * D + d0 + 8] = o[t][2];
         }
-        if (ctid == 0) v.tickets[seg] = 0u;
+        if (hv1) {
+          pacc[h1 * D + d0] = o[t][1];
+          pacc[h1 * D + d0 + 8] = o[t][3];
+        }
+      }
+      if (r0 == 0) {
+        if (hv0) v.part_ml[pidx * G + h0] = make_float2(m0, l0);
+        if (hv1) v.part_ml[pidx * G + h1] = make_float2(m1, l1);
       }
     }
-    if (ok) ok = consumer_sync(sync_bar, sync_phase, flags);  // merge buffers free again
-    if (!ok) {
-      if (lane == 0) {
-        record_error(v.err, HAM_DEVERR_TIMEOUT);
-        flags[0] = 1;
-      }
-      return;
-    }
+    if (lane == 0 && (int)blockIdx.x == first) v.seg_range[seg] = make_int2(first, last);
 #pragma unroll
-    for (int i = 0; i < G; ++i) {
-      m[i] = -INFINITY;
-#pragma unroll
-      for (int e = 0; e < E / 2; ++e) acc[i][e] = make_float2(0.f, 0.f);
-    }
-    l_own = 0.f;
+    for (int t = 0; t < S::kSteps; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
+    m0 = m1 = -INFINITY;
+    l0 = l1 = 0.f;
   }
+}
+
+// ------------------------------------------------------------------------------------
+// Combine: out[seg][h][d] = sum_k 2^(m_k - M) acc_k[h][d] / sum_k 2^(m_k - M) l_k over the
+// CTAs k = first..last of the segment, M = max_k m_k (split-softmax merge, in CTA order).
+// One thread per output element; blocks of kCombineThreads cover one segment's G*D values.
+// ------------------------------------------------------------------------------------
+constexpr int kCombineThreads = 128;
+
+template <typename OutT>
+__global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView v, int D,
+                                                                  int blocks_per_seg) {
+  grid_dependency_wait();  // the attention grid's partials and ranges are visible
+  const int G = v.group;
+  const int seg = blockIdx.x / blocks_per_seg;
+  const int idx = (blockIdx.x % blocks_per_seg) * kCombineThreads + threadIdx.x;
+  const int2 r = v.seg_range[seg];
+  if (r.x < 0 || r.x == r.y || idx >= G * D) return;
+  const int h = idx / D;
+  // Online merge in batches of 8 partials: the 8 loads of a batch are in flight together.
+  constexpr int kBatch = 8;
+  float M = -INFINITY, num = 0.f, den = 0.f;
+  for (int k0 = r.x; k0 <= r.y; k0 += kBatch) {
+    float2 ml[kBatch];
+    float acc[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int64_t p = (int64_t)k0 + j + seg;
+      const bool in = k0 + j <= r.y;
+      ml[j] = in ? __ldcg(&v.part_ml[p * G + h]) : make_float2(-INFINITY, 0.f);
+      acc[j] = in ? __ldcg(&v.part_acc[p * G * D + idx]) : 0.f;
+    }
+    float bm = M;
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) bm = fmaxf(bm, ml[j].x);
+    const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
+    num *= scale;
+    den *= scale;
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const float w = (ml[j].x == -INFINITY) ? 0.f : ex2(ml[j].x - bm);
+      num += w * acc[j];
+      den += w * ml[j].y;
+    }
+    M = bm;
+  }
+  store_out<OutT>(v.out, (int64_t)seg * G * D + idx, num / den);
+}
+
+template <typename OutT>
+cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream) {
+  const int per_seg = (v.group * head_dim + kCombineThreads - 1) / kCombineThreads;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(v.batch * v.n_kv_heads * per_seg));
+  cfg.blockDim = dim3(kCombineThreads);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, combine_kernel<OutT>, v, head_dim, per_seg);
 }
 
 // ------------------------------------------------------------------------------------
 // Dispatch
 // ------------------------------------------------------------------------------------
-template <int D, int G, int E, typename OutT>
+template <int D, typename OutT>
 struct Instance {
-  using S = Shape<D, G, E>;
-  static const void *fn() { return reinterpret_cast<const void *>(&decode_attn_kernel<D, G, E, OutT>); }
+  using S = Shape<D>;
+  static auto fn() { return &decode_attn_kernel<D, OutT>; }
   // Allow the largest dynamic shared memory any batch needs, once per device.
   static cudaError_t configure() {
     static std::mutex mu;
@@ -609,65 +641,63 @@ struct Instance {
     if (e != cudaSuccess) return e;
     std::lock_guard<std::mutex> lock(mu);
     if (dev >= 0 && dev < 64 && done[dev]) return cudaSuccess;
-    e = cudaFuncSetAttribute(&decode_attn_kernel<D, G, E, OutT>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(fn(), cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)S::smem_bytes(kMaxBatch));
     if (e == cudaSuccess && dev >= 0 && dev < 64) done[dev] = true;
     return e;
   }
-  static cudaError_t launch(const AttnView &v, cudaStream_t stream) {
+  static cudaError_t launch(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
+                            cudaStream_t stream) {
     cudaError_t e = configure();
     if (e != cudaSuccess) return e;
-    decode_attn_kernel<D, G, E, OutT>
-        <<<v.ctas, S::kThreads, S::smem_bytes(v.batch), stream>>>(v);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)v.ctas);
+    cfg.blockDim = dim3(S::kThreads);
+    cfg.dynamicSmemBytes = S::smem_bytes(v.batch);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<D, OutT>, tk, tv, v);
+    if (e != cudaSuccess) return e;
+    return launch_combine<OutT>(v, D, stream);
   }
   static int ctas_per_sm(int batch) {
     if (configure() != cudaSuccess) return 0;
     int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, &decode_attn_kernel<D, G, E, OutT>,
-                                                      S::kThreads, S::smem_bytes(batch)) !=
-        cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn(), S::kThreads,
+                                                      S::smem_bytes(batch)) != cudaSuccess)
       return 0;
     return n;
   }
 };
 
-// head_dim 128 keeps 16 elements per lane (8 lanes per slot) unless the group is 8, where
-// 8 elements per lane keep the register budget; head_dim 64 uses 8 elements per lane.
 template <typename OutT, typename F>
-cudaError_t dispatch(int head_dim, int group, F &&f) {
-  switch (head_dim * 16 + group) {
-    case 128 * 16 + 1: return f(Instance<128, 1, 16, OutT>());
-    case 128 * 16 + 2: return f(Instance<128, 2, 16, OutT>());
-    case 128 * 16 + 4: return f(Instance<128, 4, 16, OutT>());
-    case 128 * 16 + 8: return f(Instance<128, 8, 8, OutT>());
-    case 64 * 16 + 1: return f(Instance<64, 1, 8, OutT>());
-    case 64 * 16 + 2: return f(Instance<64, 2, 8, OutT>());
-    case 64 * 16 + 4: return f(Instance<64, 4, 8, OutT>());
-    case 64 * 16 + 8: return f(Instance<64, 8, 8, OutT>());
-    default: return cudaErrorInvalidValue;
-  }
+cudaError_t dispatch(int head_dim, F &&f) {
+  if (head_dim == 128) return f(Instance<128, OutT>());
+  if (head_dim == 64) return f(Instance<64, OutT>());
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
 
 bool attention_supported(int head_dim, int group) {
-  return (head_dim == 64 || head_dim == 128) &&
-         (group == 1 || group == 2 || group == 4 || group == 8);
+  return (head_dim == 64 || head_dim == 128) && group >= 1 && group <= kMaxGroup;
 }
 
-cudaError_t launch_attention(const AttnView &v, int head_dim, int group, int out_dtype,
-                             cudaStream_t stream) {
-  if (v.ctas < 1) return cudaErrorInvalidConfiguration;
-  auto go = [&](auto inst) { return decltype(inst)::launch(v, stream); };
-  return out_dtype == HAM_DTYPE_F32 ? dispatch<float>(head_dim, group, go)
-                                    : dispatch<__nv_bfloat16>(head_dim, group, go);
+cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
+                             int head_dim, int out_dtype, cudaStream_t stream) {
+  if (v.ctas < 1 || v.group < 1 || v.group > kMaxGroup) return cudaErrorInvalidConfiguration;
+  auto go = [&](auto inst) { return decltype(inst)::launch(tk, tv, v, stream); };
+  return out_dtype == HAM_DTYPE_F32 ? dispatch<float>(head_dim, go)
+                                    : dispatch<__nv_bfloat16>(head_dim, go);
 }
 
-int attention_ctas_per_sm(int head_dim, int group, int batch) {
+int attention_ctas_per_sm(int head_dim, int batch) {
   int n = 0;
-  dispatch<__nv_bfloat16>(head_dim, group, [&](auto inst) {
+  dispatch<__nv_bfloat16>(head_dim, [&](auto inst) {
     n = decltype(inst)::ctas_per_sm(batch);
     return cudaSuccess;
   });

@@ -1,8 +1,11 @@
 // Internal declarations of libham.so (not installed; the public ABI is include/ham.h).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <vector>
 
 #include "ham.h"
 
@@ -46,10 +49,11 @@ struct AttnView {
   void *out;                   // [batch][n_q_heads][head_dim], bf16 or f32
   float *part_acc;             // scratch [(ctas + batch*n_kv_heads)][group][head_dim]
   float2 *part_ml;             // scratch [(ctas + batch*n_kv_heads)][group]: (max, sum)
-  uint32_t *tickets;           // scratch [batch*n_kv_heads], zero between launches
+  int2 *seg_range;             // scratch [batch*n_kv_heads]: CTAs first..last of a segment
+                               // whose partials the combine kernel merges (-1: nothing)
   int32_t *err;                // device error word
   int64_t pool_pages;
-  int32_t batch, n_kv_heads, page_slots, max_pages, max_slots;
+  int32_t batch, n_kv_heads, group, page_slots, max_pages, max_slots;
   int32_t ctas;
 };
 
@@ -67,6 +71,7 @@ struct AppendView {
   int32_t *err;
   int64_t pool_pages;
   int32_t batch, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots, pos_mode;
+  int32_t kv_per_block;        // KV heads per append block (append_kv_per_block)
 };
 
 struct FillView {
@@ -83,12 +88,19 @@ struct FillView {
 };
 
 // Launchers (return cudaError_t of the launch; argument checks are done by the callers).
-cudaError_t launch_attention(const AttnView &v, int head_dim, int group, int out_dtype,
-                             cudaStream_t stream);
+// tk / tv: TMA maps of the layer's K and V pools (make_pool_tensor_map).
+cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
+                             int head_dim, int out_dtype, cudaStream_t stream);
 // CTAs of one SM for the attention kernel of this shape (0 if the shape is not compiled).
-int attention_ctas_per_sm(int head_dim, int group, int batch);
+int attention_ctas_per_sm(int head_dim, int batch);
 bool attention_supported(int head_dim, int group);
+// TMA map of one pool [pool_pages][n_kv_heads][page_slots][head_dim] bf16 viewed as
+// {64 elements, head_dim / 64, rows} with a box of {64, head_dim / 64, 16 rows} and the
+// 128-byte swizzle.  Returns a CUresult (0 on success).
+int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim);
 cudaError_t launch_append(const AppendView &v, cudaStream_t stream);
+// KV heads per append block (0 if the shape does not fit the append kernel).
+int append_kv_per_block(int n_q_heads, int n_kv_heads, int head_dim);
 cudaError_t launch_fill(const FillView &v, cudaStream_t stream);
 
 // Device error word: keep the first error.
@@ -105,6 +117,7 @@ struct ham_kv {
   int num_sms = 0;
   int32_t max_pages = 0;
   int32_t attn_ctas = 0;        // 0: default
+  int32_t default_ctas = 0;     // SMs x resident attention CTAs per SM (set at allocation)
   int32_t max_ctas = 0;         // scratch is sized for this many CTAs
   int64_t pool_elems = 0;       // bf16 elements of ONE pool (K or V) of one layer
   uint16_t *pool = nullptr;     // [layers][2][pool_elems]
@@ -116,7 +129,8 @@ struct ham_kv {
   int32_t *err = nullptr;
   float *part_acc = nullptr;
   float2 *part_ml = nullptr;
-  uint32_t *tickets = nullptr;
+  int2 *seg_range = nullptr;
   int64_t scratch_bytes = 0;
+  std::vector<CUtensorMap> tmaps;  // [layers][2]: TMA maps of the K and V pools
   void *host_stage = nullptr;   // pinned: counters and error word read-back
 };

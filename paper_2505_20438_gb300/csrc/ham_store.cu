@@ -4,6 +4,7 @@
 // A macro-step of HAMburger stores one KV set for all tokens it fused (Sec. 3.1, Sec. 3.6
 // "Token Fusion"), so the store is a per-sequence list of slots, each with the position it
 // was rotated at (Sec. 3.2) and its token count.
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -146,6 +147,45 @@ __global__ void fill_meta_kernel(FillView v) {
   }
 }
 
+__global__ void set_lengths_kernel(int32_t *num_slots, int64_t *num_tokens,
+                                   const int32_t *new_slots, const int64_t *new_tokens,
+                                   int32_t batch, int32_t max_slots, int32_t *err) {
+  const int32_t b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch) return;
+  const int32_t n = new_slots[b];
+  if (n < 0 || n > max_slots) {
+    record_error(err, HAM_DEVERR_SLOTS);
+    return;
+  }
+  num_slots[b] = n;
+  if (new_tokens) num_tokens[b] = new_tokens[b];
+}
+
+int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim) {
+  using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                              const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                              const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                              CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+  static Encode encode = nullptr;
+  if (!encode) {
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return -1;
+    encode = reinterpret_cast<Encode>(fn);
+  }
+  const cuuint64_t dims[3] = {64, (cuuint64_t)(head_dim / 64), (cuuint64_t)rows};
+  const cuuint64_t strides[2] = {128, (cuuint64_t)head_dim * 2};  // bytes, dims 1 and 2
+  const cuuint32_t box[3] = {64, (cuuint32_t)(head_dim / 64), (cuuint32_t)kChunkSlots};
+  const cuuint32_t estride[3] = {1, 1, 1};
+  return (int)encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(pool), dims,
+                     strides, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 cudaError_t launch_fill(const FillView &v, cudaStream_t stream) {
   if (v.lmax > 0) {
     dim3 grid((unsigned)((v.lmax + 15) / 16), (unsigned)v.batch);
@@ -185,7 +225,8 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   if (!(cfg.rope_base > 1.0) || !std::isfinite(cfg.rope_base))
     return fail(HAM_EINVAL, "rope_base must be finite and > 1");
   const int group = cfg.n_q_heads / cfg.n_kv_heads;
-  if (!ham::attention_supported(cfg.head_dim, group))
+  if (!ham::attention_supported(cfg.head_dim, group) ||
+      ham::append_kv_per_block(cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim) == 0)
     return fail(HAM_EUNSUPPORTED, "head_dim %d / group %d not compiled (head_dim 64 or 128, "
                 "group 1, 2, 4 or 8)", cfg.head_dim, group);
   const int64_t max_pages =
@@ -200,6 +241,9 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     return fail(HAM_ECAPACITY, "pool of %lld pages < %lld pages reserved by the page tables",
                 (long long)cfg.pool_pages, (long long)need_pages);
   if (cfg.pool_pages > INT32_MAX) return fail(HAM_EINVAL, "pool_pages above int32 range");
+  // TMA row coordinates of the pools are int32
+  if (cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots > INT32_MAX)
+    return fail(HAM_EINVAL, "pool_pages * n_kv_heads * page_slots above int32 range");
 
   int dev = 0;
   HAM_CUDA(cudaGetDevice(&dev));
@@ -232,9 +276,17 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   const size_t o_err = carve(sizeof(int32_t));
   const size_t o_acc = carve(n_part * group * cfg.head_dim * sizeof(float));
   const size_t o_ml = carve(n_part * group * sizeof(float2));
-  const size_t o_tk = carve(n_seg * sizeof(uint32_t));
+  const size_t o_sr = carve(n_seg * sizeof(int2));
   kv->scratch_bytes = (int64_t)(off - o_acc);
 
+  {
+    const int per_sm = ham::attention_ctas_per_sm(cfg.head_dim, cfg.batch);
+    if (per_sm <= 0) {
+      delete kv;
+      return fail(HAM_ECUDA, "attention kernel cannot be resident on an SM");
+    }
+    kv->default_ctas = std::min(sms * per_sm, kv->max_ctas);
+  }
   cudaError_t e = cudaMalloc(&kv->pool, pool_bytes);
   if (e != cudaSuccess) {
     delete kv;
@@ -257,7 +309,7 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->err = reinterpret_cast<int32_t *>(kv->meta + o_err);
   kv->part_acc = reinterpret_cast<float *>(kv->meta + o_acc);
   kv->part_ml = reinterpret_cast<float2 *>(kv->meta + o_ml);
-  kv->tickets = reinterpret_cast<uint32_t *>(kv->meta + o_tk);
+  kv->seg_range = reinterpret_cast<int2 *>(kv->meta + o_sr);
 
   // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits.
   e = cudaMemset(kv->pool, 0, pool_bytes);
@@ -276,6 +328,18 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     int rc = cuda_fail(e, "initialising the cache");
     ham_kv_free(kv);
     return rc;
+  }
+  kv->tmaps.resize((size_t)cfg.layers * 2);
+  const int64_t rows = cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots;
+  for (int layer = 0; layer < cfg.layers; ++layer) {
+    for (int which = 0; which < 2; ++which) {
+      int r = ham::make_pool_tensor_map(&kv->tmaps[(size_t)layer * 2 + which],
+                                        layer_pool(kv, layer, which), rows, cfg.head_dim);
+      if (r != 0) {
+        ham_kv_free(kv);
+        return fail(HAM_ECUDA, "cuTensorMapEncodeTiled failed (CUresult %d)", r);
+      }
+    }
   }
   *out = kv;
   return HAM_OK;
@@ -297,9 +361,7 @@ int ham_kv_get_info(const ham_kv *kv, ham_kv_info *info) {
   memset(info, 0, sizeof *info);
   info->cfg = kv->cfg;
   info->max_pages_per_seq = kv->max_pages;
-  const int group = kv->cfg.n_q_heads / kv->cfg.n_kv_heads;
-  int per_sm = ham::attention_ctas_per_sm(kv->cfg.head_dim, group, kv->cfg.batch);
-  info->attn_ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->num_sms * (per_sm > 0 ? per_sm : 1);
+  info->attn_ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->default_ctas;
   info->num_sms = kv->num_sms;
   info->device = kv->device;
   info->pool_bytes = 2 * kv->pool_elems * (int64_t)sizeof(uint16_t);
@@ -349,6 +411,7 @@ int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
   v.max_pages = kv->max_pages;
   v.max_slots = kv->cfg.max_slots_per_seq;
   v.pos_mode = kv->cfg.pos_mode;
+  v.kv_per_block = ham::append_kv_per_block(v.n_q_heads, v.n_kv_heads, v.head_dim);
   cudaError_t e = ham::launch_append(v, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "append launch");
   return HAM_OK;
@@ -364,13 +427,7 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
     return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
   DeviceGuard guard(kv->device);
   const int group = kv->cfg.n_q_heads / kv->cfg.n_kv_heads;
-  int ctas = kv->attn_ctas;
-  if (ctas <= 0) {
-    int per_sm = ham::attention_ctas_per_sm(kv->cfg.head_dim, group, kv->cfg.batch);
-    if (per_sm <= 0) return fail(HAM_ECUDA, "attention kernel cannot be resident on an SM");
-    ctas = kv->num_sms * per_sm;
-    if (ctas > kv->max_ctas) ctas = kv->max_ctas;
-  }
+  const int ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->default_ctas;
   ham::AttnView v{};
   v.k_pool = layer_pool(kv, layer, 0);
   v.v_pool = layer_pool(kv, layer, 1);
@@ -380,16 +437,18 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
   v.out = out;
   v.part_acc = kv->part_acc;
   v.part_ml = kv->part_ml;
-  v.tickets = kv->tickets;
+  v.seg_range = kv->seg_range;
   v.err = kv->err;
   v.pool_pages = kv->cfg.pool_pages;
   v.batch = kv->cfg.batch;
   v.n_kv_heads = kv->cfg.n_kv_heads;
+  v.group = group;
   v.page_slots = kv->cfg.page_slots;
   v.max_pages = kv->max_pages;
   v.max_slots = kv->cfg.max_slots_per_seq;
   v.ctas = ctas;
-  cudaError_t e = ham::launch_attention(v, kv->cfg.head_dim, group, out_dtype,
+  cudaError_t e = ham::launch_attention(kv->tmaps[(size_t)layer * 2], kv->tmaps[(size_t)layer * 2 + 1],
+                                        v, kv->cfg.head_dim, out_dtype,
                                         static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "attention launch");
   return HAM_OK;
@@ -437,13 +496,7 @@ int ham_kv_status(ham_kv *kv, void *stream, int32_t *device_code) {
   HAM_CUDA(cudaMemsetAsync(kv->err, 0, sizeof(int32_t), s));
   HAM_CUDA(cudaStreamSynchronize(s));
   if (device_code) *device_code = *h_err;
-  if (*h_err != 0) {
-    // A kernel that gave up mid-way may have left split tickets behind: clear them.
-    const size_t n_seg = (size_t)kv->cfg.batch * kv->cfg.n_kv_heads;
-    HAM_CUDA(cudaMemsetAsync(kv->tickets, 0, n_seg * sizeof(uint32_t), s));
-    HAM_CUDA(cudaStreamSynchronize(s));
-    return fail(HAM_EDEVICE, "device error word = %d", *h_err);
-  }
+  if (*h_err != 0) return fail(HAM_EDEVICE, "device error word = %d", *h_err);
   return HAM_OK;
 }
 
@@ -522,6 +575,20 @@ int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *
   if (v_dst) HAM_CUDA(cudaMemcpyAsync(v_dst, layer_pool(kv, layer, 1), pool_bytes, cudaMemcpyDefault, s));
   if (pos_dst) HAM_CUDA(cudaMemcpyAsync(pos_dst, kv->slot_pos, meta_bytes, cudaMemcpyDefault, s));
   if (ntok_dst) HAM_CUDA(cudaMemcpyAsync(ntok_dst, kv->slot_ntok, meta_bytes, cudaMemcpyDefault, s));
+  return HAM_OK;
+}
+
+int ham_kv_set_lengths(ham_kv *kv, int32_t layer, const int32_t *num_slots,
+                       const int64_t *num_tokens, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!num_slots) return fail(HAM_EINVAL, "num_slots is required");
+  DeviceGuard guard(kv->device);
+  const int B = kv->cfg.batch;
+  ham::set_lengths_kernel<<<(B + 127) / 128, 128, 0, static_cast<cudaStream_t>(stream)>>>(
+      kv->num_slots + (size_t)layer * B, kv->num_tokens + (size_t)layer * B, num_slots,
+      num_tokens, B, kv->cfg.max_slots_per_seq, kv->err);
+  HAM_CUDA(cudaGetLastError());
   return HAM_OK;
 }
 

@@ -67,6 +67,7 @@ _SIGNATURES = {
     "ham_kv_fill": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
     "ham_kv_export": [_vp, _i32, _vp, _vp, _vp, _vp, _vp],
     "ham_kv_reset": [_vp, _vp],
+    "ham_kv_set_lengths": [_vp, _i32, _vp, _vp, _vp],
     "ham_kv_set_attn_ctas": [_vp, _i32],
     "ham_split_plan": [_i32, _i32, _vp, _i32, _vp, _vp, _vp],
 }
@@ -125,7 +126,8 @@ def _dev(t, shape, dtype_name, what, nullable=False):
             return None
         raise ValueError(f"{what} is required")
     import torch
-    dtype = {"bf16": torch.bfloat16, "f32": torch.float32, "i32": torch.int32}[dtype_name]
+    dtype = {"bf16": torch.bfloat16, "f32": torch.float32, "i32": torch.int32,
+             "i64": torch.int64}[dtype_name]
     if not t.is_cuda:
         raise ValueError(f"{what} must be a CUDA tensor")
     if t.dtype != dtype:
@@ -275,6 +277,13 @@ def ham_kv_export(kv: KV, layer, stream=None):
     _check(lib().ham_kv_export(kv, layer, k.data_ptr(), v.data_ptr(), pos.data_ptr(),
                                ntok.data_ptr(), _stream_ptr(stream)))
     return k, v, pos, ntok
+
+
+def ham_kv_set_lengths(kv: KV, layer, num_slots, num_tokens=None, stream=None):
+    B = kv.batch
+    _check(lib().ham_kv_set_lengths(
+        kv, layer, _dev(num_slots, (B,), "i32", "num_slots"),
+        _dev(num_tokens, (B,), "i64", "num_tokens", nullable=True), _stream_ptr(stream)))
 
 
 def ham_kv_reset(kv: KV, stream=None):
