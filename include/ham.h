@@ -221,6 +221,40 @@ int ham_split_plan(int32_t batch, int32_t n_kv_heads, const int32_t *num_slots_h
                    int32_t ctas, int64_t *cta_begin, int32_t *seg_first_cta,
                    int32_t *seg_last_cta);
 
+/* ------------------------------------------------------------------------------------
+ * Decode attention without any allocation
+ * ------------------------------------------------------------------------------------
+ * No counterpart in the paper: this entry point exists for callers that cannot allocate
+ * device memory themselves -- code whose device memory is owned by a host framework or a
+ * fixed-size arena (an inference-server plugin, for instance), or code that must not call
+ * cudaMalloc at the point where attention runs.  They own the cache in their own layout-
+ * compatible buffers and pass every input and output; the split-attention scratch comes
+ * from an 8 MiB array compiled into libham.so, which every GPU that loads the library keeps
+ * until the process exits.  The call itself allocates nothing (no cudaMalloc, cudaFree or
+ * allocating library routine).
+ *  - The first call on each device looks up that array's device address and sets kernel
+ *    attributes; make that first call before any stream capture on the device.
+ *  - All calls share the one array: calls that overlap on the GPU (other streams, other
+ *    threads) race on it and give wrong results.  Serialize them.
+ *  - A configuration whose scratch would exceed the array ((ctas + batch*n_kv_heads) *
+ *    group * (head_dim + 2) * 4 bytes, about) is rejected with HAM_EINVAL; nothing runs.
+ * The computation is that of ham_decode_attn_ex over the given pool and page table.        */
+typedef struct ham_attn_args {
+  const void *k_pool, *v_pool;  /* device bf16 [pool_pages][n_kv_heads][page_slots][head_dim] */
+  const int32_t *page_table;    /* device [batch][max_pages]: slot n of sequence b is row
+                                   n % page_slots of page page_table[b][n / page_slots] */
+  const int32_t *num_slots;     /* device [batch]: slots to attend over, each <= max_slots */
+  const void *q;                /* device bf16 [batch][n_q_heads][head_dim], already rotated */
+  void *out;                    /* device [batch][n_q_heads][head_dim], bf16 or f32 */
+  int32_t *err;                 /* nullable device int32: first HAM_DEVERR_* seen, else kept */
+  int64_t pool_pages;
+  int32_t batch, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots;
+  int32_t ctas;                 /* 0: SMs x resident CTAs per SM */
+  int32_t out_dtype;            /* HAM_DTYPE_BF16 or HAM_DTYPE_F32 */
+} ham_attn_args;
+
+int ham_decode_attn_noalloc(const ham_attn_args *args, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

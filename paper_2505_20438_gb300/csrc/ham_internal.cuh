@@ -103,6 +103,9 @@ cudaError_t launch_append(const AppendView &v, cudaStream_t stream);
 int append_kv_per_block(int n_q_heads, int n_kv_heads, int head_dim);
 cudaError_t launch_fill(const FillView &v, cudaStream_t stream);
 
+// Record `msg` as this thread's ham_last_error() and return `status`.
+int set_last_error(int status, const char *msg);
+
 // Device error word: keep the first error.
 __device__ inline void record_error(int32_t *err, int32_t code) {
   if (err) atomicCAS(err, 0, code);

@@ -93,6 +93,8 @@ uint16_t *layer_pool(const ham_kv *kv, int32_t layer, int which) {
 // ------------------------------------------------------------------------------------
 namespace ham {
 
+int set_last_error(int status, const char *msg) { return fail(status, "%s", msg); }
+
 __global__ void fill_rows_kernel(FillView v) {
   const int32_t b = blockIdx.y;
   const int32_t count = v.counts[b];

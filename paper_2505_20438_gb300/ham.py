@@ -44,6 +44,17 @@ class ham_config(ctypes.Structure):
                 ("page_seed", ctypes.c_uint64)]
 
 
+class ham_attn_args(ctypes.Structure):
+    _fields_ = [("k_pool", ctypes.c_void_p), ("v_pool", ctypes.c_void_p),
+                ("page_table", ctypes.c_void_p), ("num_slots", ctypes.c_void_p),
+                ("q", ctypes.c_void_p), ("out", ctypes.c_void_p), ("err", ctypes.c_void_p),
+                ("pool_pages", ctypes.c_int64), ("batch", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("page_slots", ctypes.c_int32),
+                ("max_pages", ctypes.c_int32), ("max_slots", ctypes.c_int32),
+                ("ctas", ctypes.c_int32), ("out_dtype", ctypes.c_int32)]
+
+
 class ham_kv_info(ctypes.Structure):
     _fields_ = [("cfg", ham_config), ("max_pages_per_seq", ctypes.c_int32),
                 ("attn_ctas", ctypes.c_int32), ("num_sms", ctypes.c_int32),
@@ -70,6 +81,7 @@ _SIGNATURES = {
     "ham_kv_set_lengths": [_vp, _i32, _vp, _vp, _vp],
     "ham_kv_set_attn_ctas": [_vp, _i32],
     "ham_split_plan": [_i32, _i32, _vp, _i32, _vp, _vp, _vp],
+    "ham_decode_attn_noalloc": [ctypes.c_void_p, _vp],
 }
 _lib = None
 
@@ -305,3 +317,21 @@ def ham_split_plan(num_slots, n_kv_heads: int, ctas: int):
     _check(lib().ham_split_plan(B, n_kv_heads, ns.ctypes.data, ctas, begin.ctypes.data,
                                 first.ctypes.data, last.ctypes.data))
     return begin, first, last
+
+
+def ham_decode_attn_noalloc(k_pool, v_pool, page_table, num_slots, q, out, max_slots,
+                            ctas=0, err=None, stream=None):
+    """Decode attention over caller-owned buffers; the library allocates nothing (its
+    scratch is a static device array shared by all calls)."""
+    import torch
+    P, Hkv, S, d = (int(x) for x in k_pool.shape)
+    B, Hq = int(q.shape[0]), int(q.shape[1])
+    max_pages = int(page_table.shape[1])
+    f32 = out.dtype == torch.float32
+    args = ham_attn_args(
+        _dev(k_pool, (P, Hkv, S, d), "bf16", "k_pool"), _dev(v_pool, (P, Hkv, S, d), "bf16", "v_pool"),
+        _dev(page_table, (B, max_pages), "i32", "page_table"), _dev(num_slots, (B,), "i32", "num_slots"),
+        _dev(q, (B, Hq, d), "bf16", "q"), _dev(out, (B, Hq, d), "f32" if f32 else "bf16", "out"),
+        _dev(err, (1,), "i32", "err", nullable=True), P, B, Hq, Hkv, d, S, max_pages,
+        int(max_slots), int(ctas), HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16)
+    _check(lib().ham_decode_attn_noalloc(ctypes.byref(args), _stream_ptr(stream)))
