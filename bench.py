@@ -64,6 +64,27 @@ def dist_env():
             int(os.environ.get("WORLD_SIZE", "1")))
 
 
+def max_over_ranks(value, world, device):
+    """The largest of every rank's `value` (the job is as slow as its slowest rank)."""
+    if world == 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(steps_per_rank, world, elapsed_s):
+    """Whole-job macro-steps/s: every rank runs its own batch (weak scaling)."""
+    return world * steps_per_rank / elapsed_s
+
+
+def rank_cache_seed(workload_seed, rank, cache):
+    """Seed of one rank's cache: ranks own different sequences."""
+    return 1000 * workload_seed + 10 * rank + cache
+
+
 def measured_peak_hbm():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -215,7 +236,7 @@ def build_caches(w, device_index, rank):
     caches = []
     max_slots = w.slots + GRAPH_STEPS // CACHES + 16
     for r in range(CACHES):
-        seed = 1000 * w.seed + 10 * rank + r
+        seed = rank_cache_seed(w.seed, rank, r)
         kv = ham.ham_kv_alloc(1, w.batch, w.n_q_heads, w.n_kv_heads, w.head_dim, w.page_slots,
                               max_slots, pool_pages=int(math.ceil(
                                   w.batch * math.ceil(max_slots / w.page_slots) * w.pool_factor)),
@@ -331,11 +352,8 @@ def run_ours(args, w):
         probe.replay()
         t1.record(stream)
         torch.cuda.synchronize()
-    elapsed_ms = t0.elapsed_time(t1)
+    elapsed_ms = max_over_ranks(t0.elapsed_time(t1), world, "cuda")
     if world > 1:
-        tt = torch.tensor([elapsed_ms], device="cuda", dtype=torch.float64)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        elapsed_ms = float(tt.item())
         torch.distributed.barrier()
 
     # attention kernel duration (last replay of the timed region)
@@ -361,7 +379,7 @@ def run_ours(args, w):
     peak, peak_src = measured_peak_hbm()
     attn_gbs = attn_bytes_graph / (sum(attn_ms) * 1e-3) / 1e9
     ms_per_step = elapsed_ms / steps
-    value = world * steps / (elapsed_ms * 1e-3)
+    value = job_throughput(steps, world, elapsed_ms * 1e-3)
     step_gbs = world * n_graph * step_bytes_graph / (elapsed_ms * 1e-3) / 1e9
     mean_ntok = statistics.mean(c["mean_ntok"] for c in caches)
 
@@ -434,11 +452,8 @@ def run_e2e(args, w, caches, stream, rollback, world):
                 rollback()
         stream.synchronize()
         dt = time.perf_counter() - t
-    if world > 1:
-        tt = torch.tensor([dt], device="cuda", dtype=torch.float64)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        dt = float(tt.item())
-    return {"value": round(world * n / dt, 2), "unit": UNIT, "h2d_bytes_per_step": h2d,
+    dt = max_over_ranks(dt, world, "cuda")
+    return {"value": round(job_throughput(n, world, dt), 2), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": n,
             "path": "pinned host -> device copies, ham_kv_append, ham_decode_attn, "
                     "device -> pinned host copy, host sync, every step (eager)",
