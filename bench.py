@@ -1,9 +1,10 @@
 #!/usr/bin/env python3
 """Benchmark of smashed-KV decode attention (HAMburger macro-step hot path) on GB300.
 
-One step = one macro-step of one layer for the whole batch, through the C ABI:
-    ham_kv_append   (RoPE of q and k at the new slot's position, append of the slot)
-    ham_decode_attn (split-KV attention over all slots, combine)
+One step = one macro-step of one layer for the whole batch, through the C ABI.  Default
+(--path fused): ham_decode_step, which appends the macro-step's slot (RoPE of q and k at
+its position) and runs split-KV attention over all slots in one pass over the cache.
+--path split: ham_kv_append followed by ham_decode_attn (the same work in three kernels).
 The default workload is the Llama-3-8B-shaped layer: batch 8, 32 query / 8 KV heads,
 head_dim 128, 4096 slots per sequence in 16-slot pages scattered over a shared pool.
 
@@ -12,7 +13,8 @@ region is bracketed by a barrier and a device synchronize.  Four independent cac
 rotated so each step reads a cache last touched three steps earlier (4 x 128 MiB of KV,
 far above the 129 MB L2).  After each graph the four caches are rolled back to 4096 slots
 (ham_kv_set_lengths), so the attended length stays 4097..4112.  The attention kernel's
-own duration comes from CUDA events recorded around each of its launches inside the graph.
+own duration comes from CUDA events recorded around each of its launches inside the graph
+(fused: the step's attention + combine/commit kernels; split: attention + combine).
 
 Prints ONE JSON line on rank 0.  `--impl reference` times the CPU oracle instead.
 """
@@ -52,6 +54,8 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0,
                    help="CPU work budget of the oracle baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--path", choices=["fused", "split"], default="fused",
+                   help="fused: ham_decode_step; split: ham_kv_append + ham_decode_attn")
     return p.parse_args()
 
 
@@ -102,10 +106,10 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload_name):
-    """dram read+write bytes per attention launch from the committed ncu summary, if it was
-    taken on the current kernel source."""
-    path = os.path.join(ROOT, "profiles", f"decode_attn_{workload_name}.md")
+def profiled_traffic(kernel, workload_name):
+    """dram read+write bytes per launch of `kernel` (decode_step or decode_attn) from the
+    committed ncu summary, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload_name}.md")
     try:
         text = open(path).read()
     except OSError:
@@ -190,29 +194,46 @@ def workload(name):
     if name not in wl.WORKLOADS:
         raise SystemExit(f"unknown workload {name}; choose from {sorted(wl.WORKLOADS)}")
     w = wl.WORKLOADS[name]
-    if w.slot_range is not None or w.layers != 1:
-        raise SystemExit(f"bench times uniform single-layer workloads; {name} is a parity case")
+    if w.layers != 1:
+        raise SystemExit(f"bench times single-layer workloads; {name} has {w.layers} layers")
     return w
 
 
-def config_dict(w):
+def base_counts(w):
+    """Slots per sequence before the timed steps (uniform, or the workload's ragged draw)."""
+    from paper_2505_20438_gb300 import workload as wl
+    return wl.slot_counts(w, wl.rng_for(w.seed, 1))
+
+
+STEP_TEXT = {
+    "fused": "ham_decode_step: append of the slot (RoPE q,k) fused into attention over all slots",
+    "split": "ham_kv_append (RoPE q,k + append) then ham_decode_attn over all slots",
+}
+
+
+def config_dict(w, path="fused"):
+    counts = base_counts(w)
+    slots = w.slots if w.slot_range is None else (
+        f"{int(counts.min())}..{int(counts.max())} (mean {counts.mean():.0f}, uniform draw "
+        f"in [{w.slot_range[0]}, {w.slot_range[1]}])")
     return {"workload": w.name, "batch": w.batch, "n_q_heads": w.n_q_heads,
-            "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim, "slots": w.slots,
+            "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim, "slots": slots,
             "page_slots": w.page_slots, "pages": "scattered by a seeded shuffle of a shared pool",
             "tokens_per_slot": "geometric p=0.5 capped at 4 (mean 1.875)",
-            "step": "ham_kv_append (RoPE q,k + append) then ham_decode_attn over all slots",
+            "step": STEP_TEXT[path],
             "l2": f"{CACHES} independent caches rotated ({CACHES} x "
-                  f"{w.batch * w.slots * w.n_kv_heads * w.head_dim * 4 / 2**20:.0f} MiB KV "
+                  f"{int(counts.sum()) * w.n_kv_heads * w.head_dim * 4 / 2**20:.0f} MiB KV "
                   "> 129 MB L2)",
-            "graph": f"{GRAPH_STEPS} steps per CUDA graph, rollback to {w.slots} slots per graph"}
+            "graph": f"{GRAPH_STEPS} steps per CUDA graph, then each cache is rolled back "
+                     "to its starting slot counts"}
 
 
-def attn_bytes(w, L):
-    """Algorithmic bytes of one attention launch with L slots per sequence: K and V of every
-    slot once, q in, out, and the page-table entries."""
-    kv = w.batch * L * w.n_kv_heads * w.head_dim * 2 * 2
+def attn_bytes(w, lengths):
+    """Algorithmic bytes of one attention launch over sequences of `lengths` slots: K and V
+    of every slot once, q in, out, and the page-table entries."""
+    kv = sum(int(L) for L in lengths) * w.n_kv_heads * w.head_dim * 2 * 2
     qo = 2 * w.batch * w.n_q_heads * w.head_dim * 2
-    pt = w.batch * math.ceil(L / w.page_slots) * 4
+    pt = sum(math.ceil(int(L) / w.page_slots) for L in lengths) * 4
     return kv + qo + pt
 
 
@@ -234,19 +255,23 @@ def build_caches(w, device_index, rank):
     from paper_2505_20438_gb300 import workload as wl
 
     caches = []
-    max_slots = w.slots + GRAPH_STEPS // CACHES + 16
+    counts_h = base_counts(w)
+    lmax = int(counts_h.max())
+    max_slots = lmax + GRAPH_STEPS // CACHES + 16
     for r in range(CACHES):
         seed = rank_cache_seed(w.seed, rank, r)
         kv = ham.ham_kv_alloc(1, w.batch, w.n_q_heads, w.n_kv_heads, w.head_dim, w.page_slots,
                               max_slots, pool_pages=int(math.ceil(
                                   w.batch * math.ceil(max_slots / w.page_slots) * w.pool_factor)),
                               page_seed=seed + 1)
-        shape = (w.batch, w.slots, w.n_kv_heads, w.head_dim)
+        shape = (w.batch, lmax, w.n_kv_heads, w.head_dim)
         k = wl.device_normal_bf16(shape, w.value_scale, seed * 7 + 1)
         v = wl.device_normal_bf16(shape, w.value_scale, seed * 7 + 2)
         rng = wl.rng_for(seed, 5)
-        ntok = wl.ntok_capped_geometric(rng, (w.batch, w.slots))
-        counts = torch.full((w.batch,), w.slots, dtype=torch.int32, device="cuda")
+        ntok = wl.ntok_capped_geometric(rng, (w.batch, lmax))
+        for b in range(w.batch):
+            ntok[b, counts_h[b]:] = 0
+        counts = torch.from_numpy(counts_h.astype(np.int32)).cuda()
         ham.ham_kv_fill(kv, 0, k, v, counts, ntok=torch.from_numpy(ntok).cuda())
         del k, v
         tokens = torch.from_numpy(ntok.sum(axis=1).astype(np.int64)).cuda()
@@ -257,7 +282,7 @@ def build_caches(w, device_index, rank):
             "v_new": wl.device_normal_bf16((w.batch, w.n_kv_heads, w.head_dim), w.value_scale, seed * 7 + 5),
             "ntok_new": torch.from_numpy(wl.ntok_capped_geometric(rng, (w.batch,))).cuda(),
             "out": torch.empty((w.batch, w.n_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda"),
-            "mean_ntok": float(ntok.mean()),
+            "mean_ntok": float(ntok.sum() / max(1, counts_h.sum())),
         }
         caches.append(c)
     torch.cuda.synchronize()
@@ -282,9 +307,22 @@ def run_ours(args, w):
     n_warm = max(1, math.ceil(max(args.warmup, 3) / GRAPH_STEPS))
     steps = n_graph * GRAPH_STEPS
 
+    fused = args.path == "fused"
+
+    def append_part(c):
+        if not fused:
+            ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
+
+    def timed_part(c):
+        if fused:
+            ham.ham_decode_step(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"],
+                                c["out"])
+        else:
+            ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+
     def one_step(c):
-        ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
-        ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+        append_part(c)
+        timed_part(c)
 
     def rollback():
         for c in caches:
@@ -300,8 +338,10 @@ def run_ours(args, w):
     try:
         ev = [(torch.cuda.Event(enable_timing=True, external=True),
                torch.cuda.Event(enable_timing=True, external=True)) for _ in range(GRAPH_STEPS)]
-        per_launch_method = ("CUDA events around every ham_decode_attn (attention + combine "
-                             "kernels) of the last graph replay of the timed region")
+        per_launch_method = (("CUDA events around every ham_decode_step (attention + "
+                              "combine/commit kernels)" if fused else
+                              "CUDA events around every ham_decode_attn (attention + combine "
+                              "kernels)") + " of the last graph replay of the timed region")
     except TypeError:
         ev = None
         per_launch_method = "attention-only graph, CUDA events around the replay"
@@ -311,10 +351,10 @@ def run_ours(args, w):
         with torch.cuda.graph(g, stream=stream):
             for i in range(GRAPH_STEPS):
                 c = caches[i % CACHES]
-                ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
+                append_part(c)
                 if with_events:
                     ev[i][0].record()
-                ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+                timed_part(c)
                 if with_events:
                     ev[i][1].record()
             rollback()
@@ -324,12 +364,14 @@ def run_ours(args, w):
     # dependent launch between kernels); the last replay is an identical graph with events
     graph = capture(False)
     probe = capture(True) if ev is not None else graph
-    launches_per_graph = 3 * GRAPH_STEPS + CACHES   # append, attention, combine; rollbacks
+    # fused: attention + combine/commit; split: append, attention, combine; then rollbacks
+    launches_per_graph = (2 if fused else 3) * GRAPH_STEPS + CACHES
 
-    # attended lengths inside one graph: cache i % 4 sees w.slots + 1 + i // 4 slots
-    lengths = [w.slots + 1 + i // CACHES for i in range(GRAPH_STEPS)]
-    attn_bytes_graph = sum(attn_bytes(w, L) for L in lengths)
+    # attended lengths inside one graph: step i (cache i % 4) sees counts + 1 + i // 4 slots
+    counts_h = base_counts(w)
+    attn_bytes_graph = sum(attn_bytes(w, counts_h + 1 + i // CACHES) for i in range(GRAPH_STEPS))
     step_bytes_graph = attn_bytes_graph + GRAPH_STEPS * append_bytes(w)
+    timed_bytes_graph = step_bytes_graph if fused else attn_bytes_graph
 
     with torch.cuda.stream(stream):          # replay() launches on the current stream
         for _ in range(n_warm):
@@ -364,7 +406,8 @@ def run_ours(args, w):
         with torch.cuda.graph(g2, stream=stream):
             for i in range(GRAPH_STEPS):
                 c = caches[i % CACHES]
-                ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+                one_step(c)
+            rollback()
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(stream):
             a0.record(stream)
@@ -377,20 +420,20 @@ def run_ours(args, w):
             raise RuntimeError("device error during the timed region")
 
     peak, peak_src = measured_peak_hbm()
-    attn_gbs = attn_bytes_graph / (sum(attn_ms) * 1e-3) / 1e9
+    attn_gbs = timed_bytes_graph / (sum(attn_ms) * 1e-3) / 1e9
     ms_per_step = elapsed_ms / steps
     value = job_throughput(steps, world, elapsed_ms * 1e-3)
     step_gbs = world * n_graph * step_bytes_graph / (elapsed_ms * 1e-3) / 1e9
     mean_ntok = statistics.mean(c["mean_ntok"] for c in caches)
 
-    e2e = run_e2e(args, w, caches, stream, rollback, world)
+    e2e = run_e2e(args, w, caches, stream, rollback, world, one_step)
 
-    traffic = profiled_traffic(w.name)
+    traffic = profiled_traffic("decode_step" if fused else "decode_attn", w.name)
     result = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
         "steps": steps, "warmup": n_warm * GRAPH_STEPS, "ms_per_step": round(ms_per_step, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "accum_dtype": "f32", "data": "synthetic", "config": config_dict(w),
+        "accum_dtype": "f32", "data": "synthetic", "config": config_dict(w, args.path),
         "kv_gbs": round(step_gbs, 1),
         "kv_frac_of_measured_peak": round(step_gbs / world / peak, 4),
         "kv_frac_of_8tbs_spec": round(step_gbs / world / 8000.0, 4),
@@ -398,9 +441,11 @@ def run_ours(args, w):
         "tokens_per_s": round(value * w.batch * mean_ntok, 1),
         "roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(attn_gbs / peak, 4), "traffic": traffic,
-                     "kernel": "decode_attn_kernel<128,bf16> + combine_kernel<bf16>",
+                     "kernel": ("decode_attn_kernel<128,bf16,step> + combine_kernel<bf16,step>"
+                                if fused else
+                                "decode_attn_kernel<128,bf16> + combine_kernel<bf16>"),
                      "avg_launch_us": round(1e3 * statistics.mean(attn_ms), 3),
-                     "algorithmic_bytes_per_launch": int(attn_bytes_graph / GRAPH_STEPS),
+                     "algorithmic_bytes_per_launch": int(timed_bytes_graph / GRAPH_STEPS),
                      "peak_source": peak_src, "duration_method": per_launch_method},
         "gpu_launches": n_graph * launches_per_graph * world,
         "e2e": e2e,
@@ -414,12 +459,10 @@ def run_ours(args, w):
         torch.distributed.destroy_process_group()
 
 
-def run_e2e(args, w, caches, stream, rollback, world):
+def run_e2e(args, w, caches, stream, rollback, world, one_step):
     """Same steps through the public API with pinned host inputs copied in and the output
     copied back and read on the host every step."""
     import torch
-
-    from paper_2505_20438_gb300 import ham
 
     host = []
     for c in caches:
@@ -431,9 +474,7 @@ def run_e2e(args, w, caches, stream, rollback, world):
     checksum = 0.0
     with torch.cuda.stream(stream):
         for i in range(2 * CACHES):        # warm the eager path
-            c, h = caches[i % CACHES], host[i % CACHES]
-            ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
-            ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+            one_step(caches[i % CACHES])
         rollback()
         stream.synchronize()
         if world > 1:
@@ -443,8 +484,7 @@ def run_e2e(args, w, caches, stream, rollback, world):
             c, h = caches[i % CACHES], host[i % CACHES]
             for k in ("q", "k_new", "v_new", "ntok_new"):
                 c[k].copy_(h[k], non_blocking=True)
-            ham.ham_kv_append(c["kv"], 0, c["q"], c["k_new"], c["v_new"], None, c["ntok_new"])
-            ham.ham_decode_attn(c["kv"], 0, c["q"], c["out"])
+            one_step(c)
             h["out"].copy_(c["out"], non_blocking=True)
             stream.synchronize()
             checksum += float(h["out"][0, 0, 0])      # the host reads the step's result
@@ -455,7 +495,7 @@ def run_e2e(args, w, caches, stream, rollback, world):
     dt = max_over_ranks(dt, world, "cuda")
     return {"value": round(job_throughput(n, world, dt), 2), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": n,
-            "path": "pinned host -> device copies, ham_kv_append, ham_decode_attn, "
+            "path": "pinned host -> device copies, the step's C-ABI call(s), "
                     "device -> pinned host copy, host sync, every step (eager)",
             "finite": math.isfinite(checksum)}
 
@@ -507,12 +547,14 @@ def run_reference(args, w):
     # sub-case of the workload: fewer sequences, or one sequence with fewer slots, sized so
     # the whole run is about 40 full macro-steps of oracle work.  Attention work is linear
     # in the slot count, so the value is scaled by the sampled fraction of slots.
+    total = int(base_counts(w).sum())          # slots attended by one full macro-step
+    mean_l = max(1, total // w.batch)
     frac = min(1.0, 40.0 / (steps + warm))
     if frac * w.batch >= 1.0:
-        sub_b, sub_l = max(1, int(round(frac * w.batch))), w.slots
+        sub_b, sub_l = max(1, int(round(frac * w.batch))), mean_l
     else:
-        sub_b, sub_l = 1, max(16, int(round(frac * w.batch * w.slots)))
-    sub = dataclasses.replace(w, batch=sub_b, slots=sub_l)
+        sub_b, sub_l = 1, max(16, int(round(frac * total)))
+    sub = dataclasses.replace(w, batch=sub_b, slots=sub_l, slot_range=None)
     case = wl.make_case(sub, extra_slots=4)
     oc = oracle.OracleCache.from_case(case)
     def one():
@@ -526,7 +568,7 @@ def run_reference(args, w):
     for _ in range(steps):
         one()
     dt = time.perf_counter() - t0
-    share = (sub_b * sub_l) / (w.batch * w.slots)
+    share = (sub_b * sub_l) / total
     value = steps * share / dt
     sample = (f"each step: append + attention of all heads for {sub_b} sequence(s) x {sub_l} "
               f"slots = {share:.4f} of a {w.name} macro-step; {steps} steps timed")

@@ -141,6 +141,25 @@ int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
  * share the handle's scratch); serialize them on one stream. */
 int ham_decode_attn(ham_kv *kv, int32_t layer, const void *q, void *out, void *stream);
 
+/* ham_kv_append followed by ham_decode_attn in one pass over the cache (Sec. 3.1 + Sec. 3.4:
+ * the macro-step's slot is stored and every query head then attends over the slot list
+ * that includes it).  Same arguments and meaning as those two calls, with q_inout required:
+ * on return the cache, the counters and q_inout hold exactly what ham_kv_append leaves
+ * (fp64 RoPE, bf16 round-to-nearest-even), and out holds the attention of the rotated q
+ * over the n + 1 slots.  Inside the attention pass, q and the new key are rotated in fp32
+ * from a float cos/sin table, so a rotated element can differ from the stored one by one
+ * bf16 ulp; out stays within the ham_decode_attn tolerance of the two-call result.
+ * A sequence whose append fails (full, ntok < 1, bad counter) is not appended, keeps its
+ * unrotated q, attends over its old slots and sets the device error word, as the two calls
+ * would.  Two launches on `stream` (the second with programmatic dependent launch).
+ * out      device [batch][n_q_heads][head_dim], bf16 or f32 (out_dtype); must not overlap
+ *          q_inout.  k_new / v_new must not overlap the cache.
+ * Host errors: HAM_EINVAL (NULL / unaligned / overlapping pointers, layer out of range,
+ * out_dtype), HAM_ECUDA.  Same serialization rule as ham_decode_attn. */
+int ham_decode_step(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
+                    const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
+                    int32_t out_dtype, void *stream);
+
 /* Slot and token counts of every sequence after the last layer's appends (synchronous:
  * copies on `stream`, then waits for it).  num_slots_host [batch], num_tokens_host [batch]
  * (either may be NULL).  Returns HAM_EDEVICE if the device error word is set. */

@@ -1,11 +1,13 @@
 // Fused RoPE + append of the slot a macro-step produces (HAMburger Sec. 3.1: one KV set
 // per macro-step; Sec. 3.2: the merged embedding enters at an offset position).
 //
-// One cluster per sequence, one CTA per KV head (or a few).  The rotation is computed in fp64 from an fp64 frequency table
-// (base^(-2i/d), made on the host) and fp64 sin/cos, then rounded once to bf16
-// (nearest, ties to even).  Doing the whole rotation in fp64 makes the stored bits the
-// correctly rounded value of the exact rotation except within ~1e-16 relative of a bf16
-// rounding boundary, so an independent fp64 implementation reproduces them.
+// One thread-block cluster per sequence, one CTA per KV head (or a few).  The rotation is
+// computed in fp64 and rounded once to bf16 (nearest, ties to even).  cos and sin of
+// p * base^(-2i/d) come from a table the host fills at allocation with libm (positions the
+// cache can reach); past the table the kernel falls back to fp64 sincos.  With fp64
+// operands the stored bits are the correctly rounded exact rotation except within ~1e-16
+// relative of a bf16 rounding boundary, so an independent fp64 implementation reproduces
+// them (and with tabled cos/sin the operands are the ones such an implementation gets).
 #include <cuda_bf16.h>
 
 #include "ham_internal.cuh"
@@ -77,11 +79,14 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(AppendView v) {
     for (int i = threadIdx.x; i < ng * G * vec; i += blockDim.x)
       reinterpret_cast<uint4 *>(q_s)[i] = reinterpret_cast<const uint4 *>(v.q + src)[i];
   }
+  // every thread learns the position, so the cos/sin fetch overlaps the page lookup
+  const int32_t n = v.num_slots[b];
+  const int64_t p = v.pos ? (int64_t)v.pos[b] : (v.pos_mode == HAM_POS_SLOT ? (int64_t)n : v.num_tokens[b]);
+  const bool tabled = p >= 0 && p < v.rope_positions;
+  double2 cs_sn = make_double2(1.0, 0.0);
+  if (tabled && threadIdx.x < half) cs_sn = v.rope_table[p * half + threadIdx.x];
   if (threadIdx.x == 0) {
-    const int32_t n = v.num_slots[b];
     const int32_t t = v.ntok[b];
-    const int64_t tokens = v.num_tokens[b];
-    const int64_t p = v.pos ? (int64_t)v.pos[b] : (v.pos_mode == HAM_POS_SLOT ? (int64_t)n : tokens);
     int32_t err = 0;
     if (t < 1) {
       err = HAM_DEVERR_NTOK;
@@ -111,10 +116,9 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(AppendView v) {
     v.num_tokens[b] += s_ntok;
   }
   if (threadIdx.x < half) {
-    double sn, cs;
-    sincos((double)s_pos * inv_freq, &sn, &cs);
-    cos_t[threadIdx.x] = cs;
-    sin_t[threadIdx.x] = sn;
+    if (!tabled) sincos((double)p * inv_freq, &cs_sn.y, &cs_sn.x);
+    cos_t[threadIdx.x] = cs_sn.x;
+    sin_t[threadIdx.x] = cs_sn.y;
   }
   __syncthreads();
   const int64_t page = s_row_meta / v.page_slots;

@@ -44,7 +44,7 @@ namespace {
 constexpr uint32_t kFull = 0xffffffffu;
 constexpr float kRescaleSlack = 8.0f;              // log2 units
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // bounded waits: 2 s
-constexpr int kFirst = 1, kLast = 2, kPageOk = 4;  // stage flags
+constexpr int kFirst = 1, kLast = 2, kPageOk = 4, kNewRow = 8;  // stage flags
 constexpr int kMaxGroup = 8;                       // heads padded to the MMA's N = 8
 
 // ------------------------------------------------------------------------------------
@@ -196,7 +196,7 @@ __device__ __forceinline__ void store_out(void *out, int64_t i, float x) {
 // ------------------------------------------------------------------------------------
 // Shape of one kernel instance
 // ------------------------------------------------------------------------------------
-constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
+__host__ __device__ constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
 template <int D>
 struct Shape {
@@ -204,21 +204,40 @@ struct Shape {
   static constexpr int kStageBytes = 2 * kChunkBytes;
   static constexpr int kStages = 32768 / kStageBytes;       // 32 KiB ring
   static constexpr int kQBufs = kStages + 1;
-  static constexpr int kQBytes = kMaxGroup * D * 2;
   static constexpr int kThreads = 64;                       // consumer warp, producer warp
   static constexpr int kSteps = D / 16;                     // k-steps of q.k, m-tiles of p.v
   static constexpr int kLinesPerRow = D / 64;               // 128-byte swizzle lines per row
-  // shared memory map (offsets from a 1024-byte aligned base)
-  static constexpr int kOffQ = kStages * kStageBytes;
-  static constexpr int kOffBar = kOffQ + kQBufs * kQBytes;
-  static constexpr int kOffInfo = align_up(kOffBar + (2 * kStages) * 8, 16);
-  static constexpr int kOffFlags = kOffInfo + kStages * 16;
-  static constexpr int kOffCum = kOffFlags + 16;
-  static size_t smem_bytes(int batch) {
-    return 1024 + (size_t)kOffCum + 4u * (2u * batch + 1u);
-  }
+  static constexpr int kOffQ = kStages * kStageBytes;       // from a 1024-byte aligned base
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
   static_assert(kStages >= 2, "ring depth");
+};
+
+// Per-segment buffer: the group's q heads, and for the fused step also the new k and v
+// rows and the fp32 (cos, sin) of the new slot's position.
+template <int D>
+struct SegBuf {
+  int q_bytes, stride;
+  __host__ __device__ SegBuf(int group, bool step)
+      : q_bytes(group * D * 2),
+        stride(align_up(group * D * 2 + (step ? 2 * D * 2 + (D / 2) * 8 : 0), 128)) {}
+  __host__ __device__ int k_off() const { return q_bytes; }
+  __host__ __device__ int v_off() const { return q_bytes + D * 2; }
+  __host__ __device__ int cs_off() const { return q_bytes + 2 * D * 2; }
+};
+
+// Shared memory map after the per-segment buffers (runtime: depends on group and batch).
+template <int D>
+struct Layout {
+  int off_bar, off_info, off_flags, off_cum, total;
+  __host__ __device__ Layout(int group, bool step, int batch) {
+    using S = Shape<D>;
+    off_bar = S::kOffQ + S::kQBufs * SegBuf<D>(group, step).stride;
+    off_info = align_up(off_bar + 2 * S::kStages * 8, 16);
+    off_flags = off_info + S::kStages * 16;
+    off_cum = off_flags + 16;
+    // cum [B+1], lens [B], and for the fused step the new slot's position and flag [B] each
+    total = off_cum + 4 * (batch + 1) + 4 * batch * (step ? 3 : 1);
+  }
 };
 
 // Byte offset of the 16-byte piece `c` (elements c*8 .. c*8+7) of slot row `slot` inside a
@@ -230,28 +249,43 @@ __device__ __forceinline__ uint32_t tile_offset(int slot, int c) {
   return (uint32_t)(line * 128 + (((c & 7) ^ (line & 7)) << 4));
 }
 
+__device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {
+  return __uint_as_float((uint32_t)b << 16);
+}
+
+// Position of the slot a fused step appends to sequence b (slot index n or tokens so far,
+// unless given).
+__device__ __forceinline__ int64_t step_position(const StepArgs &st, int b, int n) {
+  if (st.pos) return st.pos[b];
+  return st.pos_mode == HAM_POS_SLOT ? (int64_t)n : st.num_tokens[b];
+}
+
 // ------------------------------------------------------------------------------------
 // The kernel
 // ------------------------------------------------------------------------------------
-template <int D, typename OutT>
+template <int D, typename OutT, bool kStep>
 __global__ void __launch_bounds__(Shape<D>::kThreads)
     decode_attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
                        const __grid_constant__ CUtensorMap tmap_v, const AttnView v) {
   using S = Shape<D>;
+  const int B = v.batch, Hkv = v.n_kv_heads, G = v.group;
+  const SegBuf<D> sb(G, kStep);
+  const Layout<D> lay(G, kStep, B);
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t *stages = smem;
   uint8_t *qbufs = smem + S::kOffQ;
-  uint64_t *full = reinterpret_cast<uint64_t *>(smem + S::kOffBar);
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + lay.off_bar);
   uint64_t *empty = full + S::kStages;
-  int4 *info = reinterpret_cast<int4 *>(smem + S::kOffInfo);
-  volatile int *flags = reinterpret_cast<volatile int *>(smem + S::kOffFlags);  // abort
-  int32_t *cum = reinterpret_cast<int32_t *>(smem + S::kOffCum);  // [B+1] chunk prefix
-  int32_t *lens = cum + v.batch + 1;                               // [B] slots
+  int4 *info = reinterpret_cast<int4 *>(smem + lay.off_info);
+  volatile int *flags = reinterpret_cast<volatile int *>(smem + lay.off_flags);  // abort
+  int32_t *cum = reinterpret_cast<int32_t *>(smem + lay.off_cum);  // [B+1] chunk prefix
+  int32_t *lens = cum + B + 1;                                      // [B] slots attended
+  int32_t *posb = lens + B;                                         // [B] new slot position
+  int32_t *appb = posb + B;                                         // [B] 1: append happens
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int B = v.batch, Hkv = v.n_kv_heads, G = v.group;
 
   if (tid == 0) {
     for (int s = 0; s < S::kStages; ++s) {
@@ -277,9 +311,22 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
       int n = 0;
       if (b < B) {
         int L = v.num_slots[b];
-        if (L < 0 || L > v.max_slots) {
+        const bool bad = L < 0 || L > v.max_slots;
+        if (bad) {
           record_error(v.err, HAM_DEVERR_SLOTS);
           L = L < 0 ? 0 : v.max_slots;
+        }
+        if constexpr (kStep) {  // the slot this step appends is attended too
+          const int t = v.step.ntok[b];
+          // 0: append; else the error that stops it (same order as ham_kv_append)
+          const int why = t < 1 ? HAM_DEVERR_NTOK
+                          : bad ? HAM_DEVERR_SLOTS
+                          : L == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
+          const int64_t p = step_position(v.step, b, L);
+          posb[b] = (int32_t)p;
+          appb[b] = why == 0;
+          if (blockIdx.x == 0) v.step.stash[b] = make_int4(L, why, (int32_t)p, t);
+          L += why == 0;
         }
         lens[b] = L;
         n = chunks_of(L);
@@ -318,7 +365,6 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
   // ---------------------------------------------------------------- producer warp
   if (warp == 1) {
     const uint64_t pol = policy_evict_first();
-    const uint32_t qbytes = (uint32_t)(G * D * 2);
     int it = 0, nseg = 0;
     for (int base = 0; base < nchunks; base += 32) {
       const int nb = min(32, nchunks - base);
@@ -342,6 +388,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
         row0 = ((page_ok ? page : 0) * Hkv + g) * v.page_slots + slot0 % v.page_slots;
         fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
              ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
+        if (kStep && c == nch - 1 && appb[b]) fl |= kNewRow;  // holds the appended slot
       }
       bool stop = false;
       for (int j = 0; j < nb; ++j) {
@@ -359,10 +406,19 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
             failed = 1;
           } else {
             int qb = -1;
+            bool tabled = false;
+            const int b = s_seg / Hkv;
             if (s_fl & kFirst) qb = nseg++ % S::kQBufs;
             info[stage] = make_int4(s_seg, s_valid, s_fl, qb);
             uint32_t bytes = (s_fl & kPageOk) ? (uint32_t)S::kStageBytes : 0u;
-            if (qb >= 0) bytes += qbytes;
+            if (qb >= 0) {
+              bytes += (uint32_t)sb.q_bytes;
+              if constexpr (kStep) {
+                const int64_t p = posb[b];
+                tabled = p >= 0 && p < v.step.rope_positions;
+                bytes += 2u * D * 2 + (tabled ? (uint32_t)(D / 2) * 8 : 0u);
+              }
+            }
             if (bytes) mbar_arrive_tx(&full[stage], bytes);
             else mbar_arrive(&full[stage]);
             uint8_t *dst = stages + stage * S::kStageBytes;
@@ -372,9 +428,18 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
             } else {
               record_error(v.err, HAM_DEVERR_PAGE);
             }
-            if (qb >= 0)
-              bulk_load(qbufs + qb * S::kQBytes, v.q + (int64_t)s_seg * G * D, qbytes,
-                        &full[stage]);
+            if (qb >= 0) {
+              uint8_t *qdst = qbufs + qb * sb.stride;
+              bulk_load(qdst, v.q + (int64_t)s_seg * G * D, (uint32_t)sb.q_bytes, &full[stage]);
+              if constexpr (kStep) {  // the new k, v rows and (cos, sin) of its position
+                bulk_load(qdst + sb.k_off(), v.step.k_new + (int64_t)s_seg * D, D * 2, &full[stage]);
+                bulk_load(qdst + sb.v_off(), v.step.v_new + (int64_t)s_seg * D, D * 2, &full[stage]);
+                if (tabled)
+                  bulk_load(qdst + sb.cs_off(),
+                            v.step.rope_table_f + (int64_t)posb[b] * (D / 2), (D / 2) * 8,
+                            &full[stage]);
+              }
+            }
           }
         }
         if (__shfl_sync(kFull, failed, 0)) {
@@ -408,6 +473,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
   uint32_t qb[S::kSteps][2];  // B fragments of Q^T for the current segment
   float o[S::kSteps][4];      // O^T fragments: rows = head_dim, columns = heads
   float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  int cur_qb = 0;
 #pragma unroll
   for (int t = 0; t < S::kSteps; ++t) {
     o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
@@ -425,7 +491,38 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     }
     const int4 inf = info[stage];
     if (inf.z & kFirst) {  // Q^T fragments of a new segment (heads >= G are zero)
-      const uint16_t *q = reinterpret_cast<const uint16_t *>(qbufs + inf.w * S::kQBytes);
+      cur_qb = inf.w;
+      uint16_t *q = reinterpret_cast<uint16_t *>(qbufs + cur_qb * sb.stride);
+      const int b = inf.x / Hkv;
+      if (kStep && appb[b]) {
+        // Turn q and the new key by the new slot's position (fp32 from the fp32 table; the
+        // exact fp64 rotation is committed by the combine kernel).  Lane handles pairs
+        // (i, i + D/2) for i = lane (+ 32).
+        const int64_t p = posb[b];
+        const bool tabled = p >= 0 && p < v.step.rope_positions;
+        const float2 *cs = reinterpret_cast<const float2 *>(qbufs + cur_qb * sb.stride + sb.cs_off());
+        uint16_t *kn = reinterpret_cast<uint16_t *>(qbufs + cur_qb * sb.stride + sb.k_off());
+        for (int i = lane; i < D / 2; i += 32) {
+          float c, s;
+          if (tabled) {
+            c = cs[i].x;
+            s = cs[i].y;
+          } else {
+            double sd, cd;
+            sincos((double)p * v.step.inv_freq[i], &sd, &cd);
+            c = (float)cd;
+            s = (float)sd;
+          }
+          for (int h = 0; h <= G; ++h) {  // G query heads, then the key
+            uint16_t *row = h < G ? q + h * D : kn;
+            const float x0 = bf16_bits_to_float(row[i]), x1 = bf16_bits_to_float(row[i + D / 2]);
+            row[i] = __bfloat16_as_ushort(__float2bfloat16_rn(x0 * c - x1 * s));
+            row[i + D / 2] = __bfloat16_as_ushort(__float2bfloat16_rn(x1 * c + x0 * s));
+          }
+        }
+        fence_proxy_async_smem();  // these writes vs a later bulk copy into this buffer
+        __syncwarp();
+      }
 #pragma unroll
       for (int t = 0; t < S::kSteps; ++t) {
         if (r0 < G) {
@@ -440,28 +537,38 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
       uint8_t *kt = stages + stage * S::kStageBytes;
       uint8_t *vt = kt + S::kChunkBytes;
       const int nvalid = inf.y;
+      const bool patch = nvalid < kChunkSlots || (kStep && (inf.z & kNewRow));
       if (nvalid < kChunkSlots) {  // rows past the sequence end never reach the MMA
         for (int i = lane; i < (kChunkSlots - nvalid) * (D / 8); i += 32) {
           const int slot = nvalid + i / (D / 8), c = i % (D / 8);
           *reinterpret_cast<uint4 *>(vt + tile_offset<D>(slot, c)) = make_uint4(0, 0, 0, 0);
         }
-        __syncwarp();
       }
+      if (kStep && (inf.z & kNewRow)) {  // the appended slot is the chunk's last valid row
+        const uint8_t *seg = qbufs + cur_qb * sb.stride;
+        for (int i = lane; i < 2 * (D / 8); i += 32) {
+          const int c = i % (D / 8);
+          const bool is_v = i >= D / 8;
+          const uint4 x = *reinterpret_cast<const uint4 *>(seg + (is_v ? sb.v_off() : sb.k_off()) + c * 16);
+          *reinterpret_cast<uint4 *>((is_v ? vt : kt) + tile_offset<D>(nvalid - 1, c)) = x;
+        }
+      }
+      if (patch) __syncwarp();
       const uint32_t kbase = smem_u32(kt), vbase = smem_u32(vt);
       // S^T (16 slots x 8 heads) = K (16 x D) . Q^T (D x 8), two accumulators for ILP
-      float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+      float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int t = 0; t < S::kSteps; ++t) {
         uint32_t a[4];
         ldmatrix_x4(a, kbase + tile_offset<D>(a_slot, 2 * t + a_half));
-        if (t & 1) mma_16816(sb, a, qb[t][0], qb[t][1]);
+        if (t & 1) mma_16816(sb4, a, qb[t][0], qb[t][1]);
         else mma_16816(sa, a, qb[t][0], qb[t][1]);
       }
       const bool v0 = r0 < nvalid, v1 = r0 + 8 < nvalid;
-      const float x0 = (v0 && hv0) ? (sa[0] + sb[0]) * qscale : -INFINITY;
-      const float x1 = (v0 && hv1) ? (sa[1] + sb[1]) * qscale : -INFINITY;
-      const float x2 = (v1 && hv0) ? (sa[2] + sb[2]) * qscale : -INFINITY;
-      const float x3 = (v1 && hv1) ? (sa[3] + sb[3]) * qscale : -INFINITY;
+      const float x0 = (v0 && hv0) ? (sa[0] + sb4[0]) * qscale : -INFINITY;
+      const float x1 = (v0 && hv1) ? (sa[1] + sb4[1]) * qscale : -INFINITY;
+      const float x2 = (v1 && hv0) ? (sa[2] + sb4[2]) * qscale : -INFINITY;
+      const float x3 = (v1 && hv1) ? (sa[3] + sb4[3]) * qscale : -INFINITY;
       float t0 = fmaxf(x0, x2), t1 = fmaxf(x1, x3);
 #pragma unroll
       for (int off = 4; off < 32; off <<= 1) {
@@ -502,7 +609,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
         ldmatrix_x4_trans(a, vbase + tile_offset<D>(v_slot, 2 * t + v_half));
         mma_16816(o[t], a, bp0, bp1);
       }
-      if (nvalid < kChunkSlots) fence_proxy_async_smem();  // zeroed rows vs the next TMA
+      if (patch) fence_proxy_async_smem();  // patched rows vs the next TMA into this stage
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[stage]);
@@ -566,51 +673,140 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
 // ------------------------------------------------------------------------------------
 // Combine: out[seg][h][d] = sum_k 2^(m_k - M) acc_k[h][d] / sum_k 2^(m_k - M) l_k over the
 // CTAs k = first..last of the segment, M = max_k m_k (split-softmax merge, in CTA order).
-// One thread per output element; blocks of kCombineThreads cover one segment's G*D values.
+// One thread per output element; blocks of kCombineThreads cover one segment's G*D values
+// (whole heads: kCombineThreads is a multiple of head_dim).
+//
+// For the fused step the same threads also commit the append once the whole attention grid
+// has finished (nothing may change q_inout or the counters while it still reads them):
+// element (h, d) of q_inout and, for h = 0, element d of the key and value rows.  Each is
+// the fp64 rotation of the pair (d, d +- D/2) rounded once to bf16, as ham_kv_append does.
+// The inputs that the attention pass only reads are loaded before waiting for it, so the
+// commit's dependent loads (append record -> cos/sin, page) run beside the merge's
+// (segment range -> partials).  KV head 0 writes the slot metadata and counters.
 // ------------------------------------------------------------------------------------
 constexpr int kCombineThreads = 128;
+static_assert(kCombineThreads % 128 == 0, "a block holds whole heads of head_dim 64 or 128");
 
-template <typename OutT>
-__global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView v, int D,
-                                                                  int blocks_per_seg) {
-  grid_dependency_wait();  // the attention grid's partials and ranges are visible
-  const int G = v.group;
-  const int seg = blockIdx.x / blocks_per_seg;
-  const int idx = (blockIdx.x % blocks_per_seg) * kCombineThreads + threadIdx.x;
-  const int2 r = v.seg_range[seg];
-  if (r.x < 0 || r.x == r.y || idx >= G * D) return;
-  const int h = idx / D;
-  // Online merge in batches of 8 partials: the 8 loads of a batch are in flight together.
-  constexpr int kBatch = 8;
-  float M = -INFINITY, num = 0.f, den = 0.f;
-  for (int k0 = r.x; k0 <= r.y; k0 += kBatch) {
-    float2 ml[kBatch];
-    float acc[kBatch];
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      const int64_t p = (int64_t)k0 + j + seg;
-      const bool in = k0 + j <= r.y;
-      ml[j] = in ? __ldcg(&v.part_ml[p * G + h]) : make_float2(-INFINITY, 0.f);
-      acc[j] = in ? __ldcg(&v.part_acc[p * G * D + idx]) : 0.f;
-    }
-    float bm = M;
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) bm = fmaxf(bm, ml[j].x);
-    const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
-    num *= scale;
-    den *= scale;
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      const float w = (ml[j].x == -INFINITY) ? 0.f : ex2(ml[j].x - bm);
-      num += w * acc[j];
-      den += w * ml[j].y;
-    }
-    M = bm;
-  }
-  store_out<OutT>(v.out, (int64_t)seg * G * D + idx, num / den);
+__device__ __forceinline__ double bf16_bits_to_double(uint16_t b) {
+  return (double)__uint_as_float((uint32_t)b << 16);
 }
 
-template <typename OutT>
+// One element of the rotated pair (i, i + D/2): y_i = x_i c - x_{i+D/2} s for the low half,
+// y_{i+D/2} = x_{i+D/2} c + x_i s for the high half (explicit fp64 operations, no FMA).
+__device__ __forceinline__ uint16_t rotate_elem(double self, double other, double c, double s,
+                                                bool high) {
+  const double y = high ? __dadd_rn(__dmul_rn(self, c), __dmul_rn(other, s))
+                        : __dsub_rn(__dmul_rn(self, c), __dmul_rn(other, s));
+  return __bfloat16_as_ushort(__double2bfloat16(y));
+}
+
+template <typename OutT, bool kStep>
+__global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView v, int D,
+                                                                  int blocks_per_seg) {
+  const int G = v.group, Hkv = v.n_kv_heads;
+  const int seg = blockIdx.x / blocks_per_seg;
+  const int part = blockIdx.x % blocks_per_seg;
+  const int idx = part * kCombineThreads + threadIdx.x;
+  const bool active = idx < G * D;
+  const int h = idx / D, d = idx - h * D;
+
+  // fused step: operands of this thread's commit that the attention pass only reads
+  const int half = D / 2;
+  const bool high = d >= half;
+  const int i = high ? d - half : d, partner = high ? d - half : d + half;
+  double q_self = 0.0, q_other = 0.0, k_self = 0.0, k_other = 0.0, inv_freq = 0.0;
+  uint16_t v_el = 0;
+  const int64_t qrow = (int64_t)seg * G * D + (int64_t)h * D;  // == (b*Hq + g*G + h) * D
+  if (kStep && active) {
+    const StepArgs &st = v.step;
+    q_self = bf16_bits_to_double(st.q_inout[qrow + d]);
+    q_other = bf16_bits_to_double(st.q_inout[qrow + partner]);
+    if (h == 0) {
+      k_self = bf16_bits_to_double(st.k_new[(int64_t)seg * D + d]);
+      k_other = bf16_bits_to_double(st.k_new[(int64_t)seg * D + partner]);
+      v_el = st.v_new[(int64_t)seg * D + d];
+    }
+    inv_freq = st.inv_freq[i];
+  }
+
+  grid_dependency_wait();  // the attention grid's partials, ranges and append records
+  if constexpr (kStep) __syncthreads();  // every q read above precedes any q write below
+
+  const int2 r = v.seg_range[seg];
+  int4 rec = make_int4(0, 0, 0, 0);
+  if constexpr (kStep) rec = v.step.stash[seg / Hkv];  // (n, 0 or error, position, ntok)
+
+  if (active && r.x >= 0 && r.x != r.y) {
+    // Online merge in batches of 8 partials: the 8 loads of a batch are in flight together.
+    constexpr int kBatch = 8;
+    float M = -INFINITY, num = 0.f, den = 0.f;
+    for (int k0 = r.x; k0 <= r.y; k0 += kBatch) {
+      float2 ml[kBatch];
+      float acc[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int64_t p = (int64_t)k0 + j + seg;
+        const bool in = k0 + j <= r.y;
+        ml[j] = in ? __ldcg(&v.part_ml[p * G + h]) : make_float2(-INFINITY, 0.f);
+        acc[j] = in ? __ldcg(&v.part_acc[p * G * D + idx]) : 0.f;
+      }
+      float bm = M;
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) bm = fmaxf(bm, ml[j].x);
+      const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
+      num *= scale;
+      den *= scale;
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const float w = (ml[j].x == -INFINITY) ? 0.f : ex2(ml[j].x - bm);
+        num += w * acc[j];
+        den += w * ml[j].y;
+      }
+      M = bm;
+    }
+    store_out<OutT>(v.out, (int64_t)seg * G * D + idx, num / den);
+  }
+
+  if constexpr (kStep) {
+    const StepArgs &st = v.step;
+    const int b = seg / Hkv, g = seg - b * Hkv;
+    const bool lead = g == 0 && idx == 0;  // one thread per sequence
+    if (rec.y) {                           // no append for this sequence
+      if (lead) record_error(v.err, rec.y);
+      return;
+    }
+    if (!active) return;
+    const int n = rec.x;
+    const int64_t p = rec.z;
+    double c, sn;
+    if (p >= 0 && p < st.rope_positions) {
+      const double2 e = st.rope_table[p * half + i];
+      c = e.x;
+      sn = e.y;
+    } else {
+      sincos((double)p * inv_freq, &sn, &c);
+    }
+    st.q_inout[qrow + d] = rotate_elem(q_self, q_other, c, sn, high);
+    if (h != 0) return;
+    const int page = v.page_table[(int64_t)b * v.max_pages + n / v.page_slots];
+    if (page < 0 || page >= v.pool_pages) {
+      if (lead) record_error(v.err, HAM_DEVERR_PAGE);
+      return;
+    }
+    const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
+    st.k_pool[row + d] = rotate_elem(k_self, k_other, c, sn, high);
+    st.v_pool[row + d] = v_el;
+    if (lead) {
+      const int64_t meta = (int64_t)page * v.page_slots + n % v.page_slots;
+      st.slot_pos[meta] = (int32_t)p;
+      st.slot_ntok[meta] = rec.w;
+      st.num_slots[b] = n + 1;
+      st.num_tokens[b] += rec.w;
+    }
+  }
+}
+
+template <typename OutT, bool kStep>
 cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream) {
   const int per_seg = (v.group * head_dim + kCombineThreads - 1) / kCombineThreads;
   cudaLaunchConfig_t cfg = {};
@@ -622,17 +818,20 @@ cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream)
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, combine_kernel<OutT>, v, head_dim, per_seg);
+  return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep>, v, head_dim, per_seg);
 }
 
 // ------------------------------------------------------------------------------------
 // Dispatch
 // ------------------------------------------------------------------------------------
-template <int D, typename OutT>
+template <int D, typename OutT, bool kStep>
 struct Instance {
   using S = Shape<D>;
-  static auto fn() { return &decode_attn_kernel<D, OutT>; }
-  // Allow the largest dynamic shared memory any batch needs, once per device.
+  static auto fn() { return &decode_attn_kernel<D, OutT, kStep>; }
+  static size_t smem_bytes(int group, int batch) {
+    return 1024 + (size_t)Layout<D>(group, kStep, batch).total;
+  }
+  // Allow the largest dynamic shared memory any group and batch need, once per device.
   static cudaError_t configure() {
     static std::mutex mu;
     static bool done[64] = {};
@@ -642,7 +841,7 @@ struct Instance {
     std::lock_guard<std::mutex> lock(mu);
     if (dev >= 0 && dev < 64 && done[dev]) return cudaSuccess;
     e = cudaFuncSetAttribute(fn(), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)S::smem_bytes(kMaxBatch));
+                             (int)smem_bytes(kMaxGroup, kMaxBatch));
     if (e == cudaSuccess && dev >= 0 && dev < 64) done[dev] = true;
     return e;
   }
@@ -653,31 +852,31 @@ struct Instance {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)v.ctas);
     cfg.blockDim = dim3(S::kThreads);
-    cfg.dynamicSmemBytes = S::smem_bytes(v.batch);
+    cfg.dynamicSmemBytes = smem_bytes(v.group, v.batch);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<D, OutT>, tk, tv, v);
+    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<D, OutT, kStep>, tk, tv, v);
     if (e != cudaSuccess) return e;
-    return launch_combine<OutT>(v, D, stream);
+    return launch_combine<OutT, kStep>(v, D, stream);
   }
-  static int ctas_per_sm(int batch) {
+  static int ctas_per_sm(int group, int batch) {
     if (configure() != cudaSuccess) return 0;
     int n = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn(), S::kThreads,
-                                                      S::smem_bytes(batch)) != cudaSuccess)
+                                                      smem_bytes(group, batch)) != cudaSuccess)
       return 0;
     return n;
   }
 };
 
-template <typename OutT, typename F>
+template <typename OutT, bool kStep, typename F>
 cudaError_t dispatch(int head_dim, F &&f) {
-  if (head_dim == 128) return f(Instance<128, OutT>());
-  if (head_dim == 64) return f(Instance<64, OutT>());
+  if (head_dim == 128) return f(Instance<128, OutT, kStep>());
+  if (head_dim == 64) return f(Instance<64, OutT, kStep>());
   return cudaErrorInvalidValue;
 }
 
@@ -691,16 +890,26 @@ cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const
                              int head_dim, int out_dtype, cudaStream_t stream) {
   if (v.ctas < 1 || v.group < 1 || v.group > kMaxGroup) return cudaErrorInvalidConfiguration;
   auto go = [&](auto inst) { return decltype(inst)::launch(tk, tv, v, stream); };
-  return out_dtype == HAM_DTYPE_F32 ? dispatch<float>(head_dim, go)
-                                    : dispatch<__nv_bfloat16>(head_dim, go);
+  return out_dtype == HAM_DTYPE_F32 ? dispatch<float, false>(head_dim, go)
+                                    : dispatch<__nv_bfloat16, false>(head_dim, go);
 }
 
-int attention_ctas_per_sm(int head_dim, int batch) {
+cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
+                               int head_dim, int out_dtype, cudaStream_t stream) {
+  if (v.ctas < 1 || v.group < 1 || v.group > kMaxGroup) return cudaErrorInvalidConfiguration;
+  auto go = [&](auto inst) { return decltype(inst)::launch(tk, tv, v, stream); };
+  return out_dtype == HAM_DTYPE_F32 ? dispatch<float, true>(head_dim, go)
+                                    : dispatch<__nv_bfloat16, true>(head_dim, go);
+}
+
+int attention_ctas_per_sm(int head_dim, int group, int batch, bool step) {
   int n = 0;
-  dispatch<__nv_bfloat16>(head_dim, [&](auto inst) {
-    n = decltype(inst)::ctas_per_sm(batch);
+  auto q = [&](auto inst) {
+    n = decltype(inst)::ctas_per_sm(group, batch);
     return cudaSuccess;
-  });
+  };
+  if (step) dispatch<__nv_bfloat16, true>(head_dim, q);
+  else dispatch<__nv_bfloat16, false>(head_dim, q);
   return n;
 }
 

@@ -40,6 +40,26 @@ __host__ __device__ inline int32_t chunks_of(int32_t slots) {
 }
 
 // Everything one attention launch needs; all pointers are device pointers.
+// Extra inputs when the attention launch also performs this macro-step's append (the
+// fused decode step): the attention CTAs use the new slot and the rotated q from shared
+// memory, and the combine kernel commits the slot, q and the counters after the grid.
+struct StepArgs {
+  const uint16_t *k_new, *v_new;   // [batch][n_kv_heads][head_dim]
+  uint16_t *q_inout;               // [batch][n_q_heads][head_dim], rotated in place by combine
+  const int32_t *pos;              // nullable [batch]
+  const int32_t *ntok;             // [batch]
+  int32_t *num_slots;              // [batch] of this layer (written by combine only)
+  int64_t *num_tokens;             // [batch] of this layer
+  int32_t *slot_pos, *slot_ntok;
+  uint16_t *k_pool, *v_pool;       // this layer, written by combine
+  const double *inv_freq;          // [head_dim / 2]
+  const double2 *rope_table;       // [rope_positions][head_dim / 2] (cos, sin)
+  const float2 *rope_table_f;      // same, fp32
+  int64_t rope_positions;
+  int4 *stash;                     // scratch [batch]: (slot n, 0 or HAM_DEVERR_*, position, ntok)
+  int32_t pos_mode;
+};
+
 struct AttnView {
   const uint16_t *k_pool;      // this layer: [pool_pages][n_kv_heads][page_slots][head_dim]
   const uint16_t *v_pool;
@@ -55,6 +75,7 @@ struct AttnView {
   int64_t pool_pages;
   int32_t batch, n_kv_heads, group, page_slots, max_pages, max_slots;
   int32_t ctas;
+  StepArgs step;               // used by launch_decode_step only
 };
 
 struct AppendView {
@@ -64,6 +85,8 @@ struct AppendView {
   int32_t *num_slots;          // [batch] of this layer
   int64_t *num_tokens;         // [batch] of this layer
   const double *inv_freq;      // [head_dim / 2]: base^(-2i/d)
+  const double2 *rope_table;   // [rope_positions][head_dim / 2]: (cos, sin)(p * inv_freq[i])
+  int64_t rope_positions;      // positions covered by rope_table (others use sincos)
   uint16_t *q;                 // nullable
   const uint16_t *k_new, *v_new;
   const int32_t *pos;          // nullable
@@ -91,8 +114,11 @@ struct FillView {
 // tk / tv: TMA maps of the layer's K and V pools (make_pool_tensor_map).
 cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
                              int head_dim, int out_dtype, cudaStream_t stream);
+// Fused decode step: append (v.step) + attention + combine/commit.
+cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
+                               int head_dim, int out_dtype, cudaStream_t stream);
 // CTAs of one SM for the attention kernel of this shape (0 if the shape is not compiled).
-int attention_ctas_per_sm(int head_dim, int batch);
+int attention_ctas_per_sm(int head_dim, int group, int batch, bool step);
 bool attention_supported(int head_dim, int group);
 // TMA map of one pool [pool_pages][n_kv_heads][page_slots][head_dim] bf16 viewed as
 // {64 elements, head_dim / 64, rows} with a box of {64, head_dim / 64, 16 rows} and the
@@ -121,6 +147,7 @@ struct ham_kv {
   int32_t max_pages = 0;
   int32_t attn_ctas = 0;        // 0: default
   int32_t default_ctas = 0;     // SMs x resident attention CTAs per SM (set at allocation)
+  int32_t default_step_ctas = 0;  // same for the fused decode step
   int32_t max_ctas = 0;         // scratch is sized for this many CTAs
   int64_t pool_elems = 0;       // bf16 elements of ONE pool (K or V) of one layer
   uint16_t *pool = nullptr;     // [layers][2][pool_elems]
@@ -129,6 +156,10 @@ struct ham_kv {
   int32_t *num_slots = nullptr; // [layers][batch]
   int64_t *num_tokens = nullptr;
   double *inv_freq = nullptr;
+  double2 *rope_table = nullptr;  // own allocation
+  float2 *rope_table_f = nullptr;  // own allocation
+  int64_t rope_positions = 0;
+  int4 *stash = nullptr;           // fused step: per-sequence append record
   int32_t *err = nullptr;
   float *part_acc = nullptr;
   float2 *part_ml = nullptr;

@@ -79,7 +79,7 @@ int ham_decode_attn_noalloc(const ham_attn_args *a, void *stream) {
 
   int ctas = a->ctas;
   if (ctas == 0) {
-    const int per_sm = ham::attention_ctas_per_sm(a->head_dim, a->batch);
+    const int per_sm = ham::attention_ctas_per_sm(a->head_dim, group, a->batch, false);
     if (per_sm <= 0) return noalloc_fail(HAM_ECUDA, "attention kernel cannot be resident");
     ctas = setup.num_sms * per_sm;
   }

@@ -279,15 +279,18 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   const size_t o_acc = carve(n_part * group * cfg.head_dim * sizeof(float));
   const size_t o_ml = carve(n_part * group * sizeof(float2));
   const size_t o_sr = carve(n_seg * sizeof(int2));
+  const size_t o_stash = carve((size_t)cfg.batch * sizeof(int4));
   kv->scratch_bytes = (int64_t)(off - o_acc);
 
   {
-    const int per_sm = ham::attention_ctas_per_sm(cfg.head_dim, cfg.batch);
-    if (per_sm <= 0) {
+    const int per_sm = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, false);
+    const int per_sm_step = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, true);
+    if (per_sm <= 0 || per_sm_step <= 0) {
       delete kv;
       return fail(HAM_ECUDA, "attention kernel cannot be resident on an SM");
     }
     kv->default_ctas = std::min(sms * per_sm, kv->max_ctas);
+    kv->default_step_ctas = std::min(sms * per_sm_step, kv->max_ctas);
   }
   cudaError_t e = cudaMalloc(&kv->pool, pool_bytes);
   if (e != cudaSuccess) {
@@ -312,6 +315,7 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->part_acc = reinterpret_cast<float *>(kv->meta + o_acc);
   kv->part_ml = reinterpret_cast<float2 *>(kv->meta + o_ml);
   kv->seg_range = reinterpret_cast<int2 *>(kv->meta + o_sr);
+  kv->stash = reinterpret_cast<int4 *>(kv->meta + o_stash);
 
   // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits.
   e = cudaMemset(kv->pool, 0, pool_bytes);
@@ -326,6 +330,31 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   if (e == cudaSuccess)
     e = cudaMemcpy(kv->inv_freq, inv_freq.data(), inv_freq.size() * sizeof(double),
                    cudaMemcpyHostToDevice);
+  // (cos, sin) of p * inv_freq[i] for every position a sequence can reach by slot index (or
+  // ~4 tokens per slot), capped at 64 MiB; the append kernel falls back to sincos beyond.
+  if (e == cudaSuccess) {
+    const int64_t half = cfg.head_dim / 2;
+    const int64_t reach = (int64_t)cfg.max_slots_per_seq * (cfg.pos_mode == HAM_POS_TOKEN ? 4 : 1);
+    const int64_t cap = (int64_t)(64u << 20) / (half * (int64_t)sizeof(double2));
+    kv->rope_positions = std::min(reach, cap);
+    std::vector<double2> table((size_t)(kv->rope_positions * half));
+    std::vector<float2> table_f(table.size());
+    for (int64_t p = 0; p < kv->rope_positions; ++p)
+      for (int64_t i = 0; i < half; ++i) {
+        const double theta = (double)p * inv_freq[(size_t)i];
+        const double c = cos(theta), s = sin(theta);
+        table[(size_t)(p * half + i)] = make_double2(c, s);
+        table_f[(size_t)(p * half + i)] = make_float2((float)c, (float)s);
+      }
+    e = cudaMalloc(&kv->rope_table, table.size() * sizeof(double2));
+    if (e == cudaSuccess)
+      e = cudaMemcpy(kv->rope_table, table.data(), table.size() * sizeof(double2),
+                     cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMalloc(&kv->rope_table_f, table_f.size() * sizeof(float2));
+    if (e == cudaSuccess)
+      e = cudaMemcpy(kv->rope_table_f, table_f.data(), table_f.size() * sizeof(float2),
+                     cudaMemcpyHostToDevice);
+  }
   if (e != cudaSuccess) {
     int rc = cuda_fail(e, "initialising the cache");
     ham_kv_free(kv);
@@ -353,6 +382,8 @@ int ham_kv_free(ham_kv *kv) {
   cudaDeviceSynchronize();
   if (kv->pool) cudaFree(kv->pool);
   if (kv->meta) cudaFree(kv->meta);
+  if (kv->rope_table) cudaFree(kv->rope_table);
+  if (kv->rope_table_f) cudaFree(kv->rope_table_f);
   if (kv->host_stage) cudaFreeHost(kv->host_stage);
   delete kv;
   return HAM_OK;
@@ -398,6 +429,8 @@ int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
   v.num_slots = kv->num_slots + (size_t)layer * kv->cfg.batch;
   v.num_tokens = kv->num_tokens + (size_t)layer * kv->cfg.batch;
   v.inv_freq = kv->inv_freq;
+  v.rope_table = kv->rope_table;
+  v.rope_positions = kv->rope_positions;
   v.q = static_cast<uint16_t *>(q_inout);
   v.k_new = static_cast<const uint16_t *>(k_new);
   v.v_new = static_cast<const uint16_t *>(v_new);
@@ -453,6 +486,72 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
                                         v, kv->cfg.head_dim, out_dtype,
                                         static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+  return HAM_OK;
+}
+
+int ham_decode_step(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
+                    const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
+                    int32_t out_dtype, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!q_inout || !k_new || !v_new || !ntok || !out)
+    return fail(HAM_EINVAL, "q_inout, k_new, v_new, ntok and out are required");
+  if (!aligned16(q_inout) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out))
+    return fail(HAM_EINVAL, "q/k/v/out must be 16-byte aligned");
+  if (((uintptr_t)ntok & 3u) || ((uintptr_t)pos & 3u))
+    return fail(HAM_EINVAL, "pos/ntok must be 4-byte aligned");
+  if (out_dtype != HAM_DTYPE_BF16 && out_dtype != HAM_DTYPE_F32)
+    return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
+  const ham_config &c = kv->cfg;
+  const int group = c.n_q_heads / c.n_kv_heads;
+  {  // q_inout is rewritten while out is being written: they must not overlap
+    const uintptr_t q0 = (uintptr_t)q_inout, o0 = (uintptr_t)out;
+    const uintptr_t n = (uintptr_t)c.batch * c.n_q_heads * c.head_dim;
+    const uintptr_t q1 = q0 + n * 2, o1 = o0 + n * (out_dtype == HAM_DTYPE_F32 ? 4 : 2);
+    if (q0 < o1 && o0 < q1) return fail(HAM_EINVAL, "out overlaps q_inout");
+  }
+  DeviceGuard guard(kv->device);
+  ham::AttnView v{};
+  v.k_pool = layer_pool(kv, layer, 0);
+  v.v_pool = layer_pool(kv, layer, 1);
+  v.page_table = kv->page_table;
+  v.num_slots = kv->num_slots + (size_t)layer * c.batch;
+  v.q = static_cast<const uint16_t *>(q_inout);
+  v.out = out;
+  v.part_acc = kv->part_acc;
+  v.part_ml = kv->part_ml;
+  v.seg_range = kv->seg_range;
+  v.err = kv->err;
+  v.pool_pages = c.pool_pages;
+  v.batch = c.batch;
+  v.n_kv_heads = c.n_kv_heads;
+  v.group = group;
+  v.page_slots = c.page_slots;
+  v.max_pages = kv->max_pages;
+  v.max_slots = c.max_slots_per_seq;
+  v.ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->default_step_ctas;
+  ham::StepArgs &st = v.step;
+  st.k_new = static_cast<const uint16_t *>(k_new);
+  st.v_new = static_cast<const uint16_t *>(v_new);
+  st.q_inout = static_cast<uint16_t *>(q_inout);
+  st.pos = pos;
+  st.ntok = ntok;
+  st.num_slots = kv->num_slots + (size_t)layer * c.batch;
+  st.num_tokens = kv->num_tokens + (size_t)layer * c.batch;
+  st.slot_pos = kv->slot_pos;
+  st.slot_ntok = kv->slot_ntok;
+  st.k_pool = layer_pool(kv, layer, 0);
+  st.v_pool = layer_pool(kv, layer, 1);
+  st.inv_freq = kv->inv_freq;
+  st.rope_table = kv->rope_table;
+  st.rope_table_f = kv->rope_table_f;
+  st.rope_positions = kv->rope_positions;
+  st.stash = kv->stash;
+  st.pos_mode = c.pos_mode;
+  cudaError_t e = ham::launch_decode_step(kv->tmaps[(size_t)layer * 2],
+                                          kv->tmaps[(size_t)layer * 2 + 1], v, c.head_dim,
+                                          out_dtype, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "decode step launch");
   return HAM_OK;
 }
 

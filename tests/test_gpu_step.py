@@ -1,0 +1,202 @@
+"""GPU: the fused decode step (append + attention in one pass over the cache).
+
+The cache, the counters and the rotated q it leaves are compared bit for bit with the
+oracle's append; its attention output with the oracle's attention over the n + 1 slots.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2505_20438_gb300 import ham
+from paper_2505_20438_gb300 import workload as wl
+
+from gpu_helpers import (MAX_ABS, MEAN_ABS, assert_parity, dev_bf16, dev_i32, gpu_cache,
+                         host_bits, small_case, torch)
+
+pytestmark = pytest.mark.gpu
+
+# Against the oracle: the tensor-core pass rounds each softmax weight to bf16 (relative
+# error <= 2^-9), which moves an output by at most 2^-9 * max|v_i - v_j| (~1.6e-2 for unit
+# normal values); on sequences of a few slots nothing averages it out, so the bar is the
+# bf16 one (MAX_ABS, MEAN_ABS) even with fp32 output.  GPU against GPU with the same split:
+# the same weights are rounded the same way, so only a rare one-ulp difference of an
+# fp32-rotated q or k element separates the fused step from the two separate calls.
+SAME_SPLIT_MAX, SAME_SPLIT_MEAN = 2e-3, 2e-5
+
+
+def _export_host(kv, layer=0):
+    k, v, pos, ntok = ham.ham_kv_export(kv, layer)
+    return host_bits(k), host_bits(v), pos.cpu().numpy(), ntok.cpu().numpy()
+
+
+def _assert_cache_equal(kv, oc, layer=0):
+    k, v, pos, ntok = _export_host(kv, layer)
+    assert np.array_equal(v, oc.v_pool), "V pool"
+    assert np.array_equal(k, oc.k_pool), "K pool (RoPE'd keys)"
+    assert np.array_equal(pos, oc.slot_pos) and np.array_equal(ntok, oc.slot_ntok)
+    slots, tokens = ham.ham_kv_layer_lengths(kv, layer)
+    assert np.array_equal(slots, oc.num_slots) and np.array_equal(tokens, oc.num_tokens)
+
+
+def _step(kv, q_dev, k_new, v_new, ntok, pos=None, f32=True, layer=0):
+    t = torch()
+    out = t.full(q_dev.shape, float("nan"), dtype=t.float32 if f32 else t.bfloat16,
+                 device="cuda")
+    ham.ham_decode_step(kv, layer, q_dev, dev_bf16(k_new), dev_bf16(v_new),
+                        None if pos is None else dev_i32(pos), dev_i32(ntok), out)
+    t.cuda.synchronize()
+    return out.float().cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("pos_mode", [ham.HAM_POS_SLOT, ham.HAM_POS_TOKEN])
+@pytest.mark.parametrize("d,hq,hkv,page,counts", [
+    (64, 8, 2, 16, (15, 16, 0, 47)),       # new slot ends chunk 0 / opens chunk 1 / first
+    (128, 32, 8, 32, (31, 200, 5)),        # page edge; Llama-3 8B head layout
+    (128, 8, 8, 16, (1, 64)),              # group 1
+    (64, 16, 2, 128, (127, 300)),          # group 8
+])
+def test_step_matches_oracle(pos_mode, d, hq, hkv, page, counts):
+    case = small_case(batch=len(counts), hq=hq, hkv=hkv, d=d, page=page, counts=counts,
+                      seed=11, extra_slots=8)
+    oc = oracle.OracleCache.from_case(case)
+    kv = gpu_cache(case, pos_mode=pos_mode)
+    q_host = case.q.copy()
+    q_dev = dev_bf16(case.q)
+    rng = wl.rng_for(11, 60)
+    for step in range(3):
+        k_new = wl.normal_bf16(rng, case.k_new.shape)
+        v_new = wl.normal_bf16(rng, case.v_new.shape)
+        ntok = wl.ntok_capped_geometric(rng, (case.w.batch,))
+        assert oc.append(k_new, v_new, ntok, q_inout=q_host, pos_mode=pos_mode) == 0
+        ref = oc.decode_attn(q_host)
+        got = _step(kv, q_dev, k_new, v_new, ntok)
+        assert np.array_equal(host_bits(q_dev), q_host), f"q after step {step}"
+        assert_parity(got, ref, MAX_ABS, MEAN_ABS, what=f"step {step}")
+        q_host = wl.normal_bf16(rng, case.q.shape)   # next macro-step's fresh queries
+        q_dev = dev_bf16(q_host)
+    _assert_cache_equal(kv, oc)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+def test_step_equals_append_then_attend_on_gpu():
+    """Same cache bits and q bits as the two separate calls; outputs agree closely."""
+    case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(100, 17, 640), seed=12)
+    kv1, kv2 = gpu_cache(case), gpu_cache(case)
+    for kv in (kv1, kv2):
+        ham.ham_kv_set_attn_ctas(kv, 300)          # the same split for both paths
+    q1, q2 = dev_bf16(case.q), dev_bf16(case.q)
+    t = torch()
+    out1 = t.empty(q1.shape, dtype=t.float32, device="cuda")
+    ham.ham_kv_append(kv1, 0, q1, dev_bf16(case.k_new), dev_bf16(case.v_new), None,
+                      dev_i32(case.ntok_new))
+    ham.ham_decode_attn_ex(kv1, 0, q1, out1)
+    out2 = _step(kv2, q2, case.k_new, case.v_new, case.ntok_new)
+    assert np.array_equal(host_bits(q1), host_bits(q2))
+    a, b = _export_host(kv1), _export_host(kv2)
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y)
+    assert_parity(out2, out1.cpu().numpy().astype(np.float64), SAME_SPLIT_MAX, SAME_SPLIT_MEAN,
+                  what="2-call")
+
+
+def test_step_positions_beyond_the_rope_table():
+    """Explicit positions up to ~2.6e5 take the sincos path in both kernels."""
+    case = small_case(batch=4, hq=32, hkv=8, d=128, page=16, counts=(3, 40, 0, 16), seed=13)
+    oc = oracle.OracleCache.from_case(case)
+    kv = gpu_cache(case)
+    pos = np.array([0, 4095, 131071, 262143], np.int32)
+    q_host = case.q.copy()
+    q_dev = dev_bf16(case.q)
+    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_host, pos=pos) == 0
+    ref = oc.decode_attn(q_host)
+    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new, pos=pos)
+    assert np.array_equal(host_bits(q_dev), q_host)
+    assert_parity(got, ref, MAX_ABS, MEAN_ABS, what="large positions")
+    _assert_cache_equal(kv, oc)
+
+
+@pytest.mark.parametrize("ctas", [1, 5, 37, 600])
+def test_step_split_counts(ctas):
+    """Any CTA count: identical cache and q, attention within tolerance."""
+    case = small_case(batch=3, hq=8, hkv=2, d=64, page=16, counts=(0, 333, 48), seed=14)
+    oc = oracle.OracleCache.from_case(case)
+    kv = gpu_cache(case)
+    ham.ham_kv_set_attn_ctas(kv, ctas)
+    q_host = case.q.copy()
+    q_dev = dev_bf16(case.q)
+    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_host) == 0
+    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new)
+    assert np.array_equal(host_bits(q_dev), q_host)
+    assert_parity(got, oc.decode_attn(q_host), MAX_ABS, MEAN_ABS, what=f"ctas={ctas}")
+    _assert_cache_equal(kv, oc)
+
+
+def test_step_failed_appends_behave_like_the_two_calls():
+    """A full sequence and ntok = 0: no append, q untouched, old slots attended, error set."""
+    case = small_case(batch=3, hq=8, hkv=2, d=64, page=16, counts=(20, 37, 9), seed=15,
+                      extra_slots=0)
+    oc = oracle.OracleCache.from_case(case)
+    assert case.max_slots == 37                    # sequence 1 is full
+    kv = gpu_cache(case)
+    ntok = np.array([2, 1, 0], np.int32)           # sequence 2 gives ntok = 0
+    q_host = case.q.copy()
+    q_dev = dev_bf16(case.q)
+    assert oc.append(case.k_new, case.v_new, ntok, q_inout=q_host) != 0
+    ref = oc.decode_attn(q_host)
+    got = _step(kv, q_dev, case.k_new, case.v_new, ntok)
+    assert np.array_equal(host_bits(q_dev), q_host)
+    assert np.array_equal(host_bits(q_dev)[1:], case.q[1:])   # untouched where skipped
+    assert_parity(got, ref, MAX_ABS, MEAN_ABS, what="failed appends")
+    # read (and clear) the error word first: the counter read-back refuses while it is set
+    assert ham.ham_kv_status(kv) in (ham.HAM_DEVERR_CAPACITY, ham.HAM_DEVERR_NTOK)
+    _assert_cache_equal(kv, oc)
+
+
+def test_step_host_errors():
+    case = small_case(batch=2, counts=(3, 4), seed=16)
+    kv = gpu_cache(case)
+    t = torch()
+    q = dev_bf16(case.q)
+    k, v, n = dev_bf16(case.k_new), dev_bf16(case.v_new), dev_i32(case.ntok_new)
+    out = t.empty(q.shape, dtype=t.bfloat16, device="cuda")
+    with pytest.raises(ham.HamError):
+        ham.ham_decode_step(kv, 1, q, k, v, None, n, out)          # layer out of range
+    with pytest.raises(ham.HamError):
+        ham.ham_decode_step(kv, 0, q, k, v, None, n, q)             # out aliases q_inout
+    rc = ham.lib().ham_decode_step(kv, 0, q.data_ptr() + 2, k.data_ptr(), v.data_ptr(), None,
+                                   n.data_ptr(), out.data_ptr(), ham.HAM_DTYPE_BF16, None)
+    assert rc == ham.HAM_EINVAL
+    t.cuda.synchronize()
+    slots, _ = ham.ham_slot_lengths(kv)
+    assert list(slots) == [3, 4]                   # nothing launched
+
+
+def test_step_then_attention_sees_the_slot():
+    """After a step, plain attention with the same q reproduces the step's output."""
+    case = small_case(batch=2, hq=32, hkv=8, d=128, page=32, counts=(63, 500), seed=17)
+    kv = gpu_cache(case)
+    ham.ham_kv_set_attn_ctas(kv, 200)
+    q_dev = dev_bf16(case.q)
+    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new)
+    t = torch()
+    again = t.empty(q_dev.shape, dtype=t.float32, device="cuda")
+    ham.ham_decode_attn_ex(kv, 0, q_dev, again)
+    assert_parity(got, again.cpu().numpy().astype(np.float64), SAME_SPLIT_MAX, SAME_SPLIT_MEAN,
+                  what="step vs attention after it")
+
+
+@pytest.mark.parametrize("w", [wl.C1_LLAMA8B, wl.C2_RAGGED], ids=lambda w: w.name)
+def test_step_full_size(w):
+    """The bench's workloads and launch configuration (default CTAs, bf16 output)."""
+    case = wl.make_case(w, extra_slots=4)
+    oc = oracle.OracleCache.from_case(case)
+    kv = gpu_cache(case)
+    q_host = case.q.copy()
+    q_dev = dev_bf16(case.q)
+    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_host) == 0
+    ref = oc.decode_attn(q_host)
+    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new, f32=False)
+    assert np.array_equal(host_bits(q_dev), q_host)
+    assert_parity(got, ref, what=w.name)
+    # the appended rows, bit for bit (the whole pool at this size is compared too)
+    _assert_cache_equal(kv, oc)
