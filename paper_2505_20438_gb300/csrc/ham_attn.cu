@@ -730,11 +730,32 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   }
 
   grid_dependency_wait();  // the attention grid's partials, ranges and append records
+  // The next kernel may be scheduled now; its own dependency wait still covers this grid.
+  grid_launch_dependents();
   if constexpr (kStep) __syncthreads();  // every q read above precedes any q write below
 
   const int2 r = v.seg_range[seg];
+  // fused step: the append record, then cos/sin and the page, loaded ahead of the merge so
+  // that both dependent chains are in flight together
   int4 rec = make_int4(0, 0, 0, 0);
-  if constexpr (kStep) rec = v.step.stash[seg / Hkv];  // (n, 0 or error, position, ntok)
+  double c = 1.0, sn = 0.0;
+  int page = -1;
+  if constexpr (kStep) {
+    const StepArgs &st = v.step;
+    const int b = seg / Hkv;
+    rec = st.stash[b];  // (n, 0 or error, position, ntok)
+    if (rec.y == 0 && active) {
+      const int64_t p = rec.z;
+      if (p >= 0 && p < st.rope_positions) {
+        const double2 e = st.rope_table[p * half + i];
+        c = e.x;
+        sn = e.y;
+      } else {
+        sincos((double)p * inv_freq, &sn, &c);
+      }
+      if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
+    }
+  }
 
   if (active && r.x >= 0 && r.x != r.y) {
     // Online merge in batches of 8 partials: the 8 loads of a batch are in flight together.
@@ -778,17 +799,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
     if (!active) return;
     const int n = rec.x;
     const int64_t p = rec.z;
-    double c, sn;
-    if (p >= 0 && p < st.rope_positions) {
-      const double2 e = st.rope_table[p * half + i];
-      c = e.x;
-      sn = e.y;
-    } else {
-      sincos((double)p * inv_freq, &sn, &c);
-    }
     st.q_inout[qrow + d] = rotate_elem(q_self, q_other, c, sn, high);
     if (h != 0) return;
-    const int page = v.page_table[(int64_t)b * v.max_pages + n / v.page_slots];
     if (page < 0 || page >= v.pool_pages) {
       if (lead) record_error(v.err, HAM_DEVERR_PAGE);
       return;

@@ -39,6 +39,19 @@ __host__ __device__ inline int32_t chunks_of(int32_t slots) {
   return (slots + kChunkSlots - 1) / kChunkSlots;
 }
 
+// Default attention grid: at most 4 CTAs per SM even where more would fit.  Four 32 KiB
+// rings per SM keep ~19 MB of copies in flight on 152 SMs, above what HBM needs to stay
+// busy; a fifth CTA per SM measured slower on every workload (more partials, more queueing),
+// and the spare slot lets the combine kernel, scheduled early under programmatic dependent
+// launch, sit beside the next attention grid without pushing one of its CTAs into a second
+// wave (a CTA that starts late doubles the launch: the split plan gives every CTA an equal
+// share).
+constexpr int kDefaultCtasPerSm = 4;
+inline int32_t default_attention_ctas(int32_t num_sms, int32_t resident_per_sm) {
+  const int32_t per = resident_per_sm < kDefaultCtasPerSm ? resident_per_sm : kDefaultCtasPerSm;
+  return num_sms * (per < 1 ? 1 : per);
+}
+
 // Everything one attention launch needs; all pointers are device pointers.
 // Extra inputs when the attention launch also performs this macro-step's append (the
 // fused decode step): the attention CTAs use the new slot and the rotated q from shared

@@ -81,7 +81,7 @@ int ham_decode_attn_noalloc(const ham_attn_args *a, void *stream) {
   if (ctas == 0) {
     const int per_sm = ham::attention_ctas_per_sm(a->head_dim, group, a->batch, false);
     if (per_sm <= 0) return noalloc_fail(HAM_ECUDA, "attention kernel cannot be resident");
-    ctas = setup.num_sms * per_sm;
+    ctas = ham::default_attention_ctas(setup.num_sms, per_sm);
   }
   // scratch: partial (acc, max/sum) for each (CTA, segment) incidence, then segment ranges
   const size_t n_seg = (size_t)a->batch * a->n_kv_heads;

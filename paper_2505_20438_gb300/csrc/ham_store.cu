@@ -289,8 +289,8 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
       delete kv;
       return fail(HAM_ECUDA, "attention kernel cannot be resident on an SM");
     }
-    kv->default_ctas = std::min(sms * per_sm, kv->max_ctas);
-    kv->default_step_ctas = std::min(sms * per_sm_step, kv->max_ctas);
+    kv->default_ctas = std::min(ham::default_attention_ctas(sms, per_sm), kv->max_ctas);
+    kv->default_step_ctas = std::min(ham::default_attention_ctas(sms, per_sm_step), kv->max_ctas);
   }
   cudaError_t e = cudaMalloc(&kv->pool, pool_bytes);
   if (e != cudaSuccess) {
