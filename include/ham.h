@@ -225,8 +225,8 @@ int ham_kv_set_lengths(ham_kv *kv, int32_t layer, const int32_t *num_slots,
 /* Set every sequence of every layer back to 0 slots / 0 tokens (pages stay reserved). */
 int ham_kv_reset(ham_kv *kv, void *stream);
 
-/* Number of CTAs one attention launch uses (0 = default: SMs x resident CTAs per SM).
- * Range 1 .. 8 x SMs.  Any value gives the same result up to fp32 summation order. */
+/* Number of CTAs one attention launch uses (0 = default: SMs x min(4, resident CTAs per
+ * SM)).  Range 1 .. 8 x SMs.  Any value gives the same result up to fp32 summation order. */
 int ham_kv_set_attn_ctas(ham_kv *kv, int32_t ctas);
 
 /* Host evaluation of the split plan the attention kernel uses (no GPU needed).  Chunks are
