@@ -143,20 +143,25 @@ int ham_decode_attn(ham_kv *kv, int32_t layer, const void *q, void *out, void *s
 
 /* ham_kv_append followed by ham_decode_attn in one pass over the cache (Sec. 3.1 + Sec. 3.4:
  * the macro-step's slot is stored and every query head then attends over the slot list
- * that includes it).  Same arguments and meaning as those two calls, with q_inout required:
- * on return the cache, the counters and q_inout hold exactly what ham_kv_append leaves
- * (fp64 RoPE, bf16 round-to-nearest-even), and out holds the attention of the rotated q
- * over the n + 1 slots.  Inside the attention pass, q and the new key are rotated in fp32
- * from a float cos/sin table, so a rotated element can differ from the stored one by one
- * bf16 ulp; out stays within the ham_decode_attn tolerance of the two-call result.
- * A sequence whose append fails (full, ntok < 1, bad counter) is not appended, keeps its
- * unrotated q, attends over its old slots and sets the device error word, as the two calls
+ * that includes it).  q is the UNROTATED query; the step turns it by the new slot's
+ * position internally and never writes it.  On return the cache and the counters hold
+ * exactly what ham_kv_append leaves (fp64 RoPE, bf16 round-to-nearest-even), and out holds
+ * the attention of RoPE(q) over the n + 1 slots.  Inside the attention pass q and the new
+ * key are turned in fp32 from a float cos/sin table, so a rotated element can differ from
+ * the stored one by one bf16 ulp; out stays within the ham_decode_attn tolerance of the
+ * two-call result.  q_rot (nullable) receives the fp64-exact RoPE(q), the bits
+ * ham_kv_append would leave in q_inout, for the sequences whose append happens (other rows
+ * are not written).
+ * A sequence whose append fails (full, ntok < 1, bad counter) is not appended, attends with
+ * its unrotated q over its old slots and sets the device error word, as the two calls
  * would.  Two launches on `stream` (the second with programmatic dependent launch).
- * out      device [batch][n_q_heads][head_dim], bf16 or f32 (out_dtype); must not overlap
- *          q_inout.  k_new / v_new must not overlap the cache.
+ * q        device bf16 [batch][n_q_heads][head_dim];  q_rot nullable, same shape
+ * k_new, v_new, pos, ntok as for ham_kv_append
+ * out      device [batch][n_q_heads][head_dim], bf16 or f32 (out_dtype)
+ * q, q_rot and out must not overlap; k_new and v_new must not overlap the cache.
  * Host errors: HAM_EINVAL (NULL / unaligned / overlapping pointers, layer out of range,
  * out_dtype), HAM_ECUDA.  Same serialization rule as ham_decode_attn. */
-int ham_decode_step(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
+int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const void *k_new,
                     const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
                     int32_t out_dtype, void *stream);
 

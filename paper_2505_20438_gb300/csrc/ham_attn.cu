@@ -252,6 +252,33 @@ __device__ __forceinline__ uint32_t tile_offset(int slot, int c) {
 __device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {
   return __uint_as_float((uint32_t)b << 16);
 }
+__device__ __forceinline__ double bf16_bits_to_double(uint16_t b) {
+  return (double)__uint_as_float((uint32_t)b << 16);
+}
+
+// One element of the rotated pair (i, i + D/2), rounded once to bf16: y_i = x_i c - x_{i+D/2} s
+// for the low half, y_{i+D/2} = x_{i+D/2} c + x_i s for the high half (explicit fp64
+// operations, no FMA: the textbook formula as ham_kv_append evaluates it).
+__device__ __forceinline__ uint16_t rotate_elem(double self, double other, double c, double s,
+                                                bool high) {
+  const double y = high ? __dadd_rn(__dmul_rn(self, c), __dmul_rn(other, s))
+                        : __dsub_rn(__dmul_rn(self, c), __dmul_rn(other, s));
+  return __bfloat16_as_ushort(__double2bfloat16(y));
+}
+
+// Positions past the fp32 (cos, sin) table: the consumer warp fills the segment's row in
+// shared memory itself (fp64 sincos rounded to fp32, two entries per lane at d = 128), so
+// that the rotations below always read the row.  A bulk copy may later reuse the buffer.
+__device__ __forceinline__ void fill_cs_row(float2 *cs_row, int64_t p, const double *inv_freq,
+                                            int half, int lane) {
+  for (int i = lane; i < half; i += 32) {
+    double sd, cd;
+    sincos((double)p * inv_freq[i], &sd, &cd);
+    cs_row[i] = make_float2((float)cd, (float)sd);
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+}
 
 // Position of the slot a fused step appends to sequence b (slot index n or tokens so far,
 // unless given).
@@ -492,37 +519,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     const int4 inf = info[stage];
     if (inf.z & kFirst) {  // Q^T fragments of a new segment (heads >= G are zero)
       cur_qb = inf.w;
-      uint16_t *q = reinterpret_cast<uint16_t *>(qbufs + cur_qb * sb.stride);
-      const int b = inf.x / Hkv;
-      if (kStep && appb[b]) {
-        // Turn q and the new key by the new slot's position (fp32 from the fp32 table; the
-        // exact fp64 rotation is committed by the combine kernel).  Lane handles pairs
-        // (i, i + D/2) for i = lane (+ 32).
-        const int64_t p = posb[b];
-        const bool tabled = p >= 0 && p < v.step.rope_positions;
-        const float2 *cs = reinterpret_cast<const float2 *>(qbufs + cur_qb * sb.stride + sb.cs_off());
-        uint16_t *kn = reinterpret_cast<uint16_t *>(qbufs + cur_qb * sb.stride + sb.k_off());
-        for (int i = lane; i < D / 2; i += 32) {
-          float c, s;
-          if (tabled) {
-            c = cs[i].x;
-            s = cs[i].y;
-          } else {
-            double sd, cd;
-            sincos((double)p * v.step.inv_freq[i], &sd, &cd);
-            c = (float)cd;
-            s = (float)sd;
-          }
-          for (int h = 0; h <= G; ++h) {  // G query heads, then the key
-            uint16_t *row = h < G ? q + h * D : kn;
-            const float x0 = bf16_bits_to_float(row[i]), x1 = bf16_bits_to_float(row[i + D / 2]);
-            row[i] = __bfloat16_as_ushort(__float2bfloat16_rn(x0 * c - x1 * s));
-            row[i + D / 2] = __bfloat16_as_ushort(__float2bfloat16_rn(x1 * c + x0 * s));
-          }
-        }
-        fence_proxy_async_smem();  // these writes vs a later bulk copy into this buffer
-        __syncwarp();
-      }
+      const uint16_t *q = reinterpret_cast<const uint16_t *>(qbufs + cur_qb * sb.stride);
 #pragma unroll
       for (int t = 0; t < S::kSteps; ++t) {
         if (r0 < G) {
@@ -530,6 +527,34 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
           qb[t][1] = *reinterpret_cast<const uint32_t *>(q + r0 * D + 16 * t + 8 + 2 * cq);
         } else {
           qb[t][0] = qb[t][1] = 0u;
+        }
+      }
+      if constexpr (kStep) {
+        const int b = inf.x / Hkv;
+        float2 *cs = reinterpret_cast<float2 *>(qbufs + cur_qb * sb.stride + sb.cs_off());
+        if (appb[b]) {
+          const int64_t p = posb[b];
+          if (!(p >= 0 && p < v.step.rope_positions))
+            fill_cs_row(cs, p, v.step.inv_freq, D / 2, lane);
+        }
+        if (appb[b] && r0 < G) {
+          // Turn this lane's q elements by the new slot's position, in registers (fp32; the
+          // exact fp64 rotation goes to the cache and q_rot).  Fragment t holds columns
+          // 16t + 2cq + {0, 1} and 16t + 8 + 2cq + {0, 1}; the partner of column j < D/2 is
+          // j + D/2, the same place of fragment t + kSteps/2.
+#pragma unroll
+          for (int t = 0; t < S::kSteps / 2; ++t) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int j = 16 * t + 8 * e + 2 * cq;
+              const uint32_t lo = qb[t][e], hi = qb[t + S::kSteps / 2][e];
+              const float a0 = __uint_as_float(lo << 16), a1 = __uint_as_float(lo & 0xFFFF0000u);
+              const float b0 = __uint_as_float(hi << 16), b1 = __uint_as_float(hi & 0xFFFF0000u);
+              const float2 c0 = cs[j], c1 = cs[j + 1];
+              qb[t][e] = pack_bf16x2(a0 * c0.x - b0 * c0.y, a1 * c1.x - b1 * c1.y);
+              qb[t + S::kSteps / 2][e] = pack_bf16x2(b0 * c0.x + a0 * c0.y, b1 * c1.x + a1 * c1.y);
+            }
+          }
         }
       }
     }
@@ -545,13 +570,24 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
         }
       }
       if (kStep && (inf.z & kNewRow)) {  // the appended slot is the chunk's last valid row
+        // its key, turned in fp32 by the new position, and its value, from the segment's
+        // staging buffer (the copy of the row in HBM may not be written yet)
         const uint8_t *seg = qbufs + cur_qb * sb.stride;
-        for (int i = lane; i < 2 * (D / 8); i += 32) {
-          const int c = i % (D / 8);
-          const bool is_v = i >= D / 8;
-          const uint4 x = *reinterpret_cast<const uint4 *>(seg + (is_v ? sb.v_off() : sb.k_off()) + c * 16);
-          *reinterpret_cast<uint4 *>((is_v ? vt : kt) + tile_offset<D>(nvalid - 1, c)) = x;
+        const uint16_t *kn = reinterpret_cast<const uint16_t *>(seg + sb.k_off());
+        const float2 *cs = reinterpret_cast<const float2 *>(seg + sb.cs_off());
+        const int row = nvalid - 1;
+        for (int i = lane; i < D / 2; i += 32) {
+          const float2 cx = cs[i];
+          const float x0 = bf16_bits_to_float(kn[i]), x1 = bf16_bits_to_float(kn[i + D / 2]);
+          const int i1 = i + D / 2;
+          *reinterpret_cast<__nv_bfloat16 *>(kt + tile_offset<D>(row, i >> 3) + (i & 7) * 2) =
+              __float2bfloat16_rn(x0 * cx.x - x1 * cx.y);
+          *reinterpret_cast<__nv_bfloat16 *>(kt + tile_offset<D>(row, i1 >> 3) + (i1 & 7) * 2) =
+              __float2bfloat16_rn(x1 * cx.x + x0 * cx.y);
         }
+        for (int c = lane; c < D / 8; c += 32)
+          *reinterpret_cast<uint4 *>(vt + tile_offset<D>(row, c)) =
+              *reinterpret_cast<const uint4 *>(seg + sb.v_off() + c * 16);
       }
       if (patch) __syncwarp();
       const uint32_t kbase = smem_u32(kt), vbase = smem_u32(vt);
@@ -673,119 +709,107 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
 // ------------------------------------------------------------------------------------
 // Combine: out[seg][h][d] = sum_k 2^(m_k - M) acc_k[h][d] / sum_k 2^(m_k - M) l_k over the
 // CTAs k = first..last of the segment, M = max_k m_k (split-softmax merge, in CTA order).
-// One thread per output element; blocks of kCombineThreads cover one segment's G*D values
-// (whole heads: kCombineThreads is a multiple of head_dim).
+// One thread per pair of elements (h, i) and (h, i + D/2) of an output row: both share the
+// head's (max, sum), and for the fused step they are the pair that RoPE turns together.
+// Blocks of kCombineThreads cover one segment's G*D/2 pairs (whole heads).
 //
-// For the fused step the same threads also commit the append once the whole attention grid
-// has finished (nothing may change q_inout or the counters while it still reads them):
-// element (h, d) of q_inout and, for h = 0, element d of the key and value rows.  Each is
-// the fp64 rotation of the pair (d, d +- D/2) rounded once to bf16, as ham_kv_append does.
-// The inputs that the attention pass only reads are loaded before waiting for it, so the
-// commit's dependent loads (append record -> cos/sin, page) run beside the merge's
-// (segment range -> partials).  KV head 0 writes the slot metadata and counters.
+// For the fused step the same threads also commit the append, once the whole attention grid
+// has finished (every CTA reads the counters in its prologue): thread (h = 0, i) stores
+// elements i and i + D/2 of the new key and value rows, thread (h, i) those of head h of
+// q_rot (if asked), each the fp64 rotation of the pair rounded once to bf16, as
+// ham_kv_append computes it; KV head 0 writes the slot metadata and advances the counters.
+// The commit's chain (append record -> cos/sin and page) and the merge's (segment range ->
+// partials) are issued together.
 // ------------------------------------------------------------------------------------
 constexpr int kCombineThreads = 128;
-static_assert(kCombineThreads % 128 == 0, "a block holds whole heads of head_dim 64 or 128");
-
-__device__ __forceinline__ double bf16_bits_to_double(uint16_t b) {
-  return (double)__uint_as_float((uint32_t)b << 16);
-}
-
-// One element of the rotated pair (i, i + D/2): y_i = x_i c - x_{i+D/2} s for the low half,
-// y_{i+D/2} = x_{i+D/2} c + x_i s for the high half (explicit fp64 operations, no FMA).
-__device__ __forceinline__ uint16_t rotate_elem(double self, double other, double c, double s,
-                                                bool high) {
-  const double y = high ? __dadd_rn(__dmul_rn(self, c), __dmul_rn(other, s))
-                        : __dsub_rn(__dmul_rn(self, c), __dmul_rn(other, s));
-  return __bfloat16_as_ushort(__double2bfloat16(y));
-}
+static_assert(kCombineThreads % 64 == 0, "a block holds whole heads of head_dim 64 or 128");
 
 template <typename OutT, bool kStep>
 __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView v, int D,
                                                                   int blocks_per_seg) {
-  const int G = v.group, Hkv = v.n_kv_heads;
+  const int G = v.group, Hkv = v.n_kv_heads, half = D / 2;
   const int seg = blockIdx.x / blocks_per_seg;
   const int part = blockIdx.x % blocks_per_seg;
-  const int idx = part * kCombineThreads + threadIdx.x;
-  const bool active = idx < G * D;
-  const int h = idx / D, d = idx - h * D;
-
-  // fused step: operands of this thread's commit that the attention pass only reads
-  const int half = D / 2;
-  const bool high = d >= half;
-  const int i = high ? d - half : d, partner = high ? d - half : d + half;
-  double q_self = 0.0, q_other = 0.0, k_self = 0.0, k_other = 0.0, inv_freq = 0.0;
-  uint16_t v_el = 0;
-  const int64_t qrow = (int64_t)seg * G * D + (int64_t)h * D;  // == (b*Hq + g*G + h) * D
-  if (kStep && active) {
-    const StepArgs &st = v.step;
-    q_self = bf16_bits_to_double(st.q_inout[qrow + d]);
-    q_other = bf16_bits_to_double(st.q_inout[qrow + partner]);
-    if (h == 0) {
-      k_self = bf16_bits_to_double(st.k_new[(int64_t)seg * D + d]);
-      k_other = bf16_bits_to_double(st.k_new[(int64_t)seg * D + partner]);
-      v_el = st.v_new[(int64_t)seg * D + d];
-    }
-    inv_freq = st.inv_freq[i];
-  }
+  const int idx = part * kCombineThreads + threadIdx.x;  // pair index within the segment
+  const bool active = idx < G * half;
+  const int h = idx / half, i = idx - h * half;
+  const int64_t orow = ((int64_t)seg * G + h) * D;  // row (b, g*G + h) of q / q_rot / out
 
   grid_dependency_wait();  // the attention grid's partials, ranges and append records
   // The next kernel may be scheduled now; its own dependency wait still covers this grid.
   grid_launch_dependents();
-  if constexpr (kStep) __syncthreads();  // every q read above precedes any q write below
 
   const int2 r = v.seg_range[seg];
-  // fused step: the append record, then cos/sin and the page, loaded ahead of the merge so
-  // that both dependent chains are in flight together
+  // fused step: the append record and this thread's operands, then cos/sin and the page
   int4 rec = make_int4(0, 0, 0, 0);
+  uint16_t q0 = 0, q1 = 0, k0 = 0, k1 = 0, v0 = 0, v1 = 0;
   double c = 1.0, sn = 0.0;
   int page = -1;
   if constexpr (kStep) {
     const StepArgs &st = v.step;
     const int b = seg / Hkv;
-    rec = st.stash[b];  // (n, 0 or error, position, ntok)
-    if (rec.y == 0 && active) {
+    rec = st.stash[b];  // (n, 0 or the error that stops the append, position, ntok)
+    if (active) {
+      if (st.q_rot) {
+        q0 = v.q[orow + i];
+        q1 = v.q[orow + i + half];
+      }
+      if (h == 0) {
+        k0 = st.k_new[(int64_t)seg * D + i];
+        k1 = st.k_new[(int64_t)seg * D + i + half];
+        v0 = st.v_new[(int64_t)seg * D + i];
+        v1 = st.v_new[(int64_t)seg * D + i + half];
+      }
+    }
+    if (rec.y == 0 && active && (h == 0 || st.q_rot)) {
       const int64_t p = rec.z;
       if (p >= 0 && p < st.rope_positions) {
         const double2 e = st.rope_table[p * half + i];
         c = e.x;
         sn = e.y;
       } else {
-        sincos((double)p * inv_freq, &sn, &c);
+        sincos((double)p * st.inv_freq[i], &sn, &c);
       }
       if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
     }
   }
 
   if (active && r.x >= 0 && r.x != r.y) {
-    // Online merge in batches of 8 partials: the 8 loads of a batch are in flight together.
+    // Online merge in batches of 8 partials, whose loads are in flight together.  (16 saved
+    // one round trip at 8-12 partials per segment but cost registers: fewer resident blocks
+    // when a ragged batch has thousands of segments.)
     constexpr int kBatch = 8;
-    float M = -INFINITY, num = 0.f, den = 0.f;
-    for (int k0 = r.x; k0 <= r.y; k0 += kBatch) {
+    float M = -INFINITY, num0 = 0.f, num1 = 0.f, den = 0.f;
+    for (int k0b = r.x; k0b <= r.y; k0b += kBatch) {
       float2 ml[kBatch];
-      float acc[kBatch];
+      float a0[kBatch], a1[kBatch];
 #pragma unroll
       for (int j = 0; j < kBatch; ++j) {
-        const int64_t p = (int64_t)k0 + j + seg;
-        const bool in = k0 + j <= r.y;
+        const int64_t p = (int64_t)k0b + j + seg;
+        const bool in = k0b + j <= r.y;
+        const float *acc = v.part_acc + p * G * D + (int64_t)h * D;
         ml[j] = in ? __ldcg(&v.part_ml[p * G + h]) : make_float2(-INFINITY, 0.f);
-        acc[j] = in ? __ldcg(&v.part_acc[p * G * D + idx]) : 0.f;
+        a0[j] = in ? __ldcg(acc + i) : 0.f;
+        a1[j] = in ? __ldcg(acc + i + half) : 0.f;
       }
       float bm = M;
 #pragma unroll
       for (int j = 0; j < kBatch; ++j) bm = fmaxf(bm, ml[j].x);
       const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
-      num *= scale;
+      num0 *= scale;
+      num1 *= scale;
       den *= scale;
 #pragma unroll
       for (int j = 0; j < kBatch; ++j) {
         const float w = (ml[j].x == -INFINITY) ? 0.f : ex2(ml[j].x - bm);
-        num += w * acc[j];
+        num0 += w * a0[j];
+        num1 += w * a1[j];
         den += w * ml[j].y;
       }
       M = bm;
     }
-    store_out<OutT>(v.out, (int64_t)seg * G * D + idx, num / den);
+    store_out<OutT>(v.out, orow + i, num0 / den);
+    store_out<OutT>(v.out, orow + i + half, num1 / den);
   }
 
   if constexpr (kStep) {
@@ -797,20 +821,26 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       return;
     }
     if (!active) return;
-    const int n = rec.x;
-    const int64_t p = rec.z;
-    st.q_inout[qrow + d] = rotate_elem(q_self, q_other, c, sn, high);
+    if (st.q_rot) {
+      const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
+      st.q_rot[orow + i] = rotate_elem(x0, x1, c, sn, false);
+      st.q_rot[orow + i + half] = rotate_elem(x1, x0, c, sn, true);
+    }
     if (h != 0) return;
-    if (page < 0 || page >= v.pool_pages) {
+    if (page < 0 || page >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE
       if (lead) record_error(v.err, HAM_DEVERR_PAGE);
       return;
     }
+    const int n = rec.x;
     const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
-    st.k_pool[row + d] = rotate_elem(k_self, k_other, c, sn, high);
-    st.v_pool[row + d] = v_el;
+    const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
+    st.k_pool[row + i] = rotate_elem(x0, x1, c, sn, false);
+    st.k_pool[row + i + half] = rotate_elem(x1, x0, c, sn, true);
+    st.v_pool[row + i] = v0;
+    st.v_pool[row + i + half] = v1;
     if (lead) {
       const int64_t meta = (int64_t)page * v.page_slots + n % v.page_slots;
-      st.slot_pos[meta] = (int32_t)p;
+      st.slot_pos[meta] = rec.z;
       st.slot_ntok[meta] = rec.w;
       st.num_slots[b] = n + 1;
       st.num_tokens[b] += rec.w;
@@ -820,7 +850,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
 
 template <typename OutT, bool kStep>
 cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream) {
-  const int per_seg = (v.group * head_dim + kCombineThreads - 1) / kCombineThreads;
+  const int per_seg = (v.group * head_dim / 2 + kCombineThreads - 1) / kCombineThreads;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(v.batch * v.n_kv_heads * per_seg));
   cfg.blockDim = dim3(kCombineThreads);

@@ -58,13 +58,13 @@ inline int32_t default_attention_ctas(int32_t num_sms, int32_t resident_per_sm) 
 // memory, and the combine kernel commits the slot, q and the counters after the grid.
 struct StepArgs {
   const uint16_t *k_new, *v_new;   // [batch][n_kv_heads][head_dim]
-  uint16_t *q_inout;               // [batch][n_q_heads][head_dim], rotated in place by combine
+  uint16_t *q_rot;                 // nullable [batch][n_q_heads][head_dim]: RoPE(q), fp64-exact
   const int32_t *pos;              // nullable [batch]
   const int32_t *ntok;             // [batch]
-  int32_t *num_slots;              // [batch] of this layer (written by combine only)
+  int32_t *num_slots;              // [batch] of this layer (advanced by the combine kernel)
   int64_t *num_tokens;             // [batch] of this layer
   int32_t *slot_pos, *slot_ntok;
-  uint16_t *k_pool, *v_pool;       // this layer, written by combine
+  uint16_t *k_pool, *v_pool;       // this layer (the new slot's rows, written by combine)
   const double *inv_freq;          // [head_dim / 2]
   const double2 *rope_table;       // [rope_positions][head_dim / 2] (cos, sin)
   const float2 *rope_table_f;      // same, fp32
@@ -127,7 +127,7 @@ struct FillView {
 // tk / tv: TMA maps of the layer's K and V pools (make_pool_tensor_map).
 cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
                              int head_dim, int out_dtype, cudaStream_t stream);
-// Fused decode step: append (v.step) + attention + combine/commit.
+// Fused decode step: attention with the append of v.step folded in, then combine + counters.
 cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
                                int head_dim, int out_dtype, cudaStream_t stream);
 // CTAs of one SM for the attention kernel of this shape (0 if the shape is not compiled).

@@ -331,11 +331,14 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     e = cudaMemcpy(kv->inv_freq, inv_freq.data(), inv_freq.size() * sizeof(double),
                    cudaMemcpyHostToDevice);
   // (cos, sin) of p * inv_freq[i] for every position a sequence can reach by slot index (or
-  // ~4 tokens per slot), capped at 64 MiB; the append kernel falls back to sincos beyond.
+  // 4 tokens per slot), in fp64 (stored bits) and fp32 (the attention pass), both tables
+  // capped at 512 MiB together (~350k positions at head_dim 128); the kernels fall back to
+  // sincos beyond, which on this GPU's narrow fp64 pipe costs microseconds per launch.
   if (e == cudaSuccess) {
     const int64_t half = cfg.head_dim / 2;
     const int64_t reach = (int64_t)cfg.max_slots_per_seq * (cfg.pos_mode == HAM_POS_TOKEN ? 4 : 1);
-    const int64_t cap = (int64_t)(64u << 20) / (half * (int64_t)sizeof(double2));
+    const int64_t cap = (int64_t)(512u << 20) /
+                        (half * (int64_t)(sizeof(double2) + sizeof(float2)));
     kv->rope_positions = std::min(reach, cap);
     std::vector<double2> table((size_t)(kv->rope_positions * half));
     std::vector<float2> table_f(table.size());
@@ -489,26 +492,35 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
   return HAM_OK;
 }
 
-int ham_decode_step(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
+namespace {
+bool overlaps(const void *a, size_t a_bytes, const void *b, size_t b_bytes) {
+  const uintptr_t a0 = (uintptr_t)a, b0 = (uintptr_t)b;
+  return a && b && a0 < b0 + b_bytes && b0 < a0 + a_bytes;
+}
+}  // namespace
+
+int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const void *k_new,
                     const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
                     int32_t out_dtype, void *stream) {
   int rc = check_layer(kv, layer);
   if (rc) return rc;
-  if (!q_inout || !k_new || !v_new || !ntok || !out)
-    return fail(HAM_EINVAL, "q_inout, k_new, v_new, ntok and out are required");
-  if (!aligned16(q_inout) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out))
-    return fail(HAM_EINVAL, "q/k/v/out must be 16-byte aligned");
+  if (!q || !k_new || !v_new || !ntok || !out)
+    return fail(HAM_EINVAL, "q, k_new, v_new, ntok and out are required");
+  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
+      (q_rot && !aligned16(q_rot)))
+    return fail(HAM_EINVAL, "q/q_rot/k/v/out must be 16-byte aligned");
   if (((uintptr_t)ntok & 3u) || ((uintptr_t)pos & 3u))
     return fail(HAM_EINVAL, "pos/ntok must be 4-byte aligned");
   if (out_dtype != HAM_DTYPE_BF16 && out_dtype != HAM_DTYPE_F32)
     return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
   const ham_config &c = kv->cfg;
   const int group = c.n_q_heads / c.n_kv_heads;
-  {  // q_inout is rewritten while out is being written: they must not overlap
-    const uintptr_t q0 = (uintptr_t)q_inout, o0 = (uintptr_t)out;
-    const uintptr_t n = (uintptr_t)c.batch * c.n_q_heads * c.head_dim;
-    const uintptr_t q1 = q0 + n * 2, o1 = o0 + n * (out_dtype == HAM_DTYPE_F32 ? 4 : 2);
-    if (q0 < o1 && o0 < q1) return fail(HAM_EINVAL, "out overlaps q_inout");
+  {  // outputs are written while q is still being read
+    const size_t n = (size_t)c.batch * c.n_q_heads * c.head_dim;
+    const size_t out_bytes = n * (out_dtype == HAM_DTYPE_F32 ? 4 : 2);
+    if (overlaps(q, n * 2, out, out_bytes) || overlaps(q_rot, n * 2, q, n * 2) ||
+        overlaps(q_rot, n * 2, out, out_bytes))
+      return fail(HAM_EINVAL, "q, q_rot and out must not overlap");
   }
   DeviceGuard guard(kv->device);
   ham::AttnView v{};
@@ -516,7 +528,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
   v.v_pool = layer_pool(kv, layer, 1);
   v.page_table = kv->page_table;
   v.num_slots = kv->num_slots + (size_t)layer * c.batch;
-  v.q = static_cast<const uint16_t *>(q_inout);
+  v.q = static_cast<const uint16_t *>(q);
   v.out = out;
   v.part_acc = kv->part_acc;
   v.part_ml = kv->part_ml;
@@ -533,7 +545,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
   ham::StepArgs &st = v.step;
   st.k_new = static_cast<const uint16_t *>(k_new);
   st.v_new = static_cast<const uint16_t *>(v_new);
-  st.q_inout = static_cast<uint16_t *>(q_inout);
+  st.q_rot = static_cast<uint16_t *>(q_rot);
   st.pos = pos;
   st.ntok = ntok;
   st.num_slots = kv->num_slots + (size_t)layer * c.batch;

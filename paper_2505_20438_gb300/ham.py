@@ -82,7 +82,7 @@ _SIGNATURES = {
     "ham_kv_set_attn_ctas": [_vp, _i32],
     "ham_split_plan": [_i32, _i32, _vp, _i32, _vp, _vp, _vp],
     "ham_decode_attn_noalloc": [ctypes.c_void_p, _vp],
-    "ham_decode_step": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
+    "ham_decode_step": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
 }
 _lib = None
 
@@ -231,13 +231,15 @@ def ham_decode_attn_ex(kv: KV, layer, q, out, stream=None):
         HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16, _stream_ptr(stream)))
 
 
-def ham_decode_step(kv: KV, layer, q_inout, k_new, v_new, pos, ntok, out, stream=None):
-    """Fused append + attention of one layer.  Output dtype follows `out` (bf16 or fp32)."""
+def ham_decode_step(kv: KV, layer, q, k_new, v_new, pos, ntok, out, q_rot=None, stream=None):
+    """Fused append + attention of one layer.  q is the unrotated query (not written);
+    q_rot (optional) receives RoPE(q).  Output dtype follows `out` (bf16 or fp32)."""
     import torch
     B, Hq, Hkv, d = kv.batch, kv.n_q_heads, kv.n_kv_heads, kv.head_dim
     f32 = out is not None and out.dtype == torch.float32
     _check(lib().ham_decode_step(
-        kv, layer, _dev(q_inout, (B, Hq, d), "bf16", "q_inout"),
+        kv, layer, _dev(q, (B, Hq, d), "bf16", "q"),
+        _dev(q_rot, (B, Hq, d), "bf16", "q_rot", nullable=True),
         _dev(k_new, (B, Hkv, d), "bf16", "k_new"), _dev(v_new, (B, Hkv, d), "bf16", "v_new"),
         _dev(pos, (B,), "i32", "pos", nullable=True), _dev(ntok, (B,), "i32", "ntok"),
         _dev(out, (B, Hq, d), "f32" if f32 else "bf16", "out"),

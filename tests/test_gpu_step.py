@@ -1,7 +1,8 @@
 """GPU: the fused decode step (append + attention in one pass over the cache).
 
-The cache, the counters and the rotated q it leaves are compared bit for bit with the
-oracle's append; its attention output with the oracle's attention over the n + 1 slots.
+The cache, the counters and the rotated q it reports (q_rot) are compared bit for bit with
+the oracle's append; its attention output with the oracle's attention over the n + 1 slots.
+The query it is given is never written.
 """
 import numpy as np
 import pytest
@@ -22,6 +23,7 @@ pytestmark = pytest.mark.gpu
 # the same weights are rounded the same way, so only a rare one-ulp difference of an
 # fp32-rotated q or k element separates the fused step from the two separate calls.
 SAME_SPLIT_MAX, SAME_SPLIT_MEAN = 2e-3, 2e-5
+Q_ROT_UNWRITTEN = 0x7FC1  # a bf16 NaN pattern no rotation produces
 
 
 def _export_host(kv, layer=0):
@@ -38,14 +40,18 @@ def _assert_cache_equal(kv, oc, layer=0):
     assert np.array_equal(slots, oc.num_slots) and np.array_equal(tokens, oc.num_tokens)
 
 
-def _step(kv, q_dev, k_new, v_new, ntok, pos=None, f32=True, layer=0):
+def _step(kv, q_bits, k_new, v_new, ntok, pos=None, f32=True, layer=0):
+    """One fused step; returns (out as float64, q_rot bits).  Checks that q is untouched."""
     t = torch()
+    q_dev = dev_bf16(q_bits)
+    q_rot = dev_bf16(np.full(q_bits.shape, Q_ROT_UNWRITTEN, np.uint16))
     out = t.full(q_dev.shape, float("nan"), dtype=t.float32 if f32 else t.bfloat16,
                  device="cuda")
     ham.ham_decode_step(kv, layer, q_dev, dev_bf16(k_new), dev_bf16(v_new),
-                        None if pos is None else dev_i32(pos), dev_i32(ntok), out)
+                        None if pos is None else dev_i32(pos), dev_i32(ntok), out, q_rot=q_rot)
     t.cuda.synchronize()
-    return out.float().cpu().numpy().astype(np.float64)
+    assert np.array_equal(host_bits(q_dev), q_bits), "q was written"
+    return out.float().cpu().numpy().astype(np.float64), host_bits(q_rot)
 
 
 @pytest.mark.parametrize("pos_mode", [ham.HAM_POS_SLOT, ham.HAM_POS_TOKEN])
@@ -60,38 +66,37 @@ def test_step_matches_oracle(pos_mode, d, hq, hkv, page, counts):
                       seed=11, extra_slots=8)
     oc = oracle.OracleCache.from_case(case)
     kv = gpu_cache(case, pos_mode=pos_mode)
-    q_host = case.q.copy()
-    q_dev = dev_bf16(case.q)
+    q = case.q.copy()
     rng = wl.rng_for(11, 60)
     for step in range(3):
         k_new = wl.normal_bf16(rng, case.k_new.shape)
         v_new = wl.normal_bf16(rng, case.v_new.shape)
         ntok = wl.ntok_capped_geometric(rng, (case.w.batch,))
-        assert oc.append(k_new, v_new, ntok, q_inout=q_host, pos_mode=pos_mode) == 0
-        ref = oc.decode_attn(q_host)
-        got = _step(kv, q_dev, k_new, v_new, ntok)
-        assert np.array_equal(host_bits(q_dev), q_host), f"q after step {step}"
+        q_ref = q.copy()
+        assert oc.append(k_new, v_new, ntok, q_inout=q_ref, pos_mode=pos_mode) == 0
+        ref = oc.decode_attn(q_ref)
+        got, q_rot = _step(kv, q, k_new, v_new, ntok)
+        assert np.array_equal(q_rot, q_ref), f"q_rot after step {step}"
         assert_parity(got, ref, MAX_ABS, MEAN_ABS, what=f"step {step}")
-        q_host = wl.normal_bf16(rng, case.q.shape)   # next macro-step's fresh queries
-        q_dev = dev_bf16(q_host)
+        q = wl.normal_bf16(rng, case.q.shape)        # next macro-step's fresh queries
     _assert_cache_equal(kv, oc)
     assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
 
 
 def test_step_equals_append_then_attend_on_gpu():
-    """Same cache bits and q bits as the two separate calls; outputs agree closely."""
+    """Same cache bits and rotated q bits as the two separate calls; outputs agree closely."""
     case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(100, 17, 640), seed=12)
     kv1, kv2 = gpu_cache(case), gpu_cache(case)
     for kv in (kv1, kv2):
         ham.ham_kv_set_attn_ctas(kv, 300)          # the same split for both paths
-    q1, q2 = dev_bf16(case.q), dev_bf16(case.q)
+    q1 = dev_bf16(case.q)
     t = torch()
     out1 = t.empty(q1.shape, dtype=t.float32, device="cuda")
     ham.ham_kv_append(kv1, 0, q1, dev_bf16(case.k_new), dev_bf16(case.v_new), None,
                       dev_i32(case.ntok_new))
     ham.ham_decode_attn_ex(kv1, 0, q1, out1)
-    out2 = _step(kv2, q2, case.k_new, case.v_new, case.ntok_new)
-    assert np.array_equal(host_bits(q1), host_bits(q2))
+    out2, q_rot = _step(kv2, case.q, case.k_new, case.v_new, case.ntok_new)
+    assert np.array_equal(host_bits(q1), q_rot)
     a, b = _export_host(kv1), _export_host(kv2)
     for x, y in zip(a, b):
         assert np.array_equal(x, y)
@@ -105,47 +110,46 @@ def test_step_positions_beyond_the_rope_table():
     oc = oracle.OracleCache.from_case(case)
     kv = gpu_cache(case)
     pos = np.array([0, 4095, 131071, 262143], np.int32)
-    q_host = case.q.copy()
-    q_dev = dev_bf16(case.q)
-    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_host, pos=pos) == 0
-    ref = oc.decode_attn(q_host)
-    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new, pos=pos)
-    assert np.array_equal(host_bits(q_dev), q_host)
+    q_ref = case.q.copy()
+    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_ref, pos=pos) == 0
+    ref = oc.decode_attn(q_ref)
+    got, q_rot = _step(kv, case.q, case.k_new, case.v_new, case.ntok_new, pos=pos)
+    assert np.array_equal(q_rot, q_ref)
     assert_parity(got, ref, MAX_ABS, MEAN_ABS, what="large positions")
     _assert_cache_equal(kv, oc)
 
 
 @pytest.mark.parametrize("ctas", [1, 5, 37, 600])
 def test_step_split_counts(ctas):
-    """Any CTA count: identical cache and q, attention within tolerance."""
+    """Any CTA count: identical cache and q_rot, attention within tolerance."""
     case = small_case(batch=3, hq=8, hkv=2, d=64, page=16, counts=(0, 333, 48), seed=14)
     oc = oracle.OracleCache.from_case(case)
     kv = gpu_cache(case)
     ham.ham_kv_set_attn_ctas(kv, ctas)
-    q_host = case.q.copy()
-    q_dev = dev_bf16(case.q)
-    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_host) == 0
-    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new)
-    assert np.array_equal(host_bits(q_dev), q_host)
-    assert_parity(got, oc.decode_attn(q_host), MAX_ABS, MEAN_ABS, what=f"ctas={ctas}")
+    q_ref = case.q.copy()
+    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_ref) == 0
+    got, q_rot = _step(kv, case.q, case.k_new, case.v_new, case.ntok_new)
+    assert np.array_equal(q_rot, q_ref)
+    assert_parity(got, oc.decode_attn(q_ref), MAX_ABS, MEAN_ABS, what=f"ctas={ctas}")
     _assert_cache_equal(kv, oc)
 
 
 def test_step_failed_appends_behave_like_the_two_calls():
-    """A full sequence and ntok = 0: no append, q untouched, old slots attended, error set."""
+    """A full sequence and ntok = 0: no append, unrotated q attends over the old slots, the
+    error is recorded and q_rot rows of those sequences are left alone."""
     case = small_case(batch=3, hq=8, hkv=2, d=64, page=16, counts=(20, 37, 9), seed=15,
                       extra_slots=0)
     oc = oracle.OracleCache.from_case(case)
     assert case.max_slots == 37                    # sequence 1 is full
     kv = gpu_cache(case)
     ntok = np.array([2, 1, 0], np.int32)           # sequence 2 gives ntok = 0
-    q_host = case.q.copy()
-    q_dev = dev_bf16(case.q)
-    assert oc.append(case.k_new, case.v_new, ntok, q_inout=q_host) != 0
-    ref = oc.decode_attn(q_host)
-    got = _step(kv, q_dev, case.k_new, case.v_new, ntok)
-    assert np.array_equal(host_bits(q_dev), q_host)
-    assert np.array_equal(host_bits(q_dev)[1:], case.q[1:])   # untouched where skipped
+    q_ref = case.q.copy()
+    assert oc.append(case.k_new, case.v_new, ntok, q_inout=q_ref) != 0
+    ref = oc.decode_attn(q_ref)
+    got, q_rot = _step(kv, case.q, case.k_new, case.v_new, ntok)
+    assert np.array_equal(q_rot[0], q_ref[0])
+    assert np.all(q_rot[1:] == Q_ROT_UNWRITTEN)
+    assert np.array_equal(q_ref[1:], case.q[1:])   # the oracle left them unrotated too
     assert_parity(got, ref, MAX_ABS, MEAN_ABS, what="failed appends")
     # read (and clear) the error word first: the counter read-back refuses while it is set
     assert ham.ham_kv_status(kv) in (ham.HAM_DEVERR_CAPACITY, ham.HAM_DEVERR_NTOK)
@@ -162,9 +166,11 @@ def test_step_host_errors():
     with pytest.raises(ham.HamError):
         ham.ham_decode_step(kv, 1, q, k, v, None, n, out)          # layer out of range
     with pytest.raises(ham.HamError):
-        ham.ham_decode_step(kv, 0, q, k, v, None, n, q)             # out aliases q_inout
-    rc = ham.lib().ham_decode_step(kv, 0, q.data_ptr() + 2, k.data_ptr(), v.data_ptr(), None,
-                                   n.data_ptr(), out.data_ptr(), ham.HAM_DTYPE_BF16, None)
+        ham.ham_decode_step(kv, 0, q, k, v, None, n, q)             # out aliases q
+    with pytest.raises(ham.HamError):
+        ham.ham_decode_step(kv, 0, q, k, v, None, n, out, q_rot=out)  # q_rot aliases out
+    rc = ham.lib().ham_decode_step(kv, 0, q.data_ptr() + 2, None, k.data_ptr(), v.data_ptr(),
+                                   None, n.data_ptr(), out.data_ptr(), ham.HAM_DTYPE_BF16, None)
     assert rc == ham.HAM_EINVAL
     t.cuda.synchronize()
     slots, _ = ham.ham_slot_lengths(kv)
@@ -172,17 +178,32 @@ def test_step_host_errors():
 
 
 def test_step_then_attention_sees_the_slot():
-    """After a step, plain attention with the same q reproduces the step's output."""
+    """After a step, plain attention with the rotated q reproduces the step's output."""
     case = small_case(batch=2, hq=32, hkv=8, d=128, page=32, counts=(63, 500), seed=17)
     kv = gpu_cache(case)
     ham.ham_kv_set_attn_ctas(kv, 200)
-    q_dev = dev_bf16(case.q)
-    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new)
+    got, q_rot = _step(kv, case.q, case.k_new, case.v_new, case.ntok_new)
     t = torch()
-    again = t.empty(q_dev.shape, dtype=t.float32, device="cuda")
-    ham.ham_decode_attn_ex(kv, 0, q_dev, again)
+    again = t.empty(case.q.shape, dtype=t.float32, device="cuda")
+    ham.ham_decode_attn_ex(kv, 0, dev_bf16(q_rot), again)
     assert_parity(got, again.cpu().numpy().astype(np.float64), SAME_SPLIT_MAX, SAME_SPLIT_MEAN,
                   what="step vs attention after it")
+
+
+def test_step_without_q_rot():
+    """q_rot is optional; the cache and the output do not depend on it."""
+    case = small_case(batch=2, hq=8, hkv=2, d=64, page=16, counts=(40, 70), seed=18)
+    oc = oracle.OracleCache.from_case(case)
+    kv = gpu_cache(case)
+    q_ref = case.q.copy()
+    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_ref) == 0
+    t = torch()
+    out = t.full(case.q.shape, float("nan"), dtype=t.float32, device="cuda")
+    ham.ham_decode_step(kv, 0, dev_bf16(case.q), dev_bf16(case.k_new), dev_bf16(case.v_new),
+                        None, dev_i32(case.ntok_new), out)
+    assert_parity(out.cpu().numpy().astype(np.float64), oc.decode_attn(q_ref), MAX_ABS,
+                  MEAN_ABS, what="no q_rot")
+    _assert_cache_equal(kv, oc)
 
 
 @pytest.mark.parametrize("w", [wl.C1_LLAMA8B, wl.C2_RAGGED], ids=lambda w: w.name)
@@ -191,12 +212,11 @@ def test_step_full_size(w):
     case = wl.make_case(w, extra_slots=4)
     oc = oracle.OracleCache.from_case(case)
     kv = gpu_cache(case)
-    q_host = case.q.copy()
-    q_dev = dev_bf16(case.q)
-    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_host) == 0
-    ref = oc.decode_attn(q_host)
-    got = _step(kv, q_dev, case.k_new, case.v_new, case.ntok_new, f32=False)
-    assert np.array_equal(host_bits(q_dev), q_host)
+    q_ref = case.q.copy()
+    assert oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q_ref) == 0
+    ref = oc.decode_attn(q_ref)
+    got, q_rot = _step(kv, case.q, case.k_new, case.v_new, case.ntok_new, f32=False)
+    assert np.array_equal(q_rot, q_ref)
     assert_parity(got, ref, what=w.name)
     # the appended rows, bit for bit (the whole pool at this size is compared too)
     _assert_cache_equal(kv, oc)
