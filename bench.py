@@ -99,10 +99,15 @@ def measured_peak_hbm():
 
 
 def kernel_source_hash():
+    """Hash of the attention kernels' code (comments and blank space removed), which ties an
+    ncu summary to the code it measured."""
     h = hashlib.sha256()
     for name in ("ham_attn.cu", "ham_internal.cuh"):
-        with open(os.path.join(ROOT, "paper_2505_20438_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2505_20438_gb300", "csrc", name)) as f:
+            text = f.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()[:16]
 
 
@@ -450,6 +455,7 @@ def run_ours(args, w):
         "gpu_launches": n_graph * launches_per_graph * world,
         "e2e": e2e,
         "clocks": clocks.summary(),
+        "cost_model": cost_model(mean_ntok, ms_per_step * 1e3),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
@@ -457,6 +463,17 @@ def run_ours(args, w):
         print(json.dumps(result), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
+
+
+def cost_model(n, c_s_us, c_ratio=4.0 / 32.0):
+    """Speed-up per macro-step of the paper's cost analysis (Sec. 3.7),
+    r = n C(S) / (C(S) + (n - 1) c), as a MODELLED figure: n is the mean tokens per slot of the
+    workload, C(S) this layer's measured decode step, and c (the micro-step decoder's cost per
+    token) is assumed to be 4/32 of C(S), a 4-layer decoder against a 32-layer base model."""
+    c = c_ratio * c_s_us
+    return {"r": round(n * c_s_us / (c_s_us + (n - 1) * c), 4), "n": round(n, 4),
+            "C_S_us": round(c_s_us, 3), "c_us": round(c, 3), "kind": "modelled",
+            "assumption": "c = 4/32 of C(S): 4 micro-decoder layers against 32 base layers"}
 
 
 def run_e2e(args, w, caches, stream, rollback, world, one_step):
@@ -525,11 +542,22 @@ def cpu_baseline(w, seconds):
         dt = time.perf_counter() - t0
         if dt >= seconds or n >= 10000:
             break
+    # the same steps on one host thread, for a bounded few seconds
+    n1, t1 = 0, time.perf_counter()
+    while True:
+        q = case.q.copy()
+        oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q)
+        oc.decode_attn(q, n_threads=1)
+        oc.num_slots[:] = case.num_slots
+        n1 += 1
+        dt1 = time.perf_counter() - t1
+        if dt1 >= min(3.0, seconds / 4) or n1 >= 1000:
+            break
     return {"value": round(n / dt, 4), "unit": UNIT, "cores": oracle.max_threads(),
-            "kind": "oracle",
+            "kind": "oracle", "single_thread_value": round(n1 / dt1, 4),
             "sample": f"{n} full macro-steps (append + attention of all {w.batch * w.n_q_heads} "
                       f"query heads over {w.slots} slots) of {w.name}, fp64 C oracle, "
-                      f"OpenMP over (sequence, head)"}
+                      f"OpenMP over (sequence, head); then {n1} on one thread"}
 
 
 def run_reference(args, w):

@@ -3,7 +3,7 @@
  *
  * Method: HAMburger (Liu & Zhang, arXiv 2505.20438).  A macro-step is one forward of the
  * base model that stores ONE key/value set for the whole group of 1..4 tokens it fused
- * (Sec. 3.1; Sec. 3.6 "Token Fusion"); the cache therefore holds one "slot" per macro-step,
+ * (Sec. 3.1; Sec. 3.7 "Token Fusion"); the cache therefore holds one "slot" per macro-step,
  * and each decode step attends over the slots and appends the slot just produced.  The
  * merged embedding enters the base model at an offset position reflecting the fused token
  * count (Sec. 3.2).  With one token per slot everything reduces to the base model's own

@@ -6,12 +6,12 @@
  *
  * What it computes, and where the paper fixes it:
  *  - A macro-step is one forward of the base model that stores ONE key/value set
- *    for the whole group of tokens it fused (Sec. 3.1; Sec. 3.6 "Token Fusion").
+ *    for the whole group of tokens it fused (Sec. 3.1; Sec. 3.7 "Token Fusion").
  *    The cache is therefore a list of slots, each standing for 1..4 tokens, and
  *    the attention of a decode step is ordinary softmax attention over that list:
  *    nothing in the paper weights a slot by its token count.
  *  - With a single token per slot the computation is the base model's own
- *    (Sec. 3.4; Sec. 3.6 "Minimal Overhead"), i.e. standard causal decode.
+ *    (Sec. 3.4; Sec. 3.7 "Minimal Overhead"), i.e. standard causal decode.
  *  - The base model is Llama-3.2-1B-Instruct (Sec. 4.1): rotate-half RoPE,
  *    grouped-query attention, softmax scale 1/sqrt(head_dim).
  *  - The merged embedding is sent to the base model with an offset position that

@@ -1,7 +1,7 @@
 // Split-KV GQA decode attention over the paged smashed-KV cache (sm_103a).
 //
 // What it computes (HAMburger, arXiv 2505.20438): one KV set per macro-step (Sec. 3.1,
-// Sec. 3.6 "Token Fusion"), so a decode step is plain softmax attention of each query head
+// Sec. 3.7 "Token Fusion"), so a decode step is plain softmax attention of each query head
 // over the slot list of its sequence, scale 1/sqrt(d), query head h reading KV head h / G
 // (Llama-3.2 base model, Sec. 4.1).  Decoding re-reads the whole cache every step and is
 // bound by memory bandwidth (Sec. 2.3), so the kernel moves every K/V byte from HBM once

@@ -1,7 +1,7 @@
 // Paged smashed-KV store: allocation, page tables, counters, fill/export and the C ABI
 // entry points that are not kernels of the decode path.
 //
-// A macro-step of HAMburger stores one KV set for all tokens it fused (Sec. 3.1, Sec. 3.6
+// A macro-step of HAMburger stores one KV set for all tokens it fused (Sec. 3.1, Sec. 3.7
 // "Token Fusion"), so the store is a per-sequence list of slots, each with the position it
 // was rotated at (Sec. 3.2) and its token count.
 #include <algorithm>

@@ -8,7 +8,7 @@ without sharing any of the method's code.
 Workloads stand in for the paper's decode workloads (short-context GSM8K /
 HumanEval / MGSM and long-context MultiNews / LongBench decoding, Sec. 4.3 and
 Fig. 5); the datasets and trained weights are not used.  A slot is one
-"smashed" KV entry that stands for 1..4 tokens (Sec. 3.1 and Sec. 3.6, token
+"smashed" KV entry that stands for 1..4 tokens (Sec. 3.1 and Sec. 3.7, token
 fusion), with at most 4 tokens per macro-step (Sec. 4.1).
 
 Token counts per slot follow a geometric law with p = 0.5 whose tail is folded
