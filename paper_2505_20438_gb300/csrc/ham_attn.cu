@@ -76,6 +76,12 @@ __device__ __forceinline__ void mbar_arrive_tx(uint64_t *bar, uint32_t bytes) {
                "r"(bytes)
                : "memory");
 }
+// Add `bytes` to the transaction count of the current phase without arriving.
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
 __device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -235,8 +241,9 @@ struct Layout {
     off_info = align_up(off_bar + 2 * S::kStages * 8, 16);
     off_flags = off_info + S::kStages * 16;
     off_cum = off_flags + 16;
-    // cum [B+1], lens [B], and for the fused step the new slot's position and flag [B] each
-    total = off_cum + 4 * (batch + 1) + 4 * batch * (step ? 3 : 1);
+    // cum [B+1], lens [B], and for the fused step the counter, the new slot's position and
+    // the append flag [B] each
+    total = off_cum + 4 * (batch + 1) + 4 * batch * (step ? 4 : 1);
   }
 };
 
@@ -311,8 +318,10 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
   int32_t *lens = cum + B + 1;                                      // [B] slots attended
   int32_t *posb = lens + B;                                         // [B] new slot position
   int32_t *appb = posb + B;                                         // [B] 1: append happens
+  int32_t *lraw = appb + B;  // [B] counter, clamped; -(counter + 1) if it was out of range
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const bool early = v.early != 0;
 
   if (tid == 0) {
     for (int s = 0; s < S::kStages; ++s) {
@@ -326,11 +335,16 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     prefetch_tensormap(&tmap_k);
     prefetch_tensormap(&tmap_v);
   }
-  // Programmatic dependent launch: everything above overlaps the previous kernel's tail;
-  // slot counters, q and the pools are read only after it has completed.  The combine
-  // kernel that follows may be scheduled now (it waits for this grid to finish).
-  grid_dependency_wait();
-  grid_launch_dependents();
+  // Programmatic dependent launch.  Everything above overlaps the previous kernel's tail.  If
+  // the host found that the previous launch on this stream wrote nothing of this layer
+  // (`early`), the counters, the plan, the page table and the first K/V copies also run
+  // before the dependency wait: they are this layer's library state, which no running kernel
+  // writes.  Caller inputs (q, k_new, v_new, pos, ntok) and the shared scratch are touched only
+  // after it.  The combine kernel that follows may be scheduled once the wait has returned.
+  if (!early) {
+    grid_dependency_wait();
+    grid_launch_dependents();
+  }
   if (warp == 0) {  // chunks per sequence and their prefix sums
     int run = 0;
     for (int b0 = 0; b0 < B; b0 += 32) {
@@ -343,17 +357,14 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
           record_error(v.err, HAM_DEVERR_SLOTS);
           L = L < 0 ? 0 : v.max_slots;
         }
-        if constexpr (kStep) {  // the slot this step appends is attended too
-          const int t = v.step.ntok[b];
-          // 0: append; else the error that stops it (same order as ham_kv_append)
-          const int why = t < 1 ? HAM_DEVERR_NTOK
-                          : bad ? HAM_DEVERR_SLOTS
-                          : L == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
-          const int64_t p = step_position(v.step, b, L);
-          posb[b] = (int32_t)p;
-          appb[b] = why == 0;
-          if (blockIdx.x == 0) v.step.stash[b] = make_int4(L, why, (int32_t)p, t);
-          L += why == 0;
+        // fused step: the slot it appends is attended too.  Whether the append happens also
+        // depends on ntok (a caller input); the plan counts the slot whenever there is room,
+        // and a refused slot is masked out of its chunk later.
+        if constexpr (kStep) {
+          lraw[b] = bad ? -(L + 1) : L;
+          // the new slot's position, unless the caller gives it (library state otherwise)
+          if (!v.step.pos) posb[b] = (int32_t)step_position(v.step, b, L);
+          if (!bad && L < v.max_slots) L += 1;
         }
         lens[b] = L;
         n = chunks_of(L);
@@ -372,6 +383,81 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
   __syncthreads();
 
   const int64_t W = (int64_t)Hkv * cum[B];
+  // Only min(gridDim.x, W) CTAs take part, so that every range holds at least one chunk:
+  // the CTAs touching a segment are then exactly first..last (no idle CTA in between).
+  const int C = plan_ctas(W, gridDim.x);
+  const bool active_cta = (int)blockIdx.x < C;
+  const int64_t x0 = active_cta ? plan_cta_begin(W, C, blockIdx.x) : 0;
+  const int64_t x1 = active_cta ? plan_cta_begin(W, C, (int64_t)blockIdx.x + 1) : 0;
+  const int nchunks = (int)(x1 - x0);
+
+  // Producer lanes decode 32 chunks at a time: lane j holds chunk base + j.
+  auto decode = [&](int base, int &seg, int &valid, int &fl, int &row0) {
+    const int64_t x = x0 + base + lane;
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if ((int64_t)Hkv * cum[mid] <= x) lo = mid; else hi = mid - 1;
+    }
+    const int b = lo;
+    const int nch = cum[b + 1] - cum[b];
+    const int r = (int)(x - (int64_t)Hkv * cum[b]);
+    const int g = r / nch, c = r - g * nch;
+    seg = b * Hkv + g;
+    valid = min(kChunkSlots, lens[b] - c * kChunkSlots);
+    const int slot0 = c * kChunkSlots;
+    const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
+    const bool page_ok = page >= 0 && page < v.pool_pages;
+    row0 = ((page_ok ? page : 0) * Hkv + g) * v.page_slots + slot0 % v.page_slots;
+    fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
+         ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
+    // the chunk that holds the appended slot (when the plan counted one)
+    if (kStep && c == nch - 1 && lens[b] > lraw[b]) fl |= kNewRow;
+  };
+
+  // The first ring's worth of K/V copies.  Their stages expect the K/V bytes now and arrive
+  // (with the bytes of q and the step rows, if the stage opens a segment) after the wait.
+  int seg0 = 0, valid0 = 0, fl0 = 0, row00 = 0, pre = 0;
+  if (warp == 1 && active_cta) {
+    const int nb = min(32, nchunks);
+    if (lane < nb) decode(0, seg0, valid0, fl0, row00);
+    pre = min(nb, S::kStages);
+    const uint64_t pol = policy_evict_first();
+    for (int j = 0; j < pre; ++j) {
+      const int s_fl = __shfl_sync(kFull, fl0, j);
+      const int s_row = __shfl_sync(kFull, row00, j);
+      if (lane == 0 && (s_fl & kPageOk)) {
+        uint8_t *dst = stages + j * S::kStageBytes;
+        mbar_expect_tx(&full[j], (uint32_t)S::kStageBytes);
+        tma_load_3d(dst, &tmap_k, 0, 0, s_row, &full[j], pol);
+        tma_load_3d(dst + S::kChunkBytes, &tmap_v, 0, 0, s_row, &full[j], pol);
+      }
+    }
+  }
+  if (early) {
+    grid_dependency_wait();
+    grid_launch_dependents();
+  }
+  if constexpr (kStep) {
+    // Caller inputs of the append: explicit positions, and whether each append happens.
+    // (Computing the flags after the block barrier instead, in the consumer warp alone while
+    // the producer went on, made the pass 20-35% slower.)
+    if (warp == 0) {
+      if (v.step.pos)
+        for (int b = lane; b < B; b += 32) posb[b] = v.step.pos[b];
+      for (int b = lane; b < B; b += 32) {
+        const bool bad = lraw[b] < 0;
+        const int L = bad ? -(lraw[b] + 1) : lraw[b];
+        const int t = v.step.ntok[b];
+        // 0: append; else the error that stops it (same order as ham_kv_append)
+        const int why = t < 1 ? HAM_DEVERR_NTOK
+                        : bad ? HAM_DEVERR_SLOTS
+                        : L == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
+        appb[b] = why == 0;
+        if (blockIdx.x == 0) v.step.stash[b] = make_int4(L, why, posb[b], t);
+      }
+    }
+  }
   // Sequences with no slots attend to nothing: their output is 0.  Segment s is zeroed by
   // CTA s % gridDim.x (before any CTA may leave for lack of chunks).
   for (int s = blockIdx.x; s < B * Hkv; s += gridDim.x) {
@@ -381,13 +467,8 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
       store_out<OutT>(v.out, (int64_t)s * G * D + idx, 0.f);
     if (tid == 0) v.seg_range[s] = make_int2(-1, -1);
   }
-  // Only min(gridDim.x, W) CTAs take part, so that every range holds at least one chunk:
-  // the CTAs touching a segment are then exactly first..last (no idle CTA in between).
-  const int C = plan_ctas(W, gridDim.x);
-  if ((int)blockIdx.x >= C) return;
-  const int64_t x0 = plan_cta_begin(W, C, blockIdx.x);
-  const int64_t x1 = plan_cta_begin(W, C, (int64_t)blockIdx.x + 1);
-  const int nchunks = (int)(x1 - x0);
+  __syncthreads();
+  if (!active_cta) return;
 
   // ---------------------------------------------------------------- producer warp
   if (warp == 1) {
@@ -395,39 +476,20 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     int it = 0, nseg = 0;
     for (int base = 0; base < nchunks; base += 32) {
       const int nb = min(32, nchunks - base);
-      int seg = 0, valid = 0, fl = 0, row0 = 0;
-      if (lane < nb) {  // decode chunk x0 + base + lane
-        const int64_t x = x0 + base + lane;
-        int lo = 0, hi = B - 1;
-        while (lo < hi) {
-          const int mid = (lo + hi + 1) >> 1;
-          if ((int64_t)Hkv * cum[mid] <= x) lo = mid; else hi = mid - 1;
-        }
-        const int b = lo;
-        const int nch = cum[b + 1] - cum[b];
-        const int r = (int)(x - (int64_t)Hkv * cum[b]);
-        const int g = r / nch, c = r - g * nch;
-        seg = b * Hkv + g;
-        valid = min(kChunkSlots, lens[b] - c * kChunkSlots);
-        const int slot0 = c * kChunkSlots;
-        const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
-        const bool page_ok = page >= 0 && page < v.pool_pages;
-        row0 = ((page_ok ? page : 0) * Hkv + g) * v.page_slots + slot0 % v.page_slots;
-        fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
-             ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
-        if (kStep && c == nch - 1 && appb[b]) fl |= kNewRow;  // holds the appended slot
-      }
+      int seg = seg0, valid = valid0, fl = fl0, row0 = row00;
+      if (base > 0 && lane < nb) decode(base, seg, valid, fl, row0);
       bool stop = false;
       for (int j = 0; j < nb; ++j) {
         const int s_seg = __shfl_sync(kFull, seg, j);
         const int s_valid = __shfl_sync(kFull, valid, j);
         const int s_fl = __shfl_sync(kFull, fl, j);
         const int s_row = __shfl_sync(kFull, row0, j);
+        const bool issued = it < pre;  // K/V already on their way (first ring)
         int failed = 0;
         if (lane == 0) {
           const int stage = it % S::kStages;
           const uint32_t ph = (uint32_t)(it / S::kStages) & 1u;
-          if (!thread_wait(&empty[stage], ph ^ 1u, flags, true)) {
+          if (!issued && !thread_wait(&empty[stage], ph ^ 1u, flags, true)) {
             record_error(v.err, HAM_DEVERR_TIMEOUT);
             flags[0] = 1;
             failed = 1;
@@ -437,7 +499,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
             const int b = s_seg / Hkv;
             if (s_fl & kFirst) qb = nseg++ % S::kQBufs;
             info[stage] = make_int4(s_seg, s_valid, s_fl, qb);
-            uint32_t bytes = (s_fl & kPageOk) ? (uint32_t)S::kStageBytes : 0u;
+            uint32_t bytes = ((s_fl & kPageOk) && !issued) ? (uint32_t)S::kStageBytes : 0u;
             if (qb >= 0) {
               bytes += (uint32_t)sb.q_bytes;
               if constexpr (kStep) {
@@ -449,11 +511,11 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
             if (bytes) mbar_arrive_tx(&full[stage], bytes);
             else mbar_arrive(&full[stage]);
             uint8_t *dst = stages + stage * S::kStageBytes;
-            if (s_fl & kPageOk) {
+            if (!(s_fl & kPageOk)) {
+              record_error(v.err, HAM_DEVERR_PAGE);
+            } else if (!issued) {
               tma_load_3d(dst, &tmap_k, 0, 0, s_row, &full[stage], pol);
               tma_load_3d(dst + S::kChunkBytes, &tmap_v, 0, 0, s_row, &full[stage], pol);
-            } else {
-              record_error(v.err, HAM_DEVERR_PAGE);
             }
             if (qb >= 0) {
               uint8_t *qdst = qbufs + qb * sb.stride;
@@ -561,15 +623,19 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     if (inf.z & kPageOk) {
       uint8_t *kt = stages + stage * S::kStageBytes;
       uint8_t *vt = kt + S::kChunkBytes;
-      const int nvalid = inf.y;
-      const bool patch = nvalid < kChunkSlots || (kStep && (inf.z & kNewRow));
+      // fused step: the plan counted the appended slot as this chunk's last row; if the append
+      // was refused (ntok < 1, full, bad counter) that row is masked out instead
+      const bool new_row = kStep && (inf.z & kNewRow);
+      const bool new_ok = new_row && appb[inf.x / Hkv];
+      const int nvalid = inf.y - ((new_row && !new_ok) ? 1 : 0);
+      const bool patch = nvalid < kChunkSlots || new_ok;
       if (nvalid < kChunkSlots) {  // rows past the sequence end never reach the MMA
         for (int i = lane; i < (kChunkSlots - nvalid) * (D / 8); i += 32) {
           const int slot = nvalid + i / (D / 8), c = i % (D / 8);
           *reinterpret_cast<uint4 *>(vt + tile_offset<D>(slot, c)) = make_uint4(0, 0, 0, 0);
         }
       }
-      if (kStep && (inf.z & kNewRow)) {  // the appended slot is the chunk's last valid row
+      if (new_ok) {  // the appended slot is the chunk's last valid row
         // its key, turned in fp32 by the new position, and its value, from the segment's
         // staging buffer (the copy of the row in HBM may not be written yet)
         const uint8_t *seg = qbufs + cur_qb * sb.stride;
@@ -665,7 +731,8 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     const int first = plan_owner(W, C, X0), last = plan_owner(W, C, X0 + nch - 1);
     const int64_t obase = (int64_t)seg * G * D;
     if (first == last) {  // the whole segment is ours: normalise and store
-      const float i0 = 1.f / l0, i1 = 1.f / l1;
+      // (a segment whose only slot was a refused append has l = 0: its output is 0)
+      const float i0 = l0 > 0.f ? 1.f / l0 : 0.f, i1 = l1 > 0.f ? 1.f / l1 : 0.f;
 #pragma unroll
       for (int t = 0; t < S::kSteps; ++t) {
         const int d0 = 16 * t + r0;
@@ -808,8 +875,9 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       }
       M = bm;
     }
-    store_out<OutT>(v.out, orow + i, num0 / den);
-    store_out<OutT>(v.out, orow + i + half, num1 / den);
+    const float inv = den > 0.f ? 1.f / den : 0.f;  // 0: every slot masked (refused append)
+    store_out<OutT>(v.out, orow + i, num0 * inv);
+    store_out<OutT>(v.out, orow + i + half, num1 * inv);
   }
 
   if constexpr (kStep) {

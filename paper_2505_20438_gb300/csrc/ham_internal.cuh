@@ -88,6 +88,10 @@ struct AttnView {
   int64_t pool_pages;
   int32_t batch, n_kv_heads, group, page_slots, max_pages, max_slots;
   int32_t ctas;
+  // 1: the previous launch on the stream wrote nothing of this layer's counters, page table or
+  // pools, so the kernel may read them before its programmatic-dependency wait (the host
+  // decides; 0 is always correct)
+  int32_t early;
   StepArgs step;               // used by launch_decode_step only
 };
 

@@ -9,6 +9,9 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <map>
+#include <mutex>
+#include <utility>
 #include <vector>
 
 #include "ham_internal.cuh"
@@ -84,6 +87,54 @@ struct DeviceGuard {
 
 uint16_t *layer_pool(const ham_kv *kv, int32_t layer, int which) {
   return kv->pool + ((size_t)layer * 2 + (size_t)which) * (size_t)kv->pool_elems;
+}
+
+// ---------------------------------------------------------------------------------------
+// Early start.  The attention kernels are launched with programmatic dependent launch and can
+// read their layer's counters, page table and pools before their dependency wait, which lets
+// the plan and the first K/V copies overlap the previous kernel, provided that kernel does not
+// write them.  Every kernel of this library waits for its own predecessor before letting its
+// successor start, so when an attention grid starts, everything before the immediately
+// preceding kernel has completed; only that kernel may still run.  The library remembers, per
+// stream (and per stream capture), the last launch it made and which (handle, layer) state it
+// writes, and allows the early start only when that launch is known and leaves this layer
+// alone.  Kernels of other code in between are harmless: they cannot write a handle's state
+// (only these calls do), and an unknown predecessor means no early start.
+// ---------------------------------------------------------------------------------------
+struct LastLaunch {
+  const ham_kv *kv;
+  int32_t layer;  // -1: every layer
+  bool writes;    // wrote the layer's counters, pools or slot metadata
+};
+std::mutex g_launch_mu;
+std::map<std::pair<uintptr_t, unsigned long long>, LastLaunch> g_last_launch;
+
+std::pair<uintptr_t, unsigned long long> launch_key(void *stream) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  unsigned long long id = 0;
+  if (cudaStreamGetCaptureInfo(static_cast<cudaStream_t>(stream), &st, &id) != cudaSuccess) {
+    cudaGetLastError();
+    id = ~0ull;  // unknown: gets its own (always conservative) entry
+  } else if (st != cudaStreamCaptureStatusActive) {
+    id = 0;
+  }
+  return {(uintptr_t)stream, id};
+}
+
+bool may_start_early(const ham_kv *kv, int32_t layer, void *stream) {
+  const auto key = launch_key(stream);
+  std::lock_guard<std::mutex> lock(g_launch_mu);
+  const auto it = g_last_launch.find(key);
+  if (it == g_last_launch.end()) return false;
+  const LastLaunch &l = it->second;
+  return !(l.kv == kv && l.writes && (l.layer == layer || l.layer < 0));
+}
+
+void note_launch(const ham_kv *kv, int32_t layer, void *stream, bool writes) {
+  const auto key = launch_key(stream);
+  std::lock_guard<std::mutex> lock(g_launch_mu);
+  if (g_last_launch.size() > 4096) g_last_launch.clear();  // forgetting is always safe
+  g_last_launch[key] = LastLaunch{kv, layer, writes};
 }
 
 }  // namespace
@@ -452,6 +503,7 @@ int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
   v.kv_per_block = ham::append_kv_per_block(v.n_q_heads, v.n_kv_heads, v.head_dim);
   cudaError_t e = ham::launch_append(v, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  note_launch(kv, layer, stream, true);
   return HAM_OK;
 }
 
@@ -485,10 +537,12 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
   v.max_pages = kv->max_pages;
   v.max_slots = kv->cfg.max_slots_per_seq;
   v.ctas = ctas;
+  v.early = may_start_early(kv, layer, stream) ? 1 : 0;
   cudaError_t e = ham::launch_attention(kv->tmaps[(size_t)layer * 2], kv->tmaps[(size_t)layer * 2 + 1],
                                         v, kv->cfg.head_dim, out_dtype,
                                         static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+  note_launch(kv, layer, stream, false);
   return HAM_OK;
 }
 
@@ -560,10 +614,12 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
   st.rope_positions = kv->rope_positions;
   st.stash = kv->stash;
   st.pos_mode = c.pos_mode;
+  v.early = may_start_early(kv, layer, stream) ? 1 : 0;
   cudaError_t e = ham::launch_decode_step(kv->tmaps[(size_t)layer * 2],
                                           kv->tmaps[(size_t)layer * 2 + 1], v, c.head_dim,
                                           out_dtype, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "decode step launch");
+  note_launch(kv, layer, stream, true);
   return HAM_OK;
 }
 
@@ -673,6 +729,7 @@ int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
   v.lmax = lmax;
   cudaError_t e = ham::launch_fill(v, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "fill launch");
+  note_launch(kv, layer, stream, true);
   return HAM_OK;
 }
 
@@ -702,6 +759,7 @@ int ham_kv_set_lengths(ham_kv *kv, int32_t layer, const int32_t *num_slots,
       kv->num_slots + (size_t)layer * B, kv->num_tokens + (size_t)layer * B, num_slots,
       num_tokens, B, kv->cfg.max_slots_per_seq, kv->err);
   HAM_CUDA(cudaGetLastError());
+  note_launch(kv, layer, stream, true);
   return HAM_OK;
 }
 
@@ -712,6 +770,7 @@ int ham_kv_reset(ham_kv *kv, void *stream) {
   const size_t n = (size_t)kv->cfg.layers * kv->cfg.batch;
   HAM_CUDA(cudaMemsetAsync(kv->num_slots, 0, n * sizeof(int32_t), s));
   HAM_CUDA(cudaMemsetAsync(kv->num_tokens, 0, n * sizeof(int64_t), s));
+  note_launch(kv, -1, stream, true);
   return HAM_OK;
 }
 

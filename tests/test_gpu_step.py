@@ -135,14 +135,15 @@ def test_step_split_counts(ctas):
 
 
 def test_step_failed_appends_behave_like_the_two_calls():
-    """A full sequence and ntok = 0: no append, unrotated q attends over the old slots, the
-    error is recorded and q_rot rows of those sequences are left alone."""
-    case = small_case(batch=3, hq=8, hkv=2, d=64, page=16, counts=(20, 37, 9), seed=15,
+    """A full sequence and ntok = 0 (one of them on an empty sequence): no append, unrotated
+    q attends over the old slots (none: output 0), the error is recorded and q_rot rows of
+    those sequences are left alone."""
+    case = small_case(batch=4, hq=8, hkv=2, d=64, page=16, counts=(20, 37, 9, 0), seed=15,
                       extra_slots=0)
     oc = oracle.OracleCache.from_case(case)
     assert case.max_slots == 37                    # sequence 1 is full
     kv = gpu_cache(case)
-    ntok = np.array([2, 1, 0], np.int32)           # sequence 2 gives ntok = 0
+    ntok = np.array([2, 1, 0, 0], np.int32)        # sequences 2 and 3 give ntok = 0
     q_ref = case.q.copy()
     assert oc.append(case.k_new, case.v_new, ntok, q_inout=q_ref) != 0
     ref = oc.decode_attn(q_ref)
@@ -151,9 +152,33 @@ def test_step_failed_appends_behave_like_the_two_calls():
     assert np.all(q_rot[1:] == Q_ROT_UNWRITTEN)
     assert np.array_equal(q_ref[1:], case.q[1:])   # the oracle left them unrotated too
     assert_parity(got, ref, MAX_ABS, MEAN_ABS, what="failed appends")
+    assert np.all(got[3] == 0.0)                   # nothing to attend to
     # read (and clear) the error word first: the counter read-back refuses while it is set
     assert ham.ham_kv_status(kv) in (ham.HAM_DEVERR_CAPACITY, ham.HAM_DEVERR_NTOK)
     _assert_cache_equal(kv, oc)
+
+
+def test_step_alternating_caches():
+    """Steps alternating between two caches on one stream: each launch may plan and start its
+    first copies before the previous one (other cache) has finished.  Every step is checked."""
+    cases = [small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=c, seed=s)
+             for c, s in (((300, 17, 64), 19), ((5, 250, 0), 20))]
+    ocs = [oracle.OracleCache.from_case(c) for c in cases]
+    kvs = [gpu_cache(c) for c in cases]
+    rng = wl.rng_for(19, 61)
+    for step in range(3):
+        for case, oc, kv in zip(cases, ocs, kvs):
+            q = wl.normal_bf16(rng, case.q.shape)
+            k_new = wl.normal_bf16(rng, case.k_new.shape)
+            v_new = wl.normal_bf16(rng, case.v_new.shape)
+            ntok = wl.ntok_capped_geometric(rng, (case.w.batch,))
+            q_ref = q.copy()
+            assert oc.append(k_new, v_new, ntok, q_inout=q_ref) == 0
+            got, q_rot = _step(kv, q, k_new, v_new, ntok)
+            assert np.array_equal(q_rot, q_ref)
+            assert_parity(got, oc.decode_attn(q_ref), MAX_ABS, MEAN_ABS, what=f"step {step}")
+    for oc, kv in zip(ocs, kvs):
+        _assert_cache_equal(kv, oc)
 
 
 def test_step_host_errors():
