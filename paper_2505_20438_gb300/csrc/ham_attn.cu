@@ -44,7 +44,7 @@ namespace {
 constexpr uint32_t kFull = 0xffffffffu;
 constexpr float kRescaleSlack = 8.0f;              // log2 units
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // bounded waits: 2 s
-constexpr int kFirst = 1, kLast = 2, kPageOk = 4, kNewRow = 8;  // stage flags
+constexpr int kFirst = 1, kLast = 2, kPageOk = 4;  // stage flags
 constexpr int kMaxGroup = 8;                       // heads padded to the MMA's N = 8
 
 // ------------------------------------------------------------------------------------
@@ -218,17 +218,14 @@ struct Shape {
   static_assert(kStages >= 2, "ring depth");
 };
 
-// Per-segment buffer: the group's q heads, and for the fused step also the new k and v
-// rows and the fp32 (cos, sin) of the new slot's position.
+// Per-segment buffer: the group's q heads, and for the fused step also the fp32 (cos, sin)
+// row of the new slot's position.
 template <int D>
 struct SegBuf {
   int q_bytes, stride;
   __host__ __device__ SegBuf(int group, bool step)
-      : q_bytes(group * D * 2),
-        stride(align_up(group * D * 2 + (step ? 2 * D * 2 + (D / 2) * 8 : 0), 128)) {}
-  __host__ __device__ int k_off() const { return q_bytes; }
-  __host__ __device__ int v_off() const { return q_bytes + D * 2; }
-  __host__ __device__ int cs_off() const { return q_bytes + 2 * D * 2; }
+      : q_bytes(group * D * 2), stride(align_up(group * D * 2 + (step ? (D / 2) * 8 : 0), 128)) {}
+  __host__ __device__ int cs_off() const { return q_bytes; }
 };
 
 // Shared memory map after the per-segment buffers (runtime: depends on group and batch).
@@ -241,9 +238,9 @@ struct Layout {
     off_info = align_up(off_bar + 2 * S::kStages * 8, 16);
     off_flags = off_info + S::kStages * 16;
     off_cum = off_flags + 16;
-    // cum [B+1], lens [B], and for the fused step the counter, the new slot's position and
-    // the append flag [B] each
-    total = off_cum + 4 * (batch + 1) + 4 * batch * (step ? 4 : 1);
+    // cum [B+1], lens [B], and for the fused step the new slot's position and the append
+    // flag [B] each
+    total = off_cum + 4 * (batch + 1) + 4 * batch * (step ? 3 : 1);
   }
 };
 
@@ -318,7 +315,6 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
   int32_t *lens = cum + B + 1;                                      // [B] slots attended
   int32_t *posb = lens + B;                                         // [B] new slot position
   int32_t *appb = posb + B;                                         // [B] 1: append happens
-  int32_t *lraw = appb + B;  // [B] counter, clamped; -(counter + 1) if it was out of range
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const bool early = v.early != 0;
@@ -357,14 +353,10 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
           record_error(v.err, HAM_DEVERR_SLOTS);
           L = L < 0 ? 0 : v.max_slots;
         }
-        // fused step: the slot it appends is attended too.  Whether the append happens also
-        // depends on ntok (a caller input); the plan counts the slot whenever there is room,
-        // and a refused slot is masked out of its chunk later.
+        // fused step: the pass attends over the stored slots; the combine kernel adds the
+        // appended one.  Its position, unless the caller gives it, is library state.
         if constexpr (kStep) {
-          lraw[b] = bad ? -(L + 1) : L;
-          // the new slot's position, unless the caller gives it (library state otherwise)
           if (!v.step.pos) posb[b] = (int32_t)step_position(v.step, b, L);
-          if (!bad && L < v.max_slots) L += 1;
         }
         lens[b] = L;
         n = chunks_of(L);
@@ -411,8 +403,6 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     row0 = ((page_ok ? page : 0) * Hkv + g) * v.page_slots + slot0 % v.page_slots;
     fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
          ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
-    // the chunk that holds the appended slot (when the plan counted one)
-    if (kStep && c == nch - 1 && lens[b] > lraw[b]) fl |= kNewRow;
   };
 
   // The first ring's worth of K/V copies.  Their stages expect the K/V bytes now and arrive
@@ -446,8 +436,9 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
       if (v.step.pos)
         for (int b = lane; b < B; b += 32) posb[b] = v.step.pos[b];
       for (int b = lane; b < B; b += 32) {
-        const bool bad = lraw[b] < 0;
-        const int L = bad ? -(lraw[b] + 1) : lraw[b];
+        int L = v.num_slots[b];
+        const bool bad = L < 0 || L > v.max_slots;
+        L = L < 0 ? 0 : (bad ? v.max_slots : L);
         const int t = v.step.ntok[b];
         // 0: append; else the error that stops it (same order as ham_kv_append)
         const int why = t < 1 ? HAM_DEVERR_NTOK
@@ -505,7 +496,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
               if constexpr (kStep) {
                 const int64_t p = posb[b];
                 tabled = p >= 0 && p < v.step.rope_positions;
-                bytes += 2u * D * 2 + (tabled ? (uint32_t)(D / 2) * 8 : 0u);
+                bytes += tabled ? (uint32_t)(D / 2) * 8 : 0u;
               }
             }
             if (bytes) mbar_arrive_tx(&full[stage], bytes);
@@ -520,9 +511,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
             if (qb >= 0) {
               uint8_t *qdst = qbufs + qb * sb.stride;
               bulk_load(qdst, v.q + (int64_t)s_seg * G * D, (uint32_t)sb.q_bytes, &full[stage]);
-              if constexpr (kStep) {  // the new k, v rows and (cos, sin) of its position
-                bulk_load(qdst + sb.k_off(), v.step.k_new + (int64_t)s_seg * D, D * 2, &full[stage]);
-                bulk_load(qdst + sb.v_off(), v.step.v_new + (int64_t)s_seg * D, D * 2, &full[stage]);
+              if constexpr (kStep) {  // (cos, sin) of the new slot's position
                 if (tabled)
                   bulk_load(qdst + sb.cs_off(),
                             v.step.rope_table_f + (int64_t)posb[b] * (D / 2), (D / 2) * 8,
@@ -623,37 +612,13 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     if (inf.z & kPageOk) {
       uint8_t *kt = stages + stage * S::kStageBytes;
       uint8_t *vt = kt + S::kChunkBytes;
-      // fused step: the plan counted the appended slot as this chunk's last row; if the append
-      // was refused (ntok < 1, full, bad counter) that row is masked out instead
-      const bool new_row = kStep && (inf.z & kNewRow);
-      const bool new_ok = new_row && appb[inf.x / Hkv];
-      const int nvalid = inf.y - ((new_row && !new_ok) ? 1 : 0);
-      const bool patch = nvalid < kChunkSlots || new_ok;
-      if (nvalid < kChunkSlots) {  // rows past the sequence end never reach the MMA
+      const int nvalid = inf.y;
+      const bool patch = nvalid < kChunkSlots;
+      if (patch) {  // rows past the sequence end never reach the MMA
         for (int i = lane; i < (kChunkSlots - nvalid) * (D / 8); i += 32) {
           const int slot = nvalid + i / (D / 8), c = i % (D / 8);
           *reinterpret_cast<uint4 *>(vt + tile_offset<D>(slot, c)) = make_uint4(0, 0, 0, 0);
         }
-      }
-      if (new_ok) {  // the appended slot is the chunk's last valid row
-        // its key, turned in fp32 by the new position, and its value, from the segment's
-        // staging buffer (the copy of the row in HBM may not be written yet)
-        const uint8_t *seg = qbufs + cur_qb * sb.stride;
-        const uint16_t *kn = reinterpret_cast<const uint16_t *>(seg + sb.k_off());
-        const float2 *cs = reinterpret_cast<const float2 *>(seg + sb.cs_off());
-        const int row = nvalid - 1;
-        for (int i = lane; i < D / 2; i += 32) {
-          const float2 cx = cs[i];
-          const float x0 = bf16_bits_to_float(kn[i]), x1 = bf16_bits_to_float(kn[i + D / 2]);
-          const int i1 = i + D / 2;
-          *reinterpret_cast<__nv_bfloat16 *>(kt + tile_offset<D>(row, i >> 3) + (i & 7) * 2) =
-              __float2bfloat16_rn(x0 * cx.x - x1 * cx.y);
-          *reinterpret_cast<__nv_bfloat16 *>(kt + tile_offset<D>(row, i1 >> 3) + (i1 & 7) * 2) =
-              __float2bfloat16_rn(x1 * cx.x + x0 * cx.y);
-        }
-        for (int c = lane; c < D / 8; c += 32)
-          *reinterpret_cast<uint4 *>(vt + tile_offset<D>(row, c)) =
-              *reinterpret_cast<const uint4 *>(seg + sb.v_off() + c * 16);
       }
       if (patch) __syncwarp();
       const uint32_t kbase = smem_u32(kt), vbase = smem_u32(vt);
@@ -730,7 +695,9 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     const int64_t X0 = (int64_t)Hkv * cum[b] + (int64_t)g * nch;
     const int first = plan_owner(W, C, X0), last = plan_owner(W, C, X0 + nch - 1);
     const int64_t obase = (int64_t)seg * G * D;
-    if (first == last) {  // the whole segment is ours: normalise and store
+    // The whole segment is ours: normalise and store (fused step: the combine kernel still has
+    // to add the appended slot, so the state always goes to the partials).
+    if (!kStep && first == last) {
       // (a segment whose only slot was a refused append has l = 0: its output is 0)
       const float i0 = l0 > 0.f ? 1.f / l0 : 0.f, i1 = l1 > 0.f ? 1.f / l1 : 0.f;
 #pragma unroll
@@ -780,13 +747,14 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
 // head's (max, sum), and for the fused step they are the pair that RoPE turns together.
 // Blocks of kCombineThreads cover one segment's G*D/2 pairs (whole heads).
 //
-// For the fused step the same threads also commit the append, once the whole attention grid
-// has finished (every CTA reads the counters in its prologue): thread (h = 0, i) stores
-// elements i and i + D/2 of the new key and value rows, thread (h, i) those of head h of
-// q_rot (if asked), each the fp64 rotation of the pair rounded once to bf16, as
-// ham_kv_append computes it; KV head 0 writes the slot metadata and advances the counters.
-// The commit's chain (append record -> cos/sin and page) and the merge's (segment range ->
-// partials) are issued together.
+// Fused step: the attention pass covered the stored slots only; the appended slot enters
+// here, once the whole pass has finished (every CTA reads the counters in its prologue), as
+// one more term of the merge: score q.k / sqrt(d) with q and the new key turned by the new
+// position in fp32 and rounded to bf16 as in the pass, weight 1, value v_new.  The same
+// threads commit the append: thread (h = 0, i) stores elements i and i + D/2 of the new key
+// and value rows, thread (h, i) those of head h of q_rot (if asked), each the fp64 rotation of
+// the pair rounded once to bf16, as ham_kv_append computes it; KV head 0 writes the slot
+// metadata and advances the counters.
 // ------------------------------------------------------------------------------------
 constexpr int kCombineThreads = 128;
 static_assert(kCombineThreads % 64 == 0, "a block holds whole heads of head_dim 64 or 128");
@@ -812,23 +780,21 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   uint16_t q0 = 0, q1 = 0, k0 = 0, k1 = 0, v0 = 0, v1 = 0;
   double c = 1.0, sn = 0.0;
   int page = -1;
+  bool app = false;
   if constexpr (kStep) {
     const StepArgs &st = v.step;
     const int b = seg / Hkv;
     rec = st.stash[b];  // (n, 0 or the error that stops the append, position, ntok)
+    app = rec.y == 0;
     if (active) {
-      if (st.q_rot) {
-        q0 = v.q[orow + i];
-        q1 = v.q[orow + i + half];
-      }
-      if (h == 0) {
-        k0 = st.k_new[(int64_t)seg * D + i];
-        k1 = st.k_new[(int64_t)seg * D + i + half];
-        v0 = st.v_new[(int64_t)seg * D + i];
-        v1 = st.v_new[(int64_t)seg * D + i + half];
-      }
+      q0 = v.q[orow + i];
+      q1 = v.q[orow + i + half];
+      k0 = st.k_new[(int64_t)seg * D + i];
+      k1 = st.k_new[(int64_t)seg * D + i + half];
+      v0 = st.v_new[(int64_t)seg * D + i];
+      v1 = st.v_new[(int64_t)seg * D + i + half];
     }
-    if (rec.y == 0 && active && (h == 0 || st.q_rot)) {
+    if (app && active) {
       const int64_t p = rec.z;
       if (p >= 0 && p < st.rope_positions) {
         const double2 e = st.rope_table[p * half + i];
@@ -841,12 +807,13 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
     }
   }
 
-  if (active && r.x >= 0 && r.x != r.y) {
-    // Online merge in batches of 8 partials, whose loads are in flight together.  (16 saved
-    // one round trip at 8-12 partials per segment but cost registers: fewer resident blocks
-    // when a ragged batch has thousands of segments.)
+  // Online merge in batches of 8 partials, whose loads are in flight together.  (16 saved one
+  // round trip at 8-12 partials per segment but cost registers: fewer resident blocks when a
+  // ragged batch has thousands of segments.)
+  const bool merge = r.x >= 0 && (kStep || r.x != r.y);
+  float M = -INFINITY, num0 = 0.f, num1 = 0.f, den = 0.f;
+  if (active && merge) {
     constexpr int kBatch = 8;
-    float M = -INFINITY, num0 = 0.f, num1 = 0.f, den = 0.f;
     for (int k0b = r.x; k0b <= r.y; k0b += kBatch) {
       float2 ml[kBatch];
       float a0[kBatch], a1[kBatch];
@@ -875,16 +842,49 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       }
       M = bm;
     }
-    const float inv = den > 0.f ? 1.f / den : 0.f;  // 0: every slot masked (refused append)
-    store_out<OutT>(v.out, orow + i, num0 * inv);
-    store_out<OutT>(v.out, orow + i + half, num1 * inv);
   }
 
   if constexpr (kStep) {
+    // Score of the appended slot for head h: the pair's share of q.k, summed over the D/2
+    // threads of the head (one warp at d = 64, two at d = 128, whose sums meet in shared
+    // memory).  Every thread of the block takes part, so no thread has left yet.
+    __shared__ float head_sum[kCombineThreads / 32];
+    float share = 0.f;
+    if (app && active) {
+      const float cf = (float)c, sf = (float)sn;
+      const float x0 = bf16_bits_to_float(q0), x1 = bf16_bits_to_float(q1);
+      const float y0 = bf16_bits_to_float(k0), y1 = bf16_bits_to_float(k1);
+      const float qr0 = __bfloat162float(__float2bfloat16_rn(x0 * cf - x1 * sf));
+      const float qr1 = __bfloat162float(__float2bfloat16_rn(x1 * cf + x0 * sf));
+      const float kr0 = __bfloat162float(__float2bfloat16_rn(y0 * cf - y1 * sf));
+      const float kr1 = __bfloat162float(__float2bfloat16_rn(y1 * cf + y0 * sf));
+      share = qr0 * kr0 + qr1 * kr1;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) share += __shfl_xor_sync(kFull, share, off);
+    const int warp = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) head_sum[warp] = share;
+    __syncthreads();
+    const float dot = half > 32 ? head_sum[warp & ~1] + head_sum[warp | 1] : head_sum[warp];
+    if (app && active) {
+      const float x = dot * (rsqrtf((float)D) * 1.4426950408889634f);  // log2 domain
+      const float bm = fmaxf(M, x);
+      const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
+      const float w = ex2(x - bm);
+      num0 = num0 * scale + w * bf16_bits_to_float(v0);
+      num1 = num1 * scale + w * bf16_bits_to_float(v1);
+      den = den * scale + w;
+    }
+    if (active && (merge || app)) {
+      const float inv = den > 0.f ? 1.f / den : 0.f;
+      store_out<OutT>(v.out, orow + i, num0 * inv);
+      store_out<OutT>(v.out, orow + i + half, num1 * inv);
+    }
+
     const StepArgs &st = v.step;
     const int b = seg / Hkv, g = seg - b * Hkv;
     const bool lead = g == 0 && idx == 0;  // one thread per sequence
-    if (rec.y) {                           // no append for this sequence
+    if (!app) {                            // no append for this sequence
       if (lead) record_error(v.err, rec.y);
       return;
     }
@@ -912,6 +912,12 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       st.slot_ntok[meta] = rec.w;
       st.num_slots[b] = n + 1;
       st.num_tokens[b] += rec.w;
+    }
+  } else {
+    if (active && merge) {
+      const float inv = den > 0.f ? 1.f / den : 0.f;  // 0: every slot masked
+      store_out<OutT>(v.out, orow + i, num0 * inv);
+      store_out<OutT>(v.out, orow + i + half, num1 * inv);
     }
   }
 }

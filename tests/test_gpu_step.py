@@ -20,9 +20,11 @@ pytestmark = pytest.mark.gpu
 # error <= 2^-9), which moves an output by at most 2^-9 * max|v_i - v_j| (~1.6e-2 for unit
 # normal values); on sequences of a few slots nothing averages it out, so the bar is the
 # bf16 one (MAX_ABS, MEAN_ABS) even with fp32 output.  GPU against GPU with the same split:
-# the same weights are rounded the same way, so only a rare one-ulp difference of an
-# fp32-rotated q or k element separates the fused step from the two separate calls.
-SAME_SPLIT_MAX, SAME_SPLIT_MEAN = 2e-3, 2e-5
+# the stored slots' weights are rounded the same way; what differs is the appended slot,
+# whose weight the fused step keeps in fp32 (the two calls round it to bf16 in the MMA), and a
+# rare one-ulp difference of an fp32-rotated q element.  That moves an output by at most
+# 2^-9 * w_new / sum(w) * |v|, small against the bf16 bar.
+SAME_SPLIT_MAX, SAME_SPLIT_MEAN = 2e-3, 1e-4
 Q_ROT_UNWRITTEN = 0x7FC1  # a bf16 NaN pattern no rotation produces
 
 
