@@ -781,10 +781,12 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   double c = 1.0, sn = 0.0;
   int page = -1;
   bool app = false;
+  int64_t tokens = 0;  // lead thread: the sequence's token count before the step
   if constexpr (kStep) {
     const StepArgs &st = v.step;
     const int b = seg / Hkv;
     rec = st.stash[b];  // (n, 0 or the error that stops the append, position, ntok)
+    if (idx == 0 && seg - b * Hkv == 0) tokens = st.num_tokens[b];
     app = rec.y == 0;
     if (active) {
       q0 = v.q[orow + i];
@@ -806,7 +808,6 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
     }
   }
-
   // Online merge in batches of 8 partials, whose loads are in flight together.  (16 saved one
   // round trip at 8-12 partials per segment but cost registers: fewer resident blocks when a
   // ragged batch has thousands of segments.)
@@ -841,6 +842,24 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
         den += w * ml[j].y;
       }
       M = bm;
+    }
+  }
+
+  // fused step: the exact (fp64) rotations it commits (cos/sin were loaded before the merge,
+  // whose loads are therefore not held up by them)
+  uint16_t qc0 = 0, qc1 = 0, kc0 = 0, kc1 = 0;
+  if constexpr (kStep) {
+    if (app && active) {
+      if (v.step.q_rot) {
+        const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
+        qc0 = rotate_elem(x0, x1, c, sn, false);
+        qc1 = rotate_elem(x1, x0, c, sn, true);
+      }
+      if (h == 0) {
+        const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
+        kc0 = rotate_elem(x0, x1, c, sn, false);
+        kc1 = rotate_elem(x1, x0, c, sn, true);
+      }
     }
   }
 
@@ -890,9 +909,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
     }
     if (!active) return;
     if (st.q_rot) {
-      const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
-      st.q_rot[orow + i] = rotate_elem(x0, x1, c, sn, false);
-      st.q_rot[orow + i + half] = rotate_elem(x1, x0, c, sn, true);
+      st.q_rot[orow + i] = qc0;
+      st.q_rot[orow + i + half] = qc1;
     }
     if (h != 0) return;
     if (page < 0 || page >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE
@@ -901,9 +919,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
     }
     const int n = rec.x;
     const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
-    const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
-    st.k_pool[row + i] = rotate_elem(x0, x1, c, sn, false);
-    st.k_pool[row + i + half] = rotate_elem(x1, x0, c, sn, true);
+    st.k_pool[row + i] = kc0;
+    st.k_pool[row + i + half] = kc1;
     st.v_pool[row + i] = v0;
     st.v_pool[row + i + half] = v1;
     if (lead) {
@@ -911,7 +928,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       st.slot_pos[meta] = rec.z;
       st.slot_ntok[meta] = rec.w;
       st.num_slots[b] = n + 1;
-      st.num_tokens[b] += rec.w;
+      st.num_tokens[b] = tokens + rec.w;
     }
   } else {
     if (active && merge) {
