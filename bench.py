@@ -340,35 +340,44 @@ def run_ours(args, w):
         rollback()
     stream.synchronize()
 
+    name = "ham_decode_step" if fused else "ham_decode_attn"
     try:
+        span = (torch.cuda.Event(enable_timing=True, external=True),
+                torch.cuda.Event(enable_timing=True, external=True))
         ev = [(torch.cuda.Event(enable_timing=True, external=True),
                torch.cuda.Event(enable_timing=True, external=True)) for _ in range(GRAPH_STEPS)]
-        per_launch_method = (("CUDA events around every ham_decode_step (attention + "
-                              "combine/commit kernels)" if fused else
-                              "CUDA events around every ham_decode_attn (attention + combine "
-                              "kernels)") + " of the last graph replay of the timed region")
+        per_launch_method = (f"CUDA events before and after the {GRAPH_STEPS} consecutive {name} "
+                             "calls of the last graph replay of the timed region (on the launching "
+                             f"stream; programmatic dependent launch intact between them), / "
+                             f"{GRAPH_STEPS}")
     except TypeError:
-        ev = None
-        per_launch_method = "attention-only graph, CUDA events around the replay"
+        span, ev = None, None
+        per_launch_method = "timed region / steps (events inside graphs unavailable)"
 
-    def capture(with_events):
+    def capture(events):
+        """events: None, "span" (around the steps, before the rollback) or "each" (around
+        every step; that stops consecutive launches from overlapping)."""
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
+            if events == "span":
+                span[0].record()
             for i in range(GRAPH_STEPS):
                 c = caches[i % CACHES]
                 append_part(c)
-                if with_events:
+                if events == "each":
                     ev[i][0].record()
                 timed_part(c)
-                if with_events:
+                if events == "each":
                     ev[i][1].record()
+            if events == "span":
+                span[1].record()
             rollback()
         return g
 
-    # the timed loop replays an event-free graph (events would cut the programmatic
-    # dependent launch between kernels); the last replay is an identical graph with events
-    graph = capture(False)
-    probe = capture(True) if ev is not None else graph
+    # the timed loop replays an event-free graph; the last replay is an identical graph with
+    # events around its steps only (none between them)
+    graph = capture(None)
+    probe = capture("span") if span is not None else graph
     # fused: attention + combine/commit; split: append, attention, combine; then rollbacks
     launches_per_graph = (2 if fused else 3) * GRAPH_STEPS + CACHES
 
@@ -376,7 +385,7 @@ def run_ours(args, w):
     counts_h = base_counts(w)
     attn_bytes_graph = sum(attn_bytes(w, counts_h + 1 + i // CACHES) for i in range(GRAPH_STEPS))
     step_bytes_graph = attn_bytes_graph + GRAPH_STEPS * append_bytes(w)
-    timed_bytes_graph = step_bytes_graph if fused else attn_bytes_graph
+    timed_bytes_graph = step_bytes_graph  # the span covers the whole step on both paths
 
     with torch.cuda.stream(stream):          # replay() launches on the current stream
         for _ in range(n_warm):
@@ -403,23 +412,20 @@ def run_ours(args, w):
     if world > 1:
         torch.distributed.barrier()
 
-    # attention kernel duration (last replay of the timed region)
-    if ev is not None:
-        attn_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(GRAPH_STEPS)]
+    # the timed kernels' average duration in the loop (last replay of the timed region)
+    if span is not None:
+        attn_ms = [span[0].elapsed_time(span[1]) / GRAPH_STEPS] * GRAPH_STEPS
     else:
-        g2 = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g2, stream=stream):
-            for i in range(GRAPH_STEPS):
-                c = caches[i % CACHES]
-                one_step(c)
-            rollback()
-        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        attn_ms = [elapsed_ms / steps] * GRAPH_STEPS
+    # and, after the timed region, the same launches one at a time (events around each)
+    isolated_us = None
+    if ev is not None:
+        each = capture("each")
         with torch.cuda.stream(stream):
-            a0.record(stream)
-            g2.replay()
-            a1.record(stream)
+            each.replay()
         torch.cuda.synchronize()
-        attn_ms = [a0.elapsed_time(a1) / GRAPH_STEPS] * GRAPH_STEPS
+        isolated_us = round(1e3 * statistics.mean(ev[i][0].elapsed_time(ev[i][1])
+                                                  for i in range(GRAPH_STEPS)), 3)
     for c in caches:
         if ham.ham_kv_status(c["kv"]) != ham.HAM_DEVERR_NONE:
             raise RuntimeError("device error during the timed region")
@@ -447,9 +453,10 @@ def run_ours(args, w):
         "roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(attn_gbs / peak, 4), "traffic": traffic,
                      "kernel": ("decode_attn_kernel<128,bf16,step> + combine_kernel<bf16,step>"
-                                if fused else
-                                "decode_attn_kernel<128,bf16> + combine_kernel<bf16>"),
+                                if fused else "append_kernel + decode_attn_kernel<128,bf16> + "
+                                "combine_kernel<bf16>"),
                      "avg_launch_us": round(1e3 * statistics.mean(attn_ms), 3),
+                     "isolated_launch_us": isolated_us,
                      "algorithmic_bytes_per_launch": int(timed_bytes_graph / GRAPH_STEPS),
                      "peak_source": peak_src, "duration_method": per_launch_method},
         "gpu_launches": n_graph * launches_per_graph * world,
