@@ -194,14 +194,18 @@ class ClockSampler:
 # workload
 # ---------------------------------------------------------------------------------------
 
+STACK_PREFIX = "stack_b"     # stack_b1, stack_b8, ...: the 32-layer decode stack
+STACK_GRAPH = 8              # macro-steps per CUDA graph in the stack runs
+
+
 def workload(name):
     from paper_2505_20438_gb300 import workload as wl
+    if name.startswith(STACK_PREFIX) and name[len(STACK_PREFIX):].isdigit():
+        return wl.c4_sweep(int(name[len(STACK_PREFIX):]))
     if name not in wl.WORKLOADS:
-        raise SystemExit(f"unknown workload {name}; choose from {sorted(wl.WORKLOADS)}")
-    w = wl.WORKLOADS[name]
-    if w.layers != 1:
-        raise SystemExit(f"bench times single-layer workloads; {name} has {w.layers} layers")
-    return w
+        raise SystemExit(f"unknown workload {name}; choose from {sorted(wl.WORKLOADS)} or "
+                         f"{STACK_PREFIX}<batch>")
+    return wl.WORKLOADS[name]
 
 
 def base_counts(w):
@@ -582,14 +586,14 @@ def run_reference(args, w):
     # sub-case of the workload: fewer sequences, or one sequence with fewer slots, sized so
     # the whole run is about 40 full macro-steps of oracle work.  Attention work is linear
     # in the slot count, so the value is scaled by the sampled fraction of slots.
-    total = int(base_counts(w).sum())          # slots attended by one full macro-step
+    total = int(base_counts(w).sum())          # slots attended by one layer's step
     mean_l = max(1, total // w.batch)
     frac = min(1.0, 40.0 / (steps + warm))
     if frac * w.batch >= 1.0:
         sub_b, sub_l = max(1, int(round(frac * w.batch))), mean_l
     else:
         sub_b, sub_l = 1, max(16, int(round(frac * total)))
-    sub = dataclasses.replace(w, batch=sub_b, slots=sub_l, slot_range=None)
+    sub = dataclasses.replace(w, batch=sub_b, slots=sub_l, slot_range=None, layers=1)
     case = wl.make_case(sub, extra_slots=4)
     oc = oracle.OracleCache.from_case(case)
     def one():
@@ -603,7 +607,7 @@ def run_reference(args, w):
     for _ in range(steps):
         one()
     dt = time.perf_counter() - t0
-    share = (sub_b * sub_l) / total
+    share = (sub_b * sub_l) / total / w.layers  # a macro-step runs every layer
     value = steps * share / dt
     sample = (f"each step: append + attention of all heads for {sub_b} sequence(s) x {sub_l} "
               f"slots = {share:.4f} of a {w.name} macro-step; {steps} steps timed")
@@ -619,11 +623,196 @@ def run_reference(args, w):
     }), flush=True)
 
 
+def run_stack(args, w):
+    """The decode stack: every macro-step runs ham_decode_step on each of the w.layers layers
+    (one cache, one layer after the other, as a decoder does), STACK_GRAPH macro-steps per CUDA
+    graph, then the layers are rolled back to their starting slot counts."""
+    import numpy as np
+    import torch
+
+    from paper_2505_20438_gb300 import build as build_mod
+    from paper_2505_20438_gb300 import ham
+    from paper_2505_20438_gb300 import workload as wl
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    build_mod.build()
+    B, L, layers = w.batch, w.slots, w.layers
+    seed = rank_cache_seed(w.seed, rank, 0)
+    max_slots = L + STACK_GRAPH + 16
+    kv = ham.ham_kv_alloc(layers, B, w.n_q_heads, w.n_kv_heads, w.head_dim, w.page_slots,
+                          max_slots, page_seed=seed + 1)
+    rng = wl.rng_for(seed, 5)
+    ntok_fill = wl.ntok_capped_geometric(rng, (B, L))
+    counts = torch.full((B,), L, dtype=torch.int32, device="cuda")
+    tokens = torch.from_numpy(ntok_fill.sum(axis=1).astype(np.int64)).cuda()
+    ntok_fill_dev = torch.from_numpy(ntok_fill).cuda()
+    for layer in range(layers):
+        k = wl.device_normal_bf16((B, L, w.n_kv_heads, w.head_dim), w.value_scale,
+                                  seed * 1000 + 10 * layer + 1)
+        v = wl.device_normal_bf16((B, L, w.n_kv_heads, w.head_dim), w.value_scale,
+                                  seed * 1000 + 10 * layer + 2)
+        ham.ham_kv_fill(kv, layer, k, v, counts, ntok=ntok_fill_dev)
+        del k, v
+    shape_q, shape_kv = (B, w.n_q_heads, w.head_dim), (B, w.n_kv_heads, w.head_dim)
+    q = [wl.device_normal_bf16(shape_q, w.value_scale, seed * 7 + 100 + l) for l in range(layers)]
+    k_new = [wl.device_normal_bf16(shape_kv, w.value_scale, seed * 7 + 200 + l)
+             for l in range(layers)]
+    v_new = [wl.device_normal_bf16(shape_kv, w.value_scale, seed * 7 + 300 + l)
+             for l in range(layers)]
+    ntok_new = torch.from_numpy(wl.ntok_capped_geometric(rng, (B,))).cuda()
+    out = [torch.empty(shape_q, dtype=torch.bfloat16, device="cuda") for _ in range(layers)]
+    stream = torch.cuda.Stream()
+
+    def macro_step():
+        for l in range(layers):
+            ham.ham_decode_step(kv, l, q[l], k_new[l], v_new[l], None, ntok_new, out[l])
+
+    def rollback():
+        for l in range(layers):
+            ham.ham_kv_set_lengths(kv, l, counts, tokens)
+
+    with torch.cuda.stream(stream):
+        macro_step()
+        rollback()
+    stream.synchronize()
+    span = (torch.cuda.Event(enable_timing=True, external=True),
+            torch.cuda.Event(enable_timing=True, external=True))
+
+    def capture(with_span):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            if with_span:
+                span[0].record()
+            for _ in range(STACK_GRAPH):
+                macro_step()
+            if with_span:
+                span[1].record()
+            rollback()
+        return g
+
+    graph, probe = capture(False), capture(True)
+    # a macro-step runs every layer: at most 1024 of them keep the run within a minute or so
+    n_graph = max(1, math.ceil(min(args.steps, 1024) / STACK_GRAPH))
+    n_warm = max(1, math.ceil(max(args.warmup, 3) / STACK_GRAPH))
+    steps = n_graph * STACK_GRAPH
+    with torch.cuda.stream(stream):
+        for _ in range(n_warm):
+            graph.replay()
+    torch.cuda.synchronize()
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error during warm-up")
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks, torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(n_graph - 1):
+            graph.replay()
+        probe.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed_ms = max_over_ranks(t0.elapsed_time(t1), world, "cuda")
+    if world > 1:
+        torch.distributed.barrier()
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error during the timed region")
+    counts_h = np.full(B, L)
+    macro_bytes = layers * statistics.mean(attn_bytes(w, counts_h + 1 + m) + append_bytes(w)
+                                           for m in range(STACK_GRAPH))
+    span_us = 1e3 * span[0].elapsed_time(span[1]) / STACK_GRAPH
+    peak, peak_src = measured_peak_hbm()
+    value = job_throughput(steps, world, elapsed_ms * 1e-3)
+    ms_per_step = elapsed_ms / steps
+    achieved = macro_bytes / (span_us * 1e-6) / 1e9
+
+    # end to end through the public API: every macro-step copies each layer's q, k_new, v_new
+    # from pinned host memory, runs the stack eagerly and reads the last layer's output back
+    host = {"q": [x.cpu().pin_memory() for x in q], "k": [x.cpu().pin_memory() for x in k_new],
+            "v": [x.cpu().pin_memory() for x in v_new]}
+    host_out = torch.empty(shape_q, dtype=torch.bfloat16).pin_memory()
+    h2d = layers * sum(x[0].numel() * x[0].element_size() for x in host.values())
+    d2h = host_out.numel() * host_out.element_size()
+    n_e2e = max(STACK_GRAPH, min(args.e2e_steps, 64) // STACK_GRAPH * STACK_GRAPH)
+    checksum = 0.0
+    with torch.cuda.stream(stream):
+        rollback()
+        stream.synchronize()
+        te = time.perf_counter()
+        for i in range(n_e2e):
+            for l in range(layers):
+                q[l].copy_(host["q"][l], non_blocking=True)
+                k_new[l].copy_(host["k"][l], non_blocking=True)
+                v_new[l].copy_(host["v"][l], non_blocking=True)
+            macro_step()
+            host_out.copy_(out[-1], non_blocking=True)
+            stream.synchronize()
+            checksum += float(host_out[0, 0, 0])
+            if (i + 1) % STACK_GRAPH == 0:
+                rollback()
+        stream.synchronize()
+        dte = time.perf_counter() - te
+    dte = max_over_ranks(dte, world, "cuda")
+
+    mean_ntok = float(ntok_fill.mean())
+    result = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+        "steps": steps, "warmup": n_warm * STACK_GRAPH, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "accum_dtype": "f32", "data": "synthetic",
+        "config": {"workload": w.name, "layers": layers, "batch": B, "n_q_heads": w.n_q_heads,
+                   "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+                   "slots": f"{L} at the start of each graph, +1 per macro-step",
+                   "page_slots": w.page_slots,
+                   "pages": "scattered by a seeded shuffle of the pool",
+                   "tokens_per_slot": "geometric p=0.5 capped at 4",
+                   "step": f"one macro-step: ham_decode_step on each of the {layers} layers",
+                   "l2": f"{layers} layers of KV ({layers * B * L * w.n_kv_heads * w.head_dim * 4 / 2**20:.0f} MiB) > 129 MB L2",
+                   "graph": f"{STACK_GRAPH} macro-steps per CUDA graph, then every layer is "
+                            "rolled back"},
+        "kv_gbs": round(macro_bytes * value / 1e9, 1),
+        "kv_frac_of_measured_peak": round(macro_bytes * value / world / 1e9 / peak, 4),
+        "slots_per_s": round(value * B, 1),
+        "tokens_per_s": round(value * B * mean_ntok, 1),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": None,
+                     "kernel": "decode_attn_kernel<128,bf16,step> + combine_kernel<bf16,step>, "
+                               f"{layers} layers",
+                     "avg_launch_us": round(span_us / layers, 3),
+                     "algorithmic_bytes_per_launch": int(macro_bytes / layers),
+                     "peak_source": peak_src,
+                     "duration_method": f"CUDA events around the {STACK_GRAPH} macro-steps of the "
+                                        f"last graph replay, / ({STACK_GRAPH} x {layers})"},
+        "gpu_launches": n_graph * (STACK_GRAPH * layers * 2 + layers) * world,
+        "e2e": {"value": round(job_throughput(n_e2e, world, dte), 2), "unit": UNIT,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e,
+                "finite": math.isfinite(checksum)},
+        "clocks": clocks.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import dataclasses
+        one = cpu_baseline(dataclasses.replace(w, layers=1), args.cpu_seconds)
+        one["value"] = round(one["value"] / layers, 4)
+        one["single_thread_value"] = round(one["single_thread_value"] / layers, 4)
+        one["sample"] += f"; one layer's steps, divided by {layers} layers"
+        result["cpu_baseline"] = one
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
 def main():
     args = parse_args()
     w = workload(args.workload)
     if args.impl == "reference":
         run_reference(args, w)
+    elif w.layers > 1:
+        run_stack(args, w)
     else:
         run_ours(args, w)
 

@@ -19,14 +19,17 @@ constexpr int kMaxBatch = 4096;
 
 // ---------------------------------------------------------------------------------------
 // Split plan.  The chunks of all (sequence b, KV head g) segments are numbered b-major,
-// then g, then chunk index; W is their total.  Of the launched CTAs, C = min(launched, W)
-// take part and CTA c < C takes chunks [floor(c W / C), floor((c+1) W / C)), never empty
-// because W >= C.  So the CTAs touching a segment are exactly owner(first chunk) ..
+// then g, then chunk index; W is their total.  Of the launched CTAs, C = min(launched,
+// ceil(W / kMinChunksPerCta)) take part (a small problem spread over every CTA would leave
+// each a chunk or two and every segment dozens of partials to merge) and CTA c < C takes
+// chunks [floor(c W / C), floor((c+1) W / C)), never empty because W >= C.  So the CTAs touching a segment are exactly owner(first chunk) ..
 // owner(last chunk).  A CTA writes one partial per segment it touches, at index c + s,
 // which is unique because (c, s) only ever grows along the chunk order.
 // ---------------------------------------------------------------------------------------
+constexpr int kMinChunksPerCta = 8;
 __host__ __device__ inline int32_t plan_ctas(int64_t W, int32_t launched) {
-  return (int32_t)(W < (int64_t)launched ? W : (int64_t)launched);
+  const int64_t want = (W + kMinChunksPerCta - 1) / kMinChunksPerCta;
+  return (int32_t)(want < (int64_t)launched ? want : (int64_t)launched);
 }
 __host__ __device__ inline int64_t plan_cta_begin(int64_t W, int32_t C, int64_t c) {
   return (W * c) / C;

@@ -14,6 +14,13 @@ from gpu_helpers import (MAX_ABS, MEAN_ABS, assert_parity, dev_bf16, dev_i32, gp
 
 pytestmark = pytest.mark.gpu
 
+# fp32 output: a tighter check than the bf16 bar.  The tensor-core p.V rounds each softmax
+# weight to bf16 (relative error up to 2^-9, about uniform), so an output moves by a weighted
+# sum of such errors times (v_i - out): of order 1e-3 at worst on concentrated weights, and
+# of order 1e-4 on average over a few hundred slots.  The exact value depends on how the
+# split plan cuts the segments, which changes the running maxima the weights are taken from.
+F32_MAX, F32_MEAN = 3e-3, 3e-4
+
 
 @pytest.mark.parametrize("hq,hkv,d,page,counts,scale", [
     (8, 2, 64, 16, (37, 80), 1.0),                    # ragged tails inside a chunk
@@ -35,7 +42,7 @@ def test_decode_matches_oracle(hq, hkv, d, page, counts, scale):
     out32 = gpu_decode(kv, case.q, f32=True)
     out16 = gpu_decode(kv, case.q, f32=False)
     assert_parity(out16, ref, what="bf16 out")
-    assert_parity(out32, ref, max_abs=2e-3, mean_abs=2e-4, what="f32 out")
+    assert_parity(out32, ref, max_abs=F32_MAX, mean_abs=F32_MEAN, what="f32 out")
     for b, n in enumerate(counts):                     # empty sequences give exactly 0
         if n == 0:
             assert np.all(out16[b] == 0) and np.all(out32[b] == 0)
@@ -49,7 +56,7 @@ def test_split_count_invariance(ctas):
     kv = gpu_cache(case)
     ham.ham_kv_set_attn_ctas(kv, ctas)
     out = gpu_decode(kv, case.q, f32=True)
-    assert_parity(out, ref, max_abs=2e-3, mean_abs=2e-4, what=f"ctas={ctas}")
+    assert_parity(out, ref, max_abs=F32_MAX, mean_abs=F32_MEAN, what=f"ctas={ctas}")
 
 
 def test_repeated_launches_reuse_tickets():
@@ -87,7 +94,7 @@ def test_special_cases():
         case.k[0, j, 0] = wl.f32_to_bf16_bits((q * (score * np.sqrt(128) / (q @ q))).astype(np.float32))
     ref = oracle.OracleCache.from_case(case).decode_attn(case.q)
     out = gpu_decode(gpu_cache(case), case.q, f32=True)
-    assert_parity(out, ref, max_abs=2e-3, mean_abs=2e-4, what="planted")
+    assert_parity(out, ref, max_abs=F32_MAX, mean_abs=F32_MEAN, what="planted")
     v = wl.bf16_bits_to_f32(case.v[0, 2999, 0]).astype(np.float64)
     assert np.allclose(out[0, 0], v, atol=1e-3)
 
@@ -117,7 +124,7 @@ def test_tiny_workload_step_matches_fixture():
     got = out.cpu().numpy().astype(np.float64)
     lines = open(os.path.join(here, "tiny_step_oracle.txt")).read().splitlines()
     ref = np.array([float(l) for l in lines if not l.startswith("#")]).reshape(got.shape)
-    assert_parity(got, ref, max_abs=2e-3, mean_abs=2e-4, what="tiny step")
+    assert_parity(got, ref, max_abs=F32_MAX, mean_abs=F32_MEAN, what="tiny step")
     slots, tokens = ham.ham_slot_lengths(kv)
     ref_out, oc = make_golden.tiny_step()
     assert list(slots) == [256] and list(tokens) == list(oc.num_tokens)
