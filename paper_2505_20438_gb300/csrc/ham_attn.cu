@@ -445,7 +445,6 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
                         : bad ? HAM_DEVERR_SLOTS
                         : L == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
         appb[b] = why == 0;
-        if (blockIdx.x == 0) v.step.stash[b] = make_int4(L, why, posb[b], t);
       }
     }
   }
@@ -742,62 +741,117 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
 
 // ------------------------------------------------------------------------------------
 // Combine: out[seg][h][d] = sum_k 2^(m_k - M) acc_k[h][d] / sum_k 2^(m_k - M) l_k over the
-// CTAs k = first..last of the segment, M = max_k m_k (split-softmax merge, in CTA order).
-// One thread per pair of elements (h, i) and (h, i + D/2) of an output row: both share the
-// head's (max, sum), and for the fused step they are the pair that RoPE turns together.
-// Blocks of kCombineThreads cover one segment's G*D/2 pairs (whole heads).
+// CTAs k = first..last of the segment, M = max_k m_k (split-softmax merge, in CTA order, in
+// batches of kBatch partials whose loads are in flight together).  One thread per pair of
+// elements (h, i) and (h, i + D/2) of an output row: both share the head's (max, sum), and for
+// the fused step they are the pair that RoPE turns together.  Blocks of kCombineThreads cover
+// one segment's G*D/2 pairs (whole heads).
 //
-// Fused step: the attention pass covered the stored slots only; the appended slot enters
-// here, once the whole pass has finished (every CTA reads the counters in its prologue), as
-// one more term of the merge: score q.k / sqrt(d) with q and the new key turned by the new
-// position in fp32 and rounded to bf16 as in the pass, weight 1, value v_new.  The same
-// threads commit the append: thread (h = 0, i) stores elements i and i + D/2 of the new key
-// and value rows, thread (h, i) those of head h of q_rot (if asked), each the fp64 rotation of
-// the pair rounded once to bf16, as ham_kv_append computes it; KV head 0 writes the slot
-// metadata and advances the counters.
+// The kernel is scheduled (programmatic dependent launch) once every attention CTA has passed
+// its own dependency wait, and then idles until the attention grid ends.  So everything that
+// does not depend on the attention grid runs before this kernel's wait:
+//  * the segment's CTA range first..last, from the slot counters with the attention's split
+//    plan (small batches; larger ones read the range the attention's first CTA stored);
+//  * fused step: the append record of the sequence (slot n, the error that stops the append,
+//    position, tokens), read from the counters and caller inputs as the attention pass reads
+//    them; the fp64 rotation of q (q_rot) and of the new key, rounded once to bf16 as
+//    ham_kv_append computes them, and the new slot's rows (KV head g's threads of head 0);
+//    the new slot's score for head h: q.k / sqrt(d) with q and the new key turned by the new
+//    position in fp32 and rounded to bf16 as in the pass, summed over the D/2 threads of the
+//    head.  None of these is read by the attention pass: it covers the stored slots only, and
+//    the rows of slot n that its last chunk copies are masked there.
+// After the wait: the merge, the appended slot as one more term (weight 2^(score - M'), value
+// v_new), the output, and (KV head 0's lead thread) the slot metadata and the counters, which
+// every attention CTA has read by then.
 // ------------------------------------------------------------------------------------
 constexpr int kCombineThreads = 128;
+constexpr int kCombinePlanBatch = kCombineThreads;  // batches whose plan the combine computes
 static_assert(kCombineThreads % 64 == 0, "a block holds whole heads of head_dim 64 or 128");
 
-template <typename OutT, bool kStep>
+template <typename OutT, bool kStep, int kBatch>
 __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView v, int D,
                                                                   int blocks_per_seg) {
-  const int G = v.group, Hkv = v.n_kv_heads, half = D / 2;
+  const int G = v.group, Hkv = v.n_kv_heads, half = D / 2, B = v.batch;
   const int seg = blockIdx.x / blocks_per_seg;
   const int part = blockIdx.x % blocks_per_seg;
-  const int idx = part * kCombineThreads + threadIdx.x;  // pair index within the segment
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int idx = part * kCombineThreads + tid;  // pair index within the segment
   const bool active = idx < G * half;
   const int h = idx / half, i = idx - h * half;
+  const int b = seg / Hkv, g = seg - b * Hkv;
   const int64_t orow = ((int64_t)seg * G + h) * D;  // row (b, g*G + h) of q / q_rot / out
 
-  grid_dependency_wait();  // the attention grid's partials, ranges and append records
-  // The next kernel may be scheduled now; its own dependency wait still covers this grid.
-  grid_launch_dependents();
+  // ---- before the wait: the segment's CTA range (split plan, as the attention computes it)
+  int first = -1, last = -1;
+  const bool planned = B <= kCombinePlanBatch;
+  if (planned) {
+    __shared__ int red[3][kCombineThreads / 32];
+    int n = 0;
+    if (tid < B) {
+      int L = v.num_slots[tid];
+      L = L < 0 ? 0 : (L > v.max_slots ? v.max_slots : L);
+      n = chunks_of(L);
+    }
+    int tot = n, pre = tid < b ? n : 0, own = tid == b ? n : 0;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      tot += __shfl_xor_sync(kFull, tot, off);
+      pre += __shfl_xor_sync(kFull, pre, off);
+      own += __shfl_xor_sync(kFull, own, off);
+    }
+    if (lane == 0) {
+      red[0][warp] = tot;
+      red[1][warp] = pre;
+      red[2][warp] = own;
+    }
+    __syncthreads();
+    int T = 0, P = 0, N = 0;
+#pragma unroll
+    for (int w = 0; w < kCombineThreads / 32; ++w) {
+      T += red[0][w];
+      P += red[1][w];
+      N += red[2][w];
+    }
+    if (N > 0) {
+      const int64_t W = (int64_t)Hkv * T;
+      const int C = plan_ctas(W, v.ctas);
+      const int64_t X0 = (int64_t)Hkv * P + (int64_t)g * N;
+      first = plan_owner(W, C, X0);
+      last = plan_owner(W, C, X0 + N - 1);
+    }
+  }
 
-  const int2 r = v.seg_range[seg];
-  // fused step: the append record and this thread's operands, then cos/sin and the page
-  int4 rec = make_int4(0, 0, 0, 0);
-  uint16_t q0 = 0, q1 = 0, k0 = 0, k1 = 0, v0 = 0, v1 = 0;
-  double c = 1.0, sn = 0.0;
-  int page = -1;
+  // ---- before the wait (fused step): append record, rotations, the new slot's rows, score
   bool app = false;
-  int64_t tokens = 0;  // lead thread: the sequence's token count before the step
+  int n = 0, why = 0, t = 0, page = -1;
+  int64_t p = 0, tokens = 0;
+  uint16_t v0 = 0, v1 = 0;
+  float dot = 0.f;
   if constexpr (kStep) {
     const StepArgs &st = v.step;
-    const int b = seg / Hkv;
-    rec = st.stash[b];  // (n, 0 or the error that stops the append, position, ntok)
-    if (idx == 0 && seg - b * Hkv == 0) tokens = st.num_tokens[b];
-    app = rec.y == 0;
-    if (active) {
+    {
+      int L = v.num_slots[b];
+      const bool bad = L < 0 || L > v.max_slots;
+      L = L < 0 ? 0 : (bad ? v.max_slots : L);
+      t = st.ntok[b];
+      why = t < 1 ? HAM_DEVERR_NTOK
+            : bad ? HAM_DEVERR_SLOTS
+            : L == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
+      n = L;
+      p = st.pos ? (int64_t)st.pos[b]
+                 : (st.pos_mode == HAM_POS_SLOT ? (int64_t)n : st.num_tokens[b]);
+      if (idx == 0 && g == 0) tokens = st.num_tokens[b];
+    }
+    app = why == 0;
+    uint16_t q0 = 0, q1 = 0, k0 = 0, k1 = 0;
+    double c = 1.0, sn = 0.0;
+    if (app && active) {
       q0 = v.q[orow + i];
       q1 = v.q[orow + i + half];
       k0 = st.k_new[(int64_t)seg * D + i];
       k1 = st.k_new[(int64_t)seg * D + i + half];
       v0 = st.v_new[(int64_t)seg * D + i];
       v1 = st.v_new[(int64_t)seg * D + i + half];
-    }
-    if (app && active) {
-      const int64_t p = rec.z;
       if (p >= 0 && p < st.rope_positions) {
         const double2 e = st.rope_table[p * half + i];
         c = e.x;
@@ -805,25 +859,63 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       } else {
         sincos((double)p * st.inv_freq[i], &sn, &c);
       }
-      if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
+      if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + n / v.page_slots];
     }
+    float share = 0.f;
+    if (app && active) {
+      if (st.q_rot) {
+        const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
+        st.q_rot[orow + i] = rotate_elem(x0, x1, c, sn, false);
+        st.q_rot[orow + i + half] = rotate_elem(x1, x0, c, sn, true);
+      }
+      if (h == 0 && page >= 0 && page < v.pool_pages) {
+        const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
+        const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
+        st.k_pool[row + i] = rotate_elem(x0, x1, c, sn, false);
+        st.k_pool[row + i + half] = rotate_elem(x1, x0, c, sn, true);
+        st.v_pool[row + i] = v0;
+        st.v_pool[row + i + half] = v1;
+      }
+      const float cf = (float)c, sf = (float)sn;
+      const float x0 = bf16_bits_to_float(q0), x1 = bf16_bits_to_float(q1);
+      const float y0 = bf16_bits_to_float(k0), y1 = bf16_bits_to_float(k1);
+      const float qr0 = __bfloat162float(__float2bfloat16_rn(x0 * cf - x1 * sf));
+      const float qr1 = __bfloat162float(__float2bfloat16_rn(x1 * cf + x0 * sf));
+      const float kr0 = __bfloat162float(__float2bfloat16_rn(y0 * cf - y1 * sf));
+      const float kr1 = __bfloat162float(__float2bfloat16_rn(y1 * cf + y0 * sf));
+      share = qr0 * kr0 + qr1 * kr1;
+    }
+    // the pair shares of head h: one warp at d = 64, two at d = 128 (they meet in shared
+    // memory); every thread of the block takes part
+    __shared__ float head_sum[kCombineThreads / 32];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) share += __shfl_xor_sync(kFull, share, off);
+    if (lane == 0) head_sum[warp] = share;
+    __syncthreads();
+    dot = half > 32 ? head_sum[warp & ~1] + head_sum[warp | 1] : head_sum[warp];
   }
-  // Online merge in batches of 8 partials, whose loads are in flight together.  (16 saved one
-  // round trip at 8-12 partials per segment but cost registers: fewer resident blocks when a
-  // ragged batch has thousands of segments.)
-  const bool merge = r.x >= 0 && (kStep || r.x != r.y);
+
+  grid_dependency_wait();  // the attention grid's partials (and ranges)
+  // The next kernel may be scheduled now; its own dependency wait still covers this grid.
+  grid_launch_dependents();
+
+  if (!planned) {
+    const int2 r = v.seg_range[seg];
+    first = r.x;
+    last = r.y;
+  }
+  const bool merge = first >= 0 && (kStep || first != last);
   float M = -INFINITY, num0 = 0.f, num1 = 0.f, den = 0.f;
   if (active && merge) {
-    constexpr int kBatch = 8;
-    for (int k0b = r.x; k0b <= r.y; k0b += kBatch) {
+    for (int k0b = first; k0b <= last; k0b += kBatch) {
       float2 ml[kBatch];
       float a0[kBatch], a1[kBatch];
 #pragma unroll
       for (int j = 0; j < kBatch; ++j) {
-        const int64_t p = (int64_t)k0b + j + seg;
-        const bool in = k0b + j <= r.y;
-        const float *acc = v.part_acc + p * G * D + (int64_t)h * D;
-        ml[j] = in ? __ldcg(&v.part_ml[p * G + h]) : make_float2(-INFINITY, 0.f);
+        const int64_t pi = (int64_t)k0b + j + seg;
+        const bool in = k0b + j <= last;
+        const float *acc = v.part_acc + pi * G * D + (int64_t)h * D;
+        ml[j] = in ? __ldcg(&v.part_ml[pi * G + h]) : make_float2(-INFINITY, 0.f);
         a0[j] = in ? __ldcg(acc + i) : 0.f;
         a1[j] = in ? __ldcg(acc + i + half) : 0.f;
       }
@@ -845,47 +937,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
     }
   }
 
-  // fused step: the exact (fp64) rotations it commits (cos/sin were loaded before the merge,
-  // whose loads are therefore not held up by them)
-  uint16_t qc0 = 0, qc1 = 0, kc0 = 0, kc1 = 0;
   if constexpr (kStep) {
-    if (app && active) {
-      if (v.step.q_rot) {
-        const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
-        qc0 = rotate_elem(x0, x1, c, sn, false);
-        qc1 = rotate_elem(x1, x0, c, sn, true);
-      }
-      if (h == 0) {
-        const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
-        kc0 = rotate_elem(x0, x1, c, sn, false);
-        kc1 = rotate_elem(x1, x0, c, sn, true);
-      }
-    }
-  }
-
-  if constexpr (kStep) {
-    // Score of the appended slot for head h: the pair's share of q.k, summed over the D/2
-    // threads of the head (one warp at d = 64, two at d = 128, whose sums meet in shared
-    // memory).  Every thread of the block takes part, so no thread has left yet.
-    __shared__ float head_sum[kCombineThreads / 32];
-    float share = 0.f;
-    if (app && active) {
-      const float cf = (float)c, sf = (float)sn;
-      const float x0 = bf16_bits_to_float(q0), x1 = bf16_bits_to_float(q1);
-      const float y0 = bf16_bits_to_float(k0), y1 = bf16_bits_to_float(k1);
-      const float qr0 = __bfloat162float(__float2bfloat16_rn(x0 * cf - x1 * sf));
-      const float qr1 = __bfloat162float(__float2bfloat16_rn(x1 * cf + x0 * sf));
-      const float kr0 = __bfloat162float(__float2bfloat16_rn(y0 * cf - y1 * sf));
-      const float kr1 = __bfloat162float(__float2bfloat16_rn(y1 * cf + y0 * sf));
-      share = qr0 * kr0 + qr1 * kr1;
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) share += __shfl_xor_sync(kFull, share, off);
-    const int warp = threadIdx.x >> 5;
-    if ((threadIdx.x & 31) == 0) head_sum[warp] = share;
-    __syncthreads();
-    const float dot = half > 32 ? head_sum[warp & ~1] + head_sum[warp | 1] : head_sum[warp];
-    if (app && active) {
+    if (app && active) {  // the appended slot: one more term of the merge
       const float x = dot * (rsqrtf((float)D) * 1.4426950408889634f);  // log2 domain
       const float bm = fmaxf(M, x);
       const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
@@ -899,37 +952,23 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       store_out<OutT>(v.out, orow + i, num0 * inv);
       store_out<OutT>(v.out, orow + i + half, num1 * inv);
     }
-
+    // metadata and counters: one thread per sequence
+    if (g != 0 || idx != 0) return;
+    if (!app) {
+      record_error(v.err, why);
+      return;
+    }
+    const int pg = v.page_table[(int64_t)b * v.max_pages + n / v.page_slots];
+    if (pg < 0 || pg >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE too
+      record_error(v.err, HAM_DEVERR_PAGE);
+      return;
+    }
     const StepArgs &st = v.step;
-    const int b = seg / Hkv, g = seg - b * Hkv;
-    const bool lead = g == 0 && idx == 0;  // one thread per sequence
-    if (!app) {                            // no append for this sequence
-      if (lead) record_error(v.err, rec.y);
-      return;
-    }
-    if (!active) return;
-    if (st.q_rot) {
-      st.q_rot[orow + i] = qc0;
-      st.q_rot[orow + i + half] = qc1;
-    }
-    if (h != 0) return;
-    if (page < 0 || page >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE
-      if (lead) record_error(v.err, HAM_DEVERR_PAGE);
-      return;
-    }
-    const int n = rec.x;
-    const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
-    st.k_pool[row + i] = kc0;
-    st.k_pool[row + i + half] = kc1;
-    st.v_pool[row + i] = v0;
-    st.v_pool[row + i + half] = v1;
-    if (lead) {
-      const int64_t meta = (int64_t)page * v.page_slots + n % v.page_slots;
-      st.slot_pos[meta] = rec.z;
-      st.slot_ntok[meta] = rec.w;
-      st.num_slots[b] = n + 1;
-      st.num_tokens[b] = tokens + rec.w;
-    }
+    const int64_t meta = (int64_t)pg * v.page_slots + n % v.page_slots;
+    st.slot_pos[meta] = (int32_t)p;
+    st.slot_ntok[meta] = t;
+    st.num_slots[b] = n + 1;
+    st.num_tokens[b] = tokens + t;
   } else {
     if (active && merge) {
       const float inv = den > 0.f ? 1.f / den : 0.f;  // 0: every slot masked
@@ -939,11 +978,15 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   }
 }
 
+// Partials a segment can have at most, for the merge's batch: a segment spans about
+// ctas / segments + 1 CTAs when the lengths are equal.  16 saves a round trip when there are
+// 9..16; 8 keeps registers low when a ragged batch has thousands of segments.
 template <typename OutT, bool kStep>
 cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream) {
   const int per_seg = (v.group * head_dim / 2 + kCombineThreads - 1) / kCombineThreads;
+  const int64_t segs = (int64_t)v.batch * v.n_kv_heads;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(v.batch * v.n_kv_heads * per_seg));
+  cfg.gridDim = dim3((unsigned)(segs * per_seg));
   cfg.blockDim = dim3(kCombineThreads);
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
@@ -951,7 +994,9 @@ cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream)
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep>, v, head_dim, per_seg);
+  if ((int64_t)v.ctas >= 7 * segs)
+    return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep, 16>, v, head_dim, per_seg);
+  return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep, 8>, v, head_dim, per_seg);
 }
 
 // ------------------------------------------------------------------------------------

@@ -57,8 +57,8 @@ inline int32_t default_attention_ctas(int32_t num_sms, int32_t resident_per_sm) 
 
 // Everything one attention launch needs; all pointers are device pointers.
 // Extra inputs when the attention launch also performs this macro-step's append (the
-// fused decode step): the attention CTAs use the new slot and the rotated q from shared
-// memory, and the combine kernel commits the slot, q and the counters after the grid.
+// fused decode step): the attention pass turns q in registers and covers the stored slots;
+// the combine kernel adds the new slot and commits it, q_rot and the counters.
 struct StepArgs {
   const uint16_t *k_new, *v_new;   // [batch][n_kv_heads][head_dim]
   uint16_t *q_rot;                 // nullable [batch][n_q_heads][head_dim]: RoPE(q), fp64-exact
@@ -72,7 +72,6 @@ struct StepArgs {
   const double2 *rope_table;       // [rope_positions][head_dim / 2] (cos, sin)
   const float2 *rope_table_f;      // same, fp32
   int64_t rope_positions;
-  int4 *stash;                     // scratch [batch]: (slot n, 0 or HAM_DEVERR_*, position, ntok)
   int32_t pos_mode;
 };
 
@@ -179,7 +178,6 @@ struct ham_kv {
   double2 *rope_table = nullptr;  // own allocation
   float2 *rope_table_f = nullptr;  // own allocation
   int64_t rope_positions = 0;
-  int4 *stash = nullptr;           // fused step: per-sequence append record
   int32_t *err = nullptr;
   float *part_acc = nullptr;
   float2 *part_ml = nullptr;
