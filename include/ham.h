@@ -236,8 +236,8 @@ int ham_kv_set_attn_ctas(ham_kv *kv, int32_t ctas);
 
 /* Host evaluation of the split plan the attention kernel uses (no GPU needed).  Chunks are
  * 16 slots; the chunks of (sequence b, KV head g), b-major, are numbered contiguously (W in
- * all).  The first min(ctas, ceil(W / 8)) CTAs get equal non-empty ranges (a small problem
- * gets ranges of about 8 chunks instead of being spread over every CTA), CTA c the chunks
+ * all).  The first min(ctas, ceil(W / 4)) CTAs get equal non-empty ranges (a small problem
+ * gets ranges of about 4 chunks instead of being spread over every CTA), CTA c the chunks
  * [cta_begin[c], cta_begin[c+1]); the others stay idle.  For each segment
  * s = b*n_kv_heads+g, seg_first_cta[s] .. seg_last_cta[s] are exactly the CTAs that touch
  * it (-1, -1 if empty).

@@ -428,6 +428,12 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
     grid_dependency_wait();
     grid_launch_dependents();
   }
+  // The first segment's q (buffer 0, stage 0): its copy needs nothing of what warp 0 reads
+  // next, so it is under way meanwhile.
+  if (warp == 1 && active_cta && lane == 0) {
+    mbar_expect_tx(&full[0], (uint32_t)sb.q_bytes);
+    bulk_load(qbufs, v.q + (int64_t)seg0 * G * D, (uint32_t)sb.q_bytes, &full[0]);
+  }
   if constexpr (kStep) {
     // Caller inputs of the append: explicit positions, and whether each append happens.
     // (Computing the flags after the block barrier instead, in the consumer warp alone while
@@ -491,7 +497,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
             info[stage] = make_int4(s_seg, s_valid, s_fl, qb);
             uint32_t bytes = ((s_fl & kPageOk) && !issued) ? (uint32_t)S::kStageBytes : 0u;
             if (qb >= 0) {
-              bytes += (uint32_t)sb.q_bytes;
+              if (it > 0) bytes += (uint32_t)sb.q_bytes;  // (the first one is on its way)
               if constexpr (kStep) {
                 const int64_t p = posb[b];
                 tabled = p >= 0 && p < v.step.rope_positions;
@@ -509,7 +515,8 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
             }
             if (qb >= 0) {
               uint8_t *qdst = qbufs + qb * sb.stride;
-              bulk_load(qdst, v.q + (int64_t)s_seg * G * D, (uint32_t)sb.q_bytes, &full[stage]);
+              if (it > 0)
+                bulk_load(qdst, v.q + (int64_t)s_seg * G * D, (uint32_t)sb.q_bytes, &full[stage]);
               if constexpr (kStep) {  // (cos, sin) of the new slot's position
                 if (tabled)
                   bulk_load(qdst + sb.cs_off(),
@@ -952,19 +959,18 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       store_out<OutT>(v.out, orow + i, num0 * inv);
       store_out<OutT>(v.out, orow + i + half, num1 * inv);
     }
-    // metadata and counters: one thread per sequence
+    // metadata and counters: one thread per sequence (it loaded the page before the wait)
     if (g != 0 || idx != 0) return;
     if (!app) {
       record_error(v.err, why);
       return;
     }
-    const int pg = v.page_table[(int64_t)b * v.max_pages + n / v.page_slots];
-    if (pg < 0 || pg >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE too
+    if (page < 0 || page >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE too
       record_error(v.err, HAM_DEVERR_PAGE);
       return;
     }
     const StepArgs &st = v.step;
-    const int64_t meta = (int64_t)pg * v.page_slots + n % v.page_slots;
+    const int64_t meta = (int64_t)page * v.page_slots + n % v.page_slots;
     st.slot_pos[meta] = (int32_t)p;
     st.slot_ntok[meta] = t;
     st.num_slots[b] = n + 1;
@@ -979,8 +985,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
 }
 
 // Partials a segment can have at most, for the merge's batch: a segment spans about
-// ctas / segments + 1 CTAs when the lengths are equal.  16 saves a round trip when there are
-// 9..16; 8 keeps registers low when a ragged batch has thousands of segments.
+// ctas / segments + 1 CTAs when the lengths are equal.  32 or 16 save round trips when there
+// are that many; 8 keeps registers low when a ragged batch has thousands of segments.
 template <typename OutT, bool kStep>
 cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream) {
   const int per_seg = (v.group * head_dim / 2 + kCombineThreads - 1) / kCombineThreads;
@@ -994,6 +1000,8 @@ cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream)
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  if ((int64_t)v.ctas >= 24 * segs)
+    return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep, 32>, v, head_dim, per_seg);
   if ((int64_t)v.ctas >= 7 * segs)
     return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep, 16>, v, head_dim, per_seg);
   return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep, 8>, v, head_dim, per_seg);

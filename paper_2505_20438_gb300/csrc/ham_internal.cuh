@@ -26,7 +26,7 @@ constexpr int kMaxBatch = 4096;
 // owner(last chunk).  A CTA writes one partial per segment it touches, at index c + s,
 // which is unique because (c, s) only ever grows along the chunk order.
 // ---------------------------------------------------------------------------------------
-constexpr int kMinChunksPerCta = 8;
+constexpr int kMinChunksPerCta = 4;
 __host__ __device__ inline int32_t plan_ctas(int64_t W, int32_t launched) {
   const int64_t want = (W + kMinChunksPerCta - 1) / kMinChunksPerCta;
   return (int32_t)(want < (int64_t)launched ? want : (int64_t)launched);

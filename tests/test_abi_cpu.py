@@ -100,7 +100,7 @@ def test_split_plan_partitions_every_chunk_once(libham, counts, hkv, ctas):
     W = hkv * int(sum(_chunks(int(n)) for n in counts))
     assert begin[0] == 0 and begin[-1] == W
     sizes = np.diff(begin)
-    active = min(ctas, -(-W // 8))           # small problems: ranges of about 8 chunks
+    active = min(ctas, -(-W // 4))           # small problems: ranges of about 4 chunks
     assert np.all(sizes[:active] >= 1) and np.all(sizes[active:] == 0)
     if active:
         assert sizes[:active].max() - sizes[:active].min() <= 1       # balanced
