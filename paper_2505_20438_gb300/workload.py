@@ -60,6 +60,8 @@ C0_TINY = Workload("tiny_b1_h8x2_d64_s256_p128", batch=1, n_q_heads=8, n_kv_head
 C1_LLAMA8B = Workload("llama8b_layer_b8_s4096", batch=8, n_q_heads=32, n_kv_heads=8,
                       head_dim=128, page_slots=16, layers=1, slots=4096,
                       value_scale=1.0 / math.sqrt(128.0), seed=1)
+# The same layer at 8192 slots per sequence: the smallest batch-8 case with 8k slots.
+C1_LLAMA8B_S8K = dataclasses.replace(C1_LLAMA8B, name="llama8b_layer_b8_s8192", slots=8192)
 # Ragged serving batch: 64 sequences, slots uniform in [512, 8192], attend then append.
 C2_RAGGED = Workload("ragged_b64_s512to8192", batch=64, n_q_heads=32, n_kv_heads=8,
                      head_dim=128, page_slots=16, layers=1, slot_range=(512, 8192),
@@ -76,7 +78,7 @@ def c4_sweep(batch: int, slots: int = 2048, layers: int = 32) -> Workload:
                     value_scale=1.0 / math.sqrt(128.0), seed=4)
 
 
-WORKLOADS = {w.name: w for w in (C0_TINY, C1_LLAMA8B, C2_RAGGED, C3_LONG)}
+WORKLOADS = {w.name: w for w in (C0_TINY, C1_LLAMA8B, C1_LLAMA8B_S8K, C2_RAGGED, C3_LONG)}
 
 
 def scaled(w: Workload, **changes) -> Workload:

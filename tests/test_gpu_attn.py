@@ -146,7 +146,8 @@ def _full_size(w, sample_heads=None):
     return case, kv
 
 
-@pytest.mark.parametrize("w", [wl.C1_LLAMA8B, wl.C2_RAGGED, wl.C3_LONG], ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [wl.C1_LLAMA8B, wl.C1_LLAMA8B_S8K, wl.C2_RAGGED, wl.C3_LONG],
+                         ids=lambda w: w.name)
 def test_full_size_workloads(w):
     case, kv = _full_size(w)
     # attend-then-append stays consistent: the appended slot is visible to the next step
