@@ -451,6 +451,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
                         : bad ? HAM_DEVERR_SLOTS
                         : L == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
         appb[b] = why == 0;
+        if (blockIdx.x == 0) v.step.stash[b] = make_int4(L, why, posb[b], t);
       }
     }
   }
@@ -754,26 +755,117 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
 // the fused step they are the pair that RoPE turns together.  Blocks of kCombineThreads cover
 // one segment's G*D/2 pairs (whole heads).
 //
+// Fused step: the pass covered the stored slots; the appended slot enters here as one more
+// term of the merge: score q.k / sqrt(d) with q and the new key turned by the new position in
+// fp32 and rounded to bf16 as in the pass, weight 2^(score - M'), value v_new.  The same
+// threads commit the slot: the fp64 rotation of q (q_rot) and, for h = 0, of the new key,
+// rounded once to bf16 as ham_kv_append computes them, and the new value row.  Slot metadata
+// and counters are committed once no CTA can still read the counters.
+//
 // The kernel is scheduled (programmatic dependent launch) once every attention CTA has passed
-// its own dependency wait, and then idles until the attention grid ends.  So everything that
-// does not depend on the attention grid runs before this kernel's wait:
-//  * the segment's CTA range first..last, from the slot counters with the attention's split
-//    plan (small batches; larger ones read the range the attention's first CTA stored);
-//  * fused step: the append record of the sequence (slot n, the error that stops the append,
-//    position, tokens), read from the counters and caller inputs as the attention pass reads
-//    them; the fp64 rotation of q (q_rot) and of the new key, rounded once to bf16 as
-//    ham_kv_append computes them, and the new slot's rows (KV head g's threads of head 0);
-//    the new slot's score for head h: q.k / sqrt(d) with q and the new key turned by the new
-//    position in fp32 and rounded to bf16 as in the pass, summed over the D/2 threads of the
-//    head.  None of these is read by the attention pass: it covers the stored slots only, and
-//    the rows of slot n that its last chunk copies are masked there.
-// After the wait: the merge, the appended slot as one more term (weight 2^(score - M'), value
-// v_new), the output, and (KV head 0's lead thread) the slot metadata and the counters, which
-// every attention CTA has read by then.
+// its own dependency wait, and then idles until the attention grid ends.  Two kernels use that:
+//  * combine_kernel (batches up to kCombinePlanBatch, and for the fused step a grid of at most
+//    one CTA per SM, so that it sits beside the attention grid): before the wait, the segment's
+//    CTA range from the slot counters with the attention's split plan, and for the fused step
+//    the append record as the pass forms it, the rotations, q_rot and the new slot's rows, none
+//    of which the pass reads (it covers the stored slots, and the rows of slot n that its last
+//    chunk copies are masked there).  Each CTA then reports that it has read the counters; the
+//    last one to report commits the metadata and counters of every sequence after its wait (one
+//    thread per sequence), so that no CTA of the grid reads a counter it has advanced.
+//  * combine_late_kernel (otherwise): everything after the wait, from the range and the append
+//    record the attention pass stored; each sequence's lead thread (KV head 0) commits.
+// The decode attention alone (no step) writes no counter and plans early whenever the batch
+// allows.  (Measured: with thousands of segments the grid is not resident beside the pass, and
+// the CTAs that start after it would do the early work on the critical path.)
 // ------------------------------------------------------------------------------------
 constexpr int kCombineThreads = 128;
 constexpr int kCombinePlanBatch = kCombineThreads;  // batches whose plan the combine computes
 static_assert(kCombineThreads % 64 == 0, "a block holds whole heads of head_dim 64 or 128");
+
+// (cos, sin) of position p for pair i: the fp64 table, or fp64 sincos past it.
+__device__ __forceinline__ double2 rope_cs(const StepArgs &st, int64_t p, int half, int i) {
+  if (p >= 0 && p < st.rope_positions) return st.rope_table[p * half + i];
+  double s, c;
+  sincos((double)p * st.inv_freq[i], &s, &c);
+  return make_double2(c, s);
+}
+
+// One rotation pair at (c, s): the fp64 rotations of q and of the new key, each rounded once
+// to bf16 (the stored bits), and the pair's share of the new slot's score, q.k with both turned
+// in fp32 and rounded to bf16 as in the attention pass.  Not inlined (fp64 code, two callers).
+struct PairTurn {
+  uint16_t qc0, qc1, kc0, kc1;
+  float share;
+};
+__device__ __noinline__ PairTurn turn_pair(double c, double sn, uint16_t q0, uint16_t q1,
+                                           uint16_t k0, uint16_t k1) {
+  PairTurn r;
+  const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
+  r.qc0 = rotate_elem(x0, x1, c, sn, false);
+  r.qc1 = rotate_elem(x1, x0, c, sn, true);
+  const double y0 = bf16_bits_to_double(k0), y1 = bf16_bits_to_double(k1);
+  r.kc0 = rotate_elem(y0, y1, c, sn, false);
+  r.kc1 = rotate_elem(y1, y0, c, sn, true);
+  const float cf = (float)c, sf = (float)sn;
+  const float a0 = bf16_bits_to_float(q0), a1 = bf16_bits_to_float(q1);
+  const float b0 = bf16_bits_to_float(k0), b1 = bf16_bits_to_float(k1);
+  const float qr0 = __bfloat162float(__float2bfloat16_rn(a0 * cf - a1 * sf));
+  const float qr1 = __bfloat162float(__float2bfloat16_rn(a1 * cf + a0 * sf));
+  const float kr0 = __bfloat162float(__float2bfloat16_rn(b0 * cf - b1 * sf));
+  const float kr1 = __bfloat162float(__float2bfloat16_rn(b1 * cf + b0 * sf));
+  r.share = qr0 * kr0 + qr1 * kr1;
+  return r;
+}
+
+// The append record (n, 0 or the error that stops it, position, ntok) of a sequence from its
+// slot counter, token counter and the caller's ntok / pos, as the attention pass forms it.
+__device__ __forceinline__ int4 append_record(const AttnView &v, int Lraw, int64_t tokens,
+                                              int t, const int32_t *pos_b) {
+  const bool bad = Lraw < 0 || Lraw > v.max_slots;
+  const int n = Lraw < 0 ? 0 : (bad ? v.max_slots : Lraw);
+  const int why = t < 1 ? HAM_DEVERR_NTOK
+                  : bad ? HAM_DEVERR_SLOTS
+                  : n == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
+  const int64_t p = pos_b ? (int64_t)*pos_b : (v.step.pos_mode == HAM_POS_SLOT ? (int64_t)n : tokens);
+  return make_int4(n, why, (int)p, t);
+}
+
+// Online merge of the partials of CTAs lo..hi for the pair (h, i), (h, i + D/2) of segment
+// seg, in CTA order, kBatch partials per round trip.
+template <int kBatch>
+__device__ __forceinline__ void merge_partials(const AttnView &v, int seg, int h, int i,
+                                               int half, int D, int lo, int hi, float &M,
+                                               float &num0, float &num1, float &den) {
+  const int G = v.group;
+  for (int k0b = lo; k0b <= hi; k0b += kBatch) {
+    float2 ml[kBatch];
+    float a0[kBatch], a1[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int64_t pi = (int64_t)k0b + j + seg;
+      const bool in = k0b + j <= hi;
+      const float *acc = v.part_acc + pi * G * D + (int64_t)h * D;
+      ml[j] = in ? __ldcg(&v.part_ml[pi * G + h]) : make_float2(-INFINITY, 0.f);
+      a0[j] = in ? __ldcg(acc + i) : 0.f;
+      a1[j] = in ? __ldcg(acc + i + half) : 0.f;
+    }
+    float bm = M;
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) bm = fmaxf(bm, ml[j].x);
+    const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
+    num0 *= scale;
+    num1 *= scale;
+    den *= scale;
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const float w = (ml[j].x == -INFINITY) ? 0.f : ex2(ml[j].x - bm);
+      num0 += w * a0[j];
+      num1 += w * a1[j];
+      den += w * ml[j].y;
+    }
+    M = bm;
+  }
+}
 
 template <typename OutT, bool kStep, int kBatch>
 __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView v, int D,
@@ -787,19 +879,21 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   const int h = idx / half, i = idx - h * half;
   const int b = seg / Hkv, g = seg - b * Hkv;
   const int64_t orow = ((int64_t)seg * G + h) * D;  // row (b, g*G + h) of q / q_rot / out
+  const StepArgs &st = v.step;
+  __shared__ int red[3][kCombineThreads / 32];
+  __shared__ float head_sum[kCombineThreads / 32];
+  __shared__ int commit_all;  // fused step: this CTA commits every sequence
 
-  // ---- before the wait: the segment's CTA range (split plan, as the attention computes it)
+  // ---- the segment's CTA range (split plan, as the attention computes it)
   int first = -1, last = -1;
-  const bool planned = B <= kCombinePlanBatch;
-  if (planned) {
-    __shared__ int red[3][kCombineThreads / 32];
-    int n = 0;
+  int Lt = 0;  // thread t < B: the slot counter of sequence t
+  {
+    int nch = 0;
     if (tid < B) {
-      int L = v.num_slots[tid];
-      L = L < 0 ? 0 : (L > v.max_slots ? v.max_slots : L);
-      n = chunks_of(L);
+      Lt = v.num_slots[tid];
+      nch = chunks_of(Lt < 0 ? 0 : (Lt > v.max_slots ? v.max_slots : Lt));
     }
-    int tot = n, pre = tid < b ? n : 0, own = tid == b ? n : 0;
+    int tot = nch, pre = tid < b ? nch : 0, own = tid == b ? nch : 0;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
       tot += __shfl_xor_sync(kFull, tot, off);
@@ -828,37 +922,158 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
     }
   }
 
-  // ---- before the wait (fused step): append record, rotations, the new slot's rows, score
-  bool app = false;
-  int n = 0, why = 0, t = 0, page = -1;
-  int64_t p = 0, tokens = 0;
+  // ---- fused step: record, rotations, q_rot and the new slot's rows; then the report
+  int4 rec = make_int4(0, 0, 0, 0);
   uint16_t v0 = 0, v1 = 0;
   float dot = 0.f;
+  int4 crec = make_int4(0, 0, 0, 0);  // committing CTA, thread t < B: sequence t
+  int64_t ctok = 0;
+  int cpage = -1;
   if constexpr (kStep) {
-    const StepArgs &st = v.step;
-    {
-      int L = v.num_slots[b];
-      const bool bad = L < 0 || L > v.max_slots;
-      L = L < 0 ? 0 : (bad ? v.max_slots : L);
-      t = st.ntok[b];
-      why = t < 1 ? HAM_DEVERR_NTOK
-            : bad ? HAM_DEVERR_SLOTS
-            : L == v.max_slots ? HAM_DEVERR_CAPACITY : 0;
-      n = L;
-      p = st.pos ? (int64_t)st.pos[b]
-                 : (st.pos_mode == HAM_POS_SLOT ? (int64_t)n : st.num_tokens[b]);
-      if (idx == 0 && g == 0) tokens = st.num_tokens[b];
-    }
-    app = why == 0;
     uint16_t q0 = 0, q1 = 0, k0 = 0, k1 = 0;
-    double c = 1.0, sn = 0.0;
-    if (app && active) {
+    if (active) {  // caller inputs: final once the attention grid started
       q0 = v.q[orow + i];
       q1 = v.q[orow + i + half];
       k0 = st.k_new[(int64_t)seg * D + i];
       k1 = st.k_new[(int64_t)seg * D + i + half];
       v0 = st.v_new[(int64_t)seg * D + i];
       v1 = st.v_new[(int64_t)seg * D + i + half];
+    }
+    const int64_t tb = (!st.pos && st.pos_mode == HAM_POS_TOKEN) ? st.num_tokens[b] : 0;
+    rec = append_record(v, v.num_slots[b], tb, st.ntok[b], st.pos ? st.pos + b : nullptr);
+    float share = 0.f;
+    if (rec.y == 0 && active) {
+      const double2 cs = rope_cs(st, rec.z, half, i);
+      const PairTurn pt = turn_pair(cs.x, cs.y, q0, q1, k0, k1);
+      share = pt.share;
+      if (st.q_rot) {
+        st.q_rot[orow + i] = pt.qc0;
+        st.q_rot[orow + i + half] = pt.qc1;
+      }
+      if (h == 0) {  // the new slot's rows of KV head g
+        const int page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
+        if (page >= 0 && page < v.pool_pages) {
+          const int64_t row =
+              (((int64_t)page * Hkv + g) * v.page_slots + rec.x % v.page_slots) * D;
+          st.k_pool[row + i] = pt.kc0;
+          st.k_pool[row + i + half] = pt.kc1;
+          st.v_pool[row + i] = v0;
+          st.v_pool[row + i + half] = v1;
+        }
+      }
+    }
+    // the score of head h: one warp at d = 64, two at d = 128 (they meet in shared memory)
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) share += __shfl_xor_sync(kFull, share, off);
+    if (lane == 0) head_sum[warp] = share;
+    __syncthreads();  // (also: every counter read of this CTA is consumed)
+    dot = half > 32 ? head_sum[warp & ~1] + head_sum[warp | 1] : head_sum[warp];
+    if (tid == 0) {  // report; the last CTA to report commits every sequence
+      __threadfence();
+      const bool lastcta = atomicAdd(st.arrive, 1) == (int)gridDim.x - 1;
+      if (lastcta) {
+        *st.arrive = 0;
+        __threadfence();
+      }
+      commit_all = lastcta;
+    }
+    __syncthreads();
+    if (commit_all && tid < B) {  // its record, token count and page, while the pass runs
+      ctok = st.num_tokens[tid];
+      crec = append_record(v, Lt, ctok, st.ntok[tid], st.pos ? st.pos + tid : nullptr);
+      if (crec.y == 0) cpage = v.page_table[(int64_t)tid * v.max_pages + crec.x / v.page_slots];
+    }
+  }
+
+  grid_dependency_wait();  // the attention grid's partials
+  // The next kernel may be scheduled now; its own dependency wait still covers this grid.
+  grid_launch_dependents();
+
+  const bool merge = first >= 0 && (kStep || first != last);
+  float M = -INFINITY, num0 = 0.f, num1 = 0.f, den = 0.f;
+  if (active && merge)
+    merge_partials<kBatch>(v, seg, h, i, half, D, first, last, M, num0, num1, den);
+
+  if constexpr (kStep) {
+    const bool appended = rec.y == 0;
+    if (appended && active) {  // the appended slot: one more term of the merge
+      const float x = dot * (rsqrtf((float)D) * 1.4426950408889634f);  // log2 domain
+      const float bm = fmaxf(M, x);
+      const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
+      const float w = ex2(x - bm);
+      num0 = num0 * scale + w * bf16_bits_to_float(v0);
+      num1 = num1 * scale + w * bf16_bits_to_float(v1);
+      den = den * scale + w;
+    }
+    if (active && (merge || appended)) {
+      const float inv = den > 0.f ? 1.f / den : 0.f;
+      store_out<OutT>(v.out, orow + i, num0 * inv);
+      store_out<OutT>(v.out, orow + i + half, num1 * inv);
+    }
+    // slot metadata and counters of sequence t (committing CTA, thread t), or the error that
+    // stopped its append
+    if (!commit_all || tid >= B) return;
+    if (crec.y != 0) {
+      record_error(v.err, crec.y);
+      return;
+    }
+    if (cpage < 0 || cpage >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE too
+      record_error(v.err, HAM_DEVERR_PAGE);
+      return;
+    }
+    const int64_t meta = (int64_t)cpage * v.page_slots + crec.x % v.page_slots;
+    st.slot_pos[meta] = crec.z;
+    st.slot_ntok[meta] = crec.w;
+    st.num_slots[tid] = crec.x + 1;
+    st.num_tokens[tid] = ctok + crec.w;
+  } else {
+    if (active && merge) {
+      const float inv = den > 0.f ? 1.f / den : 0.f;  // 0: every slot masked
+      store_out<OutT>(v.out, orow + i, num0 * inv);
+      store_out<OutT>(v.out, orow + i + half, num1 * inv);
+    }
+  }
+}
+
+template <typename OutT, bool kStep>
+__global__ void __launch_bounds__(kCombineThreads) combine_late_kernel(const AttnView v, int D,
+                                                                       int blocks_per_seg) {
+  const int G = v.group, Hkv = v.n_kv_heads, half = D / 2;
+  const int seg = blockIdx.x / blocks_per_seg;
+  const int part = blockIdx.x % blocks_per_seg;
+  const int idx = part * kCombineThreads + threadIdx.x;  // pair index within the segment
+  const bool active = idx < G * half;
+  const int h = idx / half, i = idx - h * half;
+  const int64_t orow = ((int64_t)seg * G + h) * D;  // row (b, g*G + h) of q / q_rot / out
+
+  grid_dependency_wait();  // the attention grid's partials, ranges and append records
+  // The next kernel may be scheduled now; its own dependency wait still covers this grid.
+  grid_launch_dependents();
+
+  const int2 r = v.seg_range[seg];
+  // fused step: the append record and this thread's operands, then cos/sin and the page
+  int4 rec = make_int4(0, 0, 0, 0);
+  uint16_t q0 = 0, q1 = 0, k0 = 0, k1 = 0, v0 = 0, v1 = 0;
+  double c = 1.0, sn = 0.0;
+  int page = -1;
+  bool app = false;
+  int64_t tokens = 0;  // lead thread: the sequence's token count before the step
+  if constexpr (kStep) {
+    const StepArgs &st = v.step;
+    const int b = seg / Hkv;
+    rec = st.stash[b];  // (n, 0 or the error that stops the append, position, ntok)
+    if (idx == 0 && seg - b * Hkv == 0) tokens = st.num_tokens[b];
+    app = rec.y == 0;
+    if (active) {
+      q0 = v.q[orow + i];
+      q1 = v.q[orow + i + half];
+      k0 = st.k_new[(int64_t)seg * D + i];
+      k1 = st.k_new[(int64_t)seg * D + i + half];
+      v0 = st.v_new[(int64_t)seg * D + i];
+      v1 = st.v_new[(int64_t)seg * D + i + half];
+    }
+    if (app && active) {
+      const int64_t p = rec.z;
       if (p >= 0 && p < st.rope_positions) {
         const double2 e = st.rope_table[p * half + i];
         c = e.x;
@@ -866,23 +1081,38 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       } else {
         sincos((double)p * st.inv_freq[i], &sn, &c);
       }
-      if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + n / v.page_slots];
+      if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
     }
+  }
+  const bool merge = r.x >= 0 && (kStep || r.x != r.y);
+  float M = -INFINITY, num0 = 0.f, num1 = 0.f, den = 0.f;
+  if (active && merge) merge_partials<8>(v, seg, h, i, half, D, r.x, r.y, M, num0, num1, den);
+
+  // fused step: the exact (fp64) rotations it commits (cos/sin were loaded before the merge,
+  // whose loads are therefore not held up by them)
+  uint16_t qc0 = 0, qc1 = 0, kc0 = 0, kc1 = 0;
+  if constexpr (kStep) {
+    if (app && active) {
+      if (v.step.q_rot) {
+        const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
+        qc0 = rotate_elem(x0, x1, c, sn, false);
+        qc1 = rotate_elem(x1, x0, c, sn, true);
+      }
+      if (h == 0) {
+        const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
+        kc0 = rotate_elem(x0, x1, c, sn, false);
+        kc1 = rotate_elem(x1, x0, c, sn, true);
+      }
+    }
+  }
+
+  if constexpr (kStep) {
+    // Score of the appended slot for head h: the pair's share of q.k, summed over the D/2
+    // threads of the head (one warp at d = 64, two at d = 128, whose sums meet in shared
+    // memory).  Every thread of the block takes part, so no thread has left yet.
+    __shared__ float head_sum[kCombineThreads / 32];
     float share = 0.f;
     if (app && active) {
-      if (st.q_rot) {
-        const double x0 = bf16_bits_to_double(q0), x1 = bf16_bits_to_double(q1);
-        st.q_rot[orow + i] = rotate_elem(x0, x1, c, sn, false);
-        st.q_rot[orow + i + half] = rotate_elem(x1, x0, c, sn, true);
-      }
-      if (h == 0 && page >= 0 && page < v.pool_pages) {
-        const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
-        const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
-        st.k_pool[row + i] = rotate_elem(x0, x1, c, sn, false);
-        st.k_pool[row + i + half] = rotate_elem(x1, x0, c, sn, true);
-        st.v_pool[row + i] = v0;
-        st.v_pool[row + i + half] = v1;
-      }
       const float cf = (float)c, sf = (float)sn;
       const float x0 = bf16_bits_to_float(q0), x1 = bf16_bits_to_float(q1);
       const float y0 = bf16_bits_to_float(k0), y1 = bf16_bits_to_float(k1);
@@ -892,60 +1122,13 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       const float kr1 = __bfloat162float(__float2bfloat16_rn(y1 * cf + y0 * sf));
       share = qr0 * kr0 + qr1 * kr1;
     }
-    // the pair shares of head h: one warp at d = 64, two at d = 128 (they meet in shared
-    // memory); every thread of the block takes part
-    __shared__ float head_sum[kCombineThreads / 32];
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) share += __shfl_xor_sync(kFull, share, off);
-    if (lane == 0) head_sum[warp] = share;
+    const int warp = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) head_sum[warp] = share;
     __syncthreads();
-    dot = half > 32 ? head_sum[warp & ~1] + head_sum[warp | 1] : head_sum[warp];
-  }
-
-  grid_dependency_wait();  // the attention grid's partials (and ranges)
-  // The next kernel may be scheduled now; its own dependency wait still covers this grid.
-  grid_launch_dependents();
-
-  if (!planned) {
-    const int2 r = v.seg_range[seg];
-    first = r.x;
-    last = r.y;
-  }
-  const bool merge = first >= 0 && (kStep || first != last);
-  float M = -INFINITY, num0 = 0.f, num1 = 0.f, den = 0.f;
-  if (active && merge) {
-    for (int k0b = first; k0b <= last; k0b += kBatch) {
-      float2 ml[kBatch];
-      float a0[kBatch], a1[kBatch];
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-        const int64_t pi = (int64_t)k0b + j + seg;
-        const bool in = k0b + j <= last;
-        const float *acc = v.part_acc + pi * G * D + (int64_t)h * D;
-        ml[j] = in ? __ldcg(&v.part_ml[pi * G + h]) : make_float2(-INFINITY, 0.f);
-        a0[j] = in ? __ldcg(acc + i) : 0.f;
-        a1[j] = in ? __ldcg(acc + i + half) : 0.f;
-      }
-      float bm = M;
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) bm = fmaxf(bm, ml[j].x);
-      const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
-      num0 *= scale;
-      num1 *= scale;
-      den *= scale;
-#pragma unroll
-      for (int j = 0; j < kBatch; ++j) {
-        const float w = (ml[j].x == -INFINITY) ? 0.f : ex2(ml[j].x - bm);
-        num0 += w * a0[j];
-        num1 += w * a1[j];
-        den += w * ml[j].y;
-      }
-      M = bm;
-    }
-  }
-
-  if constexpr (kStep) {
-    if (app && active) {  // the appended slot: one more term of the merge
+    const float dot = half > 32 ? head_sum[warp & ~1] + head_sum[warp | 1] : head_sum[warp];
+    if (app && active) {
       const float x = dot * (rsqrtf((float)D) * 1.4426950408889634f);  // log2 domain
       const float bm = fmaxf(M, x);
       const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
@@ -959,22 +1142,37 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       store_out<OutT>(v.out, orow + i, num0 * inv);
       store_out<OutT>(v.out, orow + i + half, num1 * inv);
     }
-    // metadata and counters: one thread per sequence (it loaded the page before the wait)
-    if (g != 0 || idx != 0) return;
-    if (!app) {
-      record_error(v.err, why);
-      return;
-    }
-    if (page < 0 || page >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE too
-      record_error(v.err, HAM_DEVERR_PAGE);
-      return;
-    }
+
     const StepArgs &st = v.step;
-    const int64_t meta = (int64_t)page * v.page_slots + n % v.page_slots;
-    st.slot_pos[meta] = (int32_t)p;
-    st.slot_ntok[meta] = t;
-    st.num_slots[b] = n + 1;
-    st.num_tokens[b] = tokens + t;
+    const int b = seg / Hkv, g = seg - b * Hkv;
+    const bool lead = g == 0 && idx == 0;  // one thread per sequence
+    if (!app) {                            // no append for this sequence
+      if (lead) record_error(v.err, rec.y);
+      return;
+    }
+    if (!active) return;
+    if (st.q_rot) {
+      st.q_rot[orow + i] = qc0;
+      st.q_rot[orow + i + half] = qc1;
+    }
+    if (h != 0) return;
+    if (page < 0 || page >= v.pool_pages) {  // the pass recorded HAM_DEVERR_PAGE
+      if (lead) record_error(v.err, HAM_DEVERR_PAGE);
+      return;
+    }
+    const int n = rec.x;
+    const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
+    st.k_pool[row + i] = kc0;
+    st.k_pool[row + i + half] = kc1;
+    st.v_pool[row + i] = v0;
+    st.v_pool[row + i + half] = v1;
+    if (lead) {
+      const int64_t meta = (int64_t)page * v.page_slots + n % v.page_slots;
+      st.slot_pos[meta] = rec.z;
+      st.slot_ntok[meta] = rec.w;
+      st.num_slots[b] = n + 1;
+      st.num_tokens[b] = tokens + rec.w;
+    }
   } else {
     if (active && merge) {
       const float inv = den > 0.f ? 1.f / den : 0.f;  // 0: every slot masked
@@ -984,9 +1182,14 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   }
 }
 
-// Partials a segment can have at most, for the merge's batch: a segment spans about
-// ctas / segments + 1 CTAs when the lengths are equal.  32 or 16 save round trips when there
-// are that many; 8 keeps registers low when a ragged batch has thousands of segments.
+// Early mode: the plan fits one block (batch <= kCombinePlanBatch), and for the fused step the
+// grid sits beside the attention grid (at most one CTA per SM).
+inline bool combine_early(const AttnView &v, int64_t combine_ctas, bool step) {
+  return v.batch <= kCombinePlanBatch && (!step || combine_ctas <= (int64_t)v.sms);
+}
+
+// Early mode's merge batch: a segment spans about ctas / segments + 1 CTAs when the lengths
+// are equal, and 32 or 16 partials in flight save round trips when there are that many.
 template <typename OutT, bool kStep>
 cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream) {
   const int per_seg = (v.group * head_dim / 2 + kCombineThreads - 1) / kCombineThreads;
@@ -1000,6 +1203,8 @@ cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream)
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  if (!combine_early(v, segs * per_seg, kStep))
+    return cudaLaunchKernelEx(&cfg, combine_late_kernel<OutT, kStep>, v, head_dim, per_seg);
   if ((int64_t)v.ctas >= 24 * segs)
     return cudaLaunchKernelEx(&cfg, combine_kernel<OutT, kStep, 32>, v, head_dim, per_seg);
   if ((int64_t)v.ctas >= 7 * segs)

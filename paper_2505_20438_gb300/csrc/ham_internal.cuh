@@ -72,6 +72,9 @@ struct StepArgs {
   const double2 *rope_table;       // [rope_positions][head_dim / 2] (cos, sin)
   const float2 *rope_table_f;      // same, fp32
   int64_t rope_positions;
+  int4 *stash;                     // scratch [batch]: (slot n, 0 or HAM_DEVERR_*, position, ntok)
+  int32_t *arrive;                 // scratch: combine CTAs done reading the counters (0 between
+                                   // launches; the last one to arrive resets it)
   int32_t pos_mode;
 };
 
@@ -90,6 +93,7 @@ struct AttnView {
   int64_t pool_pages;
   int32_t batch, n_kv_heads, group, page_slots, max_pages, max_slots;
   int32_t ctas;
+  int32_t sms;                 // SMs of the device (the combine's choice of mode)
   // 1: the previous launch on the stream wrote nothing of this layer's counters, page table or
   // pools, so the kernel may read them before its programmatic-dependency wait (the host
   // decides; 0 is always correct)
@@ -179,6 +183,8 @@ struct ham_kv {
   float2 *rope_table_f = nullptr;  // own allocation
   int64_t rope_positions = 0;
   int32_t *err = nullptr;
+  int4 *stash = nullptr;           // fused step: per-sequence append record
+  int32_t *arrive = nullptr;       // fused step: the combine's arrival counter
   float *part_acc = nullptr;
   float2 *part_ml = nullptr;
   int2 *seg_range = nullptr;

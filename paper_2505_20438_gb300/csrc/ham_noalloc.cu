@@ -123,6 +123,7 @@ int ham_decode_attn_noalloc(const ham_attn_args *a, void *stream) {
   v.max_pages = a->max_pages;
   v.max_slots = a->max_slots;
   v.ctas = ctas;
+  v.sms = setup.num_sms;
   cudaError_t e = ham::launch_attention(tk, tv, v, a->head_dim, a->out_dtype,
                                         static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) {

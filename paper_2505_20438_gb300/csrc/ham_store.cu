@@ -330,6 +330,8 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   const size_t o_acc = carve(n_part * group * cfg.head_dim * sizeof(float));
   const size_t o_ml = carve(n_part * group * sizeof(float2));
   const size_t o_sr = carve(n_seg * sizeof(int2));
+  const size_t o_stash = carve((size_t)cfg.batch * sizeof(int4));
+  const size_t o_arrive = carve(sizeof(int32_t));
   kv->scratch_bytes = (int64_t)(off - o_acc);
 
   {
@@ -365,6 +367,8 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->part_acc = reinterpret_cast<float *>(kv->meta + o_acc);
   kv->part_ml = reinterpret_cast<float2 *>(kv->meta + o_ml);
   kv->seg_range = reinterpret_cast<int2 *>(kv->meta + o_sr);
+  kv->stash = reinterpret_cast<int4 *>(kv->meta + o_stash);
+  kv->arrive = reinterpret_cast<int32_t *>(kv->meta + o_arrive);
 
   // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits.
   e = cudaMemset(kv->pool, 0, pool_bytes);
@@ -535,6 +539,7 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
   v.max_pages = kv->max_pages;
   v.max_slots = kv->cfg.max_slots_per_seq;
   v.ctas = ctas;
+  v.sms = kv->num_sms;
   v.early = may_start_early(kv, layer, stream) ? 1 : 0;
   cudaError_t e = ham::launch_attention(kv->tmaps[(size_t)layer * 2], kv->tmaps[(size_t)layer * 2 + 1],
                                         v, kv->cfg.head_dim, out_dtype,
@@ -594,6 +599,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
   v.max_pages = kv->max_pages;
   v.max_slots = c.max_slots_per_seq;
   v.ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->default_step_ctas;
+  v.sms = kv->num_sms;
   ham::StepArgs &st = v.step;
   st.k_new = static_cast<const uint16_t *>(k_new);
   st.v_new = static_cast<const uint16_t *>(v_new);
@@ -610,6 +616,8 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
   st.rope_table = kv->rope_table;
   st.rope_table_f = kv->rope_table_f;
   st.rope_positions = kv->rope_positions;
+  st.stash = kv->stash;
+  st.arrive = kv->arrive;
   st.pos_mode = c.pos_mode;
   v.early = may_start_early(kv, layer, stream) ? 1 : 0;
   cudaError_t e = ham::launch_decode_step(kv->tmaps[(size_t)layer * 2],

@@ -49,6 +49,34 @@ def test_decode_matches_oracle(hq, hkv, d, page, counts, scale):
     assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
 
 
+def _large_batch_counts(batch, seed):
+    """Mostly short ragged sequences, some empty, a few long enough to span many CTAs."""
+    rng = np.random.default_rng(seed)
+    counts = rng.integers(0, 70, size=batch)
+    counts[rng.choice(batch, 8, replace=False)] = 0
+    counts[rng.choice(batch, 6, replace=False)] = rng.integers(600, 1500, size=6)
+    return tuple(int(c) for c in counts)
+
+
+@pytest.mark.parametrize("f32", [True, False])
+def test_batch_above_128_merges_the_stored_ranges(f32):
+    """Batches above 128 sequences read each segment's CTA range from the attention pass
+    instead of recomputing the plan in the combine kernel."""
+    counts = _large_batch_counts(300, 5)
+    case = small_case(batch=300, hq=8, hkv=2, d=64, page=16, counts=counts, seed=5)
+    ref = oracle.OracleCache.from_case(case).decode_attn(case.q)
+    kv = gpu_cache(case)
+    out = gpu_decode(kv, case.q, f32=f32)
+    if f32:
+        assert_parity(out, ref, max_abs=F32_MAX, mean_abs=F32_MEAN, what="B300 f32")
+    else:
+        assert_parity(out, ref, what="B300 bf16")
+    for b, n in enumerate(counts):
+        if n == 0:
+            assert np.all(out[b] == 0)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
 @pytest.mark.parametrize("ctas", [1, 2, 7, 152, 0, 1216])
 def test_split_count_invariance(ctas):
     case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(2000, 35, 901), seed=11)

@@ -85,6 +85,34 @@ def test_step_matches_oracle(pos_mode, d, hq, hkv, page, counts):
     assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
 
 
+def test_step_batch_above_128():
+    """More than 128 sequences: the combine reads the stored CTA ranges; a few long sequences
+    span many CTAs, some sequences are empty (the appended slot alone)."""
+    rng = np.random.default_rng(9)
+    counts = rng.integers(0, 70, size=260)
+    counts[rng.choice(260, 6, replace=False)] = 0
+    counts[rng.choice(260, 5, replace=False)] = rng.integers(600, 1500, size=5)
+    case = small_case(batch=260, hq=16, hkv=2, d=128, page=32, counts=tuple(int(c) for c in counts),
+                      seed=9, extra_slots=4)
+    oc = oracle.OracleCache.from_case(case)
+    kv = gpu_cache(case)
+    rng2 = wl.rng_for(9, 61)
+    q = case.q.copy()
+    for step in range(2):
+        k_new = wl.normal_bf16(rng2, case.k_new.shape)
+        v_new = wl.normal_bf16(rng2, case.v_new.shape)
+        ntok = wl.ntok_capped_geometric(rng2, (case.w.batch,))
+        q_ref = q.copy()
+        assert oc.append(k_new, v_new, ntok, q_inout=q_ref) == 0
+        ref = oc.decode_attn(q_ref)
+        got, q_rot = _step(kv, q, k_new, v_new, ntok)
+        assert np.array_equal(q_rot, q_ref), f"q_rot after step {step}"
+        assert_parity(got, ref, MAX_ABS, MEAN_ABS, what=f"B260 step {step}")
+        q = wl.normal_bf16(rng2, case.q.shape)
+    _assert_cache_equal(kv, oc)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
 def test_step_equals_append_then_attend_on_gpu():
     """Same cache bits and rotated q bits as the two separate calls; outputs agree closely."""
     case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(100, 17, 640), seed=12)
