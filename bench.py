@@ -56,6 +56,10 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--path", choices=["fused", "split"], default="fused",
                    help="fused: ham_decode_step; split: ham_kv_append + ham_decode_attn")
+    p.add_argument("--caches", type=int, default=CACHES,
+                   help="independent caches rotated by the timed steps (fewer keep an ncu capture "
+                        "of a large workload within a few GB; the default keeps each step's cache "
+                        "out of L2)")
     return p.parse_args()
 
 
@@ -807,7 +811,11 @@ def run_stack(args, w):
 
 
 def main():
+    global CACHES
     args = parse_args()
+    if args.caches < 1 or GRAPH_STEPS % args.caches:
+        raise SystemExit(f"--caches must divide {GRAPH_STEPS}")
+    CACHES = args.caches
     w = workload(args.workload)
     if args.impl == "reference":
         run_reference(args, w)
