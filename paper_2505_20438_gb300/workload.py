@@ -215,3 +215,50 @@ def device_normal_bf16(shape, scale: float, seed: int, device="cuda"):
     if scale != 1.0:
         x.mul_(scale)
     return x.to(torch.bfloat16)
+
+
+# ---------------------------------------------------------------------------------------
+# Compositional embedder inputs (Sec. 3.2): the tokens each sequence produced in the last
+# macro-step (1..4, capped-geometric like the slots they become), their embeddings, and
+# synthetic module weights (the trained ones are not used).  Llama-3.2-1B width: H = 2048,
+# 32 heads of 64 (Sec. 4.1).
+# ---------------------------------------------------------------------------------------
+@dataclasses.dataclass(frozen=True)
+class EmbedWorkload:
+    name: str
+    batch: int
+    hidden: int = 2048
+    n_heads: int = 32
+    max_patch: int = MAX_TOKENS_PER_SLOT
+    seed: int = 5
+
+
+@dataclasses.dataclass
+class EmbedCase:
+    w: EmbedWorkload
+    counts: np.ndarray      # [B] tokens per sequence, 1..max_patch
+    offsets: np.ndarray     # [B+1] prefix of counts: sequence b owns rows offsets[b].. of x
+    x: np.ndarray           # bf16 bits [T][H]: token embeddings, N(0, 1)
+    wq: np.ndarray          # bf16 bits [H][H] ([out][in]), N(0, 1/H)
+    wk: np.ndarray
+    wv: np.ndarray
+    wo: np.ndarray
+    pos: np.ndarray         # bf16 bits [max_patch][H]: position embeddings, N(0, 1)
+
+
+def embed_workload(batch: int, **kw) -> EmbedWorkload:
+    return EmbedWorkload(f"embed_b{batch}", batch=batch, **kw)
+
+
+def make_embed_case(w: EmbedWorkload, counts: Optional[np.ndarray] = None) -> EmbedCase:
+    rng = rng_for(w.seed, 40)
+    if counts is None:
+        counts = ntok_capped_geometric(rng, (w.batch,), cap=w.max_patch)
+    counts = np.asarray(counts, dtype=np.int32)
+    offsets = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    H = w.hidden
+    ws = 1.0 / math.sqrt(H)
+    return EmbedCase(w, counts, offsets, normal_bf16(rng, (int(offsets[-1]), H)),
+                     normal_bf16(rng, (H, H), ws), normal_bf16(rng, (H, H), ws),
+                     normal_bf16(rng, (H, H), ws), normal_bf16(rng, (H, H), ws),
+                     normal_bf16(rng, (w.max_patch, H)))
