@@ -280,6 +280,50 @@ typedef struct ham_attn_args {
 
 int ham_decode_attn_noalloc(const ham_attn_args *args, void *stream);
 
+/* ------------------------------------------------------------------------------------
+ * Compositional embedder (Sec. 3.2, Sec. 3.4, Sec. 4.1)
+ * ------------------------------------------------------------------------------------
+ * Before a macro-step's forward, the 1..max_patch tokens each sequence produced in the last
+ * one are fused into a single hidden state of the model width H: a multi-head cross-attention
+ * whose query is the mean of the token embeddings and whose keys and values come from the
+ * embeddings plus a learned embedding of each token's place in the patch, then a linear layer.
+ * A sequence with one token skips the module: its hidden state is the token's embedding, bit
+ * for bit.  For sequence b with n >= 2 tokens x_0..x_{n-1}:
+ *   q = W_q mean(x),  k_i = W_k (x_i + P[i]),  v_i = W_v (x_i + P[i]),
+ *   per head h: o_h = sum_i softmax_i(q_h . k_{i,h} / sqrt(head_dim)) v_{i,h},   out_b = W_o o.
+ * Weights are bf16 [out][in] row-major (y = W x); accumulation is fp32, o and out are
+ * rounded to bf16.  The handle owns copies of the weights and all workspace; the dense
+ * projections run as cuBLAS GEMMs, the fusion (mean query, position terms, softmax, bypass)
+ * in this library's kernels.                                                              */
+typedef struct ham_embedder ham_embedder; /* opaque handle: weights and workspace */
+
+typedef struct ham_embed_config {
+  int32_t hidden;     /* H, the model width: a multiple of n_heads and of 8 */
+  int32_t n_heads;    /* heads; head_dim = hidden / n_heads must be 32, 64 or 128 */
+  int32_t max_batch;  /* sequences per ham_embed call, at most */
+  int32_t max_patch;  /* tokens per sequence, at most (1..8; the paper's macro-steps emit 4) */
+} ham_embed_config;
+
+/* Allocate an embedder and copy its weights (device bf16): wq, wk, wv, wo [H][H]; pos
+ * [max_patch][H].  Host errors: HAM_EINVAL (bad config, NULL or unaligned pointer),
+ * HAM_ENOMEM, HAM_ECUDA (including a cuBLAS failure). */
+int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *wk,
+                       const void *wv, const void *wo, const void *pos, ham_embedder **out);
+int ham_embedder_free(ham_embedder *e);
+
+/* Fuse the tokens of `batch` sequences.  x: device bf16 [total_tokens][H], sequence b owning
+ * rows offsets[b] .. offsets[b+1]-1; offsets: device int32 [batch + 1], offsets[0] = 0 and
+ * offsets[batch] = total_tokens; out: device bf16 [batch][H].  A sequence whose token count
+ * is outside 1..max_patch gets zeros and sets the device error word (HAM_DEVERR_NTOK).
+ * Asynchronous on `stream`.  Host errors: HAM_EINVAL (NULL/unaligned pointers, batch or
+ * total_tokens out of range), HAM_ECUDA.  Calls on one handle must not overlap in time. */
+int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t batch,
+              int32_t total_tokens, void *out, void *stream);
+
+/* Read and clear the embedder's device error word (synchronizes `stream`).  Returns
+ * HAM_EDEVICE if it was set, with the code in *device_code. */
+int ham_embedder_status(ham_embedder *e, void *stream, int32_t *device_code);
+
 #ifdef __cplusplus
 }
 #endif

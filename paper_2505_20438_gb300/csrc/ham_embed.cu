@@ -1,0 +1,312 @@
+// Compositional embedder (HAMburger, arXiv 2505.20438, Sec. 3.2, Sec. 3.4, Sec. 4.1).
+//
+// The tokens a macro-step produced for a sequence (1..max_patch) become one hidden state of
+// the model width H before the base model's next forward: a multi-head cross-attention with
+// the mean of the token embeddings as its query, keys and values from the embeddings plus a
+// learned embedding of each token's place in the patch, then a linear layer; one token skips
+// the module.  On the GPU:
+//
+//  1. QKV = X [T][H] . [W_q; W_k; W_v]^T -> fp32 [T][3H]: one dense GEMM over every token of
+//     the call (cuBLAS, bf16 in, fp32 accumulate and out).  Because the projections are linear,
+//     W_q mean(x) = mean(W_q x), and W_{k,v} (x_i + P[i]) = W_{k,v} x_i + W_{k,v} P[i]: the
+//     position terms KVP = [W_k; W_v] P^T are computed once when the handle is made.
+//  2. fuse_kernel, one warp per (sequence, head): the mean query, k_i and v_i with their
+//     position terms, the scaled scores, softmax over the patch (fp32) and o, rounded to bf16
+//     into O [B][H].  Token counts outside 1..max_patch set the error word.
+//  3. out = O . W_o^T (cuBLAS, bf16 out, fp32 accumulate).
+//  4. bypass_kernel: sequences of one token get their embedding back bit for bit (and
+//     sequences with a bad count get zeros), over the rows step 3 wrote.
+// The GEMMs stream the weights (4 H^2 bf16) once per call: memory-bound at the batches of
+// decoding, where the token rows are far fewer than the weight rows.
+#include <cublas_v2.h>
+#include <cuda_bf16.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "ham_internal.cuh"
+
+struct ham_embedder {
+  ham_embed_config cfg{};
+  int device = 0;
+  cublasHandle_t blas = nullptr;
+  void *blas_ws = nullptr;       // cuBLAS workspace (so that no call allocates, even captured)
+  __nv_bfloat16 *wqkv = nullptr; // [3H][H]
+  __nv_bfloat16 *wo = nullptr;   // [H][H]
+  float *kvp = nullptr;          // [max_patch][2H]: W_k P[i], W_v P[i]
+  float *qkv = nullptr;          // [max_batch * max_patch][3H]
+  __nv_bfloat16 *o = nullptr;    // [max_batch][H]
+  int32_t *err = nullptr;        // device error word
+  int32_t *host_err = nullptr;   // pinned read-back
+};
+
+namespace ham {
+namespace {
+
+constexpr size_t kBlasWorkspace = 32u << 20;
+
+int efail(int status, const char *fmt, ...) {
+  char msg[256];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(msg, sizeof msg, fmt, ap);
+  va_end(ap);
+  return set_last_error(status, msg);
+}
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+// One warp per (sequence b, head h); lane j owns head elements j, j + 32, ... (kPer of them).
+template <int kPer>
+__global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv,
+                                                   const float *__restrict__ kvp,
+                                                   const int32_t *__restrict__ offsets,
+                                                   __nv_bfloat16 *__restrict__ o, int32_t *err,
+                                                   int batch, int total, int H, int n_heads,
+                                                   int max_patch, float scale) {
+  const int warp = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (warp >= batch * n_heads) return;
+  const int b = warp / n_heads, h = warp - b * n_heads;
+  const int hd = kPer * 32;
+  const int t0 = offsets[b], n = offsets[b + 1] - t0;
+  // a sequence's rows must lie in the call's token rows; else it is a bad count
+  const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
+  __nv_bfloat16 *orow = o + (int64_t)b * H + (int64_t)h * hd;
+  if (bad || n == 1) {  // bypass (or a bad count): O is not used for this sequence
+    if (bad && h == 0 && lane == 0) record_error(err, HAM_DEVERR_NTOK);
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) orow[lane + 32 * e] = __float2bfloat16_rn(0.f);
+    return;
+  }
+  const int64_t ld = 3 * (int64_t)H;
+  float q[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) q[e] = 0.f;
+  for (int i = 0; i < n; ++i) {
+    const float *row = qkv + (int64_t)(t0 + i) * ld + (int64_t)h * hd;
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) q[e] += row[lane + 32 * e];
+  }
+  const float inv_n = 1.f / (float)n;
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) q[e] *= inv_n;
+  // scores of the patch's tokens (at most 8)
+  float s[8];
+  float smax = -INFINITY;
+  for (int i = 0; i < n; ++i) {
+    const float *row = qkv + (int64_t)(t0 + i) * ld + H + (int64_t)h * hd;
+    const float *pk = kvp + (int64_t)i * 2 * H + (int64_t)h * hd;
+    float part = 0.f;
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) part += q[e] * (row[lane + 32 * e] + pk[lane + 32 * e]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+    s[i] = part * scale;
+    smax = fmaxf(smax, s[i]);
+  }
+  float den = 0.f;
+  for (int i = 0; i < n; ++i) {
+    s[i] = expf(s[i] - smax);
+    den += s[i];
+  }
+  const float inv = 1.f / den;
+  float acc[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
+  for (int i = 0; i < n; ++i) {
+    const float *row = qkv + (int64_t)(t0 + i) * ld + 2 * (int64_t)H + (int64_t)h * hd;
+    const float *pv = kvp + (int64_t)i * 2 * H + H + (int64_t)h * hd;
+    const float a = s[i] * inv;
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) acc[e] += a * (row[lane + 32 * e] + pv[lane + 32 * e]);
+  }
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) orow[lane + 32 * e] = __float2bfloat16_rn(acc[e]);
+}
+
+// Sequences of one token: their embedding; bad counts: zeros.  16-byte vectors.
+__global__ void bypass_kernel(const uint4 *__restrict__ x, const int32_t *__restrict__ offsets,
+                              uint4 *__restrict__ out, int batch, int total, int vec_per_row,
+                              int max_patch) {
+  const int b = blockIdx.y;
+  if (b >= batch) return;
+  const int t0 = offsets[b], n = offsets[b + 1] - t0;
+  const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
+  if (n != 1 && !bad) return;
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < vec_per_row; j += gridDim.x * blockDim.x)
+    out[(int64_t)b * vec_per_row + j] = bad ? make_uint4(0, 0, 0, 0)
+                                            : x[(int64_t)t0 * vec_per_row + j];
+}
+
+// C[rows][n_out] (row-major, ldc) = A[rows][k] (row-major bf16) . W[n_out][k]^T (bf16).
+cublasStatus_t gemm_rows(cublasHandle_t h, int rows, int n_out, int k, const __nv_bfloat16 *a,
+                         const __nv_bfloat16 *w, void *c, cudaDataType_t c_type, int ldc) {
+  const float one = 1.f, zero = 0.f;
+  // column-major view: C^T [n_out][rows] = W (k x n_out, transposed) . A^T (k x rows)
+  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, n_out, rows, k, &one, w, CUDA_R_16BF, k, a,
+                      CUDA_R_16BF, k, &zero, c, c_type, ldc, CUBLAS_COMPUTE_32F,
+                      CUBLAS_GEMM_DEFAULT);
+}
+
+}  // namespace
+}  // namespace ham
+
+using ham::efail;
+
+extern "C" {
+
+int ham_embedder_free(ham_embedder *e) {
+  if (!e) return HAM_OK;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  cudaSetDevice(e->device);
+  if (e->blas) cublasDestroy(e->blas);
+  cudaFree(e->blas_ws);
+  cudaFree(e->wqkv);
+  cudaFree(e->wo);
+  cudaFree(e->kvp);
+  cudaFree(e->qkv);
+  cudaFree(e->o);
+  cudaFree(e->err);
+  cudaFreeHost(e->host_err);
+  cudaSetDevice(dev);
+  delete e;
+  return HAM_OK;
+}
+
+int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *wk,
+                       const void *wv, const void *wo, const void *pos, ham_embedder **out) {
+  if (!cfg || !out) return efail(HAM_EINVAL, "cfg and out are required");
+  *out = nullptr;
+  const int H = cfg->hidden, nh = cfg->n_heads;
+  if (nh < 1 || H < 1 || H % nh != 0 || H % 8 != 0)
+    return efail(HAM_EINVAL, "hidden %d must be a multiple of n_heads %d and of 8", H, nh);
+  const int hd = H / nh;
+  if (hd != 32 && hd != 64 && hd != 128)
+    return efail(HAM_EUNSUPPORTED, "head_dim %d: 32, 64 or 128", hd);
+  if (cfg->max_batch < 1 || cfg->max_patch < 1 || cfg->max_patch > 8)
+    return efail(HAM_EINVAL, "max_batch >= 1 and max_patch in 1..8");
+  if (!wq || !wk || !wv || !wo || !pos) return efail(HAM_EINVAL, "weights are required");
+  if (!ham::aligned16(wq) || !ham::aligned16(wk) || !ham::aligned16(wv) || !ham::aligned16(wo) ||
+      !ham::aligned16(pos))
+    return efail(HAM_EINVAL, "weights must be 16-byte aligned");
+  ham_embedder *e = new ham_embedder();
+  e->cfg = *cfg;
+  cudaGetDevice(&e->device);
+  const size_t hh = (size_t)H * H;
+  const size_t rows = (size_t)cfg->max_batch * cfg->max_patch;
+  cudaError_t ce = cudaSuccess;
+  auto alloc = [&](void **p, size_t bytes) {
+    if (ce == cudaSuccess) ce = cudaMalloc(p, bytes);
+  };
+  alloc(reinterpret_cast<void **>(&e->wqkv), 3 * hh * 2);
+  alloc(reinterpret_cast<void **>(&e->wo), hh * 2);
+  alloc(reinterpret_cast<void **>(&e->kvp), (size_t)cfg->max_patch * 2 * H * 4);
+  alloc(reinterpret_cast<void **>(&e->qkv), rows * 3 * H * 4);
+  alloc(reinterpret_cast<void **>(&e->o), (size_t)cfg->max_batch * H * 2);
+  alloc(reinterpret_cast<void **>(&e->err), 4);
+  alloc(&e->blas_ws, ham::kBlasWorkspace);
+  if (ce == cudaSuccess) ce = cudaMallocHost(reinterpret_cast<void **>(&e->host_err), 4);
+  if (ce != cudaSuccess) {
+    cudaGetLastError();
+    ham_embedder_free(e);
+    return efail(HAM_ENOMEM, "embedder allocation failed");
+  }
+  ce = cudaMemcpy(e->wqkv, wq, hh * 2, cudaMemcpyDeviceToDevice);
+  if (ce == cudaSuccess) ce = cudaMemcpy(e->wqkv + hh, wk, hh * 2, cudaMemcpyDeviceToDevice);
+  if (ce == cudaSuccess) ce = cudaMemcpy(e->wqkv + 2 * hh, wv, hh * 2, cudaMemcpyDeviceToDevice);
+  if (ce == cudaSuccess) ce = cudaMemcpy(e->wo, wo, hh * 2, cudaMemcpyDeviceToDevice);
+  if (ce == cudaSuccess) ce = cudaMemset(e->err, 0, 4);
+  if (ce != cudaSuccess) {
+    cudaGetLastError();
+    ham_embedder_free(e);
+    return efail(HAM_ECUDA, "embedder weight copy: %s", cudaGetErrorString(ce));
+  }
+  cublasStatus_t bs = cublasCreate(&e->blas);
+  if (bs == CUBLAS_STATUS_SUCCESS) bs = cublasSetWorkspace(e->blas, e->blas_ws, ham::kBlasWorkspace);
+  // position terms: KVP [max_patch][2H] = P [max_patch][H] . [W_k; W_v]^T
+  if (bs == CUBLAS_STATUS_SUCCESS)
+    bs = ham::gemm_rows(e->blas, cfg->max_patch, 2 * H, H,
+                        static_cast<const __nv_bfloat16 *>(pos), e->wqkv + hh, e->kvp,
+                        CUDA_R_32F, 2 * H);
+  if (bs == CUBLAS_STATUS_SUCCESS && cudaDeviceSynchronize() != cudaSuccess)
+    bs = CUBLAS_STATUS_EXECUTION_FAILED;
+  if (bs != CUBLAS_STATUS_SUCCESS) {
+    cudaGetLastError();
+    ham_embedder_free(e);
+    return efail(HAM_ECUDA, "cuBLAS set-up failed (status %d)", (int)bs);
+  }
+  *out = e;
+  return HAM_OK;
+}
+
+int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t batch,
+              int32_t total_tokens, void *out, void *stream) {
+  if (!e || !x || !offsets || !out) return efail(HAM_EINVAL, "null argument");
+  const ham_embed_config &c = e->cfg;
+  if (batch < 1 || batch > c.max_batch)
+    return efail(HAM_EINVAL, "batch %d outside 1..%d", batch, c.max_batch);
+  if (total_tokens < batch || total_tokens > batch * c.max_patch)
+    return efail(HAM_EINVAL, "total_tokens %d outside %d..%d", total_tokens, batch,
+                 batch * c.max_patch);
+  if (!ham::aligned16(x) || !ham::aligned16(out) || ((uintptr_t)offsets & 3u))
+    return efail(HAM_EINVAL, "x/out must be 16-byte aligned, offsets 4-byte aligned");
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev != e->device) cudaSetDevice(e->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int H = c.hidden, hd = H / c.n_heads;
+  int rc = HAM_OK;
+  cublasStatus_t bs = cublasSetStream(e->blas, s);
+  if (bs == CUBLAS_STATUS_SUCCESS)
+    bs = ham::gemm_rows(e->blas, total_tokens, 3 * H, H, static_cast<const __nv_bfloat16 *>(x),
+                        e->wqkv, e->qkv, CUDA_R_32F, 3 * H);
+  if (bs != CUBLAS_STATUS_SUCCESS) rc = efail(HAM_ECUDA, "projection GEMM (status %d)", (int)bs);
+  if (rc == HAM_OK) {
+    const int warps = batch * c.n_heads;
+    const dim3 grid((unsigned)((warps + 7) / 8)), block(256);
+    const float scale = 1.f / sqrtf((float)hd);
+    if (hd == 32)
+      ham::fuse_kernel<1><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets, e->o, e->err, batch,
+                                                 total_tokens, H, c.n_heads, c.max_patch, scale);
+    else if (hd == 64)
+      ham::fuse_kernel<2><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets, e->o, e->err, batch,
+                                                 total_tokens, H, c.n_heads, c.max_patch, scale);
+    else
+      ham::fuse_kernel<4><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets, e->o, e->err, batch,
+                                                 total_tokens, H, c.n_heads, c.max_patch, scale);
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "fuse launch: %s", cudaGetErrorString(ce));
+  }
+  if (rc == HAM_OK) {
+    bs = ham::gemm_rows(e->blas, batch, H, H, e->o, e->wo, out, CUDA_R_16BF, H);
+    if (bs != CUBLAS_STATUS_SUCCESS) rc = efail(HAM_ECUDA, "output GEMM (status %d)", (int)bs);
+  }
+  if (rc == HAM_OK) {
+    const int vec = H / 8;
+    const dim3 grid((unsigned)((vec + 127) / 128), (unsigned)batch), block(128);
+    ham::bypass_kernel<<<grid, block, 0, s>>>(static_cast<const uint4 *>(x), offsets,
+                                              static_cast<uint4 *>(out), batch, total_tokens, vec,
+                                              c.max_patch);
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "bypass launch: %s", cudaGetErrorString(ce));
+  }
+  if (dev != e->device) cudaSetDevice(dev);
+  return rc;
+}
+
+int ham_embedder_status(ham_embedder *e, void *stream, int32_t *device_code) {
+  if (!e) return efail(HAM_EINVAL, "null handle");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t ce = cudaMemcpyAsync(e->host_err, e->err, 4, cudaMemcpyDeviceToHost, s);
+  if (ce == cudaSuccess) ce = cudaMemsetAsync(e->err, 0, 4, s);
+  if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
+  if (ce != cudaSuccess) return efail(HAM_ECUDA, "status read: %s", cudaGetErrorString(ce));
+  if (device_code) *device_code = *e->host_err;
+  if (*e->host_err != 0) return efail(HAM_EDEVICE, "device error word = %d", *e->host_err);
+  return HAM_OK;
+}
+
+}  // extern "C"

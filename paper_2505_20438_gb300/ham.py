@@ -62,8 +62,18 @@ class ham_kv_info(ctypes.Structure):
                 ("scratch_bytes", ctypes.c_int64)]
 
 
+class ham_embed_config(ctypes.Structure):
+    _fields_ = [("hidden", ctypes.c_int32), ("n_heads", ctypes.c_int32),
+                ("max_batch", ctypes.c_int32), ("max_patch", ctypes.c_int32)]
+
+
 _vp, _i32, _i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
 _SIGNATURES = {
+    "ham_embedder_alloc": [ctypes.POINTER(ham_embed_config), _vp, _vp, _vp, _vp, _vp,
+                           ctypes.POINTER(_vp)],
+    "ham_embedder_free": [_vp],
+    "ham_embed": [_vp, _vp, _vp, _i32, _i32, _vp, _vp],
+    "ham_embedder_status": [_vp, _vp, ctypes.POINTER(_i32)],
     "ham_kv_alloc": [ctypes.POINTER(ham_config), ctypes.POINTER(_vp)],
     "ham_kv_free": [_vp],
     "ham_kv_append": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp],
@@ -351,3 +361,67 @@ def ham_decode_attn_noalloc(k_pool, v_pool, page_table, num_slots, q, out, max_s
         _dev(err, (1,), "i32", "err", nullable=True), P, B, Hq, Hkv, d, S, max_pages,
         int(max_slots), int(ctas), HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16)
     _check(lib().ham_decode_attn_noalloc(ctypes.byref(args), _stream_ptr(stream)))
+
+
+# ---------------------------------------------------------------------------------------
+# compositional embedder
+# ---------------------------------------------------------------------------------------
+
+class Embedder:
+    """Owning handle of one compositional embedder (ham_embedder*)."""
+
+    def __init__(self, ptr: int, cfg: ham_embed_config):
+        self.ptr = ptr
+        self.hidden, self.n_heads = cfg.hidden, cfg.n_heads
+        self.max_batch, self.max_patch = cfg.max_batch, cfg.max_patch
+
+    @property
+    def _as_parameter_(self):
+        return ctypes.c_void_p(self.ptr)
+
+    def close(self):
+        if self.ptr:
+            ham_embedder_free(self)
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def ham_embedder_alloc(hidden, n_heads, max_batch, max_patch, wq, wk, wv, wo, pos) -> Embedder:
+    """Weights: CUDA bf16 tensors, wq/wk/wv/wo [hidden][hidden] ([out][in]), pos
+    [max_patch][hidden].  The handle keeps its own copies."""
+    cfg = ham_embed_config(hidden, n_heads, max_batch, max_patch)
+    H = hidden
+    out = ctypes.c_void_p()
+    _check(lib().ham_embedder_alloc(
+        ctypes.byref(cfg), _dev(wq, (H, H), "bf16", "wq"), _dev(wk, (H, H), "bf16", "wk"),
+        _dev(wv, (H, H), "bf16", "wv"), _dev(wo, (H, H), "bf16", "wo"),
+        _dev(pos, (max_patch, H), "bf16", "pos"), ctypes.byref(out)))
+    return Embedder(out.value, cfg)
+
+
+def ham_embedder_free(e: Embedder):
+    ptr, e.ptr = e.ptr, 0
+    _check(lib().ham_embedder_free(ctypes.c_void_p(ptr)))
+
+
+def ham_embed(e: Embedder, x, offsets, out, stream=None):
+    """x: CUDA bf16 [total_tokens][hidden]; offsets: CUDA int32 [batch + 1]; out: CUDA bf16
+    [batch][hidden]."""
+    B = out.shape[0] if out is not None else 0
+    T = x.shape[0] if x is not None else 0
+    _check(lib().ham_embed(e, _dev(x, (T, e.hidden), "bf16", "x"),
+                           _dev(offsets, (B + 1,), "i32", "offsets"), B, T,
+                           _dev(out, (B, e.hidden), "bf16", "out"), _stream_ptr(stream)))
+
+
+def ham_embedder_status(e: Embedder, stream=None) -> int:
+    """Device error code (HAM_DEVERR_*), read and cleared; does not raise on HAM_EDEVICE."""
+    code = ctypes.c_int32(0)
+    rc = lib().ham_embedder_status(e, _stream_ptr(stream), ctypes.byref(code))
+    if rc not in (HAM_OK, HAM_EDEVICE):
+        _check(rc)
+    return code.value

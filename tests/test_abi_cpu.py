@@ -133,3 +133,29 @@ def test_split_plan_rejects_bad_arguments(libham):
         ham.ham_split_plan(np.array([-1], np.int32), 1, 4)
     with pytest.raises(ham.HamError):
         ham.ham_split_plan(np.array([5], np.int32), 1, 0)
+
+
+@pytest.mark.parametrize("hidden,heads,batch,patch,status", [
+    (100, 3, 4, 4, ham.HAM_EINVAL),          # not a multiple of the heads
+    (256, 16, 4, 4, ham.HAM_EUNSUPPORTED),   # head_dim 16
+    (256, 4, 0, 4, ham.HAM_EINVAL),          # no batch
+    (256, 4, 4, 9, ham.HAM_EINVAL),          # patch above 8
+])
+def test_embedder_alloc_rejects_bad_configs_on_the_host(libham, hidden, heads, batch, patch,
+                                                        status):
+    cfg = ham.ham_embed_config(hidden, heads, batch, patch)
+    out = ctypes.c_void_p()
+    dummy = ctypes.c_void_p(16)   # never dereferenced: the config is checked first
+    assert libham.ham_embedder_alloc(ctypes.byref(cfg), dummy, dummy, dummy, dummy, dummy,
+                                     ctypes.byref(out)) == status
+    assert out.value is None
+
+
+def test_embedder_null_arguments_are_rejected(libham):
+    cfg = ham.ham_embed_config(256, 4, 4, 4)
+    out = ctypes.c_void_p()
+    assert libham.ham_embedder_alloc(ctypes.byref(cfg), None, None, None, None, None,
+                                     ctypes.byref(out)) == ham.HAM_EINVAL
+    assert libham.ham_embed(None, None, None, 1, 1, None, None) == ham.HAM_EINVAL
+    assert libham.ham_embedder_status(None, None, None) == ham.HAM_EINVAL
+    assert libham.ham_embedder_free(None) == ham.HAM_OK

@@ -1,0 +1,90 @@
+"""GPU: the compositional embedder (Sec. 3.2, Sec. 3.4) against the fp64 oracle on the same
+seeded bits.  Fused states within the bf16 bar; single-token sequences bit for bit."""
+import numpy as np
+import pytest
+
+from oracle import embedder as oe
+from paper_2505_20438_gb300 import ham
+from paper_2505_20438_gb300 import workload as wl
+
+from gpu_helpers import MAX_ABS, MEAN_ABS, assert_parity, dev_bf16, dev_i32, host_bits, torch
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(c, offsets=None, max_batch=None):
+    t = torch()
+    w = c.w
+    e = ham.ham_embedder_alloc(w.hidden, w.n_heads, max_batch or w.batch, w.max_patch,
+                               dev_bf16(c.wq), dev_bf16(c.wk), dev_bf16(c.wv), dev_bf16(c.wo),
+                               dev_bf16(c.pos))
+    B = len(c.counts)
+    out = t.full((B, w.hidden), float("nan"), dtype=t.bfloat16, device="cuda")
+    ham.ham_embed(e, dev_bf16(c.x), dev_i32(c.offsets if offsets is None else offsets), out)
+    t.cuda.synchronize()
+    return e, out
+
+
+def _check(c, out):
+    ref = oe.embed(c.x, c.offsets, c.wq, c.wk, c.wv, c.wo, c.pos, c.w.n_heads)
+    got = out.float().cpu().numpy().astype(np.float64)
+    bits = host_bits(out)
+    fused = c.counts > 1
+    if fused.any():
+        assert_parity(got[fused], ref[fused], MAX_ABS, MEAN_ABS, what="fused states")
+    for b in np.nonzero(~fused)[0]:
+        assert np.array_equal(bits[b], c.x[c.offsets[b]]), f"bypass row {b}"
+
+
+@pytest.mark.parametrize("batch,hidden,heads", [(64, 2048, 32), (8, 256, 8), (5, 512, 4)])
+def test_embed_matches_oracle(batch, hidden, heads):
+    c = wl.make_embed_case(wl.embed_workload(batch, hidden=hidden, n_heads=heads, seed=batch))
+    e, out = _run(c)
+    _check(c, out)
+    assert ham.ham_embedder_status(e) == ham.HAM_DEVERR_NONE
+
+
+@pytest.mark.parametrize("counts", [[1] * 9, [4] * 7, [2, 1, 4, 3, 1, 1, 2]])
+def test_embed_patch_mixes(counts):
+    c = wl.make_embed_case(wl.embed_workload(len(counts), hidden=1024, n_heads=16, seed=3),
+                           counts=np.array(counts))
+    e, out = _run(c, max_batch=16)
+    _check(c, out)
+    assert ham.ham_embedder_status(e) == ham.HAM_DEVERR_NONE
+
+
+def test_bad_counts_give_zeros_and_the_error_word():
+    c = wl.make_embed_case(wl.embed_workload(6, hidden=256, n_heads=8, seed=4),
+                           counts=np.array([2, 1, 3, 2, 1, 3]))
+    offsets = c.offsets.copy()
+    offsets[2] = offsets[1]        # sequence 1: no token (sequence 2 now has 4)
+    offsets[4] = offsets[5] + 1    # sequence 4: a negative count (sequence 3 now has 4)
+    e, out = _run(c, offsets=offsets)
+    bits = host_bits(out)
+    counts = np.diff(offsets)
+    ok = (counts >= 1) & (counts <= c.w.max_patch) & (offsets[:-1] >= 0) & \
+        (offsets[1:] <= offsets[-1])
+    assert ham.ham_embedder_status(e) == ham.HAM_DEVERR_NTOK
+    for b in np.nonzero(~ok)[0]:
+        assert np.all(bits[b] == 0), b
+    ref = oe.embed(c.x, c.offsets, c.wq, c.wk, c.wv, c.wo, c.pos, c.w.n_heads)
+    for b in np.nonzero(ok)[0]:    # untouched sequences keep their own tokens and result
+        if offsets[b] == c.offsets[b] and offsets[b + 1] == c.offsets[b + 1]:
+            got = out[b].float().cpu().numpy().astype(np.float64)
+            assert np.max(np.abs(got - ref[b])) <= MAX_ABS, b
+
+
+def test_host_errors():
+    t = torch()
+    c = wl.make_embed_case(wl.embed_workload(4, hidden=256, n_heads=8, seed=2))
+    e, out = _run(c)
+    x = dev_bf16(c.x)
+    with pytest.raises(ham.HamError):          # batch above the handle's max_batch
+        big = t.zeros((5, 256), dtype=t.bfloat16, device="cuda")
+        ham.ham_embed(e, t.zeros((5, 256), dtype=t.bfloat16, device="cuda"),
+                      dev_i32(np.arange(6)), big)
+    with pytest.raises(ValueError):            # wrong offsets shape
+        ham.ham_embed(e, x, dev_i32(c.offsets[:-1]), out)
+    with pytest.raises(ham.HamError):          # head_dim 16 is not compiled
+        ham.ham_embedder_alloc(256, 16, 4, 4, *(dev_bf16(w) for w in (c.wq, c.wk, c.wv, c.wo)),
+                               dev_bf16(c.pos))
