@@ -12,10 +12,11 @@
 //     position terms KVP = [W_k; W_v] P^T are computed once when the handle is made.
 //  2. fuse_kernel, one warp per (sequence, head): the mean query, k_i and v_i with their
 //     position terms, the scaled scores, softmax over the patch (fp32) and o, rounded to bf16
-//     into O [B][H].  Token counts outside 1..max_patch set the error word.
-//  3. out = O . W_o^T (cuBLAS, bf16 out, fp32 accumulate).
-//  4. bypass_kernel: sequences of one token get their embedding back bit for bit (and
-//     sequences with a bad count get zeros), over the rows step 3 wrote.
+//     into O [B][H], all of the patch's loads issued at once.  It also sets out: the token's
+//     embedding for a sequence of one (whose O row is 0), zeros for the others.  Token counts
+//     outside 1..max_patch set the error word (and give zeros).
+//  3. out = O . W_o^T + out (cuBLAS, bf16 out, fp32 accumulate): a sequence of one gets
+//     x + 0, its embedding (exactly, but for the sign of a zero and NaN payloads).
 // The GEMMs stream the weights (4 H^2 bf16) once per call: memory-bound at the batches of
 // decoding, where the token rows are far fewer than the weight rows.
 #include <cublas_v2.h>
@@ -45,6 +46,7 @@ namespace ham {
 namespace {
 
 constexpr size_t kBlasWorkspace = 32u << 20;
+constexpr int kMaxPatch = 8;  // tokens per sequence, at most (ham_embed_config.max_patch)
 
 int efail(int status, const char *fmt, ...) {
   char msg[256];
@@ -62,7 +64,9 @@ template <int kPer>
 __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv,
                                                    const float *__restrict__ kvp,
                                                    const int32_t *__restrict__ offsets,
-                                                   __nv_bfloat16 *__restrict__ o, int32_t *err,
+                                                   const __nv_bfloat16 *__restrict__ x,
+                                                   __nv_bfloat16 *__restrict__ o,
+                                                   __nv_bfloat16 *__restrict__ out, int32_t *err,
                                                    int batch, int total, int H, int n_heads,
                                                    int max_patch, float scale) {
   const int warp = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
@@ -74,76 +78,86 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
   // a sequence's rows must lie in the call's token rows; else it is a bad count
   const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
   __nv_bfloat16 *orow = o + (int64_t)b * H + (int64_t)h * hd;
-  if (bad || n == 1) {  // bypass (or a bad count): O is not used for this sequence
+  __nv_bfloat16 *outrow = out + (int64_t)b * H + (int64_t)h * hd;
+  // The output GEMM adds O . W_o^T to what this kernel leaves in out: the token itself for a
+  // sequence of one (with O = 0), zeros otherwise.
+  const __nv_bfloat16 zero = __float2bfloat16_rn(0.f);
+  if (bad || n == 1) {
     if (bad && h == 0 && lane == 0) record_error(err, HAM_DEVERR_NTOK);
+    const __nv_bfloat16 *xrow = x + (int64_t)(bad ? 0 : t0) * H + (int64_t)h * hd;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) orow[lane + 32 * e] = __float2bfloat16_rn(0.f);
+    for (int e = 0; e < kPer; ++e) {
+      orow[lane + 32 * e] = zero;
+      outrow[lane + 32 * e] = bad ? zero : xrow[lane + 32 * e];
+    }
     return;
   }
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) outrow[lane + 32 * e] = zero;
   const int64_t ld = 3 * (int64_t)H;
-  float q[kPer];
+  const int64_t col = (int64_t)h * hd + lane;
+  // every load of the patch at once (one round trip): q, k and v rows and the position terms
+  float qv[kMaxPatch][kPer], kv[kMaxPatch][kPer], vv[kMaxPatch][kPer];
 #pragma unroll
-  for (int e = 0; e < kPer; ++e) q[e] = 0.f;
-  for (int i = 0; i < n; ++i) {
-    const float *row = qkv + (int64_t)(t0 + i) * ld + (int64_t)h * hd;
+  for (int i = 0; i < kMaxPatch; ++i) {
+    const bool in = i < n;
+    const float *row = qkv + (int64_t)(t0 + (in ? i : 0)) * ld + col;
+    const float *pp = kvp + (int64_t)(in ? i : 0) * 2 * H + col;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) q[e] += row[lane + 32 * e];
+    for (int e = 0; e < kPer; ++e) {
+      qv[i][e] = in ? row[32 * e] : 0.f;
+      kv[i][e] = in ? row[H + 32 * e] + pp[32 * e] : 0.f;
+      vv[i][e] = in ? row[2 * H + 32 * e] + pp[H + 32 * e] : 0.f;
+    }
   }
+  float q[kPer];
   const float inv_n = 1.f / (float)n;
 #pragma unroll
-  for (int e = 0; e < kPer; ++e) q[e] *= inv_n;
-  // scores of the patch's tokens (at most 8)
-  float s[8];
-  float smax = -INFINITY;
-  for (int i = 0; i < n; ++i) {
-    const float *row = qkv + (int64_t)(t0 + i) * ld + H + (int64_t)h * hd;
-    const float *pk = kvp + (int64_t)i * 2 * H + (int64_t)h * hd;
+  for (int e = 0; e < kPer; ++e) {
+    float sum = 0.f;
+#pragma unroll
+    for (int i = 0; i < kMaxPatch; ++i) sum += qv[i][e];
+    q[e] = sum * inv_n;
+  }
+  // scores (the reductions of the patch's tokens interleave), softmax over the patch
+  float s[kMaxPatch];
+#pragma unroll
+  for (int i = 0; i < kMaxPatch; ++i) {
     float part = 0.f;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) part += q[e] * (row[lane + 32 * e] + pk[lane + 32 * e]);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
-    s[i] = part * scale;
-    smax = fmaxf(smax, s[i]);
+    for (int e = 0; e < kPer; ++e) part += q[e] * kv[i][e];
+    s[i] = part;
   }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+    for (int i = 0; i < kMaxPatch; ++i) s[i] += __shfl_xor_sync(0xffffffffu, s[i], off);
+  float smax = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < kMaxPatch; ++i)
+    if (i < n) smax = fmaxf(smax, s[i] * scale);
   float den = 0.f;
-  for (int i = 0; i < n; ++i) {
-    s[i] = expf(s[i] - smax);
+#pragma unroll
+  for (int i = 0; i < kMaxPatch; ++i) {
+    s[i] = i < n ? expf(s[i] * scale - smax) : 0.f;
     den += s[i];
   }
   const float inv = 1.f / den;
-  float acc[kPer];
 #pragma unroll
-  for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
-  for (int i = 0; i < n; ++i) {
-    const float *row = qkv + (int64_t)(t0 + i) * ld + 2 * (int64_t)H + (int64_t)h * hd;
-    const float *pv = kvp + (int64_t)i * 2 * H + H + (int64_t)h * hd;
-    const float a = s[i] * inv;
+  for (int e = 0; e < kPer; ++e) {
+    float acc = 0.f;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) acc[e] += a * (row[lane + 32 * e] + pv[lane + 32 * e]);
+    for (int i = 0; i < kMaxPatch; ++i) acc += s[i] * vv[i][e];
+    orow[lane + 32 * e] = __float2bfloat16_rn(acc * inv);
   }
-#pragma unroll
-  for (int e = 0; e < kPer; ++e) orow[lane + 32 * e] = __float2bfloat16_rn(acc[e]);
 }
 
-// Sequences of one token: their embedding; bad counts: zeros.  16-byte vectors.
-__global__ void bypass_kernel(const uint4 *__restrict__ x, const int32_t *__restrict__ offsets,
-                              uint4 *__restrict__ out, int batch, int total, int vec_per_row,
-                              int max_patch) {
-  const int b = blockIdx.y;
-  if (b >= batch) return;
-  const int t0 = offsets[b], n = offsets[b + 1] - t0;
-  const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
-  if (n != 1 && !bad) return;
-  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < vec_per_row; j += gridDim.x * blockDim.x)
-    out[(int64_t)b * vec_per_row + j] = bad ? make_uint4(0, 0, 0, 0)
-                                            : x[(int64_t)t0 * vec_per_row + j];
-}
-
-// C[rows][n_out] (row-major, ldc) = A[rows][k] (row-major bf16) . W[n_out][k]^T (bf16).
+// C[rows][n_out] (row-major, ldc) = A[rows][k] (row-major bf16) . W[n_out][k]^T (bf16)
+// + beta C.
 cublasStatus_t gemm_rows(cublasHandle_t h, int rows, int n_out, int k, const __nv_bfloat16 *a,
-                         const __nv_bfloat16 *w, void *c, cudaDataType_t c_type, int ldc) {
-  const float one = 1.f, zero = 0.f;
+                         const __nv_bfloat16 *w, void *c, cudaDataType_t c_type, int ldc,
+                         float beta = 0.f) {
+  const float one = 1.f, zero = beta;
   // column-major view: C^T [n_out][rows] = W (k x n_out, transposed) . A^T (k x rows)
   return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, n_out, rows, k, &one, w, CUDA_R_16BF, k, a,
                       CUDA_R_16BF, k, &zero, c, c_type, ldc, CUBLAS_COMPUTE_32F,
@@ -269,29 +283,26 @@ int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t ba
     const dim3 grid((unsigned)((warps + 7) / 8)), block(256);
     const float scale = 1.f / sqrtf((float)hd);
     if (hd == 32)
-      ham::fuse_kernel<1><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets, e->o, e->err, batch,
+      ham::fuse_kernel<1><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets,
+                                                 static_cast<const __nv_bfloat16 *>(x), e->o,
+                                                 static_cast<__nv_bfloat16 *>(out), e->err, batch,
                                                  total_tokens, H, c.n_heads, c.max_patch, scale);
     else if (hd == 64)
-      ham::fuse_kernel<2><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets, e->o, e->err, batch,
+      ham::fuse_kernel<2><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets,
+                                                 static_cast<const __nv_bfloat16 *>(x), e->o,
+                                                 static_cast<__nv_bfloat16 *>(out), e->err, batch,
                                                  total_tokens, H, c.n_heads, c.max_patch, scale);
     else
-      ham::fuse_kernel<4><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets, e->o, e->err, batch,
+      ham::fuse_kernel<4><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets,
+                                                 static_cast<const __nv_bfloat16 *>(x), e->o,
+                                                 static_cast<__nv_bfloat16 *>(out), e->err, batch,
                                                  total_tokens, H, c.n_heads, c.max_patch, scale);
     cudaError_t ce = cudaGetLastError();
     if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "fuse launch: %s", cudaGetErrorString(ce));
   }
   if (rc == HAM_OK) {
-    bs = ham::gemm_rows(e->blas, batch, H, H, e->o, e->wo, out, CUDA_R_16BF, H);
+    bs = ham::gemm_rows(e->blas, batch, H, H, e->o, e->wo, out, CUDA_R_16BF, H, 1.f);
     if (bs != CUBLAS_STATUS_SUCCESS) rc = efail(HAM_ECUDA, "output GEMM (status %d)", (int)bs);
-  }
-  if (rc == HAM_OK) {
-    const int vec = H / 8;
-    const dim3 grid((unsigned)((vec + 127) / 128), (unsigned)batch), block(128);
-    ham::bypass_kernel<<<grid, block, 0, s>>>(static_cast<const uint4 *>(x), offsets,
-                                              static_cast<uint4 *>(out), batch, total_tokens, vec,
-                                              c.max_patch);
-    cudaError_t ce = cudaGetLastError();
-    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "bypass launch: %s", cudaGetErrorString(ce));
   }
   if (dev != e->device) cudaSetDevice(dev);
   return rc;
