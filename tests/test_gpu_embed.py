@@ -7,9 +7,25 @@ from oracle import embedder as oe
 from paper_2505_20438_gb300 import ham
 from paper_2505_20438_gb300 import workload as wl
 
-from gpu_helpers import MAX_ABS, MEAN_ABS, assert_parity, dev_bf16, dev_i32, host_bits, torch
+from gpu_helpers import MEAN_ABS, dev_bf16, dev_i32, host_bits, torch
 
 pytestmark = pytest.mark.gpu
+
+# Tolerance from the arithmetic: the GPU rounds o to bf16 before the output projection and the
+# state to bf16 at the end, each a relative error of at most 2^-9; through W_o (rows of norm
+# ~1) the first moves an element by about 2^-9 of the state's size, so the error is about
+# 2 * 2^-9 ~ 0.4% of |state| at worst.  States reach magnitude 4-5, so the bar is relative:
+# |got - ref| <= REL * max(1, |ref|) per element (REL = 1e-2, ~2.5x that), and the bf16 mean-abs
+# bar on average.
+REL = 1e-2
+
+
+def assert_states(got, ref, what):
+    assert np.all(np.isfinite(got)), what
+    err = np.abs(got - ref)
+    scaled = err / np.maximum(1.0, np.abs(ref))
+    assert scaled.max() <= REL, f"{what}: max scaled error {scaled.max():.3e}"
+    assert err.mean() <= MEAN_ABS, f"{what}: mean-abs {err.mean():.3e}"
 
 
 def _run(c, offsets=None, max_batch=None):
@@ -31,7 +47,7 @@ def _check(c, out):
     bits = host_bits(out)
     fused = c.counts > 1
     if fused.any():
-        assert_parity(got[fused], ref[fused], MAX_ABS, MEAN_ABS, what="fused states")
+        assert_states(got[fused], ref[fused], "fused states")
     for b in np.nonzero(~fused)[0]:
         assert np.array_equal(bits[b], c.x[c.offsets[b]]), f"bypass row {b}"
 
@@ -71,7 +87,7 @@ def test_bad_counts_give_zeros_and_the_error_word():
     for b in np.nonzero(ok)[0]:    # untouched sequences keep their own tokens and result
         if offsets[b] == c.offsets[b] and offsets[b + 1] == c.offsets[b + 1]:
             got = out[b].float().cpu().numpy().astype(np.float64)
-            assert np.max(np.abs(got - ref[b])) <= MAX_ABS, b
+            assert np.max(np.abs(got - ref[b]) / np.maximum(1.0, np.abs(ref[b]))) <= REL, b
 
 
 def test_host_errors():
