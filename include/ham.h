@@ -287,15 +287,15 @@ int ham_decode_attn_noalloc(const ham_attn_args *args, void *stream);
  * one are fused into a single hidden state of the model width H: a multi-head cross-attention
  * whose query is the mean of the token embeddings and whose keys and values come from the
  * embeddings plus a learned embedding of each token's place in the patch, then a linear layer.
- * A sequence with one token skips the module: its hidden state is the token's embedding
- * (bit for bit, except that a -0.0 element may come back as +0.0 and a NaN's payload may
- * change).  For sequence b with n >= 2 tokens x_0..x_{n-1}:
+ * A sequence with one token skips the module: its hidden state is the token's embedding, bit
+ * for bit.  For sequence b with n >= 2 tokens x_0..x_{n-1}:
  *   q = W_q mean(x),  k_i = W_k (x_i + P[i]),  v_i = W_v (x_i + P[i]),
  *   per head h: o_h = sum_i softmax_i(q_h . k_{i,h} / sqrt(head_dim)) v_{i,h},   out_b = W_o o.
  * Weights are bf16 [out][in] row-major (y = W x); accumulation is fp32, o and out are
- * rounded to bf16.  The handle owns copies of the weights and all workspace; the dense
- * projections run as cuBLAS GEMMs, the fusion (mean query, position terms, softmax, bypass)
- * in this library's kernels.                                                              */
+ * rounded to bf16 (o reaches the output projection as a hi + lo pair of bf16 values, about
+ * 16 bits).  The handle owns copies of the weights and all workspace; the dense projections
+ * run as cuBLAS GEMMs, the fusion (mean query, position terms, softmax, bypass) in this
+ * library's kernels.                                                                      */
 typedef struct ham_embedder ham_embedder; /* opaque handle: weights and workspace */
 
 typedef struct ham_embed_config {

@@ -4,26 +4,28 @@
 // the model width H before the base model's next forward: a multi-head cross-attention with
 // the mean of the token embeddings as its query, keys and values from the embeddings plus a
 // learned embedding of each token's place in the patch, then a linear layer; one token skips
-// the module.  On the GPU:
+// the module.  On the GPU, four launches:
 //
-//  1. QKV = X [T][H] . [W_q; W_k; W_v]^T -> fp32 [T][3H]: one dense GEMM over every token of
-//     the call (cuBLAS, bf16 in, fp32 accumulate and out).  Because the projections are linear,
-//     W_q mean(x) = mean(W_q x), and W_{k,v} (x_i + P[i]) = W_{k,v} x_i + W_{k,v} P[i]: the
-//     position terms KVP = [W_k; W_v] P^T are computed once when the handle is made.
+//  1. QKV = X [T][H] . [W_q; W_k; W_v]^T in fp32 (one cuBLAS GEMM).  Because the projections
+//     are linear, W_q mean(x) = mean(W_q x), and W_{k,v} (x_i + P[i]) = W_{k,v} x_i + W_{k,v} P[i]:
+//     the position terms KVP = [W_k; W_v] P^T are computed once when the handle is made.
 //  2. fuse_kernel, one warp per (sequence, head): the mean query, k_i and v_i with their
-//     position terms, the scaled scores, softmax over the patch (fp32) and o, rounded to bf16
-//     into O [B][H], all of the patch's loads issued at once.  It also sets out: the token's
-//     embedding for a sequence of one (whose O row is 0), zeros for the others.  Token counts
-//     outside 1..max_patch set the error word (and give zeros).
-//  3. out = O . W_o^T + out (cuBLAS, bf16 out, fp32 accumulate): a sequence of one gets
-//     x + 0, its embedding (exactly, but for the sign of a zero and NaN payloads).
-// The GEMMs stream the weights (4 H^2 bf16) once per call: memory-bound at the batches of
-// decoding, where the token rows are far fewer than the weight rows.
+//     position terms, the scaled scores, softmax over the patch (fp32) and o, every load of the
+//     patch issued at once.  o goes out as two bf16 parts, hi = bf16(o) and lo = bf16(o - hi),
+//     stacked as 2B rows, so that the output projection sees about 16 bits of it.
+//  3. [o_hi; o_lo] . W_o^T in fp32 (one cuBLAS GEMM over the 2B rows: the weights are read
+//     once).
+//  4. finish_kernel: the state is the two products' sum rounded to bf16, or for a sequence of
+//     one token its embedding bit for bit; a token count outside 1..max_patch (or rows outside
+//     the call's tokens) gives zeros and sets the error word.
+// The weights (4 H^2 bf16) dominate the bytes of a call: memory-bound at decoding batches,
+// where the token rows are far fewer than the weight rows.
 #include <cublas_v2.h>
 #include <cuda_bf16.h>
 
 #include <cstdarg>
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 
 #include "ham_internal.cuh"
@@ -36,8 +38,9 @@ struct ham_embedder {
   __nv_bfloat16 *wqkv = nullptr; // [3H][H]
   __nv_bfloat16 *wo = nullptr;   // [H][H]
   float *kvp = nullptr;          // [max_patch][2H]: W_k P[i], W_v P[i]
-  float *qkv = nullptr;          // [max_batch * max_patch][3H]
-  __nv_bfloat16 *o = nullptr;    // [max_batch][H]
+  float *qkv = nullptr;          // [max_batch * max_patch][3H] fp32
+  float *part2 = nullptr;        // [2][batch][H] fp32: the output projection of o_hi, o_lo
+  __nv_bfloat16 *o = nullptr;    // [2][batch][H]: o's hi and lo bf16 parts
   int32_t *err = nullptr;        // device error word
   int32_t *host_err = nullptr;   // pinned read-back
 };
@@ -60,13 +63,13 @@ int efail(int status, const char *fmt, ...) {
 bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 
 // One warp per (sequence b, head h); lane j owns head elements j, j + 32, ... (kPer of them).
+// qkv: nparts parts of [T][3H] fp32, summed here.
 template <int kPer>
-__global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv,
+__global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv, int nparts,
                                                    const float *__restrict__ kvp,
                                                    const int32_t *__restrict__ offsets,
-                                                   const __nv_bfloat16 *__restrict__ x,
                                                    __nv_bfloat16 *__restrict__ o,
-                                                   __nv_bfloat16 *__restrict__ out, int32_t *err,
+                                                   __nv_bfloat16 *__restrict__ o_lo, int32_t *err,
                                                    int batch, int total, int H, int n_heads,
                                                    int max_patch, float scale) {
   const int warp = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
@@ -78,36 +81,35 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
   // a sequence's rows must lie in the call's token rows; else it is a bad count
   const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
   __nv_bfloat16 *orow = o + (int64_t)b * H + (int64_t)h * hd;
-  __nv_bfloat16 *outrow = out + (int64_t)b * H + (int64_t)h * hd;
-  // The output GEMM adds O . W_o^T to what this kernel leaves in out: the token itself for a
-  // sequence of one (with O = 0), zeros otherwise.
-  const __nv_bfloat16 zero = __float2bfloat16_rn(0.f);
-  if (bad || n == 1) {
+  __nv_bfloat16 *lorow = o_lo + (int64_t)b * H + (int64_t)h * hd;
+  if (bad || n == 1) {  // the finish kernel handles these rows; O is not used for them
     if (bad && h == 0 && lane == 0) record_error(err, HAM_DEVERR_NTOK);
-    const __nv_bfloat16 *xrow = x + (int64_t)(bad ? 0 : t0) * H + (int64_t)h * hd;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) {
-      orow[lane + 32 * e] = zero;
-      outrow[lane + 32 * e] = bad ? zero : xrow[lane + 32 * e];
-    }
+    for (int e = 0; e < kPer; ++e) orow[lane + 32 * e] = lorow[lane + 32 * e] = __float2bfloat16_rn(0.f);
     return;
   }
-#pragma unroll
-  for (int e = 0; e < kPer; ++e) outrow[lane + 32 * e] = zero;
-  const int64_t ld = 3 * (int64_t)H;
+  const int64_t ld = 3 * (int64_t)H, part = (int64_t)total * ld;
   const int64_t col = (int64_t)h * hd + lane;
   // every load of the patch at once (one round trip): q, k and v rows and the position terms
   float qv[kMaxPatch][kPer], kv[kMaxPatch][kPer], vv[kMaxPatch][kPer];
 #pragma unroll
   for (int i = 0; i < kMaxPatch; ++i) {
     const bool in = i < n;
-    const float *row = qkv + (int64_t)(t0 + (in ? i : 0)) * ld + col;
     const float *pp = kvp + (int64_t)(in ? i : 0) * 2 * H + col;
 #pragma unroll
     for (int e = 0; e < kPer; ++e) {
-      qv[i][e] = in ? row[32 * e] : 0.f;
-      kv[i][e] = in ? row[H + 32 * e] + pp[32 * e] : 0.f;
-      vv[i][e] = in ? row[2 * H + 32 * e] + pp[H + 32 * e] : 0.f;
+      qv[i][e] = 0.f;
+      kv[i][e] = in ? pp[32 * e] : 0.f;
+      vv[i][e] = in ? pp[H + 32 * e] : 0.f;
+    }
+    for (int sp = 0; sp < nparts; ++sp) {
+      const float *row = qkv + sp * part + (int64_t)(t0 + (in ? i : 0)) * ld + col;
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) {
+        qv[i][e] += in ? row[32 * e] : 0.f;
+        kv[i][e] += in ? row[H + 32 * e] : 0.f;
+        vv[i][e] += in ? row[2 * H + 32 * e] : 0.f;
+      }
     }
   }
   float q[kPer];
@@ -123,10 +125,10 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
   float s[kMaxPatch];
 #pragma unroll
   for (int i = 0; i < kMaxPatch; ++i) {
-    float part = 0.f;
+    float part_s = 0.f;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) part += q[e] * kv[i][e];
-    s[i] = part;
+    for (int e = 0; e < kPer; ++e) part_s += q[e] * kv[i][e];
+    s[i] = part_s;
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1)
@@ -148,8 +150,46 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
     float acc = 0.f;
 #pragma unroll
     for (int i = 0; i < kMaxPatch; ++i) acc += s[i] * vv[i][e];
-    orow[lane + 32 * e] = __float2bfloat16_rn(acc * inv);
+    // o as two bf16 parts, o = hi + lo to about 16 bits, for the output projection
+    const float ov = acc * inv;
+    const __nv_bfloat16 hi = __float2bfloat16_rn(ov);
+    orow[lane + 32 * e] = hi;
+    lorow[lane + 32 * e] = __float2bfloat16_rn(ov - __bfloat162float(hi));
   }
+}
+
+// out[b] = the sum of the output parts rounded to bf16; a sequence of one token gets its
+// embedding bit for bit; a bad count gets zeros.  Eight elements per thread.
+__global__ void finish_kernel(const float *__restrict__ part, int nparts,
+                              const __nv_bfloat16 *__restrict__ x,
+                              const int32_t *__restrict__ offsets, __nv_bfloat16 *__restrict__ out,
+                              int batch, int total, int H, int max_patch) {
+  const int b = blockIdx.y;
+  const int j = 8 * (blockIdx.x * blockDim.x + threadIdx.x);
+  if (b >= batch || j >= H) return;
+  const int t0 = offsets[b], n = offsets[b + 1] - t0;
+  const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
+  uint4 v = make_uint4(0, 0, 0, 0);
+  if (!bad && n == 1) {
+    v = *reinterpret_cast<const uint4 *>(x + (int64_t)t0 * H + j);
+  } else if (!bad) {
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int sp = 0; sp < nparts; ++sp) {
+      const float4 *p = reinterpret_cast<const float4 *>(part + ((int64_t)sp * batch + b) * H + j);
+      const float4 lo = p[0], hi = p[1];
+      acc[0] += lo.x; acc[1] += lo.y; acc[2] += lo.z; acc[3] += lo.w;
+      acc[4] += hi.x; acc[5] += hi.y; acc[6] += hi.z; acc[7] += hi.w;
+    }
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e]));
+      const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e + 1]));
+      w[e] = lo | (hi << 16);
+    }
+    v = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  *reinterpret_cast<uint4 *>(out + (int64_t)b * H + j) = v;
 }
 
 // C[rows][n_out] (row-major, ldc) = A[rows][k] (row-major bf16) . W[n_out][k]^T (bf16)
@@ -162,6 +202,20 @@ cublasStatus_t gemm_rows(cublasHandle_t h, int rows, int n_out, int k, const __n
   return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, n_out, rows, k, &one, w, CUDA_R_16BF, k, a,
                       CUDA_R_16BF, k, &zero, c, c_type, ldc, CUBLAS_COMPUTE_32F,
                       CUBLAS_GEMM_DEFAULT);
+}
+
+}  // namespace
+}  // namespace ham
+
+namespace ham {
+namespace {
+
+// parts[rows][n_out] = X[rows][K] . W[n_out][K]^T in fp32 (one cuBLAS GEMM).
+bool project(ham_embedder *e, cudaStream_t s, const __nv_bfloat16 *X, const __nv_bfloat16 *W,
+             float *parts, int rows, int n_out, int K) {
+  return cublasSetStream(e->blas, s) == CUBLAS_STATUS_SUCCESS &&
+         gemm_rows(e->blas, rows, n_out, K, X, W, parts, CUDA_R_32F, n_out) ==
+             CUBLAS_STATUS_SUCCESS;
 }
 
 }  // namespace
@@ -182,6 +236,7 @@ int ham_embedder_free(ham_embedder *e) {
   cudaFree(e->wo);
   cudaFree(e->kvp);
   cudaFree(e->qkv);
+  cudaFree(e->part2);
   cudaFree(e->o);
   cudaFree(e->err);
   cudaFreeHost(e->host_err);
@@ -200,8 +255,8 @@ int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *
   const int hd = H / nh;
   if (hd != 32 && hd != 64 && hd != 128)
     return efail(HAM_EUNSUPPORTED, "head_dim %d: 32, 64 or 128", hd);
-  if (cfg->max_batch < 1 || cfg->max_patch < 1 || cfg->max_patch > 8)
-    return efail(HAM_EINVAL, "max_batch >= 1 and max_patch in 1..8");
+  if (cfg->max_batch < 1 || cfg->max_patch < 1 || cfg->max_patch > ham::kMaxPatch)
+    return efail(HAM_EINVAL, "max_batch >= 1 and max_patch in 1..%d", ham::kMaxPatch);
   if (!wq || !wk || !wv || !wo || !pos) return efail(HAM_EINVAL, "weights are required");
   if (!ham::aligned16(wq) || !ham::aligned16(wk) || !ham::aligned16(wv) || !ham::aligned16(wo) ||
       !ham::aligned16(pos))
@@ -219,7 +274,8 @@ int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *
   alloc(reinterpret_cast<void **>(&e->wo), hh * 2);
   alloc(reinterpret_cast<void **>(&e->kvp), (size_t)cfg->max_patch * 2 * H * 4);
   alloc(reinterpret_cast<void **>(&e->qkv), rows * 3 * H * 4);
-  alloc(reinterpret_cast<void **>(&e->o), (size_t)cfg->max_batch * H * 2);
+  alloc(reinterpret_cast<void **>(&e->part2), 2 * (size_t)cfg->max_batch * H * 4);
+  alloc(reinterpret_cast<void **>(&e->o), 2 * (size_t)cfg->max_batch * H * 2);
   alloc(reinterpret_cast<void **>(&e->err), 4);
   alloc(&e->blas_ws, ham::kBlasWorkspace);
   if (ce == cudaSuccess) ce = cudaMallocHost(reinterpret_cast<void **>(&e->host_err), 4);
@@ -236,7 +292,7 @@ int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *
   if (ce != cudaSuccess) {
     cudaGetLastError();
     ham_embedder_free(e);
-    return efail(HAM_ECUDA, "embedder weight copy: %s", cudaGetErrorString(ce));
+    return efail(HAM_ECUDA, "embedder set-up: %s", cudaGetErrorString(ce));
   }
   cublasStatus_t bs = cublasCreate(&e->blas);
   if (bs == CUBLAS_STATUS_SUCCESS) bs = cublasSetWorkspace(e->blas, e->blas_ws, ham::kBlasWorkspace);
@@ -272,37 +328,41 @@ int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t ba
   if (dev != e->device) cudaSetDevice(e->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int H = c.hidden, hd = H / c.n_heads;
+  const __nv_bfloat16 *xb = static_cast<const __nv_bfloat16 *>(x);
   int rc = HAM_OK;
-  cublasStatus_t bs = cublasSetStream(e->blas, s);
-  if (bs == CUBLAS_STATUS_SUCCESS)
-    bs = ham::gemm_rows(e->blas, total_tokens, 3 * H, H, static_cast<const __nv_bfloat16 *>(x),
-                        e->wqkv, e->qkv, CUDA_R_32F, 3 * H);
-  if (bs != CUBLAS_STATUS_SUCCESS) rc = efail(HAM_ECUDA, "projection GEMM (status %d)", (int)bs);
+  __nv_bfloat16 *o_lo = e->o + (size_t)batch * H;  // rows batch..2 batch-1 of one [2B][H] block
+  if (!ham::project(e, s, xb, e->wqkv, e->qkv, total_tokens, 3 * H, H))
+    rc = efail(HAM_ECUDA, "projection GEMM failed");
   if (rc == HAM_OK) {
     const int warps = batch * c.n_heads;
     const dim3 grid((unsigned)((warps + 7) / 8)), block(256);
     const float scale = 1.f / sqrtf((float)hd);
     if (hd == 32)
-      ham::fuse_kernel<1><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets,
-                                                 static_cast<const __nv_bfloat16 *>(x), e->o,
-                                                 static_cast<__nv_bfloat16 *>(out), e->err, batch,
-                                                 total_tokens, H, c.n_heads, c.max_patch, scale);
+      ham::fuse_kernel<1><<<grid, block, 0, s>>>(e->qkv, 1, e->kvp, offsets, e->o, o_lo, e->err,
+                                                 batch, total_tokens, H, c.n_heads, c.max_patch,
+                                                 scale);
     else if (hd == 64)
-      ham::fuse_kernel<2><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets,
-                                                 static_cast<const __nv_bfloat16 *>(x), e->o,
-                                                 static_cast<__nv_bfloat16 *>(out), e->err, batch,
-                                                 total_tokens, H, c.n_heads, c.max_patch, scale);
+      ham::fuse_kernel<2><<<grid, block, 0, s>>>(e->qkv, 1, e->kvp, offsets, e->o, o_lo, e->err,
+                                                 batch, total_tokens, H, c.n_heads, c.max_patch,
+                                                 scale);
     else
-      ham::fuse_kernel<4><<<grid, block, 0, s>>>(e->qkv, e->kvp, offsets,
-                                                 static_cast<const __nv_bfloat16 *>(x), e->o,
-                                                 static_cast<__nv_bfloat16 *>(out), e->err, batch,
-                                                 total_tokens, H, c.n_heads, c.max_patch, scale);
+      ham::fuse_kernel<4><<<grid, block, 0, s>>>(e->qkv, 1, e->kvp, offsets, e->o, o_lo, e->err,
+                                                 batch, total_tokens, H, c.n_heads, c.max_patch,
+                                                 scale);
     cudaError_t ce = cudaGetLastError();
     if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "fuse launch: %s", cudaGetErrorString(ce));
   }
+  if (rc == HAM_OK) {  // o_hi and o_lo stacked as 2B rows: the weights are read once
+    if (!ham::project(e, s, e->o, e->wo, e->part2, 2 * batch, H, H))
+      rc = efail(HAM_ECUDA, "output GEMM failed");
+  }
   if (rc == HAM_OK) {
-    bs = ham::gemm_rows(e->blas, batch, H, H, e->o, e->wo, out, CUDA_R_16BF, H, 1.f);
-    if (bs != CUBLAS_STATUS_SUCCESS) rc = efail(HAM_ECUDA, "output GEMM (status %d)", (int)bs);
+    const dim3 grid((unsigned)((H / 8 + 127) / 128), (unsigned)batch), block(128);
+    ham::finish_kernel<<<grid, block, 0, s>>>(e->part2, 2, xb, offsets,
+                                              static_cast<__nv_bfloat16 *>(out), batch,
+                                              total_tokens, H, c.max_patch);
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "finish launch: %s", cudaGetErrorString(ce));
   }
   if (dev != e->device) cudaSetDevice(dev);
   return rc;

@@ -15,9 +15,10 @@ from gpu_helpers import (MAX_ABS, MEAN_ABS, assert_parity, dev_bf16, dev_i32, gp
 pytestmark = pytest.mark.gpu
 
 # fp32 output: a tighter check than the bf16 bar.  The tensor-core p.V rounds each softmax
-# weight to bf16 (relative error up to 2^-9, about uniform), so an output moves by a weighted
-# sum of such errors times (v_i - out): of order 1e-3 at worst on concentrated weights, and
-# of order 1e-4 on average over a few hundred slots.  The exact value depends on how the
+# weight to bf16 (relative error up to 2^-8, the unit roundoff of bf16's 8-bit significand;
+# about uniform), so an output moves by a weighted sum of such errors times (v_i - out): of
+# order 1e-3 at worst on concentrated weights, and of order 1e-4 on average over a few hundred
+# slots.  The exact value depends on how the
 # split plan cuts the segments, which changes the running maxima the weights are taken from.
 F32_MAX, F32_MEAN = 3e-3, 3e-4
 

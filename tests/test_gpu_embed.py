@@ -11,12 +11,11 @@ from gpu_helpers import MEAN_ABS, dev_bf16, dev_i32, host_bits, torch
 
 pytestmark = pytest.mark.gpu
 
-# Tolerance from the arithmetic: the GPU rounds o to bf16 before the output projection and the
-# state to bf16 at the end, each a relative error of at most 2^-9; through W_o (rows of norm
-# ~1) the first moves an element by about 2^-9 of the state's size, so the error is about
-# 2 * 2^-9 ~ 0.4% of |state| at worst.  States reach magnitude 4-5, so the bar is relative:
-# |got - ref| <= REL * max(1, |ref|) per element (REL = 1e-2, ~2.5x that), and the bf16 mean-abs
-# bar on average.
+# Tolerance from the arithmetic: projections and attention accumulate in fp32, o reaches the
+# output projection as a hi + lo pair of bf16 values (about 16 bits), and the state is rounded
+# to bf16 once at the end: a relative error of at most 2^-8 (bf16's unit roundoff), 0.39% of
+# |state|.  States reach magnitude 4-5, so the bar is relative: |got - ref| <= REL * max(1,
+# |ref|) per element (REL = 1e-2, ~2.5x that), and the bf16 mean-abs bar on average.
 REL = 1e-2
 
 
@@ -52,7 +51,12 @@ def _check(c, out):
         assert np.array_equal(bits[b], c.x[c.offsets[b]]), f"bypass row {b}"
 
 
-@pytest.mark.parametrize("batch,hidden,heads", [(64, 2048, 32), (8, 256, 8), (5, 512, 4)])
+@pytest.mark.parametrize("batch,hidden,heads", [
+    (64, 2048, 32),    # the Llama-3.2-1B width; ~122 tokens: both projections streamed
+    (8, 256, 8), (5, 512, 4), (12, 320, 10),   # head dims 32 / 128; one K split (5 chunks)
+    (100, 512, 8),     # ~187 tokens: cuBLAS Q/K/V, streamed output projection
+    (160, 256, 8),     # both projections through cuBLAS
+])
 def test_embed_matches_oracle(batch, hidden, heads):
     c = wl.make_embed_case(wl.embed_workload(batch, hidden=hidden, n_heads=heads, seed=batch))
     e, out = _run(c)
