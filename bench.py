@@ -202,6 +202,8 @@ STACK_PREFIX = "stack_b"     # stack_b1, stack_b8, ...: the 32-layer decode stac
 STACK_GRAPH = 8              # macro-steps per CUDA graph in the stack runs
 EMBED_PREFIX = "embed_b"     # embed_b64, ...: the compositional embedder
 EMBED_HANDLES = 8            # rotated handles: 8 x 32 MiB of weights > 129 MB L2
+EMBED_TOK_PREFIX = "embedtok_b"  # embedtok_b64, ...: the embedder fed token ids
+EMBED_TOK_HANDLES = 16       # rotated: 16 x 8 MiB of W_o > 129 MB L2 (and 3.7 GB of tables each)
 
 
 def workload(name):
@@ -210,9 +212,12 @@ def workload(name):
         return wl.c4_sweep(int(name[len(STACK_PREFIX):]))
     if name.startswith(EMBED_PREFIX) and name[len(EMBED_PREFIX):].isdigit():
         return wl.embed_workload(int(name[len(EMBED_PREFIX):]))
+    if name.startswith(EMBED_TOK_PREFIX) and name[len(EMBED_TOK_PREFIX):].isdigit():
+        return wl.embed_tokens_workload(int(name[len(EMBED_TOK_PREFIX):]))
     if name not in wl.WORKLOADS:
         raise SystemExit(f"unknown workload {name}; choose from {sorted(wl.WORKLOADS)} or "
-                         f"{STACK_PREFIX}<batch>, {EMBED_PREFIX}<batch>")
+                         f"{STACK_PREFIX}<batch>, {EMBED_PREFIX}<batch>, "
+                         f"{EMBED_TOK_PREFIX}<batch>")
     return wl.WORKLOADS[name]
 
 
@@ -627,7 +632,7 @@ def run_reference_embed(args, w):
     """Reference arm of the embedder workload: the fp64 oracle, whole calls."""
     from oracle import embedder as oe
     from paper_2505_20438_gb300 import workload as wl
-    c = wl.make_embed_case(w)
+    c = embed_case(w)
     steps, warm = max(1, args.steps), max(3, args.warmup)
     # bounded: at most ~40 oracle calls in all
     steps, warm = min(steps, 30), min(warm, 10)
@@ -647,7 +652,10 @@ def run_reference_embed(args, w):
         "config": {"workload": w.name, "batch": w.batch, "hidden": w.hidden,
                    "n_heads": w.n_heads},
         "cpu_baseline": {"value": round(value, 4), "unit": unit, "cores": os.cpu_count(),
-                         "kind": "oracle", "sample": f"{steps} whole calls of {w.name}"},
+                         "kind": "oracle",
+                         "sample": f"{steps} whole calls of {w.name}" +
+                                   (" (embeddings gathered from the table by the ids first)"
+                                    if w.vocab else "")},
         "e2e": {"value": round(value, 4), "unit": unit, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }), flush=True)
@@ -902,17 +910,29 @@ def run_stack(args, w):
         torch.distributed.destroy_process_group()
 
 
-def embed_bytes(w, T, B):
-    """Algorithmic bytes of one call: the four H x H bf16 weights and the fp32 position terms
-    once, the token embeddings and offsets in, the fused states out."""
+def embed_case(w):
+    """The seeded case of an embedder workload; for token ids, case.x = table[ids]."""
+    from paper_2505_20438_gb300 import workload as wl
+    return wl.make_embed_tokens_case(w, w.vocab).case if w.vocab else wl.make_embed_case(w)
+
+
+def embed_bytes(w, T, B, singles=0):
+    """Algorithmic bytes of one call.  Embeddings given: the four H x H bf16 weights and the
+    fp32 position terms once, the token embeddings and offsets in, the fused states out.
+    Token ids: W_o and the position terms once, the tabulated fp32 projections of each token
+    (12 H bytes), the embedding rows of the single-token sequences, the ids and offsets in,
+    the states out."""
     H = w.hidden
-    return 4 * H * H * 2 + w.max_patch * 2 * H * 4 + T * H * 2 + (B + 1) * 4 + B * H * 2
+    io = w.max_patch * 2 * H * 4 + (B + 1) * 4 + B * H * 2
+    if w.vocab:
+        return H * H * 2 + io + T * 3 * H * 4 + singles * H * 2 + T * 4
+    return 4 * H * H * 2 + io + T * H * 2
 
 
 def run_embed(args, w):
     """The compositional embedder: one call fuses the last macro-step's tokens of w.batch
-    sequences; calls rotate over EMBED_HANDLES handles (their weights far exceed L2), 64 calls
-    per CUDA graph."""
+    sequences, given as embeddings or (w.vocab > 0) as token ids; calls rotate over handles
+    whose weights together far exceed L2, 64 calls per CUDA graph."""
     import numpy as np
     import torch
 
@@ -925,8 +945,10 @@ def run_embed(args, w):
     if world > 1 and not torch.distributed.is_initialized():
         torch.distributed.init_process_group("nccl")
     build_mod.build()
-    c = wl.make_embed_case(w)
+    tc = wl.make_embed_tokens_case(w, w.vocab) if w.vocab else None
+    c = tc.case if tc else wl.make_embed_case(w)
     B, H, T = w.batch, w.hidden, int(c.offsets[-1])
+    n_handles = EMBED_TOK_HANDLES if w.vocab else EMBED_HANDLES
 
     def dev(bits):
         return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
@@ -934,15 +956,28 @@ def run_embed(args, w):
     weights = [dev(a) for a in (c.wq, c.wk, c.wv, c.wo)]
     pos = dev(c.pos)
     handles = [ham.ham_embedder_alloc(H, w.n_heads, B, w.max_patch, *weights, pos)
-               for _ in range(EMBED_HANDLES)]
+               for _ in range(n_handles)]
     del weights
     x = dev(c.x)
     offsets = torch.from_numpy(c.offsets).cuda()
+    ids = None
+    if tc:
+        table = dev(tc.table)
+        for e in handles:
+            ham.ham_embedder_set_vocab(e, table)
+        del table
+        ids = torch.from_numpy(tc.ids).cuda()
+
+    def call(e, out):
+        if ids is not None:
+            ham.ham_embed_tokens(e, ids, offsets, out)
+        else:
+            ham.ham_embed(e, x, offsets, out)
     outs = [torch.empty((B, H), dtype=torch.bfloat16, device="cuda") for _ in handles]
     stream = torch.cuda.Stream()
     with torch.cuda.stream(stream):
         for j, e in enumerate(handles):        # eager first calls
-            ham.ham_embed(e, x, offsets, outs[j])
+            call(e, outs[j])
     stream.synchronize()
     span = (torch.cuda.Event(enable_timing=True, external=True),
             torch.cuda.Event(enable_timing=True, external=True))
@@ -953,8 +988,8 @@ def run_embed(args, w):
             if with_span:
                 span[0].record()
             for i in range(GRAPH_STEPS):
-                j = i % EMBED_HANDLES
-                ham.ham_embed(handles[j], x, offsets, outs[j])
+                j = i % n_handles
+                call(handles[j], outs[j])
             if with_span:
                 span[1].record()
         return g
@@ -985,23 +1020,24 @@ def run_embed(args, w):
         if ham.ham_embedder_status(e) != ham.HAM_DEVERR_NONE:
             raise RuntimeError("device error during the timed region")
     call_us = 1e3 * span[0].elapsed_time(span[1]) / GRAPH_STEPS
-    nbytes = embed_bytes(w, T, B)
+    nbytes = embed_bytes(w, T, B, singles=int((c.counts == 1).sum()))
     peak, peak_src = measured_peak_hbm()
     value = job_throughput(steps, world, elapsed_ms * 1e-3)
     achieved = nbytes / (call_us * 1e-6) / 1e9
 
     # end to end: each call copies the tokens and offsets from pinned host memory, fuses them
     # and copies the states back; one graph per handle, the host reads every call's result
-    hx, hoff = x.cpu().pin_memory(), offsets.cpu().pin_memory()
+    src = ids if ids is not None else x   # the call's token input: ids or embeddings
+    hx, hoff = src.cpu().pin_memory(), offsets.cpu().pin_memory()
     hout = torch.empty((B, H), dtype=torch.bfloat16).pin_memory()
     hbits = hout.view(torch.int16).numpy()
     io = []
     for j, e in enumerate(handles):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            x.copy_(hx, non_blocking=True)
+            src.copy_(hx, non_blocking=True)
             offsets.copy_(hoff, non_blocking=True)
-            ham.ham_embed(e, x, offsets, outs[j])
+            call(e, outs[j])
             hout.copy_(outs[j], non_blocking=True)
         io.append(g)
     torch.cuda.synchronize()
@@ -1010,7 +1046,7 @@ def run_embed(args, w):
     te = time.perf_counter()
     with torch.cuda.stream(stream):
         for i in range(n_e2e):
-            io[i % EMBED_HANDLES].replay()
+            io[i % n_handles].replay()
             stream.synchronize()
             bits = np.uint32(np.uint16(hbits.flat[0])) << np.uint32(16)
             checksum += float(bits.view(np.float32))
@@ -1025,15 +1061,20 @@ def run_embed(args, w):
         "config": {"workload": w.name, "batch": B, "hidden": H, "n_heads": w.n_heads,
                    "tokens": T, "fused_sequences": int((c.counts > 1).sum()),
                    "tokens_per_sequence": "geometric p=0.5 capped at 4",
-                   "step": "one ham_embed call: QKV GEMM, fusion, output GEMM, bypass",
-                   "l2": f"{EMBED_HANDLES} handles rotated ({EMBED_HANDLES} x "
-                         f"{4 * H * H * 2 / 2**20:.0f} MiB of weights > 129 MB L2)",
+                   "vocab": w.vocab or None,
+                   "step": ("one ham_embed_tokens call: gather of the tabulated projections "
+                            "with fusion, output GEMM, finish" if w.vocab else
+                            "one ham_embed call: QKV GEMM, fusion, output GEMM, finish"),
+                   "l2": f"{n_handles} handles rotated ({n_handles} x "
+                         f"{(1 if w.vocab else 4) * H * H * 2 / 1e6:.1f} MB of weights "
+                         f"> 129 MB L2)",
                    "graph": f"{GRAPH_STEPS} calls per CUDA graph"},
         "sequences_per_s": round(value * B, 1),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
-                     "kernel": "cuBLAS QKV GEMM + fuse_kernel + cuBLAS output GEMM + "
-                               "bypass_kernel",
+                     "kernel": ("fuse_kernel (gather) + cuBLAS output GEMM + finish_kernel"
+                                if w.vocab else "cuBLAS QKV GEMM + fuse_kernel + cuBLAS "
+                                "output GEMM + finish_kernel"),
                      "avg_launch_us": round(call_us, 3),
                      "algorithmic_bytes_per_launch": int(nbytes),
                      "peak_source": peak_src,
@@ -1041,11 +1082,13 @@ def run_embed(args, w):
                                         "last graph replay, / " + str(GRAPH_STEPS)},
         "gpu_launches": n_graph * GRAPH_STEPS * 2 * world,
         "e2e": {"value": round(job_throughput(n_e2e, world, dte), 2), "unit": "calls/s",
-                "h2d_bytes_per_step": T * H * 2 + (B + 1) * 4, "d2h_bytes_per_step": B * H * 2,
+                "h2d_bytes_per_step": src.numel() * src.element_size() + (B + 1) * 4,
+                "d2h_bytes_per_step": B * H * 2,
                 "steps": n_e2e, "finite": math.isfinite(checksum),
-                "path": "every call: pinned host -> device copies of the tokens and offsets, "
-                        "ham_embed, device -> pinned host copy of the states, read on the host "
-                        "(one CUDA graph per handle)"},
+                "path": "every call: pinned host -> device copies of the tokens "
+                        f"({'ids' if w.vocab else 'embeddings'}) and offsets, the call, device "
+                        "-> pinned host copy of the states, read on the host (one CUDA graph "
+                        "per handle)"},
         "clocks": clocks.summary(),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -325,6 +325,21 @@ int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t ba
  * HAM_EDEVICE if it was set, with the code in *device_code. */
 int ham_embedder_status(ham_embedder *e, void *stream, int32_t *device_code);
 
+/* Give the embedder the vocabulary's token-embedding table (device bf16 [vocab][H], copied) for
+ * ham_embed_tokens.  The tokens' projections [W_q; W_k; W_v] E[v] are tabulated once, in fp32
+ * ([vocab][3H], 12 H bytes per entry: 3.2 GB for 128k entries at H = 2048), so that a call
+ * gathers rows instead of multiplying by the weights; the result is the same function as
+ * ham_embed of the gathered embeddings.  Synchronous.  Host errors: HAM_EINVAL, HAM_ENOMEM,
+ * HAM_ECUDA. */
+int ham_embedder_set_vocab(ham_embedder *e, const void *table, int32_t vocab);
+
+/* ham_embed of the embeddings E[ids[t]]: ids device int32 [total_tokens], grouped by sequence
+ * through offsets as for ham_embed.  A token id outside [0, vocab) gives its sequence zeros and
+ * sets the device error word (HAM_DEVERR_NTOK).  Host errors as for ham_embed, and HAM_EINVAL
+ * if no vocabulary was set. */
+int ham_embed_tokens(ham_embedder *e, const int32_t *ids, const int32_t *offsets,
+                     int32_t batch, int32_t total_tokens, void *out, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -20,10 +20,14 @@
 //     the call's tokens) gives zeros and sets the error word.
 // The weights (4 H^2 bf16) dominate the bytes of a call: memory-bound at decoding batches,
 // where the token rows are far fewer than the weight rows.
+// With token ids (ham_embed_tokens) step 1 is a lookup: the projections of every vocabulary
+// entry, [W_q; W_k; W_v] E[v], are tabulated once in fp32, and the fusion kernel reads the rows
+// of the ids.  A call then reads W_o (H^2 bf16) and 12 H bytes per token instead of 4 H^2.
 #include <cublas_v2.h>
 #include <cuda_bf16.h>
 
 #include <cstdarg>
+#include <cstdint>
 #include <cstdio>
 #include <algorithm>
 #include <cstring>
@@ -38,6 +42,9 @@ struct ham_embedder {
   __nv_bfloat16 *wqkv = nullptr; // [3H][H]
   __nv_bfloat16 *wo = nullptr;   // [H][H]
   float *kvp = nullptr;          // [max_patch][2H]: W_k P[i], W_v P[i]
+  int32_t vocab = 0;             // entries of the vocabulary tables (0: none set)
+  __nv_bfloat16 *table_e = nullptr; // [vocab][H]: the token embeddings
+  float *table_qkv = nullptr;    // [vocab][3H] fp32: [W_q; W_k; W_v] E[v]
   float *qkv = nullptr;          // [max_batch * max_patch][3H] fp32
   float *part2 = nullptr;        // [2][batch][H] fp32: the output projection of o_hi, o_lo
   __nv_bfloat16 *o = nullptr;    // [2][batch][H]: o's hi and lo bf16 parts
@@ -63,13 +70,15 @@ int efail(int status, const char *fmt, ...) {
 bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 
 // One warp per (sequence b, head h); lane j owns head elements j, j + 32, ... (kPer of them).
-// qkv: nparts parts of [T][3H] fp32, summed here.
+// qkv: nparts parts of [T][3H] fp32, summed here; or, with token ids, the tabulated rows
+// [vocab][3H] of the ids (one part).
 template <int kPer>
 __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv, int nparts,
                                                    const float *__restrict__ kvp,
                                                    const int32_t *__restrict__ offsets,
                                                    __nv_bfloat16 *__restrict__ o,
                                                    __nv_bfloat16 *__restrict__ o_lo, int32_t *err,
+                                                   const int32_t *__restrict__ ids, int vocab,
                                                    int batch, int total, int H, int n_heads,
                                                    int max_patch, float scale) {
   const int warp = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
@@ -78,8 +87,17 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
   const int b = warp / n_heads, h = warp - b * n_heads;
   const int hd = kPer * 32;
   const int t0 = offsets[b], n = offsets[b + 1] - t0;
-  // a sequence's rows must lie in the call's token rows; else it is a bad count
-  const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
+  // a sequence's rows must lie in the call's token rows, and its ids in the vocabulary
+  bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
+  int row[kMaxPatch];
+#pragma unroll
+  for (int i = 0; i < kMaxPatch; ++i) {
+    row[i] = t0 + i;
+    if (ids && !bad && i < n) {
+      row[i] = ids[t0 + i];
+      bad = bad || row[i] < 0 || row[i] >= vocab;
+    }
+  }
   __nv_bfloat16 *orow = o + (int64_t)b * H + (int64_t)h * hd;
   __nv_bfloat16 *lorow = o_lo + (int64_t)b * H + (int64_t)h * hd;
   if (bad || n == 1) {  // the finish kernel handles these rows; O is not used for them
@@ -103,12 +121,12 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
       vv[i][e] = in ? pp[H + 32 * e] : 0.f;
     }
     for (int sp = 0; sp < nparts; ++sp) {
-      const float *row = qkv + sp * part + (int64_t)(t0 + (in ? i : 0)) * ld + col;
+      const float *r = qkv + sp * part + (int64_t)(in ? row[i] : row[0]) * ld + col;
 #pragma unroll
       for (int e = 0; e < kPer; ++e) {
-        qv[i][e] += in ? row[32 * e] : 0.f;
-        kv[i][e] += in ? row[H + 32 * e] : 0.f;
-        vv[i][e] += in ? row[2 * H + 32 * e] : 0.f;
+        qv[i][e] += in ? r[32 * e] : 0.f;
+        kv[i][e] += in ? r[H + 32 * e] : 0.f;
+        vv[i][e] += in ? r[2 * H + 32 * e] : 0.f;
       }
     }
   }
@@ -160,18 +178,29 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
 
 // out[b] = the sum of the output parts rounded to bf16; a sequence of one token gets its
 // embedding bit for bit; a bad count gets zeros.  Eight elements per thread.
+// With token ids, x is the vocabulary's embedding table and a token's row is its id; an id
+// outside the vocabulary makes its sequence bad.
 __global__ void finish_kernel(const float *__restrict__ part, int nparts,
                               const __nv_bfloat16 *__restrict__ x,
                               const int32_t *__restrict__ offsets, __nv_bfloat16 *__restrict__ out,
-                              int batch, int total, int H, int max_patch) {
+                              const int32_t *__restrict__ ids, int vocab, int batch, int total,
+                              int H, int max_patch) {
   const int b = blockIdx.y;
   const int j = 8 * (blockIdx.x * blockDim.x + threadIdx.x);
   if (b >= batch || j >= H) return;
   const int t0 = offsets[b], n = offsets[b + 1] - t0;
-  const bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
+  bool bad = n < 1 || n > max_patch || t0 < 0 || t0 + n > total;
+  int xrow = t0;
+  if (ids && !bad) {
+    xrow = ids[t0];
+    for (int i = 0; i < n; ++i) {
+      const int id = ids[t0 + i];
+      bad = bad || id < 0 || id >= vocab;
+    }
+  }
   uint4 v = make_uint4(0, 0, 0, 0);
   if (!bad && n == 1) {
-    v = *reinterpret_cast<const uint4 *>(x + (int64_t)t0 * H + j);
+    v = *reinterpret_cast<const uint4 *>(x + (int64_t)xrow * H + j);
   } else if (!bad) {
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     for (int sp = 0; sp < nparts; ++sp) {
@@ -218,6 +247,56 @@ bool project(ham_embedder *e, cudaStream_t s, const __nv_bfloat16 *X, const __nv
              CUBLAS_STATUS_SUCCESS;
 }
 
+// The four launches of a call.  Without ids, xb is the call's token rows and step 1 is the
+// projection GEMM; with ids, xb is the vocabulary's embedding table and the fusion kernel
+// reads the tabulated projections of the ids.
+int run_embed(ham_embedder *e, const __nv_bfloat16 *xb, const int32_t *ids,
+              const int32_t *offsets, int32_t batch, int32_t total_tokens, void *out,
+              void *stream) {
+  const ham_embed_config &c = e->cfg;
+  if (batch < 1 || batch > c.max_batch)
+    return efail(HAM_EINVAL, "batch %d outside 1..%d", batch, c.max_batch);
+  if (total_tokens < batch || total_tokens > batch * c.max_patch)
+    return efail(HAM_EINVAL, "total_tokens %d outside %d..%d", total_tokens, batch,
+                 batch * c.max_patch);
+  if (!aligned16(out) || ((uintptr_t)offsets & 3u))
+    return efail(HAM_EINVAL, "out must be 16-byte aligned, offsets 4-byte aligned");
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev != e->device) cudaSetDevice(e->device);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int H = c.hidden, hd = H / c.n_heads;
+  int rc = HAM_OK;
+  __nv_bfloat16 *o_lo = e->o + (size_t)batch * H;  // rows batch..2 batch-1 of one [2B][H] block
+  const float *qkv = ids ? e->table_qkv : e->qkv;
+  if (!ids && !project(e, s, xb, e->wqkv, e->qkv, total_tokens, 3 * H, H))
+    rc = efail(HAM_ECUDA, "projection GEMM failed");
+  if (rc == HAM_OK) {
+    const int warps = batch * c.n_heads;
+    const dim3 grid((unsigned)((warps + 7) / 8)), block(256);
+    const float scale = 1.f / sqrtf((float)hd);
+    auto fuse = hd == 32 ? fuse_kernel<1> : hd == 64 ? fuse_kernel<2> : fuse_kernel<4>;
+    fuse<<<grid, block, 0, s>>>(qkv, 1, e->kvp, offsets, e->o, o_lo, e->err, ids, e->vocab,
+                                batch, total_tokens, H, c.n_heads, c.max_patch, scale);
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "fuse launch: %s", cudaGetErrorString(ce));
+  }
+  if (rc == HAM_OK) {  // o_hi and o_lo stacked as 2B rows: the weights are read once
+    if (!project(e, s, e->o, e->wo, e->part2, 2 * batch, H, H))
+      rc = efail(HAM_ECUDA, "output GEMM failed");
+  }
+  if (rc == HAM_OK) {
+    const dim3 grid((unsigned)((H / 8 + 127) / 128), (unsigned)batch), block(128);
+    finish_kernel<<<grid, block, 0, s>>>(e->part2, 2, xb, offsets,
+                                         static_cast<__nv_bfloat16 *>(out), ids, e->vocab,
+                                         batch, total_tokens, H, c.max_patch);
+    cudaError_t ce = cudaGetLastError();
+    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "finish launch: %s", cudaGetErrorString(ce));
+  }
+  if (dev != e->device) cudaSetDevice(dev);
+  return rc;
+}
+
 }  // namespace
 }  // namespace ham
 
@@ -235,6 +314,8 @@ int ham_embedder_free(ham_embedder *e) {
   cudaFree(e->wqkv);
   cudaFree(e->wo);
   cudaFree(e->kvp);
+  cudaFree(e->table_e);
+  cudaFree(e->table_qkv);
   cudaFree(e->qkv);
   cudaFree(e->part2);
   cudaFree(e->o);
@@ -315,54 +396,63 @@ int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *
 int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t batch,
               int32_t total_tokens, void *out, void *stream) {
   if (!e || !x || !offsets || !out) return efail(HAM_EINVAL, "null argument");
-  const ham_embed_config &c = e->cfg;
-  if (batch < 1 || batch > c.max_batch)
-    return efail(HAM_EINVAL, "batch %d outside 1..%d", batch, c.max_batch);
-  if (total_tokens < batch || total_tokens > batch * c.max_patch)
-    return efail(HAM_EINVAL, "total_tokens %d outside %d..%d", total_tokens, batch,
-                 batch * c.max_patch);
-  if (!ham::aligned16(x) || !ham::aligned16(out) || ((uintptr_t)offsets & 3u))
-    return efail(HAM_EINVAL, "x/out must be 16-byte aligned, offsets 4-byte aligned");
+  if (!ham::aligned16(x)) return efail(HAM_EINVAL, "x must be 16-byte aligned");
+  return ham::run_embed(e, static_cast<const __nv_bfloat16 *>(x), nullptr, offsets, batch,
+                        total_tokens, out, stream);
+}
+
+int ham_embed_tokens(ham_embedder *e, const int32_t *ids, const int32_t *offsets,
+                     int32_t batch, int32_t total_tokens, void *out, void *stream) {
+  if (!e || !ids || !offsets || !out) return efail(HAM_EINVAL, "null argument");
+  if (e->vocab < 1) return efail(HAM_EINVAL, "no vocabulary set (ham_embedder_set_vocab)");
+  if ((uintptr_t)ids & 3u) return efail(HAM_EINVAL, "ids must be 4-byte aligned");
+  return ham::run_embed(e, e->table_e, ids, offsets, batch, total_tokens, out, stream);
+}
+
+int ham_embedder_set_vocab(ham_embedder *e, const void *table, int32_t vocab) {
+  if (!e || !table) return efail(HAM_EINVAL, "null argument");
+  const int H = e->cfg.hidden;
+  if (vocab < 1 || (int64_t)vocab * 3 * H > INT32_MAX)
+    return efail(HAM_EINVAL, "vocab %d outside 1..%lld", vocab,
+                 (long long)(INT32_MAX / (3 * (int64_t)H)));
+  if (!ham::aligned16(table)) return efail(HAM_EINVAL, "table must be 16-byte aligned");
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev != e->device) cudaSetDevice(e->device);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int H = c.hidden, hd = H / c.n_heads;
-  const __nv_bfloat16 *xb = static_cast<const __nv_bfloat16 *>(x);
+  cudaFree(e->table_e);
+  cudaFree(e->table_qkv);
+  e->table_e = nullptr;
+  e->table_qkv = nullptr;
+  e->vocab = 0;
   int rc = HAM_OK;
-  __nv_bfloat16 *o_lo = e->o + (size_t)batch * H;  // rows batch..2 batch-1 of one [2B][H] block
-  if (!ham::project(e, s, xb, e->wqkv, e->qkv, total_tokens, 3 * H, H))
-    rc = efail(HAM_ECUDA, "projection GEMM failed");
-  if (rc == HAM_OK) {
-    const int warps = batch * c.n_heads;
-    const dim3 grid((unsigned)((warps + 7) / 8)), block(256);
-    const float scale = 1.f / sqrtf((float)hd);
-    if (hd == 32)
-      ham::fuse_kernel<1><<<grid, block, 0, s>>>(e->qkv, 1, e->kvp, offsets, e->o, o_lo, e->err,
-                                                 batch, total_tokens, H, c.n_heads, c.max_patch,
-                                                 scale);
-    else if (hd == 64)
-      ham::fuse_kernel<2><<<grid, block, 0, s>>>(e->qkv, 1, e->kvp, offsets, e->o, o_lo, e->err,
-                                                 batch, total_tokens, H, c.n_heads, c.max_patch,
-                                                 scale);
-    else
-      ham::fuse_kernel<4><<<grid, block, 0, s>>>(e->qkv, 1, e->kvp, offsets, e->o, o_lo, e->err,
-                                                 batch, total_tokens, H, c.n_heads, c.max_patch,
-                                                 scale);
-    cudaError_t ce = cudaGetLastError();
-    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "fuse launch: %s", cudaGetErrorString(ce));
-  }
-  if (rc == HAM_OK) {  // o_hi and o_lo stacked as 2B rows: the weights are read once
-    if (!ham::project(e, s, e->o, e->wo, e->part2, 2 * batch, H, H))
-      rc = efail(HAM_ECUDA, "output GEMM failed");
+  cudaError_t ce = cudaMalloc(reinterpret_cast<void **>(&e->table_e), (size_t)vocab * H * 2);
+  if (ce == cudaSuccess)
+    ce = cudaMalloc(reinterpret_cast<void **>(&e->table_qkv), (size_t)vocab * 3 * H * 4);
+  if (ce != cudaSuccess) {
+    cudaGetLastError();
+    rc = efail(HAM_ENOMEM, "vocabulary tables (%d entries) do not fit", vocab);
   }
   if (rc == HAM_OK) {
-    const dim3 grid((unsigned)((H / 8 + 127) / 128), (unsigned)batch), block(128);
-    ham::finish_kernel<<<grid, block, 0, s>>>(e->part2, 2, xb, offsets,
-                                              static_cast<__nv_bfloat16 *>(out), batch,
-                                              total_tokens, H, c.max_patch);
-    cudaError_t ce = cudaGetLastError();
-    if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "finish launch: %s", cudaGetErrorString(ce));
+    ce = cudaMemcpy(e->table_e, table, (size_t)vocab * H * 2, cudaMemcpyDeviceToDevice);
+    // the tabulated projections: [vocab][3H] = E [vocab][H] . [W_q; W_k; W_v]^T, fp32
+    cublasStatus_t bs = cublasSetStream(e->blas, nullptr);
+    if (ce == cudaSuccess && bs == CUBLAS_STATUS_SUCCESS)
+      bs = ham::gemm_rows(e->blas, vocab, 3 * H, H, e->table_e, e->wqkv, e->table_qkv,
+                          CUDA_R_32F, 3 * H);
+    if (ce == cudaSuccess) ce = cudaDeviceSynchronize();
+    if (ce != cudaSuccess || bs != CUBLAS_STATUS_SUCCESS) {
+      cudaGetLastError();
+      rc = efail(HAM_ECUDA, "vocabulary tabulation: %s, cuBLAS status %d",
+                 cudaGetErrorString(ce), (int)bs);
+    }
+  }
+  if (rc == HAM_OK) {
+    e->vocab = vocab;
+  } else {
+    cudaFree(e->table_e);
+    cudaFree(e->table_qkv);
+    e->table_e = nullptr;
+    e->table_qkv = nullptr;
   }
   if (dev != e->device) cudaSetDevice(dev);
   return rc;

@@ -74,6 +74,8 @@ _SIGNATURES = {
     "ham_embedder_free": [_vp],
     "ham_embed": [_vp, _vp, _vp, _i32, _i32, _vp, _vp],
     "ham_embedder_status": [_vp, _vp, ctypes.POINTER(_i32)],
+    "ham_embedder_set_vocab": [_vp, _vp, _i32],
+    "ham_embed_tokens": [_vp, _vp, _vp, _i32, _i32, _vp, _vp],
     "ham_kv_alloc": [ctypes.POINTER(ham_config), ctypes.POINTER(_vp)],
     "ham_kv_free": [_vp],
     "ham_kv_append": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp],
@@ -416,6 +418,23 @@ def ham_embed(e: Embedder, x, offsets, out, stream=None):
     _check(lib().ham_embed(e, _dev(x, (T, e.hidden), "bf16", "x"),
                            _dev(offsets, (B + 1,), "i32", "offsets"), B, T,
                            _dev(out, (B, e.hidden), "bf16", "out"), _stream_ptr(stream)))
+
+
+def ham_embedder_set_vocab(e: Embedder, table):
+    """table: CUDA bf16 [vocab][hidden], the token embeddings (copied; the projections of every
+    entry are tabulated on the handle, synchronously)."""
+    V = table.shape[0] if table is not None and table.dim() == 2 else 0
+    _check(lib().ham_embedder_set_vocab(e, _dev(table, (V, e.hidden), "bf16", "table"), V))
+
+
+def ham_embed_tokens(e: Embedder, ids, offsets, out, stream=None):
+    """ids: CUDA int32 [total_tokens] (token ids); offsets: CUDA int32 [batch + 1]; out: CUDA
+    bf16 [batch][hidden]."""
+    B = out.shape[0] if out is not None else 0
+    T = ids.shape[0] if ids is not None else 0
+    _check(lib().ham_embed_tokens(e, _dev(ids, (T,), "i32", "ids"),
+                                  _dev(offsets, (B + 1,), "i32", "offsets"), B, T,
+                                  _dev(out, (B, e.hidden), "bf16", "out"), _stream_ptr(stream)))
 
 
 def ham_embedder_status(e: Embedder, stream=None) -> int:

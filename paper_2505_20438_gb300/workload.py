@@ -231,6 +231,7 @@ class EmbedWorkload:
     n_heads: int = 32
     max_patch: int = MAX_TOKENS_PER_SLOT
     seed: int = 5
+    vocab: int = 0          # > 0: tokens arrive as ids into a table of this many entries
 
 
 @dataclasses.dataclass
@@ -250,6 +251,12 @@ def embed_workload(batch: int, **kw) -> EmbedWorkload:
     return EmbedWorkload(f"embed_b{batch}", batch=batch, **kw)
 
 
+def embed_tokens_workload(batch: int, **kw) -> EmbedWorkload:
+    """The embedder fed token ids of the Llama-3 vocabulary (width 2048, as Llama-3.2-1B)."""
+    kw.setdefault("vocab", LLAMA3_VOCAB)
+    return EmbedWorkload(f"embedtok_b{batch}", batch=batch, **kw)
+
+
 def make_embed_case(w: EmbedWorkload, counts: Optional[np.ndarray] = None) -> EmbedCase:
     rng = rng_for(w.seed, 40)
     if counts is None:
@@ -262,3 +269,25 @@ def make_embed_case(w: EmbedWorkload, counts: Optional[np.ndarray] = None) -> Em
                      normal_bf16(rng, (H, H), ws), normal_bf16(rng, (H, H), ws),
                      normal_bf16(rng, (H, H), ws), normal_bf16(rng, (H, H), ws),
                      normal_bf16(rng, (w.max_patch, H)))
+
+
+LLAMA3_VOCAB = 128256   # entries of the Llama-3 token-embedding table (width 2048 at 1B)
+
+
+@dataclasses.dataclass
+class EmbedTokensCase:
+    case: EmbedCase         # the same weights and counts; case.x = table[ids]
+    table: np.ndarray       # bf16 bits [vocab][H]: the token-embedding table, N(0, 1)
+    ids: np.ndarray         # int32 [T]: token ids, uniform over the vocabulary
+
+
+def make_embed_tokens_case(w: EmbedWorkload, vocab: int,
+                           counts: Optional[np.ndarray] = None) -> EmbedTokensCase:
+    """An embedder case whose tokens are ids into a seeded embedding table: the weights and
+    counts of make_embed_case(w, counts), the embeddings gathered from the table."""
+    c = make_embed_case(w, counts)
+    rng = rng_for(w.seed, 41)
+    table = normal_bf16(rng, (vocab, w.hidden))
+    ids = rng.integers(0, vocab, int(c.offsets[-1]), dtype=np.int32)
+    c.x = table[ids]
+    return EmbedTokensCase(c, table, ids)

@@ -158,4 +158,6 @@ def test_embedder_null_arguments_are_rejected(libham):
                                      ctypes.byref(out)) == ham.HAM_EINVAL
     assert libham.ham_embed(None, None, None, 1, 1, None, None) == ham.HAM_EINVAL
     assert libham.ham_embedder_status(None, None, None) == ham.HAM_EINVAL
+    assert libham.ham_embedder_set_vocab(None, None, 1) == ham.HAM_EINVAL
+    assert libham.ham_embed_tokens(None, None, None, 1, 1, None, None) == ham.HAM_EINVAL
     assert libham.ham_embedder_free(None) == ham.HAM_OK

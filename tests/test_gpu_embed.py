@@ -108,3 +108,74 @@ def test_host_errors():
     with pytest.raises(ham.HamError):          # head_dim 16 is not compiled
         ham.ham_embedder_alloc(256, 16, 4, 4, *(dev_bf16(w) for w in (c.wq, c.wk, c.wv, c.wo)),
                                dev_bf16(c.pos))
+
+
+# ---- token ids through the tabulated vocabulary (ham_embedder_set_vocab / ham_embed_tokens) --
+
+def _run_tokens(tc, ids=None, max_batch=None):
+    t = torch()
+    c = tc.case
+    w = c.w
+    e = ham.ham_embedder_alloc(w.hidden, w.n_heads, max_batch or len(c.counts), w.max_patch,
+                               dev_bf16(c.wq), dev_bf16(c.wk), dev_bf16(c.wv), dev_bf16(c.wo),
+                               dev_bf16(c.pos))
+    ham.ham_embedder_set_vocab(e, dev_bf16(tc.table))
+    out = t.full((len(c.counts), w.hidden), float("nan"), dtype=t.bfloat16, device="cuda")
+    ham.ham_embed_tokens(e, dev_i32(tc.ids if ids is None else ids), dev_i32(c.offsets), out)
+    t.cuda.synchronize()
+    return e, out
+
+
+@pytest.mark.parametrize("batch,hidden,heads,vocab", [
+    (64, 2048, 32, wl.LLAMA3_VOCAB),   # the Llama-3.2-1B width and vocabulary
+    (8, 256, 8, 1000), (12, 320, 10, 777), (160, 256, 8, 5000), (5, 512, 4, 3),
+])
+def test_embed_tokens_matches_oracle(batch, hidden, heads, vocab):
+    tc = wl.make_embed_tokens_case(
+        wl.embed_workload(batch, hidden=hidden, n_heads=heads, seed=batch + 1), vocab)
+    e, out = _run_tokens(tc)
+    _check(tc.case, out)     # case.x = table[ids]: fused states and bypass rows
+    assert ham.ham_embedder_status(e) == ham.HAM_DEVERR_NONE
+
+
+def test_embed_tokens_bad_ids_give_zeros_and_the_error_word():
+    vocab = 300
+    tc = wl.make_embed_tokens_case(wl.embed_workload(6, hidden=256, n_heads=8, seed=6), vocab,
+                                   counts=np.array([2, 1, 3, 1, 4, 2]))
+    c = tc.case
+    ids = tc.ids.copy()
+    ids[c.offsets[0] + 1] = vocab     # sequence 0: an id past the end
+    ids[c.offsets[3]] = -1            # sequence 3: a single bad token
+    e, out = _run_tokens(tc, ids=ids)
+    assert ham.ham_embedder_status(e) == ham.HAM_DEVERR_NTOK
+    bits = host_bits(out)
+    for b in (0, 3):
+        assert np.all(bits[b] == 0), b
+    ref = oe.embed(c.x, c.offsets, c.wq, c.wk, c.wv, c.wo, c.pos, c.w.n_heads)
+    got = out.float().cpu().numpy().astype(np.float64)
+    for b in (2, 4, 5):
+        assert np.max(np.abs(got[b] - ref[b]) / np.maximum(1.0, np.abs(ref[b]))) <= REL, b
+    assert np.array_equal(bits[1], tc.table[ids[c.offsets[1]]])
+
+
+def test_embed_tokens_host_errors():
+    t = torch()
+    tc = wl.make_embed_tokens_case(wl.embed_workload(4, hidden=256, n_heads=8, seed=2), 50)
+    c = tc.case
+    e = ham.ham_embedder_alloc(256, 8, 4, c.w.max_patch,
+                               *(dev_bf16(w) for w in (c.wq, c.wk, c.wv, c.wo)), dev_bf16(c.pos))
+    out = t.zeros((4, 256), dtype=t.bfloat16, device="cuda")
+    with pytest.raises(ham.HamError):          # no vocabulary yet
+        ham.ham_embed_tokens(e, dev_i32(tc.ids), dev_i32(c.offsets), out)
+    with pytest.raises(ValueError):            # table of the wrong width
+        ham.ham_embedder_set_vocab(e, t.zeros((50, 128), dtype=t.bfloat16, device="cuda"))
+    ham.ham_embedder_set_vocab(e, dev_bf16(tc.table))
+    ham.ham_embedder_set_vocab(e, dev_bf16(tc.table))   # replacing the table is allowed
+    ham.ham_embed_tokens(e, dev_i32(tc.ids), dev_i32(c.offsets), out)
+    t.cuda.synchronize()
+    assert ham.ham_embedder_status(e) == ham.HAM_DEVERR_NONE
+    # one id fewer than the offsets say: the last sequence's rows leave the call's tokens
+    ham.ham_embed_tokens(e, dev_i32(tc.ids[:-1]), dev_i32(c.offsets), out)
+    t.cuda.synchronize()
+    assert ham.ham_embedder_status(e) == ham.HAM_DEVERR_NTOK
+    assert np.all(host_bits(out)[-1] == 0)
