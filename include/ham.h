@@ -171,6 +171,40 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
 int ham_slot_lengths(ham_kv *kv, int32_t *num_slots_host, int64_t *num_tokens_host,
                      void *stream);
 
+/* Chunked prefill of one layer: prompt ingestion over the smashed cache.  The paper fuses
+ * only response tokens (Figure 2, training), so each prompt token becomes its own slot;
+ * the chunk's queries attend causally over the cache and over the chunk itself.  Sequence
+ * b's new rows are rows offsets[b] .. offsets[b+1]-1 of q/k_new/v_new, in order (a sequence
+ * may have none).  With L = num_slots[layer][b] before the call, row r = offsets[b] + j:
+ *   becomes slot L + j as ham_kv_append would store it: position pos[r], or (pos == NULL)
+ *     L + j for HAM_POS_SLOT and the tokens before it (num_tokens[layer][b] plus the ntok of
+ *     the sequence's earlier rows) for HAM_POS_TOKEN; K row RoPE(k_new[r]), V row v_new[r],
+ *     slot_pos, slot_ntok = ntok[r]; num_slots += rows, num_tokens += their ntok;
+ *   q_inout[r] <- RoPE(q_inout[r]) at the same position, in place;
+ *   out[r][h] = softmax(q[r][h] K^T / sqrt(head_dim)) V over slots 0 .. L + j of the
+ *     sequence, KV head h / (n_q_heads / n_kv_heads).
+ * The rotations are evaluated to about 48 bits in fp32 pairs from the fp64 cos/sin table
+ * and rounded once to bf16: the bits ham_kv_append stores, unless the exact rotation lies
+ * within about 2^-40 (relative) of a bf16 rounding boundary.  The attention runs on the
+ * tensor cores (bf16 in, fp32 accumulation and softmax, probabilities rounded to bf16).
+ * q_inout  device bf16 [total_rows][n_q_heads][head_dim]
+ * k_new, v_new  device bf16 [total_rows][n_kv_heads][head_dim]
+ * offsets  device int32 [batch + 1]: offsets[0] = 0, non-decreasing, offsets[batch] =
+ *          total_rows
+ * pos      nullable device int32 [total_rows];  ntok  nullable device int32 [total_rows]
+ *          (NULL: 1 token per row)
+ * out      device [total_rows][n_q_heads][head_dim], bf16 or f32 (out_dtype)
+ * A sequence whose rows cannot all be stored (a token count < 1, no room for them, a bad
+ * page, offsets that leave the call's rows) gets no slot, keeps q unrotated and 0 out
+ * rows, and sets the device error word.  total_rows == 0 launches nothing.  Three launches
+ * on `stream` (plan, RoPE + append, attention).  q_inout, out, k_new and v_new must not
+ * overlap each other or the cache.  Host errors: HAM_EINVAL (NULL / unaligned / overlapping
+ * pointers, layer or out_dtype out of range, total_rows above batch * max_slots_per_seq),
+ * HAM_ECUDA.  Same serialization rule as ham_decode_attn. */
+int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, const void *v_new,
+                const int32_t *offsets, const int32_t *pos, const int32_t *ntok,
+                int32_t total_rows, void *out, int32_t out_dtype, void *stream);
+
 /* ------------------------------------------------------------------------------------
  * Helpers: inspection, test set-up, tuning
  * ------------------------------------------------------------------------------------ */

@@ -67,6 +67,7 @@ def lib():
             "oracle_decode_attn": (ctypes.c_int, [P, vp, vp, i32]),
             "oracle_attn_weights": (ctypes.c_int, [P, vp, i32, i32, vp]),
             "oracle_append": (ctypes.c_int, [P, vp, vp, vp, vp, vp, i32, f64]),
+            "oracle_prefill": (ctypes.c_int, [P, vp, vp, vp, vp, vp, vp, i32, f64, vp, vp, i32]),
             "oracle_max_threads": (ctypes.c_int, []),
         }
         for name, (res, args) in sig.items():
@@ -194,3 +195,24 @@ class OracleCache:
         return lib().oracle_append(ctypes.byref(self._c), _ptr(k_new), _ptr(v_new),
                                    _ptr(q_inout), _ptr(pos), _ptr(ntok), int(pos_mode),
                                    float(rope_base))
+
+    def prefill(self, q, k_new, v_new, offsets, ntok=None, pos=None, pos_mode=POS_SLOT,
+                rope_base=10000.0, want=None, n_threads: int = 0):
+        """Chunked prefill (oracle_prefill).  q [T][n_q_heads][d] bf16 bits is rotated in place
+        (must be C-contiguous uint16); want: optional bool [T], the rows to attend (the others
+        are appended, their out rows 0).  Returns (status, out [T][n_q_heads][d] fp64)."""
+        assert q.dtype == np.uint16 and q.flags.c_contiguous
+        k_new = np.ascontiguousarray(k_new, np.uint16)
+        v_new = np.ascontiguousarray(v_new, np.uint16)
+        offsets = np.ascontiguousarray(offsets, np.int32)
+        T = int(offsets[-1])
+        ntok = np.ones(T, np.int32) if ntok is None else np.ascontiguousarray(ntok, np.int32)
+        if pos is not None:
+            pos = np.ascontiguousarray(pos, np.int32)
+        if want is not None:
+            want = np.ascontiguousarray(want, np.uint8)
+        out = np.empty(q.shape, np.float64)
+        rc = lib().oracle_prefill(ctypes.byref(self._c), _ptr(q), _ptr(k_new), _ptr(v_new),
+                                  _ptr(offsets), _ptr(pos), _ptr(ntok), int(pos_mode),
+                                  float(rope_base), _ptr(out), _ptr(want), int(n_threads))
+        return rc, out

@@ -146,19 +146,16 @@ int oracle_fill(oracle_cache *c, const uint16_t *k_log, const uint16_t *v_log,
   return 0;
 }
 
-/* Attention of one query head over one sequence: weights w[L] and output out[d]. */
-static int attend_one(const oracle_cache *c, const uint16_t *q, int32_t b, int32_t h,
-                      double *w, double *out) {
+/* Attention of one query row qh [d] (bf16 bits) over slots 0..count-1 of sequence b, KV
+ * head g: weights w[count] and output out[d]. */
+static int attend_prefix(const oracle_cache *c, const uint16_t *qh, int32_t b, int32_t g,
+                         int64_t count, double *w, double *out) {
   const int32_t d = c->head_dim;
-  const int32_t group = c->n_q_heads / c->n_kv_heads;
-  const int32_t g = h / group;
-  const int64_t L = c->num_slots[b];
-  const uint16_t *qh = q + ((int64_t)b * c->n_q_heads + h) * d;
   const double scale = 1.0 / sqrt((double)d);
   for (int32_t i = 0; i < d; ++i) out[i] = 0.0;
-  if (L <= 0) return 0; /* empty sequence: output 0 */
+  if (count <= 0) return 0; /* empty sequence: output 0 */
   double m = -INFINITY;
-  for (int64_t j = 0; j < L; ++j) {
+  for (int64_t j = 0; j < count; ++j) {
     int64_t off = slot_row(c, b, j, g);
     if (off < 0) return ORACLE_EPAGE;
     double s = 0.0;
@@ -168,16 +165,25 @@ static int attend_one(const oracle_cache *c, const uint16_t *q, int32_t b, int32
     if (w[j] > m) m = w[j];
   }
   double l = 0.0;
-  for (int64_t j = 0; j < L; ++j) {
+  for (int64_t j = 0; j < count; ++j) {
     w[j] = exp(w[j] - m);
     l += w[j];
   }
-  for (int64_t j = 0; j < L; ++j) {
+  for (int64_t j = 0; j < count; ++j) {
     w[j] /= l;
     int64_t off = slot_row(c, b, j, g);
     for (int32_t i = 0; i < d; ++i) out[i] += w[j] * oracle_bf16_to_f64(c->v_pool[off + i]);
   }
   return 0;
+}
+
+/* Attention of one query head over one sequence: weights w[L] and output out[d]. */
+static int attend_one(const oracle_cache *c, const uint16_t *q, int32_t b, int32_t h,
+                      double *w, double *out) {
+  const int32_t d = c->head_dim;
+  const int32_t group = c->n_q_heads / c->n_kv_heads;
+  const uint16_t *qh = q + ((int64_t)b * c->n_q_heads + h) * d;
+  return attend_prefix(c, qh, b, h / group, c->num_slots[b], w, out);
 }
 
 int oracle_decode_attn(const oracle_cache *c, const uint16_t *q, double *out,
@@ -245,6 +251,86 @@ int oracle_append(oracle_cache *c, const uint16_t *k_new, const uint16_t *v_new,
     c->num_tokens[b] += ntok[b];
   }
   return status;
+}
+
+/* Chunked prefill.  A prompt's tokens are not fused (the paper fuses only response tokens:
+ * Figure 2, training, item 2), so every new row becomes its own slot.  Sequence b's new rows
+ * are offsets[b] .. offsets[b+1]-1, in order; with L = num_slots[b] before the call, row
+ * r = offsets[b] + j becomes slot L + j exactly as oracle_append would append it (position
+ * pos[r], or the slot index / the tokens so far), and its query heads then attend over slots
+ * 0 .. L + j of the sequence: the causal attention of the chunk over the cache and over
+ * itself.  want (nullable, [T]) restricts the attention to the rows it marks (the others get
+ * 0; every row is still appended), for sampled checks of large chunks.  A sequence whose rows do not all fit (a token count < 1, no room, a bad page) is
+ * left untouched and its out rows are 0.  q [T][n_q_heads][d] is rotated in place; out
+ * [T][n_q_heads][d] doubles. */
+int oracle_prefill(oracle_cache *c, uint16_t *q, const uint16_t *k_new, const uint16_t *v_new,
+                   const int32_t *offsets, const int32_t *pos, const int32_t *ntok,
+                   int32_t pos_mode, double rope_base, double *out, const uint8_t *want,
+                   int32_t n_threads) {
+  if (check_cache(c) || !q || !k_new || !v_new || !offsets || !ntok || !out || pos_mode < 0 ||
+      pos_mode > 1 || offsets[0] != 0)
+    return ORACLE_EINVAL;
+  for (int32_t b = 0; b < c->batch; ++b)
+    if (offsets[b + 1] < offsets[b]) return ORACLE_EINVAL;
+  const int32_t d = c->head_dim, hq = c->n_q_heads, hkv = c->n_kv_heads;
+  const int64_t T = offsets[c->batch];
+  int64_t *row_slot = (int64_t *)malloc(sizeof(int64_t) * (size_t)(T > 0 ? T : 1));
+  int status = 0;
+  for (int32_t b = 0; b < c->batch; ++b) {
+    const int64_t L = c->num_slots[b], n = offsets[b + 1] - offsets[b];
+    int rc = 0;
+    for (int64_t j = 0; j < n && !rc; ++j)
+      if (ntok[offsets[b] + j] < 1) rc = ORACLE_EINVAL;
+    if (!rc && L + n > c->max_slots) rc = ORACLE_ECAPACITY;
+    for (int64_t j = 0; j < n && !rc; ++j)
+      if (slot_meta(c, b, L + j) < 0) rc = ORACLE_EPAGE;
+    if (rc) {
+      if (rc < status) status = rc;
+      for (int64_t j = 0; j < n; ++j) row_slot[offsets[b] + j] = -1;
+      continue;
+    }
+    for (int64_t j = 0; j < n; ++j) {
+      const int64_t r = offsets[b] + j, slot = L + j;
+      const int64_t p = pos ? pos[r] : (pos_mode == 0 ? slot : c->num_tokens[b]);
+      for (int32_t g = 0; g < hkv; ++g) {
+        int64_t off = slot_row(c, b, slot, g);
+        oracle_rope_bf16(k_new + (r * hkv + g) * d, c->k_pool + off, 1, d, p, rope_base);
+        memcpy(c->v_pool + off, v_new + (r * hkv + g) * d, sizeof(uint16_t) * (size_t)d);
+      }
+      oracle_rope_bf16(q + r * hq * d, q + r * hq * d, hq, d, p, rope_base);
+      int64_t m = slot_meta(c, b, slot);
+      c->slot_pos[m] = (int32_t)p;
+      c->slot_ntok[m] = ntok[r];
+      c->num_slots[b] = (int32_t)(slot + 1);
+      c->num_tokens[b] += ntok[r];
+      row_slot[r] = slot;
+    }
+  }
+  /* row r, head h: slots 0 .. row_slot[r] of its sequence (b found from the offsets) */
+  const int64_t pairs = T * hq;
+  int astatus = 0;
+#ifdef _OPENMP
+  int nt = n_threads > 0 ? n_threads : omp_get_max_threads();
+#pragma omp parallel for schedule(dynamic, 16) num_threads(nt) reduction(min : astatus)
+#endif
+  for (int64_t rh = 0; rh < pairs; ++rh) {
+    const int64_t r = rh / hq;
+    const int32_t h = (int32_t)(rh % hq);
+    int32_t b = 0;
+    while (offsets[b + 1] <= r) ++b;
+    double *o = out + rh * d;
+    if (row_slot[r] < 0 || (want && !want[r])) {
+      for (int32_t i = 0; i < d; ++i) o[i] = 0.0;
+      continue;
+    }
+    double *w = (double *)malloc(sizeof(double) * (size_t)(row_slot[r] + 1));
+    int rc = attend_prefix(c, q + rh * d, b, h / (hq / hkv), row_slot[r] + 1, w, o);
+    free(w);
+    if (rc < astatus) astatus = rc;
+  }
+  (void)n_threads;
+  free(row_slot);
+  return status < astatus ? status : astatus;
 }
 
 int oracle_max_threads(void) {

@@ -82,6 +82,18 @@ int oracle_append(oracle_cache *c, const uint16_t *k_new, const uint16_t *v_new,
                   uint16_t *q_inout, const int32_t *pos, const int32_t *ntok,
                   int32_t pos_mode, double rope_base);
 
+/* Chunked prefill: sequence b's new rows offsets[b] .. offsets[b+1]-1 (offsets [batch+1],
+ * offsets[0] = 0) each become one slot, appended in order as oracle_append appends (pos [T]
+ * nullable, ntok [T]), and each row's query heads attend over the slots of its sequence up
+ * to and including its own.  q [T][n_q_heads][head_dim] rotated in place; out
+ * [T][n_q_heads][head_dim] doubles; want (nullable [T]): attend only the marked rows (others
+ * 0).  A sequence whose rows do not all fit is left untouched (out rows 0) and the error is
+ * returned. */
+int oracle_prefill(oracle_cache *c, uint16_t *q, const uint16_t *k_new, const uint16_t *v_new,
+                   const int32_t *offsets, const int32_t *pos, const int32_t *ntok,
+                   int32_t pos_mode, double rope_base, double *out, const uint8_t *want,
+                   int32_t n_threads);
+
 /* Threads an OpenMP region of this library uses by default (1 without OpenMP). */
 int oracle_max_threads(void);
 

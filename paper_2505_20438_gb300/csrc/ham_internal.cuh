@@ -133,6 +133,34 @@ struct FillView {
   int32_t batch, n_kv_heads, head_dim, page_slots, max_pages, max_slots, lmax;
 };
 
+// Chunked prefill (ham_prefill): sequence b's new rows offsets[b] .. offsets[b+1]-1.
+struct PrefillView {
+  uint16_t *k_pool, *v_pool;   // this layer
+  int32_t *slot_pos, *slot_ntok;
+  const int32_t *page_table;
+  int32_t *num_slots;          // [batch] of this layer
+  int64_t *num_tokens;         // [batch] of this layer
+  const double2 *rope_table;   // [rope_positions][head_dim / 2]: (cos, sin), fp64
+  const double *inv_freq;      // [head_dim / 2] (positions past the table)
+  int64_t rope_positions;
+  uint16_t *q;                 // [rows][n_q_heads][head_dim], rotated in place
+  const uint16_t *k_new, *v_new;
+  const int32_t *offsets, *pos, *ntok;  // pos, ntok nullable
+  void *out;                   // [rows][n_q_heads][head_dim], bf16 or f32
+  int4 *seq_info;              // scratch [batch]: (first new slot or -1, rows, query-block
+                               // start, 0)
+  int32_t *row_pos;            // scratch [rows]: position of each new row
+  int32_t *err;
+  int64_t pool_pages;
+  int32_t batch, rows, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots;
+  int32_t pos_mode;
+};
+cudaError_t launch_prefill(const CUtensorMap &tk, const CUtensorMap &tv, const PrefillView &v,
+                           int out_dtype, cudaStream_t stream);
+bool prefill_supported(int head_dim, int group);
+// Query rows of one sequence that one prefill attention CTA covers (128 / group).
+int prefill_query_rows(int group);
+
 // Launchers (return cudaError_t of the launch; argument checks are done by the callers).
 // tk / tv: TMA maps of the layer's K and V pools (make_pool_tensor_map).
 cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
@@ -188,6 +216,8 @@ struct ham_kv {
   float *part_acc = nullptr;
   float2 *part_ml = nullptr;
   int2 *seg_range = nullptr;
+  int4 *prefill_seq = nullptr;     // ham_prefill: per-sequence plan [batch]
+  int32_t *prefill_pos = nullptr;  // ham_prefill: per-row positions [batch * max_slots]
   int64_t scratch_bytes = 0;
   std::vector<CUtensorMap> tmaps;  // [layers][2]: TMA maps of the K and V pools
   void *host_stage = nullptr;   // pinned: counters and error word read-back

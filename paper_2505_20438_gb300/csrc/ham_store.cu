@@ -332,6 +332,8 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   const size_t o_sr = carve(n_seg * sizeof(int2));
   const size_t o_stash = carve((size_t)cfg.batch * sizeof(int4));
   const size_t o_arrive = carve(sizeof(int32_t));
+  const size_t o_pf_seq = carve((size_t)cfg.batch * sizeof(int4));
+  const size_t o_pf_pos = carve((size_t)cfg.batch * cfg.max_slots_per_seq * sizeof(int32_t));
   kv->scratch_bytes = (int64_t)(off - o_acc);
 
   {
@@ -369,6 +371,8 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->seg_range = reinterpret_cast<int2 *>(kv->meta + o_sr);
   kv->stash = reinterpret_cast<int4 *>(kv->meta + o_stash);
   kv->arrive = reinterpret_cast<int32_t *>(kv->meta + o_arrive);
+  kv->prefill_seq = reinterpret_cast<int4 *>(kv->meta + o_pf_seq);
+  kv->prefill_pos = reinterpret_cast<int32_t *>(kv->meta + o_pf_pos);
 
   // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits.
   e = cudaMemset(kv->pool, 0, pool_bytes);
@@ -624,6 +628,81 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
                                           kv->tmaps[(size_t)layer * 2 + 1], v, c.head_dim,
                                           out_dtype, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "decode step launch");
+  note_launch(kv, layer, stream, true);
+  return HAM_OK;
+}
+
+int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, const void *v_new,
+                const int32_t *offsets, const int32_t *pos, const int32_t *ntok,
+                int32_t total_rows, void *out, int32_t out_dtype, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!q_inout || !k_new || !v_new || !offsets || !out)
+    return fail(HAM_EINVAL, "q_inout, k_new, v_new, offsets and out are required");
+  if (out_dtype != HAM_DTYPE_BF16 && out_dtype != HAM_DTYPE_F32)
+    return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
+  const ham_config &c = kv->cfg;
+  if (total_rows < 0 || (int64_t)total_rows > (int64_t)c.batch * c.max_slots_per_seq)
+    return fail(HAM_EINVAL, "total_rows %d outside 0..batch * max_slots_per_seq", total_rows);
+  if (!aligned16(q_inout) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out))
+    return fail(HAM_EINVAL, "q/k/v/out must be 16-byte aligned");
+  if (((uintptr_t)offsets & 3u) || ((uintptr_t)pos & 3u) || ((uintptr_t)ntok & 3u))
+    return fail(HAM_EINVAL, "offsets/pos/ntok must be 4-byte aligned");
+  const int group = c.n_q_heads / c.n_kv_heads;
+  if (!ham::prefill_supported(c.head_dim, group))
+    return fail(HAM_EUNSUPPORTED, "prefill: head_dim %d / group %d not compiled", c.head_dim,
+                group);
+  const size_t T = (size_t)total_rows, d = (size_t)c.head_dim;
+  const size_t q_bytes = T * c.n_q_heads * d * 2, kv_bytes = T * c.n_kv_heads * d * 2;
+  const size_t out_bytes = T * c.n_q_heads * d * (out_dtype == HAM_DTYPE_F32 ? 4 : 2);
+  const size_t pool_bytes = (size_t)c.layers * 2 * (size_t)kv->pool_elems * 2;
+  if (overlaps(q_inout, q_bytes, out, out_bytes) || overlaps(q_inout, q_bytes, k_new, kv_bytes) ||
+      overlaps(q_inout, q_bytes, v_new, kv_bytes) || overlaps(out, out_bytes, k_new, kv_bytes) ||
+      overlaps(out, out_bytes, v_new, kv_bytes) || overlaps(q_inout, q_bytes, kv->pool, pool_bytes) ||
+      overlaps(out, out_bytes, kv->pool, pool_bytes) || overlaps(k_new, kv_bytes, kv->pool, pool_bytes) ||
+      overlaps(v_new, kv_bytes, kv->pool, pool_bytes))
+    return fail(HAM_EINVAL, "q_inout, out, k_new, v_new and the cache must not overlap");
+  const int64_t blocks = (int64_t)total_rows / ham::prefill_query_rows(group) + c.batch;
+  if (blocks > 65535)
+    return fail(HAM_EINVAL, "total_rows %d: split the chunk (at most %lld query blocks a call)",
+                total_rows, 65535LL);
+  if (total_rows == 0) return HAM_OK;
+  DeviceGuard guard(kv->device);
+  ham::PrefillView v{};
+  v.k_pool = layer_pool(kv, layer, 0);
+  v.v_pool = layer_pool(kv, layer, 1);
+  v.slot_pos = kv->slot_pos;
+  v.slot_ntok = kv->slot_ntok;
+  v.page_table = kv->page_table;
+  v.num_slots = kv->num_slots + (size_t)layer * c.batch;
+  v.num_tokens = kv->num_tokens + (size_t)layer * c.batch;
+  v.rope_table = kv->rope_table;
+  v.inv_freq = kv->inv_freq;
+  v.rope_positions = kv->rope_positions;
+  v.q = static_cast<uint16_t *>(q_inout);
+  v.k_new = static_cast<const uint16_t *>(k_new);
+  v.v_new = static_cast<const uint16_t *>(v_new);
+  v.offsets = offsets;
+  v.pos = pos;
+  v.ntok = ntok;
+  v.out = out;
+  v.seq_info = kv->prefill_seq;
+  v.row_pos = kv->prefill_pos;
+  v.err = kv->err;
+  v.pool_pages = c.pool_pages;
+  v.batch = c.batch;
+  v.rows = total_rows;
+  v.n_q_heads = c.n_q_heads;
+  v.n_kv_heads = c.n_kv_heads;
+  v.head_dim = c.head_dim;
+  v.page_slots = c.page_slots;
+  v.max_pages = kv->max_pages;
+  v.max_slots = c.max_slots_per_seq;
+  v.pos_mode = c.pos_mode;
+  cudaError_t e = ham::launch_prefill(kv->tmaps[(size_t)layer * 2],
+                                      kv->tmaps[(size_t)layer * 2 + 1], v, out_dtype,
+                                      static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
   note_launch(kv, layer, stream, true);
   return HAM_OK;
 }

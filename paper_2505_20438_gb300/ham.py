@@ -95,6 +95,7 @@ _SIGNATURES = {
     "ham_split_plan": [_i32, _i32, _vp, _i32, _vp, _vp, _vp],
     "ham_decode_attn_noalloc": [ctypes.c_void_p, _vp],
     "ham_decode_step": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
+    "ham_prefill": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _i32, _vp],
 }
 _lib = None
 
@@ -255,6 +256,24 @@ def ham_decode_step(kv: KV, layer, q, k_new, v_new, pos, ntok, out, q_rot=None, 
         _dev(k_new, (B, Hkv, d), "bf16", "k_new"), _dev(v_new, (B, Hkv, d), "bf16", "v_new"),
         _dev(pos, (B,), "i32", "pos", nullable=True), _dev(ntok, (B,), "i32", "ntok"),
         _dev(out, (B, Hq, d), "f32" if f32 else "bf16", "out"),
+        HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16, _stream_ptr(stream)))
+
+
+def ham_prefill(kv: KV, layer, q, k_new, v_new, offsets, out, pos=None, ntok=None,
+                stream=None):
+    """Chunked prefill of one layer: sequence b's new rows are offsets[b] .. offsets[b+1]-1 of
+    q [T][n_q_heads][d] (rotated in place), k_new, v_new [T][n_kv_heads][d]; each becomes one
+    slot and attends causally.  pos, ntok: optional int32 [T].  Output dtype follows `out`."""
+    import torch
+    Hq, Hkv, d = kv.n_q_heads, kv.n_kv_heads, kv.head_dim
+    T = q.shape[0] if q is not None and q.dim() == 3 else 0
+    f32 = out is not None and out.dtype == torch.float32
+    _check(lib().ham_prefill(
+        kv, layer, _dev(q, (T, Hq, d), "bf16", "q"), _dev(k_new, (T, Hkv, d), "bf16", "k_new"),
+        _dev(v_new, (T, Hkv, d), "bf16", "v_new"),
+        _dev(offsets, (kv.batch + 1,), "i32", "offsets"),
+        _dev(pos, (T,), "i32", "pos", nullable=True), _dev(ntok, (T,), "i32", "ntok", nullable=True),
+        T, _dev(out, (T, Hq, d), "f32" if f32 else "bf16", "out"),
         HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16, _stream_ptr(stream)))
 
 

@@ -203,6 +203,58 @@ def make_case(w: Workload, extra_slots: int = 1, num_slots: Optional[np.ndarray]
                     ntok_new)
 
 
+# ---------------------------------------------------------------------------------------
+# Chunked prefill (prompt ingestion): prompt tokens are not fused (Figure 2, training), so each
+# becomes one slot with one token; the chunk's rows attend causally over the cache.
+# ---------------------------------------------------------------------------------------
+@dataclasses.dataclass
+class PrefillCase:
+    base: HostCase               # the cache before the chunk (base.num_slots slots each)
+    rows: np.ndarray             # [B] int32: new rows per sequence (0 allowed)
+    offsets: np.ndarray          # [B+1] int32: sequence b owns rows offsets[b] .. offsets[b+1]-1
+    q: np.ndarray                # [T][Hq][d] uint16: unrotated queries
+    k_new: np.ndarray            # [T][Hkv][d] uint16: unrotated keys
+    v_new: np.ndarray            # [T][Hkv][d] uint16
+    ntok: np.ndarray             # [T] int32: tokens per new slot (1 for prompt tokens)
+
+    @property
+    def w(self) -> Workload:
+        return self.base.w
+
+
+def make_prefill_case(w: Workload, rows, cached=None, ntok=None,
+                      headroom: int = 0) -> PrefillCase:
+    """A chunk of rows[b] new rows per sequence over a cache holding cached[b] slots (the
+    workload's own slot counts if None), with room for `headroom` more slots."""
+    rows = np.asarray(rows, dtype=np.int32)
+    base = make_case(w, extra_slots=int(rows.max(initial=0)) + headroom, num_slots=cached)
+    offsets = np.concatenate([[0], np.cumsum(rows)]).astype(np.int32)
+    T = int(offsets[-1])
+    q = normal_bf16(rng_for(w.seed, 20), (T, w.n_q_heads, w.head_dim), w.value_scale)
+    k_new = normal_bf16(rng_for(w.seed, 21), (T, w.n_kv_heads, w.head_dim), w.value_scale)
+    v_new = normal_bf16(rng_for(w.seed, 22), (T, w.n_kv_heads, w.head_dim), w.value_scale)
+    ntok = np.ones(T, np.int32) if ntok is None else np.asarray(ntok, np.int32)
+    return PrefillCase(base, rows, offsets, q, k_new, v_new, ntok)
+
+
+@dataclasses.dataclass(frozen=True)
+class PrefillWorkload:
+    name: str
+    w: Workload                  # head shape, page size, value scale, seed
+    rows: int                    # new rows per sequence
+    cached: int                  # slots per sequence before the chunk
+
+
+# Fresh 4096-token prompts of a Llama-3-8B layer, batch 4.
+P1_PREFILL = PrefillWorkload("prefill_b4_s4096", dataclasses.replace(
+    C1_LLAMA8B, name="prefill_b4_s4096", batch=4, slots=0, seed=11), rows=4096, cached=0)
+# A 1024-row chunk over 3072 cached slots (the last chunk of a 4096-token prompt), batch 4.
+P2_CHUNK = PrefillWorkload("prefill_b4_c1024_s3072", dataclasses.replace(
+    C1_LLAMA8B, name="prefill_b4_c1024_s3072", batch=4, slots=3072, seed=12), rows=1024,
+    cached=3072)
+PREFILL_WORKLOADS = {p.name: p for p in (P1_PREFILL, P2_CHUNK)}
+
+
 def device_normal_bf16(shape, scale: float, seed: int, device="cuda"):
     """bf16 N(0, scale^2) tensor drawn on the device from a seeded torch generator.
 

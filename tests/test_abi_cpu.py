@@ -72,6 +72,8 @@ def test_null_arguments_are_rejected(libham):
     assert libham.ham_kv_free(None) == ham.HAM_OK
     assert libham.ham_decode_attn(None, 0, None, None, None) == ham.HAM_EINVAL
     assert libham.ham_kv_append(None, 0, None, None, None, None, None, None) == ham.HAM_EINVAL
+    assert libham.ham_prefill(None, 0, None, None, None, None, None, None, 0, None, 0,
+                              None) == ham.HAM_EINVAL
     assert libham.ham_slot_lengths(None, None, None, None) == ham.HAM_EINVAL
     assert libham.ham_kv_status(None, None, None) == ham.HAM_EINVAL
     assert libham.ham_kv_get_info(None, None) == ham.HAM_EINVAL
