@@ -93,6 +93,15 @@ def rank_cache_seed(workload_seed, rank, cache):
     return 1000 * workload_seed + 10 * rank + cache
 
 
+def measured_peak_bf16(sustained=False):
+    key = "bf16_tflops_sustained" if sustained else "bf16_tflops"
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)[key]), f"measured (MEASURED_PEAKS.json {key})"
+    except Exception:
+        return (1700.0 if sustained else 1900.0), "fallback"
+
+
 def measured_peak_hbm():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -214,8 +223,11 @@ def workload(name):
         return wl.embed_workload(int(name[len(EMBED_PREFIX):]))
     if name.startswith(EMBED_TOK_PREFIX) and name[len(EMBED_TOK_PREFIX):].isdigit():
         return wl.embed_tokens_workload(int(name[len(EMBED_TOK_PREFIX):]))
+    if name in wl.PREFILL_WORKLOADS:
+        return wl.PREFILL_WORKLOADS[name]
     if name not in wl.WORKLOADS:
-        raise SystemExit(f"unknown workload {name}; choose from {sorted(wl.WORKLOADS)} or "
+        raise SystemExit(f"unknown workload {name}; choose from "
+                         f"{sorted(wl.WORKLOADS) + sorted(wl.PREFILL_WORKLOADS)} or "
                          f"{STACK_PREFIX}<batch>, {EMBED_PREFIX}<batch>, "
                          f"{EMBED_TOK_PREFIX}<batch>")
     return wl.WORKLOADS[name]
@@ -668,6 +680,8 @@ def run_reference(args, w):
     from paper_2505_20438_gb300 import workload as wl
     if isinstance(w, wl.EmbedWorkload):
         return run_reference_embed(args, w)
+    if isinstance(w, wl.PrefillWorkload):
+        return run_reference_prefill(args, w)
     import dataclasses
 
     import oracle
@@ -1115,6 +1129,247 @@ def embed_cpu_baseline(c, seconds):
                       f"may use every core)"}
 
 
+# ---------------------------------------------------------------------------------------
+# chunked prefill (prompt ingestion)
+# ---------------------------------------------------------------------------------------
+
+PREFILL_METRIC = "chunked-prefill rows/s (prompt tokens ingested per second, one layer)"
+
+
+def prefill_flops(pw):
+    """Algorithmic FLOPs of one call: q.k and p.v (2 multiply-adds = 4 FLOPs per element of
+    head_dim) for every query head of every new row over the slots it attends."""
+    w = pw.w
+    n, L = pw.rows, pw.cached
+    attended = n * L + n * (n + 1) // 2          # sum over rows j of (L + j + 1)
+    return 4 * w.head_dim * w.n_q_heads * w.batch * attended
+
+
+def prefill_sample(pw, seconds, want_rows=None):
+    """Rows of the chunk the CPU oracle attends in a bounded sample: evenly spread over every
+    sequence's rows, so that their mean context is the chunk's."""
+    per_row = 4 * pw.w.head_dim * pw.w.n_q_heads * (pw.cached + pw.rows / 2)   # fp64 FLOPs
+    n = want_rows or max(8, int(seconds * 2e9 / per_row))                      # ~2 GFLOP/s
+    n = min(n, pw.rows * pw.w.batch)
+    import numpy as np
+    idx = np.linspace(0, pw.rows * pw.w.batch - 1, n).round().astype(np.int64)
+    want = np.zeros(pw.rows * pw.w.batch, bool)
+    want[idx] = True
+    return want
+
+
+def prefill_cpu(pw, seconds):
+    """The oracle as it stands on a bounded sample: every row appended, a spread sample of rows
+    attended; rows/s = sampled rows / time."""
+    import numpy as np
+
+    import oracle
+    from paper_2505_20438_gb300 import workload as wl
+    oracle.build()
+    B = pw.w.batch
+    case = wl.make_prefill_case(pw.w, [pw.rows] * B, cached=np.full(B, pw.cached, np.int32))
+    want = prefill_sample(pw, seconds)
+    oc = oracle.OracleCache.from_case(case.base)
+    q = case.q.copy()
+    t0 = time.perf_counter()
+    rc, _ = oc.prefill(q, case.k_new, case.v_new, case.offsets, ntok=case.ntok, want=want)
+    dt = time.perf_counter() - t0
+    if rc != 0:
+        raise RuntimeError(f"oracle prefill failed ({rc})")
+    return int(want.sum()) / dt, int(want.sum()), dt
+
+
+def run_reference_prefill(args, pw):
+    steps, warm = max(1, min(args.steps, 3)), 0
+    vals = []
+    for _ in range(steps):
+        v, n, dt = prefill_cpu(pw, args.cpu_seconds / steps)
+        vals.append(v)
+    value = sum(vals) / len(vals)
+    cores = oracle_threads()
+    print(json.dumps({
+        "impl": "reference", "metric": PREFILL_METRIC, "value": round(value, 3),
+        "unit": "rows/s", "n_gpus": 1, "steps": steps, "warmup": warm,
+        "ms_per_step": round(1e3 * pw.rows * pw.w.batch / value, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": pw.name, "batch": pw.w.batch, "rows": pw.rows,
+                   "cached": pw.cached},
+        "cpu_baseline": {"value": round(value, 3), "unit": "rows/s", "cores": cores,
+                         "kind": "oracle",
+                         "sample": f"each step: all {pw.rows * pw.w.batch} rows appended, "
+                                   f"{n} spread rows attended (fp64 C oracle, OpenMP)"},
+        "e2e": {"value": round(value, 3), "unit": "rows/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def oracle_threads():
+    try:
+        import oracle
+        return int(oracle.max_threads())
+    except Exception:
+        return os.cpu_count()
+
+
+def run_prefill(args, pw):
+    """One step = one ham_prefill call of the whole chunk (every sequence's rows: plan,
+    RoPE + append, causal attention).  The counters are set back to the cached length before
+    every call (one small kernel), so each step stores and attends the same slots."""
+    import numpy as np
+    import torch
+
+    from paper_2505_20438_gb300 import build as build_mod
+    from paper_2505_20438_gb300 import ham
+    from paper_2505_20438_gb300 import workload as wl
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1 and not torch.distributed.is_initialized():
+        torch.distributed.init_process_group("nccl")
+    build_mod.build()
+    w = pw.w
+    B = w.batch
+    case = wl.make_prefill_case(dataclasses_replace_seed(w, rank), [pw.rows] * B,
+                                cached=np.full(B, pw.cached, np.int32))
+    kv = ham.ham_kv_alloc(1, B, w.n_q_heads, w.n_kv_heads, w.head_dim, w.page_slots,
+                          case.base.max_slots, pool_pages=case.base.pool_pages)
+    ham.ham_kv_set_page_table(kv, case.base.page_table)
+
+    def dev(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(
+            torch.bfloat16).cuda()
+
+    if pw.cached:
+        ham.ham_kv_fill(kv, 0, dev(case.base.k), dev(case.base.v),
+                        torch.from_numpy(case.base.num_slots).cuda())
+    q, k_new, v_new = dev(case.q), dev(case.k_new), dev(case.v_new)
+    offsets = torch.from_numpy(case.offsets).cuda()
+    ntok = torch.from_numpy(case.ntok).cuda()
+    out = torch.empty_like(q)
+    lens = torch.full((B,), pw.cached, dtype=torch.int32, device="cuda")
+    toks = torch.full((B,), pw.cached, dtype=torch.int64, device="cuda")
+    stream = torch.cuda.Stream()
+    T = pw.rows * B
+
+    def step():
+        ham.ham_kv_set_lengths(kv, 0, lens, toks, stream=stream)
+        ham.ham_prefill(kv, 0, q, k_new, v_new, offsets, out, ntok=ntok, stream=stream)
+
+    steps = max(1, min(args.steps, 200))
+    warm = max(3, min(args.warmup, 20))
+    with torch.cuda.stream(stream):
+        for _ in range(warm):
+            step()
+    stream.synchronize()
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error in the warm-up")
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks, torch.cuda.stream(stream):
+        t0.record(stream)
+        for i in range(steps):
+            if i == steps - 1:
+                ham.ham_kv_set_lengths(kv, 0, lens, toks, stream=stream)
+                c0.record(stream)
+                ham.ham_prefill(kv, 0, q, k_new, v_new, offsets, out, ntok=ntok, stream=stream)
+                c1.record(stream)
+            else:
+                step()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed_ms = max_over_ranks(t0.elapsed_time(t1), world, "cuda")
+    if world > 1:
+        torch.distributed.barrier()
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error during the timed region")
+    # the call alone, timed over a short run of calls (events around each ham_prefill)
+    call_ms = []
+    with torch.cuda.stream(stream):
+        for _ in range(5):
+            ham.ham_kv_set_lengths(kv, 0, lens, toks, stream=stream)
+            c0.record(stream)
+            ham.ham_prefill(kv, 0, q, k_new, v_new, offsets, out, ntok=ntok, stream=stream)
+            c1.record(stream)
+            c1.synchronize()
+            call_ms.append(c0.elapsed_time(c1))
+    call_ms = sorted(call_ms)[len(call_ms) // 2]
+    flops = prefill_flops(pw)
+    peak, peak_src = measured_peak_bf16()
+    achieved = flops / (call_ms * 1e-3) / 1e12
+    value = world * T * steps / (elapsed_ms * 1e-3)
+
+    # end to end: pinned host -> device copies of the chunk's q, k, v and offsets, the call,
+    # device -> pinned host copy of the output, read on the host
+    hq, hk, hv = q.cpu().pin_memory(), k_new.cpu().pin_memory(), v_new.cpu().pin_memory()
+    hoff = offsets.cpu().pin_memory()
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    n_e2e = max(3, min(args.e2e_steps, 20))
+    checksum = 0.0
+    te = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for _ in range(n_e2e):
+            q.copy_(hq, non_blocking=True)
+            k_new.copy_(hk, non_blocking=True)
+            v_new.copy_(hv, non_blocking=True)
+            offsets.copy_(hoff, non_blocking=True)
+            ham.ham_kv_set_lengths(kv, 0, lens, toks, stream=stream)
+            ham.ham_prefill(kv, 0, q, k_new, v_new, offsets, out, ntok=ntok, stream=stream)
+            hout.copy_(out, non_blocking=True)
+            stream.synchronize()
+            checksum += float(hout[0, 0, 0])
+    dte = max_over_ranks(time.perf_counter() - te, world, "cuda")
+    h2d = sum(t.numel() * t.element_size() for t in (q, k_new, v_new, offsets))
+    result = {
+        "metric": PREFILL_METRIC, "value": round(value, 1), "unit": "rows/s", "n_gpus": world,
+        "steps": steps, "warmup": warm, "ms_per_step": round(elapsed_ms / steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "accum_dtype": "f32", "data": "synthetic",
+        "config": {"workload": pw.name, "batch": B, "rows_per_sequence": pw.rows,
+                   "cached_slots": pw.cached, "n_q_heads": w.n_q_heads,
+                   "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+                   "page_slots": w.page_slots, "tokens_per_row": 1,
+                   "step": "ham_kv_set_lengths + ham_prefill (plan, RoPE + append, causal "
+                           "attention) of the whole chunk",
+                   "l2": "inputs larger than L2 (q, out 134 MB each at the 4 x 4096 chunk)"},
+        "tflops": round(achieved, 1),
+        "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
+                     "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
+                     "kernel": "prefill_attn_kernel (with the plan and RoPE + append "
+                               "kernels of the same call)",
+                     "algorithmic_flops_per_launch": int(flops),
+                     "avg_launch_us": round(call_ms * 1e3, 1), "peak_source": peak_src,
+                     "duration_method": "CUDA events around one ham_prefill call (3 "
+                                        "kernels), median of 5"},
+        "gpu_launches": steps * 4 * world,
+        "e2e": {"value": round(world * T * n_e2e / dte, 1), "unit": "rows/s",
+                "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(out.numel() * out.element_size()),
+                "steps": n_e2e, "finite": math.isfinite(checksum),
+                "path": "every step: pinned host -> device copies of q, k, v and offsets, "
+                        "ham_prefill, device -> pinned host copy of the output"},
+        "clocks": clocks.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, n, dt = prefill_cpu(pw, args.cpu_seconds)
+        result["cpu_baseline"] = {
+            "value": round(v, 3), "unit": "rows/s", "cores": oracle_threads(), "kind": "oracle",
+            "sample": f"all {T} rows appended, {n} spread rows attended in {dt:.1f} s (fp64 C "
+                      f"oracle, OpenMP)"}
+    ham.ham_kv_free(kv)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+def dataclasses_replace_seed(w, rank):
+    """Rank r's sequences: the workload's seed shifted by the rank (ranks own different
+    sequences)."""
+    import dataclasses
+    return dataclasses.replace(w, seed=w.seed + 100 * rank)
+
+
 def main():
     global CACHES
     args = parse_args()
@@ -1127,6 +1382,8 @@ def main():
         run_reference(args, w)
     elif isinstance(w, wl.EmbedWorkload):
         run_embed(args, w)
+    elif isinstance(w, wl.PrefillWorkload):
+        run_prefill(args, w)
     elif w.layers > 1:
         run_stack(args, w)
     else:

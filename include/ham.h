@@ -196,7 +196,8 @@ int ham_slot_lengths(ham_kv *kv, int32_t *num_slots_host, int64_t *num_tokens_ho
  * out      device [total_rows][n_q_heads][head_dim], bf16 or f32 (out_dtype)
  * A sequence whose rows cannot all be stored (a token count < 1, no room for them, a bad
  * page, offsets that leave the call's rows) gets no slot, keeps q unrotated and 0 out
- * rows, and sets the device error word.  total_rows == 0 launches nothing.  Three launches
+ * rows, and sets the device error word.  total_rows == 0 launches nothing (the buffers may
+ * then be NULL).  Three launches
  * on `stream` (plan, RoPE + append, attention).  q_inout, out, k_new and v_new must not
  * overlap each other or the cache.  Host errors: HAM_EINVAL (NULL / unaligned / overlapping
  * pointers, layer or out_dtype out of range, total_rows above batch * max_slots_per_seq),

@@ -637,13 +637,14 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
                 int32_t total_rows, void *out, int32_t out_dtype, void *stream) {
   int rc = check_layer(kv, layer);
   if (rc) return rc;
-  if (!q_inout || !k_new || !v_new || !offsets || !out)
-    return fail(HAM_EINVAL, "q_inout, k_new, v_new, offsets and out are required");
   if (out_dtype != HAM_DTYPE_BF16 && out_dtype != HAM_DTYPE_F32)
     return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
   const ham_config &c = kv->cfg;
   if (total_rows < 0 || (int64_t)total_rows > (int64_t)c.batch * c.max_slots_per_seq)
     return fail(HAM_EINVAL, "total_rows %d outside 0..batch * max_slots_per_seq", total_rows);
+  if (total_rows == 0) return HAM_OK;  // nothing to store or attend (the buffers may be NULL)
+  if (!q_inout || !k_new || !v_new || !offsets || !out)
+    return fail(HAM_EINVAL, "q_inout, k_new, v_new, offsets and out are required");
   if (!aligned16(q_inout) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out))
     return fail(HAM_EINVAL, "q/k/v/out must be 16-byte aligned");
   if (((uintptr_t)offsets & 3u) || ((uintptr_t)pos & 3u) || ((uintptr_t)ntok & 3u))
@@ -666,7 +667,6 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
   if (blocks > 65535)
     return fail(HAM_EINVAL, "total_rows %d: split the chunk (at most %lld query blocks a call)",
                 total_rows, 65535LL);
-  if (total_rows == 0) return HAM_OK;
   DeviceGuard guard(kv->device);
   ham::PrefillView v{};
   v.k_pool = layer_pool(kv, layer, 0);
