@@ -140,7 +140,9 @@ struct PrefillView {
   const int32_t *page_table;
   int32_t *num_slots;          // [batch] of this layer
   int64_t *num_tokens;         // [batch] of this layer
-  const double2 *rope_table;   // [rope_positions][head_dim / 2]: (cos, sin), fp64
+  const float4 *rope_table_ff; // [rope_positions][head_dim / 2]: (cos, sin) of the fp64 table,
+                               // each as an fp32 pair (hi, lo) with hi + lo = the fp64 value to
+                               // about 48 bits
   const double *inv_freq;      // [head_dim / 2] (positions past the table)
   int64_t rope_positions;
   uint16_t *q;                 // [rows][n_q_heads][head_dim], rotated in place
@@ -172,9 +174,11 @@ cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, con
 int attention_ctas_per_sm(int head_dim, int group, int batch, bool step);
 bool attention_supported(int head_dim, int group);
 // TMA map of one pool [pool_pages][n_kv_heads][page_slots][head_dim] bf16 viewed as
-// {64 elements, head_dim / 64, rows} with a box of {64, head_dim / 64, 16 rows} and the
-// 128-byte swizzle.  Returns a CUresult (0 on success).
-int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim);
+// {64 elements, head_dim / 64, rows} with a box of {64, head_dim / 64, 16 rows} (half_box:
+// {64, 1, 16 rows}, one 64-column half of a chunk) and the 128-byte swizzle.  Returns a
+// CUresult (0 on success).
+int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim,
+                         bool half_box);
 cudaError_t launch_append(const AppendView &v, cudaStream_t stream);
 // KV heads per append block (0 if the shape does not fit the append kernel).
 int append_kv_per_block(int n_q_heads, int n_kv_heads, int head_dim);
@@ -209,6 +213,7 @@ struct ham_kv {
   double *inv_freq = nullptr;
   double2 *rope_table = nullptr;  // own allocation
   float2 *rope_table_f = nullptr;  // own allocation
+  float4 *rope_table_ff = nullptr;  // own allocation: fp32 (hi, lo) pairs of the fp64 table
   int64_t rope_positions = 0;
   int32_t *err = nullptr;
   int4 *stash = nullptr;           // fused step: per-sequence append record
@@ -220,5 +225,6 @@ struct ham_kv {
   int32_t *prefill_pos = nullptr;  // ham_prefill: per-row positions [batch * max_slots]
   int64_t scratch_bytes = 0;
   std::vector<CUtensorMap> tmaps;  // [layers][2]: TMA maps of the K and V pools
+  std::vector<CUtensorMap> tmaps_half;  // [layers][2]: the same, one 64-column half per box
   void *host_stage = nullptr;   // pinned: counters and error word read-back
 };

@@ -99,8 +99,8 @@ int ham_decode_attn_noalloc(const ham_attn_args *a, void *stream) {
   }
 
   CUtensorMap tk, tv;
-  if (ham::make_pool_tensor_map(&tk, a->k_pool, rows, a->head_dim) != 0 ||
-      ham::make_pool_tensor_map(&tv, a->v_pool, rows, a->head_dim) != 0)
+  if (ham::make_pool_tensor_map(&tk, a->k_pool, rows, a->head_dim, false) != 0 ||
+      ham::make_pool_tensor_map(&tv, a->v_pool, rows, a->head_dim, false) != 0)
     return noalloc_fail(HAM_ECUDA, "cuTensorMapEncodeTiled failed for the pools");
 
   unsigned char *base = static_cast<unsigned char *>(setup.scratch);

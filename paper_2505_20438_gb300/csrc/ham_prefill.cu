@@ -21,8 +21,9 @@
 //     microseconds.
 //  3. prefill_attn_kernel, one CTA per (KV head, block of 128 / G query rows of one sequence):
 //     eight consumer warps, each one 16-row m-tile of one query head, and a producer warp that
-//     streams 64-slot K/V tiles (four 16-slot chunks, TMA with the 128-byte swizzle) through a
-//     shared-memory ring.  S = Q K^T and O += P V are mma.sync m16n8k16 (bf16 in, fp32
+//     streams 64-slot K/V tiles (four 16-slot chunks, each 64-column half of a chunk one TMA
+//     copy with the 128-byte swizzle, so that ldmatrix reads are free of bank conflicts)
+//     through a shared-memory ring.  S = Q K^T and O += P V are mma.sync m16n8k16 (bf16 in, fp32
 //     accumulate); the softmax is online, fp32, in the exp2 domain; the causal mask applies to
 //     the tiles that reach past a row's own slot, and tiles past a warp's last row are skipped.
 //     CTAs are scheduled latest query block first, the longest rows of the causal triangle.
@@ -42,7 +43,7 @@ namespace ham {
 namespace {
 
 constexpr int kPlanThreads = 256;
-constexpr int kRopeThreads = 128;
+constexpr int kRopeThreads = 256;
 
 // ------------------------------------------------------------------------------------
 // 1. plan
@@ -192,6 +193,8 @@ __device__ __forceinline__ void split_double(double x, float &hi, float &lo) {
   lo = __double2float_rn(x - (double)hi);  // x - hi is exact in fp64
 }
 
+// One block per row; a thread owns four consecutive pairs (i, i + d/2), i = 4 (tid % (d/8)) ..,
+// of one head at a time (8-byte loads and stores of each half).
 template <typename OutT>
 __global__ void __launch_bounds__(kRopeThreads) prefill_rope_kernel(PrefillView v) {
   const int64_t r = blockIdx.x;
@@ -222,20 +225,22 @@ __global__ void __launch_bounds__(kRopeThreads) prefill_rope_kernel(PrefillView 
     reinterpret_cast<uint4 *>(v.v_pool + ((page * Hkv + gg) * v.page_slots + prow) * D)[k] =
         reinterpret_cast<const uint4 *>(v.v_new + (r * Hkv + gg) * D)[k];
   }
-  const int i = threadIdx.x % half;
-  double c, s;
+  const int quads = half / 4, i0 = 4 * (threadIdx.x % quads);
+  float4 cs[4];  // (c_hi, c_lo, s_hi, s_lo) of frequencies i0 .. i0 + 3
   if (p >= 0 && p < v.rope_positions) {
-    const double2 cs = v.rope_table[(int64_t)p * half + i];
-    c = cs.x;
-    s = cs.y;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) cs[e] = v.rope_table_ff[(int64_t)p * half + i0 + e];
   } else {
-    sincos((double)p * v.inv_freq[i], &s, &c);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      double c, sn;
+      sincos((double)p * v.inv_freq[i0 + e], &sn, &c);
+      split_double(c, cs[e].x, cs[e].y);
+      split_double(sn, cs[e].z, cs[e].w);
+    }
   }
-  float ch, cl, sh, sl;
-  split_double(c, ch, cl);
-  split_double(s, sh, sl);
-  // query heads in place, then the key heads into the slot; one thread owns a pair (i, i + d/2)
-  for (int hh = threadIdx.x / half; hh < Hq + Hkv; hh += kRopeThreads / half) {
+  // query heads in place, then the key heads into the slot
+  for (int hh = threadIdx.x / quads; hh < Hq + Hkv; hh += kRopeThreads / quads) {
     const uint16_t *src;
     uint16_t *dst;
     if (hh < Hq) {
@@ -245,14 +250,28 @@ __global__ void __launch_bounds__(kRopeThreads) prefill_rope_kernel(PrefillView 
       src = v.k_new + (r * Hkv + gg) * D;
       dst = v.k_pool + ((page * Hkv + gg) * v.page_slots + prow) * D;
     }
-    const float x0 = bf16_value(src[i]), x1 = bf16_value(src[i + half]);
-    const uint16_t y0 = rotate_dd(x0, x1, ch, cl, sh, sl);               // x0 c - x1 s
-    const uint16_t y1 = rotate_dd(x1, x0, ch, cl, -sh, -sl);  // x1 c + x0 s
-    dst[i] = y0;
-    dst[i + half] = y1;
+    const uint2 xl = *reinterpret_cast<const uint2 *>(src + i0);
+    const uint2 xh = *reinterpret_cast<const uint2 *>(src + i0 + half);
+    const uint32_t wl[2] = {xl.x, xl.y}, wh[2] = {xh.x, xh.y};
+    uint32_t yl[2], yh[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      uint32_t ol = 0, oh = 0;
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const float4 c4 = cs[2 * k + e];
+        const float x0 = bf16_value((uint16_t)(wl[k] >> (16 * e)));
+        const float x1 = bf16_value((uint16_t)(wh[k] >> (16 * e)));
+        ol |= (uint32_t)rotate_dd(x0, x1, c4.x, c4.y, c4.z, c4.w) << (16 * e);   // x0 c - x1 s
+        oh |= (uint32_t)rotate_dd(x1, x0, c4.x, c4.y, -c4.z, -c4.w) << (16 * e); // x1 c + x0 s
+      }
+      yl[k] = ol;
+      yh[k] = oh;
+    }
+    *reinterpret_cast<uint2 *>(dst + i0) = make_uint2(yl[0], yl[1]);
+    *reinterpret_cast<uint2 *>(dst + i0 + half) = make_uint2(yh[0], yh[1]);
   }
 }
-
 
 // ------------------------------------------------------------------------------------
 // 3. causal attention of the chunk
@@ -274,6 +293,15 @@ struct PShape {
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
   static_assert(kStages >= 2, "ring depth");
 };
+
+// A chunk tile in shared memory: its 64-column halves one after the other, each 16 slot rows
+// of 128 bytes written by its own TMA copy with the 128-byte swizzle.  Byte offset of the
+// 16-byte piece c (elements 8c .. 8c+7) of slot row `row`: the piece index inside the line is
+// XORed with the row, so the eight rows of an ldmatrix matrix hit eight different bank groups.
+constexpr int kHalfBytes = kChunkSlots * 128;
+__device__ __forceinline__ uint32_t half_tile_offset(int row, int c) {
+  return (uint32_t)((c >> 3) * kHalfBytes + row * 128 + (((c & 7) ^ (row & 7)) << 4));
+}
 
 template <typename OutT>
 __device__ __forceinline__ void store_pair(void *out, int64_t i, float x, float y) {
@@ -363,9 +391,13 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
 #pragma unroll
       for (int c = 0; c < S::kChunks; ++c) {
         if (!(mask & (1 << c))) continue;
-        tma_load_3d(dst + c * S::kChunkBytes, &tmap_k, 0, 0, rows[c], &full[s], pol);
-        tma_load_3d(dst + (S::kChunks + c) * S::kChunkBytes, &tmap_v, 0, 0, rows[c], &full[s],
-                    pol);
+#pragma unroll
+        for (int hh = 0; hh < D / 64; ++hh) {  // one 64-column half of the chunk per copy
+          tma_load_3d(dst + c * S::kChunkBytes + hh * kHalfBytes, &tmap_k, 0, hh, rows[c],
+                      &full[s], pol);
+          tma_load_3d(dst + (S::kChunks + c) * S::kChunkBytes + hh * kHalfBytes, &tmap_v, 0, hh,
+                      rows[c], &full[s], pol);
+        }
       }
       issued = t + 1;
     }
@@ -422,16 +454,16 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
 #pragma unroll
       for (int nb = 0; nb < 2 * S::kChunks; ++nb) sc[nb][0] = sc[nb][1] = sc[nb][2] = sc[nb][3] = 0.f;
       // S = Q K^T: per chunk, ldmatrix matrices (slots 0-7 | 8-15) x (d lo | hi) give the
-      // B fragments of the chunk's two 8-slot n-blocks
+      // B fragments of the chunk's two 8-slot n-blocks.  k-steps outside, chunks inside: the
+      // eight accumulators take turns instead of chaining on one.
 #pragma unroll
-      for (int c = 0; c < S::kChunks; ++c) {
-        if (tbase + c * kChunkSlots >= warp_end) continue;
-        const uint8_t *kc = kt + c * S::kChunkBytes;
+      for (int ks = 0; ks < S::kKSteps; ++ks) {
 #pragma unroll
-        for (int ks = 0; ks < S::kKSteps; ++ks) {
+        for (int c = 0; c < S::kChunks; ++c) {
+          if (tbase + c * kChunkSlots >= warp_end) continue;
           uint32_t kf[4];
-          ldmatrix_x4(kf, smem_u32(kc + swizzle128_offset((mi >> 1) * 8 + mr, 2 * ks + (mi & 1),
-                                                          D / 64)));
+          ldmatrix_x4(kf, smem_u32(kt + c * S::kChunkBytes +
+                                   half_tile_offset((mi >> 1) * 8 + mr, 2 * ks + (mi & 1))));
           mma_16816(sc[2 * c], qf[ks], kf[0], kf[1]);
           mma_16816(sc[2 * c + 1], qf[ks], kf[2], kf[3]);
         }
@@ -492,8 +524,8 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
 #pragma unroll
         for (int np = 0; np < D / 16; ++np) {
           uint32_t vf[4];
-          ldmatrix_x4_trans(vf, smem_u32(vc + swizzle128_offset((mi & 1) * 8 + mr,
-                                                                2 * np + (mi >> 1), D / 64)));
+          ldmatrix_x4_trans(vf, smem_u32(vc + half_tile_offset((mi & 1) * 8 + mr,
+                                                               2 * np + (mi >> 1))));
           mma_16816(o[2 * np], pa, vf[0], vf[1]);
           mma_16816(o[2 * np + 1], pa, vf[2], vf[3]);
         }

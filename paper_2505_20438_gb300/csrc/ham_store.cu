@@ -214,7 +214,8 @@ __global__ void set_lengths_kernel(int32_t *num_slots, int64_t *num_tokens,
   if (new_tokens) num_tokens[b] = new_tokens[b];
 }
 
-int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim) {
+int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim,
+                         bool half_box) {
   using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
                               const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
                               const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
@@ -231,7 +232,8 @@ int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int h
   }
   const cuuint64_t dims[3] = {64, (cuuint64_t)(head_dim / 64), (cuuint64_t)rows};
   const cuuint64_t strides[2] = {128, (cuuint64_t)head_dim * 2};  // bytes, dims 1 and 2
-  const cuuint32_t box[3] = {64, (cuuint32_t)(head_dim / 64), (cuuint32_t)kChunkSlots};
+  const cuuint32_t box[3] = {64, half_box ? 1u : (cuuint32_t)(head_dim / 64),
+                             (cuuint32_t)kChunkSlots};
   const cuuint32_t estride[3] = {1, 1, 1};
   return (int)encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(pool), dims,
                      strides, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -395,16 +397,20 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     const int64_t half = cfg.head_dim / 2;
     const int64_t reach = (int64_t)cfg.max_slots_per_seq * (cfg.pos_mode == HAM_POS_TOKEN ? 4 : 1);
     const int64_t cap = (int64_t)(512u << 20) /
-                        (half * (int64_t)(sizeof(double2) + sizeof(float2)));
+                        (half * (int64_t)(sizeof(double2) + sizeof(float2) + sizeof(float4)));
     kv->rope_positions = std::min(reach, cap);
     std::vector<double2> table((size_t)(kv->rope_positions * half));
     std::vector<float2> table_f(table.size());
+    std::vector<float4> table_ff(table.size());  // (c_hi, c_lo, s_hi, s_lo): c = c_hi + c_lo
     for (int64_t p = 0; p < kv->rope_positions; ++p)
       for (int64_t i = 0; i < half; ++i) {
         const double theta = (double)p * inv_freq[(size_t)i];
         const double c = cos(theta), s = sin(theta);
         table[(size_t)(p * half + i)] = make_double2(c, s);
         table_f[(size_t)(p * half + i)] = make_float2((float)c, (float)s);
+        const float ch = (float)c, sh = (float)s;
+        table_ff[(size_t)(p * half + i)] =
+            make_float4(ch, (float)(c - (double)ch), sh, (float)(s - (double)sh));
       }
     e = cudaMalloc(&kv->rope_table, table.size() * sizeof(double2));
     if (e == cudaSuccess)
@@ -414,6 +420,10 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     if (e == cudaSuccess)
       e = cudaMemcpy(kv->rope_table_f, table_f.data(), table_f.size() * sizeof(float2),
                      cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMalloc(&kv->rope_table_ff, table_ff.size() * sizeof(float4));
+    if (e == cudaSuccess)
+      e = cudaMemcpy(kv->rope_table_ff, table_ff.data(), table_ff.size() * sizeof(float4),
+                     cudaMemcpyHostToDevice);
   }
   if (e != cudaSuccess) {
     int rc = cuda_fail(e, "initialising the cache");
@@ -421,11 +431,15 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     return rc;
   }
   kv->tmaps.resize((size_t)cfg.layers * 2);
+  kv->tmaps_half.resize((size_t)cfg.layers * 2);
   const int64_t rows = cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots;
   for (int layer = 0; layer < cfg.layers; ++layer) {
     for (int which = 0; which < 2; ++which) {
       int r = ham::make_pool_tensor_map(&kv->tmaps[(size_t)layer * 2 + which],
-                                        layer_pool(kv, layer, which), rows, cfg.head_dim);
+                                        layer_pool(kv, layer, which), rows, cfg.head_dim, false);
+      if (r == 0)
+        r = ham::make_pool_tensor_map(&kv->tmaps_half[(size_t)layer * 2 + which],
+                                      layer_pool(kv, layer, which), rows, cfg.head_dim, true);
       if (r != 0) {
         ham_kv_free(kv);
         return fail(HAM_ECUDA, "cuTensorMapEncodeTiled failed (CUresult %d)", r);
@@ -444,6 +458,7 @@ int ham_kv_free(ham_kv *kv) {
   if (kv->meta) cudaFree(kv->meta);
   if (kv->rope_table) cudaFree(kv->rope_table);
   if (kv->rope_table_f) cudaFree(kv->rope_table_f);
+  if (kv->rope_table_ff) cudaFree(kv->rope_table_ff);
   if (kv->host_stage) cudaFreeHost(kv->host_stage);
   delete kv;
   return HAM_OK;
@@ -676,7 +691,7 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
   v.page_table = kv->page_table;
   v.num_slots = kv->num_slots + (size_t)layer * c.batch;
   v.num_tokens = kv->num_tokens + (size_t)layer * c.batch;
-  v.rope_table = kv->rope_table;
+  v.rope_table_ff = kv->rope_table_ff;
   v.inv_freq = kv->inv_freq;
   v.rope_positions = kv->rope_positions;
   v.q = static_cast<uint16_t *>(q_inout);
@@ -699,8 +714,8 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
   v.max_pages = kv->max_pages;
   v.max_slots = c.max_slots_per_seq;
   v.pos_mode = c.pos_mode;
-  cudaError_t e = ham::launch_prefill(kv->tmaps[(size_t)layer * 2],
-                                      kv->tmaps[(size_t)layer * 2 + 1], v, out_dtype,
+  cudaError_t e = ham::launch_prefill(kv->tmaps_half[(size_t)layer * 2],
+                                      kv->tmaps_half[(size_t)layer * 2 + 1], v, out_dtype,
                                       static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
   note_launch(kv, layer, stream, true);
