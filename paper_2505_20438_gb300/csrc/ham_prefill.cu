@@ -43,6 +43,7 @@ namespace ham {
 namespace {
 
 constexpr int kPlanThreads = 256;
+constexpr float kRescaleSlack = 8.0f;  // log2 units: the running max lags by at most 2^8
 constexpr int kRopeThreads = 256;
 
 // ------------------------------------------------------------------------------------
@@ -166,10 +167,20 @@ __device__ __forceinline__ uint16_t bf16_of_pair(float hi, float lo) {
 }
 
 // a c - b s rounded once to bf16, with c = ch + cl and s = sh + sl given as fp32 pairs and a, b
-// exact (bf16 values).  Products by FMA error terms and sums by two-sum are exact; only the
-// small terms are rounded, so the pair carries about 48 bits of the exact value.
+// exact (bf16 values).  Near a rounding boundary: products by FMA error terms and sums by
+// two-sum are exact, only the small terms are rounded, so the pair carries about 48 bits of
+// the exact value.
 __device__ __forceinline__ uint16_t rotate_dd(float a, float b, float ch, float cl, float sh,
                                               float sl) {
+  // Fast path: y = a ch - b sh in plain fp32 lies within 3 * 2^-24 (|a| + |b|) < e / 2 of the
+  // exact a c - b s.  When no bf16 rounding boundary is within e of y (the nearest one is the
+  // midpoint sharing y's upper 16 bits; the others are a quarter of a bf16 spacing away, more
+  // than e once e < 2^-11 |y|), the exact value rounds as y does.
+  const float y = __fmaf_rn(a, ch, -__fmul_rn(b, sh));
+  const float e = __fmul_rn(__fadd_rn(fabsf(a), fabsf(b)), 0x1p-21f);
+  const float mid = __uint_as_float((__float_as_uint(y) & 0xFFFF0000u) | 0x8000u);
+  if (fabsf(__fsub_rn(y, mid)) > e && e < __fmul_rn(fabsf(y), 0x1p-11f))
+    return __bfloat16_as_ushort(__float2bfloat16_rn(y));
   const float p1 = __fmul_rn(a, ch), e1 = __fmaf_rn(a, ch, -p1);
   const float p2 = __fmul_rn(b, sh), e2 = __fmaf_rn(b, sh, -p2);
   const float s = __fsub_rn(p1, p2);  // two-sum of p1 and -p2: s + t = p1 - p2
@@ -312,8 +323,10 @@ __device__ __forceinline__ void store_pair(void *out, int64_t i, float x, float 
   }
 }
 
+// One CTA per SM either way (its ring takes 96 KiB and its nine warps most of the register
+// file), so the compiler may use up to 216 registers a thread (no spills at head_dim 128).
 template <int D, typename OutT>
-__global__ void __launch_bounds__(PShape<D>::kThreads, 1)
+__global__ void __maxnreg__(216)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
                         const __grid_constant__ CUtensorMap tmap_v, const PrefillView v) {
   using S = PShape<D>;
@@ -468,16 +481,22 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
           mma_16816(sc[2 * c + 1], qf[ks], kf[2], kf[3]);
         }
       }
-      // scale, causal mask and copied chunks; row maxima over the quad
+      // causal mask and copied chunks (only on tiles that reach past the m-tile's first row or
+      // miss a chunk); row maxima of the raw scores over the quad
+      if (tbase + S::kTile - 1 > L + j0 || mask != (1 << S::kChunks) - 1) {
+#pragma unroll
+        for (int nb = 0; nb < 2 * S::kChunks; ++nb) {
+          const bool cok = (mask >> (nb >> 1)) & 1;
+          const int slot = tbase + nb * 8 + 2 * (lane & 3);
+          if (!(cok && slot <= lim_a)) sc[nb][0] = -INFINITY;
+          if (!(cok && slot + 1 <= lim_a)) sc[nb][1] = -INFINITY;
+          if (!(cok && slot <= lim_b)) sc[nb][2] = -INFINITY;
+          if (!(cok && slot + 1 <= lim_b)) sc[nb][3] = -INFINITY;
+        }
+      }
       float mx_a = -INFINITY, mx_b = -INFINITY;
 #pragma unroll
       for (int nb = 0; nb < 2 * S::kChunks; ++nb) {
-        const bool cok = (mask >> (nb >> 1)) & 1;
-        const int slot = tbase + nb * 8 + 2 * (lane & 3);
-        sc[nb][0] = cok && slot <= lim_a ? sc[nb][0] * sl2 : -INFINITY;
-        sc[nb][1] = cok && slot + 1 <= lim_a ? sc[nb][1] * sl2 : -INFINITY;
-        sc[nb][2] = cok && slot <= lim_b ? sc[nb][2] * sl2 : -INFINITY;
-        sc[nb][3] = cok && slot + 1 <= lim_b ? sc[nb][3] * sl2 : -INFINITY;
         mx_a = fmaxf(mx_a, fmaxf(sc[nb][0], sc[nb][1]));
         mx_b = fmaxf(mx_b, fmaxf(sc[nb][2], sc[nb][3]));
       }
@@ -486,30 +505,41 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
         mx_a = fmaxf(mx_a, __shfl_xor_sync(kFull, mx_a, off));
         mx_b = fmaxf(mx_b, __shfl_xor_sync(kFull, mx_b, off));
       }
-      const float mn_a = fmaxf(m_a, mx_a), mn_b = fmaxf(m_b, mx_b);
-      const float ref_a = mn_a == -INFINITY ? 0.f : mn_a;  // nothing attended yet
-      const float ref_b = mn_b == -INFINITY ? 0.f : mn_b;
-      const float al_a = ex2(m_a - ref_a), al_b = ex2(m_b - ref_b);
-      m_a = mn_a;
-      m_b = mn_b;
+      // Running maxima in the exp2 domain, raised lazily: only when a score passes them by more
+      // than kRescaleSlack (p then stays below 2^kRescaleSlack), so most tiles skip rescaling O.
+      mx_a *= sl2;
+      mx_b *= sl2;
+      float al_a = 1.f, al_b = 1.f;
+      if (mx_a > m_a + kRescaleSlack) {
+        al_a = ex2(m_a - mx_a);
+        m_a = mx_a;
+      }
+      if (mx_b > m_b + kRescaleSlack) {
+        al_b = ex2(m_b - mx_b);
+        m_b = mx_b;
+      }
+      const float ref_a = m_a == -INFINITY ? 0.f : m_a;  // nothing attended yet
+      const float ref_b = m_b == -INFINITY ? 0.f : m_b;
       float rs_a = 0.f, rs_b = 0.f;
 #pragma unroll
       for (int nb = 0; nb < 2 * S::kChunks; ++nb) {
-        sc[nb][0] = ex2(sc[nb][0] - ref_a);
-        sc[nb][1] = ex2(sc[nb][1] - ref_a);
-        sc[nb][2] = ex2(sc[nb][2] - ref_b);
-        sc[nb][3] = ex2(sc[nb][3] - ref_b);
+        sc[nb][0] = ex2(fmaf(sc[nb][0], sl2, -ref_a));
+        sc[nb][1] = ex2(fmaf(sc[nb][1], sl2, -ref_a));
+        sc[nb][2] = ex2(fmaf(sc[nb][2], sl2, -ref_b));
+        sc[nb][3] = ex2(fmaf(sc[nb][3], sl2, -ref_b));
         rs_a += sc[nb][0] + sc[nb][1];
         rs_b += sc[nb][2] + sc[nb][3];
       }
       l_a = l_a * al_a + rs_a;  // per-lane partial sums, reduced over the quad at the end
       l_b = l_b * al_b + rs_b;
+      if (__any_sync(kFull, al_a != 1.f || al_b != 1.f)) {
 #pragma unroll
-      for (int on = 0; on < S::kONBlocks; ++on) {
-        o[on][0] *= al_a;
-        o[on][1] *= al_a;
-        o[on][2] *= al_b;
-        o[on][3] *= al_b;
+        for (int on = 0; on < S::kONBlocks; ++on) {
+          o[on][0] *= al_a;
+          o[on][1] *= al_a;
+          o[on][2] *= al_b;
+          o[on][3] *= al_b;
+        }
       }
       // O += P V: P of chunk kk is the A fragment of k-step kk; V by transposing ldmatrix
       // (matrices (slots 0-7 | 8-15) x (d lo | hi))
