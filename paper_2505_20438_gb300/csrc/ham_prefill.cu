@@ -323,10 +323,11 @@ __device__ __forceinline__ void store_pair(void *out, int64_t i, float x, float 
   }
 }
 
-// One CTA per SM either way (its ring takes 96 KiB and its nine warps most of the register
-// file), so the compiler may use up to 216 registers a thread (no spills at head_dim 128).
+// One CTA per SM.  Registers are granted to a block in groups of four warps, so the nine warps
+// (twelve as allocated) may use at most 170 registers a thread: 168, with a few bytes spilled
+// at head_dim 128.
 template <int D, typename OutT>
-__global__ void __maxnreg__(216)
+__global__ void __launch_bounds__(PShape<D>::kThreads, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
                         const __grid_constant__ CUtensorMap tmap_v, const PrefillView v) {
   using S = PShape<D>;
