@@ -37,6 +37,7 @@
 #include <type_traits>
 
 #include "ham_internal.cuh"
+#include "ham_prefill.cuh"
 #include "ham_ptx.cuh"
 
 namespace ham {

@@ -15,6 +15,7 @@
 #include <vector>
 
 #include "ham_internal.cuh"
+#include "ham_prefill.cuh"
 
 namespace {
 
