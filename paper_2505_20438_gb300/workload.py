@@ -343,3 +343,37 @@ def make_embed_tokens_case(w: EmbedWorkload, vocab: int,
     ids = rng.integers(0, vocab, int(c.offsets[-1]), dtype=np.int32)
     c.x = table[ids]
     return EmbedTokensCase(c, table, ids)
+
+
+# ---------------------------------------------------------------------------------------
+# Macro-step layer front: the layer input x of width H is projected to q, k, v by one fused
+# bias-free weight [W_q; W_k; W_v] ([out][in]), as in the Llama base model (Sec. 4.1).  The
+# weights are drawn N(0, 1/H) (so q, k, v are about N(0, 1) for x ~ N(0, 1)), the inputs
+# N(0, 1), as a normalised hidden state is.
+# ---------------------------------------------------------------------------------------
+@dataclasses.dataclass(frozen=True)
+class FrontWorkload:
+    name: str
+    batch: int
+    hidden: int
+    n_q_heads: int = 32
+    n_kv_heads: int = 8
+    head_dim: int = 128
+    seed: int = 0
+
+    @property
+    def out_rows(self) -> int:
+        return (self.n_q_heads + 2 * self.n_kv_heads) * self.head_dim
+
+
+def front_workload(batch: int, hidden: int = 4096, **kw) -> FrontWorkload:
+    """Llama-3-8B-shaped layer front (H 4096, 32/8 heads of 128) unless overridden."""
+    return FrontWorkload(f"qkv_front_b{batch}_h{hidden}", batch=batch, hidden=hidden, **kw)
+
+
+def front_inputs(w: FrontWorkload, stream: int = 0):
+    """(x bits [B][H], weight bits [(Hq + 2 Hkv) d][H]) of one layer, seeded by (seed, stream)."""
+    x = normal_bf16(rng_for(w.seed, 40 + 2 * stream), (w.batch, w.hidden), 1.0)
+    wt = normal_bf16(rng_for(w.seed, 41 + 2 * stream), (w.out_rows, w.hidden),
+                     1.0 / math.sqrt(w.hidden))
+    return x, wt
