@@ -111,11 +111,15 @@ def measured_peak_hbm():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash():
-    """Hash of the attention kernels' code (comments and blank space removed), which ties an
-    ncu summary to the code it measured."""
+ATTN_SOURCES = ("ham_attn.cu", "ham_internal.cuh", "ham_ptx.cuh")
+FRONT_SOURCES = ("ham_front.cu", "ham_front.cuh", "ham_ptx.cuh")
+
+
+def kernel_source_hash(names=ATTN_SOURCES):
+    """Hash of a kernel's code (comments and blank space removed), which ties an ncu summary to
+    the code it measured."""
     h = hashlib.sha256()
-    for name in ("ham_attn.cu", "ham_internal.cuh"):
+    for name in names:
         with open(os.path.join(ROOT, "paper_2505_20438_gb300", "csrc", name)) as f:
             text = f.read()
         text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
@@ -124,8 +128,8 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel, workload_name):
-    """dram read+write bytes per launch of `kernel` (decode_step or decode_attn) from the
+def profiled_traffic(kernel, workload_name, sources=ATTN_SOURCES):
+    """dram read+write bytes per launch of `kernel` (decode_step, decode_attn, front) from the
     committed ncu summary, if it was taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", f"{kernel}_{workload_name}.md")
     try:
@@ -134,7 +138,7 @@ def profiled_traffic(kernel, workload_name):
         return None
     src = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", text)
     tr = re.search(r"traffic_bytes_per_launch:\s*([0-9]+)", text)
-    if not src or not tr or src.group(1) != kernel_source_hash():
+    if not src or not tr or src.group(1) != kernel_source_hash(sources):
         return None
     return int(tr.group(1))
 
@@ -213,6 +217,9 @@ EMBED_PREFIX = "embed_b"     # embed_b64, ...: the compositional embedder
 EMBED_HANDLES = 8            # rotated handles: 8 x 32 MiB of weights > 129 MB L2
 EMBED_TOK_PREFIX = "embedtok_b"  # embedtok_b64, ...: the embedder fed token ids
 EMBED_TOK_HANDLES = 16       # rotated: 16 x 8 MiB of W_o > 129 MB L2 (and 3.7 GB of tables each)
+FRONT_PREFIX = "qkv_front_b"  # qkv_front_b8, ...: the layer front (projection, RoPE, append)
+FRONT_LAYERS = 8             # rotated layers: 8 x 48 MiB of fused weights > 129 MB L2
+MICRO_PREFIX = "micro_b"     # micro_b8, ...: the micro-step decoder's attention
 
 
 def workload(name):
@@ -223,13 +230,18 @@ def workload(name):
         return wl.embed_workload(int(name[len(EMBED_PREFIX):]))
     if name.startswith(EMBED_TOK_PREFIX) and name[len(EMBED_TOK_PREFIX):].isdigit():
         return wl.embed_tokens_workload(int(name[len(EMBED_TOK_PREFIX):]))
+    if name.startswith(FRONT_PREFIX) and name[len(FRONT_PREFIX):].isdigit():
+        return wl.front_workload(int(name[len(FRONT_PREFIX):]))
+    if name.startswith(MICRO_PREFIX) and name[len(MICRO_PREFIX):].isdigit():
+        return wl.micro_workload(int(name[len(MICRO_PREFIX):]))
     if name in wl.PREFILL_WORKLOADS:
         return wl.PREFILL_WORKLOADS[name]
     if name not in wl.WORKLOADS:
         raise SystemExit(f"unknown workload {name}; choose from "
                          f"{sorted(wl.WORKLOADS) + sorted(wl.PREFILL_WORKLOADS)} or "
                          f"{STACK_PREFIX}<batch>, {EMBED_PREFIX}<batch>, "
-                         f"{EMBED_TOK_PREFIX}<batch>")
+                         f"{EMBED_TOK_PREFIX}<batch>, {FRONT_PREFIX}<batch>, "
+                         f"{MICRO_PREFIX}<batch>")
     return wl.WORKLOADS[name]
 
 
@@ -680,6 +692,10 @@ def run_reference(args, w):
     from paper_2505_20438_gb300 import workload as wl
     if isinstance(w, wl.EmbedWorkload):
         return run_reference_embed(args, w)
+    if isinstance(w, wl.FrontWorkload):
+        return run_reference_front(args, w)
+    if isinstance(w, wl.MicroWorkload):
+        return run_reference_micro(args, w)
     if isinstance(w, wl.PrefillWorkload):
         return run_reference_prefill(args, w)
     import dataclasses
@@ -1130,6 +1146,493 @@ def embed_cpu_baseline(c, seconds):
 
 
 # ---------------------------------------------------------------------------------------
+# macro-step layer front (q/k/v projection, RoPE, append)
+# ---------------------------------------------------------------------------------------
+
+FRONT_METRIC = "layer-front calls/s (q/k/v projection + RoPE + append) and achieved HBM GB/s"
+
+
+def front_bytes(w):
+    """Algorithmic bytes of one call: the fused weight once, x in, q_rot out, the new K and V
+    rows, and per sequence its counters, token count, page-table entry and slot metadata
+    (4 + 4 + 8 + 4 read, 4 + 4 + 4 + 8 written)."""
+    B, H, d = w.batch, w.hidden, w.head_dim
+    return (w.out_rows * H * 2 + B * H * 2 + B * w.n_q_heads * d * 2 +
+            B * 2 * w.n_kv_heads * d * 2 + B * 40)
+
+
+def front_cpu_sample(w, seconds, max_calls=1000):
+    """The fp64 oracle front (numpy) on whole calls for about `seconds`; returns (calls, s)."""
+    import dataclasses
+
+    import numpy as np
+
+    import oracle
+    from oracle import front as ofront
+    from paper_2505_20438_gb300 import workload as wl
+    oracle.build()
+    cw = wl.Workload("front_cache", batch=w.batch, n_q_heads=w.n_q_heads,
+                     n_kv_heads=w.n_kv_heads, head_dim=w.head_dim, page_slots=16, layers=1,
+                     seed=w.seed)
+    case = wl.make_case(cw, num_slots=np.zeros(w.batch, np.int32), extra_slots=16)
+    oc = oracle.OracleCache.from_case(case)
+    x, W = wl.front_inputs(w)
+    ntok = np.ones(w.batch, np.int32)
+    n, t0 = 0, time.perf_counter()
+    while True:
+        ofront.qkv_append(oc, x, W, ntok)
+        oc.num_slots[:] = 0
+        n += 1
+        dt = time.perf_counter() - t0
+        if dt >= seconds or n >= max_calls:
+            return n, dt
+
+
+def run_reference_front(args, w):
+    """Reference arm of the layer front: the fp64 oracle, whole calls (bounded)."""
+    steps, warm = min(max(1, args.steps), 30), min(max(3, args.warmup), 5)
+    front_cpu_sample(w, 0.0, max_calls=warm)
+    n, dt = front_cpu_sample(w, 1e9, max_calls=steps)
+    value = n / dt
+    print(json.dumps({
+        "impl": "reference", "metric": FRONT_METRIC, "value": round(value, 4),
+        "unit": "calls/s", "n_gpus": 1, "steps": n, "warmup": warm,
+        "ms_per_step": round(1e3 / value, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "batch": w.batch, "hidden": w.hidden,
+                   "n_q_heads": w.n_q_heads, "n_kv_heads": w.n_kv_heads,
+                   "head_dim": w.head_dim},
+        "cpu_baseline": {"value": round(value, 4), "unit": "calls/s", "cores": os.cpu_count(),
+                         "kind": "oracle", "sample": f"{n} whole calls of {w.name}"},
+        "e2e": {"value": round(value, 4), "unit": "calls/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def run_front(args, w):
+    """The layer front: one call projects x of w.batch sequences with one layer's fused
+    weight, rotates q and k at the new slot's position and appends the slot.  Calls rotate
+    over FRONT_LAYERS layers of one cache, each with its own weight (together far above L2),
+    64 calls per CUDA graph; each graph ends by rolling every layer back to its starting
+    length.  cuBLAS's GEMM of the same projection (no RoPE, no append) is timed the same way
+    for context."""
+    import numpy as np
+    import torch
+
+    from paper_2505_20438_gb300 import build as build_mod
+    from paper_2505_20438_gb300 import ham
+    from paper_2505_20438_gb300 import workload as wl
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1 and not torch.distributed.is_initialized():
+        torch.distributed.init_process_group("nccl")
+    build_mod.build()
+    B, H, L = w.batch, w.hidden, FRONT_LAYERS
+    per_layer = GRAPH_STEPS // L
+    start = 256                                   # slots per sequence before every graph
+    kv = ham.ham_kv_alloc(L, B, w.n_q_heads, w.n_kv_heads, w.head_dim, 16,
+                          start + per_layer + 8, page_seed=1 + rank)
+    lengths = torch.full((B,), start, dtype=torch.int32, device="cuda")
+    tokens = torch.full((B,), 2 * start, dtype=torch.int64, device="cuda")
+    for layer in range(L):
+        ham.ham_kv_set_lengths(kv, layer, lengths, tokens)
+    weights = [wl.device_normal_bf16((w.out_rows, H), 1.0 / math.sqrt(H), 1000 * w.seed + 10 * rank + j)
+               for j in range(L)]
+    x = wl.device_normal_bf16((B, H), 1.0, 1000 * w.seed + 10 * rank + 99)
+    ntok = torch.from_numpy(wl.ntok_capped_geometric(wl.rng_for(w.seed + rank, 9), (B,))).cuda()
+    q_rot = torch.empty((B, w.n_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    y = torch.empty((B, w.out_rows), dtype=torch.bfloat16, device="cuda")
+    stream = torch.cuda.Stream()
+    span = (torch.cuda.Event(enable_timing=True, external=True),
+            torch.cuda.Event(enable_timing=True, external=True))
+
+    def capture(fn, with_span):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            if with_span:
+                span[0].record()
+            for i in range(GRAPH_STEPS):
+                fn(i % L)
+            if with_span:
+                span[1].record()
+            for layer in range(L):
+                ham.ham_kv_set_lengths(kv, layer, lengths, tokens)
+        return g
+
+    def call(layer):
+        ham.ham_qkv_append(kv, layer, x, weights[layer], ntok, q_rot)
+
+    def gemm(layer):
+        torch.matmul(x, weights[layer].t(), out=y)
+
+    with torch.cuda.stream(stream):
+        for layer in range(L):                       # eager first calls
+            call(layer)
+            gemm(layer)
+        for layer in range(L):
+            ham.ham_kv_set_lengths(kv, layer, lengths, tokens)
+    stream.synchronize()
+    graph, probe = capture(call, False), capture(call, True)
+    n_graph = max(1, math.ceil(min(args.steps, 16384) / GRAPH_STEPS))
+    n_warm = max(1, math.ceil(max(args.warmup, 3) / GRAPH_STEPS))
+    steps = n_graph * GRAPH_STEPS
+    with torch.cuda.stream(stream):
+        for _ in range(n_warm):
+            graph.replay()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks, torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(n_graph - 1):
+            graph.replay()
+        probe.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed_ms = max_over_ranks(t0.elapsed_time(t1), world, "cuda")
+    if world > 1:
+        torch.distributed.barrier()
+    call_us = 1e3 * span[0].elapsed_time(span[1]) / GRAPH_STEPS
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error during the timed region")
+    # cuBLAS's GEMM of the same projection, timed the same way (context only)
+    gprobe = capture(gemm, True)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            gprobe.replay()
+    torch.cuda.synchronize()
+    gemm_us = 1e3 * span[0].elapsed_time(span[1]) / GRAPH_STEPS
+
+    nbytes = front_bytes(w)
+    peak, peak_src = measured_peak_hbm()
+    value = job_throughput(steps, world, elapsed_ms * 1e-3)
+    achieved = nbytes / (call_us * 1e-6) / 1e9
+
+    # end to end: each call copies x and ntok from pinned host memory, runs the front and
+    # copies q_rot back; one graph per layer, the host reads every call's result
+    hx, hn = x.cpu().pin_memory(), ntok.cpu().pin_memory()
+    hq = torch.empty_like(q_rot, device="cpu").pin_memory()
+    hbits = hq.view(torch.int16).numpy()
+    io = []
+    for layer in range(L):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            x.copy_(hx, non_blocking=True)
+            ntok.copy_(hn, non_blocking=True)
+            call(layer)
+            ham.ham_kv_set_lengths(kv, layer, lengths, tokens)
+            hq.copy_(q_rot, non_blocking=True)
+        io.append(g)
+    torch.cuda.synchronize()
+    n_e2e = max(GRAPH_STEPS, (args.e2e_steps // GRAPH_STEPS) * GRAPH_STEPS)
+    checksum = 0.0
+    te = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for i in range(n_e2e):
+            io[i % L].replay()
+            stream.synchronize()
+            bits = np.uint32(np.uint16(hbits.flat[0])) << np.uint32(16)
+            checksum += float(bits.view(np.float32))
+    dte = max_over_ranks(time.perf_counter() - te, world, "cuda")
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error in the end-to-end loop")
+
+    result = {
+        "metric": FRONT_METRIC, "value": round(value, 2), "unit": "calls/s", "n_gpus": world,
+        "steps": steps, "warmup": n_warm * GRAPH_STEPS,
+        "ms_per_step": round(elapsed_ms / steps, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "accum_dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": w.name, "batch": B, "hidden": H, "n_q_heads": w.n_q_heads,
+                   "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+                   "weights": "fused [W_q; W_k; W_v] bf16 N(0, 1/H), x N(0, 1)",
+                   "step": "one ham_qkv_append call: projection, RoPE of q and k, append",
+                   "l2": f"{L} layers' weights rotated ({L} x {w.out_rows * H * 2 / 2**20:.0f} "
+                         f"MiB > 129 MB L2)",
+                   "graph": f"{GRAPH_STEPS} calls per CUDA graph, then {L} counter rollbacks"},
+        "sequences_per_s": round(value * B, 1),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4),
+                     "traffic": profiled_traffic("front", w.name, FRONT_SOURCES),
+                     "kernel": "front_kernel", "avg_launch_us": round(call_us, 3),
+                     "algorithmic_bytes_per_launch": int(nbytes), "peak_source": peak_src,
+                     "duration_method": f"CUDA events around the {GRAPH_STEPS} calls of the "
+                                        f"last graph replay, / {GRAPH_STEPS}"},
+        "cublas_gemm_same_projection_us": round(gemm_us, 3),
+        "gpu_launches": n_graph * (GRAPH_STEPS + L) * world,
+        "e2e": {"value": round(job_throughput(n_e2e, world, dte), 2), "unit": "calls/s",
+                "h2d_bytes_per_step": B * H * 2 + B * 4,
+                "d2h_bytes_per_step": B * w.n_q_heads * w.head_dim * 2,
+                "steps": n_e2e, "finite": math.isfinite(checksum),
+                "path": "every call: pinned host -> device copies of x and ntok, the call, a "
+                        "counter rollback, device -> pinned host copy of q_rot, read on the "
+                        "host (one CUDA graph per layer)"},
+        "clocks": clocks.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n, dt = front_cpu_sample(w, args.cpu_seconds)
+        result["cpu_baseline"] = {"value": round(n / dt, 4), "unit": "calls/s",
+                                  "cores": os.cpu_count(), "kind": "oracle",
+                                  "sample": f"{n} whole calls of {w.name} (fp64 numpy oracle; "
+                                            f"its matrix product may use every core)"}
+    ham.ham_kv_free(kv)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+# ---------------------------------------------------------------------------------------
+# micro-step decoder attention (local cache of the context entries and the micro-tokens)
+# ---------------------------------------------------------------------------------------
+
+MICRO_METRIC = "micro-steps/s of the micro-step decoder's attention (all its layers, one launch each)"
+
+
+def micro_call_bytes(w, old):
+    """Algorithmic bytes of one ham_micro_step call when every sequence holds `old` slots: the old
+    K/V rows, q, k_new, v_new in, out, the new K/V rows out, per sequence its counters, token
+    count, page-table entry and slot metadata (20 B read, 20 B written)."""
+    B, Hq, Hkv, d = w.batch, w.n_q_heads, w.n_kv_heads, w.head_dim
+    return (B * old * Hkv * d * 4 + B * Hq * d * 2 * 2 + B * Hkv * d * 4 * 2 + B * 40)
+
+
+def micro_cpu_sample(w, seconds, max_steps=100000):
+    """The fp64 oracle on whole micro-steps (append + attention of every layer) of the workload;
+    returns (micro-steps, seconds)."""
+    import numpy as np
+
+    import oracle
+    from paper_2505_20438_gb300 import workload as wl
+    oracle.build()
+    case = wl.make_micro_case(w)
+    caches = [oracle.OracleCache.from_case(case) for _ in range(w.layers)]
+    n, t0 = 0, time.perf_counter()
+    while True:
+        for i in range(w.micro_steps):
+            for oc in caches:
+                q = case.q.copy()
+                oc.append(case.k_new, case.v_new, case.ntok_new, q_inout=q)
+                oc.decode_attn(q, n_threads=1)
+            n += 1
+        for oc in caches:
+            oc.num_slots[:] = case.num_slots
+        dt = time.perf_counter() - t0
+        if dt >= seconds or n >= max_steps:
+            return n, dt
+
+
+def run_reference_micro(args, w):
+    """Reference arm of the micro-step workload: the fp64 oracle, whole micro-steps (bounded)."""
+    steps, warm = min(max(1, args.steps), 3000), min(max(3, args.warmup), 30)
+    micro_cpu_sample(w, 0.0, max_steps=warm)
+    n, dt = micro_cpu_sample(w, 1e9, max_steps=steps)
+    value = n / dt
+    print(json.dumps({
+        "impl": "reference", "metric": MICRO_METRIC, "value": round(value, 4),
+        "unit": "micro-steps/s", "n_gpus": 1, "steps": n, "warmup": warm,
+        "ms_per_step": round(1e3 / value, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "batch": w.batch, "layers": w.layers,
+                   "context": w.context, "micro_steps": w.micro_steps},
+        "cpu_baseline": {"value": round(value, 4), "unit": "micro-steps/s", "cores": 1,
+                         "kind": "oracle", "sample": f"{n} micro-steps of {w.name}"},
+        "e2e": {"value": round(value, 4), "unit": "micro-steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def run_micro(args, w):
+    """The micro-step decoder's attention: each macro-step, every sequence's local cache holds
+    w.context entries (hidden states of middle layers of the base model); the decoder then runs
+    w.micro_steps micro-steps, each a ham_micro_step call on every one of its w.layers layers
+    (append the micro-token's key and value, attend over the local entries), and the local
+    cache is rolled back to the context for the next macro-step.  16 macro-steps per CUDA graph;
+    ham_decode_step on the same handle is timed the same way for context."""
+    import numpy as np
+    import torch
+
+    from paper_2505_20438_gb300 import build as build_mod
+    from paper_2505_20438_gb300 import ham
+    from paper_2505_20438_gb300 import workload as wl
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    if world > 1 and not torch.distributed.is_initialized():
+        torch.distributed.init_process_group("nccl")
+    build_mod.build()
+    B, L, C, M = w.batch, w.layers, w.context, w.micro_steps
+    case = wl.make_micro_case(dataclasses_replace_seed(w, rank))
+    kv = ham.ham_kv_alloc(L, B, w.n_q_heads, w.n_kv_heads, w.head_dim, 16, C + M + 1,
+                          page_seed=1 + rank)
+
+    def dev(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+    k_ctx, v_ctx = dev(case.k), dev(case.v)
+    counts = torch.from_numpy(case.num_slots).cuda()
+    tokens = torch.full((B,), C, dtype=torch.int64, device="cuda")
+    for layer in range(L):
+        ham.ham_kv_fill(kv, layer, k_ctx, v_ctx, counts)
+    # per (micro-step, layer) inputs: distinct draws, resident on the device
+    rng = wl.rng_for(w.seed + rank, 31)
+    qs = [[dev(wl.normal_bf16(rng, (B, w.n_q_heads, w.head_dim))) for _ in range(L)] for _ in range(M)]
+    ks = [[dev(wl.normal_bf16(rng, (B, w.n_kv_heads, w.head_dim))) for _ in range(L)] for _ in range(M)]
+    vs = [[dev(wl.normal_bf16(rng, (B, w.n_kv_heads, w.head_dim))) for _ in range(L)] for _ in range(M)]
+    ntok = torch.ones(B, dtype=torch.int32, device="cuda")
+    outs = [torch.empty((B, w.n_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+            for _ in range(L)]
+    stream = torch.cuda.Stream()
+    span = (torch.cuda.Event(enable_timing=True, external=True),
+            torch.cuda.Event(enable_timing=True, external=True))
+    MACRO = 16
+
+    def macro_step(fn, with_span=False):
+        for i in range(M):
+            if with_span and i == 0:
+                span[0].record()
+            for layer in range(L):
+                fn(kv, layer, qs[i][layer], ks[i][layer], vs[i][layer], None, ntok, outs[layer])
+            if with_span and i == M - 1:
+                span[1].record()
+        for layer in range(L):
+            ham.ham_kv_set_lengths(kv, layer, counts, tokens)
+
+    def capture(fn, with_span):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for r in range(MACRO):
+                macro_step(fn, with_span and r == MACRO - 1)
+        return g
+
+    with torch.cuda.stream(stream):
+        macro_step(ham.ham_micro_step)
+        macro_step(ham.ham_decode_step)
+    stream.synchronize()
+    graph, probe = capture(ham.ham_micro_step, False), capture(ham.ham_micro_step, True)
+    n_graph = max(1, math.ceil(min(args.steps, 40960) / (MACRO * M)))
+    n_warm = max(1, math.ceil(max(args.warmup, 3) / (MACRO * M)))
+    steps = n_graph * MACRO * M
+    with torch.cuda.stream(stream):
+        for _ in range(n_warm):
+            graph.replay()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clocks, torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(n_graph - 1):
+            graph.replay()
+        probe.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed_ms = max_over_ranks(t0.elapsed_time(t1), world, "cuda")
+    if world > 1:
+        torch.distributed.barrier()
+    call_us = 1e3 * span[0].elapsed_time(span[1]) / (M * L)
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error during the timed region")
+    dprobe = capture(ham.ham_decode_step, True)       # the general step, for context
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            dprobe.replay()
+    torch.cuda.synchronize()
+    decode_us = 1e3 * span[0].elapsed_time(span[1]) / (M * L)
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error in the decode-step comparison")
+
+    nbytes = sum(micro_call_bytes(w, C + i) for i in range(M)) / M   # per call, averaged
+    peak, peak_src = measured_peak_hbm()
+    value = job_throughput(steps, world, elapsed_ms * 1e-3)
+    achieved = nbytes / (call_us * 1e-6) / 1e9
+
+    # end to end: every micro-step copies its inputs for all layers (q, k, v, ntok) from pinned
+    # host memory, makes the L calls and copies the L outputs back; the host reads them.  One
+    # graph per micro-step position; the last also rolls the local caches back.
+    hq = [[x.cpu().pin_memory() for x in row] for row in qs]
+    hk = [[x.cpu().pin_memory() for x in row] for row in ks]
+    hv = [[x.cpu().pin_memory() for x in row] for row in vs]
+    hn = ntok.cpu().pin_memory()
+    hout = [torch.empty_like(o, device="cpu").pin_memory() for o in outs]
+    io = []
+    for i in range(M):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            ntok.copy_(hn, non_blocking=True)
+            for layer in range(L):
+                qs[i][layer].copy_(hq[i][layer], non_blocking=True)
+                ks[i][layer].copy_(hk[i][layer], non_blocking=True)
+                vs[i][layer].copy_(hv[i][layer], non_blocking=True)
+                ham.ham_micro_step(kv, layer, qs[i][layer], ks[i][layer], vs[i][layer], None,
+                                   ntok, outs[layer])
+                hout[layer].copy_(outs[layer], non_blocking=True)
+            if i == M - 1:
+                for layer in range(L):
+                    ham.ham_kv_set_lengths(kv, layer, counts, tokens)
+        io.append(g)
+    torch.cuda.synchronize()
+    n_e2e = max(M, (args.e2e_steps // M) * M)
+    checksum = 0.0
+    te = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for i in range(n_e2e):
+            io[i % M].replay()
+            stream.synchronize()
+            bits = np.uint32(np.uint16(hout[0].view(torch.int16).numpy().flat[0])) << np.uint32(16)
+            checksum += float(bits.view(np.float32))
+    dte = max_over_ranks(time.perf_counter() - te, world, "cuda")
+    if ham.ham_kv_status(kv) != ham.HAM_DEVERR_NONE:
+        raise RuntimeError("device error in the end-to-end loop")
+    in_bytes = L * B * (w.n_q_heads + 2 * w.n_kv_heads) * w.head_dim * 2 + B * 4
+
+    result = {
+        "metric": MICRO_METRIC, "value": round(value, 2), "unit": "micro-steps/s",
+        "n_gpus": world, "steps": steps, "warmup": n_warm * MACRO * M,
+        "ms_per_step": round(elapsed_ms / steps, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "accum_dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": w.name, "batch": B, "layers": L, "n_q_heads": w.n_q_heads,
+                   "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+                   "context_entries": C, "micro_steps_per_macro_step": M,
+                   "step": f"one micro-step: {L} ham_micro_step calls (one per layer) over "
+                           f"{C}..{C + M - 1} cached entries plus the new one",
+                   "graph": f"{MACRO} macro-steps per CUDA graph, each {M} micro-steps and a "
+                            f"rollback of the {L} local caches to the context",
+                   "l2": "local caches are L2-resident by nature (a few hundred KB)"},
+        "micro_tokens_per_s": round(value * B, 1),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": None,
+                     "kernel": "micro_step_kernel", "avg_launch_us": round(call_us, 3),
+                     "algorithmic_bytes_per_launch": int(nbytes), "peak_source": peak_src,
+                     "note": "latency-bound: a few hundred KB per launch",
+                     "duration_method": f"CUDA events around the {M * L} calls of the last "
+                                        f"macro-step of the last graph replay, / {M * L}"},
+        "decode_step_same_calls_us": round(decode_us, 3),
+        "gpu_launches": n_graph * MACRO * (M * L + L) * world,
+        "e2e": {"value": round(job_throughput(n_e2e, world, dte), 2), "unit": "micro-steps/s",
+                "h2d_bytes_per_step": in_bytes,
+                "d2h_bytes_per_step": L * B * w.n_q_heads * w.head_dim * 2,
+                "steps": n_e2e, "finite": math.isfinite(checksum),
+                "path": "every micro-step: pinned host -> device copies of each layer's q, k, v "
+                        "and the token counts, one call per layer, device -> pinned host copies of "
+                        "the outputs, read on the host (one CUDA graph per micro-step position)"},
+        "clocks": clocks.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n, dt = micro_cpu_sample(w, min(args.cpu_seconds, 5.0))
+        result["cpu_baseline"] = {"value": round(n / dt, 4), "unit": "micro-steps/s", "cores": 1,
+                                  "kind": "oracle",
+                                  "sample": f"{n} micro-steps of {w.name} (append + attention of "
+                                            f"every layer, one thread)"}
+    ham.ham_kv_free(kv)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+# ---------------------------------------------------------------------------------------
 # chunked prefill (prompt ingestion)
 # ---------------------------------------------------------------------------------------
 
@@ -1382,6 +1885,10 @@ def main():
         run_reference(args, w)
     elif isinstance(w, wl.EmbedWorkload):
         run_embed(args, w)
+    elif isinstance(w, wl.FrontWorkload):
+        run_front(args, w)
+    elif isinstance(w, wl.MicroWorkload):
+        run_micro(args, w)
     elif isinstance(w, wl.PrefillWorkload):
         run_prefill(args, w)
     elif w.layers > 1:

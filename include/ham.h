@@ -165,6 +165,55 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
                     const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
                     int32_t out_dtype, void *stream);
 
+/* The layer front of a macro-step: the q/k/v projection of the layer's input, RoPE at the new
+ * slot's position and the append, in one kernel (Sec. 3.1: one forward of the base model per
+ * macro-step stores one key/value set; Sec. 3.2: at an offset position; Sec. 4.1: the Llama
+ * base model, whose attention projects its normalised input with bias-free linear maps).
+ * For sequence b, with n = num_slots[layer][b] and p chosen as for ham_kv_append:
+ *   y = W x[b]  (fp32 accumulation on the tensor cores of the bf16 products), W = w_qkv
+ *   q_rot[b][h]   <- RoPE(y[h d .. h d + d), p)                          h < n_q_heads
+ *   K row of slot n, KV head g <- RoPE(y[(n_q_heads + g) d ..), p)
+ *   V row of slot n, KV head g <- y[(n_q_heads + n_kv_heads + g) d ..)
+ *   slot_pos = p, slot_ntok = ntok[b], num_slots += 1, num_tokens += ntok[b]
+ * The rotation takes the fp32 projection, is evaluated in fp64 and rounded once to bf16 (nearest,
+ * ties to even); values are the fp32 projection rounded once.  ham_decode_attn(kv, layer, q_rot,
+ * ...) then attends over the slots including the new one.
+ * x      device bf16 [batch][hidden], the layer's normalised input
+ * w_qkv  device bf16 [(n_q_heads + 2 n_kv_heads) head_dim][hidden], row-major ([out][in]): the
+ *        rows of W_q, then W_k, then W_v (a fused projection weight); caller-owned, not copied
+ * hidden a multiple of 256 (at most 2^20); head_dim 64 or 128
+ * pos    nullable device int32 [batch];  ntok  device int32 [batch], each >= 1
+ * q_rot  device bf16 [batch][n_q_heads][head_dim] (output)
+ * A sequence whose append cannot happen (full, ntok < 1, bad page or counter) gets no slot, sets
+ * the device error word and receives its unrotated projection in q_rot.  One launch on `stream`
+ * (programmatic dependent launch: the kernel may prefetch w_qkv into L2 before the previous
+ * kernel on the stream has finished; it reads x and the counters only after).  q_rot must not
+ * overlap x, w_qkv or the cache.  Host errors: HAM_EINVAL (NULL / unaligned / overlapping
+ * pointers, layer or hidden out of range), HAM_EUNSUPPORTED (head_dim), HAM_ECUDA.  Same
+ * serialization rule as ham_decode_attn. */
+int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, int32_t hidden,
+                   const int32_t *pos, const int32_t *ntok, void *q_rot, void *stream);
+
+/* One step of the micro-step decoder's attention (Sec. 3.3: the decoder that emits a
+ * macro-step's tokens one by one, conditioned on hidden states of several middle layers of the
+ * base model; Sec. 4.1: four layers with the base model's configuration).  Its cache is local to
+ * the macro-step: the context entries and the micro-tokens so far, a handful of slots, so the
+ * step costs the same at any sequence length (Sec. 3.7, the constant c).  Same operation and
+ * results as ham_decode_step (append of the new slot with RoPE at its position, attention over
+ * all slots including it, counters advanced; q_rot and out as there), for handles whose
+ * sequences hold at most 16 slots, in one kernel launch instead of two: one CTA per (sequence,
+ * KV head), the query is rotated in fp64 like the stored key (q_rot holds exactly the bits
+ * ham_kv_append leaves in q_inout), softmax and sums in fp32.  Typical use: a handle with
+ * layers = the decoder's layers, max_slots_per_seq = context entries + micro-tokens (<= 16),
+ * page_slots 16; each macro-step fills the context entries (ham_kv_fill or ham_prefill) and
+ * each micro-step calls this once per layer; ham_kv_set_lengths or ham_kv_reset clears the
+ * local cache for the next macro-step.
+ * Arguments, errors and serialization as for ham_decode_step; HAM_EUNSUPPORTED if the handle's
+ * max_slots_per_seq exceeds 16, n_kv_heads exceeds 8 or head_dim is not 64 or 128. */
+int ham_micro_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const void *k_new,
+                   const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
+                   int32_t out_dtype, void *stream);
+
 /* Slot and token counts of every sequence after the last layer's appends (synchronous:
  * copies on `stream`, then waits for it).  num_slots_host [batch], num_tokens_host [batch]
  * (either may be NULL).  Returns HAM_EDEVICE if the device error word is set. */

@@ -15,6 +15,8 @@
 #include <vector>
 
 #include "ham_internal.cuh"
+#include "ham_front.cuh"
+#include "ham_micro.cuh"
 #include "ham_prefill.cuh"
 
 namespace {
@@ -136,6 +138,46 @@ void note_launch(const ham_kv *kv, int32_t layer, void *stream, bool writes) {
   std::lock_guard<std::mutex> lock(g_launch_mu);
   if (g_last_launch.size() > 4096) g_last_launch.clear();  // forgetting is always safe
   g_last_launch[key] = LastLaunch{kv, layer, writes};
+}
+
+// Byte offsets of everything ham_kv_alloc carves out of the handle's metadata allocation (each
+// piece 256-byte aligned).  Recomputed from the configuration where a call needs a piece the
+// handle keeps no pointer to.
+struct MetaLayout {
+  size_t pos, ntok, pt, ns, nt, inv_freq, err, acc, ml, sr, stash, arrive, pf_seq, pf_pos;
+  size_t front;   // ham_qkv_append: one arrival counter per grid row
+  size_t total;
+};
+
+MetaLayout meta_layout(const ham_config &cfg, int32_t max_ctas, int64_t max_pages) {
+  const int group = cfg.n_q_heads / cfg.n_kv_heads;
+  const size_t slots_meta = (size_t)cfg.pool_pages * cfg.page_slots * sizeof(int32_t);
+  const size_t n_seg = (size_t)cfg.batch * cfg.n_kv_heads;
+  const size_t n_part = (size_t)max_ctas + n_seg;
+  size_t off = 0;
+  auto carve = [&](size_t bytes) {
+    size_t at = off;
+    off = round_up(off + bytes, 256);
+    return at;
+  };
+  MetaLayout m{};
+  m.pos = carve(slots_meta);
+  m.ntok = carve(slots_meta);
+  m.pt = carve((size_t)cfg.batch * (size_t)max_pages * sizeof(int32_t));
+  m.ns = carve((size_t)cfg.layers * cfg.batch * sizeof(int32_t));
+  m.nt = carve((size_t)cfg.layers * cfg.batch * sizeof(int64_t));
+  m.inv_freq = carve((size_t)(cfg.head_dim / 2) * sizeof(double));
+  m.err = carve(sizeof(int32_t));
+  m.acc = carve(n_part * group * cfg.head_dim * sizeof(float));
+  m.ml = carve(n_part * group * sizeof(float2));
+  m.sr = carve(n_seg * sizeof(int2));
+  m.stash = carve((size_t)cfg.batch * sizeof(int4));
+  m.arrive = carve(sizeof(int32_t));
+  m.pf_seq = carve((size_t)cfg.batch * sizeof(int4));
+  m.pf_pos = carve((size_t)cfg.batch * cfg.max_slots_per_seq * sizeof(int32_t));
+  m.front = carve((size_t)ham::kFrontMaxRows * sizeof(int32_t));
+  m.total = off;
+  return m;
 }
 
 }  // namespace
@@ -315,29 +357,9 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->pool_elems = cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots * cfg.head_dim;
 
   const size_t pool_bytes = (size_t)cfg.layers * 2 * (size_t)kv->pool_elems * sizeof(uint16_t);
-  const size_t slots_meta = (size_t)cfg.pool_pages * cfg.page_slots * sizeof(int32_t);
-  const size_t n_seg = (size_t)cfg.batch * cfg.n_kv_heads;
-  const size_t n_part = (size_t)kv->max_ctas + n_seg;
-  size_t off = 0;
-  auto carve = [&](size_t bytes) {
-    size_t at = off;
-    off = round_up(off + bytes, 256);
-    return at;
-  };
-  const size_t o_pos = carve(slots_meta), o_ntok = carve(slots_meta);
-  const size_t o_pt = carve((size_t)need_pages * sizeof(int32_t));
-  const size_t o_ns = carve((size_t)cfg.layers * cfg.batch * sizeof(int32_t));
-  const size_t o_nt = carve((size_t)cfg.layers * cfg.batch * sizeof(int64_t));
-  const size_t o_if = carve((size_t)(cfg.head_dim / 2) * sizeof(double));
-  const size_t o_err = carve(sizeof(int32_t));
-  const size_t o_acc = carve(n_part * group * cfg.head_dim * sizeof(float));
-  const size_t o_ml = carve(n_part * group * sizeof(float2));
-  const size_t o_sr = carve(n_seg * sizeof(int2));
-  const size_t o_stash = carve((size_t)cfg.batch * sizeof(int4));
-  const size_t o_arrive = carve(sizeof(int32_t));
-  const size_t o_pf_seq = carve((size_t)cfg.batch * sizeof(int4));
-  const size_t o_pf_pos = carve((size_t)cfg.batch * cfg.max_slots_per_seq * sizeof(int32_t));
-  kv->scratch_bytes = (int64_t)(off - o_acc);
+  const MetaLayout lay = meta_layout(cfg, kv->max_ctas, max_pages);
+  const size_t off = lay.total;
+  kv->scratch_bytes = (int64_t)(off - lay.acc);
 
   {
     const int per_sm = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, false);
@@ -362,20 +384,20 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     ham_kv_free(kv);
     return fail(HAM_ENOMEM, "allocation of the cache metadata failed");
   }
-  kv->slot_pos = reinterpret_cast<int32_t *>(kv->meta + o_pos);
-  kv->slot_ntok = reinterpret_cast<int32_t *>(kv->meta + o_ntok);
-  kv->page_table = reinterpret_cast<int32_t *>(kv->meta + o_pt);
-  kv->num_slots = reinterpret_cast<int32_t *>(kv->meta + o_ns);
-  kv->num_tokens = reinterpret_cast<int64_t *>(kv->meta + o_nt);
-  kv->inv_freq = reinterpret_cast<double *>(kv->meta + o_if);
-  kv->err = reinterpret_cast<int32_t *>(kv->meta + o_err);
-  kv->part_acc = reinterpret_cast<float *>(kv->meta + o_acc);
-  kv->part_ml = reinterpret_cast<float2 *>(kv->meta + o_ml);
-  kv->seg_range = reinterpret_cast<int2 *>(kv->meta + o_sr);
-  kv->stash = reinterpret_cast<int4 *>(kv->meta + o_stash);
-  kv->arrive = reinterpret_cast<int32_t *>(kv->meta + o_arrive);
-  kv->prefill_seq = reinterpret_cast<int4 *>(kv->meta + o_pf_seq);
-  kv->prefill_pos = reinterpret_cast<int32_t *>(kv->meta + o_pf_pos);
+  kv->slot_pos = reinterpret_cast<int32_t *>(kv->meta + lay.pos);
+  kv->slot_ntok = reinterpret_cast<int32_t *>(kv->meta + lay.ntok);
+  kv->page_table = reinterpret_cast<int32_t *>(kv->meta + lay.pt);
+  kv->num_slots = reinterpret_cast<int32_t *>(kv->meta + lay.ns);
+  kv->num_tokens = reinterpret_cast<int64_t *>(kv->meta + lay.nt);
+  kv->inv_freq = reinterpret_cast<double *>(kv->meta + lay.inv_freq);
+  kv->err = reinterpret_cast<int32_t *>(kv->meta + lay.err);
+  kv->part_acc = reinterpret_cast<float *>(kv->meta + lay.acc);
+  kv->part_ml = reinterpret_cast<float2 *>(kv->meta + lay.ml);
+  kv->seg_range = reinterpret_cast<int2 *>(kv->meta + lay.sr);
+  kv->stash = reinterpret_cast<int4 *>(kv->meta + lay.stash);
+  kv->arrive = reinterpret_cast<int32_t *>(kv->meta + lay.arrive);
+  kv->prefill_seq = reinterpret_cast<int4 *>(kv->meta + lay.pf_seq);
+  kv->prefill_pos = reinterpret_cast<int32_t *>(kv->meta + lay.pf_pos);
 
   // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits.
   e = cudaMemset(kv->pool, 0, pool_bytes);
@@ -576,6 +598,66 @@ bool overlaps(const void *a, size_t a_bytes, const void *b, size_t b_bytes) {
 }
 }  // namespace
 
+int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, int32_t hidden,
+                   const int32_t *pos, const int32_t *ntok, void *q_rot, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!x || !w_qkv || !ntok || !q_rot) return fail(HAM_EINVAL, "x, w_qkv, ntok and q_rot are required");
+  if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(q_rot))
+    return fail(HAM_EINVAL, "x, w_qkv and q_rot must be 16-byte aligned");
+  if (((uintptr_t)ntok & 3u) || ((uintptr_t)pos & 3u))
+    return fail(HAM_EINVAL, "pos/ntok must be 4-byte aligned");
+  if (hidden < ham::kFrontHiddenQuantum || hidden % ham::kFrontHiddenQuantum != 0 || hidden > (1 << 20))
+    return fail(HAM_EINVAL, "hidden %d must be a positive multiple of %d (at most 2^20)", hidden,
+                ham::kFrontHiddenQuantum);
+  const ham_config &c = kv->cfg;
+  if (c.head_dim != 64 && c.head_dim != 128)
+    return fail(HAM_EUNSUPPORTED, "layer front: head_dim %d not compiled", c.head_dim);
+  const size_t d = (size_t)c.head_dim, B = (size_t)c.batch;
+  const size_t x_bytes = B * (size_t)hidden * 2;
+  const size_t w_bytes = (size_t)(c.n_q_heads + 2 * c.n_kv_heads) * d * (size_t)hidden * 2;
+  const size_t q_bytes = B * (size_t)c.n_q_heads * d * 2;
+  const size_t pool_bytes = (size_t)c.layers * 2 * (size_t)kv->pool_elems * 2;
+  if (overlaps(q_rot, q_bytes, x, x_bytes) || overlaps(q_rot, q_bytes, w_qkv, w_bytes) ||
+      overlaps(q_rot, q_bytes, kv->pool, pool_bytes) || overlaps(x, x_bytes, kv->pool, pool_bytes) ||
+      overlaps(w_qkv, w_bytes, kv->pool, pool_bytes))
+    return fail(HAM_EINVAL, "q_rot, x, w_qkv and the cache must not overlap");
+  DeviceGuard guard(kv->device);
+  const MetaLayout lay = meta_layout(c, kv->max_ctas, kv->max_pages);
+  ham::FrontView v{};
+  v.x = static_cast<const uint16_t *>(x);
+  v.w = static_cast<const uint16_t *>(w_qkv);
+  v.q_rot = static_cast<uint16_t *>(q_rot);
+  v.k_pool = layer_pool(kv, layer, 0);
+  v.v_pool = layer_pool(kv, layer, 1);
+  v.slot_pos = kv->slot_pos;
+  v.slot_ntok = kv->slot_ntok;
+  v.page_table = kv->page_table;
+  v.num_slots = kv->num_slots + (size_t)layer * c.batch;
+  v.num_tokens = kv->num_tokens + (size_t)layer * c.batch;
+  v.inv_freq = kv->inv_freq;
+  v.rope_table = kv->rope_table;
+  v.rope_positions = kv->rope_positions;
+  v.pos = pos;
+  v.ntok = ntok;
+  v.arrive = reinterpret_cast<int32_t *>(kv->meta + lay.front);
+  v.err = kv->err;
+  v.pool_pages = c.pool_pages;
+  v.batch = c.batch;
+  v.hidden = hidden;
+  v.n_q_heads = c.n_q_heads;
+  v.n_kv_heads = c.n_kv_heads;
+  v.head_dim = c.head_dim;
+  v.page_slots = c.page_slots;
+  v.max_pages = kv->max_pages;
+  v.max_slots = c.max_slots_per_seq;
+  v.pos_mode = c.pos_mode;
+  cudaError_t e = ham::launch_front(v, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "layer front launch");
+  note_launch(kv, layer, stream, true);
+  return HAM_OK;
+}
+
 int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const void *k_new,
                     const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
                     int32_t out_dtype, void *stream) {
@@ -644,6 +726,73 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
                                           kv->tmaps[(size_t)layer * 2 + 1], v, c.head_dim,
                                           out_dtype, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "decode step launch");
+  note_launch(kv, layer, stream, true);
+  return HAM_OK;
+}
+
+int ham_micro_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const void *k_new,
+                   const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
+                   int32_t out_dtype, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!q || !k_new || !v_new || !ntok || !out)
+    return fail(HAM_EINVAL, "q, k_new, v_new, ntok and out are required");
+  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
+      (q_rot && !aligned16(q_rot)))
+    return fail(HAM_EINVAL, "q/q_rot/k/v/out must be 16-byte aligned");
+  if (((uintptr_t)ntok & 3u) || ((uintptr_t)pos & 3u))
+    return fail(HAM_EINVAL, "pos/ntok must be 4-byte aligned");
+  if (out_dtype != HAM_DTYPE_BF16 && out_dtype != HAM_DTYPE_F32)
+    return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
+  const ham_config &c = kv->cfg;
+  if (c.max_slots_per_seq > ham::kMicroMaxSlots || c.n_kv_heads > ham::kMicroMaxKvHeads ||
+      (c.head_dim != 64 && c.head_dim != 128))
+    return fail(HAM_EUNSUPPORTED, "micro step: needs max_slots_per_seq <= %d, n_kv_heads <= %d, "
+                "head_dim 64 or 128 (have %d, %d, %d)", ham::kMicroMaxSlots,
+                ham::kMicroMaxKvHeads, c.max_slots_per_seq, c.n_kv_heads, c.head_dim);
+  {  // outputs are written while q is still being read
+    const size_t n = (size_t)c.batch * c.n_q_heads * c.head_dim;
+    const size_t out_bytes = n * (out_dtype == HAM_DTYPE_F32 ? 4 : 2);
+    const size_t kv_bytes = (size_t)c.batch * c.n_kv_heads * c.head_dim * 2;
+    const size_t pool_bytes = (size_t)c.layers * 2 * (size_t)kv->pool_elems * 2;
+    if (overlaps(q, n * 2, out, out_bytes) || overlaps(q_rot, n * 2, q, n * 2) ||
+        overlaps(q_rot, n * 2, out, out_bytes) || overlaps(out, out_bytes, kv->pool, pool_bytes) ||
+        overlaps(q_rot, n * 2, kv->pool, pool_bytes) || overlaps(k_new, kv_bytes, kv->pool, pool_bytes) ||
+        overlaps(v_new, kv_bytes, kv->pool, pool_bytes))
+      return fail(HAM_EINVAL, "q, q_rot, out and the cache must not overlap");
+  }
+  DeviceGuard guard(kv->device);
+  ham::MicroView v{};
+  v.q = static_cast<const uint16_t *>(q);
+  v.q_rot = static_cast<uint16_t *>(q_rot);
+  v.k_new = static_cast<const uint16_t *>(k_new);
+  v.v_new = static_cast<const uint16_t *>(v_new);
+  v.pos = pos;
+  v.ntok = ntok;
+  v.out = out;
+  v.k_pool = layer_pool(kv, layer, 0);
+  v.v_pool = layer_pool(kv, layer, 1);
+  v.slot_pos = kv->slot_pos;
+  v.slot_ntok = kv->slot_ntok;
+  v.page_table = kv->page_table;
+  v.num_slots = kv->num_slots + (size_t)layer * c.batch;
+  v.num_tokens = kv->num_tokens + (size_t)layer * c.batch;
+  v.inv_freq = kv->inv_freq;
+  v.rope_table = kv->rope_table;
+  v.rope_positions = kv->rope_positions;
+  v.err = kv->err;
+  v.pool_pages = c.pool_pages;
+  v.batch = c.batch;
+  v.n_q_heads = c.n_q_heads;
+  v.n_kv_heads = c.n_kv_heads;
+  v.head_dim = c.head_dim;
+  v.page_slots = c.page_slots;
+  v.max_pages = kv->max_pages;
+  v.max_slots = c.max_slots_per_seq;
+  v.pos_mode = c.pos_mode;
+  v.out_f32 = out_dtype == HAM_DTYPE_F32 ? 1 : 0;
+  cudaError_t e = ham::launch_micro(v, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "micro step launch");
   note_launch(kv, layer, stream, true);
   return HAM_OK;
 }

@@ -96,6 +96,8 @@ _SIGNATURES = {
     "ham_decode_attn_noalloc": [ctypes.c_void_p, _vp],
     "ham_decode_step": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
     "ham_prefill": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _i32, _vp],
+    "ham_qkv_append": [_vp, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp],
+    "ham_micro_step": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
 }
 _lib = None
 
@@ -259,6 +261,21 @@ def ham_decode_step(kv: KV, layer, q, k_new, v_new, pos, ntok, out, q_rot=None, 
         HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16, _stream_ptr(stream)))
 
 
+def ham_micro_step(kv: KV, layer, q, k_new, v_new, pos, ntok, out, q_rot=None, stream=None):
+    """ham_decode_step for caches of at most 16 slots per sequence (the micro-step decoder's
+    local context), in one launch.  Output dtype follows `out` (bf16 or fp32)."""
+    import torch
+    B, Hq, Hkv, d = kv.batch, kv.n_q_heads, kv.n_kv_heads, kv.head_dim
+    f32 = out is not None and out.dtype == torch.float32
+    _check(lib().ham_micro_step(
+        kv, layer, _dev(q, (B, Hq, d), "bf16", "q"),
+        _dev(q_rot, (B, Hq, d), "bf16", "q_rot", nullable=True),
+        _dev(k_new, (B, Hkv, d), "bf16", "k_new"), _dev(v_new, (B, Hkv, d), "bf16", "v_new"),
+        _dev(pos, (B,), "i32", "pos", nullable=True), _dev(ntok, (B,), "i32", "ntok"),
+        _dev(out, (B, Hq, d), "f32" if f32 else "bf16", "out"),
+        HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16, _stream_ptr(stream)))
+
+
 def ham_prefill(kv: KV, layer, q, k_new, v_new, offsets, out, pos=None, ntok=None,
                 stream=None):
     """Chunked prefill of one layer: sequence b's new rows are offsets[b] .. offsets[b+1]-1 of
@@ -275,6 +292,19 @@ def ham_prefill(kv: KV, layer, q, k_new, v_new, offsets, out, pos=None, ntok=Non
         _dev(pos, (T,), "i32", "pos", nullable=True), _dev(ntok, (T,), "i32", "ntok", nullable=True),
         T, _dev(out, (T, Hq, d), "f32" if f32 else "bf16", "out"),
         HAM_DTYPE_F32 if f32 else HAM_DTYPE_BF16, _stream_ptr(stream)))
+
+
+def ham_qkv_append(kv: KV, layer, x, w_qkv, ntok, q_rot, pos=None, stream=None):
+    """Layer front of one macro-step: project x [B][H] with the fused weight
+    w_qkv [(Hq + 2 Hkv) d][H], rotate q and k at the new slot's position, append k and v, write
+    the rotated queries to q_rot [B][Hq][d]."""
+    B, Hq, Hkv, d = kv.batch, kv.n_q_heads, kv.n_kv_heads, kv.head_dim
+    H = x.shape[1] if x is not None and x.dim() == 2 else 0
+    _check(lib().ham_qkv_append(
+        kv, layer, _dev(x, (B, H), "bf16", "x"),
+        _dev(w_qkv, ((Hq + 2 * Hkv) * d, H), "bf16", "w_qkv"), H,
+        _dev(pos, (B,), "i32", "pos", nullable=True), _dev(ntok, (B,), "i32", "ntok"),
+        _dev(q_rot, (B, Hq, d), "bf16", "q_rot"), _stream_ptr(stream)))
 
 
 def ham_slot_lengths(kv: KV, stream=None):

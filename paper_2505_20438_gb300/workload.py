@@ -377,3 +377,39 @@ def front_inputs(w: FrontWorkload, stream: int = 0):
     wt = normal_bf16(rng_for(w.seed, 41 + 2 * stream), (w.out_rows, w.hidden),
                      1.0 / math.sqrt(w.hidden))
     return x, wt
+
+
+# ---------------------------------------------------------------------------------------
+# Micro-step decoder attention (Sec. 3.3, Sec. 4.1): four layers with the base model's
+# configuration (Llama-3.2-1B: 32 query / 8 KV heads of 64) over a local cache holding
+# `context` entries (hidden states of middle layers of the base model, already projected) and
+# the micro-tokens of the current macro-step; a macro-step emits at most 4 tokens, the first
+# from the base model itself (Sec. 3.4), so the decoder runs at most 3 micro-steps.
+# ---------------------------------------------------------------------------------------
+@dataclasses.dataclass(frozen=True)
+class MicroWorkload:
+    name: str
+    batch: int
+    layers: int = 4
+    n_q_heads: int = 32
+    n_kv_heads: int = 8
+    head_dim: int = 64
+    context: int = 4
+    micro_steps: int = MAX_TOKENS_PER_SLOT - 1
+    seed: int = 5
+
+
+def micro_workload(batch: int, **kw) -> MicroWorkload:
+    return MicroWorkload(f"micro_b{batch}", batch=batch, **kw)
+
+
+def make_micro_case(w: MicroWorkload) -> HostCase:
+    """One layer's local cache (w.context entries per sequence, one 16-slot page each) and the
+    inputs of one micro-step, values N(0, 1)."""
+    base = Workload(w.name, batch=w.batch, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
+                    head_dim=w.head_dim, page_slots=16, layers=1, value_scale=1.0, seed=w.seed,
+                    pool_factor=1.0, scatter_pages=True)
+    case = make_case(base, num_slots=np.full(w.batch, w.context, np.int32),
+                     extra_slots=w.micro_steps + 1)
+    case.ntok_new[:] = 1
+    return case
