@@ -10,9 +10,11 @@
 // built for caches of thousands of slots; here one kernel does everything:
 //  - one CTA per (sequence, KV head); the CTAs of a sequence form a thread-block cluster, whose
 //    barrier orders every CTA's read of the slot counter before rank 0 advances it;
-//  - the old entries, the new key (rotated in fp64 from the handle's cos/sin table and rounded
-//    once to bf16, the bits ham_kv_append stores) and the rotated query heads of the group are
-//    staged in shared memory;
+//  - two dependent round trips to memory: the counters and the page entry together with the
+//    query heads and the new key and value, then the cos/sin at the position together with the
+//    old entries; the new key (rotated in fp64 from the handle's cos/sin table and rounded once
+//    to bf16, the bits ham_kv_append stores) and the rotated query heads of the group are kept
+//    in shared memory;
 //  - a warp per query head: each lane holds head_dim / 32 elements, a dot product is a
 //    5-step shuffle reduction, the softmax (fp32, exact exp) and the weighted sum of values
 //    stay in registers.
@@ -53,13 +55,18 @@ __global__ void __launch_bounds__(kMicroThreads) micro_step_kernel(MicroView v) 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   __shared__ __align__(16) uint16_t ks[kMicroMaxSlots][D];
   __shared__ __align__(16) uint16_t vs[kMicroMaxSlots][D];
-  __shared__ __align__(16) uint16_t qs[8][D];
+  __shared__ __align__(16) uint16_t qs[8][D];     // the group's query heads (turned in place)
+  __shared__ __align__(16) uint16_t kn[D], vn[D]; // the new key (unrotated) and value
   __shared__ double cos_t[HALF], sin_t[HALF];
   __shared__ int32_t s_ok, s_n, s_old, s_ntok;
   __shared__ int64_t s_pos, s_page;
 
   grid_dependency_wait();
   grid_launch_dependents();
+  // First round trip: the counters and the page entry, and (not depending on them) the query
+  // heads and the new key and value.
+  const uint16_t *q_src = v.q + ((int64_t)b * v.n_q_heads + (int64_t)g * G) * D;
+  const int64_t kv_off = ((int64_t)b * Hkv + g) * D;
   if (threadIdx.x == 0) {
     const int32_t n = v.num_slots[b];
     const int32_t t = v.ntok[b];
@@ -81,7 +88,17 @@ __global__ void __launch_bounds__(kMicroThreads) micro_step_kernel(MicroView v) 
     s_page = page;
     s_pos = v.pos ? (int64_t)v.pos[b] : (v.pos_mode == HAM_POS_SLOT ? (int64_t)n : v.num_tokens[b]);
   }
+  for (int idx = threadIdx.x; idx < (G + 2) * VEC; idx += kMicroThreads) {
+    const int r = idx / VEC, e = idx % VEC;
+    if (r < G)
+      reinterpret_cast<uint4 *>(qs[r])[e] = reinterpret_cast<const uint4 *>(q_src + r * D)[e];
+    else if (r == G)
+      reinterpret_cast<uint4 *>(kn)[e] = reinterpret_cast<const uint4 *>(v.k_new + kv_off)[e];
+    else
+      reinterpret_cast<uint4 *>(vn)[e] = reinterpret_cast<const uint4 *>(v.v_new + kv_off)[e];
+  }
   __syncthreads();
+  // Second round trip: cos/sin at the position, the old entries of the page.
   const bool ok = s_ok != 0;
   const int old = s_old;
   const int64_t p = s_pos;
@@ -97,30 +114,22 @@ __global__ void __launch_bounds__(kMicroThreads) micro_step_kernel(MicroView v) 
     cos_t[threadIdx.x] = c;
     sin_t[threadIdx.x] = s;
   }
-  // old entries (16-byte pieces), unrotated query heads
   const int64_t row0 = (s_page * Hkv + g) * v.page_slots;    // row of slot 0, this KV head
   for (int idx = threadIdx.x; idx < old * VEC; idx += kMicroThreads) {
     const int j = idx / VEC, e = idx % VEC;
     reinterpret_cast<uint4 *>(ks[j])[e] = reinterpret_cast<const uint4 *>(v.k_pool + (row0 + j) * D)[e];
     reinterpret_cast<uint4 *>(vs[j])[e] = reinterpret_cast<const uint4 *>(v.v_pool + (row0 + j) * D)[e];
   }
-  const uint16_t *q_src = v.q + ((int64_t)b * v.n_q_heads + (int64_t)g * G) * D;
-  if (!ok) {
-    for (int idx = threadIdx.x; idx < G * VEC; idx += kMicroThreads)
-      reinterpret_cast<uint4 *>(qs[idx / VEC])[idx % VEC] = reinterpret_cast<const uint4 *>(q_src)[idx];
-  }
   __syncthreads();   // cos/sin ready
-  if (ok) {
+  if (ok) {   // turn the queries in place and the new key into its slot; copy the new value
     const int n = s_n;
-    const uint16_t *k_src = v.k_new + ((int64_t)b * Hkv + g) * D;
     for (int idx = threadIdx.x; idx < (G + 1) * HALF; idx += kMicroThreads) {
       const int r = idx / HALF, i = idx % HALF;
-      if (r < G) turn_pair(q_src + r * D, qs[r], i, HALF, cos_t[i], sin_t[i]);
-      else turn_pair(k_src, ks[n], i, HALF, cos_t[i], sin_t[i]);
+      if (r < G) turn_pair(qs[r], qs[r], i, HALF, cos_t[i], sin_t[i]);
+      else turn_pair(kn, ks[n], i, HALF, cos_t[i], sin_t[i]);
     }
-    const uint16_t *v_src = v.v_new + ((int64_t)b * Hkv + g) * D;
     for (int e = threadIdx.x; e < VEC; e += kMicroThreads)
-      reinterpret_cast<uint4 *>(vs[n])[e] = reinterpret_cast<const uint4 *>(v_src)[e];
+      reinterpret_cast<uint4 *>(vs[n])[e] = reinterpret_cast<const uint4 *>(vn)[e];
   }
   __syncthreads();
   if (ok) {   // the new slot's rows and the rotated queries
