@@ -1191,7 +1191,7 @@ def front_cpu_sample(w, seconds, max_calls=1000):
 def run_reference_front(args, w):
     """Reference arm of the layer front: the fp64 oracle, whole calls (bounded)."""
     steps, warm = min(max(1, args.steps), 30), min(max(3, args.warmup), 5)
-    front_cpu_sample(w, 0.0, max_calls=warm)
+    warm, _ = front_cpu_sample(w, 1e9, max_calls=warm)
     n, dt = front_cpu_sample(w, 1e9, max_calls=steps)
     value = n / dt
     print(json.dumps({
@@ -1426,7 +1426,7 @@ def micro_cpu_sample(w, seconds, max_steps=100000):
 def run_reference_micro(args, w):
     """Reference arm of the micro-step workload: the fp64 oracle, whole micro-steps (bounded)."""
     steps, warm = min(max(1, args.steps), 3000), min(max(3, args.warmup), 30)
-    micro_cpu_sample(w, 0.0, max_steps=warm)
+    warm, _ = micro_cpu_sample(w, 1e9, max_steps=warm)
     n, dt = micro_cpu_sample(w, 1e9, max_steps=steps)
     value = n / dt
     print(json.dumps({
