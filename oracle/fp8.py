@@ -9,7 +9,7 @@ instead of 16 roughly halves the bytes a step reads.  The paper itself keeps the
 precision; this is a storage format of this library, specified here so that the CUDA path can be
 checked against it bit for bit.
 
-Format (readings Q1-Q4, listed in the design notes):
+Format (readings Q1-Q4 of the paper's silence on any 8-bit cache format, taken here):
   Q1  e4m3 codes (1 sign bit, 4 exponent bits with bias 7, 3 mantissa bits; no infinities;
       S.1111.111 is NaN; largest finite 448 = 1.75 * 2^8; subnormals are multiples of 2^-9);
   Q2  one scale per stored row (one slot of one KV head), a power of two 2^e, e an int8: a row is
@@ -18,7 +18,11 @@ Format (readings Q1-Q4, listed in the design notes):
   Q3  e is chosen from the row's largest magnitude a = m 2^E (0.5 <= m < 1) as e = E - 8, so
       that a 2^-e lies in [128, 256): below 448, with every element scaled exactly (a power of
       two) and rounded once, to nearest with ties to even, onto the e4m3 grid; a row of zeros
-      gets e = 0 and zero codes;
+      gets e = 0 and zero codes.  e is then clamped to [-124, 119] so that every decoded value
+      is a finite bf16 value: the finest step of the e4m3 grid is 2^-9 and that of bf16 is 2^-133
+      (its smallest subnormal), hence e >= -124; a row maximum just below 2^128 (E = 128) would
+      round up to 256 * 2^120 = 2^128, past the largest bf16 value, hence e <= 119 (such a row's
+      largest elements then saturate at 448 * 2^119).  Rows must be finite;
   Q4  the key is rotated first (the bf16 row ham_kv_append would store), then encoded; the value
       row is encoded as given.  A decoded element code * 2^e has at most 4 significant bits and
       is therefore exact in bf16, so attention over an FP8 pool is attention over those exact
@@ -67,14 +71,17 @@ def e4m3_encode(x) -> np.ndarray:
     return code.astype(np.uint8)
 
 
+E_MIN, E_MAX = -124, 119   # Q3: the decoded values code * 2^e stay finite and exact in bf16
+
+
 def row_exponent(values) -> int:
-    """Scale exponent e of one row (Q3): e = E - 8 for the largest magnitude m 2^E, 0 if all
-    zero."""
+    """Scale exponent e of one row (Q3): e = E - 8 for the largest magnitude m 2^E, clamped to
+    [E_MIN, E_MAX]; 0 if all zero."""
     a = float(np.max(np.abs(np.asarray(values, dtype=np.float64)))) if np.size(values) else 0.0
     if a == 0.0:
         return 0
     _, E = np.frexp(a)
-    return int(E) - 8
+    return int(min(max(int(E) - 8, E_MIN), E_MAX))
 
 
 def encode_row(values):

@@ -137,3 +137,35 @@ def test_fp8_cache_attention_is_attention_over_decoded_rows():
             assert np.allclose(got[b, h], (p / p.sum()) @ vv, atol=1e-12)
     err = np.abs(got - exact)
     assert err.max() < 0.1 and err.mean() < 0.02
+
+
+@pytest.mark.parametrize("top", [2.0 ** -121, 2.0 ** -125, 2.0 ** -133, 2.0 ** -117,
+                                 2.0 ** -116, 255.0 * 2.0 ** 120, 2.0 ** 127, 1.5 * 2.0 ** 126])
+def test_row_scale_at_the_ends_of_the_bf16_range(top):
+    """Rows whose largest magnitude sits near either end of bf16's range: the exponent stays in
+    [-124, 119], every decoded value is finite and exactly representable in bf16 (checked through
+    the C oracle's rounding, not this module's), and the largest element keeps its sign and
+    lands within the e4m3 relative error of the input (or saturates at the top end)."""
+    import oracle
+    fp8 = _fp8()
+    bf16_min_sub = 2.0 ** -133
+    # a row of bf16 values: the top value, a few smaller ones, both signs, a zero
+    row = np.array([top, -top / 2, top / 3, -top / 7, 0.0, top / 64, -top / 200, top / 1000])
+    row = oracle.bf16_to_f64(oracle.f64_to_bf16(row))          # exact bf16 values
+    assert np.abs(row).max() == top
+    codes, e = fp8.encode_row(row)
+    assert -124 <= e <= 119
+    back = fp8.decode_row(codes, e)
+    assert np.all(np.isfinite(back))
+    assert np.array_equal(oracle.bf16_to_f64(oracle.f64_to_bf16(back)), back)  # exact bf16
+    assert np.all(np.abs(back[back != 0]) >= bf16_min_sub)
+    assert np.sign(back[0]) == 1.0
+    _, E = np.frexp(top)
+    assert e == min(max(int(E) - 8, -124), 119)        # the defining rule E - 8, clamped
+    if int(E) - 8 <= 119:
+        assert abs(back[0] - top) <= top * 2.0 ** -4
+    else:                            # clamped at the top: the scaled maximum may saturate at 448
+        assert back[0] <= 448.0 * 2.0 ** 119
+        assert abs(back[0] - min(top, 448.0 * 2.0 ** 119)) <= top * 2.0 ** -4
+    if top == 255.0 * 2.0 ** 120:
+        assert back[0] == 448.0 * 2.0 ** 119           # 510 after scaling: saturated
