@@ -341,8 +341,9 @@ int ham_split_plan(int32_t batch, int32_t n_kv_heads, const int32_t *num_slots_h
  * from an 8 MiB array compiled into libham.so, which every GPU that loads the library keeps
  * until the process exits.  The call itself allocates nothing (no cudaMalloc, cudaFree or
  * allocating library routine).
- *  - The first call on each device looks up that array's device address and sets kernel
- *    attributes; make that first call before any stream capture on the device.
+ *  - The first call on each device looks up that array's device address and sets the kernel
+ *    attributes of every output type and head_dim it supports (not only the first call's);
+ *    make that first call before any stream capture on the device.
  *  - All calls share the one array: calls that overlap on the GPU (other streams, other
  *    threads) race on it and give wrong results.  Serialize them.
  *  - A configuration whose scratch would exceed the array ((ctas + batch*n_kv_heads) *

@@ -1146,15 +1146,24 @@ cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, con
                                     : dispatch<__nv_bfloat16, true>(head_dim, go);
 }
 
-int attention_ctas_per_sm(int head_dim, int group, int batch, bool step) {
+int attention_ctas_per_sm(int head_dim, int group, int batch, bool step, int out_dtype) {
   int n = 0;
   auto q = [&](auto inst) {
     n = decltype(inst)::ctas_per_sm(group, batch);
     return cudaSuccess;
   };
-  if (step) dispatch<__nv_bfloat16, true>(head_dim, q);
-  else dispatch<__nv_bfloat16, false>(head_dim, q);
+  const bool f32 = out_dtype == HAM_DTYPE_F32;
+  if (step) f32 ? dispatch<float, true>(head_dim, q) : dispatch<__nv_bfloat16, true>(head_dim, q);
+  else f32 ? dispatch<float, false>(head_dim, q) : dispatch<__nv_bfloat16, false>(head_dim, q);
   return n;
+}
+
+cudaError_t configure_attention_instances() {
+  cudaError_t e = Instance<128, __nv_bfloat16, false>::configure();
+  if (e == cudaSuccess) e = Instance<64, __nv_bfloat16, false>::configure();
+  if (e == cudaSuccess) e = Instance<128, float, false>::configure();
+  if (e == cudaSuccess) e = Instance<64, float, false>::configure();
+  return e;
 }
 
 }  // namespace ham

@@ -140,8 +140,14 @@ cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const
 // Fused decode step: attention with the append of v.step folded in, then combine + counters.
 cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
                                int head_dim, int out_dtype, cudaStream_t stream);
-// CTAs of one SM for the attention kernel of this shape (0 if the shape is not compiled).
-int attention_ctas_per_sm(int head_dim, int group, int batch, bool step);
+// CTAs of one SM for the attention kernel of this shape and output type (0 if the shape is not
+// compiled).
+int attention_ctas_per_sm(int head_dim, int group, int batch, bool step,
+                          int out_dtype = HAM_DTYPE_BF16);
+// Set the shared-memory attribute of every compiled attention instance of the plain (non-step)
+// kernel, for the current device: bf16 and fp32 output at head_dim 64 and 128.  Later launches
+// of those instances then make no attribute call.
+cudaError_t configure_attention_instances();
 bool attention_supported(int head_dim, int group);
 // TMA map of one pool [pool_pages][n_kv_heads][page_slots][head_dim] bf16 viewed as
 // {64 elements, head_dim / 64, rows} with a box of {64, head_dim / 64, 16 rows} (half_box:

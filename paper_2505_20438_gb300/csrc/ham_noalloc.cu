@@ -3,8 +3,9 @@
 // owned by a ham_kv handle, and the caller passes every input and output.
 //
 // The array's name in host code is only a host-side stand-in: kernels must be given the
-// device address, which cudaGetSymbolAddress returns per device.  That lookup (and the
-// kernel attribute set-up) happens on the first call on each device.
+// device address, which cudaGetSymbolAddress returns per device.  That lookup, and the
+// shared-memory attribute of all four attention instances (bf16 / fp32 output, head_dim 64 /
+// 128), happen on the first call on each device, whatever that call's dtype and head_dim.
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -70,6 +71,12 @@ int ham_decode_attn_noalloc(const ham_attn_args *a, void *stream) {
       int sms = 0;
       if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return noalloc_fail(HAM_ECUDA, "cannot read the SM count");
+      // every attention instance this entry point can launch (bf16 / fp32 output, head_dim 64
+      // / 128) gets its attribute now, so that no later call makes one, inside a capture or not
+      if (ham::configure_attention_instances() != cudaSuccess) {
+        cudaGetLastError();
+        return noalloc_fail(HAM_ECUDA, "cannot set the attention kernels' shared-memory size");
+      }
       s.scratch = p;
       s.num_sms = sms;
       s.done = true;
@@ -79,7 +86,8 @@ int ham_decode_attn_noalloc(const ham_attn_args *a, void *stream) {
 
   int ctas = a->ctas;
   if (ctas == 0) {
-    const int per_sm = ham::attention_ctas_per_sm(a->head_dim, group, a->batch, false);
+    const int per_sm =
+        ham::attention_ctas_per_sm(a->head_dim, group, a->batch, false, a->out_dtype);
     if (per_sm <= 0) return noalloc_fail(HAM_ECUDA, "attention kernel cannot be resident");
     ctas = ham::default_attention_ctas(setup.num_sms, per_sm);
   }
