@@ -9,7 +9,7 @@ query reads keys and values computed from the token embeddings, to which a learn
 embedding of the token's place inside the patch is added; a linear layer follows.  A list of
 one token skips the module: the hidden state is that token's embedding.
 
-Readings where the paper leaves details open (each is listed in the design notes):
+Readings where the paper leaves details open, taken here:
   E1  the query comes from the mean of the raw token embeddings x_i;
   E2  keys and values come from u_i = x_i + P[i], P[i] the learned embedding of place i;
   E3  multi-head attention of the base model's head layout (H = n_heads * head_dim), scale

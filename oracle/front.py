@@ -19,7 +19,7 @@ stores the key and value as the sequence's new slot.  For sequence b:
                             slot_pos = p, slot_ntok = ntok[b];  counters advance
     q_rot[b, h] = bf16(RoPE(q_h))
 
-Readings where the paper leaves details open (each is listed in the design notes):
+Readings where the paper leaves details open, taken here:
   F1  the projections are the base model's bias-free q/k/v linear maps, one fused weight with
       the rows of W_q, then W_k, then W_v;
   F2  the rotation acts on the exact projection, and each stored value is rounded once to
