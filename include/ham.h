@@ -318,6 +318,15 @@ int ham_kv_reset(ham_kv *kv, void *stream);
  * SM)).  Range 1 .. 8 x SMs.  Any value gives the same result up to fp32 summation order. */
 int ham_kv_set_attn_ctas(ham_kv *kv, int32_t ctas);
 
+/* Limit, in nanoseconds, of the data waits of this handle's attention and prefill kernels: the
+ * waits of the shared-memory ring for copies to land and for stages to be freed.  0 restores the
+ * default, 2 s (the largest value accepted).  A wait that runs out records HAM_DEVERR_TIMEOUT
+ * (read by ham_kv_status), stops its CTA's work and leaves that launch's output undefined; the
+ * copies a CTA already issued are still waited for, with the default bound, before it exits.  This
+ * is a testing aid for the failure path (a limit of a few nanoseconds makes the waits run out on
+ * an otherwise healthy GPU); production callers leave the default. */
+int ham_kv_set_wait_limit_ns(ham_kv *kv, uint64_t ns);
+
 /* Host evaluation of the split plan the attention kernel uses (no GPU needed).  Chunks are
  * 16 slots; the chunks of (sequence b, KV head g), b-major, are numbered contiguously (W in
  * all).  The first min(ctas, ceil(W / 4)) CTAs get equal non-empty ranges (a small problem

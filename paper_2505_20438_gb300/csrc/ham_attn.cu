@@ -320,6 +320,8 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
   __syncthreads();
   if (!active_cta) return;
 
+  // ring and data waits: the launch's limit; the final drain of in-flight copies keeps 2 s
+  const uint64_t wait_lim = data_wait_limit(v.wait_ns);
   // ---------------------------------------------------------------- producer warp
   if (warp == 1) {
     const uint64_t pol = policy_evict_first();
@@ -339,7 +341,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
         if (lane == 0) {
           const int stage = it % S::kStages;
           const uint32_t ph = (uint32_t)(it / S::kStages) & 1u;
-          if (!issued && !thread_wait(&empty[stage], ph ^ 1u, flags, true)) {
+          if (!issued && !thread_wait(&empty[stage], ph ^ 1u, flags, true, wait_lim)) {
             record_error(v.err, HAM_DEVERR_TIMEOUT);
             flags[0] = 1;
             failed = 1;
@@ -420,7 +422,7 @@ __global__ void __launch_bounds__(Shape<D>::kThreads)
 
   for (int it = 0; it < nchunks; ++it) {
     const int stage = it % S::kStages;
-    if (!warp_wait(&full[stage], (uint32_t)(it / S::kStages) & 1u, flags)) {
+    if (!warp_wait(&full[stage], (uint32_t)(it / S::kStages) & 1u, flags, wait_lim)) {
       if (lane == 0) {
         record_error(v.err, HAM_DEVERR_TIMEOUT);
         flags[0] = 1;

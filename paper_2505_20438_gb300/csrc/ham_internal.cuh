@@ -98,6 +98,7 @@ struct AttnView {
   // pools, so the kernel may read them before its programmatic-dependency wait (the host
   // decides; 0 is always correct)
   int32_t early;
+  uint64_t wait_ns;            // limit of the ring and data waits (0: the default 2 s)
   StepArgs step;               // used by launch_decode_step only
 };
 
@@ -177,6 +178,7 @@ struct ham_kv {
   int num_sms = 0;
   int32_t max_pages = 0;
   int32_t attn_ctas = 0;        // 0: default
+  uint64_t wait_ns = 0;         // attention / prefill data-wait limit (0: the default 2 s)
   int32_t default_ctas = 0;     // SMs x resident attention CTAs per SM (set at allocation)
   int32_t default_step_ctas = 0;  // same for the fused decode step
   int32_t max_ctas = 0;         // scratch is sized for this many CTAs

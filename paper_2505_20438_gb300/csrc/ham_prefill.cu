@@ -370,6 +370,8 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
   }
   __syncthreads();
 
+  // ring and data waits: the launch's limit; the final drain of in-flight copies keeps 2 s
+  const uint64_t wait_lim = data_wait_limit(v.wait_ns);
   if (warp == S::kWarps) {
     // Producer: one lane streams the tiles.  A chunk past the last attended slot or on a page
     // outside the pool is not copied (its bit stays clear and the consumers mask it).
@@ -379,7 +381,8 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
     for (int t = 0; t < ntiles; ++t) {
       const int s = t % S::kStages;
       if (t >= S::kStages &&
-          !thread_wait(&empty[s], (uint32_t)((t / S::kStages) - 1) & 1u, abort_flag, true)) {
+          !thread_wait(&empty[s], (uint32_t)((t / S::kStages) - 1) & 1u, abort_flag, true,
+                       wait_lim)) {
         if (!*abort_flag) {
           record_error(v.err, HAM_DEVERR_TIMEOUT);
           *abort_flag = 1;
@@ -452,7 +455,7 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
   bool ok = true;
   for (int t = 0; t < ntiles; ++t) {
     const int s = t % S::kStages;
-    if (!warp_wait(&full[s], (uint32_t)(t / S::kStages) & 1u, abort_flag)) {
+    if (!warp_wait(&full[s], (uint32_t)(t / S::kStages) & 1u, abort_flag, wait_lim)) {
       if (lane == 0 && !*abort_flag) {
         record_error(v.err, HAM_DEVERR_TIMEOUT);
         *abort_flag = 1;

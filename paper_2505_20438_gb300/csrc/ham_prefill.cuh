@@ -28,6 +28,7 @@ struct PrefillView {
   int64_t pool_pages;
   int32_t batch, rows, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots;
   int32_t pos_mode;
+  uint64_t wait_ns;            // limit of the attention's data waits (0: the default 2 s)
 };
 cudaError_t launch_prefill(const CUtensorMap &tk, const CUtensorMap &tv, const PrefillView &v,
                            int out_dtype, cudaStream_t stream);

@@ -57,6 +57,17 @@ __device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// Non-blocking test of an mbarrier phase (never suspends the thread, unlike try_wait).
+__device__ __forceinline__ bool mbar_poll(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ uint64_t policy_evict_last() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
@@ -133,21 +144,43 @@ __device__ __forceinline__ float ex2(float x) {
 
 // One thread waits on an mbarrier phase, bounded.  honor_abort: give up early once another
 // warp has aborted (not used while draining in-flight copies).
+// limit_ns: how long to wait (the default, 2 s, unless a caller shortened its data waits).  A
+// shortened limit polls without suspending (try_wait may sleep for longer than the limit), so
+// that it is honoured to within a poll.
 __device__ bool thread_wait(uint64_t *bar, uint32_t parity, volatile int *abort_flag,
-                            bool honor_abort) {
+                            bool honor_abort, uint64_t limit_ns = kWaitLimitNs) {
+  if (limit_ns < kWaitLimitNs) {
+    const uint64_t t0 = global_timer_ns();
+    while (!mbar_poll(bar, parity)) {
+      if (honor_abort && *abort_flag) return false;
+      if (global_timer_ns() - t0 > limit_ns) return false;
+    }
+    return true;
+  }
   if (mbar_test(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t n = 1;; ++n) {
     if (mbar_test(bar, parity)) return true;
     if ((n & 15u) == 0) {
       if (honor_abort && *abort_flag) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) return false;
+      if (global_timer_ns() - t0 > limit_ns) return false;
     }
   }
 }
 
 // The whole warp waits on an mbarrier phase, bounded; the result is warp-uniform.
-__device__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort_flag) {
+__device__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort_flag,
+                          uint64_t limit_ns = kWaitLimitNs) {
+  if (limit_ns < kWaitLimitNs) {  // shortened: poll without suspending, lane 0 keeps the time
+    const uint64_t t0 = global_timer_ns();
+    for (;;) {
+      if (__all_sync(kFull, mbar_poll(bar, parity))) return true;
+      int stop = 0;
+      if ((threadIdx.x & 31) == 0)
+        stop = (*abort_flag != 0) || (global_timer_ns() - t0 > limit_ns);
+      if (__shfl_sync(kFull, stop, 0)) return false;
+    }
+  }
   if (__all_sync(kFull, mbar_test(bar, parity))) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t n = 1;; ++n) {
@@ -155,7 +188,7 @@ __device__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort_fl
     if ((n & 15u) == 0) {
       int stop = 0;
       if ((threadIdx.x & 31) == 0)
-        stop = (*abort_flag != 0) || (global_timer_ns() - t0 > kWaitLimitNs);
+        stop = (*abort_flag != 0) || (global_timer_ns() - t0 > limit_ns);
       if (__shfl_sync(kFull, stop, 0)) return false;
     }
   }
@@ -165,6 +198,11 @@ __device__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort_fl
 // TMA copy with the 128-byte swizzle: rows are split into 128-byte lines (line = row *
 // lines_per_row + c / 8) and the piece index inside a line is XORed with line % 8.  The tile
 // must start on a 1024-byte boundary.
+// Data-wait limit of a launch: the caller's (nonzero) value, else the default.
+__device__ __forceinline__ uint64_t data_wait_limit(uint64_t wait_ns) {
+  return wait_ns ? wait_ns : kWaitLimitNs;
+}
+
 __device__ __forceinline__ uint32_t swizzle128_offset(int row, int c, int lines_per_row) {
   const int line = row * lines_per_row + (c >> 3);
   return (uint32_t)(line * 128 + (((c & 7) ^ (line & 7)) << 4));

@@ -508,6 +508,16 @@ int ham_kv_set_attn_ctas(ham_kv *kv, int32_t ctas) {
   return HAM_OK;
 }
 
+int ham_kv_set_wait_limit_ns(ham_kv *kv, uint64_t ns) {
+  if (!kv) return fail(HAM_EINVAL, "null handle");
+  constexpr uint64_t kDefaultNs = 2000000000ull;  // the kernels' default bound, 2 s
+  if (ns > kDefaultNs)
+    return fail(HAM_EINVAL, "limit %llu ns above the default %llu", (unsigned long long)ns,
+                (unsigned long long)kDefaultNs);
+  kv->wait_ns = ns;
+  return HAM_OK;
+}
+
 int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
                   const void *v_new, const int32_t *pos, const int32_t *ntok, void *stream) {
   int rc = check_layer(kv, layer);
@@ -582,6 +592,7 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
   v.max_slots = kv->cfg.max_slots_per_seq;
   v.ctas = ctas;
   v.sms = kv->num_sms;
+  v.wait_ns = kv->wait_ns;
   v.early = may_start_early(kv, layer, stream) ? 1 : 0;
   cudaError_t e = ham::launch_attention(kv->tmaps[(size_t)layer * 2], kv->tmaps[(size_t)layer * 2 + 1],
                                         v, kv->cfg.head_dim, out_dtype,
@@ -702,6 +713,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
   v.max_slots = c.max_slots_per_seq;
   v.ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->default_step_ctas;
   v.sms = kv->num_sms;
+  v.wait_ns = kv->wait_ns;
   ham::StepArgs &st = v.step;
   st.k_new = static_cast<const uint16_t *>(k_new);
   st.v_new = static_cast<const uint16_t *>(v_new);
@@ -851,6 +863,7 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
   v.pos = pos;
   v.ntok = ntok;
   v.out = out;
+  v.wait_ns = kv->wait_ns;
   v.seq_info = kv->prefill_seq;
   v.row_pos = kv->prefill_pos;
   v.err = kv->err;

@@ -92,6 +92,7 @@ _SIGNATURES = {
     "ham_kv_reset": [_vp, _vp],
     "ham_kv_set_lengths": [_vp, _i32, _vp, _vp, _vp],
     "ham_kv_set_attn_ctas": [_vp, _i32],
+    "ham_kv_set_wait_limit_ns": [_vp, ctypes.c_uint64],
     "ham_split_plan": [_i32, _i32, _vp, _i32, _vp, _vp, _vp],
     "ham_decode_attn_noalloc": [ctypes.c_void_p, _vp],
     "ham_decode_step": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
@@ -382,6 +383,12 @@ def ham_kv_reset(kv: KV, stream=None):
 def ham_kv_set_attn_ctas(kv: KV, ctas: int):
     _check(lib().ham_kv_set_attn_ctas(kv, int(ctas)))
     kv.info = ham_kv_get_info(kv)
+
+
+def ham_kv_set_wait_limit_ns(kv: KV, ns: int):
+    """Limit of the attention and prefill kernels' data waits (0: the default 2 s); a testing aid
+    for the failure path."""
+    _check(lib().ham_kv_set_wait_limit_ns(kv, int(ns)))
 
 
 def ham_split_plan(num_slots, n_kv_heads: int, ctas: int):

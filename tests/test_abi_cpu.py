@@ -77,6 +77,7 @@ def test_null_arguments_are_rejected(libham):
     assert libham.ham_slot_lengths(None, None, None, None) == ham.HAM_EINVAL
     assert libham.ham_kv_status(None, None, None) == ham.HAM_EINVAL
     assert libham.ham_kv_get_info(None, None) == ham.HAM_EINVAL
+    assert libham.ham_kv_set_wait_limit_ns(None, 1000) == ham.HAM_EINVAL
 
 
 # ---------------------------------------------------------------------------------------
