@@ -154,6 +154,12 @@ bool attention_supported(int head_dim, int group);
 // {64 elements, head_dim / 64, rows} with a box of {64, head_dim / 64, 16 rows} (half_box:
 // {64, 1, 16 rows}, one 64-column half of a chunk) and the 128-byte swizzle.  Returns a
 // CUresult (0 on success).
+// TMA map of a row-major [rows][heads][head_dim] bf16 tensor viewed as {64 elements,
+// head_dim / 64, heads, rows} with a box of {64, 1, box_heads, box_rows} (one 64-column half of
+// box_heads x box_rows head rows) and the 128-byte swizzle.  Boxes past the last row read zeros.
+// Returns a CUresult (0 on success).
+int make_rows_tensor_map(CUtensorMap *map, const void *base, int64_t rows, int heads,
+                         int head_dim, int box_heads, int box_rows);
 int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim,
                          bool half_box);
 cudaError_t launch_append(const AppendView &v, cudaStream_t stream);

@@ -286,53 +286,63 @@ __global__ void __launch_bounds__(kRopeThreads) prefill_rope_kernel(PrefillView 
 }
 
 // ------------------------------------------------------------------------------------
-// 3. causal attention of the chunk
+// 3. causal attention of the chunk, on the 5th-generation tensor cores (tcgen05)
 // ------------------------------------------------------------------------------------
+// A CTA covers one KV head and two Q tiles of 128 rows each; a row is a (query row, head)
+// pair, m = (row - first row of the tile) * G + head within the group, and sits in TMEM lane m.
+// TMEM columns: S_0, S_1 (64 fp32 scores of the current K tile), O_0, O_1 (head_dim fp32).
 template <int D>
-struct PShape {
-  static constexpr int kWarps = 8;                         // consumer warps, one m-tile each
-  static constexpr int kThreads = (kWarps + 1) * 32;       // and the producer warp
-  static constexpr int kRows = kWarps * 16;                // (query row, head) pairs per CTA
-  static constexpr int kTile = 64;                         // slots per K/V tile
-  static constexpr int kChunks = kTile / kChunkSlots;      // 16-slot TMA chunks per tile
-  static constexpr int kChunkBytes = kChunkSlots * D * 2;
-  static constexpr int kStageBytes = 2 * kChunks * kChunkBytes;  // K chunks, then V chunks
-  static constexpr int kStages = 98304 / kStageBytes;      // 96 KiB ring: 3 (d 128), 6 (d 64)
-  static constexpr int kKSteps = D / 16;                   // k-steps of q.k
-  static constexpr int kONBlocks = D / 8;                  // n-blocks of o
-  static constexpr int kOffBar = kStages * kStageBytes;    // from a 1024-byte aligned base
-  static constexpr int kSmem = 1024 + kOffBar + 2 * kStages * 8 + kStages * 4 + 16;
+struct TcShape {
+  static constexpr int kTile = 64;                           // slots per K/V tile
+  static constexpr int kChunks = kTile / kChunkSlots;        // 16-slot TMA chunks per tile
+  static constexpr int kHalves = D / 64;                     // 64-column halves of a row
+  static constexpr int kHalfTileBytes = kTile * 128;         // one half of a K or V tile
+  static constexpr int kKVBytes = kHalves * kHalfTileBytes;  // a K (or V) tile
+  static constexpr int kStages = D == 128 ? 3 : 4;
+  static constexpr int kQHalfBytes = 128 * 128;              // one half of a Q tile
+  static constexpr int kQBytes = kHalves * kQHalfBytes;
+  static constexpr int kPBytes = 128 * kTile * 2;            // bf16 probabilities of a Q tile
+  static constexpr int kOffP = 2 * kQBytes;                  // Q tiles at 0
+  static constexpr int kOffRing = kOffP + 2 * kPBytes;       // stage s: K tile, then V tile
+  static constexpr int kOffBar = kOffRing + kStages * 2 * kKVBytes;
+  // k_full, v_full, kv_empty [kStages]; q_full; s_full, p_full, o_done [2]; mma_done
+  static constexpr int kBars = 3 * kStages + 8;
+  static constexpr int kSmem = 1024 + kOffBar + kBars * 8 + 16;
+  static constexpr uint32_t kTmemCols = D == 128 ? 512 : 256;
+  static constexpr int kProducerWarp = 8, kMmaWarp = 9;      // softmax: warps 0-3 and 4-7
+  static constexpr int kThreads = 10 * 32;
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
-  static_assert(kStages >= 2, "ring depth");
+  static_assert(128 + 2 * D <= (int)kTmemCols, "TMEM columns");
+  static_assert(kSmem <= 227 * 1024, "shared memory");
 };
 
-// A chunk tile in shared memory: its 64-column halves one after the other, each 16 slot rows
-// of 128 bytes written by its own TMA copy with the 128-byte swizzle.  Byte offset of the
-// 16-byte piece c (elements 8c .. 8c+7) of slot row `row`: the piece index inside the line is
-// XORed with the row, so the eight rows of an ldmatrix matrix hit eight different bank groups.
-constexpr int kHalfBytes = kChunkSlots * 128;
-__device__ __forceinline__ uint32_t half_tile_offset(int row, int c) {
-  return (uint32_t)((c >> 3) * kHalfBytes + row * 128 + (((c & 7) ^ (row & 7)) << 4));
-}
-
 template <typename OutT>
-__device__ __forceinline__ void store_pair(void *out, int64_t i, float x, float y) {
+__device__ __forceinline__ void store_row32(OutT *dst, const uint32_t (&o)[32], float scale) {
   if constexpr (std::is_same<OutT, float>::value) {
-    *reinterpret_cast<float2 *>(static_cast<float *>(out) + i) = make_float2(x, y);
+#pragma unroll
+    for (int e = 0; e < 32; e += 4)
+      *reinterpret_cast<float4 *>(dst + e) =
+          make_float4(__uint_as_float(o[e]) * scale, __uint_as_float(o[e + 1]) * scale,
+                      __uint_as_float(o[e + 2]) * scale, __uint_as_float(o[e + 3]) * scale);
   } else {
-    *reinterpret_cast<uint32_t *>(static_cast<__nv_bfloat16 *>(out) + i) = pack_bf16x2(x, y);
+#pragma unroll
+    for (int e = 0; e < 32; e += 8)
+      *reinterpret_cast<uint4 *>(dst + e) = make_uint4(
+          pack_bf16x2(__uint_as_float(o[e]) * scale, __uint_as_float(o[e + 1]) * scale),
+          pack_bf16x2(__uint_as_float(o[e + 2]) * scale, __uint_as_float(o[e + 3]) * scale),
+          pack_bf16x2(__uint_as_float(o[e + 4]) * scale, __uint_as_float(o[e + 5]) * scale),
+          pack_bf16x2(__uint_as_float(o[e + 6]) * scale, __uint_as_float(o[e + 7]) * scale));
   }
 }
 
-// One CTA per SM.  Registers are granted to a block in groups of four warps, so the nine warps
-// (twelve as allocated) may use at most 170 registers a thread: 168, with a few bytes spilled
-// at head_dim 128.
+// One CTA per SM (shared memory and 512 TMEM columns at head_dim 128).
 template <int D, typename OutT>
-__global__ void __launch_bounds__(PShape<D>::kThreads, 1)
-    prefill_attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
+__global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
+    prefill_attn_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                        const __grid_constant__ CUtensorMap tmap_k,
                         const __grid_constant__ CUtensorMap tmap_v, const PrefillView v) {
-  using S = PShape<D>;
-  const int Hq = v.n_q_heads, Hkv = v.n_kv_heads, G = Hq / Hkv, QB = S::kRows / G;
+  using S = TcShape<D>;
+  const int Hq = v.n_q_heads, Hkv = v.n_kv_heads, G = Hq / Hkv, R = 128 / G, QB = 2 * R;
   const int g = blockIdx.x;
   const int64_t xq = (int64_t)gridDim.y - 1 - blockIdx.y;  // latest query blocks first
   int lo = 0, hi = v.batch - 1;                            // the sequence of query block xq
@@ -344,272 +354,364 @@ __global__ void __launch_bounds__(PShape<D>::kThreads, 1)
   if (si.x < 0 || xq < si.z || xq >= (int64_t)si.z + (si.y + QB - 1) / QB) return;
   const int b = lo, L = si.x, n = si.y;
   const int qb0 = (int)(xq - si.z) * QB;
-  const int kv_end = L + min(qb0 + QB, n);  // the CTA's rows attend over slots 0 .. kv_end-1
-  const int ntiles = (kv_end + S::kTile - 1) / S::kTile;
   const int64_t row0 = v.offsets[b];
+  // rows of each Q tile and the K/V tiles they reach (slots 0 .. L + last row)
+  const int rows_q0 = min(R, n - qb0), rows_q1 = max(0, min(R, n - qb0 - R));
+  int ntile[2];
+  ntile[0] = (L + qb0 + rows_q0 + S::kTile - 1) / S::kTile;
+  ntile[1] = rows_q1 > 0 ? (L + qb0 + R + rows_q1 + S::kTile - 1) / S::kTile : 0;
+  const int ntiles = max(ntile[0], ntile[1]);
+  const int kv_end = L + qb0 + (rows_q1 > 0 ? R + rows_q1 : rows_q0);  // no slot >= is attended
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t *full = reinterpret_cast<uint64_t *>(smem + S::kOffBar);
-  uint64_t *empty = full + S::kStages;
-  int *chunk_ok = reinterpret_cast<int *>(empty + S::kStages);  // bit c: chunk c was copied
-  volatile int *abort_flag = chunk_ok + S::kStages;
+  uint64_t *k_full = reinterpret_cast<uint64_t *>(smem + S::kOffBar);
+  uint64_t *v_full = k_full + S::kStages, *kv_empty = v_full + S::kStages;
+  uint64_t *q_full = kv_empty + S::kStages;
+  uint64_t *s_full = q_full + 1, *p_full = q_full + 3, *o_done = q_full + 5;
+  uint64_t *mma_done = q_full + 7;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(k_full + S::kBars);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
     for (int s = 0; s < S::kStages; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], S::kWarps);
+      mbar_init(&k_full[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
     }
+    mbar_init(q_full, 1);
+    for (int q = 0; q < 2; ++q) {
+      mbar_init(&s_full[q], 1);
+      mbar_init(&p_full[q], 4);  // one arrival per warp of the softmax group
+      mbar_init(&o_done[q], 1);
+    }
+    mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (tid == S::kWarps * 32) {
+  if (warp == S::kProducerWarp && lane == 0) {
+    prefetch_tensormap(&tmap_q);
     prefetch_tensormap(&tmap_k);
     prefetch_tensormap(&tmap_v);
   }
+  if (warp == S::kMmaWarp) tmem_alloc<S::kTmemCols>(tmem_slot);
+  tc_fence_before();
   __syncthreads();
-
-  // ring and data waits: the launch's limit; the final drain of in-flight copies keeps 2 s
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  // ring and data waits: the launch's limit; draining in-flight work keeps the default 2 s
   const uint64_t wait_lim = data_wait_limit(v.wait_ns);
-  if (warp == S::kWarps) {
-    // Producer: one lane streams the tiles.  A chunk past the last attended slot or on a page
-    // outside the pool is not copied (its bit stays clear and the consumers mask it).
-    if (lane != 0) return;
-    const uint64_t pol = policy_evict_last();  // every query block of the sequence reads them
-    int issued = 0;
-    for (int t = 0; t < ntiles; ++t) {
-      const int s = t % S::kStages;
-      if (t >= S::kStages &&
-          !thread_wait(&empty[s], (uint32_t)((t / S::kStages) - 1) & 1u, abort_flag, true,
-                       wait_lim)) {
-        if (!*abort_flag) {
-          record_error(v.err, HAM_DEVERR_TIMEOUT);
-          *abort_flag = 1;
-        }
-        break;
-      }
-      int mask = 0, rows[S::kChunks];
-#pragma unroll
-      for (int c = 0; c < S::kChunks; ++c) {
-        const int slot0 = t * S::kTile + c * kChunkSlots;
-        rows[c] = 0;
-        if (slot0 >= kv_end) continue;
-        const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
-        if (page < 0 || page >= v.pool_pages) {
-          record_error(v.err, HAM_DEVERR_PAGE);
-          continue;
-        }
-        rows[c] = (page * Hkv + g) * v.page_slots + slot0 % v.page_slots;
-        mask |= 1 << c;
-      }
-      chunk_ok[s] = mask;
-      mbar_arrive_tx(&full[s], (uint32_t)(__popc(mask) * 2 * S::kChunkBytes));
-      uint8_t *dst = smem + s * S::kStageBytes;
-#pragma unroll
-      for (int c = 0; c < S::kChunks; ++c) {
-        if (!(mask & (1 << c))) continue;
-#pragma unroll
-        for (int hh = 0; hh < D / 64; ++hh) {  // one 64-column half of the chunk per copy
-          tma_load_3d(dst + c * S::kChunkBytes + hh * kHalfBytes, &tmap_k, 0, hh, rows[c],
-                      &full[s], pol);
-          tma_load_3d(dst + (S::kChunks + c) * S::kChunkBytes + hh * kHalfBytes, &tmap_v, 0, hh,
-                      rows[c], &full[s], pol);
-        }
-      }
-      issued = t + 1;
-    }
-    // copies still in flight land before the CTA exits
-    for (int t = max(0, issued - S::kStages); t < issued; ++t)
-      thread_wait(&full[t % S::kStages], (uint32_t)(t / S::kStages) & 1u, abort_flag, false);
-    return;
-  }
 
-  // Consumer warp: the m-tile of query head h = g G + (warp % G), sequence-local rows
-  // j0 .. j0 + 15.  Lane rows ra = j0 + lane / 4 and rb = ra + 8.
-  const int h = g * G + warp % G;
-  const int j0 = qb0 + (warp / G) * 16;
-  const int ra = j0 + (lane >> 2), rb = ra + 8;
-  const int warp_end = j0 < n ? L + min(j0 + 15, n - 1) + 1 : 0;  // slots < warp_end
-  const int lim_a = min(L + ra, warp_end - 1), lim_b = min(L + rb, warp_end - 1);
-  uint32_t qf[S::kKSteps][4];  // A operand: rows ra / rb, k-columns 2 (lane % 4) (+ 8)
-  {
-    const int c0 = 2 * (lane & 3);
-    const uint32_t *qa = reinterpret_cast<const uint32_t *>(v.q + ((row0 + ra) * Hq + h) * D);
-    const uint32_t *qb = reinterpret_cast<const uint32_t *>(v.q + ((row0 + rb) * Hq + h) * D);
-#pragma unroll
-    for (int ks = 0; ks < S::kKSteps; ++ks) {
-      qf[ks][0] = ra < n ? qa[(ks * 16 + c0) / 2] : 0u;
-      qf[ks][1] = rb < n ? qb[(ks * 16 + c0) / 2] : 0u;
-      qf[ks][2] = ra < n ? qa[(ks * 16 + c0 + 8) / 2] : 0u;
-      qf[ks][3] = rb < n ? qb[(ks * 16 + c0 + 8) / 2] : 0u;
-    }
-  }
-  // softmax scale and log2(e): scores in the exp2 domain
-  const float sl2 = (float)(1.4426950408889634 / sqrt((double)D));
-  float o[S::kONBlocks][4];
-#pragma unroll
-  for (int on = 0; on < S::kONBlocks; ++on) o[on][0] = o[on][1] = o[on][2] = o[on][3] = 0.f;
-  float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;
-  const int mi = lane >> 3, mr = lane & 7;  // ldmatrix: this lane's matrix and row
-  bool ok = true;
-  for (int t = 0; t < ntiles; ++t) {
-    const int s = t % S::kStages;
-    if (!warp_wait(&full[s], (uint32_t)(t / S::kStages) & 1u, abort_flag, wait_lim)) {
-      if (lane == 0 && !*abort_flag) {
-        record_error(v.err, HAM_DEVERR_TIMEOUT);
-        *abort_flag = 1;
-      }
-      ok = false;
-      break;
-    }
-    const int tbase = t * S::kTile;
-    if (tbase < warp_end) {
-      const int mask = chunk_ok[s];
-      const uint8_t *kt = smem + s * S::kStageBytes;
-      const uint8_t *vt = kt + S::kChunks * S::kChunkBytes;
-      float sc[2 * S::kChunks][4];
-#pragma unroll
-      for (int nb = 0; nb < 2 * S::kChunks; ++nb) sc[nb][0] = sc[nb][1] = sc[nb][2] = sc[nb][3] = 0.f;
-      // S = Q K^T: per chunk, ldmatrix matrices (slots 0-7 | 8-15) x (d lo | hi) give the
-      // B fragments of the chunk's two 8-slot n-blocks.  k-steps outside, chunks inside: the
-      // eight accumulators take turns instead of chaining on one.
-#pragma unroll
-      for (int ks = 0; ks < S::kKSteps; ++ks) {
+  if (warp == S::kProducerWarp) {
+    // ------------------------------------------------------------ producer: TMA copies
+    if (lane == 0) {
+      const uint64_t pol_kv = policy_evict_last();   // every query block of the sequence reads them
+      const uint64_t pol_q = policy_evict_first();
+      const int nq = rows_q1 > 0 ? 2 : 1;
+      mbar_arrive_tx(q_full, (uint32_t)(nq * S::kQBytes));
+      for (int q = 0; q < nq; ++q)
+        for (int hh = 0; hh < S::kHalves; ++hh)
+          tma_load_4d(smem + q * S::kQBytes + hh * S::kQHalfBytes, &tmap_q, 0, hh, g * G,
+                      (int)(row0 + qb0 + q * R), q_full, pol_q);
+      int issued = 0;
+      for (int t = 0; t < ntiles; ++t) {
+        const int st = t % S::kStages;
+        if (t >= S::kStages &&
+            !thread_wait(&kv_empty[st], (uint32_t)((t / S::kStages) - 1) & 1u, abort_flag, true,
+                         wait_lim)) {
+          if (!*abort_flag) {
+            record_error(v.err, HAM_DEVERR_TIMEOUT);
+            *abort_flag = 1;
+          }
+          break;
+        }
+        // chunks at or past kv_end are not copied: their rows are masked and zeroed before use
+        int64_t rows[S::kChunks];
+        int nck = 0;
+        bool bad = false;
 #pragma unroll
         for (int c = 0; c < S::kChunks; ++c) {
-          if (tbase + c * kChunkSlots >= warp_end) continue;
-          uint32_t kf[4];
-          ldmatrix_x4(kf, smem_u32(kt + c * S::kChunkBytes +
-                                   half_tile_offset((mi >> 1) * 8 + mr, 2 * ks + (mi & 1))));
-          mma_16816(sc[2 * c], qf[ks], kf[0], kf[1]);
-          mma_16816(sc[2 * c + 1], qf[ks], kf[2], kf[3]);
+          const int slot0 = t * S::kTile + c * kChunkSlots;
+          rows[c] = -1;
+          if (slot0 >= kv_end) continue;
+          const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
+          if (page < 0 || page >= v.pool_pages) {
+            bad = true;
+            continue;
+          }
+          rows[c] = ((int64_t)page * Hkv + g) * v.page_slots + slot0 % v.page_slots;
+          ++nck;
         }
-      }
-      // causal mask and copied chunks (only on tiles that reach past the m-tile's first row or
-      // miss a chunk); row maxima of the raw scores over the quad
-      if (tbase + S::kTile - 1 > L + j0 || mask != (1 << S::kChunks) - 1) {
-#pragma unroll
-        for (int nb = 0; nb < 2 * S::kChunks; ++nb) {
-          const bool cok = (mask >> (nb >> 1)) & 1;
-          const int slot = tbase + nb * 8 + 2 * (lane & 3);
-          if (!(cok && slot <= lim_a)) sc[nb][0] = -INFINITY;
-          if (!(cok && slot + 1 <= lim_a)) sc[nb][1] = -INFINITY;
-          if (!(cok && slot <= lim_b)) sc[nb][2] = -INFINITY;
-          if (!(cok && slot + 1 <= lim_b)) sc[nb][3] = -INFINITY;
+        if (bad) {  // the plan validated the table; a page outside the pool ends this CTA
+          record_error(v.err, HAM_DEVERR_PAGE);
+          *abort_flag = 1;
+          break;
         }
-      }
-      float mx_a = -INFINITY, mx_b = -INFINITY;
+        const uint32_t bytes = (uint32_t)(nck * kChunkSlots * D * 2);
+        mbar_arrive_tx(&k_full[st], bytes);
+        mbar_arrive_tx(&v_full[st], bytes);
+        uint8_t *kt = smem + S::kOffRing + st * 2 * S::kKVBytes, *vt = kt + S::kKVBytes;
 #pragma unroll
-      for (int nb = 0; nb < 2 * S::kChunks; ++nb) {
-        mx_a = fmaxf(mx_a, fmaxf(sc[nb][0], sc[nb][1]));
-        mx_b = fmaxf(mx_b, fmaxf(sc[nb][2], sc[nb][3]));
-      }
+        for (int c = 0; c < S::kChunks; ++c) {
+          if (rows[c] < 0) continue;
 #pragma unroll
-      for (int off = 1; off < 4; off <<= 1) {
-        mx_a = fmaxf(mx_a, __shfl_xor_sync(kFull, mx_a, off));
-        mx_b = fmaxf(mx_b, __shfl_xor_sync(kFull, mx_b, off));
-      }
-      // Running maxima in the exp2 domain, raised lazily: only when a score passes them by more
-      // than kRescaleSlack (p then stays below 2^kRescaleSlack), so most tiles skip rescaling O.
-      mx_a *= sl2;
-      mx_b *= sl2;
-      float al_a = 1.f, al_b = 1.f;
-      if (mx_a > m_a + kRescaleSlack) {
-        al_a = ex2(m_a - mx_a);
-        m_a = mx_a;
-      }
-      if (mx_b > m_b + kRescaleSlack) {
-        al_b = ex2(m_b - mx_b);
-        m_b = mx_b;
-      }
-      const float ref_a = m_a == -INFINITY ? 0.f : m_a;  // nothing attended yet
-      const float ref_b = m_b == -INFINITY ? 0.f : m_b;
-      float rs_a = 0.f, rs_b = 0.f;
-#pragma unroll
-      for (int nb = 0; nb < 2 * S::kChunks; ++nb) {
-        sc[nb][0] = ex2(fmaf(sc[nb][0], sl2, -ref_a));
-        sc[nb][1] = ex2(fmaf(sc[nb][1], sl2, -ref_a));
-        sc[nb][2] = ex2(fmaf(sc[nb][2], sl2, -ref_b));
-        sc[nb][3] = ex2(fmaf(sc[nb][3], sl2, -ref_b));
-        rs_a += sc[nb][0] + sc[nb][1];
-        rs_b += sc[nb][2] + sc[nb][3];
-      }
-      l_a = l_a * al_a + rs_a;  // per-lane partial sums, reduced over the quad at the end
-      l_b = l_b * al_b + rs_b;
-      if (__any_sync(kFull, al_a != 1.f || al_b != 1.f)) {
-#pragma unroll
-        for (int on = 0; on < S::kONBlocks; ++on) {
-          o[on][0] *= al_a;
-          o[on][1] *= al_a;
-          o[on][2] *= al_b;
-          o[on][3] *= al_b;
+          for (int hh = 0; hh < S::kHalves; ++hh) {
+            const int off = hh * S::kHalfTileBytes + c * kChunkSlots * 128;
+            tma_load_3d(kt + off, &tmap_k, 0, hh, (int)rows[c], &k_full[st], pol_kv);
+            tma_load_3d(vt + off, &tmap_v, 0, hh, (int)rows[c], &v_full[st], pol_kv);
+          }
         }
+        issued = t + 1;
       }
-      // O += P V: P of chunk kk is the A fragment of k-step kk; V by transposing ldmatrix
-      // (matrices (slots 0-7 | 8-15) x (d lo | hi))
+      // every copy this CTA issued lands before the CTA can exit
+      thread_wait(q_full, 0u, abort_flag, false);
+      for (int t = max(0, issued - S::kStages); t < issued; ++t) {
+        thread_wait(&k_full[t % S::kStages], (uint32_t)(t / S::kStages) & 1u, abort_flag, false);
+        thread_wait(&v_full[t % S::kStages], (uint32_t)(t / S::kStages) & 1u, abort_flag, false);
+      }
+    }
+  } else if (warp == S::kMmaWarp) {
+    // ------------------------------------------------------------ MMA issue (lane 0)
+    // Order per K/V tile t and Q tile q: O_q += P_q(t) V_t as soon as the softmax group has
+    // written P_q(t), then S_q(t+1) = Q_q K_(t+1)^T; the two Q tiles alternate, so the tensor
+    // cores work on one while the other's softmax runs.  A commit to s_full[q] therefore also
+    // covers the P V product before it (tcgen05 operations of one thread complete in order).
+    constexpr uint32_t id_s = idesc_bf16(128, S::kTile, false);  // K-major Q and K
+    constexpr uint32_t id_o = idesc_bf16(128, D, true);          // K-major P, MN-major V
+    const uint32_t q_base = smem_u32(smem), p_base = smem_u32(smem + S::kOffP);
+    const uint32_t ring = smem_u32(smem + S::kOffRing);
+    auto issue_s = [&](int q, int t) {
+      const uint32_t kt = ring + (uint32_t)((t % S::kStages) * 2 * S::kKVBytes);
 #pragma unroll
-      for (int kk = 0; kk < S::kChunks; ++kk) {
-        if (tbase + kk * kChunkSlots >= warp_end || !((mask >> kk) & 1)) continue;
-        const uint32_t pa[4] = {pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]),
-                                pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]),
-                                pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]),
-                                pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3])};
-        const uint8_t *vc = vt + kk * S::kChunkBytes;
+      for (int k = 0; k < D / 16; ++k) {
+        const uint64_t a = smem_desc_sw128(
+            q_base + q * S::kQBytes + (k >> 2) * S::kQHalfBytes + (k & 3) * 32, 16, 1024);
+        const uint64_t bk =
+            smem_desc_sw128(kt + (k >> 2) * S::kHalfTileBytes + (k & 3) * 32, 16, 1024);
+        tc_mma(tmem + q * S::kTile, a, bk, id_s, k > 0);
+      }
+    };
+    auto issue_o = [&](int q, int t) {
+      const uint32_t vt = ring + (uint32_t)((t % S::kStages) * 2 * S::kKVBytes + S::kKVBytes);
 #pragma unroll
-        for (int np = 0; np < D / 16; ++np) {
-          uint32_t vf[4];
-          ldmatrix_x4_trans(vf, smem_u32(vc + half_tile_offset((mi & 1) * 8 + mr,
-                                                               2 * np + (mi >> 1))));
-          mma_16816(o[2 * np], pa, vf[0], vf[1]);
-          mma_16816(o[2 * np + 1], pa, vf[2], vf[3]);
+      for (int k = 0; k < S::kTile / 16; ++k) {
+        const uint64_t a = smem_desc_sw128(p_base + q * S::kPBytes + k * 32, 16, 1024);
+        const uint64_t bv = smem_desc_sw128(vt + k * 2048, S::kHalfTileBytes, 1024);
+        tc_mma(tmem + 2 * S::kTile + q * D, a, bv, id_o, t > 0 || k > 0);
+      }
+    };
+    bool ok = warp_wait(q_full, 0u, abort_flag, wait_lim) &&
+              warp_wait(&k_full[0], 0u, abort_flag, wait_lim);
+    if (ok && lane == 0) {
+      tc_fence_after();
+      for (int q = 0; q < 2; ++q)
+        if (ntile[q] > 0) {
+          issue_s(q, 0);
+          tc_commit(&s_full[q]);
+        }
+    }
+    __syncwarp();
+    for (int t = 0; ok && t < ntiles; ++t) {
+      const int st = t % S::kStages;
+      if (!warp_wait(&v_full[st], (uint32_t)(t / S::kStages) & 1u, abort_flag, wait_lim)) {
+        ok = false;
+        break;
+      }
+      if (t == ntiles - 1 && kv_end < (t + 1) * S::kTile) {
+        // slots >= kv_end get p = 0; zero their value rows so that stale bits never reach O
+        const int z0 = kv_end - t * S::kTile, per_half = (S::kTile - z0) * 8;
+        uint8_t *vt = smem + S::kOffRing + st * 2 * S::kKVBytes + S::kKVBytes;
+        for (int e = lane; e < S::kHalves * per_half; e += 32) {
+          const int hh = e / per_half, r = e % per_half;
+          *reinterpret_cast<uint4 *>(vt + hh * S::kHalfTileBytes + z0 * 128 + r * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+      }
+      for (int q = 0; q < 2 && ok; ++q) {
+        if (t >= ntile[q]) continue;
+        if (!warp_wait(&p_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          tc_fence_after();
+          issue_o(q, t);
+          if (t == ntile[q] - 1) tc_commit(&o_done[q]);
+        }
+        if (t + 1 < ntile[q]) {
+          const int t1 = t + 1;
+          if (!warp_wait(&k_full[t1 % S::kStages], (uint32_t)(t1 / S::kStages) & 1u, abort_flag,
+                         wait_lim)) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            issue_s(q, t1);
+            tc_commit(&s_full[q]);
+          }
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+      if (lane == 0) tc_commit(&kv_empty[st]);  // K_t and V_t are free once these complete
+      __syncwarp();
+    }
+    if (!ok && lane == 0 && !*abort_flag) {
+      record_error(v.err, HAM_DEVERR_TIMEOUT);
+      *abort_flag = 1;
+    }
+    // every MMA issued completes before the tensor memory is freed
+    if (lane == 0) {
+      tc_commit(mma_done);
+      thread_wait(mma_done, 0u, abort_flag, false);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax groups
+    // Thread = TMEM lane = row m of Q tile q.  Each row's scores arrive whole in its own thread,
+    // so the row maximum and sum need no shuffles.
+    const int q = warp >> 2, m = tid & 127;
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t t_s = tmem + lane_base + q * S::kTile;
+    const uint32_t t_o = tmem + lane_base + 2 * S::kTile + q * D;
+    const int j = qb0 + q * R + m / G;          // the row's index in the sequence's chunk
+    const int lim = L + min(j, n - 1);          // last slot it attends (rows past n: not stored)
+    const int lim_min = L + qb0 + q * R;        // smallest limit of the tile's stored rows
+    const float sl2 = (float)(1.4426950408889634 / sqrt((double)D));  // 1/sqrt(d), log2(e)
+    uint8_t *prow = smem + S::kOffP + q * S::kPBytes + m * 128;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int t = 0; t < ntile[q]; ++t) {
+      if (!warp_wait(&s_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      uint32_t sa[32], sb[32];
+      tmem_ld32(t_s, sa);
+      tmem_ld32(t_s + 32, sb);
+      tmem_wait_ld();
+      float s[S::kTile];
+#pragma unroll
+      for (int c = 0; c < 32; ++c) {
+        s[c] = __uint_as_float(sa[c]);
+        s[c + 32] = __uint_as_float(sb[c]);
+      }
+      const int tbase = t * S::kTile;
+      if (tbase + S::kTile - 1 > lim_min) {  // the causal edge (and the chunk's end) in this tile
+#pragma unroll
+        for (int c = 0; c < S::kTile; ++c)
+          if (tbase + c > lim) s[c] = -INFINITY;
+      }
+      float mx = s[0];
+#pragma unroll
+      for (int c = 1; c < S::kTile; ++c) mx = fmaxf(mx, s[c]);
+      mx *= sl2;
+      // Running maximum in the exp2 domain, raised lazily: only when a score passes it by more
+      // than kRescaleSlack (p then stays below 2^kRescaleSlack), so O is rarely rescaled.  The
+      // first tile always raises it (slot 0 is attended by every row).
+      float alpha = 1.f;
+      if (mx > m_run + kRescaleSlack) {
+        alpha = ex2(m_run - mx);
+        m_run = mx;
+      }
+      // S_q(t) completed after O_q's last product (in-order completion), and the next product
+      // waits for p_full: O_q is stable here.
+      if (t > 0 && __any_sync(kFull, alpha != 1.f)) {
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t o[32];
+          tmem_ld32(t_o + c0, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          tmem_st32(t_o + c0, o);
+        }
+        tmem_wait_st();
+      }
+      float rs = 0.f;
+      uint32_t pk[S::kTile / 2];
+#pragma unroll
+      for (int c = 0; c < S::kTile / 2; ++c) {
+        const float p0 = ex2(fmaf(s[2 * c], sl2, -m_run));
+        const float p1 = ex2(fmaf(s[2 * c + 1], sl2, -m_run));
+        rs += p0 + p1;
+        pk[c] = pack_bf16x2(p0, p1);
+      }
+      l_run = l_run * alpha + rs;
+      // P row m: 128 bytes in the 128-byte swizzle (K-major operand of the P V product)
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        *reinterpret_cast<uint4 *>(prow + ((c ^ (m & 7)) << 4)) =
+            make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[q]);
+    }
+    if (ok && ntile[q] > 0) {
+      if (!warp_wait(&o_done[q], 0u, abort_flag, wait_lim)) {
+        ok = false;
+      } else {
+        tc_fence_after();
+        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+        const bool stored = j < n;
+        OutT *orow = static_cast<OutT *>(v.out) +
+                     ((row0 + j) * Hq + g * G + m % G) * (int64_t)D;
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t o[32];
+          tmem_ld32(t_o + c0, o);
+          tmem_wait_ld();
+          if (stored) store_row32<OutT>(orow + c0, o, inv);
         }
       }
     }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[s]);
+    if (!ok && lane == 0 && !*abort_flag) {
+      record_error(v.err, HAM_DEVERR_TIMEOUT);
+      *abort_flag = 1;
+    }
   }
-  if (!ok) return;
-#pragma unroll
-  for (int off = 1; off < 4; off <<= 1) {
-    l_a += __shfl_xor_sync(kFull, l_a, off);
-    l_b += __shfl_xor_sync(kFull, l_b, off);
-  }
-  const float inv_a = l_a > 0.f ? 1.f / l_a : 0.f, inv_b = l_b > 0.f ? 1.f / l_b : 0.f;
-  const int64_t oa = ((row0 + ra) * Hq + h) * D, ob = ((row0 + rb) * Hq + h) * D;
-#pragma unroll
-  for (int on = 0; on < S::kONBlocks; ++on) {
-    const int d = on * 8 + 2 * (lane & 3);
-    if (ra < n) store_pair<OutT>(v.out, oa + d, o[on][0] * inv_a, o[on][1] * inv_a);
-    if (rb < n) store_pair<OutT>(v.out, ob + d, o[on][2] * inv_b, o[on][3] * inv_b);
+  // all tensor-memory reads and MMAs are done: free the columns
+  tc_fence_before();
+  __syncthreads();
+  if (warp == S::kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc<S::kTmemCols>(tmem);
   }
 }
 
 template <int D, typename OutT>
-cudaError_t launch_attn(const CUtensorMap &tk, const CUtensorMap &tv, const PrefillView &v,
-                        cudaStream_t stream) {
-  using S = PShape<D>;
+cudaError_t launch_attn(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
+                        const PrefillView &v, cudaStream_t stream) {
+  using S = TcShape<D>;
   cudaError_t e = cudaFuncSetAttribute(prefill_attn_kernel<D, OutT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmem);
   if (e != cudaSuccess) return e;
-  const int QB = S::kRows / (v.n_q_heads / v.n_kv_heads);
+  const int QB = prefill_query_rows(v.n_q_heads / v.n_kv_heads);
   const dim3 grid((unsigned)v.n_kv_heads, (unsigned)(v.rows / QB + v.batch));
-  prefill_attn_kernel<D, OutT><<<grid, S::kThreads, S::kSmem, stream>>>(tk, tv, v);
+  prefill_attn_kernel<D, OutT><<<grid, S::kThreads, S::kSmem, stream>>>(tq, tk, tv, v);
   return cudaGetLastError();
 }
 
 template <typename OutT>
 cudaError_t launch_all(const CUtensorMap &tk, const CUtensorMap &tv, const PrefillView &v,
                        cudaStream_t stream) {
-  const int QB = PShape<128>::kRows / (v.n_q_heads / v.n_kv_heads);
-  prefill_plan_kernel<<<(unsigned)v.batch, kPlanThreads, 0, stream>>>(v, QB);
+  const int G = v.n_q_heads / v.n_kv_heads;
+  CUtensorMap tq;  // the chunk's queries, rotated in place by the RoPE kernel
+  if (make_rows_tensor_map(&tq, v.q, v.rows, v.n_q_heads, v.head_dim, G, 128 / G) != 0)
+    return cudaErrorInvalidValue;
+  prefill_plan_kernel<<<(unsigned)v.batch, kPlanThreads, 0, stream>>>(v, prefill_query_rows(G));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   prefill_rope_kernel<OutT><<<(unsigned)v.rows, kRopeThreads, 0, stream>>>(v);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  return v.head_dim == 128 ? launch_attn<128, OutT>(tk, tv, v, stream)
-                           : launch_attn<64, OutT>(tk, tv, v, stream);
+  return v.head_dim == 128 ? launch_attn<128, OutT>(tq, tk, tv, v, stream)
+                           : launch_attn<64, OutT>(tq, tk, tv, v, stream);
 }
 
 }  // namespace
@@ -619,7 +721,8 @@ bool prefill_supported(int head_dim, int group) {
          (group == 1 || group == 2 || group == 4 || group == 8);
 }
 
-int prefill_query_rows(int group) { return PShape<128>::kRows / group; }
+// Two Q tiles of 128 (row, head) pairs per CTA.
+int prefill_query_rows(int group) { return 256 / group; }
 
 cudaError_t launch_prefill(const CUtensorMap &tk, const CUtensorMap &tv, const PrefillView &v,
                            int out_dtype, cudaStream_t stream) {

@@ -257,22 +257,46 @@ __global__ void set_lengths_kernel(int32_t *num_slots, int64_t *num_tokens,
   if (new_tokens) num_tokens[b] = new_tokens[b];
 }
 
-int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim,
-                         bool half_box) {
-  using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
-                              const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
-                              const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
-                              CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-  static Encode encode = nullptr;
+namespace {
+using EncodeTiled = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                 const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                 const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                 CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiled tensor_map_encoder() {
+  static EncodeTiled encode = nullptr;
   if (!encode) {
     void *fn = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
                                          &q) != cudaSuccess ||
         q != cudaDriverEntryPointSuccess || !fn)
-      return -1;
-    encode = reinterpret_cast<Encode>(fn);
+      return nullptr;
+    encode = reinterpret_cast<EncodeTiled>(fn);
   }
+  return encode;
+}
+}  // namespace
+
+int make_rows_tensor_map(CUtensorMap *map, const void *base, int64_t rows, int heads,
+                         int head_dim, int box_heads, int box_rows) {
+  EncodeTiled encode = tensor_map_encoder();
+  if (!encode) return -1;
+  const cuuint64_t dims[4] = {64, (cuuint64_t)(head_dim / 64), (cuuint64_t)heads,
+                              (cuuint64_t)rows};
+  const cuuint64_t strides[3] = {128, (cuuint64_t)head_dim * 2,
+                                 (cuuint64_t)heads * head_dim * 2};  // bytes, dims 1..3
+  const cuuint32_t box[4] = {64, 1, (cuuint32_t)box_heads, (cuuint32_t)box_rows};
+  const cuuint32_t estride[4] = {1, 1, 1, 1};
+  return (int)encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims,
+                     strides, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim,
+                         bool half_box) {
+  EncodeTiled encode = tensor_map_encoder();
+  if (!encode) return -1;
   const cuuint64_t dims[3] = {64, (cuuint64_t)(head_dim / 64), (cuuint64_t)rows};
   const cuuint64_t strides[2] = {128, (cuuint64_t)head_dim * 2};  // bytes, dims 1 and 2
   const cuuint32_t box[3] = {64, half_box ? 1u : (cuuint32_t)(head_dim / 64),
