@@ -290,29 +290,34 @@ __global__ void __launch_bounds__(kRopeThreads) prefill_rope_kernel(PrefillView 
 // ------------------------------------------------------------------------------------
 // A CTA covers one KV head and two Q tiles of 128 rows each; a row is a (query row, head)
 // pair, m = (row - first row of the tile) * G + head within the group, and sits in TMEM lane m.
-// TMEM columns: S_0, S_1 (64 fp32 scores of the current K tile), O_0, O_1 (head_dim fp32).
+// TMEM columns: S_0, S_1 (128 fp32 scores of the current 128-slot K tile; the softmax writes
+// the bf16 probabilities P over the first 64 columns of its S, where the P V product reads
+// them), then O_0, O_1 (head_dim fp32).  Reading P from tensor memory and 128-slot tiles keep
+// the shared-memory traffic of the products at 2 operand bytes per 64 FLOP.
 template <int D>
 struct TcShape {
-  static constexpr int kTile = 64;                           // slots per K/V tile
+  static constexpr int kTile = 128;                          // slots per K/V tile
   static constexpr int kChunks = kTile / kChunkSlots;        // 16-slot TMA chunks per tile
   static constexpr int kHalves = D / 64;                     // 64-column halves of a row
   static constexpr int kHalfTileBytes = kTile * 128;         // one half of a K or V tile
   static constexpr int kKVBytes = kHalves * kHalfTileBytes;  // a K (or V) tile
-  static constexpr int kStages = D == 128 ? 3 : 4;
+  static constexpr int kKStages = D == 128 ? 3 : 4;          // K tiles in flight
+  static constexpr int kVStages = D == 128 ? 2 : 4;          // V tiles in flight
   static constexpr int kQHalfBytes = 128 * 128;              // one half of a Q tile
   static constexpr int kQBytes = kHalves * kQHalfBytes;
-  static constexpr int kPBytes = 128 * kTile * 2;            // bf16 probabilities of a Q tile
-  static constexpr int kOffP = 2 * kQBytes;                  // Q tiles at 0
-  static constexpr int kOffRing = kOffP + 2 * kPBytes;       // stage s: K tile, then V tile
-  static constexpr int kOffBar = kOffRing + kStages * 2 * kKVBytes;
-  // k_full, v_full, kv_empty [kStages]; q_full; s_full, p_full, o_done [2]; mma_done
-  static constexpr int kBars = 3 * kStages + 8;
+  static constexpr int kOffK = 2 * kQBytes;                  // Q tiles at 0
+  static constexpr int kOffV = kOffK + kKStages * kKVBytes;
+  static constexpr int kOffBar = kOffV + kVStages * kKVBytes;
+  // k_full, k_empty [kKStages]; v_full, v_empty [kVStages]; q_full; s_full, p_full,
+  // pv_done [2]; mma_done
+  static constexpr int kBars = 2 * kKStages + 2 * kVStages + 8;
   static constexpr int kSmem = 1024 + kOffBar + kBars * 8 + 16;
-  static constexpr uint32_t kTmemCols = D == 128 ? 512 : 256;
+  static constexpr uint32_t kTmemCols = 512;
+  static constexpr int kOffO = 2 * kTile;                    // TMEM column of O_0
   static constexpr int kProducerWarp = 8, kMmaWarp = 9;      // softmax: warps 0-3 and 4-7
   static constexpr int kThreads = 10 * 32;
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
-  static_assert(128 + 2 * D <= (int)kTmemCols, "TMEM columns");
+  static_assert(kOffO + 2 * D <= (int)kTmemCols, "TMEM columns");
   static_assert(kSmem <= 227 * 1024, "shared memory");
 };
 
@@ -367,24 +372,27 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t *k_full = reinterpret_cast<uint64_t *>(smem + S::kOffBar);
-  uint64_t *v_full = k_full + S::kStages, *kv_empty = v_full + S::kStages;
-  uint64_t *q_full = kv_empty + S::kStages;
-  uint64_t *s_full = q_full + 1, *p_full = q_full + 3, *o_done = q_full + 5;
+  uint64_t *k_empty = k_full + S::kKStages, *v_full = k_empty + S::kKStages;
+  uint64_t *v_empty = v_full + S::kVStages, *q_full = v_empty + S::kVStages;
+  uint64_t *s_full = q_full + 1, *p_full = q_full + 3, *pv_done = q_full + 5;
   uint64_t *mma_done = q_full + 7;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(k_full + S::kBars);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
-    for (int s = 0; s < S::kStages; ++s) {
+    for (int s = 0; s < S::kKStages; ++s) {
       mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < S::kVStages; ++s) {
       mbar_init(&v_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&v_empty[s], 1);
     }
     mbar_init(q_full, 1);
     for (int q = 0; q < 2; ++q) {
       mbar_init(&s_full[q], 1);
       mbar_init(&p_full[q], 4);  // one arrival per warp of the softmax group
-      mbar_init(&o_done[q], 1);
+      mbar_init(&pv_done[q], 1);
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -405,8 +413,11 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
 
   if (warp == S::kProducerWarp) {
     // ------------------------------------------------------------ producer: TMA copies
+    // Q once; then per step t the K tile t and the V tile t - 1 (keys are needed a tile before
+    // values).  A chunk at or past kv_end is not copied: its rows are masked (K) or zeroed (V).
+    const uint64_t pol_kv = policy_evict_last();   // every query block of the sequence reads them
+    int k_issued = 0, v_issued = 0;
     if (lane == 0) {
-      const uint64_t pol_kv = policy_evict_last();   // every query block of the sequence reads them
       const uint64_t pol_q = policy_evict_first();
       const int nq = rows_q1 > 0 ? 2 : 1;
       mbar_arrive_tx(q_full, (uint32_t)(nq * S::kQBytes));
@@ -414,75 +425,120 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         for (int hh = 0; hh < S::kHalves; ++hh)
           tma_load_4d(smem + q * S::kQBytes + hh * S::kQHalfBytes, &tmap_q, 0, hh, g * G,
                       (int)(row0 + qb0 + q * R), q_full, pol_q);
-      int issued = 0;
-      for (int t = 0; t < ntiles; ++t) {
-        const int st = t % S::kStages;
-        if (t >= S::kStages &&
-            !thread_wait(&kv_empty[st], (uint32_t)((t / S::kStages) - 1) & 1u, abort_flag, true,
-                         wait_lim)) {
-          if (!*abort_flag) {
-            record_error(v.err, HAM_DEVERR_TIMEOUT);
-            *abort_flag = 1;
-          }
-          break;
+    }
+    // Page-table entries of 32 chunks (4 tiles) at a time, one per lane, requested a batch
+    // ahead: lane l holds the pool row of chunk base + l (-1: at or past kv_end; -2: a page
+    // outside the pool).
+    const int nchunks = (kv_end + kChunkSlots - 1) / kChunkSlots;
+    auto lookup = [&](int base) {
+      int row = -1;
+      if (base + lane < nchunks) {
+        const int slot0 = (base + lane) * kChunkSlots;
+        const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
+        row = page < 0 || page >= v.pool_pages
+                  ? -2
+                  : (int)(((int64_t)page * Hkv + g) * v.page_slots + slot0 % v.page_slots);
+      }
+      return row;
+    };
+    constexpr int kTilesPerBatch = 32 / S::kChunks;
+    int row = lookup(0), row_next = lookup(32);
+    int rows_prev[S::kChunks];
+#pragma unroll
+    for (int c = 0; c < S::kChunks; ++c) rows_prev[c] = -1;
+    // copies of one tile into `dst` (K or V), counted on `bar`
+    auto issue_tile = [&](uint8_t *dst, const CUtensorMap *map, const int (&rows)[S::kChunks],
+                          uint64_t *bar) {
+      int nck = 0;
+#pragma unroll
+      for (int c = 0; c < S::kChunks; ++c) nck += rows[c] >= 0;
+      mbar_arrive_tx(bar, (uint32_t)(nck * kChunkSlots * D * 2));
+#pragma unroll
+      for (int c = 0; c < S::kChunks; ++c) {
+        if (rows[c] < 0) continue;
+#pragma unroll
+        for (int hh = 0; hh < S::kHalves; ++hh)
+          tma_load_3d(dst + hh * S::kHalfTileBytes + c * kChunkSlots * 128, map, 0, hh, rows[c],
+                      bar, pol_kv);
+      }
+    };
+    for (int t = 0; t <= ntiles; ++t) {
+      int rows_cur[S::kChunks];
+      bool bad = false;
+#pragma unroll
+      for (int c = 0; c < S::kChunks; ++c) rows_cur[c] = -1;
+      if (t < ntiles) {
+        if (t > 0 && t % kTilesPerBatch == 0) {
+          row = row_next;
+          row_next = lookup((t / kTilesPerBatch + 1) * 32);
         }
-        // chunks at or past kv_end are not copied: their rows are masked and zeroed before use
-        int64_t rows[S::kChunks];
-        int nck = 0;
-        bool bad = false;
 #pragma unroll
         for (int c = 0; c < S::kChunks; ++c) {
-          const int slot0 = t * S::kTile + c * kChunkSlots;
-          rows[c] = -1;
-          if (slot0 >= kv_end) continue;
-          const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
-          if (page < 0 || page >= v.pool_pages) {
-            bad = true;
-            continue;
-          }
-          rows[c] = ((int64_t)page * Hkv + g) * v.page_slots + slot0 % v.page_slots;
-          ++nck;
+          rows_cur[c] = __shfl_sync(kFull, row, (t % kTilesPerBatch) * S::kChunks + c);
+          bad |= rows_cur[c] == -2;
         }
-        if (bad) {  // the plan validated the table; a page outside the pool ends this CTA
+      }
+      int failed = 0;
+      if (lane == 0) {
+        if (bad) {  // the plan validated the table; a page outside the pool ends the CTA
           record_error(v.err, HAM_DEVERR_PAGE);
           *abort_flag = 1;
-          break;
+          failed = 1;
         }
-        const uint32_t bytes = (uint32_t)(nck * kChunkSlots * D * 2);
-        mbar_arrive_tx(&k_full[st], bytes);
-        mbar_arrive_tx(&v_full[st], bytes);
-        uint8_t *kt = smem + S::kOffRing + st * 2 * S::kKVBytes, *vt = kt + S::kKVBytes;
-#pragma unroll
-        for (int c = 0; c < S::kChunks; ++c) {
-          if (rows[c] < 0) continue;
-#pragma unroll
-          for (int hh = 0; hh < S::kHalves; ++hh) {
-            const int off = hh * S::kHalfTileBytes + c * kChunkSlots * 128;
-            tma_load_3d(kt + off, &tmap_k, 0, hh, (int)rows[c], &k_full[st], pol_kv);
-            tma_load_3d(vt + off, &tmap_v, 0, hh, (int)rows[c], &v_full[st], pol_kv);
+        if (!failed && t < ntiles) {
+          const int st = t % S::kKStages;
+          if (t >= S::kKStages &&
+              !thread_wait(&k_empty[st], (uint32_t)((t / S::kKStages) - 1) & 1u, abort_flag,
+                           true, wait_lim)) {
+            failed = 2;
+          } else {
+            issue_tile(smem + S::kOffK + st * S::kKVBytes, &tmap_k, rows_cur, &k_full[st]);
+            k_issued = t + 1;
           }
         }
-        issued = t + 1;
+        if (!failed && t >= 1) {
+          const int tv = t - 1, st = tv % S::kVStages;
+          if (tv >= S::kVStages &&
+              !thread_wait(&v_empty[st], (uint32_t)((tv / S::kVStages) - 1) & 1u, abort_flag,
+                           true, wait_lim)) {
+            failed = 2;
+          } else {
+            issue_tile(smem + S::kOffV + st * S::kKVBytes, &tmap_v, rows_prev, &v_full[st]);
+            v_issued = tv + 1;
+          }
+        }
+        if (failed == 2 && !*abort_flag) {
+          record_error(v.err, HAM_DEVERR_TIMEOUT);
+          *abort_flag = 1;
+        }
       }
+      if (__shfl_sync(kFull, failed, 0)) break;
+#pragma unroll
+      for (int c = 0; c < S::kChunks; ++c) rows_prev[c] = rows_cur[c];
+    }
+    if (lane == 0) {
       // every copy this CTA issued lands before the CTA can exit
       thread_wait(q_full, 0u, abort_flag, false);
-      for (int t = max(0, issued - S::kStages); t < issued; ++t) {
-        thread_wait(&k_full[t % S::kStages], (uint32_t)(t / S::kStages) & 1u, abort_flag, false);
-        thread_wait(&v_full[t % S::kStages], (uint32_t)(t / S::kStages) & 1u, abort_flag, false);
-      }
+      for (int t = max(0, k_issued - S::kKStages); t < k_issued; ++t)
+        thread_wait(&k_full[t % S::kKStages], (uint32_t)(t / S::kKStages) & 1u, abort_flag,
+                    false);
+      for (int t = max(0, v_issued - S::kVStages); t < v_issued; ++t)
+        thread_wait(&v_full[t % S::kVStages], (uint32_t)(t / S::kVStages) & 1u, abort_flag,
+                    false);
     }
   } else if (warp == S::kMmaWarp) {
     // ------------------------------------------------------------ MMA issue (lane 0)
-    // Order per K/V tile t and Q tile q: O_q += P_q(t) V_t as soon as the softmax group has
-    // written P_q(t), then S_q(t+1) = Q_q K_(t+1)^T; the two Q tiles alternate, so the tensor
-    // cores work on one while the other's softmax runs.  A commit to s_full[q] therefore also
-    // covers the P V product before it (tcgen05 operations of one thread complete in order).
+    // Per K/V tile t and Q tile q: O_q += P_q(t) V_t as soon as the softmax group has written
+    // P_q(t) (A operand in tensor memory), then S_q(t + 1) = Q_q K_(t+1)^T over the same columns.
+    // tcgen05 operations of one thread run in issue order, so the scores never overwrite P before
+    // the product has read it, and a commit to s_full[q] also covers the P V product before it:
+    // the softmax group may rescale O_q and overwrite S_q once it has seen S_q(t + 1).  The two
+    // Q tiles alternate, so the tensor cores work on one while the other's softmax runs.
     constexpr uint32_t id_s = idesc_bf16(128, S::kTile, false);  // K-major Q and K
-    constexpr uint32_t id_o = idesc_bf16(128, D, true);          // K-major P, MN-major V
-    const uint32_t q_base = smem_u32(smem), p_base = smem_u32(smem + S::kOffP);
-    const uint32_t ring = smem_u32(smem + S::kOffRing);
+    constexpr uint32_t id_o = idesc_bf16(128, D, true);          // P from TMEM, MN-major V
+    const uint32_t q_base = smem_u32(smem);
     auto issue_s = [&](int q, int t) {
-      const uint32_t kt = ring + (uint32_t)((t % S::kStages) * 2 * S::kKVBytes);
+      const uint32_t kt = smem_u32(smem + S::kOffK + (t % S::kKStages) * S::kKVBytes);
 #pragma unroll
       for (int k = 0; k < D / 16; ++k) {
         const uint64_t a = smem_desc_sw128(
@@ -493,12 +549,12 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       }
     };
     auto issue_o = [&](int q, int t) {
-      const uint32_t vt = ring + (uint32_t)((t % S::kStages) * 2 * S::kKVBytes + S::kKVBytes);
+      const uint32_t vt = smem_u32(smem + S::kOffV + (t % S::kVStages) * S::kKVBytes);
 #pragma unroll
       for (int k = 0; k < S::kTile / 16; ++k) {
-        const uint64_t a = smem_desc_sw128(p_base + q * S::kPBytes + k * 32, 16, 1024);
         const uint64_t bv = smem_desc_sw128(vt + k * 2048, S::kHalfTileBytes, 1024);
-        tc_mma(tmem + 2 * S::kTile + q * D, a, bv, id_o, t > 0 || k > 0);
+        tc_mma_tmem_a(tmem + S::kOffO + q * D, tmem + q * S::kTile + k * 8, bv, id_o,
+                      t > 0 || k > 0);
       }
     };
     bool ok = warp_wait(q_full, 0u, abort_flag, wait_lim) &&
@@ -510,18 +566,19 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
           issue_s(q, 0);
           tc_commit(&s_full[q]);
         }
+      tc_commit(&k_empty[0]);
     }
     __syncwarp();
     for (int t = 0; ok && t < ntiles; ++t) {
-      const int st = t % S::kStages;
-      if (!warp_wait(&v_full[st], (uint32_t)(t / S::kStages) & 1u, abort_flag, wait_lim)) {
+      const int vs = t % S::kVStages;
+      if (!warp_wait(&v_full[vs], (uint32_t)(t / S::kVStages) & 1u, abort_flag, wait_lim)) {
         ok = false;
         break;
       }
       if (t == ntiles - 1 && kv_end < (t + 1) * S::kTile) {
         // slots >= kv_end get p = 0; zero their value rows so that stale bits never reach O
         const int z0 = kv_end - t * S::kTile, per_half = (S::kTile - z0) * 8;
-        uint8_t *vt = smem + S::kOffRing + st * 2 * S::kKVBytes + S::kKVBytes;
+        uint8_t *vt = smem + S::kOffV + vs * S::kKVBytes;
         for (int e = lane; e < S::kHalves * per_half; e += 32) {
           const int hh = e / per_half, r = e % per_half;
           *reinterpret_cast<uint4 *>(vt + hh * S::kHalfTileBytes + z0 * 128 + r * 16) =
@@ -530,7 +587,9 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
       }
-      for (int q = 0; q < 2 && ok; ++q) {
+      const int t1 = t + 1;
+      bool k_next = false;  // K tile t + 1 is in shared memory
+      for (int q = 0; q < 2; ++q) {
         if (t >= ntile[q]) continue;
         if (!warp_wait(&p_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
           ok = false;
@@ -539,15 +598,15 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         if (lane == 0) {
           tc_fence_after();
           issue_o(q, t);
-          if (t == ntile[q] - 1) tc_commit(&o_done[q]);
+          tc_commit(&pv_done[q]);
         }
-        if (t + 1 < ntile[q]) {
-          const int t1 = t + 1;
-          if (!warp_wait(&k_full[t1 % S::kStages], (uint32_t)(t1 / S::kStages) & 1u, abort_flag,
-                         wait_lim)) {
+        if (t1 < ntile[q]) {
+          if (!k_next && !warp_wait(&k_full[t1 % S::kKStages], (uint32_t)(t1 / S::kKStages) & 1u,
+                                    abort_flag, wait_lim)) {
             ok = false;
             break;
           }
+          k_next = true;
           if (lane == 0) {
             issue_s(q, t1);
             tc_commit(&s_full[q]);
@@ -556,7 +615,10 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         __syncwarp();
       }
       if (!ok) break;
-      if (lane == 0) tc_commit(&kv_empty[st]);  // K_t and V_t are free once these complete
+      if (lane == 0) {
+        tc_commit(&v_empty[vs]);                          // V_t is free once these complete
+        if (k_next) tc_commit(&k_empty[t1 % S::kKStages]);  // and K_(t+1)
+      }
       __syncwarp();
     }
     if (!ok && lane == 0 && !*abort_flag) {
@@ -575,13 +637,12 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     // so the row maximum and sum need no shuffles.
     const int q = warp >> 2, m = tid & 127;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-    const uint32_t t_s = tmem + lane_base + q * S::kTile;
-    const uint32_t t_o = tmem + lane_base + 2 * S::kTile + q * D;
+    const uint32_t t_s = tmem + lane_base + q * S::kTile;  // S_q, and P_q over its first half
+    const uint32_t t_o = tmem + lane_base + S::kOffO + q * D;
     const int j = qb0 + q * R + m / G;          // the row's index in the sequence's chunk
     const int lim = L + min(j, n - 1);          // last slot it attends (rows past n: not stored)
     const int lim_min = L + qb0 + q * R;        // smallest limit of the tile's stored rows
     const float sl2 = (float)(1.4426950408889634 / sqrt((double)D));  // 1/sqrt(d), log2(e)
-    uint8_t *prow = smem + S::kOffP + q * S::kPBytes + m * 128;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int t = 0; t < ntile[q]; ++t) {
@@ -590,26 +651,33 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         break;
       }
       tc_fence_after();
-      uint32_t sa[32], sb[32];
-      tmem_ld32(t_s, sa);
-      tmem_ld32(t_s + 32, sb);
-      tmem_wait_ld();
       float s[S::kTile];
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        s[c] = __uint_as_float(sa[c]);
-        s[c + 32] = __uint_as_float(sb[c]);
+      for (int c0 = 0; c0 < S::kTile; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld32(t_s + c0, r);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) s[c0 + c] = __uint_as_float(r[c]);
       }
+      tmem_wait_ld();
       const int tbase = t * S::kTile;
       if (tbase + S::kTile - 1 > lim_min) {  // the causal edge (and the chunk's end) in this tile
 #pragma unroll
         for (int c = 0; c < S::kTile; ++c)
           if (tbase + c > lim) s[c] = -INFINITY;
       }
-      float mx = s[0];
+      float mx;
+      {  // tree maximum
+        float r[32];
 #pragma unroll
-      for (int c = 1; c < S::kTile; ++c) mx = fmaxf(mx, s[c]);
-      mx *= sl2;
+        for (int c = 0; c < 32; ++c)
+          r[c] = fmaxf(fmaxf(s[c], s[c + 32]), fmaxf(s[c + 64], s[c + 96]));
+#pragma unroll
+        for (int w = 16; w > 0; w >>= 1)
+#pragma unroll
+          for (int c = 0; c < w; ++c) r[c] = fmaxf(r[c], r[c + w]);
+        mx = r[0] * sl2;
+      }
       // Running maximum in the exp2 domain, raised lazily: only when a score passes it by more
       // than kRescaleSlack (p then stays below 2^kRescaleSlack), so O is rarely rescaled.  The
       // first tile always raises it (slot 0 is attended by every row).
@@ -618,9 +686,30 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         alpha = ex2(m_run - mx);
         m_run = mx;
       }
+      // P (bf16 pairs) over the first 64 columns of S_q: 32 scores -> 16 columns at a time
+      float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
+#pragma unroll
+      for (int c0 = 0; c0 < S::kTile; c0 += 32) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int c = 0; c < 32; c += 4) {
+          const float p0 = ex2(fmaf(s[c0 + c], sl2, -m_run));
+          const float p1 = ex2(fmaf(s[c0 + c + 1], sl2, -m_run));
+          const float p2 = ex2(fmaf(s[c0 + c + 2], sl2, -m_run));
+          const float p3 = ex2(fmaf(s[c0 + c + 3], sl2, -m_run));
+          rs0 += p0;
+          rs1 += p1;
+          rs2 += p2;
+          rs3 += p3;
+          pk[c / 2] = pack_bf16x2(p0, p1);
+          pk[c / 2 + 1] = pack_bf16x2(p2, p3);
+        }
+        tmem_st16(t_s + c0 / 2, pk);
+      }
+      l_run = l_run * alpha + ((rs0 + rs1) + (rs2 + rs3));
       // S_q(t) completed after O_q's last product (in-order completion), and the next product
       // waits for p_full: O_q is stable here.
-      if (t > 0 && __any_sync(kFull, alpha != 1.f)) {
+      if (t > 0 && __any_sync(kFull, alpha != 1.f)) {  // some row of the warp raised its max
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t o[32];
@@ -630,30 +719,14 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
           for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
           tmem_st32(t_o + c0, o);
         }
-        tmem_wait_st();
       }
-      float rs = 0.f;
-      uint32_t pk[S::kTile / 2];
-#pragma unroll
-      for (int c = 0; c < S::kTile / 2; ++c) {
-        const float p0 = ex2(fmaf(s[2 * c], sl2, -m_run));
-        const float p1 = ex2(fmaf(s[2 * c + 1], sl2, -m_run));
-        rs += p0 + p1;
-        pk[c] = pack_bf16x2(p0, p1);
-      }
-      l_run = l_run * alpha + rs;
-      // P row m: 128 bytes in the 128-byte swizzle (K-major operand of the P V product)
-#pragma unroll
-      for (int c = 0; c < 8; ++c)
-        *reinterpret_cast<uint4 *>(prow + ((c ^ (m & 7)) << 4)) =
-            make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-      fence_proxy_async_smem();
+      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[q]);
     }
     if (ok && ntile[q] > 0) {
-      if (!warp_wait(&o_done[q], 0u, abort_flag, wait_lim)) {
+      if (!warp_wait(&pv_done[q], (uint32_t)(ntile[q] - 1) & 1u, abort_flag, wait_lim)) {
         ok = false;
       } else {
         tc_fence_after();
