@@ -301,21 +301,23 @@ struct TcShape {
   static constexpr int kHalves = D / 64;                     // 64-column halves of a row
   static constexpr int kHalfTileBytes = kTile * 128;         // one half of a K or V tile
   static constexpr int kKVBytes = kHalves * kHalfTileBytes;  // a K (or V) tile
-  static constexpr int kKStages = D == 128 ? 3 : 4;          // K tiles in flight
-  static constexpr int kVStages = D == 128 ? 2 : 4;          // V tiles in flight
+  static constexpr int kKStages = D == 128 ? 2 : 4;          // K tiles in flight
+  static constexpr int kVStages = D == 128 ? 3 : 4;          // V tiles in flight
   static constexpr int kQHalfBytes = 128 * 128;              // one half of a Q tile
   static constexpr int kQBytes = kHalves * kQHalfBytes;
   static constexpr int kOffK = 2 * kQBytes;                  // Q tiles at 0
   static constexpr int kOffV = kOffK + kKStages * kKVBytes;
   static constexpr int kOffBar = kOffV + kVStages * kKVBytes;
   // k_full, k_empty [kKStages]; v_full, v_empty [kVStages]; q_full; s_full, p_full,
-  // pv_done [2]; mma_done
-  static constexpr int kBars = 2 * kKStages + 2 * kVStages + 8;
+  // pv_done, turn [2]; mma_done
+  static constexpr int kBars = 2 * kKStages + 2 * kVStages + 10;
   static constexpr int kSmem = 1024 + kOffBar + kBars * 8 + 16;
   static constexpr uint32_t kTmemCols = 512;
   static constexpr int kOffO = 2 * kTile;                    // TMEM column of O_0
-  static constexpr int kProducerWarp = 8, kMmaWarp = 9;      // softmax: warps 0-3 and 4-7
-  static constexpr int kThreads = 10 * 32;
+  // softmax: warps 0-3 and 4-7; producers of Q and K (8) and of V (10); MMA issue (9).  Eleven
+  // warps cost the registers of twelve (granted in groups of four warps): 168 a thread.
+  static constexpr int kProducerWarp = 8, kMmaWarp = 9, kVProducerWarp = 10;
+  static constexpr int kThreads = 11 * 32;
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
   static_assert(kOffO + 2 * D <= (int)kTmemCols, "TMEM columns");
   static_assert(kSmem <= 227 * 1024, "shared memory");
@@ -375,7 +377,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   uint64_t *k_empty = k_full + S::kKStages, *v_full = k_empty + S::kKStages;
   uint64_t *v_empty = v_full + S::kVStages, *q_full = v_empty + S::kVStages;
   uint64_t *s_full = q_full + 1, *p_full = q_full + 3, *pv_done = q_full + 5;
-  uint64_t *mma_done = q_full + 7;
+  uint64_t *mma_done = q_full + 7, *turn = q_full + 8;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(k_full + S::kBars);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -393,6 +395,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       mbar_init(&s_full[q], 1);
       mbar_init(&p_full[q], 4);  // one arrival per warp of the softmax group
       mbar_init(&pv_done[q], 1);
+      mbar_init(&turn[q], 4);    // the other group's four warps have done their exponentials
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -411,13 +414,14 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   // ring and data waits: the launch's limit; draining in-flight work keeps the default 2 s
   const uint64_t wait_lim = data_wait_limit(v.wait_ns);
 
-  if (warp == S::kProducerWarp) {
-    // ------------------------------------------------------------ producer: TMA copies
-    // Q once; then per step t the K tile t and the V tile t - 1 (keys are needed a tile before
-    // values).  A chunk at or past kv_end is not copied: its rows are masked (K) or zeroed (V).
+  if (warp == S::kProducerWarp || warp == S::kVProducerWarp) {
+    // ------------------------------------------------------------ producers: TMA copies
+    // One warp streams Q and the K tiles, another the V tiles, each as far ahead as its ring
+    // allows (K tiles are needed a tile before V tiles and are released earlier).  A chunk at or
+    // past kv_end is not copied: its rows are masked (K) or zeroed (V).
+    const bool is_v = warp == S::kVProducerWarp;
     const uint64_t pol_kv = policy_evict_last();   // every query block of the sequence reads them
-    int k_issued = 0, v_issued = 0;
-    if (lane == 0) {
+    if (!is_v && lane == 0) {
       const uint64_t pol_q = policy_evict_first();
       const int nq = rows_q1 > 0 ? 2 : 1;
       mbar_arrive_tx(q_full, (uint32_t)(nq * S::kQBytes));
@@ -426,6 +430,10 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
           tma_load_4d(smem + q * S::kQBytes + hh * S::kQHalfBytes, &tmap_q, 0, hh, g * G,
                       (int)(row0 + qb0 + q * R), q_full, pol_q);
     }
+    const int stages = is_v ? S::kVStages : S::kKStages;
+    uint8_t *ring = smem + (is_v ? S::kOffV : S::kOffK);
+    uint64_t *full = is_v ? v_full : k_full, *empty = is_v ? v_empty : k_empty;
+    const CUtensorMap *map = is_v ? &tmap_v : &tmap_k;
     // Page-table entries of 32 chunks (4 tiles) at a time, one per lane, requested a batch
     // ahead: lane l holds the pool row of chunk base + l (-1: at or past kv_end; -2: a page
     // outside the pool).
@@ -443,88 +451,51 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     };
     constexpr int kTilesPerBatch = 32 / S::kChunks;
     int row = lookup(0), row_next = lookup(32);
-    int rows_prev[S::kChunks];
-#pragma unroll
-    for (int c = 0; c < S::kChunks; ++c) rows_prev[c] = -1;
-    // copies of one tile into `dst` (K or V), counted on `bar`
-    auto issue_tile = [&](uint8_t *dst, const CUtensorMap *map, const int (&rows)[S::kChunks],
-                          uint64_t *bar) {
-      int nck = 0;
-#pragma unroll
-      for (int c = 0; c < S::kChunks; ++c) nck += rows[c] >= 0;
-      mbar_arrive_tx(bar, (uint32_t)(nck * kChunkSlots * D * 2));
-#pragma unroll
-      for (int c = 0; c < S::kChunks; ++c) {
-        if (rows[c] < 0) continue;
-#pragma unroll
-        for (int hh = 0; hh < S::kHalves; ++hh)
-          tma_load_3d(dst + hh * S::kHalfTileBytes + c * kChunkSlots * 128, map, 0, hh, rows[c],
-                      bar, pol_kv);
+    int issued = 0;
+    for (int t = 0; t < ntiles; ++t) {
+      if (t > 0 && t % kTilesPerBatch == 0) {
+        row = row_next;
+        row_next = lookup((t / kTilesPerBatch + 1) * 32);
       }
-    };
-    for (int t = 0; t <= ntiles; ++t) {
-      int rows_cur[S::kChunks];
-      bool bad = false;
-#pragma unroll
-      for (int c = 0; c < S::kChunks; ++c) rows_cur[c] = -1;
-      if (t < ntiles) {
-        if (t > 0 && t % kTilesPerBatch == 0) {
-          row = row_next;
-          row_next = lookup((t / kTilesPerBatch + 1) * 32);
-        }
-#pragma unroll
-        for (int c = 0; c < S::kChunks; ++c) {
-          rows_cur[c] = __shfl_sync(kFull, row, (t % kTilesPerBatch) * S::kChunks + c);
-          bad |= rows_cur[c] == -2;
-        }
-      }
-      int failed = 0;
-      if (lane == 0) {
-        if (bad) {  // the plan validated the table; a page outside the pool ends the CTA
+      int my_row = __shfl_sync(kFull, row, ((t % kTilesPerBatch) * S::kChunks + lane) & 31);
+      if (lane >= S::kChunks) my_row = -1;
+      if (__any_sync(kFull, my_row == -2)) {  // the plan validated the table: this ends the CTA
+        if (lane == 0) {
           record_error(v.err, HAM_DEVERR_PAGE);
           *abort_flag = 1;
-          failed = 1;
         }
-        if (!failed && t < ntiles) {
-          const int st = t % S::kKStages;
-          if (t >= S::kKStages &&
-              !thread_wait(&k_empty[st], (uint32_t)((t / S::kKStages) - 1) & 1u, abort_flag,
-                           true, wait_lim)) {
-            failed = 2;
-          } else {
-            issue_tile(smem + S::kOffK + st * S::kKVBytes, &tmap_k, rows_cur, &k_full[st]);
-            k_issued = t + 1;
-          }
-        }
-        if (!failed && t >= 1) {
-          const int tv = t - 1, st = tv % S::kVStages;
-          if (tv >= S::kVStages &&
-              !thread_wait(&v_empty[st], (uint32_t)((tv / S::kVStages) - 1) & 1u, abort_flag,
-                           true, wait_lim)) {
-            failed = 2;
-          } else {
-            issue_tile(smem + S::kOffV + st * S::kKVBytes, &tmap_v, rows_prev, &v_full[st]);
-            v_issued = tv + 1;
-          }
-        }
-        if (failed == 2 && !*abort_flag) {
+        break;
+      }
+      const int st = t % stages;
+      int ok_wait = 1;
+      if (lane == 0 && t >= stages)
+        ok_wait = thread_wait(&empty[st], (uint32_t)((t / stages) - 1) & 1u, abort_flag, true,
+                              wait_lim);
+      if (!__shfl_sync(kFull, ok_wait, 0)) {
+        if (lane == 0 && !*abort_flag) {
           record_error(v.err, HAM_DEVERR_TIMEOUT);
           *abort_flag = 1;
         }
+        break;
       }
-      if (__shfl_sync(kFull, failed, 0)) break;
+      // lane 0 posts the byte count, then lane c issues chunk c's boxes, so that the warp has
+      // the tile's copies in flight at once
+      const uint32_t nck = __popc(__ballot_sync(kFull, my_row >= 0));
+      if (lane == 0) mbar_arrive_tx(&full[st], nck * (uint32_t)(kChunkSlots * D * 2));
+      __syncwarp();
+      if (my_row >= 0) {
 #pragma unroll
-      for (int c = 0; c < S::kChunks; ++c) rows_prev[c] = rows_cur[c];
+        for (int hh = 0; hh < S::kHalves; ++hh)
+          tma_load_3d(ring + st * S::kKVBytes + hh * S::kHalfTileBytes + lane * kChunkSlots * 128,
+                      map, 0, hh, my_row, &full[st], pol_kv);
+      }
+      issued = t + 1;
     }
     if (lane == 0) {
-      // every copy this CTA issued lands before the CTA can exit
-      thread_wait(q_full, 0u, abort_flag, false);
-      for (int t = max(0, k_issued - S::kKStages); t < k_issued; ++t)
-        thread_wait(&k_full[t % S::kKStages], (uint32_t)(t / S::kKStages) & 1u, abort_flag,
-                    false);
-      for (int t = max(0, v_issued - S::kVStages); t < v_issued; ++t)
-        thread_wait(&v_full[t % S::kVStages], (uint32_t)(t / S::kVStages) & 1u, abort_flag,
-                    false);
+      // every copy this warp issued lands before the CTA can exit
+      if (!is_v) thread_wait(q_full, 0u, abort_flag, false);
+      for (int t = max(0, issued - stages); t < issued; ++t)
+        thread_wait(&full[t % stages], (uint32_t)(t / stages) & 1u, abort_flag, false);
     }
   } else if (warp == S::kMmaWarp) {
     // ------------------------------------------------------------ MMA issue (lane 0)
@@ -686,6 +657,15 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         alpha = ex2(m_run - mx);
         m_run = mx;
       }
+      // The two groups take turns at their exponentials (tile t of group 0, then tile t of group
+      // 1, then tile t + 1 of group 0, ...), so that each has the special-function units to
+      // itself while the tensor cores work on the other Q tile.
+      const bool take_turn = q == 0 ? (t >= 1 && t - 1 < ntile[1]) : (t < ntile[0]);
+      if (take_turn && !warp_wait(&turn[q], (uint32_t)(q == 0 ? t - 1 : t) & 1u, abort_flag,
+                                  wait_lim)) {
+        ok = false;
+        break;
+      }
       // P (bf16 pairs) over the first 64 columns of S_q: 32 scores -> 16 columns at a time
       float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
 #pragma unroll
@@ -707,6 +687,8 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         tmem_st16(t_s + c0 / 2, pk);
       }
       l_run = l_run * alpha + ((rs0 + rs1) + (rs2 + rs3));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&turn[q ^ 1]);  // the other group's turn
       // S_q(t) completed after O_q's last product (in-order completion), and the next product
       // waits for p_full: O_q is stable here.
       if (t > 0 && __any_sync(kFull, alpha != 1.f)) {  // some row of the warp raised its max
