@@ -314,10 +314,11 @@ struct TcShape {
   static constexpr int kSmem = 1024 + kOffBar + kBars * 8 + 16;
   static constexpr uint32_t kTmemCols = 512;
   static constexpr int kOffO = 2 * kTile;                    // TMEM column of O_0
-  // softmax: warps 0-3 and 4-7; producers of Q and K (8) and of V (10); MMA issue (9).  Eleven
-  // warps cost the registers of twelve (granted in groups of four warps): 168 a thread.
-  static constexpr int kProducerWarp = 8, kMmaWarp = 9, kVProducerWarp = 10;
-  static constexpr int kThreads = 11 * 32;
+  // softmax: warps 0-3 and 4-7; producers of Q and K (8) and of V (10); MMA issue for Q tile 0
+  // (9) and Q tile 1 (11).  One thread issues a 128 x 128 x 16 product about every 125 cycles
+  // (measured), half the tensor rate, so each Q tile has its own issuing warp.
+  static constexpr int kProducerWarp = 8, kMmaWarp = 9, kVProducerWarp = 10, kMmaWarp1 = 11;
+  static constexpr int kThreads = 12 * 32;
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
   static_assert(kOffO + 2 * D <= (int)kTmemCols, "TMEM columns");
   static_assert(kSmem <= 227 * 1024, "shared memory");
@@ -382,13 +383,14 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
+    // a stage is free once both MMA warps' products that read it have completed
     for (int s = 0; s < S::kKStages; ++s) {
       mbar_init(&k_full[s], 1);
-      mbar_init(&k_empty[s], 1);
+      mbar_init(&k_empty[s], 2);
     }
     for (int s = 0; s < S::kVStages; ++s) {
       mbar_init(&v_full[s], 1);
-      mbar_init(&v_empty[s], 1);
+      mbar_init(&v_empty[s], 2);
     }
     mbar_init(q_full, 1);
     for (int q = 0; q < 2; ++q) {
@@ -397,7 +399,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       mbar_init(&pv_done[q], 1);
       mbar_init(&turn[q], 4);    // the other group's four warps have done their exponentials
     }
-    mbar_init(mma_done, 1);
+    mbar_init(mma_done, 2);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -497,29 +499,35 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       for (int t = max(0, issued - stages); t < issued; ++t)
         thread_wait(&full[t % stages], (uint32_t)(t / stages) & 1u, abort_flag, false);
     }
-  } else if (warp == S::kMmaWarp) {
-    // ------------------------------------------------------------ MMA issue (lane 0)
-    // Per K/V tile t and Q tile q: O_q += P_q(t) V_t as soon as the softmax group has written
+  } else if (warp == S::kMmaWarp || warp == S::kMmaWarp1) {
+    // ------------------------------------------------------------ MMA issue (lane 0), one warp
+    // per Q tile.  Per K/V tile t: O_q += P_q(t) V_t as soon as the softmax group has written
     // P_q(t) (A operand in tensor memory), then S_q(t + 1) = Q_q K_(t+1)^T over the same columns.
     // tcgen05 operations of one thread run in issue order, so the scores never overwrite P before
     // the product has read it, and a commit to s_full[q] also covers the P V product before it:
-    // the softmax group may rescale O_q and overwrite S_q once it has seen S_q(t + 1).  The two
-    // Q tiles alternate, so the tensor cores work on one while the other's softmax runs.
+    // the softmax group may rescale O_q and overwrite S_q once it has seen S_q(t + 1).
+    // A K or V stage is released by a commit of each MMA warp; a tile that only one Q tile
+    // reaches is released twice by that warp.
+    const int q = warp == S::kMmaWarp ? 0 : 1;
+    const int nt = ntile[q], other = ntile[q ^ 1];
     constexpr uint32_t id_s = idesc_bf16(128, S::kTile, false);  // K-major Q and K
     constexpr uint32_t id_o = idesc_bf16(128, D, true);          // P from TMEM, MN-major V
-    const uint32_t q_base = smem_u32(smem);
-    auto issue_s = [&](int q, int t) {
+    const uint32_t q_base = smem_u32(smem) + q * S::kQBytes;
+    auto issue_s = [&](int t) {
       const uint32_t kt = smem_u32(smem + S::kOffK + (t % S::kKStages) * S::kKVBytes);
 #pragma unroll
       for (int k = 0; k < D / 16; ++k) {
-        const uint64_t a = smem_desc_sw128(
-            q_base + q * S::kQBytes + (k >> 2) * S::kQHalfBytes + (k & 3) * 32, 16, 1024);
+        const uint64_t a =
+            smem_desc_sw128(q_base + (k >> 2) * S::kQHalfBytes + (k & 3) * 32, 16, 1024);
         const uint64_t bk =
             smem_desc_sw128(kt + (k >> 2) * S::kHalfTileBytes + (k & 3) * 32, 16, 1024);
         tc_mma(tmem + q * S::kTile, a, bk, id_s, k > 0);
       }
+      tc_commit(&s_full[q]);
+      tc_commit(&k_empty[t % S::kKStages]);
+      if (t >= other) tc_commit(&k_empty[t % S::kKStages]);
     };
-    auto issue_o = [&](int q, int t) {
+    auto issue_o = [&](int t) {
       const uint32_t vt = smem_u32(smem + S::kOffV + (t % S::kVStages) * S::kKVBytes);
 #pragma unroll
       for (int k = 0; k < S::kTile / 16; ++k) {
@@ -527,20 +535,21 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         tc_mma_tmem_a(tmem + S::kOffO + q * D, tmem + q * S::kTile + k * 8, bv, id_o,
                       t > 0 || k > 0);
       }
+      tc_commit(&pv_done[q]);
+      tc_commit(&v_empty[t % S::kVStages]);
+      if (t >= other) tc_commit(&v_empty[t % S::kVStages]);
     };
-    bool ok = warp_wait(q_full, 0u, abort_flag, wait_lim) &&
-              warp_wait(&k_full[0], 0u, abort_flag, wait_lim);
-    if (ok && lane == 0) {
-      tc_fence_after();
-      for (int q = 0; q < 2; ++q)
-        if (ntile[q] > 0) {
-          issue_s(q, 0);
-          tc_commit(&s_full[q]);
-        }
-      tc_commit(&k_empty[0]);
+    bool ok = true;
+    if (nt > 0) {
+      ok = warp_wait(q_full, 0u, abort_flag, wait_lim) &&
+           warp_wait(&k_full[0], 0u, abort_flag, wait_lim);
+      if (ok && lane == 0) {
+        tc_fence_after();
+        issue_s(0);
+      }
+      __syncwarp();
     }
-    __syncwarp();
-    for (int t = 0; ok && t < ntiles; ++t) {
+    for (int t = 0; ok && t < nt; ++t) {
       const int vs = t % S::kVStages;
       if (!warp_wait(&v_full[vs], (uint32_t)(t / S::kVStages) & 1u, abort_flag, wait_lim)) {
         ok = false;
@@ -548,6 +557,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       }
       if (t == ntiles - 1 && kv_end < (t + 1) * S::kTile) {
         // slots >= kv_end get p = 0; zero their value rows so that stale bits never reach O
+        // (both MMA warps may write the same zeros)
         const int z0 = kv_end - t * S::kTile, per_half = (S::kTile - z0) * 8;
         uint8_t *vt = smem + S::kOffV + vs * S::kKVBytes;
         for (int e = lane; e < S::kHalves * per_half; e += 32) {
@@ -558,37 +568,22 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
       }
+      if (!warp_wait(&p_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
+        ok = false;
+        break;
+      }
+      if (lane == 0) {
+        tc_fence_after();
+        issue_o(t);
+      }
       const int t1 = t + 1;
-      bool k_next = false;  // K tile t + 1 is in shared memory
-      for (int q = 0; q < 2; ++q) {
-        if (t >= ntile[q]) continue;
-        if (!warp_wait(&p_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
+      if (t1 < nt) {
+        if (!warp_wait(&k_full[t1 % S::kKStages], (uint32_t)(t1 / S::kKStages) & 1u, abort_flag,
+                       wait_lim)) {
           ok = false;
           break;
         }
-        if (lane == 0) {
-          tc_fence_after();
-          issue_o(q, t);
-          tc_commit(&pv_done[q]);
-        }
-        if (t1 < ntile[q]) {
-          if (!k_next && !warp_wait(&k_full[t1 % S::kKStages], (uint32_t)(t1 / S::kKStages) & 1u,
-                                    abort_flag, wait_lim)) {
-            ok = false;
-            break;
-          }
-          k_next = true;
-          if (lane == 0) {
-            issue_s(q, t1);
-            tc_commit(&s_full[q]);
-          }
-        }
-        __syncwarp();
-      }
-      if (!ok) break;
-      if (lane == 0) {
-        tc_commit(&v_empty[vs]);                          // V_t is free once these complete
-        if (k_next) tc_commit(&k_empty[t1 % S::kKStages]);  // and K_(t+1)
+        if (lane == 0) issue_s(t1);
       }
       __syncwarp();
     }
