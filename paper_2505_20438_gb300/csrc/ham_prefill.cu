@@ -290,35 +290,38 @@ __global__ void __launch_bounds__(kRopeThreads) prefill_rope_kernel(PrefillView 
 // ------------------------------------------------------------------------------------
 // A CTA covers one KV head and two Q tiles of 128 rows each; a row is a (query row, head)
 // pair, m = (row - first row of the tile) * G + head within the group, and sits in TMEM lane m.
-// TMEM columns: S_0, S_1 (128 fp32 scores of the current 128-slot K tile; the softmax writes
-// the bf16 probabilities P over the first 64 columns of its S, where the P V product reads
-// them), then O_0, O_1 (head_dim fp32).  Reading P from tensor memory and 128-slot tiles keep
-// the shared-memory traffic of the products at 2 operand bytes per 64 FLOP.
+// Tensor-memory columns per Q tile q: S_q (64 fp32 scores of the current 64-slot K tile), P_q
+// (the bf16 probabilities of the tile as pairs: the A operand of O += P V) and O_q (head_dim
+// fp32).  The products of a Q tile are issued by two warps, one for S = Q K^T and one for
+// O += P V: one thread issues a tcgen05.mma only about every 125 cycles (measured on GB300),
+// so a single issuer would keep the tensor cores half idle.  Because P has columns of its own,
+// S_q(t + 1) is computed while the softmax group still works on tile t.
 template <int D>
 struct TcShape {
-  static constexpr int kTile = 128;                          // slots per K/V tile
+  static constexpr int kTile = 64;                           // slots per K/V tile
   static constexpr int kChunks = kTile / kChunkSlots;        // 16-slot TMA chunks per tile
   static constexpr int kHalves = D / 64;                     // 64-column halves of a row
   static constexpr int kHalfTileBytes = kTile * 128;         // one half of a K or V tile
   static constexpr int kKVBytes = kHalves * kHalfTileBytes;  // a K (or V) tile
-  static constexpr int kKStages = D == 128 ? 2 : 4;          // K tiles in flight
-  static constexpr int kVStages = D == 128 ? 3 : 4;          // V tiles in flight
+  static constexpr int kKStages = D == 128 ? 4 : 8;          // K tiles in flight
+  static constexpr int kVStages = D == 128 ? 5 : 8;          // V tiles in flight
   static constexpr int kQHalfBytes = 128 * 128;              // one half of a Q tile
   static constexpr int kQBytes = kHalves * kQHalfBytes;
   static constexpr int kOffK = 2 * kQBytes;                  // Q tiles at 0
   static constexpr int kOffV = kOffK + kKStages * kKVBytes;
   static constexpr int kOffBar = kOffV + kVStages * kKVBytes;
-  // k_full, k_empty [kKStages]; v_full, v_empty [kVStages]; q_full; s_full, p_full,
-  // pv_done, turn [2]; mma_done
+  // k_full, k_empty [kKStages]; v_full, v_empty [kVStages]; q_full; s_full, s_free, p_full,
+  // pv_done [2]; mma_done
   static constexpr int kBars = 2 * kKStages + 2 * kVStages + 10;
   static constexpr int kSmem = 1024 + kOffBar + kBars * 8 + 16;
   static constexpr uint32_t kTmemCols = 512;
-  static constexpr int kOffO = 2 * kTile;                    // TMEM column of O_0
-  // softmax: warps 0-3 and 4-7; producers of Q and K (8) and of V (10); MMA issue for Q tile 0
-  // (9) and Q tile 1 (11).  One thread issues a 128 x 128 x 16 product about every 125 cycles
-  // (measured), half the tensor rate, so each Q tile has its own issuing warp.
-  static constexpr int kProducerWarp = 8, kMmaWarp = 9, kVProducerWarp = 10, kMmaWarp1 = 11;
-  static constexpr int kThreads = 12 * 32;
+  static constexpr int kOffP = 2 * kTile;                    // TMEM column of P_0 (S_0 at 0)
+  static constexpr int kOffO = kOffP + kTile;                // TMEM column of O_0
+  // softmax: warps 0-3 (Q tile 0) and 4-7 (Q tile 1); TMA producers of Q and K (8) and of V
+  // (10); MMA issue of S_0 (9), S_1 (11), O_0 (12), O_1 (13).
+  static constexpr int kProducerWarp = 8, kVProducerWarp = 10;
+  static constexpr int kSWarp0 = 9, kSWarp1 = 11, kOWarp0 = 12, kOWarp1 = 13;
+  static constexpr int kThreads = 14 * 32;
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
   static_assert(kOffO + 2 * D <= (int)kTmemCols, "TMEM columns");
   static_assert(kSmem <= 227 * 1024, "shared memory");
@@ -343,7 +346,7 @@ __device__ __forceinline__ void store_row32(OutT *dst, const uint32_t (&o)[32], 
   }
 }
 
-// One CTA per SM (shared memory and 512 TMEM columns at head_dim 128).
+// One CTA per SM (shared memory and 512 TMEM columns).
 template <int D, typename OutT>
 __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap tmap_q,
@@ -377,13 +380,13 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   uint64_t *k_full = reinterpret_cast<uint64_t *>(smem + S::kOffBar);
   uint64_t *k_empty = k_full + S::kKStages, *v_full = k_empty + S::kKStages;
   uint64_t *v_empty = v_full + S::kVStages, *q_full = v_empty + S::kVStages;
-  uint64_t *s_full = q_full + 1, *p_full = q_full + 3, *pv_done = q_full + 5;
-  uint64_t *mma_done = q_full + 7, *turn = q_full + 8;
+  uint64_t *s_full = q_full + 1, *s_free = q_full + 3, *p_full = q_full + 5;
+  uint64_t *pv_done = q_full + 7, *mma_done = q_full + 9;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(k_full + S::kBars);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
-    // a stage is free once both MMA warps' products that read it have completed
+    // a stage is free once the products of both Q tiles that read it have completed
     for (int s = 0; s < S::kKStages; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&k_empty[s], 2);
@@ -395,11 +398,11 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     mbar_init(q_full, 1);
     for (int q = 0; q < 2; ++q) {
       mbar_init(&s_full[q], 1);
-      mbar_init(&p_full[q], 4);  // one arrival per warp of the softmax group
+      mbar_init(&s_free[q], 4);  // the softmax group has read S_q (one arrival per warp)
+      mbar_init(&p_full[q], 4);  // ... and written P_q
       mbar_init(&pv_done[q], 1);
-      mbar_init(&turn[q], 4);    // the other group's four warps have done their exponentials
     }
-    mbar_init(mma_done, 2);
+    mbar_init(mma_done, 4);      // the four MMA warps
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -408,7 +411,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     prefetch_tensormap(&tmap_k);
     prefetch_tensormap(&tmap_v);
   }
-  if (warp == S::kMmaWarp) tmem_alloc<S::kTmemCols>(tmem_slot);
+  if (warp == S::kSWarp0) tmem_alloc<S::kTmemCols>(tmem_slot);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -499,93 +502,86 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       for (int t = max(0, issued - stages); t < issued; ++t)
         thread_wait(&full[t % stages], (uint32_t)(t / stages) & 1u, abort_flag, false);
     }
-  } else if (warp == S::kMmaWarp || warp == S::kMmaWarp1) {
-    // ------------------------------------------------------------ MMA issue (lane 0), one warp
-    // per Q tile.  Per K/V tile t: O_q += P_q(t) V_t as soon as the softmax group has written
-    // P_q(t) (A operand in tensor memory), then S_q(t + 1) = Q_q K_(t+1)^T over the same columns.
-    // tcgen05 operations of one thread run in issue order, so the scores never overwrite P before
-    // the product has read it, and a commit to s_full[q] also covers the P V product before it:
-    // the softmax group may rescale O_q and overwrite S_q once it has seen S_q(t + 1).
-    // A K or V stage is released by a commit of each MMA warp; a tile that only one Q tile
-    // reaches is released twice by that warp.
-    const int q = warp == S::kMmaWarp ? 0 : 1;
+  } else if (warp == S::kSWarp0 || warp == S::kSWarp1 || warp == S::kOWarp0 ||
+             warp == S::kOWarp1) {
+    // ------------------------------------------------------------ MMA issue (lane 0)
+    // S warp of Q tile q: S_q(t) = Q_q K_t^T once the softmax group has read S_q(t - 1) into
+    // registers (s_free) and K_t has landed.  O warp: O_q += P_q(t) V_t once the group has
+    // written P_q(t) (p_full) and V_t has landed; the group waits for pv_done before it writes
+    // the next P or rescales O.  A K or V stage is released by a commit for each Q tile that
+    // reads it; a tile that only one Q tile reaches is released twice by that tile's warp.
+    const bool is_o = warp == S::kOWarp0 || warp == S::kOWarp1;
+    const int q = (warp == S::kSWarp0 || warp == S::kOWarp0) ? 0 : 1;
     const int nt = ntile[q], other = ntile[q ^ 1];
-    constexpr uint32_t id_s = idesc_bf16(128, S::kTile, false);  // K-major Q and K
-    constexpr uint32_t id_o = idesc_bf16(128, D, true);          // P from TMEM, MN-major V
-    const uint32_t q_base = smem_u32(smem) + q * S::kQBytes;
-    auto issue_s = [&](int t) {
-      const uint32_t kt = smem_u32(smem + S::kOffK + (t % S::kKStages) * S::kKVBytes);
-#pragma unroll
-      for (int k = 0; k < D / 16; ++k) {
-        const uint64_t a =
-            smem_desc_sw128(q_base + (k >> 2) * S::kQHalfBytes + (k & 3) * 32, 16, 1024);
-        const uint64_t bk =
-            smem_desc_sw128(kt + (k >> 2) * S::kHalfTileBytes + (k & 3) * 32, 16, 1024);
-        tc_mma(tmem + q * S::kTile, a, bk, id_s, k > 0);
-      }
-      tc_commit(&s_full[q]);
-      tc_commit(&k_empty[t % S::kKStages]);
-      if (t >= other) tc_commit(&k_empty[t % S::kKStages]);
-    };
-    auto issue_o = [&](int t) {
-      const uint32_t vt = smem_u32(smem + S::kOffV + (t % S::kVStages) * S::kKVBytes);
-#pragma unroll
-      for (int k = 0; k < S::kTile / 16; ++k) {
-        const uint64_t bv = smem_desc_sw128(vt + k * 2048, S::kHalfTileBytes, 1024);
-        tc_mma_tmem_a(tmem + S::kOffO + q * D, tmem + q * S::kTile + k * 8, bv, id_o,
-                      t > 0 || k > 0);
-      }
-      tc_commit(&pv_done[q]);
-      tc_commit(&v_empty[t % S::kVStages]);
-      if (t >= other) tc_commit(&v_empty[t % S::kVStages]);
-    };
     bool ok = true;
-    if (nt > 0) {
-      ok = warp_wait(q_full, 0u, abort_flag, wait_lim) &&
-           warp_wait(&k_full[0], 0u, abort_flag, wait_lim);
-      if (ok && lane == 0) {
-        tc_fence_after();
-        issue_s(0);
-      }
-      __syncwarp();
-    }
-    for (int t = 0; ok && t < nt; ++t) {
-      const int vs = t % S::kVStages;
-      if (!warp_wait(&v_full[vs], (uint32_t)(t / S::kVStages) & 1u, abort_flag, wait_lim)) {
-        ok = false;
-        break;
-      }
-      if (t == ntiles - 1 && kv_end < (t + 1) * S::kTile) {
-        // slots >= kv_end get p = 0; zero their value rows so that stale bits never reach O
-        // (both MMA warps may write the same zeros)
-        const int z0 = kv_end - t * S::kTile, per_half = (S::kTile - z0) * 8;
-        uint8_t *vt = smem + S::kOffV + vs * S::kKVBytes;
-        for (int e = lane; e < S::kHalves * per_half; e += 32) {
-          const int hh = e / per_half, r = e % per_half;
-          *reinterpret_cast<uint4 *>(vt + hh * S::kHalfTileBytes + z0 * 128 + r * 16) =
-              make_uint4(0u, 0u, 0u, 0u);
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-      }
-      if (!warp_wait(&p_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
-        ok = false;
-        break;
-      }
-      if (lane == 0) {
-        tc_fence_after();
-        issue_o(t);
-      }
-      const int t1 = t + 1;
-      if (t1 < nt) {
-        if (!warp_wait(&k_full[t1 % S::kKStages], (uint32_t)(t1 / S::kKStages) & 1u, abort_flag,
-                       wait_lim)) {
+    if (!is_o) {
+      constexpr uint32_t id_s = idesc_bf16(128, S::kTile, false);  // K-major Q and K
+      const uint32_t q_base = smem_u32(smem) + q * S::kQBytes;
+      if (nt > 0) ok = warp_wait(q_full, 0u, abort_flag, wait_lim);
+      for (int t = 0; ok && t < nt; ++t) {
+        const int ks = t % S::kKStages;
+        if ((t > 0 && !warp_wait(&s_free[q], (uint32_t)(t - 1) & 1u, abort_flag, wait_lim)) ||
+            !warp_wait(&k_full[ks], (uint32_t)(t / S::kKStages) & 1u, abort_flag, wait_lim)) {
           ok = false;
           break;
         }
-        if (lane == 0) issue_s(t1);
+        if (lane == 0) {
+          tc_fence_after();
+          const uint32_t kt = smem_u32(smem + S::kOffK + ks * S::kKVBytes);
+#pragma unroll
+          for (int k = 0; k < D / 16; ++k) {
+            const uint64_t a =
+                smem_desc_sw128(q_base + (k >> 2) * S::kQHalfBytes + (k & 3) * 32, 16, 1024);
+            const uint64_t bk =
+                smem_desc_sw128(kt + (k >> 2) * S::kHalfTileBytes + (k & 3) * 32, 16, 1024);
+            tc_mma(tmem + q * S::kTile, a, bk, id_s, k > 0);
+          }
+          tc_commit(&s_full[q]);
+          tc_commit(&k_empty[ks]);
+          if (t >= other) tc_commit(&k_empty[ks]);
+        }
+        __syncwarp();
       }
-      __syncwarp();
+    } else {
+      constexpr uint32_t id_o = idesc_bf16(128, D, true);  // P from TMEM, MN-major V
+      for (int t = 0; ok && t < nt; ++t) {
+        const int vs = t % S::kVStages;
+        if (!warp_wait(&v_full[vs], (uint32_t)(t / S::kVStages) & 1u, abort_flag, wait_lim)) {
+          ok = false;
+          break;
+        }
+        if (t == ntiles - 1 && kv_end < (t + 1) * S::kTile) {
+          // slots >= kv_end get p = 0; zero their value rows so that stale bits never reach O
+          // (both O warps may write the same zeros)
+          const int z0 = kv_end - t * S::kTile, per_half = (S::kTile - z0) * 8;
+          uint8_t *vt = smem + S::kOffV + vs * S::kKVBytes;
+          for (int e = lane; e < S::kHalves * per_half; e += 32) {
+            const int hh = e / per_half, r = e % per_half;
+            *reinterpret_cast<uint4 *>(vt + hh * S::kHalfTileBytes + z0 * 128 + r * 16) =
+                make_uint4(0u, 0u, 0u, 0u);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+        }
+        if (!warp_wait(&p_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          tc_fence_after();
+          const uint32_t vt = smem_u32(smem + S::kOffV + vs * S::kKVBytes);
+#pragma unroll
+          for (int k = 0; k < S::kTile / 16; ++k) {
+            const uint64_t bv = smem_desc_sw128(vt + k * 2048, S::kHalfTileBytes, 1024);
+            tc_mma_tmem_a(tmem + S::kOffO + q * D, tmem + S::kOffP + q * (S::kTile / 2) + k * 8,
+                          bv, id_o, t > 0 || k > 0);
+          }
+          tc_commit(&pv_done[q]);
+          tc_commit(&v_empty[vs]);
+          if (t >= other) tc_commit(&v_empty[vs]);
+        }
+        __syncwarp();
+      }
     }
     if (!ok && lane == 0 && !*abort_flag) {
       record_error(v.err, HAM_DEVERR_TIMEOUT);
@@ -603,7 +599,8 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     // so the row maximum and sum need no shuffles.
     const int q = warp >> 2, m = tid & 127;
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-    const uint32_t t_s = tmem + lane_base + q * S::kTile;  // S_q, and P_q over its first half
+    const uint32_t t_s = tmem + lane_base + q * S::kTile;
+    const uint32_t t_p = tmem + lane_base + S::kOffP + q * (S::kTile / 2);
     const uint32_t t_o = tmem + lane_base + S::kOffO + q * D;
     const int j = qb0 + q * R + m / G;          // the row's index in the sequence's chunk
     const int lim = L + min(j, n - 1);          // last slot it attends (rows past n: not stored)
@@ -626,6 +623,9 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         for (int c = 0; c < 32; ++c) s[c0 + c] = __uint_as_float(r[c]);
       }
       tmem_wait_ld();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[q]);  // the next scores may overwrite S_q
       const int tbase = t * S::kTile;
       if (tbase + S::kTile - 1 > lim_min) {  // the causal edge (and the chunk's end) in this tile
 #pragma unroll
@@ -634,12 +634,12 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       }
       float mx;
       {  // tree maximum
-        float r[32];
+        float r[16];
 #pragma unroll
-        for (int c = 0; c < 32; ++c)
-          r[c] = fmaxf(fmaxf(s[c], s[c + 32]), fmaxf(s[c + 64], s[c + 96]));
+        for (int c = 0; c < 16; ++c)
+          r[c] = fmaxf(fmaxf(s[c], s[c + 16]), fmaxf(s[c + 32], s[c + 48]));
 #pragma unroll
-        for (int w = 16; w > 0; w >>= 1)
+        for (int w = 8; w > 0; w >>= 1)
 #pragma unroll
           for (int c = 0; c < w; ++c) r[c] = fmaxf(r[c], r[c + w]);
         mx = r[0] * sl2;
@@ -652,51 +652,42 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         alpha = ex2(m_run - mx);
         m_run = mx;
       }
-      // The two groups take turns at their exponentials (tile t of group 0, then tile t of group
-      // 1, then tile t + 1 of group 0, ...), so that each has the special-function units to
-      // itself while the tensor cores work on the other Q tile.
-      const bool take_turn = q == 0 ? (t >= 1 && t - 1 < ntile[1]) : (t < ntile[0]);
-      if (take_turn && !warp_wait(&turn[q], (uint32_t)(q == 0 ? t - 1 : t) & 1u, abort_flag,
-                                  wait_lim)) {
-        ok = false;
-        break;
-      }
-      // P (bf16 pairs) over the first 64 columns of S_q: 32 scores -> 16 columns at a time
+      uint32_t pk[S::kTile / 2];
       float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
 #pragma unroll
-      for (int c0 = 0; c0 < S::kTile; c0 += 32) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int c = 0; c < 32; c += 4) {
-          const float p0 = ex2(fmaf(s[c0 + c], sl2, -m_run));
-          const float p1 = ex2(fmaf(s[c0 + c + 1], sl2, -m_run));
-          const float p2 = ex2(fmaf(s[c0 + c + 2], sl2, -m_run));
-          const float p3 = ex2(fmaf(s[c0 + c + 3], sl2, -m_run));
-          rs0 += p0;
-          rs1 += p1;
-          rs2 += p2;
-          rs3 += p3;
-          pk[c / 2] = pack_bf16x2(p0, p1);
-          pk[c / 2 + 1] = pack_bf16x2(p2, p3);
-        }
-        tmem_st16(t_s + c0 / 2, pk);
+      for (int c = 0; c < S::kTile; c += 4) {
+        const float p0 = ex2(fmaf(s[c], sl2, -m_run));
+        const float p1 = ex2(fmaf(s[c + 1], sl2, -m_run));
+        const float p2 = ex2(fmaf(s[c + 2], sl2, -m_run));
+        const float p3 = ex2(fmaf(s[c + 3], sl2, -m_run));
+        rs0 += p0;
+        rs1 += p1;
+        rs2 += p2;
+        rs3 += p3;
+        pk[c / 2] = pack_bf16x2(p0, p1);
+        pk[c / 2 + 1] = pack_bf16x2(p2, p3);
       }
       l_run = l_run * alpha + ((rs0 + rs1) + (rs2 + rs3));
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&turn[q ^ 1]);  // the other group's turn
-      // S_q(t) completed after O_q's last product (in-order completion), and the next product
-      // waits for p_full: O_q is stable here.
-      if (t > 0 && __any_sync(kFull, alpha != 1.f)) {  // some row of the warp raised its max
+      // O_q and P_q are free once the previous product has completed
+      if (t > 0) {
+        if (!warp_wait(&pv_done[q], (uint32_t)(t - 1) & 1u, abort_flag, wait_lim)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (__any_sync(kFull, alpha != 1.f)) {  // rescale O (some row of the warp raised its max)
 #pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
-          uint32_t o[32];
-          tmem_ld32(t_o + c0, o);
-          tmem_wait_ld();
+          for (int c0 = 0; c0 < D; c0 += 32) {
+            uint32_t o[32];
+            tmem_ld32(t_o + c0, o);
+            tmem_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-          tmem_st32(t_o + c0, o);
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+            tmem_st32(t_o + c0, o);
+          }
         }
       }
+      tmem_st32(t_p, pk);  // P_q: the tile's 64 probabilities as 32 bf16 pairs
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -708,7 +699,6 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       } else {
         tc_fence_after();
         const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-        const bool stored = j < n;
         OutT *orow = static_cast<OutT *>(v.out) +
                      ((row0 + j) * Hq + g * G + m % G) * (int64_t)D;
 #pragma unroll
@@ -716,7 +706,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
           uint32_t o[32];
           tmem_ld32(t_o + c0, o);
           tmem_wait_ld();
-          if (stored) store_row32<OutT>(orow + c0, o, inv);
+          if (j < n) store_row32<OutT>(orow + c0, o, inv);
         }
       }
     }
@@ -728,7 +718,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   // all tensor-memory reads and MMAs are done: free the columns
   tc_fence_before();
   __syncthreads();
-  if (warp == S::kMmaWarp) {
+  if (warp == S::kSWarp0) {
     tc_fence_after();
     tmem_dealloc<S::kTmemCols>(tmem);
   }
