@@ -1143,9 +1143,10 @@ def run_embed(args, w):
         "sequences_per_s": round(value * B, 1),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
-                     "kernel": ("fuse_kernel (gather) + cuBLAS output GEMM + finish_kernel"
-                                if w.vocab else "cuBLAS QKV GEMM + fuse_kernel + cuBLAS "
-                                "output GEMM + finish_kernel"),
+                     "kernel": ("fuse_kernel (gather) + gemm_xwt_kernel (output projection) "
+                                "+ finish_kernel" if w.vocab else
+                                "gemm_xwt_kernel (Q/K/V projection) + fuse_kernel + "
+                                "gemm_xwt_kernel (output projection) + finish_kernel"),
                      "avg_launch_us": round(call_us, 3),
                      "algorithmic_bytes_per_launch": int(nbytes),
                      "peak_source": peak_src,

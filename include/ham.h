@@ -387,9 +387,9 @@ int ham_decode_attn_noalloc(const ham_attn_args *args, void *stream);
  *   per head h: o_h = sum_i softmax_i(q_h . k_{i,h} / sqrt(head_dim)) v_{i,h},   out_b = W_o o.
  * Weights are bf16 [out][in] row-major (y = W x); accumulation is fp32, o and out are
  * rounded to bf16 (o reaches the output projection as a hi + lo pair of bf16 values, about
- * 16 bits).  The handle owns copies of the weights and all workspace; the dense projections
- * run as cuBLAS GEMMs, the fusion (mean query, position terms, softmax, bypass) in this
- * library's kernels.                                                                      */
+ * 16 bits).  The handle owns copies of the weights (pre-tiled for the projection kernel) and
+ * all workspace; the dense projections (tcgen05 tensor-core products that stream the weights)
+ * and the fusion (mean query, position terms, softmax, bypass) run in this library's kernels. */
 typedef struct ham_embedder ham_embedder; /* opaque handle: weights and workspace */
 
 typedef struct ham_embed_config {
@@ -401,7 +401,7 @@ typedef struct ham_embed_config {
 
 /* Allocate an embedder and copy its weights (device bf16): wq, wk, wv, wo [H][H]; pos
  * [max_patch][H].  Host errors: HAM_EINVAL (bad config, NULL or unaligned pointer),
- * HAM_ENOMEM, HAM_ECUDA (including a cuBLAS failure). */
+ * HAM_ENOMEM, HAM_ECUDA. */
 int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *wk,
                        const void *wv, const void *wo, const void *pos, ham_embedder **out);
 int ham_embedder_free(ham_embedder *e);

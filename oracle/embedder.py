@@ -42,8 +42,10 @@ def softmax(s: np.ndarray) -> np.ndarray:
     return e / np.sum(e)
 
 
-def embed(x_bits, offsets, wq_bits, wk_bits, wv_bits, wo_bits, pos_bits, n_heads):
-    """Fused hidden state of every sequence, fp64 [B][H]."""
+def embed(x_bits, offsets, wq_bits, wk_bits, wv_bits, wo_bits, pos_bits, n_heads,
+          return_o=False):
+    """Fused hidden state of every sequence, fp64 [B][H]; with return_o also the attention
+    output o [B][H] that enters the output linear (zeros for single-token sequences)."""
     x = bf16_bits_to_f64(x_bits)
     wq, wk, wv, wo = (bf16_bits_to_f64(w) for w in (wq_bits, wk_bits, wv_bits, wo_bits))
     pos = bf16_bits_to_f64(pos_bits)
@@ -51,6 +53,7 @@ def embed(x_bits, offsets, wq_bits, wk_bits, wv_bits, wo_bits, pos_bits, n_heads
     B, H = len(offsets) - 1, x.shape[1]
     hd = H // n_heads
     out = np.zeros((B, H))
+    o_rows = np.zeros((B, H))
     for b in range(B):
         xs = x[offsets[b]:offsets[b + 1]]
         n = len(xs)
@@ -70,7 +73,8 @@ def embed(x_bits, offsets, wq_bits, wk_bits, wv_bits, wo_bits, pos_bits, n_heads
             a = softmax(k[:, sl] @ q[sl] / np.sqrt(hd))
             o[sl] = a @ v[:, sl]
         out[b] = wo @ o
-    return out
+        o_rows[b] = o
+    return (out, o_rows) if return_o else out
 
 
 def attention_weights(x_bits, n_tokens_first, wq_bits, wk_bits, pos_bits, n_heads):

@@ -6,24 +6,30 @@
 // learned embedding of each token's place in the patch, then a linear layer; one token skips
 // the module.  On the GPU, four launches:
 //
-//  1. QKV = X [T][H] . [W_q; W_k; W_v]^T in fp32 (one cuBLAS GEMM).  Because the projections
+//  1. QKV = X [T][H] . [W_q; W_k; W_v]^T in fp32 (gemm_xwt_kernel, the tcgen05 weight-streaming
+//     projection of ham_gemm.cu, in split parts that the next kernel sums).  Because the projections
 //     are linear, W_q mean(x) = mean(W_q x), and W_{k,v} (x_i + P[i]) = W_{k,v} x_i + W_{k,v} P[i]:
 //     the position terms KVP = [W_k; W_v] P^T are computed once when the handle is made.
 //  2. fuse_kernel, one warp per (sequence, head): the mean query, k_i and v_i with their
-//     position terms, the scaled scores, softmax over the patch (fp32) and o, every load of the
-//     patch issued at once.  o goes out as two bf16 parts, hi = bf16(o) and lo = bf16(o - hi),
+//     position terms, the scaled scores, softmax over the patch (fp32) and o, the loads of the
+//     patch a round trip a part.  o goes out as two bf16 parts, hi = bf16(o) and lo = bf16(o - hi),
 //     stacked as 2B rows, so that the output projection sees about 16 bits of it.
-//  3. [o_hi; o_lo] . W_o^T in fp32 (one cuBLAS GEMM over the 2B rows: the weights are read
-//     once).
+//  3. [o_hi; o_lo] . W_o^T in fp32 (the same projection kernel over the 2B rows: the weights are
+//     read once; launched with programmatic dependent launch, it requests its first W_o tiles
+//     while the fusion kernel still runs).
 //  4. finish_kernel: the state is the two products' sum rounded to bf16, or for a sequence of
 //     one token its embedding bit for bit; a token count outside 1..max_patch (or rows outside
 //     the call's tokens) gives zeros and sets the error word.
+// Every launch is a programmatic dependent launch of the one before (the next call's
+// projection included): it is scheduled while its predecessor runs, reads only inputs and
+// weights until its dependency wait, and waits before the first read of what the predecessor
+// wrote; the four are a chain of short latency-bound steps, so the overlap is most of the gain.
 // The weights (4 H^2 bf16) dominate the bytes of a call: memory-bound at decoding batches,
 // where the token rows are far fewer than the weight rows.
 // With token ids (ham_embed_tokens) step 1 is a lookup: the projections of every vocabulary
 // entry, [W_q; W_k; W_v] E[v], are tabulated once in fp32, and the fusion kernel reads the rows
 // of the ids.  A call then reads W_o (H^2 bf16) and 12 H bytes per token instead of 4 H^2.
-#include <cublas_v2.h>
+#include <cuda.h>
 #include <cuda_bf16.h>
 
 #include <cstdarg>
@@ -33,20 +39,22 @@
 #include <cstring>
 
 #include "ham_internal.cuh"
+#include "ham_ptx.cuh"
 
 struct ham_embedder {
   ham_embed_config cfg{};
   int device = 0;
-  cublasHandle_t blas = nullptr;
-  void *blas_ws = nullptr;       // cuBLAS workspace (so that no call allocates, even captured)
+  CUtensorMap tmap_wkv{};        // [W_k; W_v] rows of wqkv, 128-row boxes (position terms)
+  uint8_t *wqkv_t = nullptr;     // [W_q; W_k; W_v] and W_o pre-tiled for the projection kernel
+  uint8_t *wo_t = nullptr;
   __nv_bfloat16 *wqkv = nullptr; // [3H][H]
   __nv_bfloat16 *wo = nullptr;   // [H][H]
   float *kvp = nullptr;          // [max_patch][2H]: W_k P[i], W_v P[i]
   int32_t vocab = 0;             // entries of the vocabulary tables (0: none set)
   __nv_bfloat16 *table_e = nullptr; // [vocab][H]: the token embeddings
   float *table_qkv = nullptr;    // [vocab][3H] fp32: [W_q; W_k; W_v] E[v]
-  float *qkv = nullptr;          // [max_batch * max_patch][3H] fp32
-  float *part2 = nullptr;        // [2][batch][H] fp32: the output projection of o_hi, o_lo
+  float *qkv = nullptr;          // [parts][rows][3H] fp32: split parts of the Q/K/V projection
+  float *part2 = nullptr;        // [parts][2 batch][H] fp32: the output projection of o_hi, o_lo
   __nv_bfloat16 *o = nullptr;    // [2][batch][H]: o's hi and lo bf16 parts
   int32_t *err = nullptr;        // device error word
   int32_t *host_err = nullptr;   // pinned read-back
@@ -55,7 +63,6 @@ struct ham_embedder {
 namespace ham {
 namespace {
 
-constexpr size_t kBlasWorkspace = 32u << 20;
 constexpr int kMaxPatch = 8;  // tokens per sequence, at most (ham_embed_config.max_patch)
 
 int efail(int status, const char *fmt, ...) {
@@ -81,6 +88,11 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
                                                    const int32_t *__restrict__ ids, int vocab,
                                                    int batch, int total, int H, int n_heads,
                                                    int max_patch, float scale) {
+  // the output projection may be scheduled now: it reads only its weights until its dependency
+  // wait, which waits for this whole grid
+  grid_launch_dependents();
+  // launched dependent on the Q/K/V projection: everything before the wait reads only the call's
+  // inputs and the handle's tables; the wait precedes the first read of its parts
   const int warp = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
   const int lane = threadIdx.x & 31;
   if (warp >= batch * n_heads) return;
@@ -108,7 +120,9 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
   }
   const int64_t ld = 3 * (int64_t)H, part = (int64_t)total * ld;
   const int64_t col = (int64_t)h * hd + lane;
-  // every load of the patch at once (one round trip): q, k and v rows and the position terms
+  const bool tabulated = ids != nullptr;  // the tables were written when the handle was made
+  // the patch's loads a round trip at a time: the position terms, then each part's q, k and v
+  // rows of every token at once (the parts are added in their order)
   float qv[kMaxPatch][kPer], kv[kMaxPatch][kPer], vv[kMaxPatch][kPer];
 #pragma unroll
   for (int i = 0; i < kMaxPatch; ++i) {
@@ -120,8 +134,14 @@ __global__ void __launch_bounds__(256) fuse_kernel(const float *__restrict__ qkv
       kv[i][e] = in ? pp[32 * e] : 0.f;
       vv[i][e] = in ? pp[H + 32 * e] : 0.f;
     }
-    for (int sp = 0; sp < nparts; ++sp) {
-      const float *r = qkv + sp * part + (int64_t)(in ? row[i] : row[0]) * ld + col;
+  }
+  if (!tabulated) grid_dependency_wait();
+  for (int sp = 0; sp < nparts; ++sp) {
+    const float *base = qkv + sp * part + col;
+#pragma unroll
+    for (int i = 0; i < kMaxPatch; ++i) {
+      const bool in = i < n;
+      const float *r = base + (int64_t)(in ? row[i] : row[0]) * ld;
 #pragma unroll
       for (int e = 0; e < kPer; ++e) {
         qv[i][e] += in ? r[32 * e] : 0.f;
@@ -185,6 +205,10 @@ __global__ void finish_kernel(const float *__restrict__ part, int nparts,
                               const int32_t *__restrict__ offsets, __nv_bfloat16 *__restrict__ out,
                               const int32_t *__restrict__ ids, int vocab, int batch, int total,
                               int H, int max_patch) {
+  // the next call's projection may be scheduled now (it waits for this grid before its first
+  // read of anything a call writes); launched dependent on the output projection, this kernel
+  // reads the call's inputs first and waits before the first read of the parts
+  grid_launch_dependents();
   const int b = blockIdx.y;
   const int j = 8 * (blockIdx.x * blockDim.x + threadIdx.x);
   if (b >= batch || j >= H) return;
@@ -202,12 +226,28 @@ __global__ void finish_kernel(const float *__restrict__ part, int nparts,
   if (!bad && n == 1) {
     v = *reinterpret_cast<const uint4 *>(x + (int64_t)xrow * H + j);
   } else if (!bad) {
+    grid_dependency_wait();
+    // the parts added in their order, loaded kBatch at a time (one round trip each batch)
+    constexpr int kBatch = 10;
     float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int sp = 0; sp < nparts; ++sp) {
-      const float4 *p = reinterpret_cast<const float4 *>(part + ((int64_t)sp * batch + b) * H + j);
-      const float4 lo = p[0], hi = p[1];
-      acc[0] += lo.x; acc[1] += lo.y; acc[2] += lo.z; acc[3] += lo.w;
-      acc[4] += hi.x; acc[5] += hi.y; acc[6] += hi.z; acc[7] += hi.w;
+    for (int sp0 = 0; sp0 < nparts; sp0 += kBatch) {
+      float4 lo[kBatch], hi[kBatch];
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        if (sp0 + u < nparts) {
+          const float4 *p = reinterpret_cast<const float4 *>(
+              part + ((int64_t)(sp0 + u) * batch + b) * H + j);
+          lo[u] = p[0];
+          hi[u] = p[1];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        if (sp0 + u < nparts) {
+          acc[0] += lo[u].x; acc[1] += lo[u].y; acc[2] += lo[u].z; acc[3] += lo[u].w;
+          acc[4] += hi[u].x; acc[5] += hi[u].y; acc[6] += hi[u].z; acc[7] += hi[u].w;
+        }
+      }
     }
     uint32_t w[4];
 #pragma unroll
@@ -221,30 +261,53 @@ __global__ void finish_kernel(const float *__restrict__ part, int nparts,
   *reinterpret_cast<uint4 *>(out + (int64_t)b * H + j) = v;
 }
 
-// C[rows][n_out] (row-major, ldc) = A[rows][k] (row-major bf16) . W[n_out][k]^T (bf16)
-// + beta C.
-cublasStatus_t gemm_rows(cublasHandle_t h, int rows, int n_out, int k, const __nv_bfloat16 *a,
-                         const __nv_bfloat16 *w, void *c, cudaDataType_t c_type, int ldc,
-                         float beta = 0.f) {
-  const float one = 1.f, zero = beta;
-  // column-major view: C^T [n_out][rows] = W (k x n_out, transposed) . A^T (k x rows)
-  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, n_out, rows, k, &one, w, CUDA_R_16BF, k, a,
-                      CUDA_R_16BF, k, &zero, c, c_type, ldc, CUBLAS_COMPUTE_32F,
-                      CUBLAS_GEMM_DEFAULT);
-}
-
 }  // namespace
 }  // namespace ham
 
 namespace ham {
 namespace {
 
-// parts[rows][n_out] = X[rows][K] . W[n_out][K]^T in fp32 (one cuBLAS GEMM).
-bool project(ham_embedder *e, cudaStream_t s, const __nv_bfloat16 *X, const __nv_bfloat16 *W,
-             float *parts, int rows, int n_out, int K) {
-  return cublasSetStream(e->blas, s) == CUBLAS_STATUS_SUCCESS &&
-         gemm_rows(e->blas, rows, n_out, K, X, W, parts, CUDA_R_32F, n_out) ==
-             CUBLAS_STATUS_SUCCESS;
+// parts[s][rows][ldy] = X[rows][K_s] . W[n_out][K_s]^T in fp32 on the tensor cores, W pre-tiled
+// (wt) or through a tensor map (tw); returns the number of parts (the K splits: `splits`, or 0
+// for the kernel's choice of at most kMaxSplits), or -1 on failure.
+// Split caps: each split is one more part for the fusion (Q/K/V) or finish (output) kernel to
+// read; the output projection, whose weights are fewer, needs more CTAs to stream them.
+constexpr int kMaxSplitsQKV = 3, kMaxSplitsOut = 4;
+int project(ham_embedder *e, cudaStream_t s, const CUtensorMap *tw, const void *wt,
+            const __nv_bfloat16 *X, float *parts, int rows, int n_out, int K, int64_t ldy,
+            int splits, bool pdl, int max_splits = kMaxSplitsQKV) {
+  CUtensorMap tx;
+  if (make_matrix_tensor_map(&tx, X, rows, K, gemm_row_tile(rows)) != 0) return -1;
+  const int S = splits > 0 ? splits : gemm_splits(n_out, K, rows, max_splits);
+  if (launch_gemm_xwt(tw, wt, tx, parts, ldy, e->err, rows, n_out, K, S, pdl, s) != cudaSuccess)
+    return -1;
+  return S;
+}
+
+// Largest parts x rows of a projection of up to max_rows rows (the part buffer's size).
+size_t max_part_rows(int n_out, int K, int min_rows, int max_rows, int step, int max_splits) {
+  size_t best = 0;
+  for (int r = min_rows; r <= max_rows; r += step)
+    best = std::max(best, (size_t)gemm_splits(n_out, K, r, max_splits) * (size_t)r);
+  return best;
+}
+
+// A launch with programmatic dependent launch: the kernel may start before the previous one on
+// the stream ends, and waits for it (griddepcontrol.wait) before reading what it wrote.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kernel)(KArgs...), dim3 grid, dim3 block, cudaStream_t s,
+                             Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
 // The four launches of a call.  Without ids, xb is the call's token rows and step 1 is the
@@ -269,28 +332,34 @@ int run_embed(ham_embedder *e, const __nv_bfloat16 *xb, const int32_t *ids,
   int rc = HAM_OK;
   __nv_bfloat16 *o_lo = e->o + (size_t)batch * H;  // rows batch..2 batch-1 of one [2B][H] block
   const float *qkv = ids ? e->table_qkv : e->qkv;
-  if (!ids && !project(e, s, xb, e->wqkv, e->qkv, total_tokens, 3 * H, H))
-    rc = efail(HAM_ECUDA, "projection GEMM failed");
+  int qkv_parts = 1;
+  if (!ids) {
+    qkv_parts = project(e, s, nullptr, e->wqkv_t, xb, e->qkv, total_tokens, 3 * H, H, 3 * H,
+                        0, true);
+    if (qkv_parts < 1) rc = efail(HAM_ECUDA, "Q/K/V projection launch failed");
+  }
   if (rc == HAM_OK) {
     const int warps = batch * c.n_heads;
     const dim3 grid((unsigned)((warps + 7) / 8)), block(256);
     const float scale = 1.f / sqrtf((float)hd);
     auto fuse = hd == 32 ? fuse_kernel<1> : hd == 64 ? fuse_kernel<2> : fuse_kernel<4>;
-    fuse<<<grid, block, 0, s>>>(qkv, 1, e->kvp, offsets, e->o, o_lo, e->err, ids, e->vocab,
-                                batch, total_tokens, H, c.n_heads, c.max_patch, scale);
-    cudaError_t ce = cudaGetLastError();
+    cudaError_t ce = launch_dependent(fuse, grid, block, s, qkv, qkv_parts, (const float *)e->kvp,
+                                      offsets, e->o, o_lo, e->err, ids, (int)e->vocab, (int)batch,
+                                      (int)total_tokens, H, c.n_heads, c.max_patch, scale);
     if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "fuse launch: %s", cudaGetErrorString(ce));
   }
+  int out_parts = 0;
   if (rc == HAM_OK) {  // o_hi and o_lo stacked as 2B rows: the weights are read once
-    if (!project(e, s, e->o, e->wo, e->part2, 2 * batch, H, H))
-      rc = efail(HAM_ECUDA, "output GEMM failed");
+    out_parts = project(e, s, nullptr, e->wo_t, e->o, e->part2, 2 * batch, H, H, H, 0, true,
+                        kMaxSplitsOut);
+    if (out_parts < 1) rc = efail(HAM_ECUDA, "output projection launch failed");
   }
   if (rc == HAM_OK) {
     const dim3 grid((unsigned)((H / 8 + 127) / 128), (unsigned)batch), block(128);
-    finish_kernel<<<grid, block, 0, s>>>(e->part2, 2, xb, offsets,
-                                         static_cast<__nv_bfloat16 *>(out), ids, e->vocab,
-                                         batch, total_tokens, H, c.max_patch);
-    cudaError_t ce = cudaGetLastError();
+    cudaError_t ce = launch_dependent(finish_kernel, grid, block, s, (const float *)e->part2,
+                                      2 * out_parts, xb, offsets,
+                                      static_cast<__nv_bfloat16 *>(out), ids, (int)e->vocab,
+                                      (int)batch, (int)total_tokens, H, c.max_patch);
     if (ce != cudaSuccess) rc = efail(HAM_ECUDA, "finish launch: %s", cudaGetErrorString(ce));
   }
   if (dev != e->device) cudaSetDevice(dev);
@@ -309,10 +378,10 @@ int ham_embedder_free(ham_embedder *e) {
   int dev = 0;
   cudaGetDevice(&dev);
   cudaSetDevice(e->device);
-  if (e->blas) cublasDestroy(e->blas);
-  cudaFree(e->blas_ws);
   cudaFree(e->wqkv);
   cudaFree(e->wo);
+  cudaFree(e->wqkv_t);
+  cudaFree(e->wo_t);
   cudaFree(e->kvp);
   cudaFree(e->table_e);
   cudaFree(e->table_qkv);
@@ -353,12 +422,16 @@ int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *
   };
   alloc(reinterpret_cast<void **>(&e->wqkv), 3 * hh * 2);
   alloc(reinterpret_cast<void **>(&e->wo), hh * 2);
+  alloc(reinterpret_cast<void **>(&e->wqkv_t), ham::tiled_weight_bytes(3 * H, H));
+  alloc(reinterpret_cast<void **>(&e->wo_t), ham::tiled_weight_bytes(H, H));
   alloc(reinterpret_cast<void **>(&e->kvp), (size_t)cfg->max_patch * 2 * H * 4);
-  alloc(reinterpret_cast<void **>(&e->qkv), rows * 3 * H * 4);
-  alloc(reinterpret_cast<void **>(&e->part2), 2 * (size_t)cfg->max_batch * H * 4);
+  // split parts of the projections, for the largest parts x rows any call can produce
+  alloc(reinterpret_cast<void **>(&e->qkv),
+        ham::max_part_rows(3 * H, H, 1, (int)rows, 1, ham::kMaxSplitsQKV) * 3 * H * 4);
+  alloc(reinterpret_cast<void **>(&e->part2),
+        ham::max_part_rows(H, H, 2, 2 * cfg->max_batch, 2, ham::kMaxSplitsOut) * H * 4);
   alloc(reinterpret_cast<void **>(&e->o), 2 * (size_t)cfg->max_batch * H * 2);
   alloc(reinterpret_cast<void **>(&e->err), 4);
-  alloc(&e->blas_ws, ham::kBlasWorkspace);
   if (ce == cudaSuccess) ce = cudaMallocHost(reinterpret_cast<void **>(&e->host_err), 4);
   if (ce != cudaSuccess) {
     cudaGetLastError();
@@ -375,19 +448,22 @@ int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *
     ham_embedder_free(e);
     return efail(HAM_ECUDA, "embedder set-up: %s", cudaGetErrorString(ce));
   }
-  cublasStatus_t bs = cublasCreate(&e->blas);
-  if (bs == CUBLAS_STATUS_SUCCESS) bs = cublasSetWorkspace(e->blas, e->blas_ws, ham::kBlasWorkspace);
-  // position terms: KVP [max_patch][2H] = P [max_patch][H] . [W_k; W_v]^T
-  if (bs == CUBLAS_STATUS_SUCCESS)
-    bs = ham::gemm_rows(e->blas, cfg->max_patch, 2 * H, H,
-                        static_cast<const __nv_bfloat16 *>(pos), e->wqkv + hh, e->kvp,
-                        CUDA_R_32F, 2 * H);
-  if (bs == CUBLAS_STATUS_SUCCESS && cudaDeviceSynchronize() != cudaSuccess)
-    bs = CUBLAS_STATUS_EXECUTION_FAILED;
-  if (bs != CUBLAS_STATUS_SUCCESS) {
+  // the projection kernel's tiled weights, and a tensor map of [W_k; W_v] for the position terms
+  int tr = ham::tile_weights(e->wqkv, 3 * H, H, e->wqkv_t, nullptr) == cudaSuccess &&
+                   ham::tile_weights(e->wo, H, H, e->wo_t, nullptr) == cudaSuccess
+               ? 0
+               : -1;
+  if (tr == 0) tr = ham::make_matrix_tensor_map(&e->tmap_wkv, e->wqkv + hh, 2 * (int64_t)H, H, 128);
+  // position terms: KVP [max_patch][2H] = P [max_patch][H] . [W_k; W_v]^T (one part)
+  if (tr == 0 && ham::project(e, nullptr, &e->tmap_wkv, nullptr,
+                              static_cast<const __nv_bfloat16 *>(pos), e->kvp, cfg->max_patch,
+                              2 * H, H, 2 * H, 1, false) != 1)
+    tr = -1;
+  if (tr == 0 && cudaDeviceSynchronize() != cudaSuccess) tr = -1;
+  if (tr != 0) {
     cudaGetLastError();
     ham_embedder_free(e);
-    return efail(HAM_ECUDA, "cuBLAS set-up failed (status %d)", (int)bs);
+    return efail(HAM_ECUDA, "embedder set-up (tensor maps or position terms) failed");
   }
   *out = e;
   return HAM_OK;
@@ -434,16 +510,15 @@ int ham_embedder_set_vocab(ham_embedder *e, const void *table, int32_t vocab) {
   }
   if (rc == HAM_OK) {
     ce = cudaMemcpy(e->table_e, table, (size_t)vocab * H * 2, cudaMemcpyDeviceToDevice);
-    // the tabulated projections: [vocab][3H] = E [vocab][H] . [W_q; W_k; W_v]^T, fp32
-    cublasStatus_t bs = cublasSetStream(e->blas, nullptr);
-    if (ce == cudaSuccess && bs == CUBLAS_STATUS_SUCCESS)
-      bs = ham::gemm_rows(e->blas, vocab, 3 * H, H, e->table_e, e->wqkv, e->table_qkv,
-                          CUDA_R_32F, 3 * H);
+    // the tabulated projections: [vocab][3H] = E [vocab][H] . [W_q; W_k; W_v]^T, fp32 (one part)
+    if (ce == cudaSuccess &&
+        ham::project(e, nullptr, nullptr, e->wqkv_t, e->table_e, e->table_qkv, vocab, 3 * H, H,
+                     3 * H, 1, false) != 1)
+      ce = cudaErrorLaunchFailure;
     if (ce == cudaSuccess) ce = cudaDeviceSynchronize();
-    if (ce != cudaSuccess || bs != CUBLAS_STATUS_SUCCESS) {
+    if (ce != cudaSuccess) {
       cudaGetLastError();
-      rc = efail(HAM_ECUDA, "vocabulary tabulation: %s, cuBLAS status %d",
-                 cudaGetErrorString(ce), (int)bs);
+      rc = efail(HAM_ECUDA, "vocabulary tabulation: %s", cudaGetErrorString(ce));
     }
   }
   if (rc == HAM_OK) {

@@ -154,6 +154,32 @@ bool attention_supported(int head_dim, int group);
 // {64 elements, head_dim / 64, rows} with a box of {64, head_dim / 64, 16 rows} (half_box:
 // {64, 1, 16 rows}, one 64-column half of a chunk) and the 128-byte swizzle.  Returns a
 // CUresult (0 on success).
+// TMA map of a row-major [rows][cols] bf16 matrix with a box of {64 columns, box_rows rows} (128
+// bytes of each row) and the 128-byte swizzle: one K-major operand tile of a tcgen05 product.
+// cols must be a multiple of 8; boxes past the last row or column read zeros.  Returns a CUresult.
+int make_matrix_tensor_map(CUtensorMap *map, const void *base, int64_t rows, int64_t cols,
+                           int box_rows);
+// TMA map of fp32 split parts [splits][rows][ld] (columns 0..cols-1 used) with a box of {32
+// columns, 32 rows, 1 part} and the 128-byte swizzle: the store of one epilogue warp.  ld a
+// multiple of 4 and base 16-byte aligned.  Returns a CUresult.
+int make_parts_tensor_map(CUtensorMap *map, void *base, int splits, int64_t rows, int64_t cols,
+                          int64_t ld);
+// Y[s][rows][ldy] (fp32, columns 0..F-1) = X[rows][K_s] . W[F][K_s]^T, the K columns split in
+// `splits` ranges K_s of whole 64-column tiles, as even as the tile count allows (the caller sums
+// the parts): tcgen05 products of 128 output features by up to 256 rows.  W is either pre-tiled
+// (wt, from tile_weights) or given by tw (a tensor map of make_matrix_tensor_map with box_rows
+// 128); X by tx (box_rows = gemm_row_tile(rows)).  splits <= ceil(K / 64).  With `pdl` the
+// launch may start before the previous kernel on the stream ends: it loads W tiles before its
+// dependency wait and X only after.
+int gemm_row_tile(int rows);
+int gemm_splits(int F, int K, int rows, int max_splits);
+// W [F][K] row-major bf16 -> wt: each 128 x 64 tile one contiguous 16 KiB block in the 128-byte
+// swizzle layout, tiles [ceil(F/128)][ceil(K/64)], zeros past the matrix (one launch).
+size_t tiled_weight_bytes(int F, int K);
+cudaError_t tile_weights(const void *W, int F, int K, void *wt, cudaStream_t stream);
+cudaError_t launch_gemm_xwt(const CUtensorMap *tw, const void *wt, const CUtensorMap &tx,
+                            float *Y, int64_t ldy, int32_t *err, int rows, int F, int K,
+                            int splits, bool pdl, cudaStream_t stream);
 // TMA map of a row-major [rows][heads][head_dim] bf16 tensor viewed as {64 elements,
 // head_dim / 64, heads, rows} with a box of {64, 1, box_heads, box_rows} (one 64-column half of
 // box_heads x box_rows head rows) and the 128-byte swizzle.  Boxes past the last row read zeros.

@@ -293,6 +293,33 @@ int make_rows_tensor_map(CUtensorMap *map, const void *base, int64_t rows, int h
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+int make_matrix_tensor_map(CUtensorMap *map, const void *base, int64_t rows, int64_t cols,
+                           int box_rows) {
+  EncodeTiled encode = tensor_map_encoder();
+  if (!encode) return -1;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};  // bytes of a row
+  const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+  const cuuint32_t estride[2] = {1, 1};
+  return (int)encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims,
+                     strides, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+int make_parts_tensor_map(CUtensorMap *map, void *base, int splits, int64_t rows, int64_t cols,
+                          int64_t ld) {
+  EncodeTiled encode = tensor_map_encoder();
+  if (!encode) return -1;
+  const cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)splits};
+  const cuuint64_t strides[2] = {(cuuint64_t)ld * 4, (cuuint64_t)(rows * ld) * 4};  // bytes
+  const cuuint32_t box[3] = {32, 32, 1};
+  const cuuint32_t estride[3] = {1, 1, 1};
+  return (int)encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box, estride,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim,
                          bool half_box) {
   EncodeTiled encode = tensor_map_encoder();
