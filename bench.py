@@ -59,6 +59,9 @@ def parse_args():
                         "region lasts at least this long, whatever --steps asks for")
     p.add_argument("--no-target-point", action="store_true",
                    help="default workload: skip the batch 8 x 8192 slots point")
+    p.add_argument("--kv", choices=["bf16", "fp8"], default="bf16",
+                   help="decode workloads: bf16 pools, or FP8 (e4m3) pools with one power-of-two "
+                        "scale per row (read by ham_kv_append + ham_decode_attn: --path split)")
     p.add_argument("--path", choices=["fused", "split"], default="fused",
                    help="fused: ham_decode_step; split: ham_kv_append + ham_decode_attn")
     p.add_argument("--caches", type=int, default=CACHES,
@@ -262,7 +265,7 @@ STEP_TEXT = {
 }
 
 
-def config_dict(w, path="fused"):
+def config_dict(w, path="fused", kv="bf16"):
     counts = base_counts(w)
     slots = w.slots if w.slot_range is None else (
         f"{int(counts.min())}..{int(counts.max())} (mean {counts.mean():.0f}, uniform draw "
@@ -272,33 +275,41 @@ def config_dict(w, path="fused"):
             "page_slots": w.page_slots, "pages": "scattered by a seeded shuffle of a shared pool",
             "tokens_per_slot": "geometric p=0.5 capped at 4 (mean 1.875)",
             "step": STEP_TEXT[path],
+            "kv_dtype": ("e4m3 codes + one int8 power-of-two exponent per (slot, KV head) row"
+                         if kv == "fp8" else "bf16"),
             "l2": f"{CACHES} independent caches rotated ({CACHES} x "
-                  f"{int(counts.sum()) * w.n_kv_heads * w.head_dim * 4 / 2**20:.0f} MiB KV "
-                  "> 129 MB L2)",
+                  f"{int(counts.sum()) * w.n_kv_heads * kv_row_bytes(w, kv) * 2 / 2**20:.0f} "
+                  "MiB KV > 129 MB L2)",
             "graph": f"{GRAPH_STEPS} steps per CUDA graph, then each cache is rolled back "
                      "to its starting slot counts"}
 
 
-def attn_bytes(w, lengths):
+def kv_row_bytes(w, kv="bf16"):
+    """Bytes of one stored K (or V) row of one (slot, KV head): bf16 elements, or e4m3 codes
+    plus the row's int8 exponent."""
+    return w.head_dim + 1 if kv == "fp8" else w.head_dim * 2
+
+
+def attn_bytes(w, lengths, kv="bf16"):
     """Algorithmic bytes of one attention launch over sequences of `lengths` slots: K and V
     of every slot once, q in, out, and the page-table entries."""
-    kv = sum(int(L) for L in lengths) * w.n_kv_heads * w.head_dim * 2 * 2
+    kv = sum(int(L) for L in lengths) * w.n_kv_heads * kv_row_bytes(w, kv) * 2
     qo = 2 * w.batch * w.n_q_heads * w.head_dim * 2
     pt = sum(math.ceil(int(L) / w.page_slots) for L in lengths) * 4
     return kv + qo + pt
 
 
-def append_bytes(w):
+def append_bytes(w, kv="bf16"):
     """Algorithmic bytes of one append: q read+write, k_new/v_new in, K/V rows out, metadata."""
     return (2 * w.batch * w.n_q_heads * w.head_dim * 2 + 4 * w.batch * w.n_kv_heads * w.head_dim
-            + w.batch * 4 * 6)
+            + 2 * w.batch * w.n_kv_heads * kv_row_bytes(w, kv) + w.batch * 4 * 6)
 
 
 # ---------------------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------------------
 
-def build_caches(w, device_index, rank):
+def build_caches(w, device_index, rank, kv_dtype=0):
     import numpy as np
     import torch
 
@@ -314,7 +325,7 @@ def build_caches(w, device_index, rank):
         kv = ham.ham_kv_alloc(1, w.batch, w.n_q_heads, w.n_kv_heads, w.head_dim, w.page_slots,
                               max_slots, pool_pages=int(math.ceil(
                                   w.batch * math.ceil(max_slots / w.page_slots) * w.pool_factor)),
-                              page_seed=seed + 1)
+                              page_seed=seed + 1, kv_dtype=kv_dtype)
         shape = (w.batch, lmax, w.n_kv_heads, w.head_dim)
         k = wl.device_normal_bf16(shape, w.value_scale, seed * 7 + 1)
         v = wl.device_normal_bf16(shape, w.value_scale, seed * 7 + 2)
@@ -378,7 +389,8 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
 
     from paper_2505_20438_gb300 import ham
 
-    caches = build_caches(w, local_rank, rank)
+    fp8 = args.kv == "fp8"
+    caches = build_caches(w, local_rank, rank, ham.HAM_KV_E4M3 if fp8 else ham.HAM_KV_BF16)
     stream = torch.cuda.Stream()
     n_graph = max(1, math.ceil(args.steps / GRAPH_STEPS))
     n_warm = max(1, math.ceil(max(args.warmup, 3) / GRAPH_STEPS))
@@ -454,8 +466,9 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
 
     # attended lengths inside one graph: step i (cache i % 4) sees counts + 1 + i // 4 slots
     counts_h = base_counts(w)
-    attn_bytes_graph = sum(attn_bytes(w, counts_h + 1 + i // CACHES) for i in range(GRAPH_STEPS))
-    step_bytes_graph = attn_bytes_graph + GRAPH_STEPS * append_bytes(w)
+    attn_bytes_graph = sum(attn_bytes(w, counts_h + 1 + i // CACHES, args.kv)
+                           for i in range(GRAPH_STEPS))
+    step_bytes_graph = attn_bytes_graph + GRAPH_STEPS * append_bytes(w, args.kv)
     timed_bytes_graph = step_bytes_graph  # the span covers the whole step on both paths
 
     w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -519,13 +532,15 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
 
     e2e = run_e2e(args, w, caches, stream, rollback, world, one_step) if full else None
 
-    traffic = profiled_traffic("decode_step" if fused else "decode_attn", w.name)
+    traffic = profiled_traffic(("decode_step" if fused else "decode_attn") + ("_fp8" if fp8 else ""),
+                               w.name)
     result = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
         "steps": steps, "steps_requested": args.steps, "timed_s": round(elapsed_ms * 1e-3, 3),
         "warmup": n_warm * GRAPH_STEPS, "ms_per_step": round(ms_per_step, 5),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "accum_dtype": "f32", "data": "synthetic", "config": config_dict(w, args.path),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "e4m3" if fp8 else "bf16",
+        "accum_dtype": "f32", "data": "synthetic", "config": config_dict(w, args.path, args.kv),
         "kv_gbs": round(step_gbs, 1),
         "kv_frac_of_measured_peak": round(step_gbs / world / peak, 4),
         "kv_frac_of_8tbs_spec": round(step_gbs / world / 8000.0, 4),
@@ -534,8 +549,8 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
         "roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(attn_gbs / peak, 4), "traffic": traffic,
                      "kernel": ("decode_attn_kernel<128,bf16,step> + combine_kernel<bf16,step>"
-                                if fused else "append_kernel + decode_attn_kernel<128,bf16> + "
-                                "combine_kernel<bf16>"),
+                                if fused else "append_kernel + decode_attn_kernel<128,bf16" +
+                                (",fp8" if fp8 else "") + "> + combine_kernel<bf16>"),
                      "avg_launch_us": round(1e3 * statistics.mean(attn_ms), 3),
                      "isolated_launch_us": isolated_us,
                      "algorithmic_bytes_per_launch": int(timed_bytes_graph / GRAPH_STEPS),
@@ -547,7 +562,9 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
     }
     if e2e is None:
         del result["e2e"]
-    if full and rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if fp8:
+        result["mma_dtype"] = "f16 codes x q 2^-f (scores), bf16 codes x weights (values)"
+    if full and rank == 0 and world == 1 and not args.no_cpu_baseline and not fp8:
         result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
     for c in caches:
         ham.ham_kv_free(c["kv"])
@@ -1921,6 +1938,8 @@ def main():
     if args.caches < 1 or GRAPH_STEPS % args.caches:
         raise SystemExit(f"--caches must divide {GRAPH_STEPS}")
     CACHES = args.caches
+    if args.kv == "fp8":
+        args.path = "split"  # FP8 pools are read by ham_kv_append + ham_decode_attn
     w = workload(args.workload)
     from paper_2505_20438_gb300 import workload as wl
     if args.impl == "reference":

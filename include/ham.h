@@ -64,6 +64,9 @@ enum {
 
 enum { HAM_DTYPE_BF16 = 0, HAM_DTYPE_F32 = 1 };
 
+/* Storage type of the KV pools (ham_config.kv_dtype); see "FP8 (e4m3) pools" below. */
+enum { HAM_KV_BF16 = 0, HAM_KV_E4M3 = 1 };
+
 typedef struct ham_kv ham_kv; /* opaque handle: one paged smashed-KV cache, all layers */
 
 typedef struct ham_config {
@@ -78,6 +81,7 @@ typedef struct ham_config {
   int64_t pool_pages;        /* pages in the pool; 0 = batch * ceil(max_slots_per_seq / page_slots) */
   double rope_base;          /* RoPE base (10000 for Llama-style models) */
   uint64_t page_seed;        /* 0: sequence b gets pages [b*P, (b+1)*P); else a seeded shuffle */
+  int32_t kv_dtype;          /* HAM_KV_BF16 (0) or HAM_KV_E4M3 (8-bit rows, head_dim 128) */
 } ham_config;
 
 typedef struct ham_kv_info {
@@ -86,7 +90,7 @@ typedef struct ham_kv_info {
   int32_t attn_ctas;         /* CTAs of one attention launch */
   int32_t num_sms;           /* SMs of the device the handle lives on */
   int32_t device;            /* CUDA device ordinal */
-  int64_t pool_bytes;        /* K+V bytes of ONE layer's pool */
+  int64_t pool_bytes;        /* K+V bytes of ONE layer's pool (FP8: codes and exponents) */
   int64_t scratch_bytes;     /* split-attention partials and per-segment CTA ranges */
 } ham_kv_info;
 
@@ -287,7 +291,8 @@ int ham_kv_set_page_table(ham_kv *kv, const int32_t *host_pt);
 int ham_kv_get_page_table(const ham_kv *kv, int32_t *host_pt);
 
 /* Load a logical cache into one layer: slot j < counts[b] of sequence b gets
- * k_log/v_log[b][j] (bit copy, no RoPE: keys are taken as already rotated) and, if given,
+ * k_log/v_log[b][j] (bit copy, no RoPE: keys are taken as already rotated; an FP8 pool
+ * stores the rows encoded as described under "FP8 (e4m3) pools") and, if given,
  * slot_pos = pos[b][j], slot_ntok = ntok[b][j] (defaults: j and 1).  Sets
  * num_slots[layer][b] = counts[b] and num_tokens[layer][b] = sum of the ntok.
  * k_log, v_log  device bf16 [batch][lmax][n_kv_heads][head_dim]
@@ -298,10 +303,43 @@ int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
                 void *stream);
 
 /* Copy one layer's raw pools and the slot metadata out (device or pinned host destinations,
- * cudaMemcpyDefault).  k_dst, v_dst: pool_bytes / 2 bytes each; pos_dst, ntok_dst:
+ * cudaMemcpyDefault).  k_dst, v_dst: one pool each, pool_pages * n_kv_heads * page_slots *
+ * head_dim elements (bf16, or FP8 codes in the layouts below); pos_dst, ntok_dst:
  * pool_pages * page_slots int32 each.  Any destination may be NULL. */
 int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *pos_dst,
                   int32_t *ntok_dst, void *stream);
+
+/* ------------------------------------------------------------------------------------
+ * FP8 (e4m3) pools: kv_dtype = HAM_KV_E4M3, head_dim 128
+ * ------------------------------------------------------------------------------------
+ * Decoding re-reads every stored key and value each step and is bound by memory bandwidth
+ * (Sec. 2.3; Sec. 3.7: the KV cache is what the method shrinks), so the rows of a slot may be
+ * stored in 8 bits: 2 x (128 + 1) bytes per (slot, KV head) instead of 2 x 256.  The paper
+ * keeps the base model's precision; this storage format is the library's own:
+ *  - elements: e4m3 codes (1 sign, 4 exponent bits of bias 7, 3 mantissa bits; no
+ *    infinities; largest finite 448); each element scaled exactly and rounded once, to
+ *    nearest with ties to even, saturating at +-448, the sign kept (also on zero);
+ *  - one scale per stored row (one slot of one KV head), a power of two 2^e, e an int8:
+ *    e = E - 8 for the row's largest magnitude m 2^E (0.5 <= m < 1), clamped to [-124, 119]
+ *    so that every decoded value is a finite bf16 value; a row of zeros has e = 0;
+ *  - the key is rotated first (the bf16 row a bf16 cache would hold), then encoded; the value
+ *    is encoded as given.  A decoded element code * 2^e has at most 4 significant bits and
+ *    is an exact bf16 value: attention over an FP8 pool is attention over the decoded rows.
+ * Layout of one layer's pools:
+ *   K codes    [pool_pages][n_kv_heads][page_slots][128] uint8
+ *   V codes    [pool_pages][n_kv_heads][128][page_slots] uint8  (a page's value rows
+ *              transposed: element d of slot s at [d][16 (s / 16) + b(s % 16)], the 16 slots
+ *              of a chunk in the order 0, 1, 8, 9, 2, 3, 10, 11, 4, 5, 12, 13, 6, 7, 14, 15,
+ *              i.e. b(s) = 4 ((s % 8) / 2) + 2 (s / 8) + s % 2)
+ *   exponents  [pool_pages][n_kv_heads][page_slots / 16][2][16] int8  (per 16-slot chunk:
+ *              the 16 keys' exponents, then the 16 values')
+ * FP8 caches work with ham_kv_fill (it encodes the bf16 rows it is given), ham_kv_export,
+ * ham_kv_export_scales, ham_kv_append, ham_decode_attn, ham_decode_attn_ex and the counter
+ * calls; the other calls return HAM_EUNSUPPORTED for them. */
+
+/* Copy one layer's exponent array out (layout above): pool_pages * n_kv_heads * page_slots *
+ * 2 bytes.  HAM_EINVAL for a bf16 cache. */
+int ham_kv_export_scales(ham_kv *kv, int32_t layer, void *e_dst, void *stream);
 
 /* Set the slot and token counters of one layer from device arrays (e.g. to roll back the
  * slots of a rejected macro-step): num_slots [batch] int32, num_tokens [batch] int64

@@ -1,5 +1,7 @@
 // Fused RoPE + append of the slot a macro-step produces (HAMburger Sec. 3.1: one KV set
-// per macro-step; Sec. 3.2: the merged embedding enters at an offset position).
+// per macro-step; Sec. 3.2: the merged embedding enters at an offset position).  An FP8
+// cache stores the rotated bf16 key and the value encoded as e4m3 rows with a power-of-two
+// scale (encode_e4m3_row).
 //
 // One thread-block cluster per sequence, one CTA per KV head (or a few).  The rotation is
 // computed in fp64 and rounded once to bf16 (nearest, ties to even).  cos and sin of
@@ -123,15 +125,51 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(AppendView v) {
   __syncthreads();
   const int64_t page = s_row_meta / v.page_slots;
   const int32_t row = (int32_t)(s_row_meta % v.page_slots);
-  for (int idx = threadIdx.x; idx < ng * half; idx += blockDim.x) {  // keys
-    const int j = idx / half, i = idx % half;
-    const int64_t dst = ((page * v.n_kv_heads + g0 + j) * v.page_slots + row) * d;
-    rotate_pair(k_s + j * d, v.k_pool + dst, i, half, cos_t[i], sin_t[i]);
-  }
-  for (int idx = threadIdx.x; idx < ng * vec; idx += blockDim.x) {  // values, bit copy
-    const int j = idx / vec, e = idx % vec;
-    const int64_t dst = ((page * v.n_kv_heads + g0 + j) * v.page_slots + row) * d;
-    reinterpret_cast<uint4 *>(v.v_pool + dst)[e] = reinterpret_cast<const uint4 *>(v_s + j * d)[e];
+  if (v.kv_exp) {
+    // FP8 pools (head_dim 128): the key is rotated and rounded to bf16 exactly as below, then
+    // each row is encoded by one warp (codes, V transposed within its page, and exponents)
+    // ng * (2 + G) <= kMaxRows at head_dim 128 (append_kv_per_block), G >= 1: ng <= 6
+    __shared__ __align__(16) uint16_t k_rot[(kMaxRows / 3) * kFp8HeadDim];
+    for (int idx = threadIdx.x; idx < ng * half; idx += blockDim.x) {
+      const int j = idx / half, i = idx % half;
+      rotate_pair(k_s + j * d, k_rot + j * d, i, half, cos_t[i], sin_t[i]);
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, P = v.page_slots;
+    uint8_t *kc = reinterpret_cast<uint8_t *>(v.k_pool), *vc = reinterpret_cast<uint8_t *>(v.v_pool);
+    for (int r = warp; r < 2 * ng; r += kAppendThreads / 32) {
+      const int j = r >> 1;
+      const bool is_v = (r & 1) != 0;
+      const uint16_t *src = (is_v ? v_s : k_rot) + j * d + 4 * lane;
+      float x[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) x[i] = __uint_as_float((uint32_t)src[i] << 16);
+      uint32_t codes;
+      const int e = encode_e4m3_row(x, codes);
+      const int64_t ph = page * v.n_kv_heads + g0 + j;  // (page, head) block
+      if (!is_v) {
+        *reinterpret_cast<uint32_t *>(kc + (ph * P + row) * kFp8HeadDim + 4 * lane) = codes;
+      } else {
+        const int sv = row - row % kChunkSlots + fp8_v_slot_byte(row % kChunkSlots);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          vc[(ph * kFp8HeadDim + 4 * lane + i) * P + sv] = (uint8_t)(codes >> (8 * i));
+      }
+      if (lane == 0)
+        v.kv_exp[(ph * (P / kChunkSlots) + row / kChunkSlots) * 32 + (is_v ? kChunkSlots : 0) +
+                 row % kChunkSlots] = (int8_t)e;
+    }
+  } else {
+    for (int idx = threadIdx.x; idx < ng * half; idx += blockDim.x) {  // keys
+      const int j = idx / half, i = idx % half;
+      const int64_t dst = ((page * v.n_kv_heads + g0 + j) * v.page_slots + row) * d;
+      rotate_pair(k_s + j * d, v.k_pool + dst, i, half, cos_t[i], sin_t[i]);
+    }
+    for (int idx = threadIdx.x; idx < ng * vec; idx += blockDim.x) {  // values, bit copy
+      const int j = idx / vec, e = idx % vec;
+      const int64_t dst = ((page * v.n_kv_heads + g0 + j) * v.page_slots + row) * d;
+      reinterpret_cast<uint4 *>(v.v_pool + dst)[e] = reinterpret_cast<const uint4 *>(v_s + j * d)[e];
+    }
   }
   if (v.q) {  // the query heads, turned at the same position, written back in place
     for (int idx = threadIdx.x; idx < ng * G * half; idx += blockDim.x) {

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_fp8.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -16,6 +17,33 @@ namespace ham {
 // two pages and its K (or V) rows are one contiguous 16 * head_dim * 2-byte block.
 constexpr int kChunkSlots = 16;
 constexpr int kMaxBatch = 4096;
+
+// FP8 (e4m3) pools (ham.h, "FP8 (e4m3) pools"): head_dim 128; per layer the K codes
+// [pages][Hkv][P][128], the V codes [pages][Hkv][128][P] (a page's value rows transposed) and
+// the exponents [pages][Hkv][P/16][2][16] (per chunk: 16 keys', then 16 values'), one block
+// after the other in the pool allocation.
+constexpr int kFp8HeadDim = 128;
+constexpr int kFp8ExpMin = -124, kFp8ExpMax = 119;
+// Byte of slot s (0..15) of a chunk within its transposed value rows: the slots are kept in the
+// order 0, 1, 8, 9, 2, 3, 10, 11, 4, 5, 12, 13, 6, 7, 14, 15 (the attention kernel's e4m3
+// products meet four consecutive bytes of a row with the scores of slots 2t, 2t + 1, 8 + 2t,
+// 9 + 2t).
+__host__ __device__ inline int fp8_v_slot_byte(int s) {
+  return ((s & 7) >> 1) * 4 + (s >> 3) * 2 + (s & 1);
+}
+struct Fp8Layer {
+  uint8_t *k, *v;
+  int8_t *e;
+};
+// Bytes of one layer's FP8 block: rows = pool_pages * n_kv_heads * page_slots.
+inline size_t fp8_layer_bytes(int64_t rows) {
+  return (size_t)rows * kFp8HeadDim * 2 + (((size_t)rows * 2 + 1023) / 1024) * 1024;
+}
+inline Fp8Layer fp8_layer(void *pool, int64_t rows, int layer) {
+  uint8_t *base = static_cast<uint8_t *>(pool) + (size_t)layer * fp8_layer_bytes(rows);
+  return {base, base + (size_t)rows * kFp8HeadDim,
+          reinterpret_cast<int8_t *>(base + (size_t)rows * kFp8HeadDim * 2)};
+}
 
 // ---------------------------------------------------------------------------------------
 // Split plan.  The chunks of all (sequence b, KV head g) segments are numbered b-major,
@@ -50,8 +78,13 @@ __host__ __device__ inline int32_t chunks_of(int32_t slots) {
 // wave (a CTA that starts late doubles the launch: the split plan gives every CTA an equal
 // share).
 constexpr int kDefaultCtasPerSm = 4;
-inline int32_t default_attention_ctas(int32_t num_sms, int32_t resident_per_sm) {
-  const int32_t per = resident_per_sm < kDefaultCtasPerSm ? resident_per_sm : kDefaultCtasPerSm;
+// FP8 pools: 16 KiB rings, so twice the CTAs keep the same bytes in flight, and their consumer
+// warps (which convert codes as well) get a second warp per scheduler.
+constexpr int kDefaultCtasPerSmFp8 = 8;
+inline int32_t default_attention_ctas(int32_t num_sms, int32_t resident_per_sm,
+                                      bool fp8 = false) {
+  const int32_t cap = fp8 ? kDefaultCtasPerSmFp8 : kDefaultCtasPerSm;
+  const int32_t per = resident_per_sm < cap ? resident_per_sm : cap;
   return num_sms * (per < 1 ? 1 : per);
 }
 
@@ -68,6 +101,7 @@ struct StepArgs {
   int64_t *num_tokens;             // [batch] of this layer
   int32_t *slot_pos, *slot_ntok;
   uint16_t *k_pool, *v_pool;       // this layer (the new slot's rows, written by combine)
+  int8_t *kv_exp;                  // FP8 pools: the layer's exponents (else null)
   const double *inv_freq;          // [head_dim / 2]
   const double2 *rope_table;       // [rope_positions][head_dim / 2] (cos, sin)
   const float2 *rope_table_f;      // same, fp32
@@ -80,7 +114,8 @@ struct StepArgs {
 
 struct AttnView {
   const uint16_t *k_pool;      // this layer: [pool_pages][n_kv_heads][page_slots][head_dim]
-  const uint16_t *v_pool;
+  const uint16_t *v_pool;      // (FP8 pools: the code blocks, through their TMA maps)
+  const int8_t *kv_exp;        // FP8 pools: the layer's exponents (else null)
   const int32_t *page_table;   // [batch][max_pages]
   const int32_t *num_slots;    // [batch] of this layer
   const uint16_t *q;           // [batch][n_q_heads][head_dim]
@@ -103,7 +138,8 @@ struct AttnView {
 };
 
 struct AppendView {
-  uint16_t *k_pool, *v_pool;   // this layer
+  uint16_t *k_pool, *v_pool;   // this layer (FP8 pools: uint8 codes, V transposed per page)
+  int8_t *kv_exp;              // FP8 pools: the layer's exponents (else null)
   int32_t *slot_pos, *slot_ntok;
   const int32_t *page_table;
   int32_t *num_slots;          // [batch] of this layer
@@ -122,7 +158,8 @@ struct AppendView {
 };
 
 struct FillView {
-  uint16_t *k_pool, *v_pool;
+  uint16_t *k_pool, *v_pool;   // (FP8 pools: uint8 codes, V transposed per page)
+  int8_t *kv_exp;              // FP8 pools: the layer's exponents (else null)
   int32_t *slot_pos, *slot_ntok;
   const int32_t *page_table;
   int32_t *num_slots;
@@ -144,7 +181,7 @@ cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, con
 // CTAs of one SM for the attention kernel of this shape and output type (0 if the shape is not
 // compiled).
 int attention_ctas_per_sm(int head_dim, int group, int batch, bool step,
-                          int out_dtype = HAM_DTYPE_BF16);
+                          int out_dtype = HAM_DTYPE_BF16, bool fp8 = false);
 // Set the shared-memory attribute of every compiled attention instance of the plain (non-step)
 // kernel, for the current device: bf16 and fp32 output at head_dim 64 and 128.  Later launches
 // of those instances then make no attribute call.
@@ -193,6 +230,35 @@ cudaError_t launch_append(const AppendView &v, cudaStream_t stream);
 int append_kv_per_block(int n_q_heads, int n_kv_heads, int head_dim);
 cudaError_t launch_fill(const FillView &v, cudaStream_t stream);
 
+// TMA maps of one layer's FP8 code blocks: K [rows][128] uint8 with a box of {128, 16 rows}
+// and the 128-byte swizzle; V [rows_d = pages * Hkv * 128][page_slots] uint8 with a box of
+// {16 slots, 128 rows} (one chunk's value rows, transposed), no swizzle.  Return a CUresult.
+int make_fp8_k_tensor_map(CUtensorMap *map, const void *k_codes, int64_t rows);
+int make_fp8_v_tensor_map(CUtensorMap *map, const void *v_codes, int64_t rows_d, int page_slots);
+
+// One row of 128 values (element 4 * lane + i in x[i] of lane `lane`, every lane of the warp
+// taking part) encoded as e4m3 codes with a power-of-two scale 2^e: e = E - 8 for the row's
+// largest magnitude m 2^E (0.5 <= m < 1), clamped to [-124, 119], 0 for a zero row; each element
+// x 2^-e (exact) rounded to nearest even with saturation at +-448 by the hardware conversion.
+// Returns e; `codes` gets the lane's four codes, element 4 * lane + i in byte i.
+__device__ inline int encode_e4m3_row(const float (&x)[4], uint32_t &codes) {
+  float a = fmaxf(fmaxf(fabsf(x[0]), fabsf(x[1])), fmaxf(fabsf(x[2]), fabsf(x[3])));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
+  int e = 0;
+  if (a > 0.f) {
+    int E = 0;
+    frexpf(a, &E);
+    e = min(max(E - 8, kFp8ExpMin), kFp8ExpMax);
+  }
+  const __nv_fp8x2_storage_t lo = __nv_cvt_float2_to_fp8x2(
+      make_float2(ldexpf(x[0], -e), ldexpf(x[1], -e)), __NV_SATFINITE, __NV_E4M3);
+  const __nv_fp8x2_storage_t hi = __nv_cvt_float2_to_fp8x2(
+      make_float2(ldexpf(x[2], -e), ldexpf(x[3], -e)), __NV_SATFINITE, __NV_E4M3);
+  codes = (uint32_t)lo | ((uint32_t)hi << 16);
+  return e;
+}
+
 // Record `msg` as this thread's ham_last_error() and return `status`.
 int set_last_error(int status, const char *msg);
 
@@ -214,8 +280,9 @@ struct ham_kv {
   int32_t default_ctas = 0;     // SMs x resident attention CTAs per SM (set at allocation)
   int32_t default_step_ctas = 0;  // same for the fused decode step
   int32_t max_ctas = 0;         // scratch is sized for this many CTAs
-  int64_t pool_elems = 0;       // bf16 elements of ONE pool (K or V) of one layer
-  uint16_t *pool = nullptr;     // [layers][2][pool_elems]
+  int64_t pool_elems = 0;       // elements of ONE pool (K or V) of one layer
+  int32_t fp8 = 0;              // 1: FP8 (e4m3) pools (kv_dtype HAM_KV_E4M3)
+  uint16_t *pool = nullptr;     // bf16: [layers][2][pool_elems]; FP8: [layers] x fp8_layer_bytes
   uint8_t *meta = nullptr;      // everything else, carved below
   int32_t *slot_pos = nullptr, *slot_ntok = nullptr, *page_table = nullptr;
   int32_t *num_slots = nullptr; // [layers][batch]

@@ -88,8 +88,29 @@ struct DeviceGuard {
   }
 };
 
+int64_t pool_rows(const ham_kv *kv) {
+  return kv->cfg.pool_pages * kv->cfg.n_kv_heads * (int64_t)kv->cfg.page_slots;
+}
+
+// The K (which 0) or V (1) pool of a layer: bf16 elements, or for FP8 pools the code block
+// (uint8, behind a uint16_t pointer that nothing dereferences as bf16).
 uint16_t *layer_pool(const ham_kv *kv, int32_t layer, int which) {
+  if (kv->fp8) {
+    const ham::Fp8Layer f = ham::fp8_layer(kv->pool, pool_rows(kv), layer);
+    return reinterpret_cast<uint16_t *>(which ? f.v : f.k);
+  }
   return kv->pool + ((size_t)layer * 2 + (size_t)which) * (size_t)kv->pool_elems;
+}
+int8_t *layer_exp(const ham_kv *kv, int32_t layer) {
+  return kv->fp8 ? ham::fp8_layer(kv->pool, pool_rows(kv), layer).e : nullptr;
+}
+// Bytes of one layer's pools.
+size_t layer_pool_bytes(const ham_kv *kv) {
+  return kv->fp8 ? ham::fp8_layer_bytes(pool_rows(kv))
+                 : 2 * (size_t)kv->pool_elems * sizeof(uint16_t);
+}
+int fp8_unsupported(const ham_kv *kv, const char *call) {
+  return kv->fp8 ? fail(HAM_EUNSUPPORTED, "%s: not available for an FP8 (e4m3) cache", call) : 0;
 }
 
 // ---------------------------------------------------------------------------------------
@@ -214,6 +235,47 @@ __global__ void fill_rows_kernel(FillView v) {
   }
 }
 
+// FP8 pools: one warp per (sequence b, slot j, KV head g) row pair; the K and the V row are
+// each encoded (encode_e4m3_row) and stored as codes (V transposed within its page) and
+// exponents.  Blocks of 8 warps; grid (ceil(lmax * Hkv / 8), batch).
+__global__ void fill_rows_fp8_kernel(FillView v) {
+  const int32_t b = blockIdx.y;
+  const int32_t count = v.counts[b];
+  if (count < 0 || count > v.lmax || count > v.max_slots) return;  // reported by fill_meta
+  const int lane = threadIdx.x & 31;
+  const int64_t r = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int32_t j = (int32_t)(r / v.n_kv_heads), g = (int32_t)(r % v.n_kv_heads);
+  if (j >= count) return;
+  const int32_t page = v.page_table[(int64_t)b * v.max_pages + j / v.page_slots];
+  if (page < 0 || page >= v.pool_pages) {
+    if (lane == 0) record_error(v.err, HAM_DEVERR_PAGE);
+    return;
+  }
+  const int P = v.page_slots, s = j % P;
+  const int64_t src = (((int64_t)b * v.lmax + j) * v.n_kv_heads + g) * kFp8HeadDim + 4 * lane;
+  const int64_t ph = (int64_t)page * v.n_kv_heads + g;  // (page, head) block
+  float xk[4], xv[4];
+  const uint2 kb = *reinterpret_cast<const uint2 *>(v.k_log + src);
+  const uint2 vb = *reinterpret_cast<const uint2 *>(v.v_log + src);
+  xk[0] = __uint_as_float(kb.x << 16); xk[1] = __uint_as_float(kb.x & 0xFFFF0000u);
+  xk[2] = __uint_as_float(kb.y << 16); xk[3] = __uint_as_float(kb.y & 0xFFFF0000u);
+  xv[0] = __uint_as_float(vb.x << 16); xv[1] = __uint_as_float(vb.x & 0xFFFF0000u);
+  xv[2] = __uint_as_float(vb.y << 16); xv[3] = __uint_as_float(vb.y & 0xFFFF0000u);
+  uint32_t ck, cv;
+  const int ek = encode_e4m3_row(xk, ck), ev = encode_e4m3_row(xv, cv);
+  uint8_t *kc = reinterpret_cast<uint8_t *>(v.k_pool), *vc = reinterpret_cast<uint8_t *>(v.v_pool);
+  *reinterpret_cast<uint32_t *>(kc + (ph * P + s) * kFp8HeadDim + 4 * lane) = ck;
+  const int sv = s - s % kChunkSlots + fp8_v_slot_byte(s % kChunkSlots);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    vc[(ph * kFp8HeadDim + 4 * lane + i) * P + sv] = (uint8_t)(cv >> (8 * i));
+  if (lane == 0) {
+    int8_t *e = v.kv_exp + (ph * (P / kChunkSlots) + s / kChunkSlots) * 32 + s % kChunkSlots;
+    e[0] = (int8_t)ek;
+    e[kChunkSlots] = (int8_t)ev;
+  }
+}
+
 __global__ void fill_meta_kernel(FillView v) {
   const int32_t b = blockIdx.x;
   const int32_t count = v.counts[b];
@@ -320,6 +382,32 @@ int make_parts_tensor_map(CUtensorMap *map, void *base, int splits, int64_t rows
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+int make_fp8_k_tensor_map(CUtensorMap *map, const void *k_codes, int64_t rows) {
+  EncodeTiled encode = tensor_map_encoder();
+  if (!encode) return -1;
+  const cuuint64_t dims[2] = {(cuuint64_t)kFp8HeadDim, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)kFp8HeadDim};  // bytes of a row
+  const cuuint32_t box[2] = {(cuuint32_t)kFp8HeadDim, (cuuint32_t)kChunkSlots};
+  const cuuint32_t estride[2] = {1, 1};
+  return (int)encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(k_codes), dims,
+                     strides, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+int make_fp8_v_tensor_map(CUtensorMap *map, const void *v_codes, int64_t rows_d, int page_slots) {
+  EncodeTiled encode = tensor_map_encoder();
+  if (!encode) return -1;
+  const cuuint64_t dims[2] = {(cuuint64_t)page_slots, (cuuint64_t)rows_d};
+  const cuuint64_t strides[1] = {(cuuint64_t)page_slots};  // bytes of a (page, head, d) row
+  const cuuint32_t box[2] = {(cuuint32_t)kChunkSlots, (cuuint32_t)kFp8HeadDim};
+  const cuuint32_t estride[2] = {1, 1};
+  return (int)encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(v_codes), dims,
+                     strides, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int head_dim,
                          bool half_box) {
   EncodeTiled encode = tensor_map_encoder();
@@ -336,7 +424,12 @@ int make_pool_tensor_map(CUtensorMap *map, const void *pool, int64_t rows, int h
 }
 
 cudaError_t launch_fill(const FillView &v, cudaStream_t stream) {
-  if (v.lmax > 0) {
+  if (v.lmax > 0 && v.kv_exp) {
+    dim3 grid((unsigned)(((int64_t)v.lmax * v.n_kv_heads + 7) / 8), (unsigned)v.batch);
+    fill_rows_fp8_kernel<<<grid, 256, 0, stream>>>(v);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  } else if (v.lmax > 0) {
     dim3 grid((unsigned)((v.lmax + 15) / 16), (unsigned)v.batch);
     fill_rows_kernel<<<grid, 256, 0, stream>>>(v);
     cudaError_t e = cudaGetLastError();
@@ -373,6 +466,11 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
     return fail(HAM_EINVAL, "pos_mode %d", cfg.pos_mode);
   if (!(cfg.rope_base > 1.0) || !std::isfinite(cfg.rope_base))
     return fail(HAM_EINVAL, "rope_base must be finite and > 1");
+  if (cfg.kv_dtype != HAM_KV_BF16 && cfg.kv_dtype != HAM_KV_E4M3)
+    return fail(HAM_EINVAL, "kv_dtype %d", cfg.kv_dtype);
+  if (cfg.kv_dtype == HAM_KV_E4M3 && cfg.head_dim != ham::kFp8HeadDim)
+    return fail(HAM_EUNSUPPORTED, "FP8 pools: head_dim %d (only %d is compiled)", cfg.head_dim,
+                ham::kFp8HeadDim);
   const int group = cfg.n_q_heads / cfg.n_kv_heads;
   if (!ham::attention_supported(cfg.head_dim, group) ||
       ham::append_kv_per_block(cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim) == 0)
@@ -393,6 +491,10 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   // TMA row coordinates of the pools are int32
   if (cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots > INT32_MAX)
     return fail(HAM_EINVAL, "pool_pages * n_kv_heads * page_slots above int32 range");
+  // FP8: the transposed value blocks are addressed by (page, head, element) rows
+  if (cfg.kv_dtype == HAM_KV_E4M3 &&
+      cfg.pool_pages * cfg.n_kv_heads * (int64_t)ham::kFp8HeadDim > INT32_MAX)
+    return fail(HAM_EINVAL, "pool_pages * n_kv_heads * 128 above int32 range");
 
   int dev = 0;
   HAM_CUDA(cudaGetDevice(&dev));
@@ -406,20 +508,23 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->max_pages = (int32_t)max_pages;
   kv->max_ctas = 8 * sms;
   kv->pool_elems = cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots * cfg.head_dim;
+  kv->fp8 = cfg.kv_dtype == HAM_KV_E4M3 ? 1 : 0;
 
-  const size_t pool_bytes = (size_t)cfg.layers * 2 * (size_t)kv->pool_elems * sizeof(uint16_t);
+  const size_t pool_bytes = (size_t)cfg.layers * layer_pool_bytes(kv);
   const MetaLayout lay = meta_layout(cfg, kv->max_ctas, max_pages);
   const size_t off = lay.total;
   kv->scratch_bytes = (int64_t)(off - lay.acc);
 
   {
-    const int per_sm = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, false);
+    const int per_sm = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, false,
+                                                  HAM_DTYPE_BF16, kv->fp8 != 0);
     const int per_sm_step = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, true);
     if (per_sm <= 0 || per_sm_step <= 0) {
       delete kv;
       return fail(HAM_ECUDA, "attention kernel cannot be resident on an SM");
     }
-    kv->default_ctas = std::min(ham::default_attention_ctas(sms, per_sm), kv->max_ctas);
+    kv->default_ctas =
+        std::min(ham::default_attention_ctas(sms, per_sm, kv->fp8 != 0), kv->max_ctas);
     kv->default_step_ctas = std::min(ham::default_attention_ctas(sms, per_sm_step), kv->max_ctas);
   }
   cudaError_t e = cudaMalloc(&kv->pool, pool_bytes);
@@ -450,7 +555,8 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->prefill_seq = reinterpret_cast<int4 *>(kv->meta + lay.pf_seq);
   kv->prefill_pos = reinterpret_cast<int32_t *>(kv->meta + lay.pf_pos);
 
-  // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits.
+  // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits (FP8:
+  // zero codes and exponents, the encoding of a zero row).
   e = cudaMemset(kv->pool, 0, pool_bytes);
   if (e == cudaSuccess) e = cudaMemset(kv->meta, 0, off);
   std::vector<int32_t> pt = reserve_pages(cfg.batch, kv->max_pages, cfg.pool_pages, cfg.page_seed);
@@ -508,6 +614,19 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->tmaps_half.resize((size_t)cfg.layers * 2);
   const int64_t rows = cfg.pool_pages * cfg.n_kv_heads * (int64_t)cfg.page_slots;
   for (int layer = 0; layer < cfg.layers; ++layer) {
+    if (kv->fp8) {  // the code blocks; the half-box maps (prefill) stay unused
+      const ham::Fp8Layer f = ham::fp8_layer(kv->pool, rows, layer);
+      int r = ham::make_fp8_k_tensor_map(&kv->tmaps[(size_t)layer * 2], f.k, rows);
+      if (r == 0)
+        r = ham::make_fp8_v_tensor_map(&kv->tmaps[(size_t)layer * 2 + 1], f.v,
+                                       rows / cfg.page_slots * ham::kFp8HeadDim, cfg.page_slots);
+      memset(&kv->tmaps_half[(size_t)layer * 2], 0, 2 * sizeof(CUtensorMap));
+      if (r != 0) {
+        ham_kv_free(kv);
+        return fail(HAM_ECUDA, "cuTensorMapEncodeTiled failed (CUresult %d)", r);
+      }
+      continue;
+    }
     for (int which = 0; which < 2; ++which) {
       int r = ham::make_pool_tensor_map(&kv->tmaps[(size_t)layer * 2 + which],
                                         layer_pool(kv, layer, which), rows, cfg.head_dim, false);
@@ -546,7 +665,7 @@ int ham_kv_get_info(const ham_kv *kv, ham_kv_info *info) {
   info->attn_ctas = kv->attn_ctas > 0 ? kv->attn_ctas : kv->default_ctas;
   info->num_sms = kv->num_sms;
   info->device = kv->device;
-  info->pool_bytes = 2 * kv->pool_elems * (int64_t)sizeof(uint16_t);
+  info->pool_bytes = (int64_t)layer_pool_bytes(kv);
   info->scratch_bytes = kv->scratch_bytes;
   return HAM_OK;
 }
@@ -582,6 +701,7 @@ int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
   ham::AppendView v{};
   v.k_pool = layer_pool(kv, layer, 0);
   v.v_pool = layer_pool(kv, layer, 1);
+  v.kv_exp = layer_exp(kv, layer);
   v.slot_pos = kv->slot_pos;
   v.slot_ntok = kv->slot_ntok;
   v.page_table = kv->page_table;
@@ -626,6 +746,7 @@ int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int3
   ham::AttnView v{};
   v.k_pool = layer_pool(kv, layer, 0);
   v.v_pool = layer_pool(kv, layer, 1);
+  v.kv_exp = layer_exp(kv, layer);
   v.page_table = kv->page_table;
   v.num_slots = kv->num_slots + (size_t)layer * kv->cfg.batch;
   v.q = static_cast<const uint16_t *>(q);
@@ -664,6 +785,7 @@ int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, 
                    const int32_t *pos, const int32_t *ntok, void *q_rot, void *stream) {
   int rc = check_layer(kv, layer);
   if (rc) return rc;
+  if ((rc = fp8_unsupported(kv, "ham_qkv_append")) != 0) return rc;
   if (!x || !w_qkv || !ntok || !q_rot) return fail(HAM_EINVAL, "x, w_qkv, ntok and q_rot are required");
   if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(q_rot))
     return fail(HAM_EINVAL, "x, w_qkv and q_rot must be 16-byte aligned");
@@ -725,6 +847,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
                     int32_t out_dtype, void *stream) {
   int rc = check_layer(kv, layer);
   if (rc) return rc;
+  if ((rc = fp8_unsupported(kv, "ham_decode_step")) != 0) return rc;
   if (!q || !k_new || !v_new || !ntok || !out)
     return fail(HAM_EINVAL, "q, k_new, v_new, ntok and out are required");
   if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
@@ -798,6 +921,7 @@ int ham_micro_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const 
                    int32_t out_dtype, void *stream) {
   int rc = check_layer(kv, layer);
   if (rc) return rc;
+  if ((rc = fp8_unsupported(kv, "ham_micro_step")) != 0) return rc;
   if (!q || !k_new || !v_new || !ntok || !out)
     return fail(HAM_EINVAL, "q, k_new, v_new, ntok and out are required");
   if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
@@ -865,6 +989,7 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
                 int32_t total_rows, void *out, int32_t out_dtype, void *stream) {
   int rc = check_layer(kv, layer);
   if (rc) return rc;
+  if ((rc = fp8_unsupported(kv, "ham_prefill")) != 0) return rc;
   if (out_dtype != HAM_DTYPE_BF16 && out_dtype != HAM_DTYPE_F32)
     return fail(HAM_EINVAL, "out_dtype %d", out_dtype);
   const ham_config &c = kv->cfg;
@@ -1021,6 +1146,7 @@ int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
   ham::FillView v{};
   v.k_pool = layer_pool(kv, layer, 0);
   v.v_pool = layer_pool(kv, layer, 1);
+  v.kv_exp = layer_exp(kv, layer);
   v.slot_pos = kv->slot_pos;
   v.slot_ntok = kv->slot_ntok;
   v.page_table = kv->page_table;
@@ -1052,12 +1178,23 @@ int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *
   if (rc) return rc;
   DeviceGuard guard(kv->device);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const size_t pool_bytes = (size_t)kv->pool_elems * sizeof(uint16_t);
+  const size_t pool_bytes = (size_t)kv->pool_elems * (kv->fp8 ? 1 : sizeof(uint16_t));
   const size_t meta_bytes = (size_t)kv->cfg.pool_pages * kv->cfg.page_slots * sizeof(int32_t);
   if (k_dst) HAM_CUDA(cudaMemcpyAsync(k_dst, layer_pool(kv, layer, 0), pool_bytes, cudaMemcpyDefault, s));
   if (v_dst) HAM_CUDA(cudaMemcpyAsync(v_dst, layer_pool(kv, layer, 1), pool_bytes, cudaMemcpyDefault, s));
   if (pos_dst) HAM_CUDA(cudaMemcpyAsync(pos_dst, kv->slot_pos, meta_bytes, cudaMemcpyDefault, s));
   if (ntok_dst) HAM_CUDA(cudaMemcpyAsync(ntok_dst, kv->slot_ntok, meta_bytes, cudaMemcpyDefault, s));
+  return HAM_OK;
+}
+
+int ham_kv_export_scales(ham_kv *kv, int32_t layer, void *e_dst, void *stream) {
+  int rc = check_layer(kv, layer);
+  if (rc) return rc;
+  if (!kv->fp8) return fail(HAM_EINVAL, "not an FP8 cache");
+  if (!e_dst) return fail(HAM_EINVAL, "e_dst is required");
+  DeviceGuard guard(kv->device);
+  HAM_CUDA(cudaMemcpyAsync(e_dst, layer_exp(kv, layer), (size_t)pool_rows(kv) * 2,
+                           cudaMemcpyDefault, static_cast<cudaStream_t>(stream)));
   return HAM_OK;
 }
 

@@ -27,6 +27,7 @@ STATUS_NAMES = {0: "HAM_OK", 1: "HAM_EINVAL", 2: "HAM_ENOMEM", 3: "HAM_ECAPACITY
  HAM_DEVERR_TIMEOUT) = range(6)
 HAM_POS_SLOT, HAM_POS_TOKEN = 0, 1
 HAM_DTYPE_BF16, HAM_DTYPE_F32 = 0, 1
+HAM_KV_BF16, HAM_KV_E4M3 = 0, 1
 
 
 class HamError(RuntimeError):
@@ -41,7 +42,7 @@ class ham_config(ctypes.Structure):
                 ("head_dim", ctypes.c_int32), ("page_slots", ctypes.c_int32),
                 ("max_slots_per_seq", ctypes.c_int32), ("pos_mode", ctypes.c_int32),
                 ("pool_pages", ctypes.c_int64), ("rope_base", ctypes.c_double),
-                ("page_seed", ctypes.c_uint64)]
+                ("page_seed", ctypes.c_uint64), ("kv_dtype", ctypes.c_int32)]
 
 
 class ham_attn_args(ctypes.Structure):
@@ -89,6 +90,7 @@ _SIGNATURES = {
     "ham_kv_get_page_table": [_vp, _vp],
     "ham_kv_fill": [_vp, _i32, _vp, _vp, _vp, _vp, _vp, _i32, _vp],
     "ham_kv_export": [_vp, _i32, _vp, _vp, _vp, _vp, _vp],
+    "ham_kv_export_scales": [_vp, _i32, _vp, _vp],
     "ham_kv_reset": [_vp, _vp],
     "ham_kv_set_lengths": [_vp, _i32, _vp, _vp, _vp],
     "ham_kv_set_attn_ctas": [_vp, _i32],
@@ -179,6 +181,7 @@ class KV:
         self.n_q_heads, self.n_kv_heads, self.head_dim = c.n_q_heads, c.n_kv_heads, c.head_dim
         self.page_slots, self.max_slots = c.page_slots, c.max_slots_per_seq
         self.pool_pages = c.pool_pages
+        self.kv_dtype = c.kv_dtype
         self.max_pages = self.info.max_pages_per_seq
 
     @property
@@ -202,9 +205,9 @@ class KV:
 
 def ham_kv_alloc(layers, batch, n_q_heads, n_kv_heads, head_dim, page_slots,
                  max_slots_per_seq, pos_mode=HAM_POS_SLOT, pool_pages=0, rope_base=10000.0,
-                 page_seed=0) -> KV:
+                 page_seed=0, kv_dtype=0) -> KV:
     cfg = ham_config(layers, batch, n_q_heads, n_kv_heads, head_dim, page_slots,
-                     max_slots_per_seq, pos_mode, pool_pages, rope_base, page_seed)
+                     max_slots_per_seq, pos_mode, pool_pages, rope_base, page_seed, kv_dtype)
     out = ctypes.c_void_p()
     _check(lib().ham_kv_alloc(ctypes.byref(cfg), ctypes.byref(out)))
     return KV(out.value)
@@ -357,16 +360,31 @@ def ham_kv_fill(kv: KV, layer, k_log, v_log, counts, pos=None, ntok=None, stream
 
 
 def ham_kv_export(kv: KV, layer, stream=None):
-    """Copy one layer's raw pools and slot metadata into new device tensors."""
+    """Copy one layer's raw pools and slot metadata into new device tensors (FP8 pools: uint8
+    codes, K [pages][Hkv][P][d] and V [pages][Hkv][d][P])."""
     import torch
     shape = (kv.pool_pages, kv.n_kv_heads, kv.page_slots, kv.head_dim)
-    k = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
-    v = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
+    if kv.kv_dtype == HAM_KV_E4M3:
+        k = torch.empty(shape, dtype=torch.uint8, device="cuda")
+        v = torch.empty((kv.pool_pages, kv.n_kv_heads, kv.head_dim, kv.page_slots),
+                        dtype=torch.uint8, device="cuda")
+    else:
+        k = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
+        v = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
     pos = torch.empty((kv.pool_pages, kv.page_slots), dtype=torch.int32, device="cuda")
     ntok = torch.empty_like(pos)
     _check(lib().ham_kv_export(kv, layer, k.data_ptr(), v.data_ptr(), pos.data_ptr(),
                                ntok.data_ptr(), _stream_ptr(stream)))
     return k, v, pos, ntok
+
+
+def ham_kv_export_scales(kv: KV, layer, stream=None):
+    """One layer's exponent array of an FP8 cache: int8 [pages][Hkv][P/16][2][16]."""
+    import torch
+    e = torch.empty((kv.pool_pages, kv.n_kv_heads, kv.page_slots // 16, 2, 16),
+                    dtype=torch.int8, device="cuda")
+    _check(lib().ham_kv_export_scales(kv, layer, e.data_ptr(), _stream_ptr(stream)))
+    return e
 
 
 def ham_kv_set_lengths(kv: KV, layer, num_slots, num_tokens=None, stream=None):

@@ -38,7 +38,8 @@ def test_python_binding_covers_every_symbol():
 
 def _cfg(**kw):
     base = dict(layers=1, batch=2, n_q_heads=8, n_kv_heads=2, head_dim=64, page_slots=16,
-                max_slots_per_seq=64, pos_mode=0, pool_pages=0, rope_base=10000.0, page_seed=0)
+                max_slots_per_seq=64, pos_mode=0, pool_pages=0, rope_base=10000.0, page_seed=0,
+                kv_dtype=0)
     base.update(kw)
     return ham.ham_config(**base)
 
@@ -56,6 +57,9 @@ def _cfg(**kw):
     (dict(head_dim=96), ham.HAM_EUNSUPPORTED),
     (dict(n_q_heads=32, n_kv_heads=2), ham.HAM_EUNSUPPORTED),
     (dict(pool_pages=3), ham.HAM_ECAPACITY),
+    (dict(kv_dtype=7), ham.HAM_EINVAL),
+    (dict(kv_dtype=ham.HAM_KV_E4M3), ham.HAM_EUNSUPPORTED),           # FP8 pools: head_dim 128
+    (dict(kv_dtype=ham.HAM_KV_E4M3, head_dim=128, pool_pages=3), ham.HAM_ECAPACITY),
 ])
 def test_alloc_rejects_bad_configs_on_the_host(libham, kw, status):
     out = ctypes.c_void_p(123)
@@ -71,6 +75,7 @@ def test_null_arguments_are_rejected(libham):
     assert libham.ham_kv_alloc(None, ctypes.byref(out)) == ham.HAM_EINVAL
     assert libham.ham_kv_free(None) == ham.HAM_OK
     assert libham.ham_decode_attn(None, 0, None, None, None) == ham.HAM_EINVAL
+    assert libham.ham_kv_export_scales(None, 0, None, None) == ham.HAM_EINVAL
     assert libham.ham_kv_append(None, 0, None, None, None, None, None, None) == ham.HAM_EINVAL
     assert libham.ham_prefill(None, 0, None, None, None, None, None, None, 0, None, 0,
                               None) == ham.HAM_EINVAL

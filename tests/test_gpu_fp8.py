@@ -1,0 +1,269 @@
+"""GPU: FP8 (e4m3) pools.  The stored codes and exponents match the oracle's encoder bit for
+bit (after a fill and after appends), and decode attention over an FP8 pool matches the oracle
+run on the decoded rows (every decoded value is an exact bf16 value) at the usual bar."""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import fp8
+from oracle.embedder import bf16_bits_to_f64
+from paper_2505_20438_gb300 import ham
+from paper_2505_20438_gb300 import workload as wl
+
+from gpu_helpers import (assert_parity, dev_bf16, dev_i32, host_bits, small_case, torch)
+
+pytestmark = pytest.mark.gpu
+
+F32_MAX, F32_MEAN = 3e-3, 3e-4
+
+
+def _bits_f64(bits):
+    return bf16_bits_to_f64(bits)
+
+
+def _to_bits(x):
+    """Input rows: fp64 values to bf16 bits through the generators' own conversion."""
+    return wl.f32_to_bf16_bits(np.asarray(x, np.float64).astype(np.float32))
+
+
+def _decoded(bits):
+    """bf16 bits of the rows an FP8 pool holds for these bf16 rows ([..., d] bits)."""
+    codes, es = fp8.encode_rows(_bits_f64(bits))
+    return fp8.decoded_bf16_bits(codes, es)
+
+
+# byte of slot s of a chunk within the transposed value rows (ham.h): slots 0, 1, 8, 9, 2, 3, ...
+V_SLOT_BYTE = np.array([4 * ((s % 8) // 2) + 2 * (s // 8) + s % 2 for s in range(16)])
+
+
+def _expected_pools(k_pool_bits, v_pool_bits):
+    """Expected FP8 export of an oracle layer's bf16 pools [pages][Hkv][P][d]: K codes, V codes
+    transposed per page (a chunk's slots in the documented order), exponents
+    [pages][Hkv][P/16][2][16]."""
+    kc, ke = fp8.encode_rows(_bits_f64(k_pool_bits))
+    vc, ve = fp8.encode_rows(_bits_f64(v_pool_bits))
+    pages, hkv, P, d = kc.shape
+    e = np.stack([ke.reshape(pages, hkv, P // 16, 16), ve.reshape(pages, hkv, P // 16, 16)], axis=3)
+    vt = vc.transpose(0, 1, 3, 2).reshape(pages, hkv, d, P // 16, 16)
+    vp = np.empty_like(vt)
+    vp[..., V_SLOT_BYTE] = vt
+    return kc, np.ascontiguousarray(vp.reshape(pages, hkv, d, P)), e.astype(np.int8)
+
+
+def fp8_cache(case, layers=1, pos_mode=ham.HAM_POS_SLOT, fill=True):
+    w = case.w
+    kv = ham.ham_kv_alloc(layers, w.batch, w.n_q_heads, w.n_kv_heads, w.head_dim, w.page_slots,
+                          case.max_slots, pos_mode=pos_mode, pool_pages=case.pool_pages,
+                          kv_dtype=ham.HAM_KV_E4M3)
+    ham.ham_kv_set_page_table(kv, case.page_table)
+    if fill:
+        for layer in range(layers):
+            ham.ham_kv_fill(kv, layer, dev_bf16(case.k), dev_bf16(case.v),
+                            dev_i32(case.num_slots), pos=dev_i32(case.slot_pos),
+                            ntok=dev_i32(case.slot_ntok))
+    return kv
+
+
+def _export(kv, layer=0):
+    k, v, pos, ntok = ham.ham_kv_export(kv, layer)
+    e = ham.ham_kv_export_scales(kv, layer)
+    return (k.cpu().numpy(), v.cpu().numpy(), e.cpu().numpy(), pos.cpu().numpy(),
+            ntok.cpu().numpy())
+
+
+def _decode(kv, q_bits, f32=False, layer=0):
+    t = torch()
+    q = dev_bf16(q_bits)
+    out = t.full(q.shape, float("nan"), dtype=t.float32 if f32 else t.bfloat16, device="cuda")
+    ham.ham_decode_attn_ex(kv, layer, q, out)
+    t.cuda.synchronize()
+    return out.float().cpu().numpy().astype(np.float64)
+
+
+def _reference(case):
+    """Oracle decode over the decoded rows of the case's cache."""
+    oc = oracle.OracleCache.from_case(case, fill=False)
+    oc.fill(_decoded(case.k), _decoded(case.v), case.slot_pos, case.slot_ntok, case.num_slots)
+    return oc
+
+
+@pytest.mark.parametrize("page,counts", [(16, (37, 80)), (32, (0, 100, 7)), (128, (255,))])
+def test_fill_stores_the_oracle_encoding(page, counts):
+    case = small_case(batch=len(counts), hq=32, hkv=8, d=128, page=page, counts=counts, seed=11)
+    oc = oracle.OracleCache.from_case(case)
+    kv = fp8_cache(case)
+    k, v, e, pos, ntok = _export(kv)
+    kc, vc, ee = _expected_pools(oc.k_pool, oc.v_pool)
+    assert np.array_equal(k, kc), "K codes"
+    assert np.array_equal(v, vc), "V codes (transposed)"
+    assert np.array_equal(e, ee), "exponents"
+    assert np.array_equal(pos, oc.slot_pos) and np.array_equal(ntok, oc.slot_ntok)
+    slots, tokens = ham.ham_slot_lengths(kv)
+    assert np.array_equal(slots, oc.num_slots) and np.array_equal(tokens, oc.num_tokens)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+def test_fill_encodes_extreme_row_scales():
+    """Rows whose largest magnitude ranges from bf16 subnormals to near the bf16 maximum: the
+    exponent clamps at both ends, saturation and signed zeros, bit for bit."""
+    case = small_case(batch=2, hq=8, hkv=2, d=128, page=16, counts=(40, 24), seed=12)
+    k = _bits_f64(case.k)
+    v = _bits_f64(case.v)
+    tops = 2.0 ** np.array([-133, -130, -126, -124, -117, -116, -60, 0, 30, 90, 118, 126, 127])
+    for i, top in enumerate(tops):
+        b, j = i % 2, 3 * i
+        k[b, j] *= top / np.abs(k[b, j]).max(axis=-1, keepdims=True)
+        v[b, j + 1] *= top / np.abs(v[b, j + 1]).max(axis=-1, keepdims=True)
+    k[0, 1, 0, :] = 0.0                       # a zero row
+    v[1, 2, 1, :8] = -0.0                     # negative zeros
+    k[1, 4, 0, :4] = -(2.0 ** -20) * k[1, 4, 0, :4] / np.abs(k[1, 4, 0, :4]).max()  # to -0 codes
+    case.k[...] = _to_bits(k)
+    case.v[...] = _to_bits(v)
+    oc = oracle.OracleCache.from_case(case)
+    kv = fp8_cache(case)
+    kk, vv, e, _, _ = _export(kv)
+    kc, vc, ee = _expected_pools(oc.k_pool, oc.v_pool)
+    assert np.array_equal(e, ee), "exponents"
+    assert np.array_equal(kk, kc), "K codes"
+    assert np.array_equal(vv, vc), "V codes"
+
+
+@pytest.mark.parametrize("pos_mode", [ham.HAM_POS_SLOT, ham.HAM_POS_TOKEN])
+@pytest.mark.parametrize("hq,hkv", [(32, 8), (8, 8), (32, 16)])
+def test_append_stores_the_oracle_encoding(pos_mode, hq, hkv):
+    """The rotated bf16 key (as a bf16 cache stores it) and the value, encoded bit for bit; q
+    turned in place as for a bf16 cache; several macro-steps crossing a page edge."""
+    case = small_case(batch=3, hq=hq, hkv=hkv, d=128, page=16, counts=(15, 16, 200), seed=13,
+                      extra_slots=8)
+    oc = oracle.OracleCache.from_case(case)
+    kv = fp8_cache(case, pos_mode=pos_mode)
+    q_host = case.q.copy()
+    q_dev = dev_bf16(case.q)
+    rng = wl.rng_for(13, 50)
+    for step in range(3):
+        k_new = wl.normal_bf16(rng, case.k_new.shape)
+        v_new = wl.normal_bf16(rng, case.v_new.shape)
+        ntok = wl.ntok_capped_geometric(rng, (case.w.batch,))
+        assert oc.append(k_new, v_new, ntok, q_inout=q_host, pos_mode=pos_mode) == 0
+        ham.ham_kv_append(kv, 0, q_dev, dev_bf16(k_new), dev_bf16(v_new), None, dev_i32(ntok))
+    k, v, e, pos, ntok_arr = _export(kv)
+    kc, vc, ee = _expected_pools(oc.k_pool, oc.v_pool)
+    assert np.array_equal(e, ee), "exponents"
+    assert np.array_equal(k, kc), "K codes of the rotated keys"
+    assert np.array_equal(v, vc), "V codes"
+    assert np.array_equal(pos, oc.slot_pos) and np.array_equal(ntok_arr, oc.slot_ntok)
+    assert np.array_equal(host_bits(q_dev), q_host)
+    slots, tokens = ham.ham_slot_lengths(kv)
+    assert np.array_equal(slots, oc.num_slots) and np.array_equal(tokens, oc.num_tokens)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+@pytest.mark.parametrize("hq,hkv,page,counts,scale", [
+    (32, 8, 16, (37, 80), 1.0),                       # ragged tails inside a chunk
+    (32, 8, 16, (1, 100, 1000), 1.0 / np.sqrt(128)),
+    (32, 8, 16, (0, 17, 0, 4097), 1.0),               # empty sequences
+    (32, 8, 32, (513, 2047), 1.0),
+    (32, 8, 128, (256, 3), 1.0),
+    (8, 8, 16, (300, 33), 1.0),                       # group 1
+    (16, 8, 16, (300, 33), 1.0),                      # group 2
+    (64, 8, 16, (300, 33), 1.0),                      # group 8
+    (24, 8, 16, (129, 64), 1.0),                      # group 3 (padded to 8)
+])
+def test_decode_over_fp8_matches_oracle(hq, hkv, page, counts, scale):
+    case = small_case(batch=len(counts), hq=hq, hkv=hkv, d=128, page=page, counts=counts,
+                      scale=scale, seed=sum(counts) % 89 + 3)
+    ref = _reference(case).decode_attn(case.q)
+    kv = fp8_cache(case)
+    out16 = _decode(kv, case.q)
+    out32 = _decode(kv, case.q, f32=True)
+    assert_parity(out16, ref, what="fp8 pool, bf16 out")
+    assert_parity(out32, ref, max_abs=F32_MAX, mean_abs=F32_MEAN, what="fp8 pool, f32 out")
+    for b, n in enumerate(counts):
+        if n == 0:
+            assert np.all(out16[b] == 0) and np.all(out32[b] == 0)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+def test_decode_over_fp8_rows_of_very_different_scales():
+    """Value rows whose scales differ by up to 2^40 across a sequence (the running value
+    exponent is raised mid-segment and O rescaled), keys of mixed scales, and queries whose
+    heads range from 2^-30 to 2^20."""
+    case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(700, 90, 1500), seed=31)
+    rng = wl.rng_for(31, 7)
+    k = _bits_f64(case.k)
+    v = _bits_f64(case.v)
+    L = k.shape[1]
+    vs = 2.0 ** rng.integers(-20, 21, size=(k.shape[0], L, 1, 1))
+    ks = 2.0 ** rng.integers(-6, 4, size=(k.shape[0], L, 1, 1))
+    case.k[...] = _to_bits(k * ks * 0.25)
+    case.v[...] = _to_bits(v * vs)
+    q = _bits_f64(case.q)
+    qs = 2.0 ** rng.integers(-30, 21, size=(q.shape[0], q.shape[1], 1))
+    qs[:, ::5] = 1.0
+    case.q[...] = _to_bits(np.clip(q * qs, -1e30, 1e30) * 2.0 ** -10)
+    ref = _reference(case).decode_attn(case.q)
+    kv = fp8_cache(case)
+    out32 = _decode(kv, case.q, f32=True)
+    # relative to each output row's size (the values span 2^40)
+    scale = np.maximum(np.abs(ref).max(axis=-1, keepdims=True), 1e-30)
+    err = np.abs(out32 - ref) / scale
+    assert np.all(np.isfinite(out32))
+    assert err.max() <= 3e-3, f"max relative {err.max():.3e}"
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+@pytest.mark.parametrize("ctas", [1, 7, 64, 600])
+def test_fp8_split_count_invariance(ctas):
+    case = small_case(batch=4, hq=32, hkv=8, d=128, page=16, counts=(1, 300, 2000, 45), seed=41)
+    ref = _reference(case).decode_attn(case.q)
+    kv = fp8_cache(case)
+    ham.ham_kv_set_attn_ctas(kv, ctas)
+    out = _decode(kv, case.q, f32=True)
+    assert_parity(out, ref, max_abs=F32_MAX, mean_abs=F32_MEAN, what=f"{ctas} CTAs")
+
+
+def test_fp8_append_then_decode():
+    """Macro-steps through ham_kv_append then ham_decode_attn on an FP8 cache agree with the
+    oracle's append followed by decoding over the decoded rows."""
+    case = small_case(batch=3, hq=32, hkv=8, d=128, page=16, counts=(31, 200, 64), seed=51,
+                      extra_slots=8)
+    oc = oracle.OracleCache.from_case(case)
+    kv = fp8_cache(case)
+    q_host = case.q.copy()
+    q_dev = dev_bf16(case.q)
+    rng = wl.rng_for(51, 9)
+    for step in range(4):
+        k_new = wl.normal_bf16(rng, case.k_new.shape)
+        v_new = wl.normal_bf16(rng, case.v_new.shape)
+        ntok = wl.ntok_capped_geometric(rng, (case.w.batch,))
+        assert oc.append(k_new, v_new, ntok, q_inout=q_host) == 0
+        ham.ham_kv_append(kv, 0, q_dev, dev_bf16(k_new), dev_bf16(v_new), None, dev_i32(ntok))
+    # the oracle's bf16 pools, decoded through the FP8 format, are the reference cache
+    ref_cache = oracle.OracleCache.from_case(case, fill=False)
+    ref_cache.k_pool[...] = _decoded(oc.k_pool)
+    ref_cache.v_pool[...] = _decoded(oc.v_pool)
+    ref_cache.slot_pos[...] = oc.slot_pos
+    ref_cache.slot_ntok[...] = oc.slot_ntok
+    ref_cache.num_slots[...] = oc.num_slots
+    ref_cache.num_tokens[...] = oc.num_tokens
+    ref = ref_cache.decode_attn(q_host)
+    out = _decode(kv, q_host)
+    assert_parity(out, ref, what="append then decode")
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+def test_fp8_unsupported_calls_are_refused():
+    case = small_case(batch=2, hq=8, hkv=2, d=128, page=16, counts=(5, 6), seed=61)
+    kv = fp8_cache(case)
+    t = torch()
+    q = dev_bf16(case.q)
+    out = t.empty_like(q)
+    with pytest.raises(ham.HamError) as e:
+        ham.ham_decode_step(kv, 0, q, dev_bf16(case.k_new), dev_bf16(case.v_new), None,
+                            dev_i32(case.ntok_new), out)
+    assert e.value.status == ham.HAM_EUNSUPPORTED
+    with pytest.raises(ham.HamError) as e:
+        ham.ham_kv_alloc(1, 2, 8, 2, 64, 16, 32, kv_dtype=ham.HAM_KV_E4M3)
+    assert e.value.status == ham.HAM_EUNSUPPORTED
+    slots, _ = ham.ham_slot_lengths(kv)
+    assert list(slots) == [5, 6]

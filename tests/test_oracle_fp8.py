@@ -169,3 +169,20 @@ def test_row_scale_at_the_ends_of_the_bf16_range(top):
         assert abs(back[0] - min(top, 448.0 * 2.0 ** 119)) <= top * 2.0 ** -4
     if top == 255.0 * 2.0 ** 120:
         assert back[0] == 448.0 * 2.0 ** 119           # 510 after scaling: saturated
+
+
+def test_encode_rows_is_encode_row_on_every_row():
+    """The vectorised encoding of many rows is the one-row encoding applied to each row, zero
+    rows, clamped exponents and both signs included."""
+    fp8 = _fp8()
+    rng = wl.rng_for(8, 0)
+    rows = wl.bf16_bits_to_f32(wl.normal_bf16(rng, (40, 32), 1.0)).astype(np.float64)
+    rows *= 2.0 ** rng.integers(-140, 130, size=(40, 1))
+    rows = np.clip(rows, -3.3e38, 3.3e38)
+    rows[3] = 0.0
+    rows[4, ::2] = -0.0
+    codes, es = fp8.encode_rows(rows.reshape(4, 10, 32))
+    assert codes.shape == (4, 10, 32) and es.shape == (4, 10)
+    for i, row in enumerate(rows):
+        c, e = fp8.encode_row(row)
+        assert np.array_equal(codes.reshape(40, 32)[i], c) and int(es.reshape(40)[i]) == e
