@@ -19,14 +19,19 @@
 //     lies within ~2^-44 (relative) of a rounding boundary.  This GPU's fp64 pipe would take
 //     about half a millisecond for a 16k-row chunk of a Llama-8B layer; the fp32 pairs take
 //     microseconds.
-//  3. prefill_attn_kernel, one CTA per (KV head, block of 128 / G query rows of one sequence):
-//     eight consumer warps, each one 16-row m-tile of one query head, and a producer warp that
-//     streams 64-slot K/V tiles (four 16-slot chunks, each 64-column half of a chunk one TMA
-//     copy with the 128-byte swizzle, so that ldmatrix reads are free of bank conflicts)
-//     through a shared-memory ring.  S = Q K^T and O += P V are mma.sync m16n8k16 (bf16 in, fp32
-//     accumulate); the softmax is online, fp32, in the exp2 domain; the causal mask applies to
-//     the tiles that reach past a row's own slot, and tiles past a warp's last row are skipped.
-//     CTAs are scheduled latest query block first, the longest rows of the causal triangle.
+//  3. prefill_attn_kernel, one CTA per (KV head, two Q tiles of 128 (query row, head) rows of
+//     one sequence), one CTA an SM: S = Q K^T and O += P V on the 5th-generation tensor cores
+//     (tcgen05.mma kind::f16, M = 128, bf16 operands, fp32 accumulators in tensor memory).
+//     Q, K and V reach shared memory by TMA (64-slot K/V tiles of four 16-slot chunks, each
+//     64-column half one box in the 128-byte swizzle; K and V in rings of their own, filled by
+//     two producer warps whose lanes issue the copies and look the pages up 32 chunks ahead).
+//     Two warps issue the S products of the two Q tiles and two the O products (one thread
+//     issues a tcgen05.mma only about every 125 cycles); eight softmax warps, one thread a row,
+//     read S from tensor memory, keep the online softmax in fp32 (exp2 domain, running maximum
+//     raised only past 2^8), write the bf16 probabilities to tensor memory columns of their own
+//     (the A operand of O += P V, so the next S is computed meanwhile) and rescale O there when
+//     the maximum moves.  The causal mask applies to the tiles that reach past a row's own slot;
+//     CTAs are scheduled latest query tiles first, the longest rows of the causal triangle.
 //
 // Every wait is bounded (about 2 s); a wait that runs out records HAM_DEVERR_TIMEOUT, lets the
 // CTA's copies land and returns.  No trap, no unbounded spin.
