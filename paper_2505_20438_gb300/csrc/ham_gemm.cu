@@ -6,8 +6,9 @@
 //   K_s the s-th of `splits` column ranges of whole 64-column tiles, as even as the tile count
 //   allows (the consumer sums the parts in a fixed order)
 //
-// One CTA per (128 output features, column range s, up to 128 rows; a last partial tile of
-// features or rows reads zeros past the matrix and stores nothing there), one CTA an SM: X is
+// One CTA per (128 output features, column range s, one or two row tiles of 128 rows: two when
+// the call has more than 128 rows; a last partial tile of features or rows reads zeros past the
+// matrix and stores nothing there), one CTA an SM: X is
 // the A operand (its rows in the TMEM lanes), W the B operand (N = 128 features), both K-major
 // 64-column tiles in the layout of the 128-byte swizzle, in two shared-memory rings.  W comes
 // either pre-tiled (tile_weights: each 128 x 64 tile one contiguous, already swizzled 16 KiB
@@ -49,21 +50,31 @@ constexpr int kGemmThreads = 11 * 32;
 constexpr int kGemmSmemBudget = 200 * 1024; // one CTA an SM: deep rings
 constexpr uint32_t kGemmTmemCols = 256;     // two accumulators of 128 columns
 constexpr int kGemmStages = 6;              // each ring: W tiles from HBM, X tiles from L2
+constexpr int kGemmStages2 = 4;             // the same with two row tiles a CTA
+
+// Row tiles a CTA: one up to 128 rows; above, two (both MMA warps then share each weight tile,
+// one accumulator each), so that a call's grid stays one wave and reads the weights half as often.
+inline int gemm_row_tiles(int rows) { return rows > kGemmRows ? 2 : 1; }
+constexpr int gemm_smem(int stages, int rt) {
+  return 1024 + stages * (kGemmWBytes + rt * kGemmXBytes) + (4 * stages + 1) * 8 + 16;
+}
+static_assert(gemm_smem(kGemmStages, 1) <= kGemmSmemBudget && gemm_smem(kGemmStages2, 2) <= kGemmSmemBudget,
+              "rings exceed the shared-memory budget");
+static_assert(kGemmStages2 * kGemmWBytes >= (kGemmM / 32) * 16384,
+              "the epilogue stages a row tile's 128 x 128 fp32 boxes in the weight ring");
 
 struct GemmPlan {
-  int nt, stages, smem;
+  int nt, rt, stages, smem;
 };
 
 GemmPlan gemm_plan(int rows) {
   GemmPlan p;
   p.nt = gemm_row_tile(rows);
-  p.stages = kGemmStages;
-  p.smem = 1024 + p.stages * (kGemmWBytes + kGemmXBytes) + (4 * p.stages + 1) * 8 + 16;
+  p.rt = gemm_row_tiles(rows);
+  p.stages = p.rt == 2 ? kGemmStages2 : kGemmStages;
+  p.smem = gemm_smem(p.stages, p.rt);
   return p;
 }
-static_assert(1024 + kGemmStages * (kGemmWBytes + kGemmXBytes) + (4 * kGemmStages + 1) * 8 + 16 <=
-                  kGemmSmemBudget,
-              "rings exceed the shared-memory budget");
 
 // Byte offset of element (r, k) of a 128-row x 64-column bf16 tile in the 128-byte swizzle (the
 // layout a TMA copy with that swizzle writes into 1024-byte aligned shared memory).
@@ -99,18 +110,22 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_xwt_kernel(const __grid_constant__ CUtensorMap tw, const uint8_t *__restrict__ wt,
                     int kt_total, const __grid_constant__ CUtensorMap tx,
                     const __grid_constant__ CUtensorMap ty, int tma_y, float *__restrict__ Y,
-                    int64_t ldy, int32_t *err, int rows, int F, int nt, int stages, int pdl) {
-  const int m0 = blockIdx.x * kGemmM, split = blockIdx.y, n0 = blockIdx.z * kGemmRows;
+                    int64_t ldy, int32_t *err, int rows, int F, int nt, int rt, int stages,
+                    int pdl) {
+  const int m0 = blockIdx.x * kGemmM, split = blockIdx.y, n0 = blockIdx.z * kGemmRows * rt;
   // k-tiles [kt0, kt1) of this split; columns past K read as zeros
   const int kt0 = (int)((int64_t)split * kt_total / gridDim.y);
   const int kt1 = (int)((int64_t)(split + 1) * kt_total / gridDim.y);
   const int k0 = kt0 * kGemmKTile, nk = kt1 - kt0;
-  const bool two = nk > 1;  // two accumulators (two issuing warps)
+  // one row tile: two accumulators for alternate k-tiles (two issuing warps) and their sum;
+  // two row tiles: one accumulator a row tile, every k-tile
+  const bool two = rt == 1 && nk > 1;
+  const int xs = rt * kGemmXBytes;  // an X stage
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t *wring = smem, *xring = smem + stages * kGemmWBytes;
-  uint64_t *w_full = reinterpret_cast<uint64_t *>(xring + stages * kGemmXBytes);
+  uint64_t *w_full = reinterpret_cast<uint64_t *>(xring + stages * xs);
   uint64_t *w_empty = w_full + stages, *x_full = w_empty + stages;
   uint64_t *x_empty = x_full + stages, *acc_full = x_empty + stages;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acc_full + 1);
@@ -121,9 +136,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   if (tid == 0) {
     for (int s = 0; s < stages; ++s) {
       mbar_init(&w_full[s], 1);
-      mbar_init(&w_empty[s], 1);
+      mbar_init(&w_empty[s], rt);  // every MMA warp that reads the stage commits
       mbar_init(&x_full[s], 1);
-      mbar_init(&x_empty[s], 1);
+      mbar_init(&x_empty[s], rt);
     }
     mbar_init(acc_full, 2);  // one commit per MMA warp
     *abort_flag = 0;
@@ -171,8 +186,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           wi = t + 1;
         }
         if (t >= stages && !thread_wait(&x_empty[s], par, abort_flag, true)) break;
-        mbar_arrive_tx(&x_full[s], (uint32_t)(nt * 128));
-        tma_load_2d(xring + s * kGemmXBytes, &tx, k0 + t * kGemmKTile, n0, &x_full[s], pol_x);
+        mbar_arrive_tx(&x_full[s], (uint32_t)(rt * nt * 128));
+        for (int r = 0; r < rt; ++r)  // (a row tile past the rows reads zeros)
+          tma_load_2d(xring + s * xs + r * kGemmXBytes, &tx, k0 + t * kGemmKTile,
+                      n0 + r * kGemmRows, &x_full[s], pol_x);
         xi = t + 1;
       }
       if (xi < nk && !*abort_flag) {  // a wait ran out
@@ -182,14 +199,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
   } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------------ MMA issue (lane 0)
-    // Two accumulators: warp 1 the even k-tiles into columns 0..127, warp 2 the odd ones into
-    // columns 128..255; a single k-tile: warp 1 alone.
+    // One row tile: warp 1 the even k-tiles into columns 0..127, warp 2 the odd ones into
+    // columns 128..255 (a single k-tile: warp 1 alone).  Two row tiles: warp 1 + r row tile r
+    // into columns 128 r.., every k-tile.
     const int par = warp - 1;
     const int step = two ? 2 : 1;
     const uint32_t acc = tmem + (uint32_t)(par * kGemmM);
     const uint32_t idesc = idesc_bf16(kGemmRows, kGemmM, false);  // K-major X and W
     bool ok = true, first = true;
-    const int t0 = two ? par : (par == 0 ? 0 : nk);
+    const int t0 = rt == 2 ? 0 : two ? par : (par == 0 ? 0 : nk);
+    const int xoff = rt == 2 ? par * kGemmXBytes : 0;
     for (int t = t0; t < nk; t += step) {
       const int s = t % stages;
       const uint32_t ph = (uint32_t)(t / stages) & 1u;
@@ -199,7 +218,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
       if (lane == 0) {
         tc_fence_after();
-        const uint32_t xa = smem_u32(xring + s * kGemmXBytes);
+        const uint32_t xa = smem_u32(xring + s * xs + xoff);
         const uint32_t wa = smem_u32(wring + s * kGemmWBytes);
 #pragma unroll
         for (int kk = 0; kk < kGemmKTile / 16; ++kk)
@@ -219,21 +238,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue (warps 3-10)
-    // Thread = TMEM lane = row n0 + r; the warp's half of the 128 features, 32 at a time (both
-    // accumulators added).  tcgen05.ld is warp-collective: every lane loads, lanes past the
-    // rows store nothing.
+    // Thread = TMEM lane = row of the row tile; the warp's half of the 128 features, 32 at a
+    // time (one row tile: both accumulators added; two: each row tile's own, one after the other
+    // through the same staging boxes).  tcgen05.ld is warp-collective: every lane loads, lanes
+    // past the rows store nothing.
     const int quarter = warp & 3, half = (warp - kGemmEpiWarp0) >> 2;
-    const int r = quarter * 32 + lane, n = n0 + r;
     const uint32_t t_row = tmem + ((uint32_t)(quarter * 32) << 16);
     const bool ok = warp_wait(acc_full, 0u, abort_flag) && !__any_sync(kFull, *abort_flag != 0);
-    if (ok) {
-      tc_fence_after();
-      if (tma_y && lane == 0) prefetch_tensormap(&ty);
+    if (ok) tc_fence_after();
+    if (ok && tma_y && lane == 0) prefetch_tensormap(&ty);
+    for (int rtile = 0; ok && rtile < rt; ++rtile) {
+      if (rtile > 0 && tma_y) {  // the previous row tile's boxes have left the staging area
+        if (lane == 0) bulk_wait_all();
+        __syncwarp();
+      }
+      const int nb = n0 + rtile * kGemmRows;  // the row tile's first row
+      const int n = nb + quarter * 32 + lane;
+      const uint32_t t_acc = t_row + (uint32_t)(rtile * kGemmM);
       float *yrow = Y + ((int64_t)split * rows + n) * ldy;
       const bool vec = (ldy & 3) == 0 && (reinterpret_cast<uintptr_t>(Y) & 15u) == 0;
       for (int c0 = half * (kGemmM / 2); c0 < (half + 1) * (kGemmM / 2); c0 += 32) {
         uint32_t a[32], b[32];
-        tmem_ld32(t_row + c0, a);
+        tmem_ld32(t_acc + c0, a);
         if (two) tmem_ld32(t_row + kGemmM + c0, b);
         tmem_wait_ld();
         float v[32];
@@ -249,8 +275,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
           fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0 && f < F && n0 + quarter * 32 < rows) {
-            tma_store_3d(&ty, box, f, n0 + quarter * 32, split);
+          if (lane == 0 && f < F && nb + quarter * 32 < rows) {
+            tma_store_3d(&ty, box, f, nb + quarter * 32, split);
             bulk_commit_group();
           }
         } else if (n < rows && f < F) {
@@ -266,8 +292,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
         }
       }
-      if (tma_y && lane == 0) bulk_wait_all();  // the boxes are written (and the ring read)
     }
+    if (ok && tma_y && lane == 0) bulk_wait_all();  // the boxes are written (and the ring read)
   }
   // the products are complete (acc_full) and the epilogue has read them: free the columns
   tc_fence_before();
@@ -309,7 +335,8 @@ int device_sms() {
 // Column splits: as many CTAs as fit in one wave (one resident an SM) stream the weights, at most
 // max_splits (each split is one more part to sum) and at most one split a 64-column tile.
 int gemm_splits(int F, int K, int rows, int max_splits) {
-  const int tiles = ((F + kGemmM - 1) / kGemmM) * ((rows + kGemmRows - 1) / kGemmRows);
+  const int rpc = kGemmRows * gemm_row_tiles(rows);  // rows a CTA
+  const int tiles = ((F + kGemmM - 1) / kGemmM) * ((rows + rpc - 1) / rpc);
   const int kt = (K + kGemmKTile - 1) / kGemmKTile;
   const int s = std::min(std::min(max_splits, kt), device_sms() / std::max(tiles, 1));
   return std::max(s, 1);
@@ -352,7 +379,7 @@ cudaError_t launch_gemm_xwt(const CUtensorMap *tw, const void *wt, const CUtenso
   if (!tma_y) ty = no_map;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)((F + kGemmM - 1) / kGemmM), (unsigned)splits,
-                     (unsigned)((rows + kGemmRows - 1) / kGemmRows));
+                     (unsigned)((rows + kGemmRows * p.rt - 1) / (kGemmRows * p.rt)));
   cfg.blockDim = dim3(kGemmThreads);
   cfg.dynamicSmemBytes = (size_t)p.smem;
   cfg.stream = stream;
@@ -363,7 +390,7 @@ cudaError_t launch_gemm_xwt(const CUtensorMap *tw, const void *wt, const CUtenso
   cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, gemm_xwt_kernel, tw ? *tw : no_map,
                             static_cast<const uint8_t *>(wt), (K + kGemmKTile - 1) / kGemmKTile,
-                            tx, ty, tma_y ? 1 : 0, Y, ldy, err, rows, F, p.nt, p.stages,
+                            tx, ty, tma_y ? 1 : 0, Y, ldy, err, rows, F, p.nt, p.rt, p.stages,
                             pdl ? 1 : 0);
 }
 
