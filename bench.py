@@ -61,7 +61,7 @@ def parse_args():
                    help="default workload: skip the batch 8 x 8192 slots point")
     p.add_argument("--kv", choices=["bf16", "fp8"], default="bf16",
                    help="decode workloads: bf16 pools, or FP8 (e4m3) pools with one power-of-two "
-                        "scale per row (read by ham_kv_append + ham_decode_attn: --path split)")
+                        "scale per row")
     p.add_argument("--path", choices=["fused", "split"], default="fused",
                    help="fused: ham_decode_step; split: ham_kv_append + ham_decode_attn")
     p.add_argument("--caches", type=int, default=CACHES,
@@ -548,8 +548,9 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
         "tokens_per_s": round(value * w.batch * mean_ntok, 1),
         "roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(attn_gbs / peak, 4), "traffic": traffic,
-                     "kernel": ("decode_attn_kernel<128,bf16,step> + combine_kernel<bf16,step>"
-                                if fused else "append_kernel + decode_attn_kernel<128,bf16" +
+                     "kernel": ("decode_attn_kernel<128,bf16,step" + (",fp8" if fp8 else "") +
+                                "> + combine_kernel<bf16,step>" if fused else
+                                "append_kernel + decode_attn_kernel<128,bf16" +
                                 (",fp8" if fp8 else "") + "> + combine_kernel<bf16>"),
                      "avg_launch_us": round(1e3 * statistics.mean(attn_ms), 3),
                      "isolated_launch_us": isolated_us,
@@ -563,7 +564,8 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
     if e2e is None:
         del result["e2e"]
     if fp8:
-        result["mma_dtype"] = "f16 codes x q 2^-f (scores), bf16 codes x weights (values)"
+        result["mma_dtype"] = ("codes converted to f16 (exact) in mma.sync f16 products: with q 2^-f "
+                               "(scores) and the weights p 2^(e_v - Eo + 7) (values)")
     if full and rank == 0 and world == 1 and not args.no_cpu_baseline and not fp8:
         result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
     for c in caches:
@@ -1938,8 +1940,6 @@ def main():
     if args.caches < 1 or GRAPH_STEPS % args.caches:
         raise SystemExit(f"--caches must divide {GRAPH_STEPS}")
     CACHES = args.caches
-    if args.kv == "fp8":
-        args.path = "split"  # FP8 pools are read by ham_kv_append + ham_decode_attn
     w = workload(args.workload)
     from paper_2505_20438_gb300 import workload as wl
     if args.impl == "reference":

@@ -334,8 +334,10 @@ int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *
  *   exponents  [pool_pages][n_kv_heads][page_slots / 16][2][16] int8  (per 16-slot chunk:
  *              the 16 keys' exponents, then the 16 values')
  * FP8 caches work with ham_kv_fill (it encodes the bf16 rows it is given), ham_kv_export,
- * ham_kv_export_scales, ham_kv_append, ham_decode_attn, ham_decode_attn_ex and the counter
- * calls; the other calls return HAM_EUNSUPPORTED for them. */
+ * ham_kv_export_scales, ham_kv_append, ham_decode_attn, ham_decode_attn_ex, ham_decode_step
+ * (its new slot is encoded as ham_kv_append encodes it, and attended as the cache then holds
+ * it) and the counter calls; ham_prefill, ham_micro_step and ham_qkv_append return
+ * HAM_EUNSUPPORTED for them. */
 
 /* Copy one layer's exponent array out (layout above): pool_pages * n_kv_heads * page_slots *
  * 2 bytes.  HAM_EINVAL for a bf16 cache. */

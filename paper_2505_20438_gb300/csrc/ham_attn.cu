@@ -159,7 +159,6 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
     decode_attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
                        const __grid_constant__ CUtensorMap tmap_v, const AttnView v) {
   using S = Shape<D, kFp8>;
-  static_assert(!(kFp8 && kStep), "the fused step does not read FP8 pools");
   const int B = v.batch, Hkv = v.n_kv_heads, G = v.group;
   const SegBuf<D> sb(G, kStep);
   const Layout<D, kFp8> lay(G, kStep, B);
@@ -484,19 +483,44 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
       const int4 inf = info[stage];
       if (inf.z & kFirst) {  // q of a new segment as f16, times 2^-f (heads >= G: zero)
         const uint16_t *q = reinterpret_cast<const uint16_t *>(qbufs + inf.w * sb.stride);
-        // lane (r0, cq) holds head r0's elements 16k + 4cq .. + 3 (read twice: max, convert)
-        auto q4 = [&](int k) {
-          uint2 w = make_uint2(0u, 0u);
-          if (hq) w = *reinterpret_cast<const uint2 *>(q + r0 * D + 16 * k + 4 * cq);
-          return make_float4(__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xFFFF0000u),
-                             __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xFFFF0000u));
-        };
-        float amax = 0.f;
+        // lane (r0, cq) holds head r0's elements 16k + 4cq .. + 3
+        float qv[kKSteps][4];
 #pragma unroll
         for (int k = 0; k < kKSteps; ++k) {
-          const float4 e = q4(k);
-          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(e.x), fabsf(e.y)), fmaxf(fabsf(e.z), fabsf(e.w))));
+          uint2 w = make_uint2(0u, 0u);
+          if (hq) w = *reinterpret_cast<const uint2 *>(q + r0 * D + 16 * k + 4 * cq);
+          qv[k][0] = __uint_as_float(w.x << 16);
+          qv[k][1] = __uint_as_float(w.x & 0xFFFF0000u);
+          qv[k][2] = __uint_as_float(w.y << 16);
+          qv[k][3] = __uint_as_float(w.y & 0xFFFF0000u);
         }
+        if constexpr (kStep) {
+          // the fused step: q turned by the new slot's position in fp32 and rounded to bf16, as
+          // the bf16 pass does; element j < D/2 and its partner j + D/2 sit in k-steps k, k + 4
+          const int b = inf.x / Hkv;
+          float2 *cs = reinterpret_cast<float2 *>(qbufs + inf.w * sb.stride + sb.cs_off());
+          if (appb[b]) {
+            const int64_t p = posb[b];
+            if (!(p >= 0 && p < v.step.rope_positions))
+              fill_cs_row(cs, p, v.step.inv_freq, D / 2, lane);
+          }
+          if (appb[b] && hq) {
+#pragma unroll
+            for (int k = 0; k < kKSteps / 2; ++k)
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 c = cs[16 * k + 4 * cq + e];
+                const float a = qv[k][e], bb = qv[k + kKSteps / 2][e];
+                qv[k][e] = __bfloat162float(__float2bfloat16_rn(a * c.x - bb * c.y));
+                qv[k + kKSteps / 2][e] = __bfloat162float(__float2bfloat16_rn(bb * c.x + a * c.y));
+              }
+          }
+        }
+        float amax = 0.f;
+#pragma unroll
+        for (int k = 0; k < kKSteps; ++k)
+          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(qv[k][0]), fabsf(qv[k][1])),
+                                   fmaxf(fabsf(qv[k][2]), fabsf(qv[k][3]))));
         amax = fmaxf(amax, __shfl_xor_sync(kFull, amax, 1));
         amax = fmaxf(amax, __shfl_xor_sync(kFull, amax, 2));
         int f = 0;
@@ -510,9 +534,8 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
         const float sc = pow2i(-f);
 #pragma unroll
         for (int k = 0; k < kKSteps; ++k) {
-          const float4 e = q4(k);
-          qb[k][0] = pack_f16x2(e.x * sc, e.y * sc);
-          qb[k][1] = pack_f16x2(e.z * sc, e.w * sc);
+          qb[k][0] = pack_f16x2(qv[k][0] * sc, qv[k][1] * sc);
+          qb[k][1] = pack_f16x2(qv[k][2] * sc, qv[k][3] * sc);
         }
         const float qs = qscale * pow2i(f);  // head r0's; the columns' heads are h0, h1
         qs0 = __shfl_sync(kFull, qs, 4 * h0);
@@ -626,7 +649,8 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
       // O^T back from units of 2^(Eo - 7) (0 below fp32's normal range)
       const float r0s = E0 == kNoExp ? 0.f : pow2i(max(E0 - 7, -127));
       const float r1s = E1 == kNoExp ? 0.f : pow2i(max(E1 - 7, -127));
-      if (first == last) {
+      // (fused step: the combine kernel still adds the appended slot, so always the partials)
+      if (!kStep && first == last) {
         const float i0 = l0 > 0.f ? r0s / l0 : 0.f, i1 = l1 > 0.f ? r1s / l1 : 0.f;
 #pragma unroll
         for (int i = 0; i < kMTiles; ++i) {
@@ -923,6 +947,7 @@ __device__ __forceinline__ double2 rope_cs(const StepArgs &st, int64_t p, int ha
 struct PairTurn {
   uint16_t qc0, qc1, kc0, kc1;
   float share;
+  float qr0, qr1;  // q turned in fp32 and rounded to bf16 (the pass's q)
 };
 __device__ __noinline__ PairTurn turn_pair(double c, double sn, uint16_t q0, uint16_t q1,
                                            uint16_t k0, uint16_t k1) {
@@ -941,7 +966,67 @@ __device__ __noinline__ PairTurn turn_pair(double c, double sn, uint16_t q0, uin
   const float kr0 = __bfloat162float(__float2bfloat16_rn(b0 * cf - b1 * sf));
   const float kr1 = __bfloat162float(__float2bfloat16_rn(b1 * cf + b0 * sf));
   r.share = qr0 * kr0 + qr1 * kr1;
+  r.qr0 = qr0;
+  r.qr1 = qr1;
   return r;
+}
+
+// FP8 pools, fused step: one of the new slot's rows (the rotated key, or the value) as the
+// append encodes it (encode_e4m3_row's rule: e = E - 8 of the row's largest magnitude, clamped;
+// each element times 2^-e rounded to e4m3 with saturation), from the pair (x0, x1) = elements
+// (i, i + D/2) each thread of a head holds.  The row maximum runs over the head's D/2 threads:
+// warp shuffles, and at D = 128 the head's two warps meet in `red` (one float a warp).  Every
+// thread of the block calls it (zeros where a thread has no pair).  Returns the codes, e and the
+// decoded values code 2^e (exact bf16 values: the rows the cache holds).
+struct Fp8Pair {
+  uint8_t c0, c1;
+  int e;
+  float d0, d1;
+};
+__device__ __forceinline__ Fp8Pair fp8_encode_pair(float x0, float x1, int half, float *red) {
+  float a = fmaxf(fabsf(x0), fabsf(x1));
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) a = fmaxf(a, __shfl_xor_sync(kFull, a, off));
+  if (half > 32) {
+    const int warp = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) red[warp] = a;
+    __syncthreads();
+    a = fmaxf(red[warp & ~1], red[warp | 1]);
+    __syncthreads();
+  }
+  Fp8Pair r;
+  r.e = 0;
+  if (a > 0.f) {
+    int E = 0;
+    frexpf(a, &E);
+    r.e = min(max(E - 8, kFp8ExpMin), kFp8ExpMax);
+  }
+  r.c0 = (uint8_t)__nv_cvt_float_to_fp8(ldexpf(x0, -r.e), __NV_SATFINITE, __NV_E4M3);
+  r.c1 = (uint8_t)__nv_cvt_float_to_fp8(ldexpf(x1, -r.e), __NV_SATFINITE, __NV_E4M3);
+  const float s = pow2i(r.e);
+  r.d0 = __half2float(__half(__nv_cvt_fp8_to_halfraw(r.c0, __NV_E4M3))) * s;
+  r.d1 = __half2float(__half(__nv_cvt_fp8_to_halfraw(r.c1, __NV_E4M3))) * s;
+  return r;
+}
+
+// FP8 pools, fused step: the new slot's codes of this thread's pair (elements i, i + D/2) of
+// KV head g's key and value rows, and (i == 0) their exponents, at slot n of page `page`.
+__device__ __forceinline__ void fp8_store_pair(const AttnView &v, int page, int g, int n, int i,
+                                               int half, const Fp8Pair &k, const Fp8Pair &val) {
+  const int P = v.page_slots, D = 2 * half, s = n % P;
+  const int64_t ph = (int64_t)page * v.n_kv_heads + g;
+  uint8_t *kc = reinterpret_cast<uint8_t *>(v.step.k_pool);
+  uint8_t *vc = reinterpret_cast<uint8_t *>(v.step.v_pool);
+  kc[(ph * P + s) * D + i] = k.c0;
+  kc[(ph * P + s) * D + i + half] = k.c1;
+  const int sv = s - s % kChunkSlots + fp8_v_slot_byte(s % kChunkSlots);
+  vc[(ph * D + i) * P + sv] = val.c0;
+  vc[(ph * D + i + half) * P + sv] = val.c1;
+  if (i == 0) {
+    int8_t *e = v.step.kv_exp + (ph * (P / kChunkSlots) + s / kChunkSlots) * 32 + s % kChunkSlots;
+    e[0] = (int8_t)k.e;
+    e[kChunkSlots] = (int8_t)val.e;
+  }
 }
 
 // The append record (n, 0 or the error that stops it, position, ntok) of a sequence from its
@@ -1009,7 +1094,9 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   const StepArgs &st = v.step;
   __shared__ int red[3][kCombineThreads / 32];
   __shared__ float head_sum[kCombineThreads / 32];
+  __shared__ float fp8_red[kCombineThreads / 32];
   __shared__ int commit_all;  // fused step: this CTA commits every sequence
+  const bool fp8 = v.kv_exp != nullptr;  // FP8 pools
 
   // ---- the segment's CTA range (split plan, as the attention computes it)
   int first = -1, last = -1;
@@ -1052,6 +1139,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
   // ---- fused step: record, rotations, q_rot and the new slot's rows; then the report
   int4 rec = make_int4(0, 0, 0, 0);
   uint16_t v0 = 0, v1 = 0;
+  float vd0 = 0.f, vd1 = 0.f;  // FP8 pools: the new value pair as the cache holds it
   float dot = 0.f;
   int4 crec = make_int4(0, 0, 0, 0);  // committing CTA, thread t < B: sequence t
   int64_t ctok = 0;
@@ -1069,24 +1157,37 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
     const int64_t tb = (!st.pos && st.pos_mode == HAM_POS_TOKEN) ? st.num_tokens[b] : 0;
     rec = append_record(v, v.num_slots[b], tb, st.ntok[b], st.pos ? st.pos + b : nullptr);
     float share = 0.f;
+    PairTurn pt{};
+    int page = -1;
     if (rec.y == 0 && active) {
       const double2 cs = rope_cs(st, rec.z, half, i);
-      const PairTurn pt = turn_pair(cs.x, cs.y, q0, q1, k0, k1);
+      pt = turn_pair(cs.x, cs.y, q0, q1, k0, k1);
       share = pt.share;
       if (st.q_rot) {
         st.q_rot[orow + i] = pt.qc0;
         st.q_rot[orow + i + half] = pt.qc1;
       }
-      if (h == 0) {  // the new slot's rows of KV head g
-        const int page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
-        if (page >= 0 && page < v.pool_pages) {
-          const int64_t row =
-              (((int64_t)page * Hkv + g) * v.page_slots + rec.x % v.page_slots) * D;
-          st.k_pool[row + i] = pt.kc0;
-          st.k_pool[row + i + half] = pt.kc1;
-          st.v_pool[row + i] = v0;
-          st.v_pool[row + i + half] = v1;
-        }
+      if (h == 0) page = v.page_table[(int64_t)b * v.max_pages + rec.x / v.page_slots];
+      if (h == 0 && !fp8 && page >= 0 && page < v.pool_pages) {  // the new slot's rows of head g
+        const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + rec.x % v.page_slots) * D;
+        st.k_pool[row + i] = pt.kc0;
+        st.k_pool[row + i + half] = pt.kc1;
+        st.v_pool[row + i] = v0;
+        st.v_pool[row + i + half] = v1;
+      }
+    }
+    if (fp8) {  // encode the rows as the append does; the new slot's term takes the decoded ones
+      const bool mine = rec.y == 0 && active;
+      const Fp8Pair kp = fp8_encode_pair(mine ? bf16_bits_to_float(pt.kc0) : 0.f,
+                                         mine ? bf16_bits_to_float(pt.kc1) : 0.f, half, fp8_red);
+      const Fp8Pair vp = fp8_encode_pair(mine ? bf16_bits_to_float(v0) : 0.f,
+                                         mine ? bf16_bits_to_float(v1) : 0.f, half, fp8_red);
+      if (mine) {
+        share = pt.qr0 * kp.d0 + pt.qr1 * kp.d1;
+        vd0 = vp.d0;
+        vd1 = vp.d1;
+        if (h == 0 && page >= 0 && page < v.pool_pages)
+          fp8_store_pair(v, page, g, rec.x, i, half, kp, vp);
       }
     }
     // the score of head h: one warp at d = 64, two at d = 128 (they meet in shared memory)
@@ -1128,8 +1229,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(const AttnView
       const float bm = fmaxf(M, x);
       const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
       const float w = ex2(x - bm);
-      num0 = num0 * scale + w * bf16_bits_to_float(v0);
-      num1 = num1 * scale + w * bf16_bits_to_float(v1);
+      num0 = num0 * scale + w * (fp8 ? vd0 : bf16_bits_to_float(v0));
+      num1 = num1 * scale + w * (fp8 ? vd1 : bf16_bits_to_float(v1));
       den = den * scale + w;
     }
     if (active && (merge || appended)) {
@@ -1172,6 +1273,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_late_kernel(const Att
   const bool active = idx < G * half;
   const int h = idx / half, i = idx - h * half;
   const int64_t orow = ((int64_t)seg * G + h) * D;  // row (b, g*G + h) of q / q_rot / out
+  const bool fp8 = v.kv_exp != nullptr;              // FP8 pools
 
   grid_dependency_wait();  // the attention grid's partials, ranges and append records
   // The next kernel may be scheduled now; its own dependency wait still covers this grid.
@@ -1225,7 +1327,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_late_kernel(const Att
         qc0 = rotate_elem(x0, x1, c, sn, false);
         qc1 = rotate_elem(x1, x0, c, sn, true);
       }
-      if (h == 0) {
+      if (h == 0 || fp8) {  // (FP8: every head scores the new slot with the stored key)
         const double x0 = bf16_bits_to_double(k0), x1 = bf16_bits_to_double(k1);
         kc0 = rotate_elem(x0, x1, c, sn, false);
         kc1 = rotate_elem(x1, x0, c, sn, true);
@@ -1238,16 +1340,28 @@ __global__ void __launch_bounds__(kCombineThreads) combine_late_kernel(const Att
     // threads of the head (one warp at d = 64, two at d = 128, whose sums meet in shared
     // memory).  Every thread of the block takes part, so no thread has left yet.
     __shared__ float head_sum[kCombineThreads / 32];
-    float share = 0.f;
+    __shared__ float fp8_red[kCombineThreads / 32];
+    float share = 0.f, qr0 = 0.f, qr1 = 0.f;
     if (app && active) {
       const float cf = (float)c, sf = (float)sn;
       const float x0 = bf16_bits_to_float(q0), x1 = bf16_bits_to_float(q1);
       const float y0 = bf16_bits_to_float(k0), y1 = bf16_bits_to_float(k1);
-      const float qr0 = __bfloat162float(__float2bfloat16_rn(x0 * cf - x1 * sf));
-      const float qr1 = __bfloat162float(__float2bfloat16_rn(x1 * cf + x0 * sf));
+      qr0 = __bfloat162float(__float2bfloat16_rn(x0 * cf - x1 * sf));
+      qr1 = __bfloat162float(__float2bfloat16_rn(x1 * cf + x0 * sf));
       const float kr0 = __bfloat162float(__float2bfloat16_rn(y0 * cf - y1 * sf));
       const float kr1 = __bfloat162float(__float2bfloat16_rn(y1 * cf + y0 * sf));
       share = qr0 * kr0 + qr1 * kr1;
+    }
+    // FP8 pools: the rows encoded as the append encodes them; the new slot's term takes the
+    // decoded ones (every thread of the block takes part in the row maxima)
+    Fp8Pair kp{}, vp{};
+    if (fp8) {
+      const bool mine = app && active;
+      kp = fp8_encode_pair(mine ? bf16_bits_to_float(kc0) : 0.f,
+                           mine ? bf16_bits_to_float(kc1) : 0.f, half, fp8_red);
+      vp = fp8_encode_pair(mine ? bf16_bits_to_float(v0) : 0.f,
+                           mine ? bf16_bits_to_float(v1) : 0.f, half, fp8_red);
+      if (mine) share = qr0 * kp.d0 + qr1 * kp.d1;
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) share += __shfl_xor_sync(kFull, share, off);
@@ -1260,8 +1374,8 @@ __global__ void __launch_bounds__(kCombineThreads) combine_late_kernel(const Att
       const float bm = fmaxf(M, x);
       const float scale = (M == -INFINITY) ? 0.f : ex2(M - bm);
       const float w = ex2(x - bm);
-      num0 = num0 * scale + w * bf16_bits_to_float(v0);
-      num1 = num1 * scale + w * bf16_bits_to_float(v1);
+      num0 = num0 * scale + w * (fp8 ? vp.d0 : bf16_bits_to_float(v0));
+      num1 = num1 * scale + w * (fp8 ? vp.d1 : bf16_bits_to_float(v1));
       den = den * scale + w;
     }
     if (active && (merge || app)) {
@@ -1288,11 +1402,15 @@ __global__ void __launch_bounds__(kCombineThreads) combine_late_kernel(const Att
       return;
     }
     const int n = rec.x;
-    const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
-    st.k_pool[row + i] = kc0;
-    st.k_pool[row + i + half] = kc1;
-    st.v_pool[row + i] = v0;
-    st.v_pool[row + i + half] = v1;
+    if (fp8) {
+      fp8_store_pair(v, page, g, n, i, half, kp, vp);
+    } else {
+      const int64_t row = (((int64_t)page * Hkv + g) * v.page_slots + n % v.page_slots) * D;
+      st.k_pool[row + i] = kc0;
+      st.k_pool[row + i + half] = kc1;
+      st.v_pool[row + i] = v0;
+      st.v_pool[row + i + half] = v1;
+    }
     if (lead) {
       const int64_t meta = (int64_t)page * v.page_slots + n % v.page_slots;
       st.slot_pos[meta] = rec.z;
@@ -1421,6 +1539,11 @@ cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, con
                                int head_dim, int out_dtype, cudaStream_t stream) {
   if (v.ctas < 1 || v.group < 1 || v.group > kMaxGroup) return cudaErrorInvalidConfiguration;
   auto go = [&](auto inst) { return decltype(inst)::launch(tk, tv, v, stream); };
+  if (v.kv_exp) {  // FP8 pools
+    if (head_dim != kFp8HeadDim) return cudaErrorInvalidValue;
+    return out_dtype == HAM_DTYPE_F32 ? go(Instance<kFp8HeadDim, float, true, true>())
+                                      : go(Instance<kFp8HeadDim, __nv_bfloat16, true, true>());
+  }
   return out_dtype == HAM_DTYPE_F32 ? dispatch<float, true>(head_dim, go)
                                     : dispatch<__nv_bfloat16, true>(head_dim, go);
 }
@@ -1434,9 +1557,13 @@ int attention_ctas_per_sm(int head_dim, int group, int batch, bool step, int out
   };
   const bool f32 = out_dtype == HAM_DTYPE_F32;
   if (fp8) {
-    if (head_dim != kFp8HeadDim || step) return 0;
-    f32 ? q(Instance<kFp8HeadDim, float, false, true>())
-        : q(Instance<kFp8HeadDim, __nv_bfloat16, false, true>());
+    if (head_dim != kFp8HeadDim) return 0;
+    if (step)
+      f32 ? q(Instance<kFp8HeadDim, float, true, true>())
+          : q(Instance<kFp8HeadDim, __nv_bfloat16, true, true>());
+    else
+      f32 ? q(Instance<kFp8HeadDim, float, false, true>())
+          : q(Instance<kFp8HeadDim, __nv_bfloat16, false, true>());
     return n;
   }
   if (step) f32 ? dispatch<float, true>(head_dim, q) : dispatch<__nv_bfloat16, true>(head_dim, q);

@@ -518,14 +518,16 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   {
     const int per_sm = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, false,
                                                   HAM_DTYPE_BF16, kv->fp8 != 0);
-    const int per_sm_step = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, true);
+    const int per_sm_step = ham::attention_ctas_per_sm(cfg.head_dim, group, cfg.batch, true,
+                                                       HAM_DTYPE_BF16, kv->fp8 != 0);
     if (per_sm <= 0 || per_sm_step <= 0) {
       delete kv;
       return fail(HAM_ECUDA, "attention kernel cannot be resident on an SM");
     }
     kv->default_ctas =
         std::min(ham::default_attention_ctas(sms, per_sm, kv->fp8 != 0), kv->max_ctas);
-    kv->default_step_ctas = std::min(ham::default_attention_ctas(sms, per_sm_step), kv->max_ctas);
+    kv->default_step_ctas =
+        std::min(ham::default_attention_ctas(sms, per_sm_step, kv->fp8 != 0), kv->max_ctas);
   }
   cudaError_t e = cudaMalloc(&kv->pool, pool_bytes);
   if (e != cudaSuccess) {
@@ -847,7 +849,6 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
                     int32_t out_dtype, void *stream) {
   int rc = check_layer(kv, layer);
   if (rc) return rc;
-  if ((rc = fp8_unsupported(kv, "ham_decode_step")) != 0) return rc;
   if (!q || !k_new || !v_new || !ntok || !out)
     return fail(HAM_EINVAL, "q, k_new, v_new, ntok and out are required");
   if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
@@ -870,6 +871,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
   ham::AttnView v{};
   v.k_pool = layer_pool(kv, layer, 0);
   v.v_pool = layer_pool(kv, layer, 1);
+  v.kv_exp = layer_exp(kv, layer);
   v.page_table = kv->page_table;
   v.num_slots = kv->num_slots + (size_t)layer * c.batch;
   v.q = static_cast<const uint16_t *>(q);
@@ -900,6 +902,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
   st.slot_ntok = kv->slot_ntok;
   st.k_pool = layer_pool(kv, layer, 0);
   st.v_pool = layer_pool(kv, layer, 1);
+  st.kv_exp = layer_exp(kv, layer);
   st.inv_freq = kv->inv_freq;
   st.rope_table = kv->rope_table;
   st.rope_table_f = kv->rope_table_f;

@@ -252,6 +252,97 @@ def test_fp8_append_then_decode():
     assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
 
 
+def _decoded_cache(case, oc):
+    """An oracle cache holding the decoded rows of `oc`'s bf16 pools (the rows an FP8 cache
+    holds after the same fills and appends)."""
+    ref = oracle.OracleCache.from_case(case, fill=False)
+    ref.k_pool[...] = _decoded(oc.k_pool)
+    ref.v_pool[...] = _decoded(oc.v_pool)
+    ref.slot_pos[...] = oc.slot_pos
+    ref.slot_ntok[...] = oc.slot_ntok
+    ref.num_slots[...] = oc.num_slots
+    ref.num_tokens[...] = oc.num_tokens
+    return ref
+
+
+Q_ROT_UNWRITTEN = 0x7FC1  # a bf16 NaN pattern no rotation produces
+
+
+@pytest.mark.parametrize("pos_mode", [ham.HAM_POS_SLOT, ham.HAM_POS_TOKEN])
+@pytest.mark.parametrize("hq,hkv,page,counts", [
+    (32, 8, 16, (15, 16, 0, 47)),          # new slot ends chunk 0 / opens chunk 1 / first
+    (32, 8, 32, (31, 200, 5)),             # page edge
+    (8, 8, 16, (1, 64)),                   # group 1
+    (64, 8, 128, (127, 300)),              # group 8
+])
+def test_fp8_step_matches_oracle(pos_mode, hq, hkv, page, counts):
+    """ham_decode_step on an FP8 cache: the stored codes and exponents, the counters and q_rot
+    bit for bit against the oracle's append (then encoded); the output against the oracle's
+    attention over the decoded rows of all n + 1 slots.  q is never written."""
+    case = small_case(batch=len(counts), hq=hq, hkv=hkv, d=128, page=page, counts=counts,
+                      seed=71, extra_slots=8)
+    oc = oracle.OracleCache.from_case(case)
+    kv = fp8_cache(case, pos_mode=pos_mode)
+    t = torch()
+    q = case.q.copy()
+    rng = wl.rng_for(71, 60)
+    for step in range(3):
+        k_new = wl.normal_bf16(rng, case.k_new.shape)
+        v_new = wl.normal_bf16(rng, case.v_new.shape)
+        ntok = wl.ntok_capped_geometric(rng, (case.w.batch,))
+        q_ref = q.copy()
+        assert oc.append(k_new, v_new, ntok, q_inout=q_ref, pos_mode=pos_mode) == 0
+        ref = _decoded_cache(case, oc).decode_attn(q_ref)
+        q_dev = dev_bf16(q)
+        q_rot = dev_bf16(np.full(q.shape, Q_ROT_UNWRITTEN, np.uint16))
+        out = t.full(q_dev.shape, float("nan"), dtype=t.float32, device="cuda")
+        ham.ham_decode_step(kv, 0, q_dev, dev_bf16(k_new), dev_bf16(v_new), None, dev_i32(ntok),
+                            out, q_rot=q_rot)
+        t.cuda.synchronize()
+        assert np.array_equal(host_bits(q_dev), q), "q was written"
+        assert np.array_equal(host_bits(q_rot), q_ref), f"q_rot, step {step}"
+        got = out.float().cpu().numpy().astype(np.float64)
+        assert_parity(got, ref, what=f"fp8 step {step}")
+    k, v, e, pos, ntok_arr = _export(kv)
+    kc, vc, ee = _expected_pools(oc.k_pool, oc.v_pool)
+    assert np.array_equal(e, ee), "exponents"
+    assert np.array_equal(k, kc), "K codes"
+    assert np.array_equal(v, vc), "V codes"
+    assert np.array_equal(pos, oc.slot_pos) and np.array_equal(ntok_arr, oc.slot_ntok)
+    slots, tokens = ham.ham_slot_lengths(kv)
+    assert np.array_equal(slots, oc.num_slots) and np.array_equal(tokens, oc.num_tokens)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
+@pytest.mark.parametrize("batch", [3, 200])  # early and late combine modes
+def test_fp8_step_equals_append_then_decode(batch):
+    """The fused step and ham_kv_append + ham_decode_attn on two FP8 caches from the same fill:
+    the same stored bits and counters, outputs within the bar of each other."""
+    rng = np.random.default_rng(batch)
+    counts = tuple(int(c) for c in rng.integers(0, 150, size=batch))
+    case = small_case(batch=batch, hq=32, hkv=8, d=128, page=16, counts=counts, seed=81,
+                      extra_slots=4)
+    a, b = fp8_cache(case), fp8_cache(case)
+    t = torch()
+    k_new, v_new = dev_bf16(case.k_new), dev_bf16(case.v_new)
+    ntok = dev_i32(case.ntok_new)
+    q1 = dev_bf16(case.q)
+    out1 = t.full(q1.shape, float("nan"), dtype=t.float32, device="cuda")
+    ham.ham_decode_step(a, 0, q1, k_new, v_new, None, ntok, out1)
+    q2 = dev_bf16(case.q)
+    out2 = t.full(q2.shape, float("nan"), dtype=t.float32, device="cuda")
+    ham.ham_kv_append(b, 0, q2, k_new, v_new, None, ntok)
+    ham.ham_decode_attn_ex(b, 0, q2, out2)
+    t.cuda.synchronize()
+    ea, eb = _export(a), _export(b)
+    for x, y, what in zip(ea, eb, ("K codes", "V codes", "exponents", "pos", "ntok")):
+        assert np.array_equal(x, y), what
+    o1 = out1.cpu().numpy().astype(np.float64)
+    o2 = out2.cpu().numpy().astype(np.float64)
+    assert_parity(o1, o2, what="step against append + decode")
+    assert ham.ham_kv_status(a) == ham.HAM_DEVERR_NONE and ham.ham_kv_status(b) == ham.HAM_DEVERR_NONE
+
+
 def test_fp8_unsupported_calls_are_refused():
     case = small_case(batch=2, hq=8, hkv=2, d=128, page=16, counts=(5, 6), seed=61)
     kv = fp8_cache(case)
@@ -259,8 +350,8 @@ def test_fp8_unsupported_calls_are_refused():
     q = dev_bf16(case.q)
     out = t.empty_like(q)
     with pytest.raises(ham.HamError) as e:
-        ham.ham_decode_step(kv, 0, q, dev_bf16(case.k_new), dev_bf16(case.v_new), None,
-                            dev_i32(case.ntok_new), out)
+        ham.ham_prefill(kv, 0, q, dev_bf16(case.k_new), dev_bf16(case.v_new),
+                        dev_i32(np.array([0, 1, 2], np.int32)), out)
     assert e.value.status == ham.HAM_EUNSUPPORTED
     with pytest.raises(ham.HamError) as e:
         ham.ham_kv_alloc(1, 2, 8, 2, 64, 16, 32, kv_dtype=ham.HAM_KV_E4M3)
