@@ -119,7 +119,8 @@ def measured_peak_hbm():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-ATTN_SOURCES = ("ham_attn.cu", "ham_internal.cuh", "ham_ptx.cuh")
+ATTN_SOURCES = ("ham_attn.cu", "ham_attn.cuh", "ham_internal.cuh", "ham_ptx.cuh")
+ATTN_FP8_SOURCES = ("ham_attn_fp8.cu",) + ATTN_SOURCES
 FRONT_SOURCES = ("ham_front.cu", "ham_front.cuh", "ham_ptx.cuh")
 
 
@@ -533,7 +534,7 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
     e2e = run_e2e(args, w, caches, stream, rollback, world, one_step) if full else None
 
     traffic = profiled_traffic(("decode_step" if fused else "decode_attn") + ("_fp8" if fp8 else ""),
-                               w.name)
+                               w.name, ATTN_FP8_SOURCES if fp8 else ATTN_SOURCES)
     result = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
         "steps": steps, "steps_requested": args.steps, "timed_s": round(elapsed_ms * 1e-3, 3),
@@ -548,10 +549,11 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
         "tokens_per_s": round(value * w.batch * mean_ntok, 1),
         "roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(attn_gbs / peak, 4), "traffic": traffic,
-                     "kernel": ("decode_attn_kernel<128,bf16,step" + (",fp8" if fp8 else "") +
-                                "> + combine_kernel<bf16,step>" if fused else
-                                "append_kernel + decode_attn_kernel<128,bf16" +
-                                (",fp8" if fp8 else "") + "> + combine_kernel<bf16>"),
+                     "kernel": ((("decode_attn_fp8_kernel<bf16,step>" if fp8 else
+                                  "decode_attn_kernel<128,bf16,step>") + " + combine_kernel<bf16,step>")
+                                if fused else
+                                ("append_kernel + " + ("decode_attn_fp8_kernel<bf16>" if fp8 else
+                                 "decode_attn_kernel<128,bf16>") + " + combine_kernel<bf16>")),
                      "avg_launch_us": round(1e3 * statistics.mean(attn_ms), 3),
                      "isolated_launch_us": isolated_us,
                      "algorithmic_bytes_per_launch": int(timed_bytes_graph / GRAPH_STEPS),
@@ -564,8 +566,9 @@ def measure_decode(args, w, rank, local_rank, world, min_seconds, full):
     if e2e is None:
         del result["e2e"]
     if fp8:
-        result["mma_dtype"] = ("codes converted to f16 (exact) in mma.sync f16 products: with q 2^-f "
-                               "(scores) and the weights p 2^(e_v - Eo + 7) (values)")
+        result["mma_dtype"] = ("e4m3 codes read as stored by tcgen05 kind::f8f6f4 products (fp32 "
+                               "accumulators in tensor memory); q 2^-f and the weights "
+                               "p 2^(e_v - Gv + 7) as three e4m3 pieces each (~12 significant bits)")
     if full and rank == 0 and world == 1 and not args.no_cpu_baseline and not fp8:
         result["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
     for c in caches:

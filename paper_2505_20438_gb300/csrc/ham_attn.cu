@@ -28,6 +28,9 @@
 //    timing or page ids.  (A fused last-CTA merge was measured first: one warp merging
 //    ~15 partials through L2 serialised 12-18 us at the end of every launch.)
 //
+// Caches of FP8 (e4m3) rows have their own pass (ham_attn_fp8.cu: tcgen05 products over
+// 128-slot tiles) with the same plan and partials; the combine kernels below serve both.
+//
 // Every wait is bounded (about 2 s); a wait that runs out records HAM_DEVERR_TIMEOUT,
 // lets the CTA's copies land and returns.  No trap, no unbounded spin.
 #include <cuda.h>
@@ -36,47 +39,29 @@
 #include <mutex>
 #include <type_traits>
 
+#include "ham_attn.cuh"
 #include "ham_internal.cuh"
 #include "ham_ptx.cuh"
 
 namespace ham {
 namespace {
 
-constexpr float kRescaleSlack = 8.0f;              // log2 units
-constexpr int kFirst = 1, kLast = 2, kPageOk = 4;  // stage flags
-constexpr int kMaxGroup = 8;                       // heads padded to the MMA's N = 8
-
-template <typename OutT>
-__device__ __forceinline__ void store_out(void *out, int64_t i, float x) {
-  if constexpr (std::is_same<OutT, float>::value)
-    static_cast<float *>(out)[i] = x;
-  else
-    static_cast<__nv_bfloat16 *>(out)[i] = __float2bfloat16_rn(x);
-}
+constexpr float kRescaleSlack = 8.0f;  // log2 units
 
 // ------------------------------------------------------------------------------------
 // Shape of one kernel instance
 // ------------------------------------------------------------------------------------
-__host__ __device__ constexpr int align_up(int x, int a) { return (x + a - 1) / a * a; }
-
-// kFp8: FP8 pools (head_dim 128): a stage holds a chunk's K codes (16 x 128 bytes, the
-// 128-byte swizzle), its V codes transposed (128 x 16 bytes) and, apart, its 32 exponents.
-template <int D, bool kFp8 = false>
+template <int D>
 struct Shape {
-  static constexpr int kChunkBytes = kChunkSlots * D * (kFp8 ? 1 : 2);  // K (or V) of a chunk
+  static constexpr int kChunkBytes = kChunkSlots * D * 2;   // K (or V) rows of one chunk
   static constexpr int kStageBytes = 2 * kChunkBytes;
-  // 32 KiB ring; FP8 16 KiB, for twice the CTAs an SM (its consumer has more to compute a byte)
-  static constexpr int kStages = (kFp8 ? 16384 : 32768) / kStageBytes;
+  static constexpr int kStages = 32768 / kStageBytes;       // 32 KiB ring
   static constexpr int kQBufs = kStages + 1;
   static constexpr int kThreads = 64;                       // consumer warp, producer warp
   static constexpr int kSteps = D / 16;                     // k-steps of q.k, m-tiles of p.v
   static constexpr int kLinesPerRow = D / 64;               // 128-byte swizzle lines per row
-  static constexpr int kExpBytes = kFp8 ? 2 * kChunkSlots : 0;  // a chunk's exponents
-  static constexpr int kTxBytes = kStageBytes + kExpBytes;  // bytes a stage's copies bring
-  static constexpr int kOffE = kStages * kStageBytes;       // from a 1024-byte aligned base
-  static constexpr int kOffQ = kOffE + (kStages * kExpBytes + 127) / 128 * 128;
+  static constexpr int kOffQ = kStages * kStageBytes;       // from a 1024-byte aligned base
   static_assert(D == 64 || D == 128, "head_dim 64 or 128");
-  static_assert(!kFp8 || D == 128, "FP8 pools: head_dim 128");
   static_assert(kStages >= 2, "ring depth");
 };
 
@@ -91,11 +76,11 @@ struct SegBuf {
 };
 
 // Shared memory map after the per-segment buffers (runtime: depends on group and batch).
-template <int D, bool kFp8 = false>
+template <int D>
 struct Layout {
   int off_bar, off_info, off_flags, off_cum, total;
   __host__ __device__ Layout(int group, bool step, int batch) {
-    using S = Shape<D, kFp8>;
+    using S = Shape<D>;
     off_bar = S::kOffQ + S::kQBufs * SegBuf<D>(group, step).stride;
     off_info = align_up(off_bar + 2 * S::kStages * 8, 16);
     off_flags = off_info + S::kStages * 16;
@@ -130,38 +115,17 @@ __device__ __forceinline__ uint16_t rotate_elem(double self, double other, doubl
   return __bfloat16_as_ushort(__double2bfloat16(y));
 }
 
-// Positions past the fp32 (cos, sin) table: the consumer warp fills the segment's row in
-// shared memory itself (fp64 sincos rounded to fp32, two entries per lane at d = 128), so
-// that the rotations below always read the row.  A bulk copy may later reuse the buffer.
-__device__ __forceinline__ void fill_cs_row(float2 *cs_row, int64_t p, const double *inv_freq,
-                                            int half, int lane) {
-  for (int i = lane; i < half; i += 32) {
-    double sd, cd;
-    sincos((double)p * inv_freq[i], &sd, &cd);
-    cs_row[i] = make_float2((float)cd, (float)sd);
-  }
-  fence_proxy_async_smem();
-  __syncwarp();
-}
-
-// Position of the slot a fused step appends to sequence b (slot index n or tokens so far,
-// unless given).
-__device__ __forceinline__ int64_t step_position(const StepArgs &st, int b, int n) {
-  if (st.pos) return st.pos[b];
-  return st.pos_mode == HAM_POS_SLOT ? (int64_t)n : st.num_tokens[b];
-}
-
 // ------------------------------------------------------------------------------------
 // The kernel
 // ------------------------------------------------------------------------------------
-template <int D, typename OutT, bool kStep, bool kFp8>
-__global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasPerSmFp8 : 1)
+template <int D, typename OutT, bool kStep>
+__global__ void __launch_bounds__(Shape<D>::kThreads)
     decode_attn_kernel(const __grid_constant__ CUtensorMap tmap_k,
                        const __grid_constant__ CUtensorMap tmap_v, const AttnView v) {
-  using S = Shape<D, kFp8>;
+  using S = Shape<D>;
   const int B = v.batch, Hkv = v.n_kv_heads, G = v.group;
   const SegBuf<D> sb(G, kStep);
-  const Layout<D, kFp8> lay(G, kStep, B);
+  const Layout<D> lay(G, kStep, B);
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -244,7 +208,7 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
   const int nchunks = (int)(x1 - x0);
 
   // Producer lanes decode 32 chunks at a time: lane j holds chunk base + j.
-  auto decode = [&](int base, int &seg, int &valid, int &fl, int &row0, int &ph) {
+  auto decode = [&](int base, int &seg, int &valid, int &fl, int &row0) {
     const int64_t x = x0 + base + lane;
     int lo = 0, hi = B - 1;
     while (lo < hi) {
@@ -260,46 +224,27 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
     const int slot0 = c * kChunkSlots;
     const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
     const bool page_ok = page >= 0 && page < v.pool_pages;
-    ph = (page_ok ? page : 0) * Hkv + g;  // the (page, head) block
-    row0 = ph * v.page_slots + slot0 % v.page_slots;
+    row0 = ((page_ok ? page : 0) * Hkv + g) * v.page_slots + slot0 % v.page_slots;
     fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
          ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
   };
 
-  // The K and V copies of one chunk into a stage (and for FP8 pools its 32 exponents).  row0:
-  // the chunk's first row of the pool's rows, ph its (page, head) block; for FP8 the transposed
-  // V block of ph starts at element row ph * 128, the chunk at column row0 - ph * page_slots.
-  auto issue_kv = [&](int stage, int row0, int ph, uint64_t pol) {
-    uint8_t *dst = stages + stage * S::kStageBytes;
-    if constexpr (kFp8) {
-      tma_load_2d(dst, &tmap_k, 0, row0, &full[stage], pol);
-      tma_load_2d(dst + S::kChunkBytes, &tmap_v, row0 - ph * v.page_slots, ph * D, &full[stage],
-                  pol);
-      bulk_load(stages + S::kOffE + stage * S::kExpBytes,
-                v.kv_exp + (int64_t)row0 * (S::kExpBytes / kChunkSlots), (uint32_t)S::kExpBytes,
-                &full[stage]);
-    } else {
-      (void)ph;
-      tma_load_3d(dst, &tmap_k, 0, 0, row0, &full[stage], pol);
-      tma_load_3d(dst + S::kChunkBytes, &tmap_v, 0, 0, row0, &full[stage], pol);
-    }
-  };
-
   // The first ring's worth of K/V copies.  Their stages expect the K/V bytes now and arrive
   // (with the bytes of q and the step rows, if the stage opens a segment) after the wait.
-  int seg0 = 0, valid0 = 0, fl0 = 0, row00 = 0, ph00 = 0, pre = 0;
+  int seg0 = 0, valid0 = 0, fl0 = 0, row00 = 0, pre = 0;
   if (warp == 1 && active_cta) {
     const int nb = min(32, nchunks);
-    if (lane < nb) decode(0, seg0, valid0, fl0, row00, ph00);
+    if (lane < nb) decode(0, seg0, valid0, fl0, row00);
     pre = min(nb, S::kStages);
     const uint64_t pol = policy_evict_first();
     for (int j = 0; j < pre; ++j) {
       const int s_fl = __shfl_sync(kFull, fl0, j);
       const int s_row = __shfl_sync(kFull, row00, j);
-      const int s_ph = kFp8 ? __shfl_sync(kFull, ph00, j) : 0;
       if (lane == 0 && (s_fl & kPageOk)) {
-        mbar_expect_tx(&full[j], (uint32_t)S::kTxBytes);
-        issue_kv(j, s_row, s_ph, pol);
+        uint8_t *dst = stages + j * S::kStageBytes;
+        mbar_expect_tx(&full[j], (uint32_t)S::kStageBytes);
+        tma_load_3d(dst, &tmap_k, 0, 0, s_row, &full[j], pol);
+        tma_load_3d(dst + S::kChunkBytes, &tmap_v, 0, 0, s_row, &full[j], pol);
       }
     }
   }
@@ -354,15 +299,14 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
     int it = 0, nseg = 0;
     for (int base = 0; base < nchunks; base += 32) {
       const int nb = min(32, nchunks - base);
-      int seg = seg0, valid = valid0, fl = fl0, row0 = row00, ph = ph00;
-      if (base > 0 && lane < nb) decode(base, seg, valid, fl, row0, ph);
+      int seg = seg0, valid = valid0, fl = fl0, row0 = row00;
+      if (base > 0 && lane < nb) decode(base, seg, valid, fl, row0);
       bool stop = false;
       for (int j = 0; j < nb; ++j) {
         const int s_seg = __shfl_sync(kFull, seg, j);
         const int s_valid = __shfl_sync(kFull, valid, j);
         const int s_fl = __shfl_sync(kFull, fl, j);
         const int s_row = __shfl_sync(kFull, row0, j);
-        const int s_ph = kFp8 ? __shfl_sync(kFull, ph, j) : 0;
         const bool issued = it < pre;  // K/V already on their way (first ring)
         int failed = 0;
         if (lane == 0) {
@@ -378,7 +322,7 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
             const int b = s_seg / Hkv;
             if (s_fl & kFirst) qb = nseg++ % S::kQBufs;
             info[stage] = make_int4(s_seg, s_valid, s_fl, qb);
-            uint32_t bytes = ((s_fl & kPageOk) && !issued) ? (uint32_t)S::kTxBytes : 0u;
+            uint32_t bytes = ((s_fl & kPageOk) && !issued) ? (uint32_t)S::kStageBytes : 0u;
             if (qb >= 0) {
               if (it > 0) bytes += (uint32_t)sb.q_bytes;  // (the first one is on its way)
               if constexpr (kStep) {
@@ -389,10 +333,12 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
             }
             if (bytes) mbar_arrive_tx(&full[stage], bytes);
             else mbar_arrive(&full[stage]);
+            uint8_t *dst = stages + stage * S::kStageBytes;
             if (!(s_fl & kPageOk)) {
               record_error(v.err, HAM_DEVERR_PAGE);
             } else if (!issued) {
-              issue_kv(stage, s_row, s_ph, pol);
+              tma_load_3d(dst, &tmap_k, 0, 0, s_row, &full[stage], pol);
+              tma_load_3d(dst + S::kChunkBytes, &tmap_v, 0, 0, s_row, &full[stage], pol);
             }
             if (qb >= 0) {
               uint8_t *qdst = qbufs + qb * sb.stride;
@@ -419,277 +365,6 @@ __global__ void __launch_bounds__(Shape<D, kFp8>::kThreads, kFp8 ? kDefaultCtasP
     if (lane == 0) {
       for (int i = max(0, it - S::kStages); i < it; ++i)
         thread_wait(&full[i % S::kStages], (uint32_t)(i / S::kStages) & 1u, flags, false);
-    }
-    return;
-  }
-
-  if constexpr (kFp8) {
-    // ------------------------------------------------------------ consumer warp, FP8 pools
-    // The codes become f16 values (cvt, exact: every e4m3 value is an f16 value) in the
-    // registers of f16 products (mma.sync m16n8k16, fp32 accumulate): S^T = K Q^T (16 slots x
-    // 8 heads) and O^T += V^T P^T, as for bf16 pools.  (The e4m3 form of mma.sync ran about
-    // 1.3x slower here: the tensor path for e4m3 operands on this GPU is tcgen05.)  Scales are
-    // powers of two: q enters as q 2^-f per head (its largest element in [2^14, 2^15)), the key
-    // exponents scale the scores exactly in fp32, and the weights enter as p 2^(e_v - Eo + 7),
-    // where Eo of a head is the largest e_v + exponent(p) of its segment so far (lowered by the
-    // whole binades a raised maximum takes off the earlier weights): every weight stays below
-    // 2^8, and the ones that matter far above f16's smallest values, however far apart the rows'
-    // scales are.  One k-step takes a lane's four consecutive code bytes as its columns 2cq,
-    // 2cq + 1, 2cq + 8, 2cq + 9: in the scores the head dims 16k + 4cq .. + 3 (a dot product
-    // does not depend on the order of its terms; q takes the same order), in the values the
-    // slots 2cq, 2cq + 1, 8 + 2cq, 9 + 2cq, the order in which a chunk's transposed value rows
-    // keep their slots (ham.h, "FP8 (e4m3) pools").
-    const int r0 = lane >> 2, cq = lane & 3;   // fragment row (slot / head dim), column pair
-    const int h0 = 2 * cq, h1 = 2 * cq + 1;    // the heads of this lane's S^T / O^T columns
-    const bool hv0 = h0 < G, hv1 = h1 < G, hq = r0 < G;
-    const float qscale = rsqrtf((float)D) * 1.4426950408889634f;  // 1/sqrt(d) * log2(e)
-    constexpr int kNoExp = -1000;
-    constexpr int kKSteps = D / 16, kMTiles = D / 16;
-    uint32_t qb[kKSteps][2];     // B fragments of Q^T (f16, scaled by 2^-f)
-    float o[kMTiles][4];         // O^T: rows = head dims, columns = heads h0, h1
-    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f, qs0 = 0.f, qs1 = 0.f;
-    int E0 = kNoExp, E1 = kNoExp;  // O^T column h0 (h1) is in units of 2^(E0 - 7) (2^(E1 - 7))
-#pragma unroll
-    for (int i = 0; i < kMTiles; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-#pragma unroll
-    for (int k = 0; k < kKSteps; ++k) qb[k][0] = qb[k][1] = 0u;
-    // one head's rescale: the maximum m rises to mn and (fp8) Eo by whole binades
-    auto raise = [](float m, float mn, int Eo, float &a, float &al, int &Eo1) {
-      a = 1.f;
-      al = 1.f;
-      Eo1 = Eo;
-      if (mn > m) {
-        if (m == -INFINITY) {
-          al = 0.f;  // nothing accumulated yet
-        } else {
-          const float dm = mn - m;
-          const int k = dm < 1.0e6f ? (int)dm : 1000000;
-          a = ex2((float)k - dm);
-          al = ex2(m - mn);
-          if (Eo != kNoExp) Eo1 = max(Eo - k, kNoExp + 1);
-        }
-      }
-    };
-    auto pexp = [](float p) { return (int)((__float_as_uint(p) >> 23) & 0xFFu) - 127; };
-    for (int it = 0; it < nchunks; ++it) {
-      const int stage = it % S::kStages;
-      if (!warp_wait(&full[stage], (uint32_t)(it / S::kStages) & 1u, flags, wait_lim)) {
-        if (lane == 0) {
-          record_error(v.err, HAM_DEVERR_TIMEOUT);
-          flags[0] = 1;
-        }
-        return;
-      }
-      const int4 inf = info[stage];
-      if (inf.z & kFirst) {  // q of a new segment as f16, times 2^-f (heads >= G: zero)
-        const uint16_t *q = reinterpret_cast<const uint16_t *>(qbufs + inf.w * sb.stride);
-        // lane (r0, cq) holds head r0's elements 16k + 4cq .. + 3
-        float qv[kKSteps][4];
-#pragma unroll
-        for (int k = 0; k < kKSteps; ++k) {
-          uint2 w = make_uint2(0u, 0u);
-          if (hq) w = *reinterpret_cast<const uint2 *>(q + r0 * D + 16 * k + 4 * cq);
-          qv[k][0] = __uint_as_float(w.x << 16);
-          qv[k][1] = __uint_as_float(w.x & 0xFFFF0000u);
-          qv[k][2] = __uint_as_float(w.y << 16);
-          qv[k][3] = __uint_as_float(w.y & 0xFFFF0000u);
-        }
-        if constexpr (kStep) {
-          // the fused step: q turned by the new slot's position in fp32 and rounded to bf16, as
-          // the bf16 pass does; element j < D/2 and its partner j + D/2 sit in k-steps k, k + 4
-          const int b = inf.x / Hkv;
-          float2 *cs = reinterpret_cast<float2 *>(qbufs + inf.w * sb.stride + sb.cs_off());
-          if (appb[b]) {
-            const int64_t p = posb[b];
-            if (!(p >= 0 && p < v.step.rope_positions))
-              fill_cs_row(cs, p, v.step.inv_freq, D / 2, lane);
-          }
-          if (appb[b] && hq) {
-#pragma unroll
-            for (int k = 0; k < kKSteps / 2; ++k)
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const float2 c = cs[16 * k + 4 * cq + e];
-                const float a = qv[k][e], bb = qv[k + kKSteps / 2][e];
-                qv[k][e] = __bfloat162float(__float2bfloat16_rn(a * c.x - bb * c.y));
-                qv[k + kKSteps / 2][e] = __bfloat162float(__float2bfloat16_rn(bb * c.x + a * c.y));
-              }
-          }
-        }
-        float amax = 0.f;
-#pragma unroll
-        for (int k = 0; k < kKSteps; ++k)
-          amax = fmaxf(amax, fmaxf(fmaxf(fabsf(qv[k][0]), fabsf(qv[k][1])),
-                                   fmaxf(fabsf(qv[k][2]), fabsf(qv[k][3]))));
-        amax = fmaxf(amax, __shfl_xor_sync(kFull, amax, 1));
-        amax = fmaxf(amax, __shfl_xor_sync(kFull, amax, 2));
-        int f = 0;
-        if (amax > 0.f) {
-          int E = 0;
-          frexpf(amax, &E);
-          // (clamped so that 2^+-f stays a normal float: a head whose largest element lies
-          // below 2^-85 keeps fewer bits of its smallest elements)
-          f = min(max(E - 15, -100), 100);
-        }
-        const float sc = pow2i(-f);
-#pragma unroll
-        for (int k = 0; k < kKSteps; ++k) {
-          qb[k][0] = pack_f16x2(qv[k][0] * sc, qv[k][1] * sc);
-          qb[k][1] = pack_f16x2(qv[k][2] * sc, qv[k][3] * sc);
-        }
-        const float qs = qscale * pow2i(f);  // head r0's; the columns' heads are h0, h1
-        qs0 = __shfl_sync(kFull, qs, 4 * h0);
-        qs1 = __shfl_sync(kFull, qs, 4 * h1);
-      }
-      if (inf.z & kPageOk) {
-        const uint8_t *kt = stages + stage * S::kStageBytes;
-        const uint8_t *vt = kt + S::kChunkBytes;
-        const int8_t *ex = reinterpret_cast<const int8_t *>(stages + S::kOffE + stage * S::kExpBytes);
-        const int nvalid = inf.y;
-        // A fragments of K: code rows r0 and 8 + r0, bytes 16k + 4cq ..: 16-byte piece k, at
-        // piece k ^ (row & 7) in the 128-byte swizzle, i.e. the address of piece 0 XOR 16 k
-        // (the tile is 1024-byte aligned)
-        const uint32_t ka = smem_u32(kt) + r0 * 128 + ((r0 & 7) << 4) + 4 * cq;
-        const uint32_t kb = ka + 8 * 128;
-        float sh[4] = {0.f, 0.f, 0.f, 0.f}, sl[4] = {0.f, 0.f, 0.f, 0.f};  // even, odd k-steps
-#pragma unroll
-        for (int k = 0; k < kKSteps; ++k) {
-          uint32_t a[4];
-          e4m3x4_to_f16x2(ld_shared_u32(ka ^ (uint32_t)(k << 4)), a[0], a[2]);
-          e4m3x4_to_f16x2(ld_shared_u32(kb ^ (uint32_t)(k << 4)), a[1], a[3]);
-          if (k & 1) mma_16816_f16(sl, a, qb[k][0], qb[k][1]);
-          else mma_16816_f16(sh, a, qb[k][0], qb[k][1]);
-        }
-        const bool v0 = r0 < nvalid, v1 = r0 + 8 < nvalid;
-        const float ka0 = pow2i(ex[r0]), ka1 = pow2i(ex[r0 + 8]);
-        const float x0 = (v0 && hv0) ? (sh[0] + sl[0]) * ka0 * qs0 : -INFINITY;  // (k-steps)
-        const float x1 = (v0 && hv1) ? (sh[1] + sl[1]) * ka0 * qs1 : -INFINITY;
-        const float x2 = (v1 && hv0) ? (sh[2] + sl[2]) * ka1 * qs0 : -INFINITY;
-        const float x3 = (v1 && hv1) ? (sh[3] + sl[3]) * ka1 * qs1 : -INFINITY;
-        float t0 = fmaxf(x0, x2), t1 = fmaxf(x1, x3);
-#pragma unroll
-        for (int off = 4; off < 32; off <<= 1) {
-          t0 = fmaxf(t0, __shfl_xor_sync(kFull, t0, off));
-          t1 = fmaxf(t1, __shfl_xor_sync(kFull, t1, off));
-        }
-        const float n0 = t0 > m0 + kRescaleSlack ? fmaxf(m0, t0) : m0;
-        const float n1 = t1 > m1 + kRescaleSlack ? fmaxf(m1, t1) : m1;
-        float a0, al0, a1, al1;
-        int F0, F1;
-        raise(m0, n0, E0, a0, al0, F0);
-        raise(m1, n1, E1, a1, al1, F1);
-        const float p0 = (x0 == -INFINITY) ? 0.f : ex2(x0 - n0);
-        const float p1 = (x1 == -INFINITY) ? 0.f : ex2(x1 - n1);
-        const float p2 = (x2 == -INFINITY) ? 0.f : ex2(x2 - n0);
-        const float p3 = (x3 == -INFINITY) ? 0.f : ex2(x3 - n1);
-        // Eo of each head: the largest e_v + exponent(p) over the chunk's slots
-        const int ev0 = ex[kChunkSlots + r0], ev1 = ex[kChunkSlots + r0 + 8];
-        int c0 = max(p0 > 0.f ? ev0 + pexp(p0) : kNoExp, p2 > 0.f ? ev1 + pexp(p2) : kNoExp);
-        int c1 = max(p1 > 0.f ? ev0 + pexp(p1) : kNoExp, p3 > 0.f ? ev1 + pexp(p3) : kNoExp);
-#pragma unroll
-        for (int off = 4; off < 32; off <<= 1) {
-          c0 = max(c0, __shfl_xor_sync(kFull, c0, off));
-          c1 = max(c1, __shfl_xor_sync(kFull, c1, off));
-        }
-        const int G0 = max(F0, c0), G1 = max(F1, c1);
-        if (__any_sync(kFull, n0 != m0 || n1 != m1 || G0 != E0 || G1 != E1)) {
-          const float f0 = a0 * ((G0 > F0 && F0 != kNoExp) ? pow2i(max(F0 - G0, -127)) : 1.f);
-          const float f1 = a1 * ((G1 > F1 && F1 != kNoExp) ? pow2i(max(F1 - G1, -127)) : 1.f);
-#pragma unroll
-          for (int i = 0; i < kMTiles; ++i) {
-            o[i][0] *= f0;
-            o[i][2] *= f0;
-            o[i][1] *= f1;
-            o[i][3] *= f1;
-          }
-        }
-        l0 = l0 * al0 + (p0 + p2);
-        l1 = l1 * al1 + (p1 + p3);
-        m0 = n0;
-        m1 = n1;
-        E0 = G0;
-        E1 = G1;
-        // the weights p 2^(e_v - Eo + 7) (< 2^8) as f16 pairs (slot r0 | r0 + 8: heads h0, h1),
-        // moved into the B layout: P^T rows (slots) 2cq, 2cq + 1 | 8 + 2cq, 9 + 2cq of head r0
-        auto wgt = [](float p, int ev, int Eo) {
-          return p > 0.f ? p * pow2i(min(ev - Eo + 7, 127)) : 0.f;
-        };
-        const uint32_t bp0 = movmatrix_trans(pack_f16x2(wgt(p0, ev0, G0), wgt(p1, ev0, G1)));
-        const uint32_t bp1 = movmatrix_trans(pack_f16x2(wgt(p2, ev1, G0), wgt(p3, ev1, G1)));
-        // O^T += V^T P^T: V^T rows 16i + r0 and 16i + r0 + 8, bytes 4cq .. 4cq + 3 (slots
-        // 2cq, 2cq + 1 -> columns 2cq, 2cq + 1; slots 8 + 2cq, 9 + 2cq -> columns 2cq + 8, + 9)
-#pragma unroll
-        for (int i = 0; i < kMTiles; ++i) {
-          uint32_t a[4];
-          e4m3x4_to_f16x2(*reinterpret_cast<const uint32_t *>(vt + (16 * i + r0) * 16 + 4 * cq),
-                          a[0], a[2]);
-          e4m3x4_to_f16x2(
-              *reinterpret_cast<const uint32_t *>(vt + (16 * i + r0 + 8) * 16 + 4 * cq), a[1],
-              a[3]);
-          mma_16816_f16(o[i], a, bp0, bp1);
-        }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[stage]);
-
-      if (!(inf.z & kLast)) continue;
-
-      // ---------------------------------------------------------- end of a segment
-      const int seg = inf.x;
-#pragma unroll
-      for (int off = 4; off < 32; off <<= 1) {
-        l0 += __shfl_xor_sync(kFull, l0, off);
-        l1 += __shfl_xor_sync(kFull, l1, off);
-      }
-      const int b = seg / Hkv, gk = seg - b * Hkv;
-      const int nch = cum[b + 1] - cum[b];
-      const int64_t X0 = (int64_t)Hkv * cum[b] + (int64_t)gk * nch;
-      const int first = plan_owner(W, C, X0), last = plan_owner(W, C, X0 + nch - 1);
-      const int64_t obase = (int64_t)seg * G * D;
-      // O^T back from units of 2^(Eo - 7) (0 below fp32's normal range)
-      const float r0s = E0 == kNoExp ? 0.f : pow2i(max(E0 - 7, -127));
-      const float r1s = E1 == kNoExp ? 0.f : pow2i(max(E1 - 7, -127));
-      // (fused step: the combine kernel still adds the appended slot, so always the partials)
-      if (!kStep && first == last) {
-        const float i0 = l0 > 0.f ? r0s / l0 : 0.f, i1 = l1 > 0.f ? r1s / l1 : 0.f;
-#pragma unroll
-        for (int i = 0; i < kMTiles; ++i) {
-          const int d0 = 16 * i + r0;
-          if (hv0) {
-            store_out<OutT>(v.out, obase + (int64_t)h0 * D + d0, o[i][0] * i0);
-            store_out<OutT>(v.out, obase + (int64_t)h0 * D + d0 + 8, o[i][2] * i0);
-          }
-          if (hv1) {
-            store_out<OutT>(v.out, obase + (int64_t)h1 * D + d0, o[i][1] * i1);
-            store_out<OutT>(v.out, obase + (int64_t)h1 * D + d0 + 8, o[i][3] * i1);
-          }
-        }
-      } else {  // partial state of this CTA; the combine kernel merges first..last
-        const int64_t pidx = (int64_t)blockIdx.x + seg;
-        float *pacc = v.part_acc + pidx * G * D;
-#pragma unroll
-        for (int i = 0; i < kMTiles; ++i) {
-          const int d0 = 16 * i + r0;
-          if (hv0) {
-            pacc[h0 * D + d0] = o[i][0] * r0s;
-            pacc[h0 * D + d0 + 8] = o[i][2] * r0s;
-          }
-          if (hv1) {
-            pacc[h1 * D + d0] = o[i][1] * r1s;
-            pacc[h1 * D + d0 + 8] = o[i][3] * r1s;
-          }
-        }
-        if (r0 == 0) {
-          if (hv0) v.part_ml[pidx * G + h0] = make_float2(m0, l0);
-          if (hv1) v.part_ml[pidx * G + h1] = make_float2(m1, l1);
-        }
-      }
-      if (lane == 0 && (int)blockIdx.x == first) v.seg_range[seg] = make_int2(first, last);
-#pragma unroll
-      for (int i = 0; i < kMTiles; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-      m0 = m1 = -INFINITY;
-      l0 = l1 = 0.f;
-      E0 = E1 = kNoExp;
     }
     return;
   }
@@ -1460,12 +1135,12 @@ cudaError_t launch_combine(const AttnView &v, int head_dim, cudaStream_t stream)
 // ------------------------------------------------------------------------------------
 // Dispatch
 // ------------------------------------------------------------------------------------
-template <int D, typename OutT, bool kStep, bool kFp8 = false>
+template <int D, typename OutT, bool kStep>
 struct Instance {
-  using S = Shape<D, kFp8>;
-  static auto fn() { return &decode_attn_kernel<D, OutT, kStep, kFp8>; }
+  using S = Shape<D>;
+  static auto fn() { return &decode_attn_kernel<D, OutT, kStep>; }
   static size_t smem_bytes(int group, int batch) {
-    return 1024 + (size_t)Layout<D, kFp8>(group, kStep, batch).total;
+    return 1024 + (size_t)Layout<D>(group, kStep, batch).total;
   }
   // Allow the largest dynamic shared memory any group and batch need, once per device.
   static cudaError_t configure() {
@@ -1495,7 +1170,7 @@ struct Instance {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<D, OutT, kStep, kFp8>, tk, tv, v);
+    e = cudaLaunchKernelEx(&cfg, decode_attn_kernel<D, OutT, kStep>, tk, tv, v);
     if (e != cudaSuccess) return e;
     return launch_combine<OutT, kStep>(v, D, stream);
   }
@@ -1526,10 +1201,12 @@ cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const
                              int head_dim, int out_dtype, cudaStream_t stream) {
   if (v.ctas < 1 || v.group < 1 || v.group > kMaxGroup) return cudaErrorInvalidConfiguration;
   auto go = [&](auto inst) { return decltype(inst)::launch(tk, tv, v, stream); };
-  if (v.kv_exp) {  // FP8 pools
+  if (v.kv_exp) {  // FP8 pools: the tcgen05 pass, then the same combine kernel
     if (head_dim != kFp8HeadDim) return cudaErrorInvalidValue;
-    return out_dtype == HAM_DTYPE_F32 ? go(Instance<kFp8HeadDim, float, false, true>())
-                                      : go(Instance<kFp8HeadDim, __nv_bfloat16, false, true>());
+    cudaError_t e = launch_fp8_attention_pass(tk, tv, v, out_dtype, false, stream);
+    if (e != cudaSuccess) return e;
+    return out_dtype == HAM_DTYPE_F32 ? launch_combine<float, false>(v, kFp8HeadDim, stream)
+                                      : launch_combine<__nv_bfloat16, false>(v, kFp8HeadDim, stream);
   }
   return out_dtype == HAM_DTYPE_F32 ? dispatch<float, false>(head_dim, go)
                                     : dispatch<__nv_bfloat16, false>(head_dim, go);
@@ -1539,10 +1216,12 @@ cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, con
                                int head_dim, int out_dtype, cudaStream_t stream) {
   if (v.ctas < 1 || v.group < 1 || v.group > kMaxGroup) return cudaErrorInvalidConfiguration;
   auto go = [&](auto inst) { return decltype(inst)::launch(tk, tv, v, stream); };
-  if (v.kv_exp) {  // FP8 pools
+  if (v.kv_exp) {  // FP8 pools: the tcgen05 pass, then the same combine kernel
     if (head_dim != kFp8HeadDim) return cudaErrorInvalidValue;
-    return out_dtype == HAM_DTYPE_F32 ? go(Instance<kFp8HeadDim, float, true, true>())
-                                      : go(Instance<kFp8HeadDim, __nv_bfloat16, true, true>());
+    cudaError_t e = launch_fp8_attention_pass(tk, tv, v, out_dtype, true, stream);
+    if (e != cudaSuccess) return e;
+    return out_dtype == HAM_DTYPE_F32 ? launch_combine<float, true>(v, kFp8HeadDim, stream)
+                                      : launch_combine<__nv_bfloat16, true>(v, kFp8HeadDim, stream);
   }
   return out_dtype == HAM_DTYPE_F32 ? dispatch<float, true>(head_dim, go)
                                     : dispatch<__nv_bfloat16, true>(head_dim, go);
@@ -1550,22 +1229,14 @@ cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, con
 
 int attention_ctas_per_sm(int head_dim, int group, int batch, bool step, int out_dtype,
                           bool fp8) {
+  if (fp8)
+    return head_dim == kFp8HeadDim ? fp8_attention_ctas_per_sm(group, batch, step, out_dtype) : 0;
   int n = 0;
   auto q = [&](auto inst) {
     n = decltype(inst)::ctas_per_sm(group, batch);
     return cudaSuccess;
   };
   const bool f32 = out_dtype == HAM_DTYPE_F32;
-  if (fp8) {
-    if (head_dim != kFp8HeadDim) return 0;
-    if (step)
-      f32 ? q(Instance<kFp8HeadDim, float, true, true>())
-          : q(Instance<kFp8HeadDim, __nv_bfloat16, true, true>());
-    else
-      f32 ? q(Instance<kFp8HeadDim, float, false, true>())
-          : q(Instance<kFp8HeadDim, __nv_bfloat16, false, true>());
-    return n;
-  }
   if (step) f32 ? dispatch<float, true>(head_dim, q) : dispatch<__nv_bfloat16, true>(head_dim, q);
   else f32 ? dispatch<float, false>(head_dim, q) : dispatch<__nv_bfloat16, false>(head_dim, q);
   return n;

@@ -78,9 +78,8 @@ __host__ __device__ inline int32_t chunks_of(int32_t slots) {
 // wave (a CTA that starts late doubles the launch: the split plan gives every CTA an equal
 // share).
 constexpr int kDefaultCtasPerSm = 4;
-// FP8 pools: 16 KiB rings, so twice the CTAs keep the same bytes in flight, and their consumer
-// warps (which convert codes as well) get a second warp per scheduler.
-constexpr int kDefaultCtasPerSmFp8 = 8;
+// FP8 pools: two CTAs an SM, each with a ring of three 32 KiB tiles (ham_attn_fp8.cu).
+constexpr int kDefaultCtasPerSmFp8 = 2;
 inline int32_t default_attention_ctas(int32_t num_sms, int32_t resident_per_sm,
                                       bool fp8 = false) {
   const int32_t cap = fp8 ? kDefaultCtasPerSmFp8 : kDefaultCtasPerSm;
@@ -178,6 +177,13 @@ cudaError_t launch_attention(const CUtensorMap &tk, const CUtensorMap &tv, const
 // Fused decode step: attention with the append of v.step folded in, then combine + counters.
 cudaError_t launch_decode_step(const CUtensorMap &tk, const CUtensorMap &tv, const AttnView &v,
                                int head_dim, int out_dtype, cudaStream_t stream);
+// The attention pass over FP8 pools (ham_attn_fp8.cu: tcgen05 products of e4m3 operands over
+// 128-slot tiles), without the combine kernel that follows it; step: the fused decode step's
+// pass.  Same plan, partials and errors as the bf16 pass.
+cudaError_t launch_fp8_attention_pass(const CUtensorMap &tk, const CUtensorMap &tv,
+                                      const AttnView &v, int out_dtype, bool step,
+                                      cudaStream_t stream);
+int fp8_attention_ctas_per_sm(int group, int batch, bool step, int out_dtype);
 // CTAs of one SM for the attention kernel of this shape and output type (0 if the shape is not
 // compiled).
 int attention_ctas_per_sm(int head_dim, int group, int batch, bool step,
