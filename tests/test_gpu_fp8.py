@@ -166,8 +166,10 @@ def test_append_stores_the_oracle_encoding(pos_mode, hq, hkv):
     (32, 8, 128, (256, 3), 1.0),
     (8, 8, 16, (300, 33), 1.0),                       # group 1
     (16, 8, 16, (300, 33), 1.0),                      # group 2
-    (64, 8, 16, (300, 33), 1.0),                      # group 8
-    (24, 8, 16, (129, 64), 1.0),                      # group 3 (padded to 8)
+    (64, 8, 16, (300, 33), 1.0),                      # group 8 (32 product columns)
+    (24, 8, 16, (129, 64), 1.0),                      # group 3
+    (40, 8, 16, (1000, 129), 1.0),                    # group 5: every one of 16 columns in use
+    (48, 8, 32, (700, 15), 1.0),                      # group 6: 32 columns, 18 in use
 ])
 def test_decode_over_fp8_matches_oracle(hq, hkv, page, counts, scale):
     case = small_case(batch=len(counts), hq=hq, hkv=hkv, d=128, page=page, counts=counts,
@@ -274,6 +276,7 @@ Q_ROT_UNWRITTEN = 0x7FC1  # a bf16 NaN pattern no rotation produces
     (32, 8, 32, (31, 200, 5)),             # page edge
     (8, 8, 16, (1, 64)),                   # group 1
     (64, 8, 128, (127, 300)),              # group 8
+    (40, 8, 16, (127, 128, 129)),          # group 5; one slot short of / exactly / past a tile
 ])
 def test_fp8_step_matches_oracle(pos_mode, hq, hkv, page, counts):
     """ham_decode_step on an FP8 cache: the stored codes and exponents, the counters and q_rot

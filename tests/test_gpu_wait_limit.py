@@ -41,6 +41,30 @@ def test_decode_attention_wait_runs_out_then_recovers():
     assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
 
 
+def test_fp8_decode_attention_wait_runs_out_then_recovers():
+    """The FP8 pass (tcgen05 over 128-slot tiles): its ring, product and four-warp waits give up
+    on the shortened limit; the copies and products in flight are waited for, the tensor memory
+    freed, and the handle decodes at parity afterwards."""
+    from test_gpu_fp8 import fp8_cache, _reference, _decode
+    t = torch()
+    case = small_case(batch=1, hq=32, hkv=8, d=128, page=16, counts=(8192,), seed=45)
+    kv = fp8_cache(case)
+    ham.ham_kv_set_attn_ctas(kv, 1)          # one CTA: 512 chunks through one 3-tile ring
+    ham.ham_kv_set_wait_limit_ns(kv, 1)
+    q = dev_bf16(case.q)
+    out = t.zeros(q.shape, dtype=t.float32, device="cuda")
+    ham.ham_decode_attn_ex(kv, 0, q, out)
+    t.cuda.synchronize()
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_TIMEOUT
+    ham.ham_kv_set_wait_limit_ns(kv, 0)
+    ref = _reference(case).decode_attn(case.q)
+    assert_parity(_decode(kv, case.q, f32=True), ref, max_abs=3e-3, mean_abs=3e-4,
+                  what="FP8 after the timeout, one CTA")
+    ham.ham_kv_set_attn_ctas(kv, 0)
+    assert_parity(_decode(kv, case.q), ref, what="FP8 after the timeout, default CTAs")
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+
+
 def test_prefill_wait_runs_out_then_recovers():
     t = torch()
     w = wl.Workload("prefill_timeout", batch=1, n_q_heads=32, n_kv_heads=8, head_dim=128,
