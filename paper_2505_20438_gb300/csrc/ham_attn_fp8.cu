@@ -61,6 +61,7 @@ constexpr int kSoftWarps = 4, kSoftThreads = 32 * kSoftWarps;
 constexpr int kProducerWarp = 4, kIssuerWarp = 5;
 constexpr int kThreads8 = 32 * 6;
 constexpr int kEnd = 8;                                 // tile flag: the CTA's last tile
+constexpr int kPreTiles = 1;  // tiles whose copies `early` issues before the dependency wait
 static_assert(kTileSlots == kSoftThreads && kD8 == kSoftThreads, "one TMEM lane per thread");
 
 template <int kCols>
@@ -247,6 +248,74 @@ __global__ void __launch_bounds__(kThreads8, 2)
   const int64_t x1 = active_cta ? plan_cta_begin(W, C, (int64_t)blockIdx.x + 1) : 0;
   const int nchunks = (int)(x1 - x0);
 
+  // ---- the producer's first 32 chunks, decoded before the dependency wait (their counters and
+  // page-table entries are this layer's state).  With `early`, the K / V / exponent copies of
+  // the first tile are issued then too, and the first segment's q is prefetched into L2 (a
+  // prefetch reads nothing into the CTA; the copy of q after the wait takes it as the previous
+  // kernel left it).  (Three tiles before the wait measured slower: their 72 copies take ~2.5 us
+  // to issue and held back the first tile's q when the wait returned sooner.)
+  auto decode = [&](int64_t x, int &seg, int &valid, int &fl, int &row0, int &ph, int &c) {
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if ((int64_t)Hkv * cum[mid] <= x) lo = mid; else hi = mid - 1;
+    }
+    const int b = lo;
+    const int nch = cum[b + 1] - cum[b];
+    const int r = (int)(x - (int64_t)Hkv * cum[b]);
+    const int g = r / nch;
+    c = r - g * nch;
+    seg = b * Hkv + g;
+    valid = min(kChunkSlots, lens[b] - c * kChunkSlots);
+    const int slot0 = c * kChunkSlots;
+    const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
+    const bool page_ok = page >= 0 && page < v.pool_pages;
+    ph = (page_ok ? page : 0) * Hkv + g;
+    row0 = ph * v.page_slots + slot0 % v.page_slots;
+    fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
+         ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
+  };
+  const uint64_t pol = policy_evict_first();
+  const uint32_t q_bytes = (uint32_t)(G * kD8 * 2);
+  // 16-slot pages: a chunk's transposed value rows are one contiguous 2 KiB block
+  const bool v_block = v.page_slots == kChunkSlots;
+  const uint8_t *v_codes = reinterpret_cast<const uint8_t *>(v.v_pool);
+  // this lane's chunk's copies into position `pos` of a stage's tile
+  auto issue_chunk = [&](int stage, int pos, int row0, int ph) {
+    uint8_t *dst = ring + stage * kStage8 + pos * kBox8;
+    tma_load_2d(dst, &tmap_k, 0, row0, &full[stage], pol);
+    if (v_block)
+      bulk_load(dst + kHalf8, v_codes + (int64_t)ph * kD8 * kChunkSlots, (uint32_t)kBox8,
+                &full[stage]);
+    else
+      tma_load_2d(dst + kHalf8, &tmap_v, row0 - ph * v.page_slots, ph * kD8, &full[stage], pol);
+    bulk_load(exps + (stage * kTileChunks + pos) * kChunkExp,
+              v.kv_exp + (int64_t)row0 * (kChunkExp / kChunkSlots), (uint32_t)kChunkExp,
+              &full[stage]);
+  };
+  int d_seg = 0, d_valid = 0, d_fl = 0, d_row0 = 0, d_ph = 0, d_c = 0;  // lane: chunk x0 + lane
+  int pre = 0;  // tiles whose K / V copies are under way before the wait
+  if (active_cta && warp == kProducerWarp) {
+    const int nb = min(32, nchunks);
+    if (lane < nb) decode(x0 + lane, d_seg, d_valid, d_fl, d_row0, d_ph, d_c);
+    if (early) {
+      const uint32_t closes =
+          __ballot_sync(kFull, lane < nb && ((d_fl & kLast) || (d_c & 7) == 7));
+      const uint32_t okm = __ballot_sync(kFull, lane < nb && (d_fl & kPageOk));
+      const int last = 31 - __clz(closes);
+      if (lane == 0) bulk_prefetch_l2(v.q + (int64_t)d_seg * G * kD8, q_bytes);  // chunk x0's
+      for (int ts = 0; ts <= last && pre < kPreTiles;) {
+        const int te = ts + __ffs(closes >> ts) - 1;
+        const uint32_t tm = (okm >> ts) & ((1u << (te - ts + 1)) - 1u);
+        if (lane == 0) mbar_expect_tx(&full[pre], (uint32_t)__popc(tm) * (uint32_t)kChunkTx);
+        __syncwarp();
+        if (lane >= ts && lane <= te && (d_fl & kPageOk)) issue_chunk(pre, lane - ts, d_row0, d_ph);
+        ++pre;
+        ts = te + 1;
+      }
+    }
+  }
+
   if (early) {
     grid_dependency_wait();
     grid_launch_dependents();
@@ -289,40 +358,14 @@ __global__ void __launch_bounds__(kThreads8, 2)
     // (whole tiles of them); per tile lane 0 waits for the stage and posts the bytes to expect,
     // the tile's lanes issue the copies of their chunks together (the K box, the V block, the
     // 32 exponent bytes), and lane 0 records the tile and arrives.
-    auto decode = [&](int64_t x, int &seg, int &valid, int &fl, int &row0, int &ph, int &c) {
-      int lo = 0, hi = B - 1;
-      while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if ((int64_t)Hkv * cum[mid] <= x) lo = mid; else hi = mid - 1;
-      }
-      const int b = lo;
-      const int nch = cum[b + 1] - cum[b];
-      const int r = (int)(x - (int64_t)Hkv * cum[b]);
-      const int g = r / nch;
-      c = r - g * nch;
-      seg = b * Hkv + g;
-      valid = min(kChunkSlots, lens[b] - c * kChunkSlots);
-      const int slot0 = c * kChunkSlots;
-      const int page = v.page_table[(int64_t)b * v.max_pages + slot0 / v.page_slots];
-      const bool page_ok = page >= 0 && page < v.pool_pages;
-      ph = (page_ok ? page : 0) * Hkv + g;
-      row0 = ph * v.page_slots + slot0 % v.page_slots;
-      fl = (page_ok ? kPageOk : 0) | ((c == 0 || x == x0) ? kFirst : 0) |
-           ((c == nch - 1 || x == x1 - 1) ? kLast : 0);
-    };
-    const uint64_t pol = policy_evict_first();
-    const uint32_t q_bytes = (uint32_t)(G * kD8 * 2);
-    // 16-slot pages: a chunk's transposed value rows are one contiguous 2 KiB block
-    const bool v_block = v.page_slots == kChunkSlots;
-    const uint8_t *v_codes = reinterpret_cast<const uint8_t *>(v.v_pool);
     int tiles = 0, nseg = 0;
     bool stop = false;
     for (int base = 0; base < nchunks && !stop;) {
       const int nb = min(32, nchunks - base);
       const bool in = lane < nb;
       const int64_t x = x0 + base + lane;
-      int seg = 0, valid = 0, fl = 0, row0 = 0, ph = 0, c = 0;
-      if (in) decode(x, seg, valid, fl, row0, ph, c);
+      int seg = d_seg, valid = d_valid, fl = d_fl, row0 = d_row0, ph = d_ph, c = d_c;
+      if (base > 0 && in) decode(x, seg, valid, fl, row0, ph, c);
       const uint32_t closes = __ballot_sync(kFull, in && ((fl & kLast) || (c & 7) == 7));
       const uint32_t okm = __ballot_sync(kFull, in && (fl & kPageOk));
       // (the batch's last chunk closes a tile when nb < 32, and 32 chunks hold closes)
@@ -335,6 +378,7 @@ __global__ void __launch_bounds__(kThreads8, 2)
         const int t_seg = __shfl_sync(kFull, seg, ts);
         const int vlast = __shfl_sync(kFull, valid, te);
         const uint32_t tm = (okm >> ts) & ((1u << n) - 1u);  // chunks whose page is valid
+        const bool kv_issued = tiles < pre;                   // (before the wait)
         int failed = 0, qb = 0;
         if (lane == 0) {
           const uint32_t par = ((uint32_t)(tiles / kStages8) & 1u) ^ 1u;
@@ -343,7 +387,7 @@ __global__ void __launch_bounds__(kThreads8, 2)
             flags[0] = 1;
             failed = 1;
           } else {
-            uint32_t bytes = (uint32_t)__popc(tm) * (uint32_t)kChunkTx;
+            uint32_t bytes = kv_issued ? 0u : (uint32_t)__popc(tm) * (uint32_t)kChunkTx;
             bool tabled = false;
             int64_t p = 0;
             if (f0 & kFirst) {
@@ -370,19 +414,8 @@ __global__ void __launch_bounds__(kThreads8, 2)
           break;
         }
         __syncwarp();
-        if (lane >= ts && lane <= te && (fl & kPageOk)) {
-          uint8_t *dst = ring + stage * kStage8 + (lane - ts) * kBox8;
-          tma_load_2d(dst, &tmap_k, 0, row0, &full[stage], pol);
-          if (v_block)
-            bulk_load(dst + kHalf8, v_codes + (int64_t)ph * kD8 * kChunkSlots, (uint32_t)kBox8,
-                      &full[stage]);
-          else
-            tma_load_2d(dst + kHalf8, &tmap_v, row0 - ph * v.page_slots, ph * kD8, &full[stage],
-                        pol);
-          bulk_load(exps + (stage * kTileChunks + (lane - ts)) * kChunkExp,
-                    v.kv_exp + (int64_t)row0 * (kChunkExp / kChunkSlots), (uint32_t)kChunkExp,
-                    &full[stage]);
-        }
+        if (!kv_issued && lane >= ts && lane <= te && (fl & kPageOk))
+          issue_chunk(stage, lane - ts, row0, ph);
         __syncwarp();
         if (lane == 0) {
           const bool end = x0 + base + te == x1 - 1;

@@ -90,6 +90,11 @@ __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t b
       "l"(src), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
 }
+// Prefetch `bytes` of global memory (16-byte aligned, a multiple of 16) into L2: no shared memory,
+// no barrier, nothing returned to the thread.
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
 // Rank-3 tiled TMA copy of the box at (x, y, z) of `map` into shared memory.
 __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int x, int y,
                                             int z, uint64_t *bar, uint64_t policy) {
