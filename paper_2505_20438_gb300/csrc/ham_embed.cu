@@ -471,6 +471,7 @@ int ham_embedder_alloc(const ham_embed_config *cfg, const void *wq, const void *
 
 int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t batch,
               int32_t total_tokens, void *out, void *stream) {
+  ham::ApiRange nvtx_range("ham_embed");
   if (!e || !x || !offsets || !out) return efail(HAM_EINVAL, "null argument");
   if (!ham::aligned16(x)) return efail(HAM_EINVAL, "x must be 16-byte aligned");
   return ham::run_embed(e, static_cast<const __nv_bfloat16 *>(x), nullptr, offsets, batch,
@@ -479,6 +480,7 @@ int ham_embed(ham_embedder *e, const void *x, const int32_t *offsets, int32_t ba
 
 int ham_embed_tokens(ham_embedder *e, const int32_t *ids, const int32_t *offsets,
                      int32_t batch, int32_t total_tokens, void *out, void *stream) {
+  ham::ApiRange nvtx_range("ham_embed_tokens");
   if (!e || !ids || !offsets || !out) return efail(HAM_EINVAL, "null argument");
   if (e->vocab < 1) return efail(HAM_EINVAL, "no vocabulary set (ham_embedder_set_vocab)");
   if ((uintptr_t)ids & 3u) return efail(HAM_EINVAL, "ids must be 4-byte aligned");

@@ -8,6 +8,8 @@
 
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "ham.h"
 
 namespace ham {
@@ -265,6 +267,15 @@ __device__ inline int encode_e4m3_row(const float (&x)[4], uint32_t &codes) {
   return e;
 }
 
+// An NVTX range named after a C-ABI call, for the duration of the call (host side: the call's
+// launches and checks).  NVTX v3 is header-only; without a profiler attached a push and a pop
+// cost a load and a branch each.
+struct ApiRange {
+  explicit ApiRange(const char *name) { nvtxRangePushA(name); }
+  ~ApiRange() { nvtxRangePop(); }
+  ApiRange(const ApiRange &) = delete;
+  ApiRange &operator=(const ApiRange &) = delete;
+};
 // Record `msg` as this thread's ham_last_error() and return `status`.
 int set_last_error(int status, const char *msg);
 

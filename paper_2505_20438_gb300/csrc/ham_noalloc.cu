@@ -36,6 +36,7 @@ size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 extern "C" {
 
 int ham_decode_attn_noalloc(const ham_attn_args *a, void *stream) {
+  ham::ApiRange nvtx_range("ham_decode_attn_noalloc");
   if (!a) return noalloc_fail(HAM_EINVAL, "args is NULL");
   if (!a->k_pool || !a->v_pool || !a->page_table || !a->num_slots || !a->q || !a->out)
     return noalloc_fail(HAM_EINVAL, "k_pool, v_pool, page_table, num_slots, q and out are required");

@@ -692,6 +692,7 @@ int ham_kv_set_wait_limit_ns(ham_kv *kv, uint64_t ns) {
 
 int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
                   const void *v_new, const int32_t *pos, const int32_t *ntok, void *stream) {
+  ham::ApiRange nvtx_range("ham_kv_append");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if (!k_new || !v_new || !ntok) return fail(HAM_EINVAL, "k_new, v_new and ntok are required");
@@ -736,6 +737,7 @@ int ham_kv_append(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new,
 
 int ham_decode_attn_ex(ham_kv *kv, int32_t layer, const void *q, void *out, int32_t out_dtype,
                        void *stream) {
+  ham::ApiRange nvtx_range("ham_decode_attn_ex");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if (!q || !out) return fail(HAM_EINVAL, "q and out are required");
@@ -785,6 +787,7 @@ bool overlaps(const void *a, size_t a_bytes, const void *b, size_t b_bytes) {
 
 int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, int32_t hidden,
                    const int32_t *pos, const int32_t *ntok, void *q_rot, void *stream) {
+  ham::ApiRange nvtx_range("ham_qkv_append");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if ((rc = fp8_unsupported(kv, "ham_qkv_append")) != 0) return rc;
@@ -847,6 +850,7 @@ int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, 
 int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const void *k_new,
                     const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
                     int32_t out_dtype, void *stream) {
+  ham::ApiRange nvtx_range("ham_decode_step");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if (!q || !k_new || !v_new || !ntok || !out)
@@ -922,6 +926,7 @@ int ham_decode_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const
 int ham_micro_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const void *k_new,
                    const void *v_new, const int32_t *pos, const int32_t *ntok, void *out,
                    int32_t out_dtype, void *stream) {
+  ham::ApiRange nvtx_range("ham_micro_step");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if ((rc = fp8_unsupported(kv, "ham_micro_step")) != 0) return rc;
@@ -990,6 +995,7 @@ int ham_micro_step(ham_kv *kv, int32_t layer, const void *q, void *q_rot, const 
 int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, const void *v_new,
                 const int32_t *offsets, const int32_t *pos, const int32_t *ntok,
                 int32_t total_rows, void *out, int32_t out_dtype, void *stream) {
+  ham::ApiRange nvtx_range("ham_prefill");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if ((rc = fp8_unsupported(kv, "ham_prefill")) != 0) return rc;
@@ -1139,6 +1145,7 @@ int ham_kv_get_page_table(const ham_kv *kv, int32_t *host_pt) {
 int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
                 const int32_t *pos, const int32_t *ntok, const int32_t *counts, int32_t lmax,
                 void *stream) {
+  ham::ApiRange nvtx_range("ham_kv_fill");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if (!counts || lmax < 0 || (lmax > 0 && (!k_log || !v_log)))
@@ -1177,6 +1184,7 @@ int ham_kv_fill(ham_kv *kv, int32_t layer, const void *k_log, const void *v_log,
 
 int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *pos_dst,
                   int32_t *ntok_dst, void *stream) {
+  ham::ApiRange nvtx_range("ham_kv_export");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   DeviceGuard guard(kv->device);
@@ -1203,6 +1211,7 @@ int ham_kv_export_scales(ham_kv *kv, int32_t layer, void *e_dst, void *stream) {
 
 int ham_kv_set_lengths(ham_kv *kv, int32_t layer, const int32_t *num_slots,
                        const int64_t *num_tokens, void *stream) {
+  ham::ApiRange nvtx_range("ham_kv_set_lengths");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
   if (!num_slots) return fail(HAM_EINVAL, "num_slots is required");
