@@ -1712,6 +1712,15 @@ def prefill_flops(pw):
     return 4 * w.head_dim * w.n_q_heads * w.batch * attended
 
 
+def prefill_bytes(pw):
+    """Algorithmic bytes of one call: the K and V rows of every attended slot once per KV head
+    (cached and new), q in and out, k_new / v_new in."""
+    w = pw.w
+    T = pw.rows * w.batch
+    kv = w.batch * w.n_kv_heads * (pw.cached + pw.rows) * w.head_dim * 2 * 2
+    return kv + T * w.n_q_heads * w.head_dim * 2 * 2 + T * w.n_kv_heads * w.head_dim * 2 * 2
+
+
 def prefill_sample(pw, seconds, want_rows=None):
     """Rows of the chunk the CPU oracle attends in a bounded sample: evenly spread over every
     sequence's rows, so that their mean context is the chunk's."""
@@ -1866,6 +1875,12 @@ def run_prefill(args, pw):
     flops = prefill_flops(pw)
     peak, peak_src = measured_peak_bf16()
     achieved = flops / (call_ms * 1e-3) / 1e12
+    # the roofline that bounds the call: the contraction, or (a short chunk over a long cache)
+    # the stream of the cached rows
+    nbytes = prefill_bytes(pw)
+    hbm_peak, hbm_src = measured_peak_hbm()
+    gbs = nbytes / (call_ms * 1e-3) / 1e9
+    hbm_bound = nbytes / hbm_peak > flops / (peak * 1e3)  # seconds x 1e9, both sides
     value = world * T * steps / (elapsed_ms * 1e-3)
 
     # end to end: pinned host -> device copies of the chunk's q, k, v and offsets, the call,
@@ -1900,16 +1915,24 @@ def run_prefill(args, pw):
                    "page_slots": w.page_slots, "tokens_per_row": 1,
                    "step": "ham_kv_set_lengths + ham_prefill (plan, RoPE + append, causal "
                            "attention) of the whole chunk",
-                   "l2": "inputs larger than L2 (q, out 134 MB each at the 4 x 4096 chunk)"},
+                   "l2": ("inputs larger than L2 (q, out 134 MB each at the 4 x 4096 chunk)"
+                          if pw.rows * B >= 4096 else
+                          f"cached K and V ({prefill_bytes(pw) / 2**20:.0f} MiB) larger than L2")},
         "tflops": round(achieved, 1),
-        "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
-                     "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
-                     "kernel": "prefill_attn_kernel (with the plan and RoPE + append "
-                               "kernels of the same call)",
-                     "algorithmic_flops_per_launch": int(flops),
-                     "avg_launch_us": round(call_ms * 1e3, 1), "peak_source": peak_src,
-                     "duration_method": "CUDA events around one ham_prefill call (3 "
-                                        "kernels), median of 5"},
+        "roofline": dict(
+            ({"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+              "frac": round(gbs / hbm_peak, 4), "algorithmic_bytes_per_launch": int(nbytes),
+              "peak_source": hbm_src, "tensor_frac_of_measured": round(achieved / peak, 4)}
+             if hbm_bound else
+             {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
+              "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+              "algorithmic_flops_per_launch": int(flops), "peak_source": peak_src,
+              "hbm_frac_of_measured": round(gbs / hbm_peak, 4)}),
+            traffic=None,
+            kernel="prefill_attn_kernel (with the plan, RoPE + append and, when the grid "
+                   "splits over the cached slots, merge kernels of the same call)",
+            avg_launch_us=round(call_ms * 1e3, 1),
+            duration_method="CUDA events around one ham_prefill call, median of 5"),
         "gpu_launches": steps * 4 * world,
         "e2e": {"value": round(world * T * n_e2e / dte, 1), "unit": "rows/s",
                 "h2d_bytes_per_step": int(h2d),

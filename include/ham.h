@@ -251,7 +251,9 @@ int ham_slot_lengths(ham_kv *kv, int32_t *num_slots_host, int64_t *num_tokens_ho
  * page, offsets that leave the call's rows) gets no slot, keeps q unrotated and 0 out
  * rows, and sets the device error word.  total_rows == 0 launches nothing (the buffers may
  * then be NULL).  Three launches
- * on `stream` (plan, RoPE + append, attention).  q_inout, out, k_new and v_new must not
+ * on `stream` (plan, RoPE + append, attention), four when a short chunk lets the attention
+ * split over the cached slots (a merge of the splits' partials, kept in the handle's scratch;
+ * the result does not depend on the split).  q_inout, out, k_new and v_new must not
  * overlap each other or the cache.  Host errors: HAM_EINVAL (NULL / unaligned / overlapping
  * pointers, layer or out_dtype out of range, total_rows above batch * max_slots_per_seq),
  * HAM_ECUDA.  Same serialization rule as ham_decode_attn. */

@@ -317,6 +317,8 @@ struct ham_kv {
   int2 *seg_range = nullptr;
   int4 *prefill_seq = nullptr;     // ham_prefill: per-sequence plan [batch]
   int32_t *prefill_pos = nullptr;  // ham_prefill: per-row positions [batch * max_slots]
+  float *prefill_part = nullptr;   // ham_prefill: split partials (bf16 caches)
+  float2 *prefill_part_ml = nullptr;
   int64_t scratch_bytes = 0;
   std::vector<CUtensorMap> tmaps;  // [layers][2]: TMA maps of the K and V pools
   std::vector<CUtensorMap> tmaps_half;  // [layers][2]: the same, one 64-column half per box

@@ -8,7 +8,7 @@
 // softmax scale 1/sqrt(d), query head h reads KV head h / G).  Unlike decode this is a dense
 // contraction: every K/V tile serves 128 query rows, so it runs on the tensor cores.
 //
-// Three launches:
+// Three launches (four when the attention splits over the cached slots):
 //  1. prefill_plan_kernel, one block per sequence: checks that the sequence's rows fit
 //     (counts, capacity, pages), gives each row its position (slot index, running token count
 //     or the caller's), numbers the query blocks, and advances the counters.
@@ -32,6 +32,13 @@
 //     (the A operand of O += P V, so the next S is computed meanwhile) and rescale O there when
 //     the maximum moves.  The causal mask applies to the tiles that reach past a row's own slot;
 //     CTAs are scheduled latest query tiles first, the longest rows of the causal triangle.
+//     When the grid would leave SMs idle (a short chunk: few query blocks) it gets a third
+//     dimension, the split over slots: a sequence with L cached slots is cut into up to
+//     floor(L / 512) contiguous ranges of 64-slot tiles (the last range also takes the chunk's
+//     own slots), each CTA streams one range, and a split that is not alone leaves its rows'
+//     unnormalised output, running maximum and sum as a partial.
+//  4. prefill_merge_kernel (split launches only), one warp per (row, head): the split-softmax
+//     merge of the partials in split order (as the decode combine merges its CTAs').
 //
 // Every wait is bounded (about 2 s); a wait that runs out records HAM_DEVERR_TIMEOUT, lets the
 // CTA's copies land and returns.  No trap, no unbounded spin.
@@ -378,6 +385,16 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   ntile[1] = rows_q1 > 0 ? (L + qb0 + R + rows_q1 + S::kTile - 1) / S::kTile : 0;
   const int ntiles = max(ntile[0], ntile[1]);
   const int kv_end = L + qb0 + (rows_q1 > 0 ? R + rows_q1 : rows_q0);  // no slot >= is attended
+  // Split z of the sequence's zs takes tiles t0 .. t1 - 1: the cached part's whole tiles cut
+  // evenly, the last split also the rest (the chunk's own slots, the causal edge).  Every split
+  // starts at or before slot L - 64, which every row attends, so no row of a split is empty.
+  const int zs = prefill_splits(L, (int)gridDim.z), z = (int)blockIdx.z;
+  if (z >= zs) return;
+  const int Lt = L / S::kTile;
+  const int t0 = (int)((int64_t)z * Lt / zs);
+  const int t1 = z + 1 == zs ? ntiles : (int)((int64_t)(z + 1) * Lt / zs);
+  const int ntq[2] = {max(0, min(t1, ntile[0]) - t0), max(0, min(t1, ntile[1]) - t0)};
+  const int nts = max(ntq[0], ntq[1]);  // tiles this CTA streams
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -460,14 +477,15 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       return row;
     };
     constexpr int kTilesPerBatch = 32 / S::kChunks;
-    int row = lookup(0), row_next = lookup(32);
+    const int cbase = t0 * S::kChunks;  // the split's first chunk
+    int row = lookup(cbase), row_next = lookup(cbase + 32);
     int issued = 0;
-    for (int t = 0; t < ntiles; ++t) {
-      if (t > 0 && t % kTilesPerBatch == 0) {
+    for (int i = 0; i < nts; ++i) {  // tile t0 + i, the i-th of this CTA's ring
+      if (i > 0 && i % kTilesPerBatch == 0) {
         row = row_next;
-        row_next = lookup((t / kTilesPerBatch + 1) * 32);
+        row_next = lookup(cbase + (i / kTilesPerBatch + 1) * 32);
       }
-      int my_row = __shfl_sync(kFull, row, ((t % kTilesPerBatch) * S::kChunks + lane) & 31);
+      int my_row = __shfl_sync(kFull, row, ((i % kTilesPerBatch) * S::kChunks + lane) & 31);
       if (lane >= S::kChunks) my_row = -1;
       if (__any_sync(kFull, my_row == -2)) {  // the plan validated the table: this ends the CTA
         if (lane == 0) {
@@ -476,10 +494,10 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
         }
         break;
       }
-      const int st = t % stages;
+      const int st = i % stages;
       int ok_wait = 1;
-      if (lane == 0 && t >= stages)
-        ok_wait = thread_wait(&empty[st], (uint32_t)((t / stages) - 1) & 1u, abort_flag, true,
+      if (lane == 0 && i >= stages)
+        ok_wait = thread_wait(&empty[st], (uint32_t)((i / stages) - 1) & 1u, abort_flag, true,
                               wait_lim);
       if (!__shfl_sync(kFull, ok_wait, 0)) {
         if (lane == 0 && !*abort_flag) {
@@ -499,7 +517,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
           tma_load_3d(ring + st * S::kKVBytes + hh * S::kHalfTileBytes + lane * kChunkSlots * 128,
                       map, 0, hh, my_row, &full[st], pol_kv);
       }
-      issued = t + 1;
+      issued = i + 1;
     }
     if (lane == 0) {
       // every copy this warp issued lands before the CTA can exit
@@ -517,16 +535,16 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     // reads it; a tile that only one Q tile reaches is released twice by that tile's warp.
     const bool is_o = warp == S::kOWarp0 || warp == S::kOWarp1;
     const int q = (warp == S::kSWarp0 || warp == S::kOWarp0) ? 0 : 1;
-    const int nt = ntile[q], other = ntile[q ^ 1];
+    const int nt = ntq[q], other = ntile[q ^ 1];  // (tile t0 + i; other: absolute)
     bool ok = true;
     if (!is_o) {
       constexpr uint32_t id_s = idesc_bf16(128, S::kTile, false);  // K-major Q and K
       const uint32_t q_base = smem_u32(smem) + q * S::kQBytes;
       if (nt > 0) ok = warp_wait(q_full, 0u, abort_flag, wait_lim);
-      for (int t = 0; ok && t < nt; ++t) {
-        const int ks = t % S::kKStages;
-        if ((t > 0 && !warp_wait(&s_free[q], (uint32_t)(t - 1) & 1u, abort_flag, wait_lim)) ||
-            !warp_wait(&k_full[ks], (uint32_t)(t / S::kKStages) & 1u, abort_flag, wait_lim)) {
+      for (int i = 0; ok && i < nt; ++i) {
+        const int t = t0 + i, ks = i % S::kKStages;
+        if ((i > 0 && !warp_wait(&s_free[q], (uint32_t)(i - 1) & 1u, abort_flag, wait_lim)) ||
+            !warp_wait(&k_full[ks], (uint32_t)(i / S::kKStages) & 1u, abort_flag, wait_lim)) {
           ok = false;
           break;
         }
@@ -549,9 +567,9 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       }
     } else {
       constexpr uint32_t id_o = idesc_bf16(128, D, true);  // P from TMEM, MN-major V
-      for (int t = 0; ok && t < nt; ++t) {
-        const int vs = t % S::kVStages;
-        if (!warp_wait(&v_full[vs], (uint32_t)(t / S::kVStages) & 1u, abort_flag, wait_lim)) {
+      for (int i = 0; ok && i < nt; ++i) {
+        const int t = t0 + i, vs = i % S::kVStages;
+        if (!warp_wait(&v_full[vs], (uint32_t)(i / S::kVStages) & 1u, abort_flag, wait_lim)) {
           ok = false;
           break;
         }
@@ -568,7 +586,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
           fence_proxy_async_smem();
           __syncwarp();
         }
-        if (!warp_wait(&p_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
+        if (!warp_wait(&p_full[q], (uint32_t)i & 1u, abort_flag, wait_lim)) {
           ok = false;
           break;
         }
@@ -579,7 +597,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
           for (int k = 0; k < S::kTile / 16; ++k) {
             const uint64_t bv = smem_desc_sw128(vt + k * 2048, S::kHalfTileBytes, 1024);
             tc_mma_tmem_a(tmem + S::kOffO + q * D, tmem + S::kOffP + q * (S::kTile / 2) + k * 8,
-                          bv, id_o, t > 0 || k > 0);
+                          bv, id_o, i > 0 || k > 0);
           }
           tc_commit(&pv_done[q]);
           tc_commit(&v_empty[vs]);
@@ -613,8 +631,9 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
     const float sl2 = (float)(1.4426950408889634 / sqrt((double)D));  // 1/sqrt(d), log2(e)
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    for (int t = 0; t < ntile[q]; ++t) {
-      if (!warp_wait(&s_full[q], (uint32_t)t & 1u, abort_flag, wait_lim)) {
+    for (int i = 0; i < ntq[q]; ++i) {
+      const int t = t0 + i;
+      if (!warp_wait(&s_full[q], (uint32_t)i & 1u, abort_flag, wait_lim)) {
         ok = false;
         break;
       }
@@ -651,7 +670,7 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       }
       // Running maximum in the exp2 domain, raised lazily: only when a score passes it by more
       // than kRescaleSlack (p then stays below 2^kRescaleSlack), so O is rarely rescaled.  The
-      // first tile always raises it (slot 0 is attended by every row).
+      // split's first tile always raises it (its first slot is attended by every row).
       float alpha = 1.f;
       if (mx > m_run + kRescaleSlack) {
         alpha = ex2(m_run - mx);
@@ -674,8 +693,8 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       }
       l_run = l_run * alpha + ((rs0 + rs1) + (rs2 + rs3));
       // O_q and P_q are free once the previous product has completed
-      if (t > 0) {
-        if (!warp_wait(&pv_done[q], (uint32_t)(t - 1) & 1u, abort_flag, wait_lim)) {
+      if (i > 0) {
+        if (!warp_wait(&pv_done[q], (uint32_t)(i - 1) & 1u, abort_flag, wait_lim)) {
           ok = false;
           break;
         }
@@ -698,20 +717,33 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[q]);
     }
-    if (ok && ntile[q] > 0) {
-      if (!warp_wait(&pv_done[q], (uint32_t)(ntile[q] - 1) & 1u, abort_flag, wait_lim)) {
+    if (ok && ntq[q] > 0) {
+      if (!warp_wait(&pv_done[q], (uint32_t)(ntq[q] - 1) & 1u, abort_flag, wait_lim)) {
         ok = false;
       } else {
         tc_fence_after();
-        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-        OutT *orow = static_cast<OutT *>(v.out) +
-                     ((row0 + j) * Hq + g * G + m % G) * (int64_t)D;
+        const int64_t rh = (row0 + j) * Hq + g * G + m % G;  // (row, head) of the call
+        if (zs == 1) {  // the whole row: normalised output
+          const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+          OutT *orow = static_cast<OutT *>(v.out) + rh * (int64_t)D;
 #pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
-          uint32_t o[32];
-          tmem_ld32(t_o + c0, o);
-          tmem_wait_ld();
-          if (j < n) store_row32<OutT>(orow + c0, o, inv);
+          for (int c0 = 0; c0 < D; c0 += 32) {
+            uint32_t o[32];
+            tmem_ld32(t_o + c0, o);
+            tmem_wait_ld();
+            if (j < n) store_row32<OutT>(orow + c0, o, inv);
+          }
+        } else {  // this split's partial: O in units of 2^m_run, the running max and sum
+          const int64_t pr = (int64_t)z * v.rows * Hq + rh;
+          float *prow = v.part_o + pr * D;
+#pragma unroll
+          for (int c0 = 0; c0 < D; c0 += 32) {
+            uint32_t o[32];
+            tmem_ld32(t_o + c0, o);
+            tmem_wait_ld();
+            if (j < n) store_row32<float>(prow + c0, o, 1.f);
+          }
+          if (j < n) v.part_ml[pr] = make_float2(m_run, l_run);
         }
       }
     }
@@ -729,6 +761,52 @@ __global__ void __launch_bounds__(TcShape<D>::kThreads, 1)
   }
 }
 
+// ------------------------------------------------------------------------------------
+// 4. merge of the split partials (only when the attention grid has splits)
+// ------------------------------------------------------------------------------------
+// out = sum_z 2^(m_z - M) O_z / sum_z 2^(m_z - M) l_z over the splits z of the row's sequence, in
+// split order (M = max_z m_z; the split-softmax merge of the decode combine).  One warp per
+// (row, head), D / 32 elements a lane; rows of sequences that were not split (written by the
+// attention itself) or that the plan refused are left alone.
+constexpr int kMergeWarps = 8;
+template <typename OutT>
+__global__ void __launch_bounds__(kMergeWarps * 32) prefill_merge_kernel(const PrefillView v) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Hq = v.n_q_heads, D = v.head_dim;
+  const int64_t rh = (int64_t)blockIdx.x * kMergeWarps + warp;  // (row, head)
+  if (rh >= (int64_t)v.rows * Hq) return;
+  const int r = (int)(rh / Hq);
+  int lo = 0, hi = v.batch - 1;  // the row's sequence: the last b with offsets[b] <= r
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (v.offsets[mid] <= r) lo = mid; else hi = mid - 1;
+  }
+  const int4 si = v.seq_info[lo];
+  if (si.x < 0) return;
+  const int zs = prefill_splits(si.x, v.splits);
+  if (zs <= 1) return;
+  const int64_t zstride = (int64_t)v.rows * Hq;
+  float M = -INFINITY;
+  for (int z = 0; z < zs; ++z) M = fmaxf(M, v.part_ml[z * zstride + rh].x);
+  const int per = D / 32;  // 4 or 2
+  float num[4] = {0.f, 0.f, 0.f, 0.f}, den = 0.f;
+  for (int z = 0; z < zs; ++z) {
+    const float2 ml = v.part_ml[z * zstride + rh];
+    const float w = ml.x == -INFINITY ? 0.f : ex2(ml.x - M);
+    den += w * ml.y;
+    const float *po = v.part_o + (z * zstride + rh) * D + lane * per;
+    for (int e = 0; e < per; ++e) num[e] += w * po[e];
+  }
+  const float inv = den > 0.f ? 1.f / den : 0.f;
+  OutT *dst = static_cast<OutT *>(v.out) + rh * D + lane * per;
+  for (int e = 0; e < per; ++e) {
+    if constexpr (std::is_same<OutT, float>::value)
+      dst[e] = num[e] * inv;
+    else
+      dst[e] = __float2bfloat16_rn(num[e] * inv);
+  }
+}
+
 template <int D, typename OutT>
 cudaError_t launch_attn(const CUtensorMap &tq, const CUtensorMap &tk, const CUtensorMap &tv,
                         const PrefillView &v, cudaStream_t stream) {
@@ -737,8 +815,14 @@ cudaError_t launch_attn(const CUtensorMap &tq, const CUtensorMap &tk, const CUte
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, S::kSmem);
   if (e != cudaSuccess) return e;
   const int QB = prefill_query_rows(v.n_q_heads / v.n_kv_heads);
-  const dim3 grid((unsigned)v.n_kv_heads, (unsigned)(v.rows / QB + v.batch));
+  const int Z = v.splits < 1 ? 1 : v.splits;
+  const dim3 grid((unsigned)v.n_kv_heads, (unsigned)(v.rows / QB + v.batch), (unsigned)Z);
   prefill_attn_kernel<D, OutT><<<grid, S::kThreads, S::kSmem, stream>>>(tq, tk, tv, v);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || Z == 1) return e;
+  const int64_t pairs = (int64_t)v.rows * v.n_q_heads;
+  prefill_merge_kernel<OutT><<<(unsigned)((pairs + kMergeWarps - 1) / kMergeWarps),
+                               kMergeWarps * 32, 0, stream>>>(v);
   return cudaGetLastError();
 }
 

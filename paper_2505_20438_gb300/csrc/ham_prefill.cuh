@@ -29,7 +29,28 @@ struct PrefillView {
   int32_t batch, rows, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots;
   int32_t pos_mode;
   uint64_t wait_ns;            // limit of the attention's data waits (0: the default 2 s)
+  // Split over slots (a short chunk over a long cache): the attention grid's z dimension.  A
+  // sequence of L cached slots uses prefill_splits(L, splits) of them; a split that is not alone
+  // leaves its rows' unnormalised partials (output, running maximum and sum) here, and the merge
+  // kernel combines them: part_o [splits][rows][n_q_heads][head_dim], part_ml [same without d].
+  float *part_o;
+  float2 *part_ml;
+  int32_t splits;
 };
+// Slots a prefill split covers at least (whole 64-slot tiles of the cached part), and the most
+// splits a launch uses.
+constexpr int kPrefillSplitMinTiles = 8, kPrefillMaxSplits = 32;
+// Splits of a sequence holding L cached slots, at most Z: each takes at least
+// kPrefillSplitMinTiles tiles of the cached part, the last one also the chunk's own slots.
+__host__ __device__ inline int prefill_splits(int L, int Z) {
+  const int by_len = (L / 64) / kPrefillSplitMinTiles;
+  return by_len < 1 ? 1 : (by_len < Z ? by_len : Z);
+}
+// Scratch floats the split partials may use: SMs x 256 (row, head) pairs x head_dim (a launch
+// splits only while its CTAs, 256 pairs each, fit the SMs).
+inline size_t prefill_part_floats(int sms, int head_dim) {
+  return (size_t)sms * 256 * (size_t)head_dim;
+}
 cudaError_t launch_prefill(const CUtensorMap &tk, const CUtensorMap &tv, const PrefillView &v,
                            int out_dtype, cudaStream_t stream);
 bool prefill_supported(int head_dim, int group);

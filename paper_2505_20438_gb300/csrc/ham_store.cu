@@ -166,6 +166,7 @@ void note_launch(const ham_kv *kv, int32_t layer, void *stream, bool writes) {
 // handle keeps no pointer to.
 struct MetaLayout {
   size_t pos, ntok, pt, ns, nt, inv_freq, err, acc, ml, sr, stash, arrive, pf_seq, pf_pos;
+  size_t pf_part, pf_ml;  // ham_prefill's split partials (bf16 caches; empty for FP8)
   size_t front;   // ham_qkv_append: one arrival counter per grid row
   size_t total;
 };
@@ -196,6 +197,12 @@ MetaLayout meta_layout(const ham_config &cfg, int32_t max_ctas, int64_t max_page
   m.arrive = carve(sizeof(int32_t));
   m.pf_seq = carve((size_t)cfg.batch * sizeof(int4));
   m.pf_pos = carve((size_t)cfg.batch * cfg.max_slots_per_seq * sizeof(int32_t));
+  {  // (max_ctas is 8 x the SMs)
+    const bool fp8 = cfg.kv_dtype == HAM_KV_E4M3;
+    const size_t floats = fp8 ? 0 : ham::prefill_part_floats(max_ctas / 8, cfg.head_dim);
+    m.pf_part = carve(floats * sizeof(float));
+    m.pf_ml = carve(floats / (size_t)cfg.head_dim * sizeof(float2));
+  }
   m.front = carve((size_t)ham::kFrontMaxRows * sizeof(int32_t));
   m.total = off;
   return m;
@@ -556,6 +563,10 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->arrive = reinterpret_cast<int32_t *>(kv->meta + lay.arrive);
   kv->prefill_seq = reinterpret_cast<int4 *>(kv->meta + lay.pf_seq);
   kv->prefill_pos = reinterpret_cast<int32_t *>(kv->meta + lay.pf_pos);
+  if (!kv->fp8) {
+    kv->prefill_part = reinterpret_cast<float *>(kv->meta + lay.pf_part);
+    kv->prefill_part_ml = reinterpret_cast<float2 *>(kv->meta + lay.pf_ml);
+  }
 
   // Zeroed pool: slots past a sequence's length hold zeros, never uninitialised bits (FP8:
   // zero codes and exponents, the encoding of a zero row).
@@ -1051,6 +1062,21 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
   v.wait_ns = kv->wait_ns;
   v.seq_info = kv->prefill_seq;
   v.row_pos = kv->prefill_pos;
+  // Split over slots when the grid would leave SMs idle (a short chunk, whatever the cache
+  // holds: the kernel keeps one split for sequences with few cached slots).
+  {
+    const int64_t base = (int64_t)c.n_kv_heads * blocks;
+    int Z = 1;
+    if (kv->prefill_part && 2 * base <= kv->num_sms) {
+      Z = (int)std::min<int64_t>(ham::kPrefillMaxSplits, kv->num_sms / base);
+      while (Z > 1 && (size_t)Z * T * c.n_q_heads * d >
+                          ham::prefill_part_floats(kv->num_sms, c.head_dim))
+        --Z;
+    }
+    v.splits = Z;
+    v.part_o = kv->prefill_part;
+    v.part_ml = kv->prefill_part_ml;
+  }
   v.err = kv->err;
   v.pool_pages = c.pool_pages;
   v.batch = c.batch;

@@ -252,7 +252,12 @@ P1_PREFILL = PrefillWorkload("prefill_b4_s4096", dataclasses.replace(
 P2_CHUNK = PrefillWorkload("prefill_b4_c1024_s3072", dataclasses.replace(
     C1_LLAMA8B, name="prefill_b4_c1024_s3072", batch=4, slots=3072, seed=12), rows=1024,
     cached=3072)
-PREFILL_WORKLOADS = {p.name: p for p in (P1_PREFILL, P2_CHUNK)}
+# A 64-row chunk over 65,536 cached slots, batch 1: few query blocks over a long cache (the
+# attention splits over the cached slots).
+P3_SHORT = PrefillWorkload("prefill_b1_c64_s65536", dataclasses.replace(
+    C1_LLAMA8B, name="prefill_b1_c64_s65536", batch=1, slots=65536, seed=13), rows=64,
+    cached=65536)
+PREFILL_WORKLOADS = {p.name: p for p in (P1_PREFILL, P2_CHUNK, P3_SHORT)}
 
 
 def device_normal_bf16(shape, scale: float, seed: int, device="cuda"):

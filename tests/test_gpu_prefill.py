@@ -75,6 +75,28 @@ def test_prefill_matches_oracle(hq, hkv, d, page, cached, rows):
     assert_parity(_out(out), ref, what="prefill output")
 
 
+# Short chunks over long caches: the attention grid is split over the cached slots (each split at
+# least 8 tiles of 64 cached slots) and a merge kernel combines the splits' partials; sequences
+# with few cached slots in the same call stay whole.
+@pytest.mark.parametrize("hq,hkv,d,page,cached,rows,f32", [
+    (32, 8, 128, 16, (4096, 1500), (40, 9), False),      # 8 and 2 splits; Llama-8B heads
+    (32, 8, 128, 16, (4096, 1500), (40, 9), True),       # the same, fp32 output
+    (8, 2, 64, 16, (3000, 0, 700), (17, 5, 64), False),  # 5 splits, an empty cache, one split
+    (16, 2, 64, 16, (2600,), (20,), False),              # group 8, 5 splits
+    (8, 8, 128, 32, (5000,), (100,), False),             # group 1, 9 splits
+    (8, 4, 128, 64, (2048, 4000), (1, 70), True),        # group 2; a one-row chunk
+])
+def test_prefill_split_over_slots_matches_oracle(hq, hkv, d, page, cached, rows, f32):
+    w = _w(len(rows), hq, hkv, d, page, seed=sum(cached) % 97 + 5)
+    case = wl.make_prefill_case(w, rows, cached=np.array(cached, np.int32))
+    kv, q, out = _gpu(case, f32=f32)
+    oc, q_ref, rc, ref = _oracle(case)
+    assert rc == 0
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+    _check_state(kv, q, oc, q_ref)
+    assert_parity(_out(out), ref, what="split prefill output" + (" (f32)" if f32 else ""))
+
+
 @pytest.mark.parametrize("mode", ["token", "explicit"])
 def test_prefill_positions(mode):
     w = _w(2, 8, 2, 128, 16, seed=31)
@@ -175,7 +197,7 @@ def test_prefill_host_errors():
     assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
 
 
-@pytest.mark.parametrize("pw", [wl.P1_PREFILL, wl.P2_CHUNK], ids=lambda p: p.name)
+@pytest.mark.parametrize("pw", [wl.P1_PREFILL, wl.P2_CHUNK, wl.P3_SHORT], ids=lambda p: p.name)
 def test_prefill_full_size_sampled(pw):
     """The bench workloads at full size: every stored bit, and the output rows of a sample
     (first, last and spread rows of every sequence) against the oracle."""
@@ -186,8 +208,8 @@ def test_prefill_full_size_sampled(pw):
     want = np.zeros(int(case.offsets[-1]), bool)
     for b in range(B):
         a = int(case.offsets[b])
-        want[a + np.array([0, 1, 31, 32, 33, 63, 64, 127, pw.rows // 2, pw.rows - 2,
-                           pw.rows - 1])] = True
+        idx = np.array([0, 1, 31, 32, 33, 63, 64, 127, pw.rows // 2, pw.rows - 2, pw.rows - 1])
+        want[a + idx[idx < pw.rows]] = True
     oc, q_ref, rc, ref = _oracle(case, want=want)
     assert rc == 0
     assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
