@@ -1216,13 +1216,14 @@ def embed_cpu_baseline(c, seconds):
 FRONT_METRIC = "layer-front calls/s (q/k/v projection + RoPE + append) and achieved HBM GB/s"
 
 
-def front_bytes(w):
+def front_bytes(w, kv="bf16"):
     """Algorithmic bytes of one call: the fused weight once, x in, q_rot out, the new K and V
-    rows, and per sequence its counters, token count, page-table entry and slot metadata
-    (4 + 4 + 8 + 4 read, 4 + 4 + 4 + 8 written)."""
+    rows (FP8 pools: codes and one exponent byte a row), and per sequence its counters, token
+    count, page-table entry and slot metadata (4 + 4 + 8 + 4 read, 4 + 4 + 4 + 8 written)."""
     B, H, d = w.batch, w.hidden, w.head_dim
+    row = d + 1 if kv == "fp8" else d * 2
     return (w.out_rows * H * 2 + B * H * 2 + B * w.n_q_heads * d * 2 +
-            B * 2 * w.n_kv_heads * d * 2 + B * 40)
+            B * 2 * w.n_kv_heads * row + B * 40)
 
 
 def front_cpu_sample(w, seconds, max_calls=1000):
@@ -1295,8 +1296,10 @@ def run_front(args, w):
     B, H, L = w.batch, w.hidden, FRONT_LAYERS
     per_layer = GRAPH_STEPS // L
     start = 256                                   # slots per sequence before every graph
+    fp8 = args.kv == "fp8"
     kv = ham.ham_kv_alloc(L, B, w.n_q_heads, w.n_kv_heads, w.head_dim, 16,
-                          start + per_layer + 8, page_seed=1 + rank)
+                          start + per_layer + 8, page_seed=1 + rank,
+                          kv_dtype=ham.HAM_KV_E4M3 if fp8 else ham.HAM_KV_BF16)
     lengths = torch.full((B,), start, dtype=torch.int32, device="cuda")
     tokens = torch.full((B,), 2 * start, dtype=torch.int64, device="cuda")
     for layer in range(L):
@@ -1370,7 +1373,7 @@ def run_front(args, w):
     torch.cuda.synchronize()
     gemm_us = 1e3 * span[0].elapsed_time(span[1]) / GRAPH_STEPS
 
-    nbytes = front_bytes(w)
+    nbytes = front_bytes(w, args.kv)
     peak, peak_src = measured_peak_hbm()
     value = job_throughput(steps, world, elapsed_ms * 1e-3)
     achieved = nbytes / (call_us * 1e-6) / 1e9
@@ -1414,13 +1417,15 @@ def run_front(args, w):
                    "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
                    "weights": "fused [W_q; W_k; W_v] bf16 N(0, 1/H), x N(0, 1)",
                    "step": "one ham_qkv_append call: projection, RoPE of q and k, append",
+                   "kv_dtype": ("e4m3 codes + one int8 power-of-two exponent per row (encoded "
+                                "by the front)" if fp8 else "bf16"),
                    "l2": f"{L} layers' weights rotated ({L} x {w.out_rows * H * 2 / 2**20:.0f} "
                          f"MiB > 129 MB L2)",
                    "graph": f"{GRAPH_STEPS} calls per CUDA graph, then {L} counter rollbacks"},
         "sequences_per_s": round(value * B, 1),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4),
-                     "traffic": profiled_traffic("front", w.name, FRONT_SOURCES),
+                     "traffic": None if fp8 else profiled_traffic("front", w.name, FRONT_SOURCES),
                      "kernel": "front_kernel", "avg_launch_us": round(call_us, 3),
                      "algorithmic_bytes_per_launch": int(nbytes), "peak_source": peak_src,
                      "duration_method": f"CUDA events around the {GRAPH_STEPS} calls of the "

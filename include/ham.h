@@ -338,8 +338,9 @@ int ham_kv_export(ham_kv *kv, int32_t layer, void *k_dst, void *v_dst, int32_t *
  * FP8 caches work with ham_kv_fill (it encodes the bf16 rows it is given), ham_kv_export,
  * ham_kv_export_scales, ham_kv_append, ham_decode_attn, ham_decode_attn_ex, ham_decode_step
  * (its new slot is encoded as ham_kv_append encodes it, and attended as the cache then holds
- * it) and the counter calls; ham_prefill, ham_micro_step and ham_qkv_append return
- * HAM_EUNSUPPORTED for them. */
+ * it), ham_qkv_append (the projected rows, the key rotated, rounded to bf16 as for a bf16 cache
+ * and then encoded by the same rule) and the counter calls; ham_prefill and ham_micro_step
+ * return HAM_EUNSUPPORTED for them. */
 
 /* Copy one layer's exponent array out (layout above): pool_pages * n_kv_heads * page_slots *
  * 2 bytes.  HAM_EINVAL for a bf16 cache. */

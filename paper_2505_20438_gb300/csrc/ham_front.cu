@@ -208,8 +208,10 @@ __global__ void __launch_bounds__(kFrontThreads, NT == 1 ? 3 : 2) front_kernel(F
   }
   __syncthreads();
   // Every CTA of this row has read the counters once it gets here (the reads precede the
-  // barrier above); the last one to arrive commits them after its stores.
-  if (threadIdx.x == 0) {
+  // barrier above); the last one to arrive commits them after its stores.  (FP8 pools: the
+  // arrival comes after the stores instead, see below.)
+  const bool fp8 = v.kv_exp != nullptr;
+  if (threadIdx.x == 0 && !fp8) {
     __threadfence();
     s_last = atomicAdd(&v.arrive[blockIdx.y], 1) == (int)gridDim.x - 1;
   }
@@ -243,6 +245,16 @@ __global__ void __launch_bounds__(kFrontThreads, NT == 1 ? 3 : 2) front_kernel(F
           dst[i] = bf16_bits_f(a0);
           dst[i + half] = bf16_bits_f(a1);
         }
+      } else if (row >= 0 && fp8) {  // staged as bf16; the row's last CTA encodes it
+        const int g = rotated ? hh - Hq : hh - Hq - Hkv;
+        uint16_t *dst = v.stage + (((int64_t)b * Hkv + g) * 2 + (rotated ? 0 : 1)) * d;
+        if (rotated) {
+          const double2 cs = s_cs[bl][gid];
+          rotate_store(a0, a1, cs.x, cs.y, dst + i, dst + i + half);
+        } else {
+          dst[i] = bf16_bits_f(a0);
+          dst[i + half] = bf16_bits_f(a1);
+        }
       } else if (row >= 0) {
         const int g = rotated ? hh - Hq : hh - Hq - Hkv;
         const int64_t page = row / v.page_slots, r = row % v.page_slots;
@@ -258,6 +270,49 @@ __global__ void __launch_bounds__(kFrontThreads, NT == 1 ? 3 : 2) front_kernel(F
     }
   }
   __syncthreads();
+  if (fp8) {
+    // FP8 pools: the row's last CTA to finish its stores encodes every staged row of the row's
+    // sequences as ham_kv_append does (encode_e4m3_row: one warp a row of 128 elements, 4 a
+    // lane; codes, V transposed within its page, exponents), then commits the counters.
+    if (threadIdx.x == 0) {
+      __threadfence();
+      s_last = atomicAdd(&v.arrive[blockIdx.y], 1) == (int)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (s_last) {
+      __threadfence();
+      const int Hkv = v.n_kv_heads, P = v.page_slots;
+      const int nb = min(kFrontBatchTile, v.batch - b_base);
+      uint8_t *kc = reinterpret_cast<uint8_t *>(v.k_pool);
+      uint8_t *vc = reinterpret_cast<uint8_t *>(v.v_pool);
+      for (int r = warp; r < nb * Hkv * 2; r += kFrontWarps + 1) {
+        const int bl = r / (Hkv * 2), g = (r >> 1) % Hkv;
+        const bool is_v = (r & 1) != 0;
+        const int64_t row = s_row[bl];
+        if (row < 0) continue;  // (uniform over the warp)
+        const uint16_t *src = v.stage + (((int64_t)(b_base + bl) * Hkv + g) * 2 + (is_v ? 1 : 0)) *
+                                            kFp8HeadDim + 4 * lane;
+        float x[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) x[e] = __uint_as_float((uint32_t)__ldcg(src + e) << 16);
+        uint32_t codes;
+        const int ex = encode_e4m3_row(x, codes);
+        const int64_t page = row / P, s = row % P;
+        const int64_t ph = page * Hkv + g;  // (page, head) block
+        if (!is_v) {
+          *reinterpret_cast<uint32_t *>(kc + (ph * P + s) * kFp8HeadDim + 4 * lane) = codes;
+        } else {
+          const int64_t sv = s - s % kChunkSlots + fp8_v_slot_byte((int)(s % kChunkSlots));
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            vc[(ph * kFp8HeadDim + 4 * lane + e) * P + sv] = (uint8_t)(codes >> (8 * e));
+        }
+        if (lane == 0)
+          v.kv_exp[(ph * (P / kChunkSlots) + s / kChunkSlots) * 32 + (is_v ? kChunkSlots : 0) +
+                   s % kChunkSlots] = (int8_t)ex;
+      }
+    }
+  }
   if (s_last && threadIdx.x < kFrontBatchTile) {
     __threadfence();
     const int b = b_base + threadIdx.x;

@@ -29,6 +29,11 @@ struct FrontView {
   const int32_t *ntok;         // [batch]
   int32_t *arrive;             // scratch [ceil(batch / 32)]: CTAs of a row done with the
                                // counters (0 between launches; the last to arrive resets it)
+  // FP8 (e4m3) pools (head_dim 128): the layer's exponents, and scratch for the new slot's key
+  // (rotated) and value rows as bf16, [batch][n_kv_heads][2][head_dim], which the row's last CTA
+  // encodes (else both null)
+  int8_t *kv_exp;
+  uint16_t *stage;
   int32_t *err;
   int64_t pool_pages;
   int32_t batch, hidden, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots;

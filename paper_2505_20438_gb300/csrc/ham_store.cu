@@ -167,6 +167,7 @@ void note_launch(const ham_kv *kv, int32_t layer, void *stream, bool writes) {
 struct MetaLayout {
   size_t pos, ntok, pt, ns, nt, inv_freq, err, acc, ml, sr, stash, arrive, pf_seq, pf_pos;
   size_t pf_part, pf_ml;  // ham_prefill's split partials (bf16 caches; empty for FP8)
+  size_t front_stage;     // ham_qkv_append on FP8 caches: the new rows as bf16 (else empty)
   size_t front;   // ham_qkv_append: one arrival counter per grid row
   size_t total;
 };
@@ -204,6 +205,9 @@ MetaLayout meta_layout(const ham_config &cfg, int32_t max_ctas, int64_t max_page
     m.pf_ml = carve(floats / (size_t)cfg.head_dim * sizeof(float2));
   }
   m.front = carve((size_t)ham::kFrontMaxRows * sizeof(int32_t));
+  m.front_stage = carve(cfg.kv_dtype == HAM_KV_E4M3
+                            ? (size_t)cfg.batch * cfg.n_kv_heads * 2 * cfg.head_dim * sizeof(uint16_t)
+                            : 0);
   m.total = off;
   return m;
 }
@@ -801,7 +805,6 @@ int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, 
   ham::ApiRange nvtx_range("ham_qkv_append");
   int rc = check_layer(kv, layer);
   if (rc) return rc;
-  if ((rc = fp8_unsupported(kv, "ham_qkv_append")) != 0) return rc;
   if (!x || !w_qkv || !ntok || !q_rot) return fail(HAM_EINVAL, "x, w_qkv, ntok and q_rot are required");
   if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(q_rot))
     return fail(HAM_EINVAL, "x, w_qkv and q_rot must be 16-byte aligned");
@@ -817,7 +820,7 @@ int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, 
   const size_t x_bytes = B * (size_t)hidden * 2;
   const size_t w_bytes = (size_t)(c.n_q_heads + 2 * c.n_kv_heads) * d * (size_t)hidden * 2;
   const size_t q_bytes = B * (size_t)c.n_q_heads * d * 2;
-  const size_t pool_bytes = (size_t)c.layers * 2 * (size_t)kv->pool_elems * 2;
+  const size_t pool_bytes = (size_t)c.layers * layer_pool_bytes(kv);
   if (overlaps(q_rot, q_bytes, x, x_bytes) || overlaps(q_rot, q_bytes, w_qkv, w_bytes) ||
       overlaps(q_rot, q_bytes, kv->pool, pool_bytes) || overlaps(x, x_bytes, kv->pool, pool_bytes) ||
       overlaps(w_qkv, w_bytes, kv->pool, pool_bytes))
@@ -841,6 +844,8 @@ int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, 
   v.pos = pos;
   v.ntok = ntok;
   v.arrive = reinterpret_cast<int32_t *>(kv->meta + lay.front);
+  v.kv_exp = layer_exp(kv, layer);  // FP8 pools: encoded by the front's last CTAs
+  v.stage = kv->fp8 ? reinterpret_cast<uint16_t *>(kv->meta + lay.front_stage) : nullptr;
   v.err = kv->err;
   v.pool_pages = c.pool_pages;
   v.batch = c.batch;

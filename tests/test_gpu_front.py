@@ -201,3 +201,59 @@ def test_front_rejects_bad_arguments():
         ham.ham_qkv_append(kv, 1, x, W, ntok, q_rot)                     # layer out of range
     slots, _ = ham.ham_slot_lengths(kv)
     assert list(slots) == [3, 4]                                          # nothing ran
+
+
+@pytest.mark.parametrize("hq,hkv,H,counts", [
+    (32, 8, 4096, (5, 16, 100, 31, 0, 7, 64, 200)),   # Llama-3-8B shapes, batch 8
+    (8, 8, 512, tuple((7 * i) % 50 for i in range(37))),  # 2 grid rows (two last CTAs)
+])
+def test_front_over_fp8_pools(hq, hkv, H, counts):
+    """FP8 (e4m3) pools: the row's last CTA encodes the new slot's rows.  Slot metadata and
+    counters exactly as the oracle's; attention over the cache against the oracle's attention
+    over its own front rows decoded through the FP8 format (the decode bar).  And, between two
+    CUDA paths, the same call on a bf16 cache: the same q_rot bits, and its stored rows, encoded
+    by the oracle's FP8 encoder, the FP8 cache's codes and exponents bit for bit."""
+    import torch
+    from oracle import fp8 as ofp8
+    from test_gpu_fp8 import fp8_cache, _decoded_cache, _export as fp8_export
+    d, B = 128, len(counts)
+    case = small_case(batch=B, hq=hq, hkv=hkv, d=d, page=16, counts=counts, seed=hq + 7,
+                      extra_slots=4)
+    oc = oracle.OracleCache.from_case(case)
+    kv8 = fp8_cache(case)
+    kvb = gpu_cache(case)
+    fw = wl.front_workload(B, hidden=H, n_q_heads=hq, n_kv_heads=hkv, head_dim=d, seed=hq + 7)
+    rng = wl.rng_for(hq + 7, 78)
+    for step in range(2):
+        x, W = wl.front_inputs(fw, stream=step)
+        ntok = wl.ntok_capped_geometric(rng, (B,))
+        st, q_ref, _ = ofront.qkv_append(oc, x, W, ntok)
+        assert st == 0
+        q8 = torch.full((B, hq, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+        qb = torch.full_like(q8, float("nan"))
+        ham.ham_qkv_append(kv8, 0, dev_bf16(x), dev_bf16(W), dev_i32(ntok), q8)
+        ham.ham_qkv_append(kvb, 0, dev_bf16(x), dev_bf16(W), dev_i32(ntok), qb)
+        torch.cuda.synchronize()
+        assert np.array_equal(host_bits(q8), host_bits(qb)), "q_rot, FP8 against bf16 pools"
+    assert ham.ham_kv_status(kv8) == ham.HAM_DEVERR_NONE
+    slots, tokens = ham.ham_slot_lengths(kv8)
+    assert np.array_equal(slots, oc.num_slots) and np.array_equal(tokens, oc.num_tokens)
+    k8, v8, e8, pos8, ntok8 = fp8_export(kv8)
+    assert np.array_equal(pos8, oc.slot_pos) and np.array_equal(ntok8, oc.slot_ntok)
+    # parity: attention over the FP8 cache against the oracle over its front rows, decoded
+    got = gpu_decode(kv8, host_bits(q8))
+    ref = _decoded_cache(case, oc).decode_attn(q_ref)
+    assert_parity(got, ref, what="attention over FP8 pools after the front")
+    # consistency with the bf16 pools' front (the oracle's encoder on its stored rows)
+    kb, vb, _, _ = _export(kvb)
+    kc, ke = ofp8.encode_rows(ofront.bf16_bits_to_f64(kb))
+    vc, ve = ofp8.encode_rows(ofront.bf16_bits_to_f64(vb))
+    pages, hk, P, _ = kc.shape
+    assert np.array_equal(k8, kc), "K codes"
+    perm = np.array([4 * ((s % 8) // 2) + 2 * (s // 8) + s % 2 for s in range(16)])
+    vt = vc.transpose(0, 1, 3, 2).reshape(pages, hk, d, P // 16, 16)
+    vp = np.empty_like(vt)
+    vp[..., perm] = vt
+    assert np.array_equal(v8, vp.reshape(pages, hk, d, P)), "V codes"
+    e = np.stack([ke.reshape(pages, hk, P // 16, 16), ve.reshape(pages, hk, P // 16, 16)], axis=3)
+    assert np.array_equal(e8, e.astype(np.int8)), "exponents"
