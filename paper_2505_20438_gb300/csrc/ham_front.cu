@@ -208,10 +208,9 @@ __global__ void __launch_bounds__(kFrontThreads, NT == 1 ? 3 : 2) front_kernel(F
   }
   __syncthreads();
   // Every CTA of this row has read the counters once it gets here (the reads precede the
-  // barrier above); the last one to arrive commits them after its stores.  (FP8 pools: the
-  // arrival comes after the stores instead, see below.)
+  // barrier above); the last one to arrive commits them after its stores.
   const bool fp8 = v.kv_exp != nullptr;
-  if (threadIdx.x == 0 && !fp8) {
+  if (threadIdx.x == 0) {
     __threadfence();
     s_last = atomicAdd(&v.arrive[blockIdx.y], 1) == (int)gridDim.x - 1;
   }
@@ -269,25 +268,29 @@ __global__ void __launch_bounds__(kFrontThreads, NT == 1 ? 3 : 2) front_kernel(F
       }
     }
   }
+  if (fp8) __threadfence();  // each thread's staged elements: visible to the encoding CTA
   __syncthreads();
-  if (fp8) {
-    // FP8 pools: the row's last CTA to finish its stores encodes every staged row of the row's
-    // sequences as ham_kv_append does (encode_e4m3_row: one warp a row of 128 elements, 4 a
-    // lane; codes, V transposed within its page, exponents), then commits the counters.
+  if (fp8 && hh >= v.n_q_heads) {
+    // FP8 pools: the 8 CTAs of one key (or value) head each staged 16 elements of its rows; the
+    // last of them to finish encodes the head's rows of this CTA row as ham_kv_append does
+    // (encode_e4m3_row: one warp a row of 128 elements, 4 a lane; codes, V transposed within
+    // its page, exponents).  Sixteen heads encode in parallel, a round trip each.
+    __shared__ int32_t s_enc;
+    const int Hkv = v.n_kv_heads, kv_head = hh - v.n_q_heads;  // keys 0 .. Hkv-1, then values
+    int32_t *cnt = v.enc_arrive + (int64_t)blockIdx.y * 2 * Hkv + kv_head;
     if (threadIdx.x == 0) {
       __threadfence();
-      s_last = atomicAdd(&v.arrive[blockIdx.y], 1) == (int)gridDim.x - 1;
+      s_enc = atomicAdd(cnt, 1) == tiles_per_head - 1;
     }
     __syncthreads();
-    if (s_last) {
+    if (s_enc) {
       __threadfence();
-      const int Hkv = v.n_kv_heads, P = v.page_slots;
+      const bool is_v = !rotated;
+      const int g = is_v ? kv_head - Hkv : kv_head, P = v.page_slots;
       const int nb = min(kFrontBatchTile, v.batch - b_base);
       uint8_t *kc = reinterpret_cast<uint8_t *>(v.k_pool);
       uint8_t *vc = reinterpret_cast<uint8_t *>(v.v_pool);
-      for (int r = warp; r < nb * Hkv * 2; r += kFrontWarps + 1) {
-        const int bl = r / (Hkv * 2), g = (r >> 1) % Hkv;
-        const bool is_v = (r & 1) != 0;
+      for (int bl = warp; bl < nb; bl += kFrontWarps + 1) {
         const int64_t row = s_row[bl];
         if (row < 0) continue;  // (uniform over the warp)
         const uint16_t *src = v.stage + (((int64_t)(b_base + bl) * Hkv + g) * 2 + (is_v ? 1 : 0)) *
@@ -297,20 +300,21 @@ __global__ void __launch_bounds__(kFrontThreads, NT == 1 ? 3 : 2) front_kernel(F
         for (int e = 0; e < 4; ++e) x[e] = __uint_as_float((uint32_t)__ldcg(src + e) << 16);
         uint32_t codes;
         const int ex = encode_e4m3_row(x, codes);
-        const int64_t page = row / P, s = row % P;
+        const int64_t page = row / P, sl = row % P;
         const int64_t ph = page * Hkv + g;  // (page, head) block
         if (!is_v) {
-          *reinterpret_cast<uint32_t *>(kc + (ph * P + s) * kFp8HeadDim + 4 * lane) = codes;
+          *reinterpret_cast<uint32_t *>(kc + (ph * P + sl) * kFp8HeadDim + 4 * lane) = codes;
         } else {
-          const int64_t sv = s - s % kChunkSlots + fp8_v_slot_byte((int)(s % kChunkSlots));
+          const int64_t sv = sl - sl % kChunkSlots + fp8_v_slot_byte((int)(sl % kChunkSlots));
 #pragma unroll
           for (int e = 0; e < 4; ++e)
             vc[(ph * kFp8HeadDim + 4 * lane + e) * P + sv] = (uint8_t)(codes >> (8 * e));
         }
         if (lane == 0)
-          v.kv_exp[(ph * (P / kChunkSlots) + s / kChunkSlots) * 32 + (is_v ? kChunkSlots : 0) +
-                   s % kChunkSlots] = (int8_t)ex;
+          v.kv_exp[(ph * (P / kChunkSlots) + sl / kChunkSlots) * 32 + (is_v ? kChunkSlots : 0) +
+                   sl % kChunkSlots] = (int8_t)ex;
       }
+      if (threadIdx.x == 0) *cnt = 0;  // for the next call
     }
   }
   if (s_last && threadIdx.x < kFrontBatchTile) {

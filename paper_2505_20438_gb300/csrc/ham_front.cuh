@@ -34,6 +34,8 @@ struct FrontView {
   // encodes (else both null)
   int8_t *kv_exp;
   uint16_t *stage;
+  int32_t *enc_arrive;         // FP8 pools: [ceil(batch / 32)][2 n_kv_heads] arrivals of a head's
+                               // CTAs (0 between launches; the last to arrive resets it)
   int32_t *err;
   int64_t pool_pages;
   int32_t batch, hidden, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots;

@@ -168,6 +168,7 @@ struct MetaLayout {
   size_t pos, ntok, pt, ns, nt, inv_freq, err, acc, ml, sr, stash, arrive, pf_seq, pf_pos;
   size_t pf_part, pf_ml;  // ham_prefill's split partials (bf16 caches; empty for FP8)
   size_t front_stage;     // ham_qkv_append on FP8 caches: the new rows as bf16 (else empty)
+  size_t front_enc;       // ... and the per-head arrival counters of its encoding
   size_t front;   // ham_qkv_append: one arrival counter per grid row
   size_t total;
 };
@@ -208,6 +209,9 @@ MetaLayout meta_layout(const ham_config &cfg, int32_t max_ctas, int64_t max_page
   m.front_stage = carve(cfg.kv_dtype == HAM_KV_E4M3
                             ? (size_t)cfg.batch * cfg.n_kv_heads * 2 * cfg.head_dim * sizeof(uint16_t)
                             : 0);
+  m.front_enc = carve(cfg.kv_dtype == HAM_KV_E4M3
+                          ? (size_t)ham::kFrontMaxRows * 2 * cfg.n_kv_heads * sizeof(int32_t)
+                          : 0);
   m.total = off;
   return m;
 }
@@ -846,6 +850,7 @@ int ham_qkv_append(ham_kv *kv, int32_t layer, const void *x, const void *w_qkv, 
   v.arrive = reinterpret_cast<int32_t *>(kv->meta + lay.front);
   v.kv_exp = layer_exp(kv, layer);  // FP8 pools: encoded by the front's last CTAs
   v.stage = kv->fp8 ? reinterpret_cast<uint16_t *>(kv->meta + lay.front_stage) : nullptr;
+  v.enc_arrive = kv->fp8 ? reinterpret_cast<int32_t *>(kv->meta + lay.front_enc) : nullptr;
   v.err = kv->err;
   v.pool_pages = c.pool_pages;
   v.batch = c.batch;
