@@ -316,7 +316,7 @@ struct ham_kv {
   float2 *part_ml = nullptr;
   int2 *seg_range = nullptr;
   int4 *prefill_seq = nullptr;     // ham_prefill: per-sequence plan [batch]
-  int32_t *prefill_pos = nullptr;  // ham_prefill: per-row positions [batch * max_slots]
+  int2 *prefill_rows = nullptr;    // ham_prefill: per-row (position, pool row) [batch * max_slots]
   float *prefill_part = nullptr;   // ham_prefill: split partials (bf16 caches)
   float2 *prefill_part_ml = nullptr;
   int64_t scratch_bytes = 0;

@@ -11,7 +11,8 @@
 // Three launches (four when the attention splits over the cached slots):
 //  1. prefill_plan_kernel, one block per sequence: checks that the sequence's rows fit
 //     (counts, capacity, pages), gives each row its position (slot index, running token count
-//     or the caller's), numbers the query blocks, and advances the counters.
+//     or the caller's) and pool row (or -1: not stored), numbers the query blocks, and advances
+//     the counters.
 //  2. prefill_rope_kernel, one block per row: turns q and k at the row's position and stores
 //     k and v into the row's slot.  The rotation x0 c - x1 s is evaluated from the fp64 cos/sin
 //     table in pairs of fp32 values (error-free products and sums, about 48 bits) and rounded
@@ -56,6 +57,7 @@ namespace ham {
 namespace {
 
 constexpr int kPlanThreads = 256;
+constexpr int kPlanRun = 8;  // consecutive rows a plan thread takes per tile
 constexpr float kRescaleSlack = 8.0f;  // log2 units: the running max lags by at most 2^8
 constexpr int kRopeThreads = 256;
 
@@ -133,32 +135,48 @@ __global__ void __launch_bounds__(kPlanThreads) prefill_plan_kernel(PrefillView 
   bad_page = __syncthreads_or(bad_page);
   if (!err && bad_tok) err = HAM_DEVERR_NTOK;
   if (!err && bad_page) err = HAM_DEVERR_PAGE;
-  if (err) {
+  if (err) {  // none of the rows is stored
+    for (int j = tid; j < n; j += kPlanThreads) v.row_info[a + j] = make_int2(0, -1);
     if (tid == 0) {
       record_error(v.err, err);
-      v.seq_info[b] = make_int4(-1, n, qb, 0);
+      v.seq_info[b] = make_int4(-1, n, qb, 1);
     }
     return;
   }
-  // positions: the caller's, the slot index, or the tokens before the row
+  // positions (the caller's, the slot index, or the tokens before the row) and pool rows.  A
+  // thread takes kPlanRun consecutive rows of each tile of kPlanThreads * kPlanRun rows: their
+  // token counts, positions and page-table entries are loaded together, and one block scan of
+  // the threads' sums a tile gives every row its tokens before it.
   const int64_t t0 = v.num_tokens[b];
   int64_t carry = 0;
-  for (int j0 = 0; j0 < n; j0 += kPlanThreads) {
-    const int j = j0 + tid;
-    const int t = j < n ? (v.ntok ? v.ntok[a + j] : 1) : 0;
+  for (int j0 = 0; j0 < n; j0 += kPlanThreads * kPlanRun) {
+    const int jb = j0 + tid * kPlanRun;
+    int t[kPlanRun], run = 0;
+#pragma unroll
+    for (int k = 0; k < kPlanRun; ++k) {
+      t[k] = jb + k < n ? (v.ntok ? v.ntok[a + jb + k] : 1) : 0;
+      run += t[k];
+    }
     int total = 0;
-    const int excl = block_scan(t, red, &total) - t;
-    if (j < n) {
-      int64_t p;
-      if (v.pos) p = v.pos[a + j];
-      else if (v.pos_mode == HAM_POS_SLOT) p = (int64_t)L + j;
-      else p = t0 + carry + excl;
-      v.row_pos[a + j] = (int32_t)p;
+    int64_t before = t0 + carry + (block_scan(run, red, &total) - run);
+#pragma unroll
+    for (int k = 0; k < kPlanRun; ++k) {
+      const int j = jb + k;
+      if (j < n) {
+        int64_t p;
+        if (v.pos) p = v.pos[a + j];
+        else if (v.pos_mode == HAM_POS_SLOT) p = (int64_t)L + j;
+        else p = before;
+        const int slot = L + j, pg = slot / v.page_slots;
+        const int page = v.page_table[(int64_t)b * v.max_pages + pg];
+        v.row_info[a + j] = make_int2((int32_t)p, page * v.page_slots + (slot - pg * v.page_slots));
+      }
+      before += t[k];
     }
     carry += total;
   }
   if (tid == 0) {
-    v.seq_info[b] = make_int4(L, n, qb, 0);
+    v.seq_info[b] = make_int4(L, n, qb, 1);
     v.num_slots[b] = L + n;
     v.num_tokens[b] = t0 + carry;
   }
@@ -179,21 +197,25 @@ __device__ __forceinline__ uint16_t bf16_of_pair(float hi, float lo) {
   return __bfloat16_as_ushort(__float2bfloat16_rn(hi));
 }
 
-// a c - b s rounded once to bf16, with c = ch + cl and s = sh + sl given as fp32 pairs and a, b
-// exact (bf16 values).  Near a rounding boundary: products by FMA error terms and sums by
-// two-sum are exact, only the small terms are rounded, so the pair carries about 48 bits of
-// the exact value.
-__device__ __forceinline__ uint16_t rotate_dd(float a, float b, float ch, float cl, float sh,
-                                              float sl) {
-  // Fast path: y = a ch - b sh in plain fp32 lies within 3 * 2^-24 (|a| + |b|) < e / 2 of the
-  // exact a c - b s.  When no bf16 rounding boundary is within e of y (the nearest one is the
-  // midpoint sharing y's upper 16 bits; the others are a quarter of a bf16 spacing away, more
-  // than e once e < 2^-11 |y|), the exact value rounds as y does.
+// Fast evaluation of a c - b s, with c = ch + cl and s = sh + sl given as fp32 pairs and a, b
+// exact (bf16 values): y = a ch - b sh in plain fp32 lies within 3 * 2^-24 (|a| + |b|) < e / 2
+// of the exact value, e = (|a| + |b|) 2^-21.  When no bf16 rounding boundary is within e of y
+// (the nearest one is the midpoint sharing y's upper 16 bits; the others are a quarter of a
+// bf16 spacing away, more than e once e < 2^-11 |y|), the exact value rounds as y does and
+// *sure is set; otherwise rotate_exact gives the rounding.
+__device__ __forceinline__ float rotate_fast(float a, float b, float ch, float sh, float e,
+                                             bool *sure) {
   const float y = __fmaf_rn(a, ch, -__fmul_rn(b, sh));
-  const float e = __fmul_rn(__fadd_rn(fabsf(a), fabsf(b)), 0x1p-21f);
   const float mid = __uint_as_float((__float_as_uint(y) & 0xFFFF0000u) | 0x8000u);
-  if (fabsf(__fsub_rn(y, mid)) > e && e < __fmul_rn(fabsf(y), 0x1p-11f))
-    return __bfloat16_as_ushort(__float2bfloat16_rn(y));
+  *sure = fabsf(__fsub_rn(y, mid)) > e && e < __fmul_rn(fabsf(y), 0x1p-11f);
+  return y;
+}
+
+// a c - b s rounded once to bf16 near a rounding boundary: products by FMA error terms and sums
+// by two-sum are exact, only the small terms are rounded, so the pair carries about 48 bits of
+// the exact value.
+__device__ __noinline__ uint16_t rotate_exact(float a, float b, float ch, float cl, float sh,
+                                              float sl) {
   const float p1 = __fmul_rn(a, ch), e1 = __fmaf_rn(a, ch, -p1);
   const float p2 = __fmul_rn(b, sh), e2 = __fmaf_rn(b, sh, -p2);
   const float s = __fsub_rn(p1, p2);  // two-sum of p1 and -p2: s + t = p1 - p2
@@ -217,84 +239,133 @@ __device__ __forceinline__ void split_double(double x, float &hi, float &lo) {
   lo = __double2float_rn(x - (double)hi);  // x - hi is exact in fp64
 }
 
-// One block per row; a thread owns four consecutive pairs (i, i + d/2), i = 4 (tid % (d/8)) ..,
-// of one head at a time (8-byte loads and stores of each half).
-template <typename OutT>
+// Shared-memory index of frequency i of the (cos, sin) row: the eight frequencies a thread
+// reads, 8 (i / 8) .. + 7, rotated by i / 8 within their group of eight, so that the eight
+// threads of a head (distinct i / 8, same step) read eight distinct 16-byte bank groups.
+__device__ __forceinline__ int cs_index(int i) { return (i & ~7) | ((i + (i >> 3)) & 7); }
+
+// One block per row.  Thread t owns the eight pairs (i, i + d/2), i = 8 (t % (d/16)) .. + 7, of
+// heads t / (d/16), t / (d/16) + 256 / (d/16), ... (query heads, then key heads): a 16-byte load
+// and store of each half.  The plan left the row's position and pool row in row_info, so every
+// load the block makes needs only the row index, and is issued at once: the first two heads'
+// halves, a 16-byte piece of the value row, and then the (cos, sin) row of the position, which
+// goes to shared memory, read by the threads of every head.
+template <int D, typename OutT>
 __global__ void __launch_bounds__(kRopeThreads) prefill_rope_kernel(PrefillView v) {
+  constexpr int kHalf = D / 2, kOcts = kHalf / 8, kHeadsPass = kRopeThreads / kOcts;
+  constexpr int kVPieces = D / 8;  // 16-byte pieces of one head's value row
+  static_assert(kHalf <= kRopeThreads, "one thread a frequency");
+  __shared__ float4 cs_s[kHalf];   // (c_hi, c_lo, s_hi, s_lo) of frequency i at cs_index(i)
   const int64_t r = blockIdx.x;
-  const int D = v.head_dim, half = D / 2, Hq = v.n_q_heads, Hkv = v.n_kv_heads;
-  int lo = 0, hi = v.batch - 1;  // the sequence of row r
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (v.offsets[mid] <= r) lo = mid; else hi = mid - 1;
-  }
-  const int b = lo;
-  const int4 si = v.seq_info[b];
-  const int a = v.offsets[b];
-  if (si.x < 0 || r < a || r >= (int64_t)a + si.y) {  // not stored: its output rows are 0
+  const int tid = threadIdx.x, j = tid % kOcts, h0 = tid / kOcts, h1 = h0 + kHeadsPass;
+  const int Hq = v.n_q_heads, Hkv = v.n_kv_heads, H = Hq + Hkv, nv = Hkv * kVPieces;
+  uint16_t *const qrow = v.q + r * Hq * D;
+  const uint16_t *const krow = v.k_new + r * Hkv * D;
+  const uint4 *const vrow = reinterpret_cast<const uint4 *>(v.v_new + r * Hkv * D);
+  auto half_of = [&](int h, int upper) {  // 16-byte piece j of head h's lower or upper half
+    const uint16_t *src = h < Hq ? qrow + h * D : krow + (h - Hq) * D;
+    return *reinterpret_cast<const uint4 *>(src + upper * kHalf + 8 * j);
+  };
+  // 1. the loads (the row's pool row is -1 when it is not stored; the call's offsets are valid
+  //    when sequence 0's plan entry says so)
+  const int2 ri = v.row_info[r];
+  const int offsets_ok = v.seq_info[0].w;
+  uint4 x0l{}, x0h{}, x1l{}, x1h{}, vv{};
+  if (h0 < H) { x0l = half_of(h0, 0); x0h = half_of(h0, 1); }
+  if (h1 < H) { x1l = half_of(h1, 0); x1h = half_of(h1, 1); }
+  if (tid < nv) vv = vrow[tid];
+  const int p = ri.x;
+  const bool in_table = p >= 0 && p < v.rope_positions;
+  float4 c4{};
+  if (tid < kHalf && in_table) c4 = v.rope_table_ff[(int64_t)p * kHalf + tid];
+  if (!offsets_ok || ri.y < 0) {  // not stored: its output rows are 0
     OutT *o = static_cast<OutT *>(v.out) + r * Hq * D;
-    for (int e = threadIdx.x; e < Hq * D; e += kRopeThreads) o[e] = OutT(0.f);
+    for (int e = tid; e < Hq * D; e += kRopeThreads) o[e] = OutT(0.f);
     return;
   }
-  const int slot = si.x + (int)(r - a);
-  const int p = v.row_pos[r];
-  const int64_t page = v.page_table[(int64_t)b * v.max_pages + slot / v.page_slots];
-  const int prow = slot % v.page_slots;
-  if (threadIdx.x == 0) {
-    v.slot_pos[page * v.page_slots + prow] = p;
-    v.slot_ntok[page * v.page_slots + prow] = v.ntok ? v.ntok[r] : 1;
-  }
-  for (int e = threadIdx.x; e < Hkv * D / 8; e += kRopeThreads) {  // values: bit copy
-    const int gg = e / (D / 8), k = e % (D / 8);
-    reinterpret_cast<uint4 *>(v.v_pool + ((page * Hkv + gg) * v.page_slots + prow) * D)[k] =
-        reinterpret_cast<const uint4 *>(v.v_new + (r * Hkv + gg) * D)[k];
-  }
-  const int quads = half / 4, i0 = 4 * (threadIdx.x % quads);
-  float4 cs[4];  // (c_hi, c_lo, s_hi, s_lo) of frequencies i0 .. i0 + 3
-  if (p >= 0 && p < v.rope_positions) {
-#pragma unroll
-    for (int e = 0; e < 4; ++e) cs[e] = v.rope_table_ff[(int64_t)p * half + i0 + e];
-  } else {
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
+  // 2. the (cos, sin) row in shared memory (past the table: from fp64 sincos) and the slot's
+  //    page and row in it
+  __shared__ int2 where;  // (page, row in page)
+  if (tid < kHalf) {
+    if (!in_table) {
       double c, sn;
-      sincos((double)p * v.inv_freq[i0 + e], &sn, &c);
-      split_double(c, cs[e].x, cs[e].y);
-      split_double(sn, cs[e].z, cs[e].w);
+      sincos((double)p * v.inv_freq[tid], &sn, &c);
+      split_double(c, c4.x, c4.y);
+      split_double(sn, c4.z, c4.w);
     }
+    cs_s[cs_index(tid)] = c4;
   }
-  // query heads in place, then the key heads into the slot
-  for (int hh = threadIdx.x / quads; hh < Hq + Hkv; hh += kRopeThreads / quads) {
-    const uint16_t *src;
-    uint16_t *dst;
-    if (hh < Hq) {
-      src = dst = v.q + (r * Hq + hh) * D;
-    } else {
-      const int gg = hh - Hq;
-      src = v.k_new + (r * Hkv + gg) * D;
-      dst = v.k_pool + ((page * Hkv + gg) * v.page_slots + prow) * D;
-    }
-    const uint2 xl = *reinterpret_cast<const uint2 *>(src + i0);
-    const uint2 xh = *reinterpret_cast<const uint2 *>(src + i0 + half);
-    const uint32_t wl[2] = {xl.x, xl.y}, wh[2] = {xh.x, xh.y};
-    uint32_t yl[2], yh[2];
+  if (tid == 0) {
+    where = make_int2(ri.y / v.page_slots, ri.y % v.page_slots);
+    v.slot_pos[ri.y] = p;
+    v.slot_ntok[ri.y] = v.ntok ? v.ntok[r] : 1;
+  }
+  __syncthreads();
+  const int64_t page = where.x;
+  const int prow = where.y;
+  auto pool_row = [&](uint16_t *pool, int g) {
+    return pool + ((page * Hkv + g) * v.page_slots + prow) * D;
+  };
+  // 3. the value row (a bit copy)
+  if (tid < nv) reinterpret_cast<uint4 *>(pool_row(v.v_pool, tid / kVPieces))[tid % kVPieces] = vv;
+  for (int e = tid + kRopeThreads; e < nv; e += kRopeThreads)
+    reinterpret_cast<uint4 *>(pool_row(v.v_pool, e / kVPieces))[e % kVPieces] = vrow[e];
+  // 4. query heads in place, key heads into the slot
+  // Every output by the fast path, two to a conversion; the rare outputs whose rounding the
+  // fast path leaves open (bit 2 m + u of `open`: pair m, lower (u = 0) or upper half) are
+  // redone exactly in a loop of their own, so the exact path costs nothing where it is not used.
+  auto rotate_store = [&](int h, const uint4 &xl, const uint4 &xh) {
+    uint16_t *dst = h < Hq ? qrow + h * D : pool_row(v.k_pool, h - Hq);
+    uint32_t wl[4] = {xl.x, xl.y, xl.z, xl.w}, wh[4] = {xh.x, xh.y, xh.z, xh.w};
+    uint32_t open = 0;
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      uint32_t ol = 0, oh = 0;
+    for (int k = 0; k < 4; ++k) {
+      float yl[2], yh[2];
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
-        const float4 c4 = cs[2 * k + e];
+        const float4 c = cs_s[cs_index(8 * j + 2 * k + e)];
         const float x0 = bf16_value((uint16_t)(wl[k] >> (16 * e)));
         const float x1 = bf16_value((uint16_t)(wh[k] >> (16 * e)));
-        ol |= (uint32_t)rotate_dd(x0, x1, c4.x, c4.y, c4.z, c4.w) << (16 * e);   // x0 c - x1 s
-        oh |= (uint32_t)rotate_dd(x1, x0, c4.x, c4.y, -c4.z, -c4.w) << (16 * e); // x1 c + x0 s
+        const float err = __fmul_rn(__fadd_rn(fabsf(x0), fabsf(x1)), 0x1p-21f);
+        bool sure_l, sure_h;
+        yl[e] = rotate_fast(x0, x1, c.x, c.z, err, &sure_l);   // x0 c - x1 s
+        yh[e] = rotate_fast(x1, x0, c.x, -c.z, err, &sure_h);  // x1 c + x0 s
+        open |= (sure_l ? 0u : 1u) << (2 * (2 * k + e));
+        open |= (sure_h ? 0u : 2u) << (2 * (2 * k + e));
       }
-      yl[k] = ol;
-      yh[k] = oh;
+      const __nv_bfloat162 ol = __floats2bfloat162_rn(yl[0], yl[1]);
+      const __nv_bfloat162 oh = __floats2bfloat162_rn(yh[0], yh[1]);
+      const uint32_t uol = *reinterpret_cast<const uint32_t *>(&ol);
+      const uint32_t uoh = *reinterpret_cast<const uint32_t *>(&oh);
+      wl[k] = uol;  // wl/wh now hold outputs; the exact path reads the inputs from xl/xh
+      wh[k] = uoh;
     }
-    *reinterpret_cast<uint2 *>(dst + i0) = make_uint2(yl[0], yl[1]);
-    *reinterpret_cast<uint2 *>(dst + i0 + half) = make_uint2(yh[0], yh[1]);
-  }
+    while (open) {
+      const int bit = __ffs(open) - 1;
+      open &= open - 1;
+      const int m = bit >> 1, k = m >> 1, e = m & 1, upper = bit & 1;
+      const uint32_t in_l = k == 0 ? xl.x : k == 1 ? xl.y : k == 2 ? xl.z : xl.w;
+      const uint32_t in_h = k == 0 ? xh.x : k == 1 ? xh.y : k == 2 ? xh.z : xh.w;
+      const float4 c = cs_s[cs_index(8 * j + m)];
+      const float x0 = bf16_value((uint16_t)(in_l >> (16 * e)));
+      const float x1 = bf16_value((uint16_t)(in_h >> (16 * e)));
+      const uint32_t y = upper ? rotate_exact(x1, x0, c.x, c.y, -c.z, -c.w)
+                               : rotate_exact(x0, x1, c.x, c.y, c.z, c.w);
+      const uint32_t keep = e ? 0x0000FFFFu : 0xFFFF0000u, put = y << (16 * e);
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        if (kk != k) continue;
+        if (upper) wh[kk] = (wh[kk] & keep) | put;
+        else wl[kk] = (wl[kk] & keep) | put;
+      }
+    }
+    *reinterpret_cast<uint4 *>(dst + 8 * j) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+    *reinterpret_cast<uint4 *>(dst + kHalf + 8 * j) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+  };
+  if (h0 < H) rotate_store(h0, x0l, x0h);
+  if (h1 < H) rotate_store(h1, x1l, x1h);
+  for (int h = h1 + kHeadsPass; h < H; h += kHeadsPass)
+    rotate_store(h, half_of(h, 0), half_of(h, 1));
 }
 
 // ------------------------------------------------------------------------------------
@@ -836,7 +907,10 @@ cudaError_t launch_all(const CUtensorMap &tk, const CUtensorMap &tv, const Prefi
   prefill_plan_kernel<<<(unsigned)v.batch, kPlanThreads, 0, stream>>>(v, prefill_query_rows(G));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  prefill_rope_kernel<OutT><<<(unsigned)v.rows, kRopeThreads, 0, stream>>>(v);
+  if (v.head_dim == 128)
+    prefill_rope_kernel<128, OutT><<<(unsigned)v.rows, kRopeThreads, 0, stream>>>(v);
+  else
+    prefill_rope_kernel<64, OutT><<<(unsigned)v.rows, kRopeThreads, 0, stream>>>(v);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   return v.head_dim == 128 ? launch_attn<128, OutT>(tq, tk, tv, v, stream)

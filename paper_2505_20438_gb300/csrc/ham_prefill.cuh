@@ -22,8 +22,9 @@ struct PrefillView {
   const int32_t *offsets, *pos, *ntok;  // pos, ntok nullable
   void *out;                   // [rows][n_q_heads][head_dim], bf16 or f32
   int4 *seq_info;              // scratch [batch]: (first new slot or -1, rows, query-block
-                               // start, 0)
-  int32_t *row_pos;            // scratch [rows]: position of each new row
+                               // start, 1 when the call's offsets are valid, else 0)
+  int2 *row_info;              // scratch [rows]: (position, pool row page * page_slots + row
+                               // in page, or -1 when the row is not stored) of each new row
   int32_t *err;
   int64_t pool_pages;
   int32_t batch, rows, n_q_heads, n_kv_heads, head_dim, page_slots, max_pages, max_slots;

@@ -198,7 +198,7 @@ MetaLayout meta_layout(const ham_config &cfg, int32_t max_ctas, int64_t max_page
   m.stash = carve((size_t)cfg.batch * sizeof(int4));
   m.arrive = carve(sizeof(int32_t));
   m.pf_seq = carve((size_t)cfg.batch * sizeof(int4));
-  m.pf_pos = carve((size_t)cfg.batch * cfg.max_slots_per_seq * sizeof(int32_t));
+  m.pf_pos = carve((size_t)cfg.batch * cfg.max_slots_per_seq * sizeof(int2));
   {  // (max_ctas is 8 x the SMs)
     const bool fp8 = cfg.kv_dtype == HAM_KV_E4M3;
     const size_t floats = fp8 ? 0 : ham::prefill_part_floats(max_ctas / 8, cfg.head_dim);
@@ -570,7 +570,7 @@ int ham_kv_alloc(const ham_config *cfg_in, ham_kv **out) {
   kv->stash = reinterpret_cast<int4 *>(kv->meta + lay.stash);
   kv->arrive = reinterpret_cast<int32_t *>(kv->meta + lay.arrive);
   kv->prefill_seq = reinterpret_cast<int4 *>(kv->meta + lay.pf_seq);
-  kv->prefill_pos = reinterpret_cast<int32_t *>(kv->meta + lay.pf_pos);
+  kv->prefill_rows = reinterpret_cast<int2 *>(kv->meta + lay.pf_pos);
   if (!kv->fp8) {
     kv->prefill_part = reinterpret_cast<float *>(kv->meta + lay.pf_part);
     kv->prefill_part_ml = reinterpret_cast<float2 *>(kv->meta + lay.pf_ml);
@@ -1071,7 +1071,7 @@ int ham_prefill(ham_kv *kv, int32_t layer, void *q_inout, const void *k_new, con
   v.out = out;
   v.wait_ns = kv->wait_ns;
   v.seq_info = kv->prefill_seq;
-  v.row_pos = kv->prefill_pos;
+  v.row_info = kv->prefill_rows;
   // Split over slots when the grid would leave SMs idle (a short chunk, whatever the cache
   // holds: the kernel keeps one split for sequences with few cached slots).
   {
