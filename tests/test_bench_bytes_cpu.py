@@ -49,3 +49,44 @@ def test_workload_names_resolve():
     assert isinstance(m, wl.MicroWorkload) and (m.layers, m.context, m.micro_steps) == (4, 4, 3)
     c = wl.make_micro_case(m)
     assert c.max_slots == 8 and list(c.num_slots) == [4] * 8 and all(c.ntok_new == 1)
+
+
+def test_fp8_attention_bytes_of_the_llama8b_layer():
+    w = wl.C1_LLAMA8B
+    b = _bench()
+    # an e4m3 row is 128 codes and one exponent byte: 129 B against 256 B in bf16
+    assert b.kv_row_bytes(w, "fp8") == 129 and b.kv_row_bytes(w) == 256
+    kv8 = 8 * 4096 * 8 * 129 * 2
+    assert b.attn_bytes(w, [4096] * 8, "fp8") == kv8 + 2 * 8 * 32 * 128 * 2 + 8 * 256 * 4
+    # the appended rows shrink the same way; q, k_new and v_new stay bf16
+    assert b.append_bytes(w) - b.append_bytes(w, "fp8") == 2 * 8 * 8 * (256 - 129)
+
+
+def test_fp8_front_bytes_of_the_llama8b_layer():
+    w = wl.front_workload(8)
+    b = _bench()
+    assert b.front_bytes(w) - b.front_bytes(w, "fp8") == 8 * 2 * 8 * (256 - 129)
+
+
+def test_prefill_flops_count_every_attended_pair():
+    b = _bench()
+    # brute force on small chunks: every new row j of every sequence attends L + j + 1 slots
+    for rows, cached in ((1, 0), (5, 3), (7, 64), (64, 1000)):
+        pw = wl.PrefillWorkload("t", wl.C1_LLAMA8B, rows=rows, cached=cached)
+        w = pw.w
+        pairs = sum(cached + j + 1 for j in range(rows)) * w.batch
+        assert b.prefill_flops(pw) == 4 * w.head_dim * w.n_q_heads * pairs
+    # the bench workloads: 549.9 GFLOP for 4 fresh prompts of 4096 rows, 68.8 GFLOP for 64 rows
+    # over 65,536 cached slots
+    p1, p3 = wl.PREFILL_WORKLOADS["prefill_b4_s4096"], wl.PREFILL_WORKLOADS["prefill_b1_c64_s65536"]
+    assert b.prefill_flops(p1) == 4 * 128 * 32 * 4 * (4096 * 4097 // 2) == 549_890_031_616
+    assert b.prefill_flops(p3) == 4 * 128 * 32 * (64 * 65536 + 64 * 65 // 2)
+
+
+def test_prefill_bytes_of_the_short_chunk():
+    p3 = _bench().workload("prefill_b1_c64_s65536")
+    # K and V of 65,536 + 64 slots x 8 heads x 128 x 2 B; q in and out (32 heads); k, v in
+    kv = (65536 + 64) * 8 * 128 * 2 * 2
+    q = 64 * 32 * 128 * 2 * 2
+    new = 64 * 8 * 128 * 2 * 2
+    assert _bench().prefill_bytes(p3) == kv + q + new == 270_008_320
