@@ -1974,8 +1974,12 @@ def main():
     w = workload(args.workload)
     from paper_2505_20438_gb300 import workload as wl
     if args.impl == "reference":
-        run_reference(args, w)
-    elif isinstance(w, wl.EmbedWorkload):
+        return run_reference(args, w)
+    import torch
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py: this arm runs the library's CUDA kernels and needs a GPU "
+                         "(GB300); there is no CPU path (--impl reference times the oracle)")
+    if isinstance(w, wl.EmbedWorkload):
         run_embed(args, w)
     elif isinstance(w, wl.FrontWorkload):
         run_front(args, w)
