@@ -169,3 +169,55 @@ def test_embedder_null_arguments_are_rejected(libham):
     assert libham.ham_embedder_set_vocab(None, None, 1) == ham.HAM_EINVAL
     assert libham.ham_embed_tokens(None, None, None, 1, 1, None, None) == ham.HAM_EINVAL
     assert libham.ham_embedder_free(None) == ham.HAM_OK
+
+
+# ---------------------------------------------------------------------------------------
+# the binding never hands a host pointer to a kernel: every tensor argument is checked for
+# device, dtype, shape and layout before the library is called
+# ---------------------------------------------------------------------------------------
+
+def _fake_kv():
+    import types
+    return types.SimpleNamespace(batch=2, n_q_heads=8, n_kv_heads=2, head_dim=64, max_pages=4)
+
+
+def _host_tensors():
+    import torch
+    B, Hq, Hkv, d = 2, 8, 2, 64
+    return dict(q=torch.zeros(B, Hq, d, dtype=torch.bfloat16),
+                kn=torch.zeros(B, Hkv, d, dtype=torch.bfloat16),
+                vn=torch.zeros(B, Hkv, d, dtype=torch.bfloat16),
+                ntok=torch.ones(B, dtype=torch.int32),
+                out=torch.zeros(B, Hq, d, dtype=torch.bfloat16),
+                x=torch.zeros(B, 256, dtype=torch.bfloat16),
+                w=torch.zeros((Hq + 2 * Hkv) * d, 256, dtype=torch.bfloat16),
+                off=torch.tensor([0, 1, 2], dtype=torch.int32),
+                q1=torch.zeros(2, Hq, d, dtype=torch.bfloat16),
+                k1=torch.zeros(2, Hkv, d, dtype=torch.bfloat16))
+
+
+@pytest.mark.parametrize("call,first", [
+    (lambda kv, t: ham.ham_kv_append(kv, 0, t["q"], t["kn"], t["vn"], None, t["ntok"]), "q_inout"),
+    (lambda kv, t: ham.ham_decode_attn(kv, 0, t["q"], t["out"]), "q"),
+    (lambda kv, t: ham.ham_decode_attn_ex(kv, 0, t["q"], t["out"]), "q"),
+    (lambda kv, t: ham.ham_decode_step(kv, 0, t["q"], t["kn"], t["vn"], None, t["ntok"],
+                                       t["out"]), "q"),
+    (lambda kv, t: ham.ham_micro_step(kv, 0, t["q"], t["kn"], t["vn"], None, t["ntok"],
+                                      t["out"]), "q"),
+    (lambda kv, t: ham.ham_prefill(kv, 0, t["q1"], t["k1"], t["k1"], t["off"], t["q1"]), "q"),
+    (lambda kv, t: ham.ham_qkv_append(kv, 0, t["x"], t["w"], t["ntok"], t["q"]), "x"),
+    (lambda kv, t: ham.ham_kv_fill(kv, 0, t["kn"][:, None], t["vn"][:, None], t["ntok"]), "k"),
+])
+def test_binding_rejects_host_tensors_before_the_library(call, first):
+    with pytest.raises(ValueError, match="must be a CUDA tensor") as e:
+        call(_fake_kv(), _host_tensors())
+    assert str(e.value).startswith(first)
+
+
+def test_binding_rejects_host_tensors_without_a_handle():
+    import torch
+    t = _host_tensors()
+    pool = torch.zeros(4, 2, 16, 64, dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="k_pool must be a CUDA tensor"):
+        ham.ham_decode_attn_noalloc(pool, pool, torch.zeros(2, 4, dtype=torch.int32),
+                                    t["ntok"], t["q"], t["out"], 64)
