@@ -90,3 +90,17 @@ def test_prefill_bytes_of_the_short_chunk():
     q = 64 * 32 * 128 * 2 * 2
     new = 64 * 8 * 128 * 2 * 2
     assert _bench().prefill_bytes(p3) == kv + q + new == 270_008_320
+
+
+def test_cost_model_follows_the_papers_speedup_formula():
+    # Sec. 3.7: r = n C(S) / (C(S) + (n - 1) c); one token per slot gives no speed-up, a free
+    # micro-step decoder gives n, and any c < C(S) with n > 1 gives r > 1
+    cm = _bench().cost_model
+    assert cm(1.0, 30.0)["r"] == 1.0
+    assert cm(3.0, 30.0, c_ratio=0.0)["r"] == 3.0
+    assert math.isclose(cm(2.0, 40.0, c_ratio=1 / 8)["r"], 16 / 9, abs_tol=1e-4)
+    for n in (1.5, 1.875, 4.0):
+        for ratio in (0.05, 0.125, 0.9):
+            d = cm(n, 25.0, c_ratio=ratio)
+            assert d["r"] > 1.0 and d["kind"] == "modelled"
+            assert math.isclose(d["c_us"], ratio * 25.0, rel_tol=1e-3)
