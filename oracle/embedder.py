@@ -44,8 +44,11 @@ def softmax(s: np.ndarray) -> np.ndarray:
 
 def embed(x_bits, offsets, wq_bits, wk_bits, wv_bits, wo_bits, pos_bits, n_heads,
           return_o=False):
-    """Fused hidden state of every sequence, fp64 [B][H]; with return_o also the attention
-    output o [B][H] that enters the output linear (zeros for single-token sequences)."""
+    """Fused hidden state of every sequence, fp64 [B][H] (Sec. 3.2 "Compositional Embedder":
+    the mean of a sequence's token embeddings queries the embeddings plus their in-patch position
+    embeddings, multi-head, then a linear layer; Sec. 3.4: a single token bypasses it); with
+    return_o also the attention output o [B][H] that enters the output linear (zeros for
+    single-token sequences)."""
     x = bf16_bits_to_f64(x_bits)
     wq, wk, wv, wo = (bf16_bits_to_f64(w) for w in (wq_bits, wk_bits, wv_bits, wo_bits))
     pos = bf16_bits_to_f64(pos_bits)
@@ -78,7 +81,8 @@ def embed(x_bits, offsets, wq_bits, wk_bits, wv_bits, wo_bits, pos_bits, n_heads
 
 
 def attention_weights(x_bits, n_tokens_first, wq_bits, wk_bits, pos_bits, n_heads):
-    """Softmax weights [n_heads][n] of the first sequence (for the sum-to-one pin)."""
+    """Softmax weights [n_heads][n] of the first sequence (for the sum-to-one pin): the
+    cross-attention of `embed` (Sec. 3.2), weights only."""
     x = bf16_bits_to_f64(x_bits)[:n_tokens_first]
     wq, wk = bf16_bits_to_f64(wq_bits), bf16_bits_to_f64(wk_bits)
     pos = bf16_bits_to_f64(pos_bits)

@@ -37,7 +37,8 @@ E4M3_NAN_CODES = (0x7F, 0xFF)
 
 
 def e4m3_value(code) -> np.ndarray:
-    """Exact value of e4m3 codes (uint8), NaN for the two NaN codes."""
+    """Exact value of e4m3 codes (uint8), NaN for the two NaN codes (reading Q1: the OCP e4m3
+    "fn" format; the paper keeps the base model's precision and fixes no 8-bit format)."""
     c = np.asarray(code, dtype=np.int64)
     sign = np.where(c & 0x80, -1.0, 1.0)
     exp = (c >> 3) & 0xF
@@ -85,14 +86,15 @@ def row_exponent(values) -> int:
 
 
 def encode_row(values):
-    """(codes uint8 [n], e int) of one row of exact values (bf16 values given as float)."""
+    """(codes uint8 [n], e int) of one row of exact values (bf16 values given as float): one
+    power-of-two scale per stored row (Q2, Q3), each element rounded once (Q1)."""
     v = np.asarray(values, dtype=np.float64)
     e = row_exponent(v)
     return e4m3_encode(np.ldexp(v, -e)), e
 
 
 def decode_row(codes, e) -> np.ndarray:
-    """Exact values code * 2^e of one row."""
+    """Exact values code * 2^e of one row (Q4: what attention over an FP8 pool reads)."""
     return np.ldexp(e4m3_value(codes), int(e))
 
 

@@ -67,14 +67,16 @@ def f64_to_bf16_bits(x) -> np.ndarray:
 
 
 def project(x_bits, w_bits) -> np.ndarray:
-    """y[b, o] = sum_k W[o, k] x[b, k] in fp64 (the linear map of F1)."""
+    """y[b, o] = sum_k W[o, k] x[b, k] in fp64 (the linear map of F1: the base model's q/k/v
+    projections, Sec. 4.1, fused into one weight)."""
     x = bf16_bits_to_f64(x_bits)
     w = bf16_bits_to_f64(w_bits)
     return x @ w.T
 
 
 def rope_values(y, pos: int, base: float = 10000.0) -> np.ndarray:
-    """Rotate-half RoPE of fp64 rows y [..., d] at integer position pos (fp64 throughout)."""
+    """Rotate-half RoPE of fp64 rows y [..., d] at integer position pos (fp64 throughout): the
+    base model's rotary embedding (Sec. 4.1) at the macro-step's offset position (Sec. 3.2)."""
     y = np.asarray(y, dtype=np.float64)
     d = y.shape[-1]
     half = d // 2
@@ -86,7 +88,9 @@ def rope_values(y, pos: int, base: float = 10000.0) -> np.ndarray:
 
 
 def qkv_append(cache, x_bits, w_bits, ntok, pos=None, pos_mode=POS_SLOT, rope_base=10000.0):
-    """One layer front of one macro-step on an oracle.OracleCache (its arrays are edited).
+    """One layer front of one macro-step on an oracle.OracleCache (its arrays are edited): the
+    macro-step's one forward stores one key/value set (Sec. 3.1), projected, rotated at the
+    offset position (Sec. 3.2) and appended as the append oracle appends it.
 
     x_bits [B][H], w_bits [(Hq + 2 Hkv) d][H] bf16 bits; ntok [B]; pos nullable [B].
     Returns (status, q_rot bits [B][Hq][d], y fp64 [B][(Hq + 2 Hkv) d]): status 0, or the
