@@ -188,6 +188,20 @@ def test_rows_that_do_not_fit_leave_the_sequence_untouched():
     assert rc2 == o.EINVAL and list(oc2.num_slots) == [16, 20] and np.all(out2[6:] == 0)
 
 
+def test_capacity_boundary_is_exact():
+    # a chunk that fills the sequence to its capacity is stored; one row more is refused whole
+    o = _o()
+    for cap, fits in ((29, True), (28, False)):
+        case = wl.make_prefill_case(_w(seed=8), [6, 9], cached=np.array([10, 20], np.int32))
+        case.base.max_slots = cap
+        oc, _, rc, out = _run(case)
+        if fits:
+            assert rc == 0 and list(oc.num_slots) == [16, 29]
+        else:
+            assert rc == o.ECAPACITY and list(oc.num_slots) == [16, 20]
+            assert np.all(out[int(case.offsets[1]):] == 0)
+
+
 def test_row_mask_only_skips_attention():
     case = wl.make_prefill_case(_w(seed=9), [12, 7], cached=np.array([4, 0], np.int32))
     oc_all, q_all, _, out_all = _run(case)
