@@ -361,3 +361,54 @@ def test_fp8_unsupported_calls_are_refused():
     assert e.value.status == ham.HAM_EUNSUPPORTED
     slots, _ = ham.ham_slot_lengths(kv)
     assert list(slots) == [5, 6]
+
+
+# ---------------------------------------------------------------------------------------
+# full size, in the bench's launch configuration (default CTA count)
+# ---------------------------------------------------------------------------------------
+
+FULL_SIZE_PAGES = 16   # pages of the checked sequence whose codes are compared
+
+
+def _full_size_reference(case, b):
+    """Oracle attention with sequence b's rows decoded through the FP8 format (the other
+    sequences' rows are left as bf16: their outputs are not compared, and the oracle's encoder
+    is brute force, about 10 s per 4M elements)."""
+    kd, vd = case.k.copy(), case.v.copy()
+    kd[b], vd[b] = _decoded(case.k[b]), _decoded(case.v[b])
+    ref = oracle.OracleCache.from_case(case, fill=False)
+    ref.fill(kd, vd, case.slot_pos, case.slot_ntok, case.num_slots)
+    return ref.decode_attn(case.q)
+
+
+def _full_size_pages(case, b):
+    """A spread of the pages sequence b uses."""
+    used = -(-int(case.num_slots[b]) // case.w.page_slots)
+    idx = np.unique(np.linspace(0, used - 1, FULL_SIZE_PAGES).round().astype(np.int64))
+    return case.page_table[b, idx].astype(np.int64)
+
+
+@pytest.mark.parametrize("w", [wl.C1_LLAMA8B, wl.C1_LLAMA8B_S8K], ids=lambda w: w.name)
+def test_fp8_full_size_workloads(w):
+    """The bench's Llama-8B layer at 4096 and 8192 slots over an FP8 pool: every output
+    finite, the last sequence's attention (all 32 heads) against the oracle on its decoded rows
+    at the usual bar, and the codes and exponents of a spread of its pages bit for bit."""
+    case = wl.make_case(w, extra_slots=4)
+    kv = fp8_cache(case)
+    out = _decode(kv, case.q)
+    assert np.all(np.isfinite(out))
+    b = w.batch - 1
+    ref = _full_size_reference(case, b)
+    assert_parity(out[b], ref[b], what=f"{w.name}, sequence {b}")
+    pages = _full_size_pages(case, b)
+    raw = oracle.OracleCache.from_case(case)
+    kc, vc, ee = _expected_pools(raw.k_pool[pages], raw.v_pool[pages])
+    k, v, e, pos, ntok = _export(kv)
+    assert np.array_equal(k[pages], kc), "K codes"
+    assert np.array_equal(v[pages], vc), "V codes (transposed)"
+    assert np.array_equal(e[pages], ee), "exponents"
+    assert np.array_equal(pos, raw.slot_pos) and np.array_equal(ntok, raw.slot_ntok)
+    slots, _ = ham.ham_slot_lengths(kv)
+    assert np.array_equal(slots, case.num_slots)
+    assert ham.ham_kv_status(kv) == ham.HAM_DEVERR_NONE
+    ham.ham_kv_free(kv)
